@@ -1,0 +1,587 @@
+"""CPU oracle for one grid iteration of Lipizzaner's coevolutionary GAN training.
+
+TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU
+baseline / reference arm may import or run this module. The product path (the CUDA library
+and its Python binding) never calls it, and this module never imports the product.
+
+What it computes follows the method section of arXiv 1811.12843 (Section 3, "Coevolutionary GAN
+Training", steps 1-3 and 5) and its settings table (Table 1), written as plain numpy in float64:
+
+  1. every cell of an R x C toroidal grid holds one generator (params u_i, learning rate delta_i)
+     and one discriminator (v_j, gamma_j), randomly initialised (step 1);
+  2. each generator is evaluated against each discriminator of its cell's 5-cell von Neumann
+     neighbourhood (centre, N, S, W, E; Section 2 "Scaling Evolutionary Computing for ML"),
+     L(u_i, v_j) on one minibatch; a discriminator's fitness averages its interactions, a
+     generator's averages its own (step 2);
+  3. size-2 tournament selection in each neighbourhood, then one gradient (Adam) update of the
+     selected pair, with optional Gaussian mutation of the learning rate (step 3, Table 1).
+
+Readings where the paper is silent (each is listed in the design doc with its reason):
+  * fitness is a loss for both populations, lower is better: f_G = mean_j L_G, f_D = mean_i L_D;
+  * L_D is the SUM of the real-batch and fake-batch BCE means; L_G is the non-saturating loss;
+  * iterations run on a synchronous snapshot of all centres;
+  * tournament entrants are distinct slots; a tie goes to the lower slot; the centre is replaced
+    by the winner only if the winner's fitness is strictly lower (``if_better``) -- or always;
+  * the pair is trained on the same minibatch that was used for its evaluation, with the fake
+    batch detached for the discriminator gradient and both gradients taken at the pre-update
+    parameters; one Adam step (Kingma & Ba 2015, Algorithm 1) per iteration;
+  * random draws come from Philox4x32-10 (Salmon et al., SC'11) keyed by the seed, with the
+    counter (block index, cell, iteration, stream);
+  * in bf16 mode every operand of a matrix product (weights, activations, back-propagated
+    deltas) is rounded to bfloat16 (round to nearest even), products accumulate exactly (here:
+    float64), biases, logits, losses, gradients and optimiser state stay unrounded.
+
+Parity of the whole iteration against the paper is pinned only through its pieces (Philox
+known-answer vectors, torus invariants, the ln 2 BCE case, finite-difference gradients, Adam's
+closed-form first step, torch cross-checks, exhaustive tournament checks); see tests/.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, List, Optional, Tuple
+
+import numpy as np
+
+# --------------------------------------------------------------------------------------------
+# Counter-based random numbers: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random
+# numbers: as easy as 1, 2, 3", SC'11). Multipliers and Weyl key increments are the ones that
+# paper publishes for the 4x32 variant.
+# --------------------------------------------------------------------------------------------
+_PHILOX_M0 = np.uint64(0xD2511F53)
+_PHILOX_M1 = np.uint64(0xCD9E8D57)
+_PHILOX_W0 = 0x9E3779B9
+_PHILOX_W1 = 0xBB67AE85
+_MASK32 = np.uint64(0xFFFFFFFF)
+
+# Stream ids (the fourth counter word); part of the library's documented contract.
+STREAM_INIT_G = 1
+STREAM_INIT_D = 2
+STREAM_BATCH = 3
+STREAM_NOISE = 4
+STREAM_TOUR_G = 5
+STREAM_TOUR_D = 6
+STREAM_MUT_G = 7
+STREAM_MUT_D = 8
+
+
+def philox4x32_10(ctr: np.ndarray, key: Tuple[int, int]) -> np.ndarray:
+    """Ten Philox rounds on counters ``ctr`` ([..., 4] of 32-bit values) with key (k0, k1).
+
+    One round: the products M0*c0 and M1*c2 are split into high/low halves; the new counter is
+    (hi1 ^ c1 ^ k0, lo1, hi0 ^ c3 ^ k1, lo0). The key is bumped by the Weyl constants between
+    rounds.
+    """
+    ctr = np.asarray(ctr, dtype=np.uint64)
+    c0, c1, c2, c3 = (ctr[..., i].copy() for i in range(4))
+    k0, k1 = int(key[0]) & 0xFFFFFFFF, int(key[1]) & 0xFFFFFFFF
+    for rnd in range(10):
+        if rnd:
+            k0 = (k0 + _PHILOX_W0) & 0xFFFFFFFF
+            k1 = (k1 + _PHILOX_W1) & 0xFFFFFFFF
+        p0 = _PHILOX_M0 * c0
+        p1 = _PHILOX_M1 * c2
+        hi0, lo0 = p0 >> np.uint64(32), p0 & _MASK32
+        hi1, lo1 = p1 >> np.uint64(32), p1 & _MASK32
+        c0, c1, c2, c3 = hi1 ^ c1 ^ np.uint64(k0), lo1, hi0 ^ c3 ^ np.uint64(k1), lo0
+    return np.stack([c0, c1, c2, c3], axis=-1)
+
+
+def draw_words(seed: int, stream: int, t: int, cell: int, n: int) -> np.ndarray:
+    """The first ``n`` 32-bit words of the (stream, t, cell) sequence: word k is output word
+    k % 4 of the Philox block with counter (k // 4, cell, t, stream), key = (seed lo, seed hi)."""
+    nb = (n + 3) // 4
+    ctr = np.zeros((nb, 4), dtype=np.uint64)
+    ctr[:, 0] = np.arange(nb, dtype=np.uint64)
+    ctr[:, 1] = cell
+    ctr[:, 2] = t
+    ctr[:, 3] = stream
+    out = philox4x32_10(ctr, (seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF))
+    return out.reshape(-1)[:n]
+
+
+def mulhi(w: np.ndarray, n: int) -> np.ndarray:
+    """floor(w * n / 2^32): maps a uniform 32-bit word onto {0, .., n-1} without floats."""
+    return (np.asarray(w, dtype=np.uint64) * np.uint64(n)) >> np.uint64(32)
+
+
+def box_muller(wa: np.ndarray, wb: np.ndarray) -> Tuple[np.ndarray, np.ndarray]:
+    """Two standard normals from two words (Box & Muller 1958): u1 = (top 24 bits + 1) / 2^24 in
+    (0, 1], v = (top 24 bits) / 2^24 in [0, 1); r = sqrt(-2 ln u1); (r cos 2 pi v, r sin 2 pi v)."""
+    u1 = ((np.asarray(wa, dtype=np.uint64) >> np.uint64(8)).astype(np.float64) + 1.0) * 2.0 ** -24
+    v = (np.asarray(wb, dtype=np.uint64) >> np.uint64(8)).astype(np.float64) * 2.0 ** -24
+    r = np.sqrt(-2.0 * np.log(u1))
+    return r * np.cos(2.0 * math.pi * v), r * np.sin(2.0 * math.pi * v)
+
+
+def draw_normals(seed: int, stream: int, t: int, cell: int, n: int) -> np.ndarray:
+    """``n`` normals: block i's words (w0, w1, w2, w3) give normals 4i..4i+3 as
+    box_muller(w0, w1) followed by box_muller(w2, w3)."""
+    nb = (n + 3) // 4
+    w = draw_words(seed, stream, t, cell, 4 * nb).reshape(nb, 4)
+    out = np.empty((nb, 4), dtype=np.float64)
+    out[:, 0], out[:, 1] = box_muller(w[:, 0], w[:, 1])
+    out[:, 2], out[:, 3] = box_muller(w[:, 2], w[:, 3])
+    return out.reshape(-1)[:n]
+
+
+# --------------------------------------------------------------------------------------------
+# Configuration (Table 1 for the MLP/MNIST column) and parameter layout.
+# --------------------------------------------------------------------------------------------
+@dataclasses.dataclass
+class Arch:
+    z_dim: int = 64          # input neurons (Table 1)
+    hidden: int = 256        # neurons per hidden layer, 2 hidden layers (Table 1)
+    x_dim: int = 784         # output neurons (Table 1)
+    batch: int = 100         # batch size (Table 1)
+    precision: str = "fp32"  # "fp32" or "bf16"
+    lr: float = 2e-4         # initial learning rate (Table 1)
+    beta1: float = 0.5
+    beta2: float = 0.999
+    eps: float = 1e-8
+    tournament_size: int = 2  # Table 1
+    replace_mode: str = "if_better"  # or "always"
+    lr_mutation: bool = False
+    lr_mut_std: float = 1e-4  # mutation rate (Table 1)
+    lr_mut_prob: float = 0.5  # mutation probability (Table 1)
+    leaky_slope: float = 0.2
+
+
+def g_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
+    """Generator tensors in storage order; weights are [out][in] row-major."""
+    return [("W1", (a.hidden, a.z_dim)), ("b1", (a.hidden,)),
+            ("W2", (a.hidden, a.hidden)), ("b2", (a.hidden,)),
+            ("W3", (a.x_dim, a.hidden)), ("b3", (a.x_dim,))]
+
+
+def d_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
+    """Discriminator tensors in storage order; weights are [out][in] row-major."""
+    return [("W1", (a.hidden, a.x_dim)), ("b1", (a.hidden,)),
+            ("W2", (a.hidden, a.hidden)), ("b2", (a.hidden,)),
+            ("W3", (1, a.hidden)), ("b3", (1,))]
+
+
+def n_params(layout) -> int:
+    return sum(int(np.prod(s)) for _, s in layout)
+
+
+def unflatten(flat: np.ndarray, layout) -> Dict[str, np.ndarray]:
+    """Views of the named tensors inside one flat parameter vector."""
+    out, off = {}, 0
+    for name, shape in layout:
+        n = int(np.prod(shape))
+        out[name] = flat[off:off + n].reshape(shape)
+        off += n
+    return out
+
+
+def neighbors(rows: int, cols: int) -> np.ndarray:
+    """nbr[c] = (centre, north, south, west, east) on the torus, cells numbered r * cols + col.
+    Duplicates are kept (a 1x1 grid has the centre in all five slots)."""
+    nbr = np.empty((rows * cols, 5), dtype=np.int64)
+    for r in range(rows):
+        for q in range(cols):
+            nbr[r * cols + q] = [r * cols + q,
+                                 ((r - 1) % rows) * cols + q,
+                                 ((r + 1) % rows) * cols + q,
+                                 r * cols + (q - 1) % cols,
+                                 r * cols + (q + 1) % cols]
+    return nbr
+
+
+def xavier_bound(fan_in: int, fan_out: int) -> np.float32:
+    """Glorot & Bengio (2010) uniform bound sqrt(6 / (fan_in + fan_out)), stored as float32."""
+    return np.float32(math.sqrt(6.0 / (fan_in + fan_out)))
+
+
+def init_params(seed: int, stream: int, cell: int, layout) -> np.ndarray:
+    """Step 1: random weights. Element k of a weight tensor takes word k of the flat vector's
+    sequence: s = word >> 8, q = (2 s + 1 - 2^24) / 2^24 in (-1, 1), w = float32(a * q) with a the
+    tensor's Xavier bound. Biases start at zero."""
+    total = n_params(layout)
+    words = draw_words(seed, stream, 0, cell, total)
+    flat = np.zeros(total, dtype=np.float64)
+    off = 0
+    for name, shape in layout:
+        n = int(np.prod(shape))
+        if name.startswith("W"):
+            s = (words[off:off + n] >> np.uint64(8)).astype(np.float64)
+            q = (2.0 * s + 1.0 - 2.0 ** 24) * 2.0 ** -24
+            a = float(xavier_bound(shape[1], shape[0]))
+            flat[off:off + n] = (a * q).astype(np.float32)
+        off += n
+    return flat
+
+
+# --------------------------------------------------------------------------------------------
+# Arithmetic helpers.
+# --------------------------------------------------------------------------------------------
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bfloat16 value (8 significant bits), ties to even."""
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)
+    return np.ldexp(np.round(m * 256.0), e - 8)
+
+
+def softplus(x: np.ndarray) -> np.ndarray:
+    """log(1 + e^x), written max(x, 0) + log1p(e^-|x|) so that it never overflows."""
+    return np.maximum(x, 0.0) + np.log1p(np.exp(-np.abs(x)))
+
+
+def sigmoid(x: np.ndarray) -> np.ndarray:
+    return 0.5 * (1.0 + np.tanh(0.5 * x))
+
+
+class _Rounder:
+    def __init__(self, arch: Arch):
+        if arch.precision not in ("fp32", "bf16"):
+            raise ValueError("precision must be fp32 or bf16")
+        self.bf16 = arch.precision == "bf16"
+
+    def __call__(self, x):
+        return round_bf16(x) if self.bf16 else np.asarray(x, dtype=np.float64)
+
+
+def g_forward(P: Dict[str, np.ndarray], z: np.ndarray, arch: Arch) -> Dict[str, np.ndarray]:
+    """Generator MLP: z -> ReLU(256) -> ReLU(256) -> tanh(784). Returns every activation."""
+    rb = _Rounder(arch)
+    zq = rb(z)
+    h1 = rb(np.maximum(zq @ rb(P["W1"]).T + P["b1"], 0.0))
+    h2 = rb(np.maximum(h1 @ rb(P["W2"]).T + P["b2"], 0.0))
+    F = rb(np.tanh(h2 @ rb(P["W3"]).T + P["b3"]))
+    return {"z": zq, "h1": h1, "h2": h2, "F": F}
+
+
+def _lrelu(x, slope):
+    return np.where(x > 0.0, x, slope * x)
+
+
+def d_forward(P: Dict[str, np.ndarray], X: np.ndarray, arch: Arch) -> Dict[str, np.ndarray]:
+    """Discriminator MLP: x -> LeakyReLU(256) -> LeakyReLU(256) -> logit (sigmoid in the loss)."""
+    rb = _Rounder(arch)
+    Xq = rb(X)
+    g1 = rb(_lrelu(Xq @ rb(P["W1"]).T + P["b1"], arch.leaky_slope))
+    g2 = rb(_lrelu(g1 @ rb(P["W2"]).T + P["b2"], arch.leaky_slope))
+    logit = g2 @ rb(P["W3"])[0] + P["b3"][0]
+    return {"X": Xq, "g1": g1, "g2": g2, "logit": logit}
+
+
+def pair_losses(logit_real: np.ndarray, logit_fake: np.ndarray) -> Tuple[float, float]:
+    """L_D = mean BCE(D(x), 1) + mean BCE(D(G(z)), 0);  L_G = mean BCE(D(G(z)), 1).
+    With sigmoid outputs, BCE(l, 1) = softplus(-l) and BCE(l, 0) = softplus(l)."""
+    ld = float(np.mean(softplus(-logit_real)) + np.mean(softplus(logit_fake)))
+    lg = float(np.mean(softplus(-logit_fake)))
+    return lg, ld
+
+
+# --------------------------------------------------------------------------------------------
+# Grid state.
+# --------------------------------------------------------------------------------------------
+@dataclasses.dataclass
+class State:
+    rows: int
+    cols: int
+    arch: Arch
+    seed: int
+    t: int
+    Gw: np.ndarray   # [cells, PG] parameters (float64 holding float32 values after init)
+    Gm: np.ndarray
+    Gv: np.ndarray
+    Gstep: np.ndarray  # [cells] int64
+    Glr: np.ndarray    # [cells]
+    Dw: np.ndarray
+    Dm: np.ndarray
+    Dv: np.ndarray
+    Dstep: np.ndarray
+    Dlr: np.ndarray
+
+    @property
+    def cells(self) -> int:
+        return self.rows * self.cols
+
+    def copy(self) -> "State":
+        return dataclasses.replace(self, **{f: getattr(self, f).copy() for f in
+                                            ("Gw", "Gm", "Gv", "Gstep", "Glr",
+                                             "Dw", "Dm", "Dv", "Dstep", "Dlr")})
+
+
+def create(rows: int, cols: int, arch: Arch, seed: int) -> State:
+    """Step 1 for every cell: Xavier weights, zero biases and moments, lr = arch.lr, step 0."""
+    if rows < 1 or cols < 1:
+        raise ValueError("grid needs rows, cols >= 1")
+    gl, dl = g_layout(arch), d_layout(arch)
+    cells = rows * cols
+    Gw = np.stack([init_params(seed, STREAM_INIT_G, c, gl) for c in range(cells)])
+    Dw = np.stack([init_params(seed, STREAM_INIT_D, c, dl) for c in range(cells)])
+    lr = float(np.float32(arch.lr))
+    return State(rows, cols, arch, seed, 0,
+                 Gw, np.zeros_like(Gw), np.zeros_like(Gw), np.zeros(cells, np.int64),
+                 np.full(cells, lr), Dw, np.zeros_like(Dw), np.zeros_like(Dw),
+                 np.zeros(cells, np.int64), np.full(cells, lr))
+
+
+def draw_batch(seed: int, t: int, cell: int, pool: np.ndarray, arch: Arch
+               ) -> Tuple[np.ndarray, np.ndarray]:
+    """Cell ``cell``'s minibatch at iteration ``t``: B pool rows at indices mulhi(word_b, n)
+    (stream BATCH) and z = B x z_dim normals (stream NOISE), row-major."""
+    w = draw_words(seed, STREAM_BATCH, t, cell, arch.batch)
+    idx = mulhi(w, pool.shape[0]).astype(np.int64)
+    x = pool[idx].astype(np.float64)
+    z = draw_normals(seed, STREAM_NOISE, t, cell, arch.batch * arch.z_dim)
+    return x, z.reshape(arch.batch, arch.z_dim)
+
+
+def batches(state: State, pool: Optional[np.ndarray], x_host: Optional[np.ndarray] = None):
+    """Per-cell (x, z) for the state's current iteration. ``x_host`` ([cells, B, x_dim]) replaces
+    the pool draw when the caller supplies the real minibatches itself."""
+    a = state.arch
+    out = []
+    for c in range(state.cells):
+        if x_host is not None:
+            z = draw_normals(state.seed, STREAM_NOISE, state.t, c, a.batch * a.z_dim)
+            out.append((np.asarray(x_host[c], np.float64), z.reshape(a.batch, a.z_dim)))
+        else:
+            out.append(draw_batch(state.seed, state.t, c, pool, a))
+    return out
+
+
+# --------------------------------------------------------------------------------------------
+# Step 2: all-pairs evaluation and fitness.
+# --------------------------------------------------------------------------------------------
+def eval_neighborhoods(state: State, data) -> Dict[str, np.ndarray]:
+    """For each cell c and slots (i, j): generator nbr[c][i] against discriminator nbr[c][j] on
+    cell c's minibatch. Returns L_G, L_D [cells, 5(i), 5(j)], fitness f_G = mean_j L_G[c, i, :],
+    f_D = mean_i L_D[c, :, j], and the logits [cells, 5(j), 6B] (real rows, then the fakes of
+    generator slots 0..4)."""
+    a = state.arch
+    gl, dl = g_layout(a), d_layout(a)
+    nbr = neighbors(state.rows, state.cols)
+    cells, B = state.cells, a.batch
+    LG = np.zeros((cells, 5, 5))
+    LD = np.zeros((cells, 5, 5))
+    logits = np.zeros((cells, 5, 6 * B))
+    for c in range(cells):
+        x, z = data[c]
+        fakes = [g_forward(unflatten(state.Gw[nbr[c][i]], gl), z, a)["F"] for i in range(5)]
+        X = np.vstack([x] + fakes)
+        for j in range(5):
+            lg = d_forward(unflatten(state.Dw[nbr[c][j]], dl), X, a)["logit"]
+            logits[c, j] = lg
+            for i in range(5):
+                LG[c, i, j], LD[c, i, j] = pair_losses(lg[:B], lg[B * (i + 1):B * (i + 2)])
+    return {"LG": LG, "LD": LD, "fG": LG.mean(axis=2), "fD": LD.mean(axis=1), "logits": logits}
+
+
+# --------------------------------------------------------------------------------------------
+# Step 3a: tournament selection, replacement, learning-rate mutation.
+# --------------------------------------------------------------------------------------------
+def tournament(f5: np.ndarray, words: np.ndarray, size: int) -> int:
+    """Draw ``size`` distinct slots (entrant m is the mulhi(word_m, 5 - m)-th slot not yet drawn,
+    in ascending order) and return the entrant with the lowest fitness, the lower slot on a tie."""
+    if not 1 <= size <= 5:
+        raise ValueError("tournament size must be in 1..5")
+    remaining = [0, 1, 2, 3, 4]
+    entrants = [remaining.pop(int(mulhi(words[m], 5 - m))) for m in range(size)]
+    best = entrants[0]
+    for e in entrants[1:]:
+        if f5[e] < f5[best] or (f5[e] == f5[best] and e < best):
+            best = e
+    return best
+
+
+def select_slot(f5: np.ndarray, words: np.ndarray, arch: Arch) -> int:
+    """The slot whose individual becomes the new centre: the tournament winner if it is strictly
+    fitter than the centre (``if_better``) or unconditionally (``always``); else the centre."""
+    win = tournament(f5, words, arch.tournament_size)
+    if arch.replace_mode == "always":
+        return win
+    if arch.replace_mode != "if_better":
+        raise ValueError("replace_mode must be if_better or always")
+    return win if f5[win] < f5[0] else 0
+
+
+def mutate_lr(lr: float, seed: int, stream: int, t: int, cell: int, arch: Arch) -> float:
+    """Gaussian hyper-parameter update (step 3; Table 1 rate and probability): with probability
+    p (word0 < floor(p * 2^32)) add std * N(0, 1) (Box-Muller on word1, word2, cosine branch);
+    the result is kept >= 1e-8."""
+    w = draw_words(seed, stream, t, cell, 4)
+    thr = min(int(math.floor(arch.lr_mut_prob * 4294967296.0)), 4294967296)
+    if int(w[0]) >= thr:
+        return lr
+    n, _ = box_muller(w[1:2], w[2:3])
+    return max(lr + arch.lr_mut_std * float(n[0]), 1e-8)
+
+
+def select_replace(state: State, ev) -> Dict[str, np.ndarray]:
+    """Slots chosen for every cell's new centre generator and discriminator."""
+    a = state.arch
+    sel_g = np.zeros(state.cells, np.int64)
+    sel_d = np.zeros(state.cells, np.int64)
+    for c in range(state.cells):
+        sel_g[c] = select_slot(ev["fG"][c], draw_words(state.seed, STREAM_TOUR_G, state.t, c,
+                                                       a.tournament_size), a)
+        sel_d[c] = select_slot(ev["fD"][c], draw_words(state.seed, STREAM_TOUR_D, state.t, c,
+                                                       a.tournament_size), a)
+    return {"sel_g": sel_g, "sel_d": sel_d}
+
+
+# --------------------------------------------------------------------------------------------
+# Step 3b: gradients of the selected pair and the Adam update.
+# --------------------------------------------------------------------------------------------
+def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.ndarray,
+                   arch: Arch) -> Tuple[np.ndarray, np.ndarray, Dict[str, float]]:
+    """dL_D/dv (fake batch detached) and dL_G/du (through D at its pre-update parameters), by
+    the chain rule, layer by layer. Returns flat gradients in the parameter layouts."""
+    a = arch
+    rb = _Rounder(a)
+    gl, dl = g_layout(a), d_layout(a)
+    G, D = unflatten(Gflat, gl), unflatten(Dflat, dl)
+    B = x.shape[0]
+    fg = g_forward(G, z, a)
+    fd = d_forward(D, np.vstack([x, fg["F"]]), a)
+    logit = fd["logit"]
+    s = sigmoid(logit)
+    dl_d = np.concatenate([(s[:B] - 1.0) / B, s[B:] / B])   # dL_D / d logit, real then fake rows
+    dl_g = (s[B:] - 1.0) / B                                 # dL_G / d logit of fake rows
+    slope = a.leaky_slope
+
+    gD = {name: np.zeros(shape) for name, shape in dl}
+    gG = {name: np.zeros(shape) for name, shape in gl}
+    g1, g2, X = fd["g1"], fd["g2"], fd["X"]
+    # Rows of the discriminator chain: [real, fake (D loss), fake (G loss)].
+    dl3 = np.concatenate([dl_d, dl_g])
+    g2_3 = np.vstack([g2, g2[B:]])
+    g1_3 = np.vstack([g1, g1[B:]])
+    w3 = rb(D["W3"])[0]
+    gD["W3"][0] = dl_d @ g2
+    gD["b3"][0] = dl_d.sum()
+    d2 = rb(dl3[:, None] * w3[None, :] * np.where(g2_3 > 0.0, 1.0, slope))
+    gD["W2"][:] = d2[:2 * B].T @ g1
+    gD["b2"][:] = d2[:2 * B].sum(axis=0)
+    d1 = rb((d2 @ rb(D["W2"])) * np.where(g1_3 > 0.0, 1.0, slope))
+    gD["W1"][:] = d1[:2 * B].T @ X
+    gD["b1"][:] = d1[:2 * B].sum(axis=0)
+    # Generator chain: through D's first layer into the fakes, then back through G.
+    dF = d1[2 * B:] @ rb(D["W1"])
+    F, h2, h1, zq = fg["F"], fg["h2"], fg["h1"], fg["z"]
+    a3 = rb(dF * (1.0 - F * F))
+    gG["W3"][:] = a3.T @ h2
+    gG["b3"][:] = a3.sum(axis=0)
+    a2 = rb((a3 @ rb(G["W3"])) * (h2 > 0.0))
+    gG["W2"][:] = a2.T @ h1
+    gG["b2"][:] = a2.sum(axis=0)
+    a1 = rb((a2 @ rb(G["W2"])) * (h1 > 0.0))
+    gG["W1"][:] = a1.T @ zq
+    gG["b1"][:] = a1.sum(axis=0)
+    lg, ld = pair_losses(logit[:B], logit[B:])
+    flatG = np.concatenate([gG[n].reshape(-1) for n, _ in gl])
+    flatD = np.concatenate([gD[n].reshape(-1) for n, _ in dl])
+    return flatG, flatD, {"LG": lg, "LD": ld}
+
+
+def adam_step(w, m, v, step, g, lr, arch: Arch):
+    """One Adam update (Kingma & Ba 2015, Algorithm 1) with the individual's own step count."""
+    t1 = step + 1
+    m1 = arch.beta1 * m + (1.0 - arch.beta1) * g
+    v1 = arch.beta2 * v + (1.0 - arch.beta2) * g * g
+    mhat = m1 / (1.0 - arch.beta1 ** t1)
+    vhat = v1 / (1.0 - arch.beta2 ** t1)
+    return w - lr * mhat / (np.sqrt(vhat) + arch.eps), m1, v1, t1
+
+
+def train_step(state: State, sel, data, keep_grads: bool = False):
+    """Every cell's new centre pair (the selected slots' individuals with their optimiser state)
+    takes one Adam step on the cell's minibatch. Reads only the snapshot ``state``."""
+    a = state.arch
+    nbr = neighbors(state.rows, state.cols)
+    new = state.copy()
+    grads = {"gG": np.zeros_like(state.Gw), "gD": np.zeros_like(state.Dw)}
+    for c in range(state.cells):
+        sg = int(nbr[c][sel["sel_g"][c]])
+        sd = int(nbr[c][sel["sel_d"][c]])
+        lr_g, lr_d = float(state.Glr[sg]), float(state.Dlr[sd])
+        if a.lr_mutation:
+            lr_g = mutate_lr(lr_g, state.seed, STREAM_MUT_G, state.t, c, a)
+            lr_d = mutate_lr(lr_d, state.seed, STREAM_MUT_D, state.t, c, a)
+        x, z = data[c]
+        gG, gD, _ = pair_gradients(state.Gw[sg], state.Dw[sd], x, z, a)
+        new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c] = adam_step(
+            state.Gw[sg], state.Gm[sg], state.Gv[sg], state.Gstep[sg], gG, lr_g, a)
+        new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c] = adam_step(
+            state.Dw[sd], state.Dm[sd], state.Dv[sd], state.Dstep[sd], gD, lr_d, a)
+        new.Glr[c], new.Dlr[c] = lr_g, lr_d
+        grads["gG"][c], grads["gD"][c] = gG, gD
+    new.t = state.t + 1
+    return (new, grads) if keep_grads else new
+
+
+def iterate(state: State, pool: Optional[np.ndarray], n_iters: int = 1,
+            x_host: Optional[np.ndarray] = None, record: bool = False):
+    """Steps 2, 3 and 5: ``n_iters`` synchronous grid iterations. Returns the new state (and,
+    with ``record``, the per-iteration evaluations and selections)."""
+    log = []
+    for _ in range(n_iters):
+        data = batches(state, pool, x_host)
+        ev = eval_neighborhoods(state, data)
+        sel = select_replace(state, ev)
+        state = train_step(state, sel, data)
+        if record:
+            log.append({"eval": ev, "sel": sel})
+    return (state, log) if record else state
+
+
+# --------------------------------------------------------------------------------------------
+# State bytes: the engine's documented export layout (little-endian), so that a state can move
+# between the engine and the oracle.
+#   header (64 bytes): u32 magic 0x5A50494C ("LIPZ"), u32 version 1, i32 rows, i32 cols,
+#     i32 z_dim, i32 hidden, i32 x_dim, i32 batch, i32 precision (0 fp32, 1 bf16), i32 0,
+#     i64 t, u64 seed, 8 zero bytes
+#   then f32 Gw[cells][PG], Gm, Gv, Dw[cells][PD], Dm, Dv, i32 Gstep[cells], Dstep[cells],
+#     f32 Glr[cells], Dlr[cells].
+# --------------------------------------------------------------------------------------------
+_MAGIC = 0x5A50494C
+
+
+def state_to_bytes(s: State) -> bytes:
+    a = s.arch
+    hdr = np.zeros(16, dtype=np.uint32)
+    hdr[0], hdr[1] = _MAGIC, 1
+    hdr[2:10] = [s.rows, s.cols, a.z_dim, a.hidden, a.x_dim, a.batch,
+                 1 if a.precision == "bf16" else 0, 0]
+    h = hdr.tobytes()
+    h = h[:40] + np.array([s.t], np.int64).tobytes() + np.array([s.seed], np.uint64).tobytes() \
+        + bytes(8)
+    parts = [h] + [getattr(s, f).astype(np.float32).tobytes()
+                   for f in ("Gw", "Gm", "Gv", "Dw", "Dm", "Dv")]
+    parts += [s.Gstep.astype(np.int32).tobytes(), s.Dstep.astype(np.int32).tobytes(),
+              s.Glr.astype(np.float32).tobytes(), s.Dlr.astype(np.float32).tobytes()]
+    return b"".join(parts)
+
+
+def state_from_bytes(buf: bytes, arch: Arch) -> State:
+    hdr = np.frombuffer(buf[:40], dtype=np.int32)
+    if int(np.frombuffer(buf[:4], np.uint32)[0]) != _MAGIC:
+        raise ValueError("not a grid state")
+    rows, cols = int(hdr[2]), int(hdr[3])
+    if (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7])) != (arch.z_dim, arch.hidden,
+                                                              arch.x_dim, arch.batch):
+        raise ValueError("state does not match the architecture")
+    t = int(np.frombuffer(buf[40:48], np.int64)[0])
+    seed = int(np.frombuffer(buf[48:56], np.uint64)[0])
+    cells = rows * cols
+    PG, PD = n_params(g_layout(arch)), n_params(d_layout(arch))
+    off = 64
+    arrs = {}
+    for f, p in (("Gw", PG), ("Gm", PG), ("Gv", PG), ("Dw", PD), ("Dm", PD), ("Dv", PD)):
+        n = cells * p
+        arrs[f] = np.frombuffer(buf[off:off + 4 * n], np.float32).astype(np.float64).reshape(cells, p)
+        off += 4 * n
+    for f, dt in (("Gstep", np.int32), ("Dstep", np.int32), ("Glr", np.float32),
+                  ("Dlr", np.float32)):
+        v = np.frombuffer(buf[off:off + 4 * cells], dt)
+        arrs[f] = v.astype(np.int64 if dt == np.int32 else np.float64)
+        off += 4 * cells
+    if off != len(buf):
+        raise ValueError("state size mismatch")
+    return State(rows, cols, arch, seed, t, **arrs)
