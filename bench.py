@@ -1,0 +1,360 @@
+"""Throughput of the grid iteration: G-D pair evaluations per second and grid iterations per
+second on one GB300, with the roofline fraction of the dominant kernel, an end-to-end number
+through the C ABI with host buffers, and the CPU oracle timed on a bounded sample.
+
+Workload: 12x12 toroidal grid (144 cells, 720 neighbourhood slots, 3600 G-D pairs per
+iteration), MLP G (64-256-256-784) and D (784-256-256-1), bf16 operands with fp32 accumulation
+and fp32 Adam masters, minibatch 100, real data from a seeded 10-blob 784-dim pool. One step is
+one full grid iteration (minibatch draw, all-pairs evaluation, fitness, selection, backward and
+Adam of every cell's new centre pair).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (torchrun, one process per GPU) every rank runs its own 12x12 grid (replicas: the
+per-GPU work is fixed, scaling "weak"); value = all ranks' pairs / the slowest rank's time.
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+ROWS, COLS, BATCH = 12, 12, 100
+Z_DIM, HIDDEN, X_DIM = 64, 256, 784
+POOL_N, SEED = 60000, 1811
+CELLS = ROWS * COLS
+PAIRS = 25 * CELLS
+METRIC = "G-D pair evals/sec and grid iterations/sec on 1 GB300; % of bf16 tensor peak"
+UNIT = "pair-evals/s"
+WORKLOAD = "12x12 torus MLP G/D bf16 B=100 (3600 pairs/iter)"
+
+# Algorithmic work per iteration (no padding, no recomputation):
+#   evaluation: generator slots 5 B rows x (z*h + h*h + h*x) MACs per cell; discriminator slots
+#   5 * 6B rows x (x*h + h*h + h) MACs per cell.
+G_MAC_ROW = Z_DIM * HIDDEN + HIDDEN * HIDDEN + HIDDEN * X_DIM            # 282,624
+D_MAC_ROW = X_DIM * HIDDEN + HIDDEN * HIDDEN + HIDDEN                    # 266,496
+EVAL_G_FLOP = 2 * CELLS * 5 * BATCH * G_MAC_ROW
+EVAL_D_FLOP = 2 * CELLS * 30 * BATCH * D_MAC_ROW
+PG = HIDDEN * Z_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + X_DIM * HIDDEN + X_DIM
+PD = HIDDEN * X_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + HIDDEN + 1
+# Adam + replacement per parameter: read w, m, v, g (16 B), write w, m, v (12 B) + bf16 copy (2 B)
+ADAM_BYTES = CELLS * (PG + PD) * 30
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1900.0), \
+            d.get("bf16_tflops_sustained", 1700.0), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during a timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+        return False
+
+    def summary(self):
+        rows = [r.split(", ") for r in (self.out or "").strip().splitlines() if r.strip()]
+        rows = [r for r in rows if len(r) >= 9]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def _dist():
+    n = int(os.environ.get("WORLD_SIZE", "1"))
+    if n > 1:
+        import torch.distributed as dist
+        if not dist.is_initialized():
+            dist.init_process_group("nccl" if os.environ.get("LIPZ_BENCH_GLOO") is None else "gloo")
+        return dist, dist.get_rank(), n
+    return None, 0, 1
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    dist, rank, world = _dist()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import lipz_synth
+    import paper_1811_12843_gb300 as L
+
+    pool = lipz_synth.blob_pool(SEED, n=POOL_N, dim=X_DIM)
+    g = L.Grid(ROWS, COLS, seed=SEED + rank, precision="bf16", batch=BATCH)
+    g.set_data(pool)
+    stream = torch.cuda.Stream()
+    g.set_stream(stream.cuda_stream)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+
+    # warm-up
+    for _ in range(args.warmup):
+        L.lipz_iterate(g.h, 1)
+    g.synchronize()
+    L.lipz_profile_read(g.h)  # reset counters
+
+    # ---- timed region: K grid iterations on the grid's stream (device time)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    with Clocks(local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            L.lipz_iterate(g.h, 1)
+        e1.record(stream)
+        g.synchronize()
+    barrier()
+    ms = e0.elapsed_time(e1)
+    prof0 = L.lipz_profile_read(g.h)
+    launches = sum(v[2] for v in prof0.values())
+    t_max = ms
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_max = float(t.item())
+    ms_step = t_max / args.steps
+    iters_s = 1000.0 / ms_step
+    value = PAIRS * world * iters_s
+
+    # ---- per-phase device time (separate pass with phase events on the same stream)
+    L.lipz_profile_enable(g.h, True)
+    for _ in range(args.steps):
+        L.lipz_iterate(g.h, 1)
+    prof = L.lipz_profile_read(g.h)
+    L.lipz_profile_enable(g.h, False)
+    phase_ms = {k: v[0] / max(v[1], 1) for k, v in prof.items()}
+
+    # ---- end to end through the public API: pinned host minibatches in, fitness out
+    nbuf = 2
+    xs = [torch.from_numpy(lipz_synth.host_batch(SEED + 7 + i, CELLS, BATCH, X_DIM)).pin_memory()
+          for i in range(nbuf)]
+    fg = torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()
+    fd = torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()
+    for i in range(2):
+        L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
+    barrier()
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
+    e2e_s = time.perf_counter() - t0
+    if dist:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_value = PAIRS * world * args.steps / e2e_s
+    h2d = CELLS * BATCH * X_DIM * 4
+    d2h = 2 * CELLS * 5 * 4
+
+    # ---- roofline of the dominant kernel phase
+    hbm, tf_burst, tf_sus, peak_kind = _peaks()
+    dom = max(("g_fwd", "d_fwd", "train_fwd", "train_bwd", "adam"), key=lambda k: phase_ms[k])
+    if dom == "d_fwd":
+        ach = EVAL_D_FLOP / (phase_ms["d_fwd"] * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
+                "kernel": "discriminator evaluation forward (all 720 slots, fused 3 layers + logit)",
+                "algorithmic_flop_per_launch": EVAL_D_FLOP}
+    elif dom == "g_fwd":
+        ach = EVAL_G_FLOP / (phase_ms["g_fwd"] * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
+                "kernel": "generator evaluation forward (all 720 slots)",
+                "algorithmic_flop_per_launch": EVAL_G_FLOP}
+    elif dom == "adam":
+        ach = ADAM_BYTES / (phase_ms["adam"] * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                "kernel": "fused Adam + replacement", "algorithmic_bytes_per_launch": ADAM_BYTES}
+    else:
+        flop = 2 * CELLS * BATCH * (G_MAC_ROW - HIDDEN * X_DIM) + 2 * CELLS * 2 * BATCH * D_MAC_ROW \
+            if dom == "train_fwd" else 2 * CELLS * BATCH * 1479936
+        ach = flop / (phase_ms[dom] * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
+                "kernel": "selected-pair " + dom.replace("_", " "),
+                "algorithmic_flop_per_launch": flop}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["peak_source"] = peak_kind + (" sustained bf16" if roof["unit"] == "TFLOP/s" else " HBM copy")
+    roof["traffic"] = None
+    roof["phase"] = dom
+
+    if rank != 0:
+        return None
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
+        "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+                   "pairs_per_iter": PAIRS, "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (population 2.2 GB + pool 188 MB per iteration)"},
+        "grid_iterations_per_sec": iters_s * world,
+        "pair_evals_per_sec_eval_only": PAIRS * world * 1000.0 /
+        (phase_ms["batch"] + phase_ms["g_fwd"] + phase_ms["d_fwd"] + phase_ms["fitness"]),
+        "phase_ms": phase_ms,
+        "roofline": roof,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+    return line
+
+
+def _oracle_sample(seconds, max_cells=None):
+    """Run the oracle's full iteration cell by cell on the 12x12 workload until ``seconds`` of
+    CPU work are spent; return (cells done, elapsed seconds)."""
+    import numpy as np
+    import lipz_synth
+    from oracle import lipz_oracle as O
+
+    pool = lipz_synth.blob_pool(SEED, n=POOL_N, dim=X_DIM)
+    arch = O.Arch(precision="bf16", batch=BATCH)
+    # a state for the whole grid (initialisation is not part of the timed sample)
+    state = _oracle_state(arch)
+    nbr = O.neighbors(ROWS, COLS)
+    done, t0 = 0, time.perf_counter()
+    c = 0
+    while True:
+        cells = [c]
+        data = O.batches(state, pool, cells=cells)
+        ev = O.eval_neighborhoods(state, data, cells=cells)
+        a = state.arch
+        sg = O.select_slot(ev["fG"][c], O.draw_words(state.seed, O.STREAM_TOUR_G, state.t, c,
+                                                     a.tournament_size), a)
+        sd = O.select_slot(ev["fD"][c], O.draw_words(state.seed, O.STREAM_TOUR_D, state.t, c,
+                                                     a.tournament_size), a)
+        x, z = data[c]
+        gG, gD, _ = O.pair_gradients(state.Gw[nbr[c][sg]], state.Dw[nbr[c][sd]], x, z, a)
+        O.adam_step(state.Gw[nbr[c][sg]], state.Gm[nbr[c][sg]], state.Gv[nbr[c][sg]], 0, gG,
+                    a.lr, a)
+        O.adam_step(state.Dw[nbr[c][sd]], state.Dm[nbr[c][sd]], state.Dv[nbr[c][sd]], 0, gD,
+                    a.lr, a)
+        done += 1
+        c = (c + 1) % CELLS
+        el = time.perf_counter() - t0
+        if el >= seconds or (max_cells and done >= max_cells):
+            return done, el
+
+
+_STATE_CACHE = {}
+
+
+def _oracle_state(arch):
+    """Oracle grid state for the workload: Xavier weights from the seed (cells drawn lazily would
+    change nothing: every cell's weights come from its own Philox stream)."""
+    from oracle import lipz_oracle as O
+    if "s" not in _STATE_CACHE:
+        _STATE_CACHE["s"] = O.create(ROWS, COLS, arch, SEED)
+    return _STATE_CACHE["s"]
+
+
+def _threads():
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(k):
+            return int(os.environ[k])
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(seconds):
+    done, el = _oracle_sample(seconds)
+    return {"value": 25.0 * done / el, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+            "sample": "%d cells of the 12x12 bf16 B=100 workload (eval of 25 pairs + selection + "
+                      "gradients + Adam per cell), %.1f s, numpy float64 + OpenBLAS" % (done, el)}
+
+
+def run_reference(args):
+    _, rank, world = _dist()
+    if rank != 0:
+        return None
+    from oracle import lipz_oracle as O
+    arch = O.Arch(precision="bf16", batch=BATCH)
+    _oracle_state(arch)
+    per_step_cells = 2
+    for _ in range(args.warmup):
+        _oracle_sample(1e9, max_cells=1)
+    times = []
+    total_cells = 0
+    for _ in range(args.steps):
+        done, el = _oracle_sample(1e9, max_cells=per_step_cells)
+        times.append(el)
+        total_cells += done
+    el = sum(times)
+    value = 25.0 * total_cells / el
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
+            "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+                       "pairs_per_iter": PAIRS, "parallelism": "cpu"},
+            "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+                             "sample": "%d cells per step of the 12x12 bf16 B=100 workload"
+                                       % per_step_cells},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

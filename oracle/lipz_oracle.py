@@ -332,13 +332,17 @@ def draw_batch(seed: int, t: int, cell: int, pool: np.ndarray, arch: Arch
     return x, z.reshape(arch.batch, arch.z_dim)
 
 
-def batches(state: State, pool: Optional[np.ndarray], x_host: Optional[np.ndarray] = None):
+def batches(state: State, pool: Optional[np.ndarray], x_host: Optional[np.ndarray] = None,
+            cells=None):
     """Per-cell (x, z) for the state's current iteration. ``x_host`` ([cells, B, x_dim]) replaces
-    the pool draw when the caller supplies the real minibatches itself."""
+    the pool draw when the caller supplies the real minibatches itself. With ``cells``, only
+    those cells' batches are drawn (the others are None)."""
     a = state.arch
     out = []
     for c in range(state.cells):
-        if x_host is not None:
+        if cells is not None and c not in cells:
+            out.append(None)
+        elif x_host is not None:
             z = draw_normals(state.seed, STREAM_NOISE, state.t, c, a.batch * a.z_dim)
             out.append((np.asarray(x_host[c], np.float64), z.reshape(a.batch, a.z_dim)))
         else:
@@ -349,19 +353,20 @@ def batches(state: State, pool: Optional[np.ndarray], x_host: Optional[np.ndarra
 # --------------------------------------------------------------------------------------------
 # Step 2: all-pairs evaluation and fitness.
 # --------------------------------------------------------------------------------------------
-def eval_neighborhoods(state: State, data) -> Dict[str, np.ndarray]:
+def eval_neighborhoods(state: State, data, cells=None) -> Dict[str, np.ndarray]:
     """For each cell c and slots (i, j): generator nbr[c][i] against discriminator nbr[c][j] on
     cell c's minibatch. Returns L_G, L_D [cells, 5(i), 5(j)], fitness f_G = mean_j L_G[c, i, :],
     f_D = mean_i L_D[c, :, j], and the logits [cells, 5(j), 6B] (real rows, then the fakes of
-    generator slots 0..4)."""
+    generator slots 0..4). With ``cells``, only those cells are evaluated (others stay 0)."""
     a = state.arch
     gl, dl = g_layout(a), d_layout(a)
     nbr = neighbors(state.rows, state.cols)
+    only = cells
     cells, B = state.cells, a.batch
     LG = np.zeros((cells, 5, 5))
     LD = np.zeros((cells, 5, 5))
     logits = np.zeros((cells, 5, 6 * B))
-    for c in range(cells):
+    for c in (range(cells) if only is None else only):
         x, z = data[c]
         fakes = [g_forward(unflatten(state.Gw[nbr[c][i]], gl), z, a)["F"] for i in range(5)]
         X = np.vstack([x] + fakes)

@@ -1,0 +1,1041 @@
+// C ABI and host scheduler of the grid-iteration engine (declared in include/lipz.h).
+//
+// The grid owns two population snapshots per population (ping-pong A/B): an iteration reads
+// snapshot `cur` (evaluation, selection, gradients) and writes every cell's new centre into
+// snapshot 1 - cur, so no cell can see a neighbour's half-updated state. Work is enqueued on
+// one CUDA stream; the host waits only when the caller asks for host-side results.
+#include <climits>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "engine.h"
+#include "fwd_tc.h"
+#include "lipz.h"
+
+using namespace lipz;
+
+namespace {
+
+enum Phase { PH_IDLE = 0, PH_EVALUATED = 1, PH_SELECTED = 2 };
+
+thread_local std::string t_create_err;
+
+struct Descs {
+  // evaluation (per parity of the snapshot): generator layers over (cell, slot i),
+  // discriminator layers over (cell, slot j)
+  GemmDesc *g1, *g2, *g3, *d1, *d2;
+  GemvDesc* d3;
+  // training (per parity): forward of the selected pair and its backward
+  GemmDesc *tg1, *tg2, *td1, *td2, *bw2d, *bd1, *bw1d, *ba3, *bw3g, *ba2, *bw2g, *ba1, *bw1g;
+  GemvDesc* tgv;
+  ColSumDesc *cb2d, *cb1d, *cb3g, *cb2g, *cb1g;
+};
+
+}  // namespace
+
+struct lipz_grid {
+  int rows = 0, cols = 0, cells = 0;
+  lipz_arch a{};
+  uint64_t seed = 0;
+  int64_t t = 0;
+  bool bf = false;
+  size_t esz = 4;
+  Layout lg{}, ld{};
+  int64_t PG = 0, PD = 0, PGs = 0, PDs = 0;
+  int64_t e_cell = 0;  // elements per cell of the evaluation input E (6B rows)
+  cudaStream_t st = nullptr;
+  int device = 0;
+  PopView G[2]{}, D[2]{};
+  int cur = 0;
+  int phase = PH_IDLE;
+  bool use_tc = false;
+  std::vector<void*> allocs;
+  std::string err;
+
+  // data and work buffers
+  float* pool = nullptr;
+  int64_t pool_n = 0, pool_cap = 0;
+  float* xin = nullptr;  // caller-supplied minibatch staging [cells][B][x_dim]
+  void *Z = nullptr, *E = nullptr, *H1g = nullptr, *H2g = nullptr, *H1d = nullptr, *H2d = nullptr;
+  float *logits = nullptr, *LG = nullptr, *LD = nullptr, *fG = nullptr, *fD = nullptr;
+  int *nbr = nullptr, *sel_g = nullptr, *sel_d = nullptr, *src_g = nullptr, *src_d = nullptr;
+  float *lrn_g = nullptr, *lrn_d = nullptr;
+  void *TH1 = nullptr, *TH2 = nullptr, *TX = nullptr, *TG1 = nullptr, *TG2 = nullptr;
+  float* TL = nullptr;
+  void *J2 = nullptr, *D1 = nullptr, *A3 = nullptr, *A2 = nullptr, *A1 = nullptr;
+  float *gG = nullptr, *gD = nullptr;
+  int* flag = nullptr;
+  Descs dsc[2]{};
+  TcPlan* tc[2]{};
+
+  // tracing: event pairs per phase execution, resolved at lipz_profile_read
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_free;
+  struct Mark {
+    int phase;
+    cudaEvent_t a, b;
+  };
+  std::vector<Mark> marks;
+  cudaEvent_t open_ev[LIPZ_N_PHASES]{};
+  int64_t launches[LIPZ_N_PHASES]{};
+  int64_t counts[LIPZ_N_PHASES]{};
+};
+
+namespace {
+
+int fail(lipz_grid* g, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (g) g->err = buf;
+  else t_create_err = buf;
+  return code;
+}
+
+#define CK(g, call)                                                                   \
+  do {                                                                                \
+    cudaError_t e_ = (call);                                                          \
+    if (e_ != cudaSuccess)                                                            \
+      return fail((g), e_ == cudaErrorMemoryAllocation ? LIPZ_ERR_OOM : LIPZ_ERR_CUDA, \
+                  "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__,   \
+                  __LINE__);                                                          \
+  } while (0)
+
+#define CKL(g)                                                                               \
+  do {                                                                                       \
+    cudaError_t e_ = cudaGetLastError();                                                     \
+    if (e_ != cudaSuccess)                                                                   \
+      return fail((g), LIPZ_ERR_CUDA, "kernel launch failed: %s (%s:%d)", cudaGetErrorString(e_), \
+                  __FILE__, __LINE__);                                                       \
+  } while (0)
+
+template <typename T>
+int dalloc(lipz_grid* g, T** p, size_t bytes) {
+  void* q = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(&q, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(g, e == cudaErrorMemoryAllocation ? LIPZ_ERR_OOM : LIPZ_ERR_CUDA,
+                "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+  }
+  g->allocs.push_back(q);
+  *p = (T*)q;
+  return LIPZ_OK;
+}
+
+cudaEvent_t take_event(lipz_grid* g) {
+  if (!g->ev_free.empty()) {
+    cudaEvent_t e = g->ev_free.back();
+    g->ev_free.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return e;
+}
+
+void phase_begin(lipz_grid* g, int ph) {
+  if (!g->prof) return;
+  cudaEvent_t e = take_event(g);
+  if (e) cudaEventRecord(e, g->st);
+  g->open_ev[ph] = e;
+}
+
+// Closes a phase: counts its kernel launches and, when tracing, records its stop event.
+void phase_end(lipz_grid* g, int ph, int n_launches) {
+  g->launches[ph] += n_launches;
+  g->counts[ph] += 1;
+  if (!g->prof || !g->open_ev[ph]) return;
+  cudaEvent_t e = take_event(g);
+  if (!e) return;
+  cudaEventRecord(e, g->st);
+  g->marks.push_back({ph, g->open_ev[ph], e});
+  g->open_ev[ph] = nullptr;
+}
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+// Layouts (PyTorch Linear convention, W [out][in] row-major).
+void make_layouts(lipz_grid* g) {
+  const int64_t z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
+  auto build = [](Layout& L, const int64_t shapes[6][2]) {
+    L.n = 6;
+    L.off[0] = 0;
+    for (int t = 0; t < 6; ++t) {
+      L.off[t + 1] = L.off[t] + shapes[t][0] * shapes[t][1];
+      L.bound[t] = (t % 2 == 0)
+                       ? (float)std::sqrt(6.0 / (double)(shapes[t][0] + shapes[t][1]))
+                       : 0.f;
+    }
+  };
+  const int64_t gs[6][2] = {{h, z}, {1, h}, {h, h}, {1, h}, {x, h}, {1, x}};
+  const int64_t ds[6][2] = {{h, x}, {1, h}, {h, h}, {1, h}, {1, h}, {1, 1}};
+  build(g->lg, gs);
+  build(g->ld, ds);
+  g->PG = g->lg.off[6];
+  g->PD = g->ld.off[6];
+  g->PGs = round_up(g->PG, 64);
+  g->PDs = round_up(g->PD, 64);
+}
+
+const void* act_w(const PopView& p) { return p.wb ? (const void*)p.wb : (const void*)p.w; }
+
+char* eoff(const void* base, int64_t elems, size_t esz) {
+  return (char*)base + elems * (int64_t)esz;
+}
+
+GemmDesc gd(const void* A, int64_t sam, int64_t sak, const void* B, int64_t sbk, int64_t sbn,
+            void* C, int64_t scm, int64_t scn, int M, int N, int K) {
+  GemmDesc d;
+  memset(&d, 0, sizeof d);
+  d.A = A;
+  d.B = B;
+  d.C = C;
+  d.sam = sam;
+  d.sak = sak;
+  d.sbk = sbk;
+  d.sbn = sbn;
+  d.scm = scm;
+  d.scn = scn;
+  d.M = M;
+  d.N = N;
+  d.K = K;
+  return d;
+}
+
+template <typename T>
+int upload(lipz_grid* g, T** dst, const std::vector<T>& v) {
+  int rc = dalloc(g, dst, v.size() * sizeof(T));
+  if (rc) return rc;
+  CK(g, cudaMemcpy(*dst, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice));
+  return LIPZ_OK;
+}
+
+int build_descs(lipz_grid* g, int p) {
+  const int C = g->cells, B = g->a.batch, z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
+  const size_t es = g->esz;
+  const PopView &Gp = g->G[p], &Dp = g->D[p];
+  const void* Gw = act_w(Gp);
+  const void* Dw = act_w(Dp);
+  const Layout &L = g->lg, &M = g->ld;
+  std::vector<int> nbr(C * 5);
+  for (int r = 0; r < g->rows; ++r)
+    for (int q = 0; q < g->cols; ++q) {
+      int* n = &nbr[(r * g->cols + q) * 5];
+      n[0] = r * g->cols + q;
+      n[1] = ((r - 1 + g->rows) % g->rows) * g->cols + q;
+      n[2] = ((r + 1) % g->rows) * g->cols + q;
+      n[3] = r * g->cols + (q - 1 + g->cols) % g->cols;
+      n[4] = r * g->cols + (q + 1) % g->cols;
+    }
+  std::vector<GemmDesc> g1, g2, g3, d1, d2;
+  std::vector<GemvDesc> d3;
+  for (int c = 0; c < C; ++c)
+    for (int s = 0; s < 5; ++s) {
+      const int k = nbr[c * 5 + s];
+      const int64_t pg = (int64_t)k * g->PGs, pd = (int64_t)k * g->PDs;
+      const int64_t cs = (int64_t)c * 5 + s;
+      GemmDesc a = gd(eoff(g->Z, (int64_t)c * B * z, es), z, 1, eoff(Gw, pg + L.off[0], es), 1, z,
+                      eoff(g->H1g, cs * B * h, es), h, 1, B, h, z);
+      a.bias = Gp.w + pg + L.off[1];
+      g1.push_back(a);
+      GemmDesc b = gd(eoff(g->H1g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[2], es), 1, h,
+                      eoff(g->H2g, cs * B * h, es), h, 1, B, h, h);
+      b.bias = Gp.w + pg + L.off[3];
+      g2.push_back(b);
+      GemmDesc e = gd(eoff(g->H2g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[4], es), 1, h,
+                      eoff(g->E, (int64_t)c * g->e_cell + (int64_t)(1 + s) * B * x, es), x, 1, B,
+                      x, h);
+      e.bias = Gp.w + pg + L.off[5];
+      g3.push_back(e);
+      GemmDesc f = gd(eoff(g->E, (int64_t)c * g->e_cell, es), x, 1, eoff(Dw, pd + M.off[0], es), 1,
+                      x, eoff(g->H1d, cs * 6 * B * h, es), h, 1, 6 * B, h, x);
+      f.bias = Dp.w + pd + M.off[1];
+      d1.push_back(f);
+      GemmDesc q2 = gd(eoff(g->H1d, cs * 6 * B * h, es), h, 1, eoff(Dw, pd + M.off[2], es), 1, h,
+                       eoff(g->H2d, cs * 6 * B * h, es), h, 1, 6 * B, h, h);
+      q2.bias = Dp.w + pd + M.off[3];
+      d2.push_back(q2);
+      GemvDesc v;
+      memset(&v, 0, sizeof v);
+      v.X = eoff(g->H2d, cs * 6 * B * h, es);
+      v.w = eoff(Dw, pd + M.off[4], es);
+      v.bias = Dp.w + pd + M.off[5];
+      v.out = g->logits + cs * 6 * B;
+      v.ld = h;
+      v.rows = 6 * B;
+      v.K = h;
+      d3.push_back(v);
+    }
+  if (p == 0) {
+    int rc = upload(g, &g->nbr, nbr);
+    if (rc) return rc;
+  }
+  Descs& D = g->dsc[p];
+  int rc;
+  if ((rc = upload(g, &D.g1, g1)) || (rc = upload(g, &D.g2, g2)) || (rc = upload(g, &D.g3, g3)) ||
+      (rc = upload(g, &D.d1, d1)) || (rc = upload(g, &D.d2, d2)) || (rc = upload(g, &D.d3, d3)))
+    return rc;
+
+  // ---- training descriptors: weights of the selected individual (wsel = src_g / src_d)
+  std::vector<GemmDesc> tg1, tg2, td1, td2, bw2d, bd1, bw1d, ba3, bw3g, ba2, bw2g, ba1, bw1g;
+  std::vector<GemvDesc> tgv;
+  std::vector<ColSumDesc> cb2d, cb1d, cb3g, cb2g, cb1g;
+  auto selg = [&](GemmDesc d, int c) {
+    d.wsel = g->src_g;
+    d.wsel_stride = g->PGs;
+    d.wsel_op = 2;
+    d.cell = c;
+    return d;
+  };
+  auto seld = [&](GemmDesc d, int c) {
+    d.wsel = g->src_d;
+    d.wsel_stride = g->PDs;
+    d.wsel_op = 2;
+    d.cell = c;
+    return d;
+  };
+  auto cs = [](const void* X, float* out, int64_t ld, int rows, int cols) {
+    ColSumDesc d;
+    d.X = X;
+    d.out = out;
+    d.ld = ld;
+    d.rows = rows;
+    d.cols = cols;
+    return d;
+  };
+  for (int c = 0; c < C; ++c) {
+    const void* Zc = eoff(g->Z, (int64_t)c * B * z, es);
+    void* TH1c = eoff(g->TH1, (int64_t)c * B * h, es);
+    void* TH2c = eoff(g->TH2, (int64_t)c * B * h, es);
+    void* TXc = eoff(g->TX, (int64_t)c * 2 * B * x, es);
+    void* TG1c = eoff(g->TG1, (int64_t)c * 2 * B * h, es);
+    void* TG2c = eoff(g->TG2, (int64_t)c * 2 * B * h, es);
+    void* J2c = eoff(g->J2, (int64_t)c * 3 * B * h, es);
+    void* D1c = eoff(g->D1, (int64_t)c * 3 * B * h, es);
+    void* A3c = eoff(g->A3, (int64_t)c * B * x, es);
+    void* A2c = eoff(g->A2, (int64_t)c * B * h, es);
+    void* A1c = eoff(g->A1, (int64_t)c * B * h, es);
+    float* gGc = g->gG + (int64_t)c * g->PGs;
+    float* gDc = g->gD + (int64_t)c * g->PDs;
+
+    GemmDesc a = selg(gd(Zc, z, 1, eoff(Gw, L.off[0], es), 1, z, TH1c, h, 1, B, h, z), c);
+    a.bias = Gp.w + L.off[1];
+    tg1.push_back(a);
+    a = selg(gd(TH1c, h, 1, eoff(Gw, L.off[2], es), 1, h, TH2c, h, 1, B, h, h), c);
+    a.bias = Gp.w + L.off[3];
+    tg2.push_back(a);
+    a = seld(gd(TXc, x, 1, eoff(Dw, M.off[0], es), 1, x, TG1c, h, 1, 2 * B, h, x), c);
+    a.bias = Dp.w + M.off[1];
+    td1.push_back(a);
+    a = seld(gd(TG1c, h, 1, eoff(Dw, M.off[2], es), 1, h, TG2c, h, 1, 2 * B, h, h), c);
+    a.bias = Dp.w + M.off[3];
+    td2.push_back(a);
+    GemvDesc v;
+    memset(&v, 0, sizeof v);
+    v.X = TG2c;
+    v.w = eoff(Dw, M.off[4], es);
+    v.bias = Dp.w + M.off[5];
+    v.out = g->TL + (int64_t)c * 2 * B;
+    v.wsel = g->src_d;
+    v.wsel_stride = g->PDs;
+    v.cell = c;
+    v.ld = h;
+    v.rows = 2 * B;
+    v.K = h;
+    tgv.push_back(v);
+    // discriminator backward
+    bw2d.push_back(gd(J2c, 1, h, TG1c, h, 1, gDc + M.off[2], h, 1, h, h, 2 * B));
+    cb2d.push_back(cs(J2c, gDc + M.off[3], h, 2 * B, h));
+    a = seld(gd(J2c, h, 1, eoff(Dw, M.off[2], es), h, 1, D1c, h, 1, 2 * B, h, h), c);
+    a.aux = TG1c;
+    a.sxm = h;
+    a.sxn = 1;
+    bd1.push_back(a);
+    a = seld(gd(eoff(J2c, 2 * (int64_t)B * h, es), h, 1, eoff(Dw, M.off[2], es), h, 1,
+                eoff(D1c, 2 * (int64_t)B * h, es), h, 1, B, h, h), c);
+    a.aux = eoff(TG1c, (int64_t)B * h, es);
+    a.sxm = h;
+    a.sxn = 1;
+    bd1.push_back(a);
+    bw1d.push_back(gd(D1c, 1, h, TXc, x, 1, gDc + M.off[0], x, 1, h, x, 2 * B));
+    cb1d.push_back(cs(D1c, gDc + M.off[1], h, 2 * B, h));
+    // generator backward: into the fakes through D's first layer, then through G
+    a = seld(gd(eoff(D1c, 2 * (int64_t)B * h, es), h, 1, eoff(Dw, M.off[0], es), x, 1, A3c, x, 1,
+                B, x, h), c);
+    a.aux = eoff(TXc, (int64_t)B * x, es);
+    a.sxm = x;
+    a.sxn = 1;
+    ba3.push_back(a);
+    bw3g.push_back(gd(A3c, 1, x, TH2c, h, 1, gGc + L.off[4], h, 1, x, h, B));
+    cb3g.push_back(cs(A3c, gGc + L.off[5], x, B, x));
+    a = selg(gd(A3c, x, 1, eoff(Gw, L.off[4], es), h, 1, A2c, h, 1, B, h, x), c);
+    a.aux = TH2c;
+    a.sxm = h;
+    a.sxn = 1;
+    ba2.push_back(a);
+    bw2g.push_back(gd(A2c, 1, h, TH1c, h, 1, gGc + L.off[2], h, 1, h, h, B));
+    cb2g.push_back(cs(A2c, gGc + L.off[3], h, B, h));
+    a = selg(gd(A2c, h, 1, eoff(Gw, L.off[2], es), h, 1, A1c, h, 1, B, h, h), c);
+    a.aux = TH1c;
+    a.sxm = h;
+    a.sxn = 1;
+    ba1.push_back(a);
+    bw1g.push_back(gd(A1c, 1, h, Zc, z, 1, gGc + L.off[0], z, 1, h, z, B));
+    cb1g.push_back(cs(A1c, gGc + L.off[1], h, B, h));
+  }
+  if ((rc = upload(g, &D.tg1, tg1)) || (rc = upload(g, &D.tg2, tg2)) ||
+      (rc = upload(g, &D.td1, td1)) || (rc = upload(g, &D.td2, td2)) ||
+      (rc = upload(g, &D.tgv, tgv)) || (rc = upload(g, &D.bw2d, bw2d)) ||
+      (rc = upload(g, &D.bd1, bd1)) || (rc = upload(g, &D.bw1d, bw1d)) ||
+      (rc = upload(g, &D.ba3, ba3)) || (rc = upload(g, &D.bw3g, bw3g)) ||
+      (rc = upload(g, &D.ba2, ba2)) || (rc = upload(g, &D.bw2g, bw2g)) ||
+      (rc = upload(g, &D.ba1, ba1)) || (rc = upload(g, &D.bw1g, bw1g)) ||
+      (rc = upload(g, &D.cb2d, cb2d)) || (rc = upload(g, &D.cb1d, cb1d)) ||
+      (rc = upload(g, &D.cb3g, cb3g)) || (rc = upload(g, &D.cb2g, cb2g)) ||
+      (rc = upload(g, &D.cb1g, cb1g)))
+    return rc;
+  return LIPZ_OK;
+}
+
+// Grouped GEMM in the grid's precision; out_f32 selects an fp32 output (gradients).
+void gemm(lipz_grid* g, const GemmDesc* d, int n, int M, int N, int epi, int act, bool out_f32) {
+  const float sl = g->a.leaky_slope;
+  if (g->bf) {
+    if (out_f32) launch_gemm<bf16, float, EPI_STORE>(d, n, M, N, act, sl, g->st);
+    else if (epi == EPI_BIAS_ACT) launch_gemm<bf16, bf16, EPI_BIAS_ACT>(d, n, M, N, act, sl, g->st);
+    else launch_gemm<bf16, bf16, EPI_DACT>(d, n, M, N, act, sl, g->st);
+  } else {
+    if (out_f32 && epi == EPI_STORE) launch_gemm<float, float, EPI_STORE>(d, n, M, N, act, sl, g->st);
+    else if (epi == EPI_BIAS_ACT) launch_gemm<float, float, EPI_BIAS_ACT>(d, n, M, N, act, sl, g->st);
+    else launch_gemm<float, float, EPI_DACT>(d, n, M, N, act, sl, g->st);
+  }
+}
+
+void gemv(lipz_grid* g, const GemvDesc* d, int n, int rows) {
+  if (g->bf) launch_gemv<bf16>(d, n, rows, g->st);
+  else launch_gemv<float>(d, n, rows, g->st);
+}
+
+void colsum(lipz_grid* g, const ColSumDesc* d, int n, int cols) {
+  if (g->bf) launch_colsum<bf16>(d, n, cols, g->st);
+  else launch_colsum<float>(d, n, cols, g->st);
+}
+
+int check_arch(const lipz_arch* a) {
+  if (!a) return fail(nullptr, LIPZ_ERR_INVALID, "arch is null");
+  if (a->struct_size != sizeof(lipz_arch))
+    return fail(nullptr, LIPZ_ERR_INVALID, "arch.struct_size is %u, expected %zu", a->struct_size,
+                sizeof(lipz_arch));
+  if (a->kind != LIPZ_MLP) return fail(nullptr, LIPZ_ERR_INVALID, "arch.kind must be LIPZ_MLP");
+  if (a->precision != LIPZ_FP32 && a->precision != LIPZ_BF16)
+    return fail(nullptr, LIPZ_ERR_INVALID, "arch.precision must be LIPZ_FP32 or LIPZ_BF16");
+  if (a->z_dim < 1 || a->hidden < 1 || a->x_dim < 1 || a->batch < 1 || a->hidden > 1024 ||
+      a->batch > 4096 || a->z_dim > 65536 || a->x_dim > 65536)
+    return fail(nullptr, LIPZ_ERR_INVALID, "arch sizes out of range");
+  if (a->tournament_size < 1 || a->tournament_size > 5)
+    return fail(nullptr, LIPZ_ERR_INVALID, "tournament_size must be in 1..5");
+  if (a->replace_mode != LIPZ_REPLACE_IF_BETTER && a->replace_mode != LIPZ_REPLACE_ALWAYS)
+    return fail(nullptr, LIPZ_ERR_INVALID, "bad replace_mode");
+  if (!(a->lr >= 0.f) || !(a->beta1 >= 0.f && a->beta1 < 1.f) ||
+      !(a->beta2 >= 0.f && a->beta2 < 1.f) || !(a->eps > 0.f) || !(a->lr_mut_prob >= 0.f) ||
+      !(a->lr_mut_prob <= 1.f))
+    return fail(nullptr, LIPZ_ERR_INVALID, "bad optimiser / mutation hyper-parameters");
+  return LIPZ_OK;
+}
+
+int alloc_pop(lipz_grid* g, PopView* p, int64_t Ps) {
+  const size_t n = (size_t)g->cells * Ps;
+  int rc;
+  if ((rc = dalloc(g, &p->w, n * 4)) || (rc = dalloc(g, &p->m, n * 4)) ||
+      (rc = dalloc(g, &p->v, n * 4)) || (rc = dalloc(g, &p->step, g->cells * 4)) ||
+      (rc = dalloc(g, &p->lr, g->cells * 4)))
+    return rc;
+  p->wb = nullptr;
+  if (g->bf && (rc = dalloc(g, &p->wb, n * 2))) return rc;
+  CK(g, cudaMemset(p->w, 0, n * 4));
+  CK(g, cudaMemset(p->m, 0, n * 4));
+  CK(g, cudaMemset(p->v, 0, n * 4));
+  CK(g, cudaMemset(p->step, 0, g->cells * 4));
+  if (p->wb) CK(g, cudaMemset(p->wb, 0, n * 2));
+  return LIPZ_OK;
+}
+
+int create_impl(lipz_grid* g) {
+  const int C = g->cells, B = g->a.batch, z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
+  const size_t es = g->esz;
+  int rc;
+  CK(g, cudaGetDevice(&g->device));
+  make_layouts(g);
+  g->e_cell = (int64_t)6 * B * x;
+  for (int p = 0; p < 2; ++p) {
+    if ((rc = alloc_pop(g, &g->G[p], g->PGs)) || (rc = alloc_pop(g, &g->D[p], g->PDs))) return rc;
+  }
+  const size_t CB = (size_t)C * B;
+  if ((rc = dalloc(g, &g->Z, CB * z * es)) || (rc = dalloc(g, &g->E, (size_t)C * g->e_cell * es)) ||
+      (rc = dalloc(g, &g->H1g, CB * 5 * h * es)) || (rc = dalloc(g, &g->H2g, CB * 5 * h * es)) ||
+      (rc = dalloc(g, &g->H1d, CB * 30 * h * es)) || (rc = dalloc(g, &g->H2d, CB * 30 * h * es)) ||
+      (rc = dalloc(g, &g->logits, CB * 30 * 4)) || (rc = dalloc(g, &g->LG, C * 25 * 4)) ||
+      (rc = dalloc(g, &g->LD, C * 25 * 4)) || (rc = dalloc(g, &g->fG, C * 5 * 4)) ||
+      (rc = dalloc(g, &g->fD, C * 5 * 4)) || (rc = dalloc(g, &g->sel_g, C * 4)) ||
+      (rc = dalloc(g, &g->sel_d, C * 4)) || (rc = dalloc(g, &g->src_g, C * 4)) ||
+      (rc = dalloc(g, &g->src_d, C * 4)) || (rc = dalloc(g, &g->lrn_g, C * 4)) ||
+      (rc = dalloc(g, &g->lrn_d, C * 4)) || (rc = dalloc(g, &g->TH1, CB * h * es)) ||
+      (rc = dalloc(g, &g->TH2, CB * h * es)) || (rc = dalloc(g, &g->TX, CB * 2 * x * es)) ||
+      (rc = dalloc(g, &g->TG1, CB * 2 * h * es)) || (rc = dalloc(g, &g->TG2, CB * 2 * h * es)) ||
+      (rc = dalloc(g, &g->TL, CB * 2 * 4)) || (rc = dalloc(g, &g->J2, CB * 3 * h * es)) ||
+      (rc = dalloc(g, &g->D1, CB * 3 * h * es)) || (rc = dalloc(g, &g->A3, CB * x * es)) ||
+      (rc = dalloc(g, &g->A2, CB * h * es)) || (rc = dalloc(g, &g->A1, CB * h * es)) ||
+      (rc = dalloc(g, &g->gG, (size_t)C * g->PGs * 4)) ||
+      (rc = dalloc(g, &g->gD, (size_t)C * g->PDs * 4)) || (rc = dalloc(g, &g->flag, 4)) ||
+      (rc = dalloc(g, &g->xin, CB * x * 4)))
+    return rc;
+  CK(g, cudaMemset(g->gG, 0, (size_t)C * g->PGs * 4));
+  CK(g, cudaMemset(g->gD, 0, (size_t)C * g->PDs * 4));
+  const int big = INT_MAX;
+  CK(g, cudaMemcpy(g->flag, &big, 4, cudaMemcpyHostToDevice));
+  // step 1: random initialisation of snapshot 0
+  launch_init_params(g->G[0].w, g->G[0].wb, g->PG, g->PGs, g->lg, C, g->seed, LIPZ_STREAM_INIT_G,
+                     g->st);
+  launch_init_params(g->D[0].w, g->D[0].wb, g->PD, g->PDs, g->ld, C, g->seed, LIPZ_STREAM_INIT_D,
+                     g->st);
+  CKL(g);
+  std::vector<float> lr(C, g->a.lr);
+  CK(g, cudaMemcpy(g->G[0].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpy(g->D[0].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpy(g->G[1].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpy(g->D[1].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
+  if ((rc = build_descs(g, 0)) || (rc = build_descs(g, 1))) return rc;
+  g->use_tc = g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
+  if (g->use_tc) {
+    for (int p = 0; p < 2; ++p) {
+      TcShape s{C, B, z, h, x, g->a.leaky_slope};
+      std::string msg;
+      g->tc[p] = tc_plan_create(s, g->Z, g->E, g->e_cell, g->logits, g->nbr, g->G[p].wb,
+                                g->G[p].w, g->PGs, g->lg.off, g->D[p].wb, g->D[p].w, g->PDs,
+                                g->ld.off, &msg);
+      if (!g->tc[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core plan: %s", msg.c_str());
+    }
+  }
+  CK(g, cudaStreamSynchronize(g->st));
+  return LIPZ_OK;
+}
+
+int eval_impl(lipz_grid* g, const float* xin_dev) {
+  const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
+  if (!xin_dev && g->pool_n <= 0)
+    return fail(g, LIPZ_ERR_STATE, "no real-data pool: call lipz_set_data first");
+  const int p = g->cur;
+  phase_begin(g, LIPZ_PHASE_BATCH);
+  if (g->bf)
+    launch_draw_batch<bf16>(g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell, (bf16*)g->Z, C,
+                            B, x, z, g->seed, (uint32_t)g->t, g->st);
+  else
+    launch_draw_batch<float>(g->pool, g->pool_n, xin_dev, (float*)g->E, g->e_cell, (float*)g->Z,
+                             C, B, x, z, g->seed, (uint32_t)g->t, g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_BATCH, 1);
+  if (g->use_tc) {
+    std::string msg;
+    phase_begin(g, LIPZ_PHASE_G_FWD);
+    if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_G_FWD, 1);
+    phase_begin(g, LIPZ_PHASE_D_FWD);
+    if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_D_FWD, 1);
+  } else {
+    const Descs& D = g->dsc[p];
+    phase_begin(g, LIPZ_PHASE_G_FWD);
+    gemm(g, D.g1, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
+    phase_end(g, LIPZ_PHASE_G_FWD, 3);
+    phase_begin(g, LIPZ_PHASE_D_FWD);
+    gemm(g, D.d1, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+    gemm(g, D.d2, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+    gemv(g, D.d3, C * 5, 6 * B);
+    phase_end(g, LIPZ_PHASE_D_FWD, 3);
+  }
+  CKL(g);
+  phase_begin(g, LIPZ_PHASE_FITNESS);
+  launch_fitness(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_FITNESS, 1);
+  g->phase = PH_EVALUATED;
+  return LIPZ_OK;
+}
+
+int select_impl(lipz_grid* g) {
+  if (g->phase != PH_EVALUATED)
+    return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
+  SelectParams sp;
+  sp.seed = g->seed;
+  sp.t = (uint32_t)g->t;
+  sp.tournament_size = g->a.tournament_size;
+  sp.replace_always = g->a.replace_mode == LIPZ_REPLACE_ALWAYS;
+  sp.lr_mutation = g->a.lr_mutation;
+  sp.lr_mut_std = g->a.lr_mut_std;
+  double thr = std::floor((double)g->a.lr_mut_prob * 4294967296.0);
+  sp.lr_mut_thr = (uint64_t)(thr < 0 ? 0 : (thr > 4294967296.0 ? 4294967296.0 : thr));
+  const int p = g->cur;
+  phase_begin(g, LIPZ_PHASE_SELECT);
+  launch_select(g->fG, g->fD, g->nbr, g->cells, sp, g->G[p].lr, g->D[p].lr, g->sel_g, g->sel_d,
+                g->src_g, g->src_d, g->lrn_g, g->lrn_d, g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_SELECT, 1);
+  g->phase = PH_SELECTED;
+  return LIPZ_OK;
+}
+
+int train_impl(lipz_grid* g) {
+  if (g->phase != PH_SELECTED)
+    return fail(g, LIPZ_ERR_STATE, "lipz_train_step must follow lipz_select_replace");
+  const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
+  const int p = g->cur;
+  const Descs& D = g->dsc[p];
+  phase_begin(g, LIPZ_PHASE_TRAIN_FWD);
+  if (g->bf)
+    launch_train_prep<bf16>((const bf16*)g->E, g->e_cell, g->sel_g, (bf16*)g->TX, C, B, x, g->st);
+  else
+    launch_train_prep<float>((const float*)g->E, g->e_cell, g->sel_g, (float*)g->TX, C, B, x,
+                             g->st);
+  // forward of the selected pair
+  gemm(g, D.tg1, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+  gemm(g, D.tg2, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+  gemm(g, D.td1, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+  gemm(g, D.td2, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+  gemv(g, D.tgv, C, 2 * B);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_TRAIN_FWD, 6);
+  phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
+  // logit deltas, then the discriminator's backward
+  if (g->bf)
+    launch_dlogit<bf16>(g->TL, (const bf16*)g->TG2, g->D[p].wb, g->PDs, g->ld.off[4], g->src_d, C,
+                        B, h, g->a.leaky_slope, (bf16*)g->J2, g->gD, g->PDs, g->ld.off[4],
+                        g->ld.off[5], g->st);
+  else
+    launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
+                         C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
+                         g->ld.off[5], g->st);
+  gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
+  colsum(g, D.cb2d, C, h);
+  gemm(g, D.bd1, 2 * C, 2 * B, h, EPI_DACT, ACT_LRELU, false);
+  gemm(g, D.bw1d, C, h, x, EPI_STORE, ACT_NONE, true);
+  colsum(g, D.cb1d, C, h);
+  // generator's backward through D
+  gemm(g, D.ba3, C, B, x, EPI_DACT, ACT_TANH, false);
+  gemm(g, D.bw3g, C, x, h, EPI_STORE, ACT_NONE, true);
+  colsum(g, D.cb3g, C, x);
+  gemm(g, D.ba2, C, B, h, EPI_DACT, ACT_RELU, false);
+  gemm(g, D.bw2g, C, h, h, EPI_STORE, ACT_NONE, true);
+  colsum(g, D.cb2g, C, h);
+  gemm(g, D.ba1, C, B, h, EPI_DACT, ACT_RELU, false);
+  gemm(g, D.bw1g, C, h, z, EPI_STORE, ACT_NONE, true);
+  colsum(g, D.cb1g, C, h);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_TRAIN_BWD, 17);
+  phase_begin(g, LIPZ_PHASE_ADAM);
+  // Adam + replacement into the other snapshot
+  launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->lrn_g, C, g->PG, g->PGs, g->a.beta1,
+              g->a.beta2, g->a.eps, g->st);
+  launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->lrn_d, C, g->PD, g->PDs, g->a.beta1,
+              g->a.beta2, g->a.eps, g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_ADAM, 2);
+  g->cur = 1 - p;
+  g->t += 1;
+  g->phase = PH_IDLE;
+  return LIPZ_OK;
+}
+
+int check_flag(lipz_grid* g) {
+  int v = INT_MAX;
+  CK(g, cudaMemcpy(&v, g->flag, 4, cudaMemcpyDeviceToHost));
+  if (v != INT_MAX) {
+    const int big = INT_MAX;
+    CK(g, cudaMemcpy(g->flag, &big, 4, cudaMemcpyHostToDevice));
+    return fail(g, LIPZ_ERR_NONFINITE, "non-finite loss in cell %d", v);
+  }
+  return LIPZ_OK;
+}
+
+float bf16_bits_to_float(uint16_t b) {
+  uint32_t u = (uint32_t)b << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+
+// Copies `rows` blocks of `n` activation elements (device pitch `pitch` elements) to fp32 host.
+int act_to_host(lipz_grid* g, const void* src, int64_t pitch, int64_t rows, int64_t n, float* out) {
+  std::vector<char> tmp((size_t)(rows * n * g->esz));
+  CK(g, cudaMemcpy2DAsync(tmp.data(), n * g->esz, src, pitch * g->esz, n * g->esz, rows,
+                          cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
+  if (g->bf) {
+    const uint16_t* s = (const uint16_t*)tmp.data();
+    for (int64_t i = 0; i < rows * n; ++i) out[i] = bf16_bits_to_float(s[i]);
+  } else {
+    memcpy(out, tmp.data(), (size_t)(rows * n * 4));
+  }
+  return LIPZ_OK;
+}
+
+}  // namespace
+
+// =============================================================================================
+// C ABI
+// =============================================================================================
+extern "C" {
+
+int lipz_arch_default(lipz_arch* a) {
+  if (!a) return LIPZ_ERR_INVALID;
+  memset(a, 0, sizeof *a);
+  a->struct_size = sizeof(lipz_arch);
+  a->kind = LIPZ_MLP;
+  a->precision = LIPZ_FP32;
+  a->z_dim = 64;
+  a->hidden = 256;
+  a->x_dim = 784;
+  a->batch = 100;
+  a->lr = 2e-4f;
+  a->beta1 = 0.5f;
+  a->beta2 = 0.999f;
+  a->eps = 1e-8f;
+  a->tournament_size = 2;
+  a->replace_mode = LIPZ_REPLACE_IF_BETTER;
+  a->lr_mutation = 0;
+  a->lr_mut_std = 1e-4f;
+  a->lr_mut_prob = 0.5f;
+  a->leaky_slope = 0.2f;
+  a->keep_grads = 0;
+  a->force_simt = 0;
+  return LIPZ_OK;
+}
+
+int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_t seed, lipz_grid** out) {
+  t_create_err.clear();
+  if (!out) return fail(nullptr, LIPZ_ERR_INVALID, "out is null");
+  *out = nullptr;
+  if (rows < 1 || cols < 1 || (int64_t)rows * cols > (1 << 20))
+    return fail(nullptr, LIPZ_ERR_INVALID, "grid needs 1 <= rows, cols and rows*cols <= 2^20");
+  int rc = check_arch(arch);
+  if (rc) return rc;
+  lipz_grid* g = new (std::nothrow) lipz_grid();
+  if (!g) return fail(nullptr, LIPZ_ERR_OOM, "host allocation failed");
+  g->rows = rows;
+  g->cols = cols;
+  g->cells = rows * cols;
+  g->a = *arch;
+  g->seed = seed;
+  g->bf = arch->precision == LIPZ_BF16;
+  g->esz = g->bf ? 2 : 4;
+  rc = create_impl(g);
+  if (rc) {
+    t_create_err = g->err;
+    lipz_grid_destroy(g);
+    return rc;
+  }
+  *out = g;
+  return LIPZ_OK;
+}
+
+int lipz_grid_destroy(lipz_grid* g) {
+  if (!g) return LIPZ_OK;
+  if (g->st || true) cudaStreamSynchronize(g->st);
+  for (int p = 0; p < 2; ++p)
+    if (g->tc[p]) tc_plan_destroy(g->tc[p]);
+  for (auto& m : g->marks) {
+    cudaEventDestroy(m.a);
+    cudaEventDestroy(m.b);
+  }
+  for (auto e : g->ev_free) cudaEventDestroy(e);
+  for (auto e : g->open_ev)
+    if (e) cudaEventDestroy(e);
+  for (void* p : g->allocs) cudaFree(p);
+  delete g;
+  return LIPZ_OK;
+}
+
+int lipz_set_stream(lipz_grid* g, void* stream) {
+  if (!g) return LIPZ_ERR_INVALID;
+  g->st = (cudaStream_t)stream;
+  return LIPZ_OK;
+}
+
+int lipz_synchronize(lipz_grid* g) {
+  if (!g) return LIPZ_ERR_INVALID;
+  CK(g, cudaStreamSynchronize(g->st));
+  return check_flag(g);
+}
+
+int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t dim) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (!host_pool || n_rows < 1 || n_rows > 0xFFFFFFFFll || dim != g->a.x_dim)
+    return fail(g, LIPZ_ERR_INVALID, "set_data needs a pool of 1..2^32-1 rows of x_dim=%d",
+                g->a.x_dim);
+  CK(g, cudaStreamSynchronize(g->st));
+  if (n_rows > g->pool_cap) {
+    if (g->pool) {
+      for (auto& p : g->allocs)
+        if (p == g->pool) p = nullptr;
+      cudaFree(g->pool);
+      g->pool = nullptr;
+      g->pool_cap = 0;
+    }
+    int rc = dalloc(g, &g->pool, (size_t)n_rows * dim * 4);
+    if (rc) return rc;
+    g->pool_cap = n_rows;
+  }
+  CK(g, cudaMemcpy(g->pool, host_pool, (size_t)n_rows * dim * 4, cudaMemcpyHostToDevice));
+  g->pool_n = n_rows;
+  return LIPZ_OK;
+}
+
+int lipz_eval_neighborhoods(lipz_grid* g, float* fit_g, float* fit_d, float* pair_lg,
+                            float* pair_ld) {
+  if (!g) return LIPZ_ERR_INVALID;
+  int rc = eval_impl(g, nullptr);
+  if (rc) return rc;
+  if (fit_g || fit_d || pair_lg || pair_ld) {
+    const size_t C = g->cells;
+    if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
+    if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
+    if (pair_lg) CK(g, cudaMemcpyAsync(pair_lg, g->LG, C * 100, cudaMemcpyDeviceToHost, g->st));
+    if (pair_ld) CK(g, cudaMemcpyAsync(pair_ld, g->LD, C * 100, cudaMemcpyDeviceToHost, g->st));
+    CK(g, cudaStreamSynchronize(g->st));
+    return check_flag(g);
+  }
+  return LIPZ_OK;
+}
+
+int lipz_select_replace(lipz_grid* g, int32_t* sel_g, int32_t* sel_d) {
+  if (!g) return LIPZ_ERR_INVALID;
+  int rc = select_impl(g);
+  if (rc) return rc;
+  if (sel_g || sel_d) {
+    if (sel_g) CK(g, cudaMemcpyAsync(sel_g, g->sel_g, g->cells * 4, cudaMemcpyDeviceToHost, g->st));
+    if (sel_d) CK(g, cudaMemcpyAsync(sel_d, g->sel_d, g->cells * 4, cudaMemcpyDeviceToHost, g->st));
+    CK(g, cudaStreamSynchronize(g->st));
+  }
+  return LIPZ_OK;
+}
+
+int lipz_train_step(lipz_grid* g) {
+  if (!g) return LIPZ_ERR_INVALID;
+  return train_impl(g);
+}
+
+int lipz_iterate(lipz_grid* g, int n_iters) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (n_iters < 0) return fail(g, LIPZ_ERR_INVALID, "n_iters < 0");
+  for (int i = 0; i < n_iters; ++i) {
+    int rc;
+    if ((rc = eval_impl(g, nullptr)) || (rc = select_impl(g)) || (rc = train_impl(g))) return rc;
+  }
+  return LIPZ_OK;
+}
+
+int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* fit_d) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
+  const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
+  CK(g, cudaMemcpyAsync(g->xin, x_host, bytes, cudaMemcpyHostToDevice, g->st));
+  int rc;
+  if ((rc = eval_impl(g, g->xin)) || (rc = select_impl(g)) || (rc = train_impl(g))) return rc;
+  const size_t C = g->cells;
+  if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
+  if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
+  return check_flag(g);
+}
+
+int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {
+  if (!g || !bytes) return LIPZ_ERR_INVALID;
+  const size_t C = g->cells;
+  *bytes = 64 + C * (size_t)(g->PG + g->PD) * 3 * 4 + C * 16;
+  return LIPZ_OK;
+}
+
+int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
+  if (!g) return LIPZ_ERR_INVALID;
+  size_t need = 0;
+  lipz_state_bytes(g, &need);
+  if (!host || bytes != need)
+    return fail(g, LIPZ_ERR_INVALID, "export_state needs a %zu-byte buffer", need);
+  char* o = (char*)host;
+  uint32_t hdr[10] = {0x5A50494Cu, 1u, (uint32_t)g->rows, (uint32_t)g->cols,
+                      (uint32_t)g->a.z_dim, (uint32_t)g->a.hidden, (uint32_t)g->a.x_dim,
+                      (uint32_t)g->a.batch, (uint32_t)g->a.precision, 0u};
+  memset(o, 0, 64);
+  memcpy(o, hdr, 40);
+  memcpy(o + 40, &g->t, 8);
+  memcpy(o + 48, &g->seed, 8);
+  o += 64;
+  CK(g, cudaStreamSynchronize(g->st));
+  const int p = g->cur;
+  const size_t C = g->cells;
+  auto put = [&](const float* src, int64_t P, int64_t Ps) -> int {
+    CK(g, cudaMemcpy2D(o, P * 4, src, Ps * 4, P * 4, C, cudaMemcpyDeviceToHost));
+    o += C * P * 4;
+    return LIPZ_OK;
+  };
+  int rc;
+  if ((rc = put(g->G[p].w, g->PG, g->PGs)) || (rc = put(g->G[p].m, g->PG, g->PGs)) ||
+      (rc = put(g->G[p].v, g->PG, g->PGs)) || (rc = put(g->D[p].w, g->PD, g->PDs)) ||
+      (rc = put(g->D[p].m, g->PD, g->PDs)) || (rc = put(g->D[p].v, g->PD, g->PDs)))
+    return rc;
+  CK(g, cudaMemcpy(o, g->G[p].step, C * 4, cudaMemcpyDeviceToHost));
+  o += C * 4;
+  CK(g, cudaMemcpy(o, g->D[p].step, C * 4, cudaMemcpyDeviceToHost));
+  o += C * 4;
+  CK(g, cudaMemcpy(o, g->G[p].lr, C * 4, cudaMemcpyDeviceToHost));
+  o += C * 4;
+  CK(g, cudaMemcpy(o, g->D[p].lr, C * 4, cudaMemcpyDeviceToHost));
+  return LIPZ_OK;
+}
+
+int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
+  if (!g) return LIPZ_ERR_INVALID;
+  size_t need = 0;
+  lipz_state_bytes(g, &need);
+  if (!host || bytes != need) return fail(g, LIPZ_ERR_INVALID, "import_state needs %zu bytes", need);
+  const char* s = (const char*)host;
+  uint32_t hdr[10];
+  memcpy(hdr, s, 40);
+  if (hdr[0] != 0x5A50494Cu || hdr[1] != 1u)
+    return fail(g, LIPZ_ERR_INVALID, "not a version-1 grid state");
+  if ((int)hdr[2] != g->rows || (int)hdr[3] != g->cols || (int)hdr[4] != g->a.z_dim ||
+      (int)hdr[5] != g->a.hidden || (int)hdr[6] != g->a.x_dim || (int)hdr[7] != g->a.batch)
+    return fail(g, LIPZ_ERR_INVALID, "state shape does not match this grid");
+  CK(g, cudaStreamSynchronize(g->st));
+  int64_t t;
+  uint64_t seed;
+  memcpy(&t, s + 40, 8);
+  memcpy(&seed, s + 48, 8);
+  s += 64;
+  const int p = g->cur;
+  const size_t C = g->cells;
+  auto get = [&](float* dst, int64_t P, int64_t Ps) -> int {
+    CK(g, cudaMemcpy2D(dst, Ps * 4, s, P * 4, P * 4, C, cudaMemcpyHostToDevice));
+    s += C * P * 4;
+    return LIPZ_OK;
+  };
+  int rc;
+  if ((rc = get(g->G[p].w, g->PG, g->PGs)) || (rc = get(g->G[p].m, g->PG, g->PGs)) ||
+      (rc = get(g->G[p].v, g->PG, g->PGs)) || (rc = get(g->D[p].w, g->PD, g->PDs)) ||
+      (rc = get(g->D[p].m, g->PD, g->PDs)) || (rc = get(g->D[p].v, g->PD, g->PDs)))
+    return rc;
+  CK(g, cudaMemcpy(g->G[p].step, s, C * 4, cudaMemcpyHostToDevice));
+  s += C * 4;
+  CK(g, cudaMemcpy(g->D[p].step, s, C * 4, cudaMemcpyHostToDevice));
+  s += C * 4;
+  CK(g, cudaMemcpy(g->G[p].lr, s, C * 4, cudaMemcpyHostToDevice));
+  s += C * 4;
+  CK(g, cudaMemcpy(g->D[p].lr, s, C * 4, cudaMemcpyHostToDevice));
+  if (g->bf) {
+    launch_to_bf16(g->G[p].w, g->G[p].wb, (int64_t)C * g->PGs, g->st);
+    launch_to_bf16(g->D[p].w, g->D[p].wb, (int64_t)C * g->PDs, g->st);
+    CKL(g);
+  }
+  CK(g, cudaStreamSynchronize(g->st));
+  g->t = t;
+  g->seed = seed;
+  g->phase = PH_IDLE;
+  return LIPZ_OK;
+}
+
+int lipz_get_iteration(const lipz_grid* g, int64_t* t) {
+  if (!g || !t) return LIPZ_ERR_INVALID;
+  *t = g->t;
+  return LIPZ_OK;
+}
+
+int lipz_get_batch(lipz_grid* g, float* x, float* z) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (g->phase == PH_IDLE) return fail(g, LIPZ_ERR_STATE, "no evaluation since the last train step");
+  const int64_t B = g->a.batch;
+  int rc;
+  if (x && (rc = act_to_host(g, g->E, g->e_cell, g->cells, B * g->a.x_dim, x))) return rc;
+  if (z && (rc = act_to_host(g, g->Z, B * g->a.z_dim, g->cells, B * g->a.z_dim, z))) return rc;
+  return LIPZ_OK;
+}
+
+int lipz_get_logits(lipz_grid* g, float* logits) {
+  if (!g || !logits) return LIPZ_ERR_INVALID;
+  if (g->phase == PH_IDLE) return fail(g, LIPZ_ERR_STATE, "no evaluation since the last train step");
+  CK(g, cudaMemcpyAsync(logits, g->logits, (size_t)g->cells * 30 * g->a.batch * 4,
+                        cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
+  return LIPZ_OK;
+}
+
+int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (!g->a.keep_grads) return fail(g, LIPZ_ERR_STATE, "grid was created without keep_grads");
+  CK(g, cudaStreamSynchronize(g->st));
+  const size_t C = g->cells;
+  if (grad_g)
+    CK(g, cudaMemcpy2D(grad_g, g->PG * 4, g->gG, g->PGs * 4, g->PG * 4, C, cudaMemcpyDeviceToHost));
+  if (grad_d)
+    CK(g, cudaMemcpy2D(grad_d, g->PD * 4, g->gD, g->PDs * 4, g->PD * 4, C, cudaMemcpyDeviceToHost));
+  return LIPZ_OK;
+}
+
+int lipz_profile_enable(lipz_grid* g, int enable) {
+  if (!g) return LIPZ_ERR_INVALID;
+  g->prof = enable != 0;
+  return LIPZ_OK;
+}
+
+int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t* launches, int n) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (n < 0 || n > LIPZ_N_PHASES) return fail(g, LIPZ_ERR_INVALID, "n must be in 0..%d", LIPZ_N_PHASES);
+  CK(g, cudaStreamSynchronize(g->st));
+  double acc[LIPZ_N_PHASES] = {0};
+  for (auto& m : g->marks) {
+    float t = 0.f;
+    CK(g, cudaEventElapsedTime(&t, m.a, m.b));
+    acc[m.phase] += t;
+    g->ev_free.push_back(m.a);
+    g->ev_free.push_back(m.b);
+  }
+  g->marks.clear();
+  for (int i = 0; i < n; ++i) {
+    if (ms) ms[i] = acc[i];
+    if (count) count[i] = g->counts[i];
+    if (launches) launches[i] = g->launches[i];
+  }
+  for (int i = 0; i < LIPZ_N_PHASES; ++i) g->counts[i] = g->launches[i] = 0;
+  return LIPZ_OK;
+}
+
+const char* lipz_last_error(const lipz_grid* g) {
+  return g ? g->err.c_str() : t_create_err.c_str();
+}
+
+const char* lipz_status_string(int status) {
+  switch (status) {
+    case LIPZ_OK: return "ok";
+    case LIPZ_ERR_INVALID: return "invalid argument";
+    case LIPZ_ERR_CUDA: return "CUDA error";
+    case LIPZ_ERR_OOM: return "out of memory";
+    case LIPZ_ERR_NONFINITE: return "non-finite loss";
+    case LIPZ_ERR_TIMEOUT: return "device wait timed out";
+    case LIPZ_ERR_STATE: return "call out of order";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

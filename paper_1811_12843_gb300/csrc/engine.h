@@ -1,0 +1,78 @@
+// Internal interface between the host scheduler (api.cu) and the kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lipz {
+
+struct GemmDesc;
+struct GemvDesc;
+struct ColSumDesc;
+typedef __nv_bfloat16 bf16;
+
+// Flat parameter layout of one individual: tensor t occupies [off[t], off[t+1]); bound[t] is
+// its Xavier bound (0 for biases).
+struct Layout {
+  int n;
+  int64_t off[7];
+  float bound[6];
+};
+
+// One population snapshot (all cells): fp32 master weights, Adam moments, bf16 copy (bf16
+// mode, else null), per-individual step count and learning rate. Per-cell stride Ps elements.
+struct PopView {
+  float* w;
+  float* m;
+  float* v;
+  bf16* wb;
+  int* step;
+  float* lr;
+};
+
+struct SelectParams {
+  uint64_t seed;
+  uint32_t t;
+  int tournament_size;
+  int replace_always;
+  int lr_mutation;
+  float lr_mut_std;
+  uint64_t lr_mut_thr;  // mutate iff word < thr (= floor(prob * 2^32))
+};
+
+void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout& lay, int cells,
+                        uint64_t seed, uint32_t stream, cudaStream_t st);
+void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st);
+
+template <typename T>
+void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
+                       T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
+                       cudaStream_t st);
+
+template <typename TI, typename TO, int EPI>
+void launch_gemm(const GemmDesc* descs, int n_problems, int max_m, int max_n, int act,
+                 float slope, cudaStream_t st);
+template <typename T>
+void launch_gemv(const GemvDesc* descs, int n_problems, int max_rows, cudaStream_t st);
+template <typename T>
+void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st);
+
+void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
+                    float* fD, int* flag, cudaStream_t st);
+void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
+                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old, int* sel_g,
+                   int* sel_d, int* src_g, int* src_d, float* lr_g_new, float* lr_d_new,
+                   cudaStream_t st);
+template <typename T>
+void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
+                       int x_dim, cudaStream_t st);
+template <typename T>
+void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
+                   const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
+                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st);
+void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, const int* src,
+                 const float* lr_new, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
+                 float eps, cudaStream_t st);
+
+}  // namespace lipz

@@ -1,0 +1,41 @@
+// Tensor-core (tcgen05 / TMEM / TMA) forward of the evaluation phase, bf16 operands with fp32
+// accumulation: every generator slot's fakes and every discriminator slot's logits of every
+// cell, for the MLP shapes it supports.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+namespace lipz {
+
+struct TcShape {
+  int cells, B, z, h, x;
+  float slope;
+};
+
+struct TcPlan;
+
+// hidden == 256, z and x multiples of 16, 16 <= z <= 256, 16 <= x, batch >= 1.
+bool tc_supported(int z, int h, int x, int B);
+
+// Builds the TMA descriptors and launch parameters for one population snapshot. Z: [cells][B][z]
+// bf16; E: [cells][6B][x] bf16 (rows [0, B) real, then the fakes of slots 0..4, which the
+// generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5] on the device. Weights:
+// bf16 copies (Gwb, Dwb) and fp32 masters (for the biases), per-cell strides PGs / PDs, tensor
+// offsets goff / doff (W1, b1, W2, b2, W3, b3). Returns null and a message on failure.
+TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float* logits,
+                       const int* nbr, const __nv_bfloat16* Gwb, const float* Gw, int64_t PGs,
+                       const int64_t* goff, const __nv_bfloat16* Dwb, const float* Dw,
+                       int64_t PDs, const int64_t* doff, std::string* msg);
+
+// Enqueue the generator kernel (fakes of every (cell, slot)) / the discriminator kernel (logits
+// of every (cell, slot)) on `st`. 0 on success.
+int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
+int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
+
+void tc_plan_destroy(TcPlan* p);
+
+}  // namespace lipz

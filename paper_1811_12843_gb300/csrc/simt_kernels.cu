@@ -1,0 +1,539 @@
+// CUDA-core kernels of the grid iteration: initialisation, minibatch draw, grouped GEMM for
+// every layer and its transposes, the discriminator's last layer, BCE fitness, tournament
+// selection, the logit-delta epilogue, column sums and the fused Adam/replacement update.
+#include "common.cuh"
+#include "engine.h"
+
+namespace lipz {
+
+// ------------------------------------------------------------------------------------------
+// Step 1: Xavier-uniform weights. Element k of the flat vector takes word k of the
+// (stream, 0, individual) sequence; s = word >> 8; q = (2 s + 1 - 2^24) 2^-24; w = a q.
+// ------------------------------------------------------------------------------------------
+__global__ void k_init_params(float* __restrict__ w, bf16* __restrict__ wb, int64_t P,
+                              int64_t Ps, Layout lay, uint64_t seed, uint32_t stream) {
+  const int cell = blockIdx.y;
+  const int64_t k0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (k0 >= Ps) return;
+  const U4 r = philox_block(seed, stream, 0u, (uint32_t)cell, (uint32_t)(k0 >> 2));
+  const uint32_t words[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int64_t k = k0 + e;
+    if (k >= Ps) break;
+    float v = 0.f;
+    if (k < P) {
+      int t = 0;
+      while (t + 1 < lay.n && k >= lay.off[t + 1]) ++t;
+      const float a = lay.bound[t];
+      if (a != 0.f) {
+        const float q = (float)(2 * (int32_t)(words[e] >> 8) + 1 - (1 << 24)) * 5.9604644775390625e-8f;
+        v = a * q;
+      }
+    }
+    w[(int64_t)cell * Ps + k] = v;
+    if (wb) wb[(int64_t)cell * Ps + k] = __float2bfloat16_rn(v);
+  }
+}
+
+void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout& lay, int cells,
+                        uint64_t seed, uint32_t stream, cudaStream_t st) {
+  dim3 grid((unsigned)((Ps / 4 + 255) / 256), cells);
+  k_init_params<<<grid, 256, 0, st>>>(w, wb, P, Ps, lay, seed, stream);
+}
+
+__global__ void k_to_bf16(const float* __restrict__ w, bf16* __restrict__ wb, int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    wb[i] = __float2bfloat16_rn(w[i]);
+}
+
+void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st) {
+  k_to_bf16<<<1216, 256, 0, st>>>(w, wb, n);
+}
+
+// ------------------------------------------------------------------------------------------
+// Minibatch of cell c at iteration t: row b = pool row mulhi(word_b, n_pool) of stream BATCH
+// (or row b of the caller's batch), z[b][d] = normal b*z_dim + d of stream NOISE.
+// Rows go to E[c][b] (the first B rows of the cell's evaluation input).
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_draw_batch(const float* __restrict__ pool, int64_t n_pool,
+                             const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
+                             T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
+                             uint32_t t) {
+  const int b = blockIdx.x, c = blockIdx.y;
+  const float* src;
+  if (xin) {
+    src = xin + ((int64_t)c * B + b) * x_dim;
+  } else {
+    const U4 r = philox_block(seed, 3u, t, (uint32_t)c, (uint32_t)(b >> 2));
+    const uint32_t w = (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
+    src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
+  }
+  T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
+  for (int k = threadIdx.x; k < x_dim; k += blockDim.x) dst[k] = from_f<T>(src[k]);
+  T* zr = Z + ((int64_t)c * B + b) * z_dim;
+  for (int d = threadIdx.x; d < z_dim; d += blockDim.x) {
+    const uint32_t n = (uint32_t)b * (uint32_t)z_dim + (uint32_t)d;
+    const U4 r = philox_block(seed, 4u, t, (uint32_t)c, n >> 2);
+    const int q = n & 3;
+    const float2 g = q < 2 ? box_muller(r.x, r.y) : box_muller(r.z, r.w);
+    zr[d] = from_f<T>((q & 1) ? g.y : g.x);
+  }
+}
+
+template <typename T>
+void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
+                       T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
+                       cudaStream_t st) {
+  k_draw_batch<T><<<dim3(B, cells), 256, 0, st>>>(pool, n_pool, xin, E, e_cell, Z, B, x_dim,
+                                                  z_dim, seed, t);
+}
+template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
+                                       float*, int, int, int, int, uint64_t, uint32_t,
+                                       cudaStream_t);
+template void launch_draw_batch<bf16>(const float*, int64_t, const float*, bf16*, int64_t, bf16*,
+                                      int, int, int, int, uint64_t, uint32_t, cudaStream_t);
+
+// ------------------------------------------------------------------------------------------
+// Grouped GEMM on CUDA cores: 64x64 output tile per block, k-slices of 16 staged in shared
+// memory as fp32, 4x4 outputs per thread, fp32 accumulation in k order.
+// ------------------------------------------------------------------------------------------
+template <typename TI, typename TO, int EPI>
+__global__ void __launch_bounds__(256) k_gemm(const GemmDesc* __restrict__ descs, int act,
+                                              float slope) {
+  const GemmDesc d = descs[blockIdx.z];
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  if (m0 >= d.M || n0 >= d.N) return;
+  const TI* A = (const TI*)d.A;
+  const TI* Bm = (const TI*)d.B;
+  const float* bias = d.bias;
+  if (d.wsel) {
+    const int64_t off = (int64_t)d.wsel[d.cell] * d.wsel_stride;
+    if (d.wsel_op == 1) A += off; else Bm += off;
+    if (bias) bias += off;
+  }
+  __shared__ float As[16][64 + 4];
+  __shared__ float Bs[16][64 + 4];
+  const int tid = threadIdx.x;
+  const int tm = (tid >> 4) * 4, tn = (tid & 15) * 4;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  const bool a_kfast = d.sak == 1, b_nfast = d.sbn == 1;
+  for (int k0 = 0; k0 < d.K; k0 += 16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int idx = tid + 256 * i;
+      int m, k;
+      if (a_kfast) { m = idx >> 4; k = idx & 15; } else { m = idx & 63; k = idx >> 6; }
+      float v = 0.f;
+      if (m0 + m < d.M && k0 + k < d.K)
+        v = to_f<TI>(A[(int64_t)(m0 + m) * d.sam + (int64_t)(k0 + k) * d.sak]);
+      As[k][m] = v;
+      int n, kk;
+      if (b_nfast) { n = idx & 63; kk = idx >> 6; } else { n = idx >> 4; kk = idx & 15; }
+      float w = 0.f;
+      if (n0 + n < d.N && k0 + kk < d.K)
+        w = to_f<TI>(Bm[(int64_t)(k0 + kk) * d.sbk + (int64_t)(n0 + n) * d.sbn]);
+      Bs[kk][n] = w;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[k][tm + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Bs[k][tn + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  TO* C = (TO*)d.C;
+  const TI* aux = (const TI*)d.aux;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int m = m0 + tm + i;
+    if (m >= d.M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = n0 + tn + j;
+      if (n >= d.N) continue;
+      float v = acc[i][j];
+      if (EPI == EPI_BIAS_ACT) {
+        v = act_fwd(act, v + (bias ? bias[n] : 0.f), slope);
+      } else if (EPI == EPI_DACT) {
+        v *= act_bwd(act, to_f<TI>(aux[(int64_t)m * d.sxm + (int64_t)n * d.sxn]), slope);
+      }
+      C[(int64_t)m * d.scm + (int64_t)n * d.scn] = from_f<TO>(v);
+    }
+  }
+}
+
+template <typename TI, typename TO, int EPI>
+void launch_gemm(const GemmDesc* descs, int n_problems, int max_m, int max_n, int act,
+                 float slope, cudaStream_t st) {
+  if (n_problems <= 0 || max_m <= 0 || max_n <= 0) return;
+  dim3 grid((max_n + 63) / 64, (max_m + 63) / 64, n_problems);
+  k_gemm<TI, TO, EPI><<<grid, 256, 0, st>>>(descs, act, slope);
+}
+#define LIPZ_INST_GEMM(TI, TO, EPI) \
+  template void launch_gemm<TI, TO, EPI>(const GemmDesc*, int, int, int, int, float, cudaStream_t);
+LIPZ_INST_GEMM(float, float, EPI_STORE)
+LIPZ_INST_GEMM(float, float, EPI_BIAS_ACT)
+LIPZ_INST_GEMM(float, float, EPI_DACT)
+LIPZ_INST_GEMM(bf16, float, EPI_STORE)
+LIPZ_INST_GEMM(bf16, bf16, EPI_BIAS_ACT)
+LIPZ_INST_GEMM(bf16, bf16, EPI_DACT)
+
+// ------------------------------------------------------------------------------------------
+// Discriminator output layer: one warp per row, lanes stride over k, fixed shuffle tree.
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_gemv(const GemvDesc* __restrict__ descs) {
+  const GemvDesc d = descs[blockIdx.y];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (r >= d.rows) return;
+  const T* w = (const T*)d.w;
+  const float* bias = d.bias;
+  if (d.wsel) {
+    const int64_t off = (int64_t)d.wsel[d.cell] * d.wsel_stride;
+    w += off;
+    bias += off;
+  }
+  const T* x = (const T*)d.X + (int64_t)r * d.ld;
+  float s = 0.f;
+  for (int k = lane; k < d.K; k += 32) s = fmaf(to_f<T>(x[k]), to_f<T>(w[k]), s);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) d.out[r] = s + bias[0];
+}
+
+template <typename T>
+void launch_gemv(const GemvDesc* descs, int n_problems, int max_rows, cudaStream_t st) {
+  if (n_problems <= 0 || max_rows <= 0) return;
+  k_gemv<T><<<dim3((max_rows + 7) / 8, n_problems), 256, 0, st>>>(descs);
+}
+template void launch_gemv<float>(const GemvDesc*, int, int, cudaStream_t);
+template void launch_gemv<bf16>(const GemvDesc*, int, int, cudaStream_t);
+
+// ------------------------------------------------------------------------------------------
+// Column sums (bias gradients): one thread per column, rows in order.
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_colsum(const ColSumDesc* __restrict__ descs) {
+  const ColSumDesc d = descs[blockIdx.y];
+  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= d.cols) return;
+  const T* x = (const T*)d.X;
+  float s = 0.f;
+  for (int r = 0; r < d.rows; ++r) s += to_f<T>(x[(int64_t)r * d.ld + n]);
+  d.out[n] = s;
+}
+
+template <typename T>
+void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st) {
+  if (n_problems <= 0 || max_cols <= 0) return;
+  k_colsum<T><<<dim3((max_cols + 255) / 256, n_problems), 256, 0, st>>>(descs);
+}
+template void launch_colsum<float>(const ColSumDesc*, int, int, cudaStream_t);
+template void launch_colsum<bf16>(const ColSumDesc*, int, int, cudaStream_t);
+
+// ------------------------------------------------------------------------------------------
+// Pair losses and fitness of every cell (one block per cell). logits[c][j][6B]: rows [0, B)
+// real, rows [B (1 + i), B (2 + i)) fakes of generator slot i.
+//   L_D[c][i][j] = mean softplus(-real_j) + mean softplus(fake_ij)
+//   L_G[c][i][j] = mean softplus(-fake_ij)
+//   f_G[c][i] = mean_j L_G,  f_D[c][j] = mean_i L_D
+// Each mean is one warp's fixed-order reduction: the result does not depend on scheduling.
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ float softplusf(float x) { return fmaxf(x, 0.f) + log1pf(expf(-fabsf(x))); }
+
+__global__ void k_fitness(const float* __restrict__ logits, int B, float* __restrict__ LG,
+                          float* __restrict__ LD, float* __restrict__ fG, float* __restrict__ fD,
+                          int* __restrict__ flag) {
+  const int c = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __shared__ float real_s[5], fake_d[25], fake_g[25];
+  const float* lc = logits + (int64_t)c * 5 * 6 * B;
+  for (int task = warp; task < 30; task += nw) {
+    float s1 = 0.f, s2 = 0.f;
+    if (task < 5) {
+      const float* l = lc + (int64_t)task * 6 * B;
+      for (int b = lane; b < B; b += 32) s1 += softplusf(-l[b]);
+    } else {
+      const int i = (task - 5) / 5, j = (task - 5) % 5;
+      const float* l = lc + (int64_t)j * 6 * B + (int64_t)(1 + i) * B;
+      for (int b = lane; b < B; b += 32) {
+        s1 += softplusf(l[b]);
+        s2 += softplusf(-l[b]);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+    }
+    if (lane == 0) {
+      if (task < 5) real_s[task] = s1 / (float)B;
+      else {
+        fake_d[task - 5] = s1 / (float)B;
+        fake_g[task - 5] = s2 / (float)B;
+      }
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < 25) {
+    const int i = threadIdx.x / 5, j = threadIdx.x % 5;
+    const float ld = real_s[j] + fake_d[threadIdx.x];
+    const float lg = fake_g[threadIdx.x];
+    LD[c * 25 + threadIdx.x] = ld;
+    LG[c * 25 + threadIdx.x] = lg;
+    if (!isfinite(ld) || !isfinite(lg)) atomicMin(flag, c);
+    (void)i;
+  }
+  __syncthreads();
+  if (threadIdx.x < 5) {
+    const int i = threadIdx.x;
+    float sg = 0.f, sd = 0.f;
+    for (int j = 0; j < 5; ++j) {
+      sg += fake_g[i * 5 + j];
+      sd += real_s[i] + fake_d[j * 5 + i];  // f_D of slot i: mean over generator slots j
+    }
+    fG[c * 5 + i] = sg / 5.f;
+    fD[c * 5 + i] = sd / 5.f;
+  }
+}
+
+void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
+                    float* fD, int* flag, cudaStream_t st) {
+  k_fitness<<<cells, 256, 0, st>>>(logits, B, LG, LD, fG, fD, flag);
+}
+
+// ------------------------------------------------------------------------------------------
+// Tournament selection, replacement and learning-rate mutation: one thread per cell.
+// ------------------------------------------------------------------------------------------
+__device__ int tournament_slot(const float* f5, const uint32_t* w, int size) {
+  int remaining[5] = {0, 1, 2, 3, 4};
+  int left = 5, best = -1;
+  for (int m = 0; m < size; ++m) {
+    const int r = (int)mulhi_u32(w[m], (uint32_t)(5 - m));
+    const int e = remaining[r];
+    for (int q = r; q + 1 < left; ++q) remaining[q] = remaining[q + 1];
+    --left;
+    if (best < 0 || f5[e] < f5[best] || (f5[e] == f5[best] && e < best)) best = e;
+  }
+  return best;
+}
+
+__device__ float mutate(float lr, uint64_t seed, uint32_t stream, uint32_t t, uint32_t c,
+                        float std, uint64_t thr) {
+  const U4 r = philox_block(seed, stream, t, c, 0u);
+  if ((uint64_t)r.x >= thr) return lr;
+  const float n = box_muller(r.y, r.z).x;
+  return fmaxf(lr + std * n, 1e-8f);
+}
+
+__global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
+                         const int* __restrict__ nbr, int cells, SelectParams p,
+                         const float* __restrict__ lr_g_old, const float* __restrict__ lr_d_old,
+                         int* __restrict__ sel_g, int* __restrict__ sel_d, int* __restrict__ src_g,
+                         int* __restrict__ src_d, float* __restrict__ lr_g_new,
+                         float* __restrict__ lr_d_new) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= cells) return;
+  for (int pop = 0; pop < 2; ++pop) {
+    const float* f5 = (pop ? fD : fG) + c * 5;
+    const U4 a = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 0u);
+    const U4 b = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 1u);
+    const uint32_t w[5] = {a.x, a.y, a.z, a.w, b.x};
+    const int win = tournament_slot(f5, w, p.tournament_size);
+    const int s = p.replace_always ? win : (f5[win] < f5[0] ? win : 0);
+    const int src = nbr[c * 5 + s];
+    float lr = (pop ? lr_d_old : lr_g_old)[src];
+    if (p.lr_mutation) lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std,
+                                   p.lr_mut_thr);
+    if (pop) {
+      sel_d[c] = s;
+      src_d[c] = src;
+      lr_d_new[c] = lr;
+    } else {
+      sel_g[c] = s;
+      src_g[c] = src;
+      lr_g_new[c] = lr;
+    }
+  }
+}
+
+void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
+                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old, int* sel_g,
+                   int* sel_d, int* src_g, int* src_d, float* lr_g_new, float* lr_d_new,
+                   cudaStream_t st) {
+  k_select<<<(cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old, sel_g,
+                                                sel_d, src_g, src_d, lr_g_new, lr_d_new);
+}
+
+// ------------------------------------------------------------------------------------------
+// Training input of cell c: TX[c] = [E[c] rows [0, B); E[c] rows of generator slot sel_g[c]].
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_train_prep(const T* __restrict__ E, int64_t e_cell, const int* __restrict__ sel_g,
+                             T* __restrict__ TX, int B, int x_dim) {
+  const int r = blockIdx.x, c = blockIdx.y;
+  const int src_row = r < B ? r : B * (1 + sel_g[c]) + (r - B);
+  const T* s = E + (int64_t)c * e_cell + (int64_t)src_row * x_dim;
+  T* d = TX + ((int64_t)c * 2 * B + r) * x_dim;
+  for (int k = threadIdx.x; k < x_dim; k += blockDim.x) d[k] = s[k];
+}
+
+template <typename T>
+void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
+                       int x_dim, cudaStream_t st) {
+  k_train_prep<T><<<dim3(2 * B, cells), 256, 0, st>>>(E, e_cell, sel_g, TX, B, x_dim);
+}
+template void launch_train_prep<float>(const float*, int64_t, const int*, float*, int, int, int,
+                                       cudaStream_t);
+template void launch_train_prep<bf16>(const bf16*, int64_t, const int*, bf16*, int, int, int,
+                                      cudaStream_t);
+
+// ------------------------------------------------------------------------------------------
+// Logit deltas of the selected pair of cell c, rows [real, fake (D loss), fake (G loss)]:
+//   dl = (s - 1)/B (real), s/B (fake, D loss), (s - 1)/B (fake, G loss), s = sigmoid(logit);
+//   J2[r][k] = dl_r * w3[k] * lrelu'(g2[r'][k])  (r' = r, or r - B for the G-loss rows);
+//   dW3 = sum_{r < 2B} dl_r g2[r],  db3 = sum_{r < 2B} dl_r.
+// One block per cell, one thread per hidden unit.
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_dlogit(const float* __restrict__ TL, const T* __restrict__ TG2,
+                         const T* __restrict__ wD, int64_t wD_stride, int64_t off_w3,
+                         const int* __restrict__ src_d, int B, int H, float slope,
+                         T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride,
+                         int64_t off_gw3, int64_t off_gb3) {
+  extern __shared__ float dl[];
+  const int c = blockIdx.x;
+  const float* l = TL + (int64_t)c * 2 * B;
+  for (int r = threadIdx.x; r < 3 * B; r += blockDim.x) {
+    const float x = r < 2 * B ? l[r] : l[r - B];
+    const float s = 1.f / (1.f + expf(-x));
+    dl[r] = (r < B || r >= 2 * B) ? (s - 1.f) / (float)B : s / (float)B;
+  }
+  __syncthreads();
+  const T* w3 = wD + (int64_t)src_d[c] * wD_stride + off_w3;
+  const T* g2 = TG2 + (int64_t)c * 2 * B * H;
+  T* j2 = J2 + (int64_t)c * 3 * B * H;
+  float* g = gD + (int64_t)c * gD_stride;
+  for (int k = threadIdx.x; k < H; k += blockDim.x) {
+    const float wk = to_f<T>(w3[k]);
+    float acc = 0.f;
+    for (int r = 0; r < 3 * B; ++r) {
+      const int rr = r < 2 * B ? r : r - B;
+      const float gv = to_f<T>(g2[(int64_t)rr * H + k]);
+      j2[(int64_t)r * H + k] = from_f<T>(dl[r] * wk * (gv > 0.f ? 1.f : slope));
+      if (r < 2 * B) acc = fmaf(dl[r], gv, acc);
+    }
+    g[off_gw3 + k] = acc;
+  }
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int r = 0; r < 2 * B; ++r) s += dl[r];
+    g[off_gb3] = s;
+  }
+}
+
+template <typename T>
+void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
+                   const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
+                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st) {
+  const int threads = H >= 256 ? 256 : ((H + 31) / 32) * 32;
+  k_dlogit<T><<<cells, threads, 3 * B * sizeof(float), st>>>(
+      TL, TG2, wD, wD_stride, off_w3, src_d, B, H, slope, J2, gD, gD_stride, off_gw3, off_gb3);
+}
+template void launch_dlogit<float>(const float*, const float*, const float*, int64_t, int64_t,
+                                   const int*, int, int, int, float, float*, float*, int64_t,
+                                   int64_t, int64_t, cudaStream_t);
+template void launch_dlogit<bf16>(const float*, const bf16*, const bf16*, int64_t, int64_t,
+                                  const int*, int, int, int, float, bf16*, float*, int64_t,
+                                  int64_t, int64_t, cudaStream_t);
+
+// ------------------------------------------------------------------------------------------
+// Adam (Kingma & Ba 2015, Algorithm 1) fused with the replacement copy: the new centre of
+// cell c starts from individual src[c] of the old snapshot and is written to cell c of the
+// new snapshot (fp32 master, m, v, bf16 copy, step, lr).
+// ------------------------------------------------------------------------------------------
+__global__ void k_adam(PopView old_p, PopView new_p, const float* __restrict__ grad,
+                       const int* __restrict__ src, const float* __restrict__ lr_new,
+                       int64_t P, int64_t Ps, float beta1, float beta2, float eps) {
+  const int c = blockIdx.y;
+  const int s = src[c];
+  __shared__ float coef[2];
+  if (threadIdx.x == 0) {
+    const int step1 = old_p.step[s] + 1;
+    const double bc1 = 1.0 - pow((double)beta1, (double)step1);
+    const double bc2 = 1.0 - pow((double)beta2, (double)step1);
+    coef[0] = (float)(1.0 / bc1);
+    coef[1] = (float)(1.0 / bc2);
+    if (blockIdx.x == 0) {
+      new_p.step[c] = step1;
+      new_p.lr[c] = lr_new[c];
+    }
+  }
+  __syncthreads();
+  const float lr = lr_new[c], ib1 = coef[0], ib2 = coef[1];
+  const int64_t so = (int64_t)s * Ps, co = (int64_t)c * Ps;
+  const int64_t k0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (k0 >= P) return;
+  if (k0 + 3 < P) {
+    const float4 w = *(const float4*)(old_p.w + so + k0);
+    const float4 m = *(const float4*)(old_p.m + so + k0);
+    const float4 v = *(const float4*)(old_p.v + so + k0);
+    const float4 g = *(const float4*)(grad + co + k0);
+    float wv[4] = {w.x, w.y, w.z, w.w}, mv[4] = {m.x, m.y, m.z, m.w};
+    float vv[4] = {v.x, v.y, v.z, v.w};
+    const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      mv[e] = beta1 * mv[e] + (1.f - beta1) * gv[e];
+      vv[e] = beta2 * vv[e] + (1.f - beta2) * gv[e] * gv[e];
+      wv[e] = wv[e] - lr * (mv[e] * ib1) / (sqrtf(vv[e] * ib2) + eps);
+    }
+    *(float4*)(new_p.w + co + k0) = make_float4(wv[0], wv[1], wv[2], wv[3]);
+    *(float4*)(new_p.m + co + k0) = make_float4(mv[0], mv[1], mv[2], mv[3]);
+    *(float4*)(new_p.v + co + k0) = make_float4(vv[0], vv[1], vv[2], vv[3]);
+    if (new_p.wb) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(wv[0], wv[1]);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(wv[2], wv[3]);
+      uint2 pk;
+      pk.x = *(uint32_t*)&lo;
+      pk.y = *(uint32_t*)&hi;
+      *(uint2*)(new_p.wb + co + k0) = pk;
+    }
+  } else {
+    for (int64_t k = k0; k < P; ++k) {
+      const float gk = grad[co + k];
+      const float mk = beta1 * old_p.m[so + k] + (1.f - beta1) * gk;
+      const float vk = beta2 * old_p.v[so + k] + (1.f - beta2) * gk * gk;
+      const float wk = old_p.w[so + k] - lr * (mk * ib1) / (sqrtf(vk * ib2) + eps);
+      new_p.w[co + k] = wk;
+      new_p.m[co + k] = mk;
+      new_p.v[co + k] = vk;
+      if (new_p.wb) new_p.wb[co + k] = __float2bfloat16_rn(wk);
+    }
+  }
+}
+
+void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, const int* src,
+                 const float* lr_new, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
+                 float eps, cudaStream_t st) {
+  dim3 grid((unsigned)((P / 4 + 1 + 255) / 256), cells);
+  k_adam<<<grid, 256, 0, st>>>(old_p, new_p, grad, src, lr_new, P, Ps, beta1, beta2, eps);
+}
+
+}  // namespace lipz

@@ -1,0 +1,280 @@
+"""GPU parity: the CUDA engine (through the C ABI) against the CPU oracle, step by step.
+
+Tolerances (max-norm relative error per tensor, max|gpu - ref| / max|ref|): 1e-4 for the fp32
+path and 2e-2 for the bf16-operand / fp32-accumulate path. Integer work (neighbourhoods,
+minibatch indices, tournament choices given the same fitness) is compared bit-exactly.
+"""
+
+import numpy as np
+import pytest
+
+from oracle import lipz_oracle as O
+
+from helpers import max_rel, oracle_arch, per_tensor
+
+pytestmark = pytest.mark.gpu
+
+TOL = {0: 1e-4, 1: 2e-2}
+
+
+@pytest.fixture(scope="module")
+def L():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_1811_12843_gb300 import _build
+    _build.build()
+    import paper_1811_12843_gb300 as lib
+    return lib
+
+
+def _pool(seed, n, dim):
+    import lipz_synth
+    return lipz_synth.blob_pool(seed, n=n, dim=dim)
+
+
+def _grid(L, rows, cols, seed, pool, **kw):
+    g = L.Grid(rows, cols, seed=seed, **kw)
+    g.set_data(pool)
+    return g
+
+
+def _to_oracle(g, arch):
+    return O.state_from_bytes(g.export_state(), oracle_arch(arch))
+
+
+# ------------------------------------------------------------------------------------------
+def test_init_is_bit_exact(L):
+    g = L.Grid(2, 3, seed=1811)
+    s = _to_oracle(g, g.arch)
+    ref = O.create(2, 3, oracle_arch(g.arch), 1811)
+    assert np.array_equal(s.Gw, ref.Gw) and np.array_equal(s.Dw, ref.Dw)
+    assert np.all(s.Gm == 0) and np.all(s.Dv == 0) and np.all(s.Gstep == 0)
+    assert np.allclose(s.Glr, np.float32(2e-4))
+
+
+@pytest.mark.parametrize("precision", ["fp32", "bf16"])
+def test_minibatch_draw(L, precision):
+    pool = _pool(3, 5000, 784)
+    g = _grid(L, 2, 2, 77, pool, precision=precision)
+    g.eval()
+    x, z = g.batch()
+    s = _to_oracle(g, g.arch)
+    data = O.batches(s, pool)
+    for c in range(4):
+        xr, zr = data[c]
+        if precision == "fp32":
+            assert np.array_equal(x[c], xr.astype(np.float32))        # indices bit-exact
+            assert np.max(np.abs(z[c] - zr)) < 2e-6 * max(1.0, np.max(np.abs(zr)))
+        else:
+            assert np.array_equal(x[c], O.round_bf16(xr))
+            assert np.max(np.abs(z[c] - O.round_bf16(zr))) <= 2 ** -7 * np.max(np.abs(zr))
+
+
+def _check_eval(g, s, ev_ref, tol, cells=None):
+    ev = g.eval(pairs=True)
+    logits = g.logits()
+    sl = slice(None) if cells is None else list(cells)
+    assert max_rel(logits[sl], ev_ref["logits"][sl]) < tol
+    for k in ("LG", "LD", "fG", "fD"):
+        assert max_rel(ev[k][sl], ev_ref[k][sl]) < tol, k
+    return ev
+
+
+@pytest.mark.parametrize("precision,rows,cols,batch", [
+    ("fp32", 2, 2, 100),    # 2x2 fp32, B=100 (one-iteration parity config)
+    ("fp32", 1, 1, 37),     # degenerate 1x1 torus, ragged batch
+    ("fp32", 1, 4, 64),
+    ("bf16", 2, 2, 100),
+    ("bf16", 3, 3, 129),    # ragged tile tails on the tensor-core path
+])
+def test_eval_parity(L, precision, rows, cols, batch):
+    pool = _pool(5, 3000, 784)
+    g = _grid(L, rows, cols, 11, pool, precision=precision, batch=batch)
+    s = _to_oracle(g, g.arch)
+    ref = O.eval_neighborhoods(s, O.batches(s, pool))
+    _check_eval(g, s, ref, TOL[g.arch.precision])
+
+
+def test_eval_parity_tiny_arch_simt(L):
+    """Shapes the tensor-core kernels do not take run on the CUDA-core kernels."""
+    pool = _pool(6, 200, 5)
+    g = _grid(L, 2, 3, 4, pool, z_dim=3, hidden=4, x_dim=5, batch=7)
+    s = _to_oracle(g, g.arch)
+    ref = O.eval_neighborhoods(s, O.batches(s, pool))
+    _check_eval(g, s, ref, 1e-4)
+
+
+def _one_iteration_check(L, g, pool, tol, x_host=None):
+    """Eval, select (bit-exact given the engine's own fitness), train (gradients and weights)."""
+    a = oracle_arch(g.arch)
+    s = _to_oracle(g, g.arch)
+    data = O.batches(s, pool, x_host)
+    ref = O.eval_neighborhoods(s, data)
+    ev = _check_eval(g, s, ref, tol)
+    sel = g.select()
+    # the tournament is a pure function of (fitness, Philox words): feed the engine's fitness
+    ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                   "fD": ev["fD"].astype(np.float64)})
+    assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+    assert np.array_equal(sel["sel_d"], ref_sel["sel_d"])
+    g.train()
+    new, grads = O.train_step(s, ref_sel, data, keep_grads=True)
+    gg, gd = g.gradients()
+    got = _to_oracle(g, g.arch)
+    assert got.t == s.t + 1
+    assert np.array_equal(got.Gstep, new.Gstep) and np.array_equal(got.Dstep, new.Dstep)
+    for name, err in per_tensor(gg, grads["gG"], O.g_layout(a)).items():
+        assert err < tol, ("grad G", name, err)
+    for name, err in per_tensor(gd, grads["gD"], O.d_layout(a)).items():
+        assert err < tol, ("grad D", name, err)
+    # Adam given the engine's own gradient: fp32 arithmetic against float64
+    nbr = O.neighbors(s.rows, s.cols)
+    for c in range(s.cells):
+        sg = nbr[c][sel["sel_g"][c]]
+        w1 = O.adam_step(s.Gw[sg], s.Gm[sg], s.Gv[sg], s.Gstep[sg], gg[c].astype(np.float64),
+                         float(np.float32(s.Glr[sg])), a)[0]
+        assert np.max(np.abs(got.Gw[c] - w1)) <= 1e-6 * np.max(np.abs(w1)) + 1e-9
+    # updated weights against the oracle's own iteration; an element beyond the tolerance is
+    # allowed only where Adam's sign-like first step follows a gradient whose sign is within the
+    # engine's accumulation noise (|g_ref| <= |g_gpu - g_ref|)
+    flagged = 0
+    for pop, lay, gref, ggpu in (("Gw", O.g_layout(a), grads["gG"], gg),
+                                 ("Dw", O.d_layout(a), grads["gD"], gd)):
+        w_got, w_ref = getattr(got, pop), getattr(new, pop)
+        off = 0
+        for name, shape in lay:
+            n = int(np.prod(shape))
+            sl = slice(off, off + n)
+            off += n
+            d = np.abs(w_got[:, sl] - w_ref[:, sl])
+            bad = d > tol * np.max(np.abs(w_ref[:, sl]))
+            if np.any(bad):
+                gr, gq = gref[:, sl][bad], ggpu[:, sl][bad].astype(np.float64)
+                assert np.all(np.abs(gr) <= np.abs(gq - gr) + 1e-12), (pop, name)
+                flagged += int(bad.sum())
+    return flagged
+
+
+def test_one_iteration_fp32_2x2(L):
+    """2x2 torus, fp32, B = 100, one grid iteration."""
+    pool = _pool(1811, 60000, 784)
+    g = _grid(L, 2, 2, 1811, pool, keep_grads=1)
+    flagged = _one_iteration_check(L, g, pool, 1e-4)
+    assert flagged <= 20
+
+
+def test_lockstep_fp32_3x3_twenty_iterations(L):
+    """3x3 torus, fp32, B = 100: twenty iterations, each checked against the oracle started from
+    the engine's previous state."""
+    pool = _pool(1811, 60000, 784)
+    g = _grid(L, 3, 3, 0, pool, keep_grads=1)
+    for it in range(20):
+        _one_iteration_check(L, g, pool, 1e-4)
+    assert g.t == 20
+
+
+def test_one_iteration_bf16_5x5_b256(L):
+    """5x5 torus, bf16 operands / fp32 accumulation and Adam masters, B = 256."""
+    pool = _pool(2, 60000, 784)
+    g = _grid(L, 5, 5, 2, pool, precision="bf16", batch=256, keep_grads=1)
+    _one_iteration_check(L, g, pool, 2e-2)
+    _one_iteration_check(L, g, pool, 2e-2)
+
+
+def test_selection_modes_and_mutation(L):
+    pool = _pool(8, 4000, 784)
+    g = _grid(L, 3, 4, 8, pool, keep_grads=1, tournament_size=5, replace_mode="always",
+              lr_mutation=1, lr_mut_prob=1.0, lr_mut_std=1e-4)
+    for _ in range(2):
+        s = _to_oracle(g, g.arch)
+        data = O.batches(s, pool)
+        ev = g.eval()
+        sel = g.select()
+        ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                       "fD": ev["fD"].astype(np.float64)})
+        assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+        assert np.array_equal(sel["sel_g"], np.argmin(ev["fG"], axis=1))
+        g.train()
+        new = O.train_step(s, ref_sel, data)
+        got = _to_oracle(g, g.arch)
+        assert np.allclose(got.Glr, new.Glr, rtol=1e-6, atol=1e-12)
+        assert np.allclose(got.Dlr, new.Dlr, rtol=1e-6, atol=1e-12)
+        assert not np.allclose(got.Glr, 2e-4)
+
+
+def test_host_batch_iteration(L):
+    import lipz_synth
+    g = L.Grid(2, 3, seed=5, keep_grads=1)
+    g.set_data(_pool(1, 100, 784))
+    x = lipz_synth.host_batch(9, 6, 100)
+    s = _to_oracle(g, g.arch)
+    fg, fd = np.zeros((6, 5), np.float32), np.zeros((6, 5), np.float32)
+    L.lipz_iterate_batch(g.h, x, fg, fd)
+    data = O.batches(s, None, x)
+    ref = O.eval_neighborhoods(s, data)
+    assert max_rel(fg, ref["fG"]) < 1e-4 and max_rel(fd, ref["fD"]) < 1e-4
+    sel = O.select_replace(s, {"fG": fg.astype(np.float64), "fD": fd.astype(np.float64)})
+    new = O.train_step(s, sel, data)
+    got = _to_oracle(g, g.arch)
+    assert max_rel(got.Dm, new.Dm) < 1e-4
+
+
+def test_determinism_and_resume(L):
+    pool = _pool(4, 2000, 784)
+    a = _grid(L, 3, 3, 21, pool, precision="bf16")
+    b = _grid(L, 3, 3, 21, pool, precision="bf16")
+    a.iterate(3)
+    b.iterate(2)
+    mid = b.export_state()
+    c = _grid(L, 3, 3, 999, pool, precision="bf16")
+    c.import_state(mid)                 # resume replaces seed and iteration counter too
+    b.iterate(1)
+    c.iterate(1)
+    sa, sb, sc = a.export_state(), b.export_state(), c.export_state()
+    assert sa == sb == sc
+
+
+def test_call_order_and_nonfinite_detection(L):
+    pool = _pool(4, 500, 784)
+    g = _grid(L, 2, 2, 3, pool)
+    with pytest.raises(L.LipzError) as e:
+        g.select()
+    assert e.value.code == L.LIPZ_ERR_STATE
+    g.eval()
+    with pytest.raises(L.LipzError) as e:
+        g.train()
+    assert e.value.code == L.LIPZ_ERR_STATE
+    # plant a NaN in cell 2's discriminator through the state interface (a host-side fault)
+    s = _to_oracle(g, g.arch)
+    s.Dw[2, 5] = np.nan
+    g.import_state(O.state_to_bytes(s))
+    with pytest.raises(L.LipzError) as e:
+        g.eval()
+    assert e.value.code == L.LIPZ_ERR_NONFINITE
+
+
+def test_full_size_12x12_bf16_sampled_cells(L):
+    """The benchmark workload (12x12 torus, bf16, B = 100, tensor-core path): pair losses of a
+    sample of cells against the oracle computed cell by cell, then invariants of one full
+    iteration at that size."""
+    pool = _pool(1811, 60000, 784)
+    g = _grid(L, 12, 12, 1811, pool, precision="bf16")
+    s = _to_oracle(g, g.arch)
+    cells = [0, 13, 77, 143]
+    data = O.batches(s, pool, cells=cells)
+    ref = O.eval_neighborhoods(s, data, cells=cells)
+    ev = _check_eval(g, s, ref, 2e-2, cells=cells)
+    assert np.all(np.isfinite(ev["fG"])) and np.all(np.isfinite(ev["fD"]))
+    sel = g.select()
+    ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                   "fD": ev["fD"].astype(np.float64)})
+    assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+    assert np.array_equal(sel["sel_d"], ref_sel["sel_d"])
+    g.train()
+    got = _to_oracle(g, g.arch)
+    assert np.all(got.Gstep == 1) and np.all(got.Dstep == 1)
+    # every weight moved by at most lr (Adam's first step is bounded by lr per element)
+    nbr = O.neighbors(12, 12)
+    src = nbr[np.arange(144), sel["sel_g"]]
+    assert np.max(np.abs(got.Gw - s.Gw[src])) <= 2e-4 * (1 + 1e-5)
