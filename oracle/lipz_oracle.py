@@ -482,7 +482,12 @@ def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.nd
     lg, ld = pair_losses(logit[:B], logit[B:])
     flatG = np.concatenate([gG[n].reshape(-1) for n, _ in gl])
     flatD = np.concatenate([gD[n].reshape(-1) for n, _ in dl])
-    return flatG, flatD, {"LG": lg, "LD": ld}
+    # Distance of the closest pre-activation to a kink of ReLU / LeakyReLU (where the derivative
+    # jumps): a diagnostic for comparisons with implementations that round differently.
+    pre = [zq @ rb(G["W1"]).T + G["b1"], h1 @ rb(G["W2"]).T + G["b2"],
+           X @ rb(D["W1"]).T + D["b1"], g1 @ rb(D["W2"]).T + D["b2"]]
+    kink = min(float(np.min(np.abs(p))) for p in pre)
+    return flatG, flatD, {"LG": lg, "LD": ld, "kink": kink}
 
 
 def adam_step(w, m, v, step, g, lr, arch: Arch):
@@ -501,7 +506,8 @@ def train_step(state: State, sel, data, keep_grads: bool = False):
     a = state.arch
     nbr = neighbors(state.rows, state.cols)
     new = state.copy()
-    grads = {"gG": np.zeros_like(state.Gw), "gD": np.zeros_like(state.Dw)}
+    grads = {"gG": np.zeros_like(state.Gw), "gD": np.zeros_like(state.Dw),
+             "kink": np.zeros(state.cells)}
     for c in range(state.cells):
         sg = int(nbr[c][sel["sel_g"][c]])
         sd = int(nbr[c][sel["sel_d"][c]])
@@ -510,7 +516,8 @@ def train_step(state: State, sel, data, keep_grads: bool = False):
             lr_g = mutate_lr(lr_g, state.seed, STREAM_MUT_G, state.t, c, a)
             lr_d = mutate_lr(lr_d, state.seed, STREAM_MUT_D, state.t, c, a)
         x, z = data[c]
-        gG, gD, _ = pair_gradients(state.Gw[sg], state.Dw[sd], x, z, a)
+        gG, gD, info = pair_gradients(state.Gw[sg], state.Dw[sd], x, z, a)
+        grads["kink"][c] = info["kink"]
         new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c] = adam_step(
             state.Gw[sg], state.Gm[sg], state.Gv[sg], state.Gstep[sg], gG, lr_g, a)
         new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c] = adam_step(

@@ -660,6 +660,16 @@ int train_impl(lipz_grid* g) {
 }
 
 int check_flag(lipz_grid* g) {
+  for (int p = 0; p < 2; ++p) {
+    int* f = g->tc[p] ? tc_error_flag(g->tc[p]) : nullptr;
+    if (!f) continue;
+    int code = 0;
+    CK(g, cudaMemcpy(&code, f, 4, cudaMemcpyDeviceToHost));
+    if (code) {
+      CK(g, cudaMemset(f, 0, 4));
+      return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core forward stopped: bounded wait %d expired", code);
+    }
+  }
   int v = INT_MAX;
   CK(g, cudaMemcpy(&v, g->flag, 4, cudaMemcpyDeviceToHost));
   if (v != INT_MAX) {

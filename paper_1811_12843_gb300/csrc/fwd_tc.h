@@ -36,6 +36,10 @@ TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
 
+// Device int that a kernel of the plan sets to a non-zero code when one of its bounded waits
+// expired (the kernel then stopped early); the host reads and clears it.
+int* tc_error_flag(TcPlan* p);
+
 void tc_plan_destroy(TcPlan* p);
 
 }  // namespace lipz
