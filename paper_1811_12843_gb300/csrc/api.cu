@@ -14,6 +14,7 @@
 
 #include "common.cuh"
 #include "engine.h"
+#include "bwd_tc.h"
 #include "fwd_tc.h"
 #include "lipz.h"
 
@@ -65,6 +66,7 @@ struct lipz_grid {
   float *logits = nullptr, *LG = nullptr, *LD = nullptr, *fG = nullptr, *fD = nullptr;
   int *nbr = nullptr, *sel_g = nullptr, *sel_d = nullptr, *src_g = nullptr, *src_d = nullptr;
   float *lrn_g = nullptr, *lrn_d = nullptr;
+  float4 *coef_g = nullptr, *coef_d = nullptr;  // per cell: lr, 1/bc1, 1/bc2, step + 1
   void *TH1 = nullptr, *TH2 = nullptr, *TX = nullptr, *TG1 = nullptr, *TG2 = nullptr;
   float* TL = nullptr;
   void *J2 = nullptr, *D1 = nullptr, *A3 = nullptr, *A2 = nullptr, *A1 = nullptr;
@@ -72,6 +74,8 @@ struct lipz_grid {
   int* flag = nullptr;
   Descs dsc[2]{};
   TcPlan* tc[2]{};
+  TcbPlan* tcb[2]{};
+  bool use_tcb = false;
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
   bool prof = false;
@@ -491,7 +495,8 @@ int create_impl(lipz_grid* g) {
       (rc = dalloc(g, &g->fD, C * 5 * 4)) || (rc = dalloc(g, &g->sel_g, C * 4)) ||
       (rc = dalloc(g, &g->sel_d, C * 4)) || (rc = dalloc(g, &g->src_g, C * 4)) ||
       (rc = dalloc(g, &g->src_d, C * 4)) || (rc = dalloc(g, &g->lrn_g, C * 4)) ||
-      (rc = dalloc(g, &g->lrn_d, C * 4)) || (rc = dalloc(g, &g->TH1, CB * h * es)) ||
+      (rc = dalloc(g, &g->lrn_d, C * 4)) || (rc = dalloc(g, &g->coef_g, C * 16)) ||
+      (rc = dalloc(g, &g->coef_d, C * 16)) || (rc = dalloc(g, &g->TH1, CB * h * es)) ||
       (rc = dalloc(g, &g->TH2, CB * h * es)) || (rc = dalloc(g, &g->TX, CB * 2 * x * es)) ||
       (rc = dalloc(g, &g->TG1, CB * 2 * h * es)) || (rc = dalloc(g, &g->TG2, CB * 2 * h * es)) ||
       (rc = dalloc(g, &g->TL, CB * 2 * 4)) || (rc = dalloc(g, &g->J2, CB * 3 * h * es)) ||
@@ -521,11 +526,59 @@ int create_impl(lipz_grid* g) {
   if (g->use_tc) {
     for (int p = 0; p < 2; ++p) {
       TcShape s{C, B, z, h, x, g->a.leaky_slope};
+      TcBuffers b{};
+      b.Z = g->Z;
+      b.E = g->E;
+      b.e_cell = g->e_cell;
+      b.logits = g->logits;
+      b.nbr = g->nbr;
+      b.Gwb = g->G[p].wb;
+      b.Gw = g->G[p].w;
+      b.PGs = g->PGs;
+      b.goff = g->lg.off;
+      b.Dwb = g->D[p].wb;
+      b.Dw = g->D[p].w;
+      b.PDs = g->PDs;
+      b.doff = g->ld.off;
+      b.TX = g->TX;
+      b.src_g = g->src_g;
+      b.src_d = g->src_d;
+      b.TH1 = g->TH1;
+      b.TH2 = g->TH2;
+      b.TG1 = g->TG1;
+      b.TG2 = g->TG2;
+      b.TL = g->TL;
       std::string msg;
-      g->tc[p] = tc_plan_create(s, g->Z, g->E, g->e_cell, g->logits, g->nbr, g->G[p].wb,
-                                g->G[p].w, g->PGs, g->lg.off, g->D[p].wb, g->D[p].w, g->PDs,
-                                g->ld.off, &msg);
+      g->tc[p] = tc_plan_create(s, b, &msg);
       if (!g->tc[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core plan: %s", msg.c_str());
+    }
+    g->use_tcb = tcb_supported(z, h, x, B);
+    for (int p = 0; p < 2 && g->use_tcb; ++p) {
+      TcbShape s{C, B, z, h, x, g->a.leaky_slope, C};
+      TcbBuffers b{};
+      b.Z = g->Z;
+      b.TX = g->TX;
+      b.TH1 = g->TH1;
+      b.TH2 = g->TH2;
+      b.TG1 = g->TG1;
+      b.J2 = g->J2;
+      b.D1 = g->D1;
+      b.A3 = g->A3;
+      b.A2 = g->A2;
+      b.A1 = g->A1;
+      b.gG = g->gG;
+      b.gD = g->gD;
+      b.Gwb = g->G[p].wb;
+      b.Dwb = g->D[p].wb;
+      b.PGs = g->PGs;
+      b.PDs = g->PDs;
+      b.goff = g->lg.off;
+      b.doff = g->ld.off;
+      b.src_g = g->src_g;
+      b.src_d = g->src_d;
+      std::string msg;
+      g->tcb[p] = tcb_plan_create(s, b, &msg);
+      if (!g->tcb[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core backward plan: %s", msg.c_str());
     }
   }
   CK(g, cudaStreamSynchronize(g->st));
@@ -590,8 +643,11 @@ int select_impl(lipz_grid* g) {
   sp.lr_mut_thr = (uint64_t)(thr < 0 ? 0 : (thr > 4294967296.0 ? 4294967296.0 : thr));
   const int p = g->cur;
   phase_begin(g, LIPZ_PHASE_SELECT);
-  launch_select(g->fG, g->fD, g->nbr, g->cells, sp, g->G[p].lr, g->D[p].lr, g->sel_g, g->sel_d,
-                g->src_g, g->src_d, g->lrn_g, g->lrn_d, g->st);
+  sp.beta1 = g->a.beta1;
+  sp.beta2 = g->a.beta2;
+  launch_select(g->fG, g->fD, g->nbr, g->cells, sp, g->G[p].lr, g->D[p].lr, g->G[p].step,
+                g->D[p].step, g->sel_g, g->sel_d, g->src_g, g->src_d, g->lrn_g, g->lrn_d,
+                g->coef_g, g->coef_d, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_SELECT, 1);
   g->phase = PH_SELECTED;
@@ -611,13 +667,20 @@ int train_impl(lipz_grid* g) {
     launch_train_prep<float>((const float*)g->E, g->e_cell, g->sel_g, (float*)g->TX, C, B, x,
                              g->st);
   // forward of the selected pair
-  gemm(g, D.tg1, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
-  gemm(g, D.tg2, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
-  gemm(g, D.td1, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
-  gemm(g, D.td2, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
-  gemv(g, D.tgv, C, 2 * B);
+  if (g->use_tc) {
+    std::string msg;
+    if (tc_run_train_g(g->tc[p], g->st, &msg) || tc_run_train_d(g->tc[p], g->st, &msg))
+      return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_TRAIN_FWD, 3);
+  } else {
+    gemm(g, D.tg1, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.tg2, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.td1, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+    gemm(g, D.td2, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
+    gemv(g, D.tgv, C, 2 * B);
+    phase_end(g, LIPZ_PHASE_TRAIN_FWD, 6);
+  }
   CKL(g);
-  phase_end(g, LIPZ_PHASE_TRAIN_FWD, 6);
   phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
   // logit deltas, then the discriminator's backward
   if (g->bf)
@@ -628,28 +691,45 @@ int train_impl(lipz_grid* g) {
     launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
                          g->ld.off[5], g->st);
-  gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
-  colsum(g, D.cb2d, C, h);
-  gemm(g, D.bd1, 2 * C, 2 * B, h, EPI_DACT, ACT_LRELU, false);
-  gemm(g, D.bw1d, C, h, x, EPI_STORE, ACT_NONE, true);
-  colsum(g, D.cb1d, C, h);
-  // generator's backward through D
-  gemm(g, D.ba3, C, B, x, EPI_DACT, ACT_TANH, false);
-  gemm(g, D.bw3g, C, x, h, EPI_STORE, ACT_NONE, true);
-  colsum(g, D.cb3g, C, x);
-  gemm(g, D.ba2, C, B, h, EPI_DACT, ACT_RELU, false);
-  gemm(g, D.bw2g, C, h, h, EPI_STORE, ACT_NONE, true);
-  colsum(g, D.cb2g, C, h);
-  gemm(g, D.ba1, C, B, h, EPI_DACT, ACT_RELU, false);
-  gemm(g, D.bw1g, C, h, z, EPI_STORE, ACT_NONE, true);
-  colsum(g, D.cb1g, C, h);
-  CKL(g);
-  phase_end(g, LIPZ_PHASE_TRAIN_BWD, 17);
+  if (g->use_tcb) {
+    std::string msg;
+    TcbPlan* P = g->tcb[p];
+    // D1, dW2(D) | A3, dW1(D) | A2, dW3(G) | A1, dW2(G), dW1(G), with the bias column sums
+    if (tcb_run(P, 0, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    colsum(g, D.cb2d, C, h);
+    colsum(g, D.cb1d, C, h);
+    if (tcb_run(P, 2, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    colsum(g, D.cb3g, C, x);
+    if (tcb_run(P, 4, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    colsum(g, D.cb2g, C, h);
+    if (tcb_run(P, 6, 3, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    colsum(g, D.cb1g, C, h);
+    CKL(g);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
+  } else {
+    gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
+    colsum(g, D.cb2d, C, h);
+    gemm(g, D.bd1, 2 * C, 2 * B, h, EPI_DACT, ACT_LRELU, false);
+    gemm(g, D.bw1d, C, h, x, EPI_STORE, ACT_NONE, true);
+    colsum(g, D.cb1d, C, h);
+    // generator's backward through D
+    gemm(g, D.ba3, C, B, x, EPI_DACT, ACT_TANH, false);
+    gemm(g, D.bw3g, C, x, h, EPI_STORE, ACT_NONE, true);
+    colsum(g, D.cb3g, C, x);
+    gemm(g, D.ba2, C, B, h, EPI_DACT, ACT_RELU, false);
+    gemm(g, D.bw2g, C, h, h, EPI_STORE, ACT_NONE, true);
+    colsum(g, D.cb2g, C, h);
+    gemm(g, D.ba1, C, B, h, EPI_DACT, ACT_RELU, false);
+    gemm(g, D.bw1g, C, h, z, EPI_STORE, ACT_NONE, true);
+    colsum(g, D.cb1g, C, h);
+    CKL(g);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 17);
+  }
   phase_begin(g, LIPZ_PHASE_ADAM);
   // Adam + replacement into the other snapshot
-  launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->lrn_g, C, g->PG, g->PGs, g->a.beta1,
+  launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
-  launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->lrn_d, C, g->PD, g->PDs, g->a.beta1,
+  launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_ADAM, 2);
@@ -660,14 +740,15 @@ int train_impl(lipz_grid* g) {
 }
 
 int check_flag(lipz_grid* g) {
-  for (int p = 0; p < 2; ++p) {
-    int* f = g->tc[p] ? tc_error_flag(g->tc[p]) : nullptr;
+  for (int p = 0; p < 4; ++p) {
+    int* f = p < 2 ? (g->tc[p] ? tc_error_flag(g->tc[p]) : nullptr)
+                   : (g->tcb[p - 2] ? tcb_error_flag(g->tcb[p - 2]) : nullptr);
     if (!f) continue;
     int code = 0;
     CK(g, cudaMemcpy(&code, f, 4, cudaMemcpyDeviceToHost));
     if (code) {
       CK(g, cudaMemset(f, 0, 4));
-      return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core forward stopped: bounded wait %d expired", code);
+      return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
   int v = INT_MAX;
@@ -764,8 +845,10 @@ int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_t seed, l
 int lipz_grid_destroy(lipz_grid* g) {
   if (!g) return LIPZ_OK;
   if (g->st || true) cudaStreamSynchronize(g->st);
-  for (int p = 0; p < 2; ++p)
+  for (int p = 0; p < 2; ++p) {
     if (g->tc[p]) tc_plan_destroy(g->tc[p]);
+    if (g->tcb[p]) tcb_plan_destroy(g->tcb[p]);
+  }
   for (auto& m : g->marks) {
     cudaEventDestroy(m.a);
     cudaEventDestroy(m.b);

@@ -1,0 +1,535 @@
+// Tensor-core backward of the training step (Section 3, step 3: the gradient update of every
+// cell's selected generator and discriminator), bf16 operands and fp32 accumulation in TMEM.
+//
+// One grouped GEMM kernel serves every product of the backward: per cell, a 128 x BN output
+// tile of C = A * B^T over K, where each operand is read by TMA either K-major (rows of K) or
+// MN-major (rows of M or N, K in the outer dimension; used for the transposed products dW =
+// delta^T X and delta W, so no transposed copy is ever written). Epilogues: fp32 store
+// (weight gradients) or bf16 delta times the activation derivative read from the stored
+// forward output. The z coordinate of a weight operand is the cell's selected individual.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+
+#include "bwd_tc.h"
+#include "common.cuh"
+#include "tc_ptx.cuh"
+
+namespace lipz {
+namespace tcb {
+
+using namespace lipz::tc;
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int STAGES = 2;
+constexpr int A_BYTES = BM * BK * 2;        // 16 KB
+constexpr int B_BYTES = 256 * BK * 2;       // 32 KB (BN <= 256)
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int MN_BOX_BYTES = 64 * BK * 2;   // one {64 MN, 64 K} box
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+
+enum { EPI_F32 = 0, EPI_DACT = 1 };
+
+struct GParams {
+  int M, N, K, BN;
+  int mtiles, ntiles, kchunks;
+  int a_mn, b_mn;       // operand layouts (1 = MN-major)
+  int a_row0, b_row0;   // first row of a K-major operand
+  const int* a_sel;     // z coordinate of A: a_sel[cell] (weights of the selected individual)
+  const int* b_sel;     //   or the cell itself when null
+  int epi, act;
+  float slope;
+  void* C;
+  int64_t c_cell, scm, scn;  // C[cell * c_cell + m * scm + n * scn]
+  const bf16* aux;
+  int64_t aux_cell, sxm, sxn;
+  int aux_wrap_at, aux_wrap_sub;  // aux row of m: m < wrap_at ? m : m - wrap_sub
+  int* err;
+};
+
+__device__ __forceinline__ float dact(int act, float y, float slope) {
+  switch (act) {
+    case ACT_RELU: return y > 0.f ? 1.f : 0.f;
+    case ACT_LRELU: return y > 0.f ? 1.f : slope;
+    case ACT_TANH: return 1.f - y * y;
+    default: return 1.f;
+  }
+}
+
+__global__ void __launch_bounds__(THREADS, 2)
+    k_gemm_tc(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+              const GParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  uint8_t* misc = gbase + STAGES * STAGE_BYTES;
+  const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES, bAcc = bEmpty + 8 * STAGES;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 128);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 132);
+
+  const int per_cell = p.mtiles * p.ntiles;
+  const int cell = blockIdx.x / per_cell;
+  const int rem = blockIdx.x % per_cell;
+  const int m0 = (rem / p.ntiles) * BM;
+  const int n0 = (rem % p.ntiles) * p.BN;
+  int n = min(p.BN, p.N - n0);
+  n = (n + 15) & ~15;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(bFull + 8 * s, 1);
+      mbar_init(bEmpty + 8 * s, 1);
+    }
+    mbar_init(bAcc, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t b_bytes = p.b_mn ? (uint32_t)((p.BN / 64) * MN_BOX_BYTES) : (uint32_t)(p.BN * 128);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const int za = p.a_sel ? __ldg(&p.a_sel[cell]) : cell;
+      const int zb = p.b_sel ? __ldg(&p.b_sel[cell]) : cell;
+      int issued[STAGES] = {0, 0};
+      bool ok = true;
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int kc = 0; kc < p.kchunks; ++kc) {
+        if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 11)) {
+          ok = false;
+          break;
+        }
+        const uint32_t full = bFull + 8 * stage;
+        mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
+        const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+        if (p.a_mn) {
+          tma_load_3d(sA, &mA, full, m0, kc * BK, za);
+          tma_load_3d(sA + MN_BOX_BYTES, &mA, full, m0 + 64, kc * BK, za);
+        } else {
+          tma_load_3d(sA, &mA, full, kc * BK, p.a_row0 + m0, za);
+        }
+        if (p.b_mn) {
+          for (int i = 0; i < p.BN / 64; ++i)
+            tma_load_3d(sB + i * MN_BOX_BYTES, &mB, full, n0 + 64 * i, kc * BK, zb);
+        } else {
+          tma_load_3d(sB, &mB, full, kc * BK, p.b_row0 + n0, zb);
+        }
+        issued[stage]++;
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) {
+        for (int s = 0; s < STAGES; ++s)
+          if (issued[s] > 0) {
+            volatile int never = 0;
+            mbar_wait(bFull + 8 * s, (uint32_t)((issued[s] - 1) & 1), &never, p.err, 11);
+          }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_major(BM, n, p.a_mn, p.b_mn);
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int kc = 0; kc < p.kchunks; ++kc) {
+        if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 12)) break;
+        tc_fence_after();
+        const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          const uint64_t ad = p.a_mn ? sw128_mn_desc(sA + kk * 2048, MN_BOX_BYTES)
+                                     : sw128_desc(sA + kk * 32);
+          const uint64_t bd = p.b_mn ? sw128_mn_desc(sB + kk * 2048, MN_BOX_BYTES)
+                                     : sw128_desc(sB + kk * 32);
+          tc_mma(tmem, ad, bd, idesc, (kc | kk) != 0 ? 1u : 0u);
+        }
+        tc_commit(bEmpty + 8 * stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      tc_commit(bAcc);
+      // the MMAs must be complete before the tensor memory is released, even if the
+      // epilogue gave up waiting
+      volatile int never = 0;
+      mbar_wait(bAcc, 0u, &never, p.err, 14);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
+    const int row = q * 32 + lane;
+    const int m = m0 + row;
+    if (mbar_wait(bAcc, 0u, abort_flag, p.err, 13)) {
+      tc_fence_after();
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+      const int ng = n / 16;
+      const int half = (ng + 1) / 2;
+      const int g0 = hf ? half : 0, g1 = hf ? ng : half;
+      const bool row_ok = m < p.M;
+      const int arow = m < p.aux_wrap_at ? m : m - p.aux_wrap_sub;
+      for (int gi = g0; gi < g1; ++gi) {
+        uint32_t r[16];
+        LIPZ_TMEM_LD16(tbase + gi * 16, r);
+        tmem_wait_ld();
+        const int col0 = n0 + gi * 16;
+        if (!row_ok) continue;
+        if (p.epi == EPI_F32) {
+          float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+          if (p.scn == 1 && col0 + 16 <= p.N) {
+            float4* o = reinterpret_cast<float4*>(C + col0);
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+              o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
+                                 __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
+          } else {
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __uint_as_float(r[e]);
+          }
+        } else {
+          bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+          const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
+          float v[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int col = col0 + e;
+            const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
+            v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
+          }
+          if (p.scn == 1 && col0 + 16 <= p.N) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int e = 0; e < 16; e += 2) {
+              __nv_bfloat162 b2 = __floats2bfloat162_rn(v[e], v[e + 1]);
+              pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
+            }
+            uint4* o = reinterpret_cast<uint4*>(C + col0);
+            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __float2bfloat16_rn(v[e]);
+          }
+        }
+      }
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+  }
+}
+
+}  // namespace tcb
+
+// ---- host side -----------------------------------------------------------------------------
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
+
+bool encoder(std::string* msg) {
+  if (g_enc) return true;
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                   cudaEnableDefault, &q);
+  if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) {
+    cudaGetLastError();
+    if (msg) *msg = "cuTensorMapEncodeTiled is unavailable";
+    return false;
+  }
+  g_enc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  return true;
+}
+
+// bf16 3-D map {inner, rows, depth}; box {64, box_rows, 1}, 128-byte swizzle.
+bool map3(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t depth,
+          uint64_t depth_elems, uint32_t box_rows, std::string* msg) {
+  cuuint64_t dims[3] = {inner, rows, depth};
+  cuuint64_t strides[2] = {inner * 2, depth_elems * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
+struct Gemm {
+  CUtensorMap a, b;
+  tcb::GParams p;
+  int grid;
+};
+
+}  // namespace
+
+struct TcbPlan {
+  // order of execution: D1, dW2d, A3, dW1d, A2, dW3g, A1, dW2g, dW1g
+  Gemm g[9];
+  int n;
+  int* err;
+};
+
+bool tcb_supported(int z, int h, int x, int B) {
+  return h == 256 && z == 64 && x % 16 == 0 && x >= 64 && B >= 1 && B <= 256;
+}
+
+TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* msg) {
+  if (!tcb_supported(s.z, s.h, s.x, s.B)) {
+    if (msg) *msg = "shape not supported by the tensor-core backward";
+    return nullptr;
+  }
+  if (!encoder(msg)) return nullptr;
+  if (cudaFuncSetAttribute(tcb::k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tcb::SMEM_BYTES) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "cannot reserve shared memory for the tensor-core backward";
+    return nullptr;
+  }
+  TcbPlan* P = new TcbPlan();
+  memset(P, 0, sizeof *P);
+  if (cudaMalloc(&P->err, 4) != cudaSuccess || cudaMemset(P->err, 0, 4) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "cudaMalloc for the error flag failed";
+    delete P;
+    return nullptr;
+  }
+  const int C = s.cells, B = s.B, h = s.h, x = s.x, z = s.z;
+  const uint64_t NI = s.n_indiv;
+  const int BNr = ((B + 15) / 16) * 16;  // rows of a batch as an MMA N
+  const bf16* Gw = b.Gwb;
+  const bf16* Dw = b.Dwb;
+  auto base_params = [&](int M, int N, int K, int BN) {
+    tcb::GParams q;
+    memset(&q, 0, sizeof q);
+    q.M = M;
+    q.N = N;
+    q.K = K;
+    q.BN = BN;
+    q.mtiles = (M + 127) / 128;
+    q.ntiles = (N + BN - 1) / BN;
+    q.kchunks = (K + 63) / 64;
+    q.slope = s.slope;
+    q.aux_wrap_at = 1 << 30;
+    q.err = P->err;
+    return q;
+  };
+  bool ok = true;
+  int i = 0;
+  auto finish = [&](Gemm& G) { G.grid = C * G.p.mtiles * G.p.ntiles; };
+
+  // 1. D1 = (J2 @ W2d) * lrelu'(TG1 rows r or r - B): M = 3B rows, N = 256, K = 256
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(3 * B, h, h, 256);
+    G.p.b_mn = 1;
+    G.p.b_sel = b.src_d;
+    G.p.epi = tcb::EPI_DACT;
+    G.p.act = ACT_LRELU;
+    G.p.C = b.D1;
+    G.p.c_cell = (int64_t)3 * B * h;
+    G.p.scm = h;
+    G.p.scn = 1;
+    G.p.aux = (const bf16*)b.TG1;
+    G.p.aux_cell = (int64_t)2 * B * h;
+    G.p.sxm = h;
+    G.p.sxn = 1;
+    G.p.aux_wrap_at = 2 * B;
+    G.p.aux_wrap_sub = B;
+    ok = ok && map3(&G.a, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 128, msg) &&
+         map3(&G.b, Dw + b.doff[2], h, h, NI, b.PDs, 64, msg);
+    finish(G);
+  }
+  // 2. dW2d^T[i][o] = sum_{r < 2B} TG1[r][i] J2[r][o]: M = i, N = o, K = 2B (TG1 ends at 2B)
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(h, h, 2 * B, 256);
+    G.p.a_mn = 1;
+    G.p.b_mn = 1;
+    G.p.epi = tcb::EPI_F32;
+    G.p.C = b.gD + b.doff[2];
+    G.p.c_cell = b.PDs;
+    G.p.scm = 1;
+    G.p.scn = h;
+    ok = ok && map3(&G.a, b.TG1, h, 2 * B, C, (uint64_t)2 * B * h, 64, msg) &&
+         map3(&G.b, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg);
+    finish(G);
+  }
+  // 3. A3^T[i][r] = (sum_o W1d[o][i] D1[2B + r][o]) * (1 - F[r][i]^2): M = x, N = B, K = 256
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(x, B, h, BNr);
+    G.p.a_mn = 1;
+    G.p.a_sel = b.src_d;
+    G.p.b_row0 = 2 * B;
+    G.p.epi = tcb::EPI_DACT;
+    G.p.act = ACT_TANH;
+    G.p.C = b.A3;
+    G.p.c_cell = (int64_t)B * x;
+    G.p.scm = 1;
+    G.p.scn = x;
+    G.p.aux = (const bf16*)b.TX + (int64_t)B * x;
+    G.p.aux_cell = (int64_t)2 * B * x;
+    G.p.sxm = 1;
+    G.p.sxn = x;
+    ok = ok && map3(&G.a, Dw + b.doff[0], x, h, NI, b.PDs, 64, msg) &&
+         map3(&G.b, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, BNr, msg);
+    finish(G);
+  }
+  // 4. dW1d^T[i][o] = sum_{r < 2B} TX[r][i] D1[r][o]: M = x, N = 256, K = 2B (TX ends at 2B)
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(x, h, 2 * B, 256);
+    G.p.a_mn = 1;
+    G.p.b_mn = 1;
+    G.p.epi = tcb::EPI_F32;
+    G.p.C = b.gD + b.doff[0];
+    G.p.c_cell = b.PDs;
+    G.p.scm = 1;
+    G.p.scn = x;
+    ok = ok && map3(&G.a, b.TX, x, 2 * B, C, (uint64_t)2 * B * x, 64, msg) &&
+         map3(&G.b, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg);
+    finish(G);
+  }
+  // 5. A2 = (A3 @ W3g) * relu'(TH2): M = B, N = 256, K = x
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(B, h, x, 256);
+    G.p.b_mn = 1;
+    G.p.b_sel = b.src_g;
+    G.p.epi = tcb::EPI_DACT;
+    G.p.act = ACT_RELU;
+    G.p.C = b.A2;
+    G.p.c_cell = (int64_t)B * h;
+    G.p.scm = h;
+    G.p.scn = 1;
+    G.p.aux = (const bf16*)b.TH2;
+    G.p.aux_cell = (int64_t)B * h;
+    G.p.sxm = h;
+    G.p.sxn = 1;
+    ok = ok && map3(&G.a, b.A3, x, B, C, (uint64_t)B * x, 128, msg) &&
+         map3(&G.b, Gw + b.goff[4], h, x, NI, b.PGs, 64, msg);
+    finish(G);
+  }
+  // 6. dW3g[o][i] = sum_r A3[r][o] TH2[r][i]: M = x (o), N = 256 (i), K = B
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(x, h, B, 256);
+    G.p.a_mn = 1;
+    G.p.b_mn = 1;
+    G.p.epi = tcb::EPI_F32;
+    G.p.C = b.gG + b.goff[4];
+    G.p.c_cell = b.PGs;
+    G.p.scm = h;
+    G.p.scn = 1;
+    ok = ok && map3(&G.a, b.A3, x, B, C, (uint64_t)B * x, 64, msg) &&
+         map3(&G.b, b.TH2, h, B, C, (uint64_t)B * h, 64, msg);
+    finish(G);
+  }
+  // 7. A1 = (A2 @ W2g) * relu'(TH1): M = B, N = 256, K = 256
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(B, h, h, 256);
+    G.p.b_mn = 1;
+    G.p.b_sel = b.src_g;
+    G.p.epi = tcb::EPI_DACT;
+    G.p.act = ACT_RELU;
+    G.p.C = b.A1;
+    G.p.c_cell = (int64_t)B * h;
+    G.p.scm = h;
+    G.p.scn = 1;
+    G.p.aux = (const bf16*)b.TH1;
+    G.p.aux_cell = (int64_t)B * h;
+    G.p.sxm = h;
+    G.p.sxn = 1;
+    ok = ok && map3(&G.a, b.A2, h, B, C, (uint64_t)B * h, 128, msg) &&
+         map3(&G.b, Gw + b.goff[2], h, h, NI, b.PGs, 64, msg);
+    finish(G);
+  }
+  // 8. dW2g^T[i][o] = sum_r TH1[r][i] A2[r][o]: M = 256 (i), N = 256 (o), K = B
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(h, h, B, 256);
+    G.p.a_mn = 1;
+    G.p.b_mn = 1;
+    G.p.epi = tcb::EPI_F32;
+    G.p.C = b.gG + b.goff[2];
+    G.p.c_cell = b.PGs;
+    G.p.scm = 1;
+    G.p.scn = h;
+    ok = ok && map3(&G.a, b.TH1, h, B, C, (uint64_t)B * h, 64, msg) &&
+         map3(&G.b, b.A2, h, B, C, (uint64_t)B * h, 64, msg);
+    finish(G);
+  }
+  // 9. dW1g[o][i] = sum_r A1[r][o] Z[r][i]: M = 256 (o), N = z (i), K = B
+  {
+    Gemm& G = P->g[i++];
+    G.p = base_params(h, z, B, z);
+    G.p.a_mn = 1;
+    G.p.b_mn = 1;
+    G.p.epi = tcb::EPI_F32;
+    G.p.C = b.gG + b.goff[0];
+    G.p.c_cell = b.PGs;
+    G.p.scm = z;
+    G.p.scn = 1;
+    ok = ok && map3(&G.a, b.A1, h, B, C, (uint64_t)B * h, 64, msg) &&
+         map3(&G.b, b.Z, z, B, C, (uint64_t)B * z, 64, msg);
+    finish(G);
+  }
+  P->n = i;
+  if (!ok) {
+    cudaFree(P->err);
+    delete P;
+    return nullptr;
+  }
+  return P;
+}
+
+int tcb_run(TcbPlan* P, int first, int count, cudaStream_t st, std::string* msg) {
+  for (int i = first; i < first + count && i < P->n; ++i) {
+    Gemm& G = P->g[i];
+    tcb::k_gemm_tc<<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+      if (msg) *msg = std::string("tensor-core backward launch: ") + cudaGetErrorString(e);
+      return 1;
+    }
+  }
+  return 0;
+}
+
+int* tcb_error_flag(TcbPlan* P) { return P ? P->err : nullptr; }
+
+void tcb_plan_destroy(TcbPlan* P) {
+  if (!P) return;
+  if (P->err) cudaFree(P->err);
+  delete P;
+}
+
+}  // namespace lipz

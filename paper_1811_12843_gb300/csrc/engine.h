@@ -39,6 +39,7 @@ struct SelectParams {
   int lr_mutation;
   float lr_mut_std;
   uint64_t lr_mut_thr;  // mutate iff word < thr (= floor(prob * 2^32))
+  float beta1, beta2;
 };
 
 void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout& lay, int cells,
@@ -60,10 +61,13 @@ void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaSt
 
 void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
                     float* fD, int* flag, cudaStream_t st);
+// Also writes, per cell and population, the Adam coefficients of the new centre's next step:
+// (lr, 1 / (1 - beta1^(step+1)), 1 / (1 - beta2^(step+1)), step + 1).
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
-                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old, int* sel_g,
-                   int* sel_d, int* src_g, int* src_d, float* lr_g_new, float* lr_d_new,
-                   cudaStream_t st);
+                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old,
+                   const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
+                   int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
+                   float4* coef_d, cudaStream_t st);
 template <typename T>
 void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
                        int x_dim, cudaStream_t st);
@@ -72,7 +76,7 @@ void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride
                    const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
                    int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st);
 void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, const int* src,
-                 const float* lr_new, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
+                 const float4* coef, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
                  float eps, cudaStream_t st);
 
 }  // namespace lipz

@@ -25,6 +25,7 @@
 
 #include "common.cuh"
 #include "fwd_tc.h"
+#include "tc_ptx.cuh"
 
 namespace lipz {
 namespace tc {
@@ -43,10 +44,9 @@ constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr int MISC_BYTES = 2048;
 constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + H_BYTES + MISC_BYTES;
-constexpr unsigned long long WAIT_NS = 1000000000ull;  // bound on any single wait
 
 enum { KIND_G = 0, KIND_D = 1 };
-enum { EPI_TO_H = 0, EPI_LOGIT = 1, EPI_TO_E = 2 };
+enum { EPI_TO_H = 0, EPI_LOGIT = 1, EPI_TO_E = 2, EPI_ACT_OUT = 3 };
 
 struct KParams {
   int kind;
@@ -66,6 +66,12 @@ struct KParams {
   float* logits;
   float slope;
   int* err;
+  // training forward: one problem per cell, weights of individual wsel[cell], and the
+  // activations of both hidden layers stored ([problem][rows][256] bf16) for the backward
+  int train;
+  const int* wsel;
+  bf16* act1;
+  bf16* act2;
 };
 
 struct Job {
@@ -84,7 +90,8 @@ __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   if (j == 0) {
     J = Job{0, p.kc1, HID, 0, 0, 0, HID, EPI_TO_H};
   } else if (j == 1) {
-    J = Job{1, HID / BK, HID, 1, 1, 0, HID, p.kind == KIND_D ? EPI_LOGIT : EPI_TO_H};
+    const int epi = p.kind == KIND_D ? EPI_LOGIT : (p.train ? EPI_ACT_OUT : EPI_TO_H);
+    J = Job{1, HID / BK, HID, 1, 1, 0, HID, epi};
   } else {
     const int nb = j - 2;
     const int n = min(N3, p.x - nb * N3);
@@ -93,132 +100,16 @@ __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   return J;
 }
 
-__device__ __forceinline__ int n_jobs(const KParams& p) { return p.kind == KIND_D ? 2 : 2 + p.n3; }
-
-// ---- PTX wrappers ------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
+__device__ __forceinline__ int n_jobs(const KParams& p) {
+  return (p.kind == KIND_D || p.train) ? 2 : 2 + p.n3;
 }
 
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+// Problem -> (cell whose activations are the A operand, individual whose weights are B).
+__device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
+  return p.train ? prob : prob / 5;
 }
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ unsigned long long globaltimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-// Bounded wait for the phase of `parity` to complete. Returns false (and raises the CTA's
-// abort flag and the kernel's error code) if it does not complete within WAIT_NS, or if
-// another role of the CTA has aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* err, int code) {
-  if (mbar_try(bar, parity)) return true;
-  const unsigned long long t0 = globaltimer();
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try(bar, parity)) return true;
-    if ((it & 255u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > WAIT_NS) {
-        *abort_flag = 1;
-        atomicExch(err, code);
-        return false;
-      }
-    }
-  }
-}
-
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int x, int y, int z) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"((uint64_t)map), "r"(x), "r"(y), "r"(z), "r"(bar)
-      : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   bar)
-               : "memory");
-}
-__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
-                                       uint32_t acc) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
-      "l"(a), "l"(b), "r"(idesc), "r"(acc)
-      : "memory");
-}
-
-// Shared-memory matrix descriptor of a K-major operand in the 128-byte swizzle layout: rows of
-// 128 bytes, 8-row groups 1024 bytes apart (stride byte offset), descriptor version 1.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)1 << 16;            // leading byte offset (unused for swizzled K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset
-  d |= (uint64_t)1 << 46;            // version
-  d |= (uint64_t)2 << 61;            // 128-byte swizzle
-  return d;
-}
-
-// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both K-major, N, M.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
-         ((uint32_t)(M >> 4) << 24);
-}
-
-#define LIPZ_TMEM_LD32(taddr, r)                                                                 \
-  asm volatile(                                                                                  \
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14," \
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"             \
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),      \
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),  \
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),            \
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),            \
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])             \
-      : "r"(taddr))
-
-#define LIPZ_TMEM_LD16(taddr, r)                                                                 \
-  asm volatile(                                                                                  \
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14," \
-      "%15}, [%16];"                                                                             \
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),      \
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),  \
-        "=r"(r[14]), "=r"(r[15])                                                                 \
-      : "r"(taddr))
-
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
+__device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
+  return p.train ? __ldg(&p.wsel[prob]) : __ldg(&p.nbr[prob]);
 }
 
 // ---- the kernel ----------------------------------------------------------------------------
@@ -282,8 +173,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
-        const int c = prob / 5;
-        const int k = __ldg(&p.nbr[prob]);
+        const int c = prob_cell(p, prob);
+        const int k = prob_individual(p, prob);
         for (int j = 0; j < nj && ok; ++j) {
           const Job J = get_job(p, j);
           const CUtensorMap* mb = J.bmap == 0 ? &mB1 : (J.bmap == 1 ? &mB2 : &mB3);
@@ -386,9 +277,12 @@ __global__ void __launch_bounds__(THREADS, 1)
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
-      const int c = prob / 5, slot = prob % 5;
-      const int k = __ldg(&p.nbr[prob]);
+      const int c = prob_cell(p, prob), slot = prob % 5;
+      const int k = prob_individual(p, prob);
       const float* wm = p.wmaster + (int64_t)k * p.pstride;
+      const int rr = m0 + row;
+      const bool row_ok = rr < p.rows;
+      const int64_t act_off = ((int64_t)prob * p.rows + rr) * HID;
       for (int j = 0; j < nj && ok; ++j) {
         const Job J = get_job(p, j);
         const int R = J.region;
@@ -398,9 +292,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         tc_fence_after();
         const uint32_t tbase = tmem + lane_base + (uint32_t)(R * HID);
-        if (J.epi == EPI_TO_H) {
+        if (J.epi == EPI_TO_H || J.epi == EPI_ACT_OUT) {
           const float* bias = wm + (j == 0 ? p.off_b1 : p.off_b2);
           const bool lrelu = p.kind == KIND_D;
+          const bool to_h = J.epi == EPI_TO_H;
+          bf16* gout = j == 0 ? p.act1 : p.act2;
 #pragma unroll 1
           for (int cg = hf * 4; cg < hf * 4 + 4; ++cg) {
             uint32_t r[32];
@@ -415,21 +311,29 @@ __global__ void __launch_bounds__(THREADS, 1)
               a1 = a1 > 0.f ? a1 : (lrelu ? p.slope * a1 : 0.f);
               pk[e >> 1] = pack_bf16(a0, a1);
             }
-            const uint32_t chunk = sH + (uint32_t)((cg >> 1) * H_CHUNK) + (uint32_t)row * 128u;
+            if (to_h) {
+              const uint32_t chunk = sH + (uint32_t)((cg >> 1) * H_CHUNK) + (uint32_t)row * 128u;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const uint32_t unit = (uint32_t)((cg & 1) * 4 + u);
-              const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
-              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
-                           "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]),
-                           "r"(pk[4 * u + 3])
-                           : "memory");
+              for (int u = 0; u < 4; ++u) {
+                const uint32_t unit = (uint32_t)((cg & 1) * 4 + u);
+                const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
+                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                             "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]),
+                             "r"(pk[4 * u + 3])
+                             : "memory");
+              }
+            }
+            if (gout && row_ok) {
+              uint4* o = reinterpret_cast<uint4*>(gout + act_off + cg * 32);
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
             }
           }
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          if (to_h) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           tc_fence_before();
           mbar_arrive(bReg + 8 * R);
-          mbar_arrive(bH);
+          if (to_h) mbar_arrive(bH);
         } else if (J.epi == EPI_LOGIT) {
           const float* bias = wm + p.off_b2;
           const bf16* w3 = p.wb + (int64_t)k * p.pstride + p.off_w3;
@@ -439,12 +343,23 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t r[32];
             LIPZ_TMEM_LD32(tbase + cg * 32, r);
             tmem_wait_ld();
+            uint32_t pk[16];
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              float a = __uint_as_float(r[e]) + __ldg(&bias[cg * 32 + e]);
-              a = a > 0.f ? a : p.slope * a;
-              a = __bfloat162float(__float2bfloat16_rn(a));
-              acc = fmaf(a, __bfloat162float(w3[cg * 32 + e]), acc);
+            for (int e = 0; e < 32; e += 2) {
+              float a0 = __uint_as_float(r[e]) + __ldg(&bias[cg * 32 + e]);
+              float a1 = __uint_as_float(r[e + 1]) + __ldg(&bias[cg * 32 + e + 1]);
+              a0 = a0 > 0.f ? a0 : p.slope * a0;
+              a1 = a1 > 0.f ? a1 : p.slope * a1;
+              pk[e >> 1] = pack_bf16(a0, a1);
+              const __nv_bfloat162 q2 = *reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]);
+              acc = fmaf(__low2float(q2), __bfloat162float(w3[cg * 32 + e]), acc);
+              acc = fmaf(__high2float(q2), __bfloat162float(w3[cg * 32 + e + 1]), acc);
+            }
+            if (p.act2 && row_ok) {
+              uint4* o = reinterpret_cast<uint4*>(p.act2 + act_off + cg * 32);
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
             }
           }
           tc_fence_before();
@@ -459,15 +374,13 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             const float logit = acc + part[row] + __ldg(wm + p.off_b3);
             mbar_arrive(bReg + 8 * R);
-            const int rr = m0 + row;
-            if (rr < p.rows) p.logits[(int64_t)prob * p.rows + rr] = logit;
+            if (row_ok) p.logits[(int64_t)prob * p.rows + rr] = logit;
           }
         } else {
           // generator output block: bias + tanh, bf16, into the fake rows of E[c]
           const float* bias = wm + p.off_b3;
           const int ng = J.n / 16;
           const int g0 = hf ? 4 : 0, g1 = hf ? ng : min(4, ng);
-          const int rr = m0 + row;
           bf16* dst = p.E + (int64_t)c * p.e_cell + (int64_t)((1 + slot) * p.B + rr) * p.x;
 #pragma unroll 1
           for (int gi = g0; gi < g1; ++gi) {
@@ -508,9 +421,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 // ---- host side -----------------------------------------------------------------------------
 struct TcPlan {
   TcShape s;
-  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2;
-  tc::KParams pg, pd;
-  int grid_g, grid_d;
+  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mTX;
+  tc::KParams pg, pd, pgt, pdt;
+  int grid_g, grid_d, grid_gt, grid_dt;
   int* err;
 };
 
@@ -557,10 +470,7 @@ bool tc_supported(int z, int h, int x, int B) {
   return h == tc::HID && z % 16 == 0 && z >= 64 && z <= 256 && x % 16 == 0 && x >= 64 && B >= 1;
 }
 
-TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float* logits,
-                       const int* nbr, const __nv_bfloat16* Gwb, const float* Gw, int64_t PGs,
-                       const int64_t* goff, const __nv_bfloat16* Dwb, const float* Dw,
-                       int64_t PDs, const int64_t* doff, std::string* msg) {
+TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   if (!tc_supported(s.z, s.h, s.x, s.B)) {
     if (msg) *msg = "shape not supported by the tensor-core forward";
     return nullptr;
@@ -570,18 +480,20 @@ TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float
   memset(p, 0, sizeof *p);
   p->s = s;
   const uint64_t C = s.cells, B = s.B, z = s.z, x = s.x, h = s.h;
-  bool ok = make_map(&p->mZ, Z, z, B, C, z * 2, B * z * 2, 128, msg) &&
-            make_map(&p->mE, E, x, 6 * B, C, x * 2, (uint64_t)e_cell * 2, 128, msg) &&
-            make_map(&p->mG1, Gwb + goff[0], z, h, C, z * 2, PGs * 2, 256, msg) &&
-            make_map(&p->mG2, Gwb + goff[2], h, h, C, h * 2, PGs * 2, 256, msg) &&
-            make_map(&p->mG3, Gwb + goff[4], h, x, C, h * 2, PGs * 2, tc::N3, msg) &&
-            make_map(&p->mD1, Dwb + doff[0], x, h, C, x * 2, PDs * 2, 256, msg) &&
-            make_map(&p->mD2, Dwb + doff[2], h, h, C, h * 2, PDs * 2, 256, msg);
+  bool ok = make_map(&p->mZ, b.Z, z, B, C, z * 2, B * z * 2, 128, msg) &&
+            make_map(&p->mE, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 128, msg) &&
+            make_map(&p->mTX, b.TX, x, 2 * B, C, x * 2, 2 * B * x * 2, 128, msg) &&
+            make_map(&p->mG1, b.Gwb + b.goff[0], z, h, C, z * 2, b.PGs * 2, 256, msg) &&
+            make_map(&p->mG2, b.Gwb + b.goff[2], h, h, C, h * 2, b.PGs * 2, 256, msg) &&
+            make_map(&p->mG3, b.Gwb + b.goff[4], h, x, C, h * 2, b.PGs * 2, tc::N3, msg) &&
+            make_map(&p->mD1, b.Dwb + b.doff[0], x, h, C, x * 2, b.PDs * 2, 256, msg) &&
+            make_map(&p->mD2, b.Dwb + b.doff[2], h, h, C, h * 2, b.PDs * 2, 256, msg);
   if (!ok) {
     delete p;
     return nullptr;
   }
-  if (cudaMalloc(&p->err, sizeof(int)) != cudaSuccess || cudaMemset(p->err, 0, sizeof(int)) != cudaSuccess) {
+  if (cudaMalloc(&p->err, sizeof(int)) != cudaSuccess ||
+      cudaMemset(p->err, 0, sizeof(int)) != cudaSuccess) {
     cudaGetLastError();
     if (msg) *msg = "cudaMalloc for the error flag failed";
     delete p;
@@ -598,6 +510,7 @@ TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float
     delete p;
     return nullptr;
   }
+  auto tiles = [](int rows) { return (rows + tc::BM - 1) / tc::BM; };
   tc::KParams g{};
   g.kind = tc::KIND_G;
   g.cells = s.cells;
@@ -605,64 +518,95 @@ TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float
   g.z = s.z;
   g.x = s.x;
   g.rows = s.B;
-  g.mtiles = (s.B + tc::BM - 1) / tc::BM;
+  g.mtiles = tiles(s.B);
   g.n_tiles = s.cells * 5 * g.mtiles;
   g.kc1 = (s.z + tc::BK - 1) / tc::BK;
   g.n3 = (s.x + tc::N3 - 1) / tc::N3;
-  g.nbr = nbr;
-  g.wmaster = Gw;
-  g.wb = Gwb;
-  g.pstride = PGs;
-  g.off_b1 = goff[1];
-  g.off_b2 = goff[3];
-  g.off_b3 = goff[5];
-  g.off_w3 = goff[4];
-  g.E = (bf16*)E;
-  g.e_cell = e_cell;
-  g.logits = logits;
+  g.nbr = b.nbr;
+  g.wmaster = b.Gw;
+  g.wb = b.Gwb;
+  g.pstride = b.PGs;
+  g.off_b1 = b.goff[1];
+  g.off_b2 = b.goff[3];
+  g.off_b3 = b.goff[5];
+  g.off_w3 = b.goff[4];
+  g.E = (bf16*)b.E;
+  g.e_cell = b.e_cell;
+  g.logits = b.logits;
   g.slope = s.slope;
   g.err = p->err;
   tc::KParams d = g;
   d.kind = tc::KIND_D;
   d.rows = 6 * s.B;
-  d.mtiles = (6 * s.B + tc::BM - 1) / tc::BM;
+  d.mtiles = tiles(6 * s.B);
   d.n_tiles = s.cells * 5 * d.mtiles;
   d.kc1 = (s.x + tc::BK - 1) / tc::BK;
   d.n3 = 0;
-  d.wmaster = Dw;
-  d.wb = Dwb;
-  d.pstride = PDs;
-  d.off_b1 = doff[1];
-  d.off_b2 = doff[3];
-  d.off_b3 = doff[5];
-  d.off_w3 = doff[4];
+  d.wmaster = b.Dw;
+  d.wb = b.Dwb;
+  d.pstride = b.PDs;
+  d.off_b1 = b.doff[1];
+  d.off_b2 = b.doff[3];
+  d.off_b3 = b.doff[5];
+  d.off_w3 = b.doff[4];
+  tc::KParams gt = g;  // selected generator of each cell on its own z: both hidden layers
+  gt.train = 1;
+  gt.wsel = b.src_g;
+  gt.n_tiles = s.cells * g.mtiles;
+  gt.act1 = (bf16*)b.TH1;
+  gt.act2 = (bf16*)b.TH2;
+  tc::KParams dt = d;  // selected discriminator on [x_c; selected fakes]
+  dt.train = 1;
+  dt.wsel = b.src_d;
+  dt.rows = 2 * s.B;
+  dt.mtiles = tiles(2 * s.B);
+  dt.n_tiles = s.cells * dt.mtiles;
+  dt.act1 = (bf16*)b.TG1;
+  dt.act2 = (bf16*)b.TG2;
+  dt.logits = b.TL;
   p->pg = g;
   p->pd = d;
-  p->grid_g = g.n_tiles < sms ? g.n_tiles : sms;
-  p->grid_d = d.n_tiles < sms ? d.n_tiles : sms;
+  p->pgt = gt;
+  p->pdt = dt;
+  auto grid = [sms](int n) { return n < sms ? n : sms; };
+  p->grid_g = grid(g.n_tiles);
+  p->grid_d = grid(d.n_tiles);
+  p->grid_gt = grid(gt.n_tiles);
+  p->grid_dt = grid(dt.n_tiles);
   return p;
 }
 
-int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg) {
-  tc::k_mlp_fwd<<<p->grid_g, tc::THREADS, tc::SMEM_BYTES, st>>>(p->mZ, p->mG1, p->mG2, p->mG3,
-                                                                p->pg);
+namespace {
+int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensorMap& b2,
+           const CUtensorMap& b3, const tc::KParams& kp, cudaStream_t st, const char* what,
+           std::string* msg) {
+  tc::k_mlp_fwd<<<grid, tc::THREADS, tc::SMEM_BYTES, st>>>(a, b1, b2, b3, kp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
-    if (msg) *msg = std::string("generator forward launch: ") + cudaGetErrorString(e);
+    if (msg) *msg = std::string(what) + " launch: " + cudaGetErrorString(e);
     return 1;
   }
   return 0;
 }
+}  // namespace
+
+int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg) {
+  return launch(p->grid_g, p->mZ, p->mG1, p->mG2, p->mG3, p->pg, st, "generator forward", msg);
+}
 
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg) {
-  tc::k_mlp_fwd<<<p->grid_d, tc::THREADS, tc::SMEM_BYTES, st>>>(p->mE, p->mD1, p->mD2, p->mD2,
-                                                                p->pd);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) {
-    if (msg) *msg = std::string("discriminator forward launch: ") + cudaGetErrorString(e);
-    return 1;
-  }
-  return 0;
+  return launch(p->grid_d, p->mE, p->mD1, p->mD2, p->mD2, p->pd, st, "discriminator forward",
+                msg);
+}
+
+int tc_run_train_g(TcPlan* p, cudaStream_t st, std::string* msg) {
+  return launch(p->grid_gt, p->mZ, p->mG1, p->mG2, p->mG3, p->pgt, st, "generator training forward",
+                msg);
+}
+
+int tc_run_train_d(TcPlan* p, cudaStream_t st, std::string* msg) {
+  return launch(p->grid_dt, p->mTX, p->mD1, p->mD2, p->mD2, p->pdt, st,
+                "discriminator training forward", msg);
 }
 
 int* tc_error_flag(TcPlan* p) { return p ? p->err : nullptr; }

@@ -21,20 +21,47 @@ struct TcPlan;
 // hidden == 256, z and x multiples of 16, 16 <= z <= 256, 16 <= x, batch >= 1.
 bool tc_supported(int z, int h, int x, int B);
 
-// Builds the TMA descriptors and launch parameters for one population snapshot. Z: [cells][B][z]
-// bf16; E: [cells][6B][x] bf16 (rows [0, B) real, then the fakes of slots 0..4, which the
-// generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5] on the device. Weights:
-// bf16 copies (Gwb, Dwb) and fp32 masters (for the biases), per-cell strides PGs / PDs, tensor
-// offsets goff / doff (W1, b1, W2, b2, W3, b3). Returns null and a message on failure.
-TcPlan* tc_plan_create(const TcShape& s, void* Z, void* E, int64_t e_cell, float* logits,
-                       const int* nbr, const __nv_bfloat16* Gwb, const float* Gw, int64_t PGs,
-                       const int64_t* goff, const __nv_bfloat16* Dwb, const float* Dw,
-                       int64_t PDs, const int64_t* doff, std::string* msg);
+// Device buffers of one population snapshot that the tensor-core forward reads and writes.
+//   Z: [cells][B][z] bf16; E: [cells][6B][x] bf16 (rows [0, B) real, then the fakes of slots
+//   0..4, which the generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5].
+//   Weights: bf16 copies (Gwb, Dwb) and fp32 masters (biases), per-individual strides
+//   PGs / PDs, tensor offsets goff / doff (W1, b1, W2, b2, W3, b3).
+//   Training forward of the selected pairs: TX [cells][2B][x] bf16 (real rows, then the
+//   selected generator's fakes), src_g / src_d [cells] (selected individuals), outputs
+//   TH1, TH2 [cells][B][256], TG1, TG2 [cells][2B][256] bf16 and TL [cells][2B] fp32.
+struct TcBuffers {
+  void* Z;
+  void* E;
+  int64_t e_cell;
+  float* logits;
+  const int* nbr;
+  const __nv_bfloat16* Gwb;
+  const float* Gw;
+  int64_t PGs;
+  const int64_t* goff;
+  const __nv_bfloat16* Dwb;
+  const float* Dw;
+  int64_t PDs;
+  const int64_t* doff;
+  void* TX;
+  const int* src_g;
+  const int* src_d;
+  void *TH1, *TH2, *TG1, *TG2;
+  float* TL;
+};
+
+// Builds the TMA descriptors and launch parameters for one population snapshot. Returns null
+// and a message on failure.
+TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg);
 
 // Enqueue the generator kernel (fakes of every (cell, slot)) / the discriminator kernel (logits
 // of every (cell, slot)) on `st`. 0 on success.
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
+// Training forward of every cell's selected generator (hidden activations into TH1, TH2) and
+// selected discriminator (TG1, TG2 and the logits TL).
+int tc_run_train_g(TcPlan* p, cudaStream_t st, std::string* msg);
+int tc_run_train_d(TcPlan* p, cudaStream_t st, std::string* msg);
 
 // Device int that a kernel of the plan sets to a non-zero code when one of its bounded waits
 // expired (the kernel then stopped early); the host reads and clears it.

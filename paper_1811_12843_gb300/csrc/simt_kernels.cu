@@ -345,9 +345,11 @@ __device__ float mutate(float lr, uint64_t seed, uint32_t stream, uint32_t t, ui
 __global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
                          const int* __restrict__ nbr, int cells, SelectParams p,
                          const float* __restrict__ lr_g_old, const float* __restrict__ lr_d_old,
+                         const int* __restrict__ step_g_old, const int* __restrict__ step_d_old,
                          int* __restrict__ sel_g, int* __restrict__ sel_d, int* __restrict__ src_g,
                          int* __restrict__ src_d, float* __restrict__ lr_g_new,
-                         float* __restrict__ lr_d_new) {
+                         float* __restrict__ lr_d_new, float4* __restrict__ coef_g,
+                         float4* __restrict__ coef_d) {
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= cells) return;
   for (int pop = 0; pop < 2; ++pop) {
@@ -361,6 +363,11 @@ __global__ void k_select(const float* __restrict__ fG, const float* __restrict__
     float lr = (pop ? lr_d_old : lr_g_old)[src];
     if (p.lr_mutation) lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std,
                                    p.lr_mut_thr);
+    const int step1 = (pop ? step_d_old : step_g_old)[src] + 1;
+    const float4 cf = make_float4(lr, (float)(1.0 / (1.0 - pow((double)p.beta1, (double)step1))),
+                                  (float)(1.0 / (1.0 - pow((double)p.beta2, (double)step1))),
+                                  (float)step1);
+    (pop ? coef_d : coef_g)[c] = cf;
     if (pop) {
       sel_d[c] = s;
       src_d[c] = src;
@@ -374,11 +381,13 @@ __global__ void k_select(const float* __restrict__ fG, const float* __restrict__
 }
 
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
-                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old, int* sel_g,
-                   int* sel_d, int* src_g, int* src_d, float* lr_g_new, float* lr_d_new,
-                   cudaStream_t st) {
-  k_select<<<(cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old, sel_g,
-                                                sel_d, src_g, src_d, lr_g_new, lr_d_new);
+                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old,
+                   const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
+                   int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
+                   float4* coef_d, cudaStream_t st) {
+  k_select<<<(cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old,
+                                                step_g_old, step_d_old, sel_g, sel_d, src_g, src_d,
+                                                lr_g_new, lr_d_new, coef_g, coef_d);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -466,74 +475,87 @@ template void launch_dlogit<bf16>(const float*, const bf16*, const bf16*, int64_
 // ------------------------------------------------------------------------------------------
 // Adam (Kingma & Ba 2015, Algorithm 1) fused with the replacement copy: the new centre of
 // cell c starts from individual src[c] of the old snapshot and is written to cell c of the
-// new snapshot (fp32 master, m, v, bf16 copy, step, lr).
+// new snapshot (fp32 master, m, v, bf16 copy, step, lr). HBM-bound: 16-byte loads/stores,
+// each thread walks float4 groups of its cell with a grid stride.
 // ------------------------------------------------------------------------------------------
-__global__ void k_adam(PopView old_p, PopView new_p, const float* __restrict__ grad,
-                       const int* __restrict__ src, const float* __restrict__ lr_new,
-                       int64_t P, int64_t Ps, float beta1, float beta2, float eps) {
+__device__ __forceinline__ void adam4(float4& w, float4& m, float4& v, const float4 g, float b1,
+                                      float b2, float lr, float ib1, float ib2, float eps) {
+  float* wv = &w.x;
+  float* mv = &m.x;
+  float* vv = &v.x;
+  const float* gv = &g.x;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    mv[e] = b1 * mv[e] + (1.f - b1) * gv[e];
+    vv[e] = b2 * vv[e] + (1.f - b2) * gv[e] * gv[e];
+    wv[e] = wv[e] - lr * (mv[e] * ib1) / (sqrtf(vv[e] * ib2) + eps);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_adam(PopView old_p, PopView new_p,
+                                              const float* __restrict__ grad,
+                                              const int* __restrict__ src,
+                                              const float4* __restrict__ coef, int64_t P,
+                                              int64_t Ps, float beta1, float beta2, float eps) {
   const int c = blockIdx.y;
   const int s = src[c];
-  __shared__ float coef[2];
-  if (threadIdx.x == 0) {
-    const int step1 = old_p.step[s] + 1;
-    const double bc1 = 1.0 - pow((double)beta1, (double)step1);
-    const double bc2 = 1.0 - pow((double)beta2, (double)step1);
-    coef[0] = (float)(1.0 / bc1);
-    coef[1] = (float)(1.0 / bc2);
-    if (blockIdx.x == 0) {
-      new_p.step[c] = step1;
-      new_p.lr[c] = lr_new[c];
+  const float4 cf = coef[c];
+  const float lr = cf.x, ib1 = cf.y, ib2 = cf.z;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    new_p.step[c] = (int)cf.w;
+    new_p.lr[c] = lr;
+  }
+  const int64_t so = (int64_t)s * Ps, co = (int64_t)c * Ps;
+  const int64_t n4 = P >> 2;
+  const float4* __restrict__ w_in = reinterpret_cast<const float4*>(old_p.w + so);
+  const float4* __restrict__ m_in = reinterpret_cast<const float4*>(old_p.m + so);
+  const float4* __restrict__ v_in = reinterpret_cast<const float4*>(old_p.v + so);
+  const float4* __restrict__ g_in = reinterpret_cast<const float4*>(grad + co);
+  float4* w_out = reinterpret_cast<float4*>(new_p.w + co);
+  float4* m_out = reinterpret_cast<float4*>(new_p.m + co);
+  float4* v_out = reinterpret_cast<float4*>(new_p.v + co);
+  uint2* b_out = new_p.wb ? reinterpret_cast<uint2*>(new_p.wb + co) : nullptr;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    float4 w = __ldcs(w_in + i), m = __ldcs(m_in + i), v = __ldcs(v_in + i);
+    const float4 g = __ldcs(g_in + i);
+    adam4(w, m, v, g, beta1, beta2, lr, ib1, ib2, eps);
+    __stcs(w_out + i, w);
+    __stcs(m_out + i, m);
+    __stcs(v_out + i, v);
+    if (b_out) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(w.x, w.y);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(w.z, w.w);
+      uint2 pk;
+      pk.x = *reinterpret_cast<uint32_t*>(&lo);
+      pk.y = *reinterpret_cast<uint32_t*>(&hi);
+      b_out[i] = pk;
     }
   }
-  __syncthreads();
-  const float lr = lr_new[c], ib1 = coef[0], ib2 = coef[1];
-  const int64_t so = (int64_t)s * Ps, co = (int64_t)c * Ps;
-  const int64_t k0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
-  if (k0 >= P) return;
-  if (k0 + 3 < P) {
-    const float4 w = *(const float4*)(old_p.w + so + k0);
-    const float4 m = *(const float4*)(old_p.m + so + k0);
-    const float4 v = *(const float4*)(old_p.v + so + k0);
-    const float4 g = *(const float4*)(grad + co + k0);
-    float wv[4] = {w.x, w.y, w.z, w.w}, mv[4] = {m.x, m.y, m.z, m.w};
-    float vv[4] = {v.x, v.y, v.z, v.w};
-    const float gv[4] = {g.x, g.y, g.z, g.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      mv[e] = beta1 * mv[e] + (1.f - beta1) * gv[e];
-      vv[e] = beta2 * vv[e] + (1.f - beta2) * gv[e] * gv[e];
-      wv[e] = wv[e] - lr * (mv[e] * ib1) / (sqrtf(vv[e] * ib2) + eps);
-    }
-    *(float4*)(new_p.w + co + k0) = make_float4(wv[0], wv[1], wv[2], wv[3]);
-    *(float4*)(new_p.m + co + k0) = make_float4(mv[0], mv[1], mv[2], mv[3]);
-    *(float4*)(new_p.v + co + k0) = make_float4(vv[0], vv[1], vv[2], vv[3]);
-    if (new_p.wb) {
-      __nv_bfloat162 lo = __floats2bfloat162_rn(wv[0], wv[1]);
-      __nv_bfloat162 hi = __floats2bfloat162_rn(wv[2], wv[3]);
-      uint2 pk;
-      pk.x = *(uint32_t*)&lo;
-      pk.y = *(uint32_t*)&hi;
-      *(uint2*)(new_p.wb + co + k0) = pk;
-    }
-  } else {
-    for (int64_t k = k0; k < P; ++k) {
-      const float gk = grad[co + k];
-      const float mk = beta1 * old_p.m[so + k] + (1.f - beta1) * gk;
-      const float vk = beta2 * old_p.v[so + k] + (1.f - beta2) * gk * gk;
-      const float wk = old_p.w[so + k] - lr * (mk * ib1) / (sqrtf(vk * ib2) + eps);
-      new_p.w[co + k] = wk;
-      new_p.m[co + k] = mk;
-      new_p.v[co + k] = vk;
-      if (new_p.wb) new_p.wb[co + k] = __float2bfloat16_rn(wk);
-    }
+  // tail (P not a multiple of 4)
+  if (blockIdx.x == 0 && threadIdx.x < (P & 3)) {
+    const int64_t k = (n4 << 2) + threadIdx.x;
+    const float gk = grad[co + k];
+    const float mk = beta1 * old_p.m[so + k] + (1.f - beta1) * gk;
+    const float vk = beta2 * old_p.v[so + k] + (1.f - beta2) * gk * gk;
+    const float wk = old_p.w[so + k] - lr * (mk * ib1) / (sqrtf(vk * ib2) + eps);
+    new_p.w[co + k] = wk;
+    new_p.m[co + k] = mk;
+    new_p.v[co + k] = vk;
+    if (new_p.wb) new_p.wb[co + k] = __float2bfloat16_rn(wk);
   }
 }
 
 void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, const int* src,
-                 const float* lr_new, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
+                 const float4* coef, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
                  float eps, cudaStream_t st) {
-  dim3 grid((unsigned)((P / 4 + 1 + 255) / 256), cells);
-  k_adam<<<grid, 256, 0, st>>>(old_p, new_p, grad, src, lr_new, P, Ps, beta1, beta2, eps);
+  // about 8 resident 256-thread blocks per SM over the whole population
+  int per_cell = (int)((P / 4 + 255) / 256);
+  const int target = (152 * 8 + cells - 1) / cells;
+  if (per_cell > target * 4) per_cell = target * 4;
+  if (per_cell < 1) per_cell = 1;
+  dim3 grid(per_cell, cells);
+  k_adam<<<grid, 256, 0, st>>>(old_p, new_p, grad, src, coef, P, Ps, beta1, beta2, eps);
 }
 
 }  // namespace lipz

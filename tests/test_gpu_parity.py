@@ -148,9 +148,10 @@ def _one_iteration_check(L, g, pool, tol, x_host=None, kink_band=1e-5):
         w1 = O.adam_step(s.Gw[sg], s.Gm[sg], s.Gv[sg], s.Gstep[sg], gg[c].astype(np.float64),
                          float(np.float32(s.Glr[sg])), a)[0]
         assert np.max(np.abs(got.Gw[c] - w1)) <= 1e-6 * np.max(np.abs(w1)) + 1e-9
-    # updated weights against the oracle's own iteration; an element beyond the tolerance is
-    # allowed only where Adam's sign-like first step follows a gradient whose sign is within the
-    # engine's accumulation noise (|g_ref| <= |g_gpu - g_ref|)
+    # updated weights against the oracle's own iteration. Adam's early steps move an element by
+    # about lr * sign(g), so an element whose gradient lies within the comparison's noise band
+    # of zero may move the other way: such an element (|g_ref| <= 2 |g_gpu - g_ref| +
+    # tol * max|g_ref| of its tensor) is allowed to differ; all others meet the tolerance.
     flagged = 0
     for pop, lay, gref, ggpu in (("Gw", O.g_layout(a), grads["gG"], gg),
                                  ("Dw", O.d_layout(a), grads["gD"], gd)):
@@ -164,7 +165,8 @@ def _one_iteration_check(L, g, pool, tol, x_host=None, kink_band=1e-5):
             bad = (d > tol * np.max(np.abs(w_ref[:, sl]))) & ok[:, None]
             if np.any(bad):
                 gr, gq = gref[:, sl][bad], ggpu[:, sl][bad].astype(np.float64)
-                assert np.all(np.abs(gr) <= np.abs(gq - gr) + 1e-12), (pop, name)
+                band = tol * np.max(np.abs(gref[:, sl]))
+                assert np.all(np.abs(gr) <= 2 * np.abs(gq - gr) + band + 1e-12), (pop, name)
                 flagged += int(bad.sum())
     return flagged
 
@@ -290,4 +292,5 @@ def test_full_size_12x12_bf16_sampled_cells(L):
     # every weight moved by at most lr (Adam's first step is bounded by lr per element)
     nbr = O.neighbors(12, 12)
     src = nbr[np.arange(144), sel["sel_g"]]
-    assert np.max(np.abs(got.Gw - s.Gw[src])) <= 2e-4 * (1 + 1e-5)
+    ulp = 2 * np.spacing(np.float32(np.max(np.abs(s.Gw))))
+    assert np.max(np.abs(got.Gw - s.Gw[src])) <= 2e-4 * (1 + 1e-5) + ulp
