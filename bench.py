@@ -164,14 +164,53 @@ def run_ours(args):
     value = PAIRS * world * iters_s
 
     # ---- per-phase device time (separate pass with phase events on the same stream)
-    L.lipz_profile_enable(g.h, True)
-    for _ in range(args.steps):
-        L.lipz_iterate(g.h, 1)
-    prof = L.lipz_profile_read(g.h)
-    L.lipz_profile_enable(g.h, False)
-    phase_ms = {k: v[0] / max(v[1], 1) for k, v in prof.items()}
+    phase_ms = {k: float("nan") for k in L.PHASES}
+    if not args.no_phases:
+        L.lipz_profile_enable(g.h, True)
+        for _ in range(args.steps):
+            L.lipz_iterate(g.h, 1)
+        prof = L.lipz_profile_read(g.h)
+        L.lipz_profile_enable(g.h, False)
+        phase_ms = {k: v[0] / max(v[1], 1) for k, v in prof.items()}
 
     # ---- end to end through the public API: pinned host minibatches in, fitness out
+    if args.no_e2e:
+        e2e_value = None
+    else:
+        e2e_value = _e2e(args, L, g, torch, dist, world)
+    h2d = CELLS * BATCH * X_DIM * 4
+    d2h = 2 * CELLS * 5 * 4
+    if args.no_phases:
+        roof = None
+    else:
+        roof = _roofline(phase_ms)
+    if rank != 0:
+        return None
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
+        "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+                   "pairs_per_iter": PAIRS, "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (population 2.2 GB + pool 188 MB per iteration)"},
+        "grid_iterations_per_sec": iters_s * world,
+        "pair_evals_per_sec_eval_only": PAIRS * world * 1000.0 /
+        (phase_ms["batch"] + phase_ms["g_fwd"] + phase_ms["d_fwd"] + phase_ms["fitness"]),
+        "phase_ms": phase_ms,
+        "roofline": roof,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+    return line
+
+
+def _e2e(args, L, g, torch, dist, world):
+    import lipz_synth
     nbuf = 2
     xs = [torch.from_numpy(lipz_synth.host_batch(SEED + 7 + i, CELLS, BATCH, X_DIM)).pin_memory()
           for i in range(nbuf)]
@@ -179,7 +218,9 @@ def run_ours(args):
     fd = torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()
     for i in range(2):
         L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
-    barrier()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
     t0 = time.perf_counter()
     for i in range(args.steps):
         L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
@@ -188,11 +229,11 @@ def run_ours(args):
         t = torch.tensor([e2e_s], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
-    e2e_value = PAIRS * world * args.steps / e2e_s
-    h2d = CELLS * BATCH * X_DIM * 4
-    d2h = 2 * CELLS * 5 * 4
+    return PAIRS * world * args.steps / e2e_s
 
-    # ---- roofline of the dominant kernel phase
+
+def _roofline(phase_ms):
+    """Roofline of the phase with the largest device time."""
     hbm, tf_burst, tf_sus, peak_kind = _peaks()
     dom = max(("g_fwd", "d_fwd", "train_fwd", "train_bwd", "adam"), key=lambda k: phase_ms[k])
     if dom == "d_fwd":
@@ -220,30 +261,7 @@ def run_ours(args):
     roof["peak_source"] = peak_kind + (" sustained bf16" if roof["unit"] == "TFLOP/s" else " HBM copy")
     roof["traffic"] = None
     roof["phase"] = dom
-
-    if rank != 0:
-        return None
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
-        "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
-                   "pairs_per_iter": PAIRS, "parallelism": "replicas" if world > 1 else "single",
-                   "l2": "inputs larger than L2 (population 2.2 GB + pool 188 MB per iteration)"},
-        "grid_iterations_per_sec": iters_s * world,
-        "pair_evals_per_sec_eval_only": PAIRS * world * 1000.0 /
-        (phase_ms["batch"] + phase_ms["g_fwd"] + phase_ms["d_fwd"] + phase_ms["fitness"]),
-        "phase_ms": phase_ms,
-        "roofline": roof,
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
-        "gpu_launches": launches,
-        "clocks": clk.summary(),
-    }
-    if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
-    return line
+    return roof
 
 
 def _oracle_sample(seconds, max_cells=None):
@@ -348,6 +366,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass")
+    ap.add_argument("--no-phases", action="store_true", help="skip the per-phase timing pass")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
