@@ -208,11 +208,24 @@ __global__ void __launch_bounds__(THREADS, 2)
           bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
           const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
           float v[16];
+          if (p.sxn == 1 && col0 + 16 <= p.N) {
+            // the row's 16 aux values are contiguous: two 16-byte loads
+            const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
+            const uint4 q0 = __ldg(x4), q1 = __ldg(x4 + 1);
+            const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
 #pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const int col = col0 + e;
-            const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
-            v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
+            for (int e = 0; e < 16; e += 2) {
+              const __nv_bfloat162 y2 = *reinterpret_cast<const __nv_bfloat162*>(&w[e >> 1]);
+              v[e] = __uint_as_float(r[e]) * dact(p.act, __low2float(y2), p.slope);
+              v[e + 1] = __uint_as_float(r[e + 1]) * dact(p.act, __high2float(y2), p.slope);
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              const int col = col0 + e;
+              const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
+              v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
+            }
           }
           if (p.scn == 1 && col0 + 16 <= p.N) {
             uint32_t pk[8];

@@ -226,23 +226,43 @@ template void launch_gemv<float>(const GemvDesc*, int, int, cudaStream_t);
 template void launch_gemv<bf16>(const GemvDesc*, int, int, cudaStream_t);
 
 // ------------------------------------------------------------------------------------------
-// Column sums (bias gradients): one thread per column, rows in order.
+// Column sums (bias gradients). A block takes 64 columns of one problem: 32 lanes own two
+// adjacent columns each, 8 row groups stride over the rows, and the 8 partial sums are added
+// in a fixed order (deterministic).
 // ------------------------------------------------------------------------------------------
 template <typename T>
-__global__ void k_colsum(const ColSumDesc* __restrict__ descs) {
+__global__ void __launch_bounds__(256) k_colsum(const ColSumDesc* __restrict__ descs) {
   const ColSumDesc d = descs[blockIdx.y];
-  const int n = blockIdx.x * blockDim.x + threadIdx.x;
-  if (n >= d.cols) return;
+  const int lane = threadIdx.x & 31, rg = threadIdx.x >> 5;
+  const int n = blockIdx.x * 64 + 2 * lane;
   const T* x = (const T*)d.X;
-  float s = 0.f;
-  for (int r = 0; r < d.rows; ++r) s += to_f<T>(x[(int64_t)r * d.ld + n]);
-  d.out[n] = s;
+  float s0 = 0.f, s1 = 0.f;
+  if (n < d.cols) {
+    const bool pair = n + 1 < d.cols;
+#pragma unroll 4
+    for (int r = rg; r < d.rows; r += 8) {
+      const T* p = x + (int64_t)r * d.ld + n;
+      s0 += to_f<T>(p[0]);
+      if (pair) s1 += to_f<T>(p[1]);
+    }
+  }
+  __shared__ float part[8][64];
+  part[rg][2 * lane] = s0;
+  part[rg][2 * lane + 1] = s1;
+  __syncthreads();
+  if (threadIdx.x < 64) {
+    const int c = blockIdx.x * 64 + threadIdx.x;
+    float t = 0.f;
+#pragma unroll
+    for (int g = 0; g < 8; ++g) t += part[g][threadIdx.x];
+    if (c < d.cols) d.out[c] = t;
+  }
 }
 
 template <typename T>
 void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st) {
   if (n_problems <= 0 || max_cols <= 0) return;
-  k_colsum<T><<<dim3((max_cols + 255) / 256, n_problems), 256, 0, st>>>(descs);
+  k_colsum<T><<<dim3((max_cols + 63) / 64, n_problems), 256, 0, st>>>(descs);
 }
 template void launch_colsum<float>(const ColSumDesc*, int, int, cudaStream_t);
 template void launch_colsum<bf16>(const ColSumDesc*, int, int, cudaStream_t);
@@ -364,9 +384,11 @@ __global__ void k_select(const float* __restrict__ fG, const float* __restrict__
     if (p.lr_mutation) lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std,
                                    p.lr_mut_thr);
     const int step1 = (pop ? step_d_old : step_g_old)[src] + 1;
-    const float4 cf = make_float4(lr, (float)(1.0 / (1.0 - pow((double)p.beta1, (double)step1))),
-                                  (float)(1.0 / (1.0 - pow((double)p.beta2, (double)step1))),
-                                  (float)step1);
+    // 1 - beta^t = -expm1(t * log1p(-(1 - beta))): 1 - beta is exact in fp32 for beta in
+    // [0.5, 1), and the expm1 form keeps full relative precision for beta^t near 1
+    const float bc1 = -expm1f((float)step1 * log1pf(-(1.f - p.beta1)));
+    const float bc2 = -expm1f((float)step1 * log1pf(-(1.f - p.beta2)));
+    const float4 cf = make_float4(lr, 1.f / bc1, 1.f / bc2, (float)step1);
     (pop ? coef_d : coef_g)[c] = cf;
     if (pop) {
       sel_d[c] = s;
@@ -396,17 +418,26 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
 template <typename T>
 __global__ void k_train_prep(const T* __restrict__ E, int64_t e_cell, const int* __restrict__ sel_g,
                              T* __restrict__ TX, int B, int x_dim) {
-  const int r = blockIdx.x, c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
+  if (r >= 2 * B) return;
   const int src_row = r < B ? r : B * (1 + sel_g[c]) + (r - B);
   const T* s = E + (int64_t)c * e_cell + (int64_t)src_row * x_dim;
   T* d = TX + ((int64_t)c * 2 * B + r) * x_dim;
-  for (int k = threadIdx.x; k < x_dim; k += blockDim.x) d[k] = s[k];
+  const int bytes = x_dim * (int)sizeof(T);
+  if ((bytes & 15) == 0 && (((uintptr_t)s | (uintptr_t)d) & 15) == 0) {
+    const uint4* s4 = reinterpret_cast<const uint4*>(s);
+    uint4* d4 = reinterpret_cast<uint4*>(d);
+    for (int k = lane; k < bytes / 16; k += 32) d4[k] = s4[k];
+  } else {
+    for (int k = lane; k < x_dim; k += 32) d[k] = s[k];
+  }
 }
 
 template <typename T>
 void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
                        int x_dim, cudaStream_t st) {
-  k_train_prep<T><<<dim3(2 * B, cells), 256, 0, st>>>(E, e_cell, sel_g, TX, B, x_dim);
+  k_train_prep<T><<<dim3((2 * B + 7) / 8, cells), 256, 0, st>>>(E, e_cell, sel_g, TX, B, x_dim);
 }
 template void launch_train_prep<float>(const float*, int64_t, const int*, float*, int, int, int,
                                        cudaStream_t);
@@ -421,13 +452,16 @@ template void launch_train_prep<bf16>(const bf16*, int64_t, const int*, bf16*, i
 // One block per cell, one thread per hidden unit.
 // ------------------------------------------------------------------------------------------
 template <typename T>
-__global__ void k_dlogit(const float* __restrict__ TL, const T* __restrict__ TG2,
-                         const T* __restrict__ wD, int64_t wD_stride, int64_t off_w3,
-                         const int* __restrict__ src_d, int B, int H, float slope,
-                         T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride,
-                         int64_t off_gw3, int64_t off_gb3) {
-  extern __shared__ float dl[];
+__global__ void __launch_bounds__(1024) k_dlogit(
+    const float* __restrict__ TL, const T* __restrict__ TG2, const T* __restrict__ wD,
+    int64_t wD_stride, int64_t off_w3, const int* __restrict__ src_d, int B, int H, float slope,
+    T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride, int64_t off_gw3,
+    int64_t off_gb3) {
+  extern __shared__ float dl[];            // [3B] deltas, then [4][H] partial sums
+  float* part = dl + 3 * B;
   const int c = blockIdx.x;
+  const int groups = blockDim.x / H;        // row groups (1..4)
+  const int k = threadIdx.x % H, rg = threadIdx.x / H;
   const float* l = TL + (int64_t)c * 2 * B;
   for (int r = threadIdx.x; r < 3 * B; r += blockDim.x) {
     const float x = r < 2 * B ? l[r] : l[r - B];
@@ -438,22 +472,28 @@ __global__ void k_dlogit(const float* __restrict__ TL, const T* __restrict__ TG2
   const T* w3 = wD + (int64_t)src_d[c] * wD_stride + off_w3;
   const T* g2 = TG2 + (int64_t)c * 2 * B * H;
   T* j2 = J2 + (int64_t)c * 3 * B * H;
-  float* g = gD + (int64_t)c * gD_stride;
-  for (int k = threadIdx.x; k < H; k += blockDim.x) {
+  float acc = 0.f;
+  if (rg < groups) {
     const float wk = to_f<T>(w3[k]);
-    float acc = 0.f;
-    for (int r = 0; r < 3 * B; ++r) {
+    for (int r = rg; r < 3 * B; r += groups) {
       const int rr = r < 2 * B ? r : r - B;
       const float gv = to_f<T>(g2[(int64_t)rr * H + k]);
       j2[(int64_t)r * H + k] = from_f<T>(dl[r] * wk * (gv > 0.f ? 1.f : slope));
       if (r < 2 * B) acc = fmaf(dl[r], gv, acc);
     }
-    g[off_gw3 + k] = acc;
+    part[rg * H + k] = acc;
+  }
+  __syncthreads();
+  float* g = gD + (int64_t)c * gD_stride;
+  if (threadIdx.x < H) {
+    float t = 0.f;
+    for (int q = 0; q < groups; ++q) t += part[q * H + threadIdx.x];
+    g[off_gw3 + threadIdx.x] = t;
   }
   if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int r = 0; r < 2 * B; ++r) s += dl[r];
-    g[off_gb3] = s;
+    float t = 0.f;
+    for (int r = 0; r < 2 * B; ++r) t += dl[r];
+    g[off_gb3] = t;
   }
 }
 
@@ -461,9 +501,13 @@ template <typename T>
 void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
                    const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
                    int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st) {
-  const int threads = H >= 256 ? 256 : ((H + 31) / 32) * 32;
-  k_dlogit<T><<<cells, threads, 3 * B * sizeof(float), st>>>(
-      TL, TG2, wD, wD_stride, off_w3, src_d, B, H, slope, J2, gD, gD_stride, off_gw3, off_gb3);
+  int groups = 1024 / H;
+  if (groups > 4) groups = 4;
+  if (groups < 1) groups = 1;
+  const int threads = groups * H;
+  const size_t smem = (3 * (size_t)B + 4 * (size_t)H) * sizeof(float);
+  k_dlogit<T><<<cells, threads, smem, st>>>(TL, TG2, wD, wD_stride, off_w3, src_d, B, H, slope, J2,
+                                            gD, gD_stride, off_gw3, off_gb3);
 }
 template void launch_dlogit<float>(const float*, const float*, const float*, int64_t, int64_t,
                                    const int*, int, int, int, float, float*, float*, int64_t,
