@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(THREADS, 2)
   const int m0 = (rem / p.ntiles) * BM;
   const int n0 = (rem % p.ntiles) * p.BN;
   int n = min(p.BN, p.N - n0);
-  n = (n + 15) & ~15;
+  n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -335,7 +335,6 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
   }
   const int C = s.cells, B = s.B, h = s.h, x = s.x, z = s.z;
   const uint64_t NI = s.n_indiv;
-  const int BNr = ((B + 15) / 16) * 16;  // rows of a batch as an MMA N
   const bf16* Gw = b.Gwb;
   const bf16* Dw = b.Dwb;
   auto base_params = [&](int M, int N, int K, int BN) {
@@ -394,25 +393,25 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg);
     finish(G);
   }
-  // 3. A3^T[i][r] = (sum_o W1d[o][i] D1[2B + r][o]) * (1 - F[r][i]^2): M = x, N = B, K = 256
+  // 3. A3 = (D1[2B + r] @ W1d) * (1 - F^2): M = B, N = x (tiles of 256), K = 256
   {
     Gemm& G = P->g[i++];
-    G.p = base_params(x, B, h, BNr);
-    G.p.a_mn = 1;
-    G.p.a_sel = b.src_d;
-    G.p.b_row0 = 2 * B;
+    G.p = base_params(B, x, h, 256);
+    G.p.a_row0 = 2 * B;
+    G.p.b_mn = 1;
+    G.p.b_sel = b.src_d;
     G.p.epi = tcb::EPI_DACT;
     G.p.act = ACT_TANH;
     G.p.C = b.A3;
     G.p.c_cell = (int64_t)B * x;
-    G.p.scm = 1;
-    G.p.scn = x;
+    G.p.scm = x;
+    G.p.scn = 1;
     G.p.aux = (const bf16*)b.TX + (int64_t)B * x;
     G.p.aux_cell = (int64_t)2 * B * x;
-    G.p.sxm = 1;
-    G.p.sxn = x;
-    ok = ok && map3(&G.a, Dw + b.doff[0], x, h, NI, b.PDs, 64, msg) &&
-         map3(&G.b, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, BNr, msg);
+    G.p.sxm = x;
+    G.p.sxn = 1;
+    ok = ok && map3(&G.a, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 128, msg) &&
+         map3(&G.b, Dw + b.doff[0], x, h, NI, b.PDs, 64, msg);
     finish(G);
   }
   // 4. dW1d^T[i][o] = sum_{r < 2B} TX[r][i] D1[r][o]: M = x, N = 256, K = 2B (TX ends at 2B)
