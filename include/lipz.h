@@ -218,6 +218,29 @@ enum {
 LIPZ_API int lipz_profile_enable(lipz_grid* g, int enable);
 LIPZ_API int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t* launches, int n);
 
+/*
+ * Fitness of every cell from logits already in device memory, allocating nothing.
+ * Not part of the method: the paper has no counterpart. It is for callers that cannot call
+ * cudaMalloc when they need the fitness: code running while a CUDA graph is being captured
+ * (allocation calls are not allowed there), a serving loop whose device memory is fully
+ * reserved by another allocator (a new allocation would fail), or a latency-critical path
+ * that cannot afford the implicit synchronisation of cudaMalloc / cudaFree. The per-pair
+ * losses that the computation needs go to one file-scope device array of about 800 KB, which
+ * every GPU that loads this library holds until the process exits.
+ *   logits: device, [cells][5 (j)][6 * batch] fp32, laid out as lipz_get_logits returns it;
+ *   fit_g, fit_d: device outputs [cells][5] fp32 (as lipz_eval_neighborhoods computes them);
+ *   stream: the cudaStream_t to run on (0 = legacy default). The call is asynchronous.
+ * Limits: 1 <= cells <= LIPZ_NOALLOC_MAX_CELLS and batch >= 1, else LIPZ_ERR_INVALID with
+ * nothing launched; a null pointer also gives LIPZ_ERR_INVALID. LIPZ_ERR_CUDA if a CUDA call
+ * fails. The first call on a device looks up the array's device address (once per device,
+ * with that device current): make that first call before any stream capture. All calls share
+ * the array, and each call overwrites what it uses, so two calls whose work overlaps on the
+ * GPU (different streams, no ordering) race. Non-finite losses show up as NaN/Inf fitness.
+ */
+#define LIPZ_NOALLOC_MAX_CELLS 4096
+LIPZ_API int lipz_fitness_from_logits_noalloc(const float* logits, int32_t cells, int32_t batch,
+                                             float* fit_g, float* fit_d, void* stream);
+
 /* Message of the grid's last failure ("" if none); for a null grid, of the last failed
  * lipz_grid_create on this thread. The pointer stays valid until the next call on the grid. */
 LIPZ_API const char* lipz_last_error(const lipz_grid* g);

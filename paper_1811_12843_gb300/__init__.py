@@ -19,7 +19,7 @@ __all__ = [
     "lipz_train_step", "lipz_iterate", "lipz_iterate_batch", "lipz_state_bytes",
     "lipz_export_state", "lipz_import_state", "lipz_get_iteration", "lipz_get_batch",
     "lipz_get_logits", "lipz_get_gradients", "lipz_profile_enable", "lipz_profile_read",
-    "lipz_last_error", "lipz_status_string", "PHASES",
+    "lipz_fitness_from_logits_noalloc", "lipz_last_error", "lipz_status_string", "PHASES",
     "EXPORTED", "Grid", "param_counts",
 ]
 
@@ -78,6 +78,7 @@ _SIGS = {
     "lipz_get_gradients": (_I, [_P, _P, _P]),
     "lipz_profile_enable": (_I, [_P, _I]),
     "lipz_profile_read": (_I, [_P, _P, _P, _P, _I]),
+    "lipz_fitness_from_logits_noalloc": (_I, [_P, ctypes.c_int32, ctypes.c_int32, _P, _P, _P]),
     "lipz_last_error": (ctypes.c_char_p, [_P]),
     "lipz_status_string": (ctypes.c_char_p, [_I]),
 }
@@ -226,6 +227,17 @@ def lipz_profile_read(g):
     la = np.zeros(n, np.int64)
     _check(g, load().lipz_profile_read(g, _ptr(ms), _ptr(cnt), _ptr(la), n))
     return {p: (float(ms[i]), int(cnt[i]), int(la[i])) for i, p in enumerate(PHASES)}
+
+
+def lipz_fitness_from_logits_noalloc(logits, cells, batch, fit_g, fit_d, stream=0):
+    """Fitness from device logits with no device allocation (all buffers are device tensors
+    the caller owns). Raises LipzError with the status code on failure."""
+    s = stream if isinstance(stream, int) else getattr(stream, "cuda_stream", stream)
+    rc = load().lipz_fitness_from_logits_noalloc(_ptr(logits), int(cells), int(batch),
+                                                 _ptr(fit_g), _ptr(fit_d), _P(int(s or 0)))
+    if rc != LIPZ_OK:
+        raise LipzError(rc, "lipz_fitness_from_logits_noalloc: " + lipz_status_string(rc))
+    return rc
 
 
 def lipz_last_error(g) -> str:
