@@ -449,19 +449,20 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Gw + b.goff[4], h, x, NI, b.PGs, 64, msg);
     finish(G);
   }
-  // 6. dW3g[o][i] = sum_r A3[r][o] TH2[r][i]: M = x (o), N = 256 (i), K = B
+  // 6. dW3g^T[i][o] = sum_r TH2[r][i] A3[r][o]: M = 256 (i), N = x (o), K = B; the
+  //    transposed output makes a warp's stores contiguous
   {
     Gemm& G = P->g[i++];
-    G.p = base_params(x, h, B, 256);
+    G.p = base_params(h, x, B, 256);
     G.p.a_mn = 1;
     G.p.b_mn = 1;
     G.p.epi = tcb::EPI_F32;
     G.p.C = b.gG + b.goff[4];
     G.p.c_cell = b.PGs;
-    G.p.scm = h;
-    G.p.scn = 1;
-    ok = ok && map3(&G.a, b.A3, x, B, C, (uint64_t)B * x, 64, msg) &&
-         map3(&G.b, b.TH2, h, B, C, (uint64_t)B * h, 64, msg);
+    G.p.scm = 1;
+    G.p.scn = h;
+    ok = ok && map3(&G.a, b.TH2, h, B, C, (uint64_t)B * h, 64, msg) &&
+         map3(&G.b, b.A3, x, B, C, (uint64_t)B * x, 64, msg);
     finish(G);
   }
   // 7. A1 = (A2 @ W2g) * relu'(TH1): M = B, N = 256, K = 256
