@@ -39,7 +39,7 @@ constexpr int B_BYTES = HID * BK * 2;        // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int H_CHUNK = BM * BK * 2;         // one 64-column chunk of the on-chip activation
 constexpr int H_BYTES = BM * HID * 2;        // 64 KB
-constexpr int N3 = 112;                      // generator output columns per MMA block
+constexpr int N3 = 256;                      // generator output columns per MMA block
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr int MISC_BYTES = 2048;
@@ -95,9 +95,9 @@ __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   } else {
     const int nb = j - 2;
     const int n = min(N3, p.x - nb * N3);
-    // output blocks start in region 1 so that, with an odd block count, a tile ends in
-    // region 1 and the next tile's first layer (region 0) need not wait for its last epilogue
-    J = Job{1, HID / BK, n, (nb + 1) & 1, 2, nb * N3, N3, EPI_TO_E};
+    // the last output block always lands in region 1, so the next tile's first layer
+    // (region 0) need not wait for the tile's last epilogue
+    J = Job{1, HID / BK, (n + 15) & ~15, (nb + p.n3) & 1, 2, nb * N3, N3, EPI_TO_E};
   }
   return J;
 }
@@ -420,7 +420,8 @@ __global__ void __launch_bounds__(THREADS, 1)
           // generator output block: bias + tanh, bf16, into the fake rows of E[c]
           const float* bias = wm + p.off_b3;
           const int ng = J.n / 16;
-          const int g0 = hf ? 4 : 0, g1 = hf ? ng : min(4, ng);
+          const int split = (ng + 1) / 2;
+          const int g0 = hf ? split : 0, g1 = hf ? ng : split;
           bf16* dst = p.E + (int64_t)c * p.e_cell + (int64_t)((1 + slot) * p.B + rr) * p.x;
 #pragma unroll 1
           for (int gi = g0; gi < g1; ++gi) {
@@ -445,7 +446,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int e = 0; e < 16; e += 2)
               pk[e >> 1] = pack_bf16(tanh_approx(__uint_as_float(r[e]) + bv[e]),
                                      tanh_approx(__uint_as_float(r[e + 1]) + bv[e + 1]));
-            if (rr < p.B) {
+            if (rr < p.B && col0 < p.x) {
               uint4* o = reinterpret_cast<uint4*>(dst + col0);
               o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
               o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
