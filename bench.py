@@ -45,6 +45,14 @@ PG = HIDDEN * Z_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + X_DIM * HIDDEN + X_DIM
 PD = HIDDEN * X_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + HIDDEN + 1
 # Adam + replacement per parameter: read w, m, v, g (16 B), write w, m, v (12 B) + bf16 copy (2 B)
 ADAM_BYTES = CELLS * (PG + PD) * 30
+# Training: forward of the selected pair (G layers 1-2 on B rows, D on 2B rows) and backward.
+TRAIN_FWD_FLOP = 2 * CELLS * BATCH * (Z_DIM * HIDDEN + HIDDEN * HIDDEN) + 2 * CELLS * 2 * BATCH * D_MAC_ROW
+TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
+
+# DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels, from
+# the ncu launch list in profiles/launches_12x12_bf16_iteration.md (same kernels as this build).
+PHASE_TRAFFIC = {"batch": 41.4e6, "g_fwd": 159.5e6, "d_fwd": 226.9e6, "fitness": 1.7e6,
+                 "select": 0.0, "train_fwd": 160.7e6, "train_bwd": 557.9e6, "adam": 2105.9e6}
 
 
 def _peaks():
@@ -199,6 +207,7 @@ def run_ours(args):
         (phase_ms["batch"] + phase_ms["g_fwd"] + phase_ms["d_fwd"] + phase_ms["fitness"]),
         "phase_ms": phase_ms,
         "roofline": roof,
+        "phase_rooflines": None if args.no_phases else _phase_roofs(phase_ms),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
@@ -232,36 +241,39 @@ def _e2e(args, L, g, torch, dist, world):
     return PAIRS * world * args.steps / e2e_s
 
 
+def _phase_roofs(phase_ms):
+    """Roofline of every heavy phase: algorithmic work / device time against the measured peak."""
+    hbm, tf_burst, tf_sus, peak_kind = _peaks()
+    work = {"g_fwd": ("tensor", EVAL_G_FLOP, "generator evaluation forward (all 720 slots, 3 fused layers)"),
+            "d_fwd": ("tensor", EVAL_D_FLOP,
+                      "discriminator evaluation forward (all 720 slots, 3 fused layers + logit)"),
+            "train_fwd": ("tensor", TRAIN_FWD_FLOP, "forward of every cell's selected pair"),
+            "train_bwd": ("tensor", TRAIN_BWD_FLOP, "backward of every cell's selected pair"),
+            "adam": ("hbm", ADAM_BYTES, "Adam + replacement (both populations)")}
+    out = {}
+    for ph, (bound, units, what) in work.items():
+        t = phase_ms.get(ph)
+        if not t or t != t:
+            continue
+        if bound == "hbm":
+            ach, peak, unit = units / (t * 1e-3) / 1e9, hbm, "GB/s"
+            src = peak_kind + " HBM copy"
+        else:
+            ach, peak, unit = units / (t * 1e-3) / 1e12, tf_sus, "TFLOP/s"
+            src = peak_kind + " sustained bf16"
+        out[ph] = {"bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
+                   "traffic": PHASE_TRAFFIC.get(ph), "kernel": what, "peak_source": src,
+                   ("algorithmic_bytes" if bound == "hbm" else "algorithmic_flop"): units}
+    return out
+
+
 def _roofline(phase_ms):
     """Roofline of the phase with the largest device time."""
-    hbm, tf_burst, tf_sus, peak_kind = _peaks()
-    dom = max(("g_fwd", "d_fwd", "train_fwd", "train_bwd", "adam"), key=lambda k: phase_ms[k])
-    if dom == "d_fwd":
-        ach = EVAL_D_FLOP / (phase_ms["d_fwd"] * 1e-3) / 1e12
-        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
-                "kernel": "discriminator evaluation forward (all 720 slots, fused 3 layers + logit)",
-                "algorithmic_flop_per_launch": EVAL_D_FLOP}
-    elif dom == "g_fwd":
-        ach = EVAL_G_FLOP / (phase_ms["g_fwd"] * 1e-3) / 1e12
-        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
-                "kernel": "generator evaluation forward (all 720 slots)",
-                "algorithmic_flop_per_launch": EVAL_G_FLOP}
-    elif dom == "adam":
-        ach = ADAM_BYTES / (phase_ms["adam"] * 1e-3) / 1e9
-        roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
-                "kernel": "fused Adam + replacement", "algorithmic_bytes_per_launch": ADAM_BYTES}
-    else:
-        flop = 2 * CELLS * BATCH * (G_MAC_ROW - HIDDEN * X_DIM) + 2 * CELLS * 2 * BATCH * D_MAC_ROW \
-            if dom == "train_fwd" else 2 * CELLS * BATCH * 1479936
-        ach = flop / (phase_ms[dom] * 1e-3) / 1e12
-        roof = {"bound": "tensor", "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
-                "kernel": "selected-pair " + dom.replace("_", " "),
-                "algorithmic_flop_per_launch": flop}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["peak_source"] = peak_kind + (" sustained bf16" if roof["unit"] == "TFLOP/s" else " HBM copy")
-    roof["traffic"] = None
-    roof["phase"] = dom
-    return roof
+    roofs = _phase_roofs(phase_ms)
+    dom = max(roofs, key=lambda k: phase_ms[k])
+    r = dict(roofs[dom])
+    r["phase"] = dom
+    return r
 
 
 def _oracle_sample(seconds, max_cells=None):
