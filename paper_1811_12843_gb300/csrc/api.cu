@@ -76,6 +76,8 @@ struct lipz_grid {
   TcPlan* tc[2]{};
   TcbPlan* tcb[2]{};
   bool use_tcb = false;
+  cudaStream_t side = nullptr;  // second stream of the training step (owned)
+  cudaEvent_t ev_fork = nullptr, ev_d1 = nullptr, ev_join = nullptr;
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
   bool prof = false;
@@ -432,10 +434,12 @@ void gemv(lipz_grid* g, const GemvDesc* d, int n, int rows) {
   else launch_gemv<float>(d, n, rows, g->st);
 }
 
-void colsum(lipz_grid* g, const ColSumDesc* d, int n, int cols) {
-  if (g->bf) launch_colsum<bf16>(d, n, cols, g->st);
-  else launch_colsum<float>(d, n, cols, g->st);
+void colsum_on(lipz_grid* g, const ColSumDesc* d, int n, int cols, cudaStream_t st) {
+  if (g->bf) launch_colsum<bf16>(d, n, cols, st);
+  else launch_colsum<float>(d, n, cols, st);
 }
+
+void colsum(lipz_grid* g, const ColSumDesc* d, int n, int cols) { colsum_on(g, d, n, cols, g->st); }
 
 int check_arch(const lipz_arch* a) {
   if (!a) return fail(nullptr, LIPZ_ERR_INVALID, "arch is null");
@@ -481,6 +485,10 @@ int create_impl(lipz_grid* g) {
   const size_t es = g->esz;
   int rc;
   CK(g, cudaGetDevice(&g->device));
+  CK(g, cudaStreamCreateWithFlags(&g->side, cudaStreamNonBlocking));
+  CK(g, cudaEventCreateWithFlags(&g->ev_fork, cudaEventDisableTiming));
+  CK(g, cudaEventCreateWithFlags(&g->ev_d1, cudaEventDisableTiming));
+  CK(g, cudaEventCreateWithFlags(&g->ev_join, cudaEventDisableTiming));
   make_layouts(g);
   g->e_cell = (int64_t)6 * B * x;
   for (int p = 0; p < 2; ++p) {
@@ -691,6 +699,44 @@ int train_impl(lipz_grid* g) {
     launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
                          g->ld.off[5], g->st);
+  if (g->use_tcb && !g->prof) {
+    // Two streams. The delta chain through D into G (D1 -> A3 -> A2 -> A1) and the generator's
+    // weight gradients stay on the grid's stream; the discriminator's weight gradients and its
+    // Adam step (HBM-bound) run on the side stream as soon as their inputs exist, overlapping
+    // the latency-bound chain. The side stream rejoins before the generator's Adam ends the
+    // step. (With tracing on, the serial order below is used so phases do not overlap.)
+    std::string msg;
+    TcbPlan* P = g->tcb[p];
+    cudaStream_t ms = g->st, ss = g->side;
+    CK(g, cudaEventRecord(g->ev_fork, ms));
+    CK(g, cudaStreamWaitEvent(ss, g->ev_fork, 0));
+    if (tcb_run(P, 1, 1, ss, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW2(D)
+    colsum_on(g, D.cb2d, C, h, ss);
+    if (tcb_run(P, 0, 1, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // D1
+    CK(g, cudaEventRecord(g->ev_d1, ms));
+    CK(g, cudaStreamWaitEvent(ss, g->ev_d1, 0));
+    if (tcb_run(P, 3, 1, ss, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW1(D)
+    colsum_on(g, D.cb1d, C, h, ss);
+    launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
+                g->a.beta2, g->a.eps, ss);
+    CK(g, cudaEventRecord(g->ev_join, ss));
+    if (tcb_run(P, 2, 1, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // A3
+    colsum_on(g, D.cb3g, C, x, ms);
+    if (tcb_run(P, 4, 3, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // A2 dW3 A1
+    colsum_on(g, D.cb2g, C, h, ms);
+    if (tcb_run(P, 7, 2, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW2 dW1
+    colsum_on(g, D.cb1g, C, h, ms);
+    launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
+                g->a.beta2, g->a.eps, ms);
+    CK(g, cudaStreamWaitEvent(ms, g->ev_join, 0));
+    CKL(g);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
+    phase_end(g, LIPZ_PHASE_ADAM, 2);
+    g->cur = 1 - p;
+    g->t += 1;
+    g->phase = PH_IDLE;
+    return LIPZ_OK;
+  }
   if (g->use_tcb) {
     std::string msg;
     TcbPlan* P = g->tcb[p];
@@ -855,6 +901,12 @@ int lipz_grid_destroy(lipz_grid* g) {
   }
   for (auto e : g->ev_free) cudaEventDestroy(e);
   for (auto e : g->open_ev)
+    if (e) cudaEventDestroy(e);
+  if (g->side) {
+    cudaStreamSynchronize(g->side);
+    cudaStreamDestroy(g->side);
+  }
+  for (cudaEvent_t e : {g->ev_fork, g->ev_d1, g->ev_join})
     if (e) cudaEventDestroy(e);
   for (void* p : g->allocs) cudaFree(p);
   delete g;
