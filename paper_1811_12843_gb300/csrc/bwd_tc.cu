@@ -23,18 +23,19 @@ using namespace lipz::tc;
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int STAGES = 2;
+constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;        // 16 KB
 constexpr int B_BYTES = 256 * BK * 2;       // 32 KB (BN <= 256)
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int MN_BOX_BYTES = 64 * BK * 2;   // one {64 MN, 64 K} box
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;  // one CTA per SM
 
 enum { EPI_F32 = 0, EPI_DACT = 1 };
 
 struct GParams {
+  int cells;
   int M, N, K, BN;
   int mtiles, ntiles, kchunks;
   int a_mn, b_mn;       // operand layouts (1 = MN-major)
@@ -60,7 +61,11 @@ __device__ __forceinline__ float dact(int act, float y, float slope) {
   }
 }
 
-__global__ void __launch_bounds__(THREADS, 2)
+// Persistent: CTAs walk the product's tiles (cell, m-tile, n-tile); the accumulator of
+// consecutive tiles alternates between two 256-column TMEM regions, so the epilogue of one
+// tile overlaps the loads and MMAs of the next.
+template <int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
               const GParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -68,18 +73,13 @@ __global__ void __launch_bounds__(THREADS, 2)
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
   uint8_t* misc = gbase + STAGES * STAGE_BYTES;
-  const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES, bAcc = bEmpty + 8 * STAGES;
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 128);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 132);
+  const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES;
+  const uint32_t bAcc = bEmpty + 8 * STAGES, bReg = bAcc + 16, bFinal = bReg + 16;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
 
   const int per_cell = p.mtiles * p.ntiles;
-  const int cell = blockIdx.x / per_cell;
-  const int rem = blockIdx.x % per_cell;
-  const int m0 = (rem / p.ntiles) * BM;
-  const int n0 = (rem % p.ntiles) * p.BN;
-  int n = min(p.BN, p.N - n0);
-  n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
-
+  const int n_tiles = p.cells * per_cell;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -87,12 +87,16 @@ __global__ void __launch_bounds__(THREADS, 2)
       mbar_init(bEmpty + 8 * s, 1);
     }
     mbar_init(bAcc, 1);
+    mbar_init(bAcc + 8, 1);
+    mbar_init(bReg, 32 * NUM_EPI_WARPS);
+    mbar_init(bReg + 8, 32 * NUM_EPI_WARPS);
+    mbar_init(bFinal, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
         smem_u32((const void*)tmem_slot)));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
@@ -104,36 +108,40 @@ __global__ void __launch_bounds__(THREADS, 2)
 
   if (warp == 0) {
     if (lane == 0) {
-      const int za = p.a_sel ? __ldg(&p.a_sel[cell]) : cell;
-      const int zb = p.b_sel ? __ldg(&p.b_sel[cell]) : cell;
-      int issued[STAGES] = {0, 0};
+      int issued[STAGES] = {0, 0, 0, 0};
       bool ok = true;
       int stage = 0;
       uint32_t phase = 0;
-      for (int kc = 0; kc < p.kchunks; ++kc) {
-        if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 11)) {
-          ok = false;
-          break;
-        }
-        const uint32_t full = bFull + 8 * stage;
-        mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
-        const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
-        if (p.a_mn) {
-          tma_load_3d(sA, &mA, full, m0, kc * BK, za);
-          tma_load_3d(sA + MN_BOX_BYTES, &mA, full, m0 + 64, kc * BK, za);
-        } else {
-          tma_load_3d(sA, &mA, full, kc * BK, p.a_row0 + m0, za);
-        }
-        if (p.b_mn) {
-          for (int i = 0; i < p.BN / 64; ++i)
-            tma_load_3d(sB + i * MN_BOX_BYTES, &mB, full, n0 + 64 * i, kc * BK, zb);
-        } else {
-          tma_load_3d(sB, &mB, full, kc * BK, p.b_row0 + n0, zb);
-        }
-        issued[stage]++;
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1u;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        const int cell = tile / per_cell, rem = tile % per_cell;
+        const int m0 = (rem / p.ntiles) * BM, n0 = (rem % p.ntiles) * p.BN;
+        const int za = p.a_sel ? __ldg(&p.a_sel[cell]) : cell;
+        const int zb = p.b_sel ? __ldg(&p.b_sel[cell]) : cell;
+        for (int kc = 0; kc < p.kchunks; ++kc) {
+          if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 11)) {
+            ok = false;
+            break;
+          }
+          const uint32_t full = bFull + 8 * stage;
+          mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
+          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+          if (p.a_mn) {
+            tma_load_3d(sA, &mA, full, m0, kc * BK, za);
+            tma_load_3d(sA + MN_BOX_BYTES, &mA, full, m0 + 64, kc * BK, za);
+          } else {
+            tma_load_3d(sA, &mA, full, kc * BK, p.a_row0 + m0, za);
+          }
+          if (p.b_mn) {
+            for (int i = 0; i < p.BN / 64; ++i)
+              tma_load_3d(sB + i * MN_BOX_BYTES, &mB, full, n0 + 64 * i, kc * BK, zb);
+          } else {
+            tma_load_3d(sB, &mB, full, kc * BK, p.b_row0 + n0, zb);
+          }
+          issued[stage]++;
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
         }
       }
       if (!ok) {
@@ -146,40 +154,67 @@ __global__ void __launch_bounds__(THREADS, 2)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_major(BM, n, p.a_mn, p.b_mn);
       int stage = 0;
       uint32_t phase = 0;
-      for (int kc = 0; kc < p.kchunks; ++kc) {
-        if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 12)) break;
+      bool ok = true;
+      int lt = 0;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++lt) {
+        const int rem = tile % per_cell;
+        const int n0 = (rem % p.ntiles) * p.BN;
+        int n = min(p.BN, p.N - n0);
+        n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
+        const int R = lt & 1, use = lt >> 1;
+        if (use > 0 &&
+            !mbar_wait(bReg + 8 * R, (uint32_t)((use - 1) & 1), abort_flag, p.err, 15)) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+        const uint32_t d = tmem + (uint32_t)(R * 256);
+        const uint32_t idesc = idesc_bf16_major(BM, n, p.a_mn, p.b_mn);
+        for (int kc = 0; kc < p.kchunks; ++kc) {
+          if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 12)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk) {
-          const uint64_t ad = p.a_mn ? sw128_mn_desc(sA + kk * 2048, MN_BOX_BYTES)
-                                     : sw128_desc(sA + kk * 32);
-          const uint64_t bd = p.b_mn ? sw128_mn_desc(sB + kk * 2048, MN_BOX_BYTES)
-                                     : sw128_desc(sB + kk * 32);
-          tc_mma(tmem, ad, bd, idesc, (kc | kk) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t ad = p.a_mn ? sw128_mn_desc(sA + kk * 2048, MN_BOX_BYTES)
+                                       : sw128_desc(sA + kk * 32);
+            const uint64_t bd = p.b_mn ? sw128_mn_desc(sB + kk * 2048, MN_BOX_BYTES)
+                                       : sw128_desc(sB + kk * 32);
+            tc_mma(d, ad, bd, idesc, (kc | kk) != 0 ? 1u : 0u);
+          }
+          tc_commit(bEmpty + 8 * stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
         }
-        tc_commit(bEmpty + 8 * stage);
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1u;
-        }
+        if (!ok) break;
+        tc_commit(bAcc + 8 * R);
       }
-      tc_commit(bAcc);
-      // the MMAs must be complete before the tensor memory is released, even if the
-      // epilogue gave up waiting
+      // every MMA issued here completes before the tensor memory is released
+      tc_commit(bFinal);
       volatile int never = 0;
-      mbar_wait(bAcc, 0u, &never, p.err, 14);
+      mbar_wait(bFinal, 0u, &never, p.err, 14);
     }
   } else {
     const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
     const int row = q * 32 + lane;
-    const int m = m0 + row;
-    if (mbar_wait(bAcc, 0u, abort_flag, p.err, 13)) {
+    int lt = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++lt) {
+      const int cell = tile / per_cell, rem = tile % per_cell;
+      const int m0 = (rem / p.ntiles) * BM, n0 = (rem % p.ntiles) * p.BN;
+      int n = min(p.BN, p.N - n0);
+      n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
+      const int R = lt & 1, use = lt >> 1;
+      if (!mbar_wait(bAcc + 8 * R, (uint32_t)(use & 1), abort_flag, p.err, 13)) break;
       tc_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+      const int m = m0 + row;
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
       const int ng = n / 16;
       const int half = (ng + 1) / 2;
       const int g0 = hf ? half : 0, g1 = hf ? ng : half;
@@ -191,7 +226,7 @@ __global__ void __launch_bounds__(THREADS, 2)
         tmem_wait_ld();
         const int col0 = n0 + gi * 16;
         if (!row_ok) continue;
-        if (p.epi == EPI_F32) {
+        if (EPI == EPI_F32) {
           float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
           if (p.scn == 1 && col0 + 16 <= p.N) {
             float4* o = reinterpret_cast<float4*>(C + col0);
@@ -209,7 +244,6 @@ __global__ void __launch_bounds__(THREADS, 2)
           const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
           float v[16];
           if (p.sxn == 1 && col0 + 16 <= p.N) {
-            // the row's 16 aux values are contiguous: two 16-byte loads
             const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
             const uint4 q0 = __ldg(x4), q1 = __ldg(x4 + 1);
             const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
@@ -244,6 +278,8 @@ __global__ void __launch_bounds__(THREADS, 2)
           }
         }
       }
+      tc_fence_before();
+      mbar_arrive(bReg + 8 * R);
     }
   }
   __syncwarp();
@@ -251,7 +287,7 @@ __global__ void __launch_bounds__(THREADS, 2)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
   }
 }
 
@@ -319,8 +355,13 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     return nullptr;
   }
   if (!encoder(msg)) return nullptr;
-  if (cudaFuncSetAttribute(tcb::k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           tcb::SMEM_BYTES) != cudaSuccess) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (cudaFuncSetAttribute(tcb::k_gemm_tc<tcb::EPI_F32>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, tcb::SMEM_BYTES) != cudaSuccess ||
+      cudaFuncSetAttribute(tcb::k_gemm_tc<tcb::EPI_DACT>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, tcb::SMEM_BYTES) != cudaSuccess) {
     cudaGetLastError();
     if (msg) *msg = "cannot reserve shared memory for the tensor-core backward";
     return nullptr;
@@ -350,11 +391,15 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     q.slope = s.slope;
     q.aux_wrap_at = 1 << 30;
     q.err = P->err;
+    q.cells = C;
     return q;
   };
   bool ok = true;
   int i = 0;
-  auto finish = [&](Gemm& G) { G.grid = C * G.p.mtiles * G.p.ntiles; };
+  auto finish = [&](Gemm& G) {
+    const int tiles = C * G.p.mtiles * G.p.ntiles;
+    G.grid = tiles < sms ? tiles : sms;
+  };
 
   // 1. D1 = (J2 @ W2d) * lrelu'(TG1 rows r or r - B): M = 3B rows, N = 256, K = 256
   {
@@ -527,7 +572,10 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
 int tcb_run(TcbPlan* P, int first, int count, cudaStream_t st, std::string* msg) {
   for (int i = first; i < first + count && i < P->n; ++i) {
     Gemm& G = P->g[i];
-    tcb::k_gemm_tc<<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
+    if (G.p.epi == tcb::EPI_DACT)
+      tcb::k_gemm_tc<tcb::EPI_DACT><<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
+    else
+      tcb::k_gemm_tc<tcb::EPI_F32><<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
       if (msg) *msg = std::string("tensor-core backward launch: ") + cudaGetErrorString(e);
