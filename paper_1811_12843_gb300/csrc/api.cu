@@ -78,6 +78,7 @@ struct lipz_grid {
   bool use_tcb = false;
   cudaStream_t side = nullptr;  // second stream of the training step (owned)
   cudaEvent_t ev_fork = nullptr, ev_d1 = nullptr, ev_join = nullptr;
+  bool side_pending = false;    // the side stream's last work is not yet joined into st
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
   bool prof = false;
@@ -168,6 +169,14 @@ void phase_end(lipz_grid* g, int ph, int n_launches) {
   cudaEventRecord(e, g->st);
   g->marks.push_back({ph, g->open_ev[ph], e});
   g->open_ev[ph] = nullptr;
+}
+
+// Makes the grid's stream wait for the side stream's outstanding work (the discriminator's
+// Adam step of the last training step), if any.
+cudaError_t join_side(lipz_grid* g) {
+  if (!g->side_pending) return cudaSuccess;
+  g->side_pending = false;
+  return cudaStreamWaitEvent(g->st, g->ev_join, 0);
 }
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -612,6 +621,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);
+    CK(g, join_side(g));
     phase_begin(g, LIPZ_PHASE_D_FWD);
     if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_D_FWD, 1);
@@ -622,6 +632,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
     phase_end(g, LIPZ_PHASE_G_FWD, 3);
+    CK(g, join_side(g));
     phase_begin(g, LIPZ_PHASE_D_FWD);
     gemm(g, D.d1, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemm(g, D.d2, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
@@ -638,6 +649,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
 }
 
 int select_impl(lipz_grid* g) {
+  CK(g, join_side(g));
   if (g->phase != PH_EVALUATED)
     return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
   SelectParams sp;
@@ -663,6 +675,7 @@ int select_impl(lipz_grid* g) {
 }
 
 int train_impl(lipz_grid* g) {
+  CK(g, join_side(g));
   if (g->phase != PH_SELECTED)
     return fail(g, LIPZ_ERR_STATE, "lipz_train_step must follow lipz_select_replace");
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
@@ -703,8 +716,9 @@ int train_impl(lipz_grid* g) {
     // Two streams. The delta chain through D into G (D1 -> A3 -> A2 -> A1) and the generator's
     // weight gradients stay on the grid's stream; the discriminator's weight gradients and its
     // Adam step (HBM-bound) run on the side stream as soon as their inputs exist, overlapping
-    // the latency-bound chain. The side stream rejoins before the generator's Adam ends the
-    // step. (With tracing on, the serial order below is used so phases do not overlap.)
+    // the latency-bound chain and the next evaluation's generator kernel; the grid's stream
+    // waits for it before anything reads the discriminator population again. (With tracing
+    // on, the serial order below is used so phases do not overlap.)
     std::string msg;
     TcbPlan* P = g->tcb[p];
     cudaStream_t ms = g->st, ss = g->side;
@@ -728,7 +742,9 @@ int train_impl(lipz_grid* g) {
     colsum_on(g, D.cb1g, C, h, ms);
     launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
                 g->a.beta2, g->a.eps, ms);
-    CK(g, cudaStreamWaitEvent(ms, g->ev_join, 0));
+    // The discriminator's Adam may still run: the next evaluation's generator kernel does not
+    // need it, so the join is deferred to just before the discriminator kernel (join_side).
+    g->side_pending = true;
     CKL(g);
     phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
     phase_end(g, LIPZ_PHASE_ADAM, 2);
@@ -915,18 +931,21 @@ int lipz_grid_destroy(lipz_grid* g) {
 
 int lipz_set_stream(lipz_grid* g, void* stream) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   g->st = (cudaStream_t)stream;
   return LIPZ_OK;
 }
 
 int lipz_synchronize(lipz_grid* g) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   CK(g, cudaStreamSynchronize(g->st));
   return check_flag(g);
 }
 
 int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t dim) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   if (!host_pool || n_rows < 1 || n_rows > 0xFFFFFFFFll || dim != g->a.x_dim)
     return fail(g, LIPZ_ERR_INVALID, "set_data needs a pool of 1..2^32-1 rows of x_dim=%d",
                 g->a.x_dim);
@@ -1015,6 +1034,7 @@ int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {
 
 int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   size_t need = 0;
   lipz_state_bytes(g, &need);
   if (!host || bytes != need)
@@ -1053,6 +1073,7 @@ int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
 
 int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   size_t need = 0;
   lipz_state_bytes(g, &need);
   if (!host || bytes != need) return fail(g, LIPZ_ERR_INVALID, "import_state needs %zu bytes", need);
@@ -1109,6 +1130,7 @@ int lipz_get_iteration(const lipz_grid* g, int64_t* t) {
 
 int lipz_get_batch(lipz_grid* g, float* x, float* z) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   if (g->phase == PH_IDLE) return fail(g, LIPZ_ERR_STATE, "no evaluation since the last train step");
   const int64_t B = g->a.batch;
   int rc;
@@ -1128,6 +1150,7 @@ int lipz_get_logits(lipz_grid* g, float* logits) {
 
 int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   if (!g->a.keep_grads) return fail(g, LIPZ_ERR_STATE, "grid was created without keep_grads");
   CK(g, cudaStreamSynchronize(g->st));
   const size_t C = g->cells;
@@ -1146,6 +1169,7 @@ int lipz_profile_enable(lipz_grid* g, int enable) {
 
 int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t* launches, int n) {
   if (!g) return LIPZ_ERR_INVALID;
+  CK(g, join_side(g));
   if (n < 0 || n > LIPZ_N_PHASES) return fail(g, LIPZ_ERR_INVALID, "n must be in 0..%d", LIPZ_N_PHASES);
   CK(g, cudaStreamSynchronize(g->st));
   double acc[LIPZ_N_PHASES] = {0};
