@@ -712,62 +712,37 @@ int train_impl(lipz_grid* g) {
     launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
                          g->ld.off[5], g->st);
-  if (g->use_tcb && !g->prof) {
-    // Two streams. The delta chain through D into G (D1 -> A3 -> A2 -> A1) and the generator's
-    // weight gradients stay on the grid's stream; the discriminator's weight gradients and its
-    // Adam step (HBM-bound) run on the side stream as soon as their inputs exist, overlapping
-    // the latency-bound chain and the next evaluation's generator kernel; the grid's stream
-    // waits for it before anything reads the discriminator population again. (With tracing
-    // on, the serial order below is used so phases do not overlap.)
-    std::string msg;
-    TcbPlan* P = g->tcb[p];
-    cudaStream_t ms = g->st, ss = g->side;
-    CK(g, cudaEventRecord(g->ev_fork, ms));
-    CK(g, cudaStreamWaitEvent(ss, g->ev_fork, 0));
-    if (tcb_run(P, 1, 1, ss, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW2(D)
-    colsum_on(g, D.cb2d, C, h, ss);
-    if (tcb_run(P, 0, 1, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // D1
-    CK(g, cudaEventRecord(g->ev_d1, ms));
-    CK(g, cudaStreamWaitEvent(ss, g->ev_d1, 0));
-    if (tcb_run(P, 3, 1, ss, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW1(D)
-    colsum_on(g, D.cb1d, C, h, ss);
-    launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
-                g->a.beta2, g->a.eps, ss);
-    CK(g, cudaEventRecord(g->ev_join, ss));
-    if (tcb_run(P, 2, 1, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // A3
-    colsum_on(g, D.cb3g, C, x, ms);
-    if (tcb_run(P, 4, 3, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // A2 dW3 A1
-    colsum_on(g, D.cb2g, C, h, ms);
-    if (tcb_run(P, 7, 2, ms, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());  // dW2 dW1
-    colsum_on(g, D.cb1g, C, h, ms);
-    launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
-                g->a.beta2, g->a.eps, ms);
-    // The discriminator's Adam may still run: the next evaluation's generator kernel does not
-    // need it, so the join is deferred to just before the discriminator kernel (join_side).
-    g->side_pending = true;
-    CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
-    phase_end(g, LIPZ_PHASE_ADAM, 2);
-    g->cur = 1 - p;
-    g->t += 1;
-    g->phase = PH_IDLE;
-    return LIPZ_OK;
-  }
   if (g->use_tcb) {
+    // the nine backward products of every cell in one launch, then the bias column sums
     std::string msg;
-    TcbPlan* P = g->tcb[p];
-    // D1, dW2(D) | A3, dW1(D) | A2, dW3(G) | A1, dW2(G), dW1(G), with the bias column sums
-    if (tcb_run(P, 0, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    if (tcb_run_cells(g->tcb[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     colsum(g, D.cb2d, C, h);
     colsum(g, D.cb1d, C, h);
-    if (tcb_run(P, 2, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     colsum(g, D.cb3g, C, x);
-    if (tcb_run(P, 4, 2, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     colsum(g, D.cb2g, C, h);
-    if (tcb_run(P, 6, 3, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     colsum(g, D.cb1g, C, h);
     CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 6);
+    if (!g->prof) {
+      // The discriminator's Adam runs on the side stream, overlapping the generator's Adam and
+      // the next evaluation's generator kernel; the grid's stream waits for it before anything
+      // reads the discriminator population again (join_side).
+      phase_begin(g, LIPZ_PHASE_ADAM);
+      CK(g, cudaEventRecord(g->ev_fork, g->st));
+      CK(g, cudaStreamWaitEvent(g->side, g->ev_fork, 0));
+      launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs,
+                  g->a.beta1, g->a.beta2, g->a.eps, g->side);
+      CK(g, cudaEventRecord(g->ev_join, g->side));
+      g->side_pending = true;
+      launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs,
+                  g->a.beta1, g->a.beta2, g->a.eps, g->st);
+      CKL(g);
+      phase_end(g, LIPZ_PHASE_ADAM, 2);
+      g->cur = 1 - p;
+      g->t += 1;
+      g->phase = PH_IDLE;
+      return LIPZ_OK;
+    }
   } else {
     gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
     colsum(g, D.cb2d, C, h);

@@ -211,7 +211,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int n = min(p.BN, p.N - n0);
       n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
       const int R = lt & 1, use = lt >> 1;
-      if (!mbar_wait(bAcc + 8 * R, (uint32_t)(use & 1), abort_flag, p.err, 13)) break;
+      if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(use & 1), abort_flag, p.err, 13)) break;
       tc_fence_after();
       const int m = m0 + row;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
@@ -291,6 +291,337 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------------------------------------
+// The whole backward of one cell in one CTA: the nine products run as consecutive stages of a
+// single tile stream (double-buffered TMEM, one TMA ring). A stage that reads an earlier
+// stage's output waits until the epilogue has finished that stage's last tile: the epilogue
+// threads fence their global stores into the async proxy, meet on an mbarrier, and one of
+// them advances a tile counter in shared memory that the producer polls before loading.
+// ---------------------------------------------------------------------------------------------
+constexpr int MAX_STAGES = 9;
+
+struct Stage {
+  GParams p;
+  int dep;    // stage whose output this one reads (-1: none)
+  int tile0;  // tiles of the cell before this stage
+};
+
+struct CellPlan {
+  Stage st[MAX_STAGES];
+  int n_stages, tiles_per_cell, cells;
+  int* err;
+};
+
+struct StageMaps {
+  CUtensorMap a[MAX_STAGES];
+  CUtensorMap b[MAX_STAGES];
+};
+
+__device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int& n0, int& n) {
+  m0 = (t / p.ntiles) * BM;
+  n0 = (t % p.ntiles) * p.BN;
+  n = min(p.BN, p.N - n0);
+  n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
+}
+
+__device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0, int n0, int n,
+                                              uint32_t tbase, int hf, int row) {
+  const int m = m0 + row;
+  const int ng = n / 16;
+  const int half = (ng + 1) / 2;
+  const int g0 = hf ? half : 0, g1 = hf ? ng : half;
+  const bool row_ok = m < p.M;
+  const int arow = m < p.aux_wrap_at ? m : m - p.aux_wrap_sub;
+  for (int gi = g0; gi < g1; ++gi) {
+    uint32_t r[16];
+    LIPZ_TMEM_LD16(tbase + gi * 16, r);
+    tmem_wait_ld();
+    const int col0 = n0 + gi * 16;
+    if (!row_ok) continue;
+    if (p.epi == EPI_F32) {
+      float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+      if (p.scn == 1 && col0 + 16 <= p.N) {
+        float4* o = reinterpret_cast<float4*>(C + col0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
+                             __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e)
+          if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __uint_as_float(r[e]);
+      }
+    } else {
+      bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+      const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
+      float v[16];
+      if (p.sxn == 1 && col0 + 16 <= p.N) {
+        const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
+        const uint4 q0 = x4[0], q1 = x4[1];
+        const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          const __nv_bfloat162 y2 = *reinterpret_cast<const __nv_bfloat162*>(&w[e >> 1]);
+          v[e] = __uint_as_float(r[e]) * dact(p.act, __low2float(y2), p.slope);
+          v[e + 1] = __uint_as_float(r[e + 1]) * dact(p.act, __high2float(y2), p.slope);
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int col = col0 + e;
+          const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
+          v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
+        }
+      }
+      if (p.scn == 1 && col0 + 16 <= p.N) {
+        uint32_t pk[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          __nv_bfloat162 b2 = __floats2bfloat162_rn(v[e], v[e + 1]);
+          pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
+        }
+        uint4* o = reinterpret_cast<uint4*>(C + col0);
+        o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e)
+          if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __float2bfloat16_rn(v[e]);
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    k_bwd_cells(const __grid_constant__ StageMaps maps, const __grid_constant__ CellPlan cp) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  uint8_t* misc = gbase + STAGES * STAGE_BYTES;
+  const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES;
+  const uint32_t bAcc = bEmpty + 8 * STAGES, bReg = bAcc + 16, bFinal = bReg + 16;
+  const uint32_t bEpi = bFinal + 8;  // [2], alternating by tile
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
+  volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 200);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(bFull + 8 * s, 1);
+      mbar_init(bEmpty + 8 * s, 1);
+    }
+    mbar_init(bAcc, 1);
+    mbar_init(bAcc + 8, 1);
+    mbar_init(bReg, 32 * NUM_EPI_WARPS);
+    mbar_init(bReg + 8, 32 * NUM_EPI_WARPS);
+    mbar_init(bFinal, 1);
+    mbar_init(bEpi, 32 * NUM_EPI_WARPS);
+    mbar_init(bEpi + 8, 32 * NUM_EPI_WARPS);
+    *abort_flag = 0;
+    *done_tiles = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  int* err = cp.err;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued[STAGES] = {0, 0, 0, 0};
+      bool ok = true;
+      int stage = 0;
+      uint32_t phase = 0;
+      int cells_done = 0;
+      for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x, ++cells_done) {
+        for (int si = 0; si < cp.n_stages && ok; ++si) {
+          const GParams& p = cp.st[si].p;
+          const int dep = cp.st[si].dep;
+          if (dep >= 0) {
+            // the stage reads the output of stage `dep` of this cell: wait for its last tile
+            const GParams& pd = cp.st[dep].p;
+            const int need = cells_done * cp.tiles_per_cell + cp.st[dep].tile0 +
+                             pd.mtiles * pd.ntiles;
+            const unsigned long long t0 = globaltimer();
+            uint32_t it = 0;
+            while (*done_tiles < need) {
+              if ((++it & 255u) == 0) {
+                if (*abort_flag) {
+                  ok = false;
+                  break;
+                }
+                if (globaltimer() - t0 > WAIT_NS) {
+                  *abort_flag = 1;
+                  atomicExch(err, 16);
+                  ok = false;
+                  break;
+                }
+              }
+            }
+            if (!ok) break;
+            __threadfence_block();
+          }
+          const CUtensorMap* mA = &maps.a[si];
+          const CUtensorMap* mB = &maps.b[si];
+          const int za = p.a_sel ? __ldg(&p.a_sel[cell]) : cell;
+          const int zb = p.b_sel ? __ldg(&p.b_sel[cell]) : cell;
+          const uint32_t b_bytes =
+              p.b_mn ? (uint32_t)((p.BN / 64) * MN_BOX_BYTES) : (uint32_t)(p.BN * 128);
+          const int nt = p.mtiles * p.ntiles;
+          for (int t = 0; t < nt && ok; ++t) {
+            int m0, n0, n;
+            stage_tile(p, t, m0, n0, n);
+            for (int kc = 0; kc < p.kchunks; ++kc) {
+              if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, err, 11)) {
+                ok = false;
+                break;
+              }
+              const uint32_t full = bFull + 8 * stage;
+              mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
+              const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+              if (p.a_mn) {
+                tma_load_3d(sA, mA, full, m0, kc * BK, za);
+                tma_load_3d(sA + MN_BOX_BYTES, mA, full, m0 + 64, kc * BK, za);
+              } else {
+                tma_load_3d(sA, mA, full, kc * BK, p.a_row0 + m0, za);
+              }
+              if (p.b_mn) {
+                for (int i = 0; i < p.BN / 64; ++i)
+                  tma_load_3d(sB + i * MN_BOX_BYTES, mB, full, n0 + 64 * i, kc * BK, zb);
+              } else {
+                tma_load_3d(sB, mB, full, kc * BK, p.b_row0 + n0, zb);
+              }
+              issued[stage]++;
+              if (++stage == STAGES) {
+                stage = 0;
+                phase ^= 1u;
+              }
+            }
+          }
+        }
+      }
+      if (!ok) {
+        for (int s = 0; s < STAGES; ++s)
+          if (issued[s] > 0) {
+            volatile int never = 0;
+            mbar_wait(bFull + 8 * s, (uint32_t)((issued[s] - 1) & 1), &never, err, 11);
+          }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int lt = 0;
+      for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
+        for (int si = 0; si < cp.n_stages && ok; ++si) {
+          const GParams& p = cp.st[si].p;
+          const int nt = p.mtiles * p.ntiles;
+          for (int t = 0; t < nt && ok; ++t, ++lt) {
+            int m0, n0, n;
+            stage_tile(p, t, m0, n0, n);
+            const int R = lt & 1, use = lt >> 1;
+            if (use > 0 &&
+                !mbar_wait(bReg + 8 * R, (uint32_t)((use - 1) & 1), abort_flag, err, 15)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t d = tmem + (uint32_t)(R * 256);
+            const uint32_t idesc = idesc_bf16_major(BM, n, p.a_mn, p.b_mn);
+            for (int kc = 0; kc < p.kchunks; ++kc) {
+              if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, err, 12)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+#pragma unroll
+              for (int kk = 0; kk < BK / 16; ++kk) {
+                const uint64_t ad = p.a_mn ? sw128_mn_desc(sA + kk * 2048, MN_BOX_BYTES)
+                                           : sw128_desc(sA + kk * 32);
+                const uint64_t bd = p.b_mn ? sw128_mn_desc(sB + kk * 2048, MN_BOX_BYTES)
+                                           : sw128_desc(sB + kk * 32);
+                tc_mma(d, ad, bd, idesc, (kc | kk) != 0 ? 1u : 0u);
+              }
+              tc_commit(bEmpty + 8 * stage);
+              if (++stage == STAGES) {
+                stage = 0;
+                phase ^= 1u;
+              }
+            }
+            if (!ok) break;
+            tc_commit(bAcc + 8 * R);
+          }
+        }
+      }
+      tc_commit(bFinal);
+      volatile int never = 0;
+      mbar_wait(bFinal, 0u, &never, err, 14);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
+    const int row = q * 32 + lane;
+    bool ok = true;
+    int lt = 0;
+    for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
+      for (int si = 0; si < cp.n_stages && ok; ++si) {
+        const GParams& p = cp.st[si].p;
+        const int nt = p.mtiles * p.ntiles;
+        for (int t = 0; t < nt; ++t, ++lt) {
+          int m0, n0, n;
+          stage_tile(p, t, m0, n0, n);
+          const int R = lt & 1, use = lt >> 1;
+          if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(use & 1), abort_flag, err, 13)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
+          epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+          // publish the tile's global stores to the async proxy (later TMA loads), then count
+          // it. The tile's arrival on bEpi[lt & 1] comes before its arrival on bReg, so no
+          // thread can reach tile lt + 2 (same barrier) before every thread has arrived here.
+          asm volatile("fence.proxy.async;" ::: "memory");
+          mbar_arrive(bEpi + 8 * (lt & 1));
+          tc_fence_before();
+          mbar_arrive(bReg + 8 * R);
+          if (warp == 2) {
+            // one warp counts the tile once all epilogue threads have published their stores
+            if (!mbar_wait_warp(bEpi + 8 * (lt & 1), (uint32_t)((lt >> 1) & 1), abort_flag, err,
+                                17)) {
+              ok = false;
+              break;
+            }
+            if (lane == 0) {
+              __threadfence_block();
+              *done_tiles = lt + 1;
+            }
+            __syncwarp();
+          }
+        }
+      }
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+  }
+}
+
 }  // namespace tcb
 
 // ---- host side -----------------------------------------------------------------------------
@@ -343,6 +674,9 @@ struct TcbPlan {
   Gemm g[9];
   int n;
   int* err;
+  tcb::StageMaps maps;  // the same nine products as one per-cell kernel
+  tcb::CellPlan cells;
+  int grid_cells;
 };
 
 bool tcb_supported(int z, int h, int x, int B) {
@@ -561,6 +895,30 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     finish(G);
   }
   P->n = i;
+  if (ok) {
+    // per-cell megakernel: stage order as above; each stage's dependency on an earlier output
+    const int deps[9] = {-1, -1, 0, 0, 2, 2, 4, 4, 6};
+    int tile0 = 0;
+    for (int k = 0; k < i; ++k) {
+      P->maps.a[k] = P->g[k].a;
+      P->maps.b[k] = P->g[k].b;
+      P->cells.st[k].p = P->g[k].p;
+      P->cells.st[k].dep = deps[k];
+      P->cells.st[k].tile0 = tile0;
+      tile0 += P->g[k].p.mtiles * P->g[k].p.ntiles;
+    }
+    P->cells.n_stages = i;
+    P->cells.tiles_per_cell = tile0;
+    P->cells.cells = C;
+    P->cells.err = P->err;
+    P->grid_cells = C < sms ? C : sms;
+    if (cudaFuncSetAttribute(tcb::k_bwd_cells, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tcb::SMEM_BYTES) != cudaSuccess) {
+      cudaGetLastError();
+      if (msg) *msg = "cannot reserve shared memory for the per-cell backward";
+      ok = false;
+    }
+  }
   if (!ok) {
     cudaFree(P->err);
     delete P;
@@ -581,6 +939,16 @@ int tcb_run(TcbPlan* P, int first, int count, cudaStream_t st, std::string* msg)
       if (msg) *msg = std::string("tensor-core backward launch: ") + cudaGetErrorString(e);
       return 1;
     }
+  }
+  return 0;
+}
+
+int tcb_run_cells(TcbPlan* P, cudaStream_t st, std::string* msg) {
+  tcb::k_bwd_cells<<<P->grid_cells, tcb::THREADS, tcb::SMEM_BYTES, st>>>(P->maps, P->cells);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    if (msg) *msg = std::string("per-cell backward launch: ") + cudaGetErrorString(e);
+    return 1;
   }
   return 0;
 }

@@ -309,7 +309,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int j = 0; j < nj && ok; ++j) {
         const Job J = get_job(p, j);
         const int R = J.region;
-        if (!mbar_wait(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
+        if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
           ok = false;
           break;
         }
@@ -408,7 +408,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_arrive(bPart);
             mbar_arrive(bReg + 8 * R);
           } else {
-            if (!mbar_wait(bPart, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 7)) {
+            if (!mbar_wait_warp(bPart, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 7)) {
               ok = false;
               break;
             }
