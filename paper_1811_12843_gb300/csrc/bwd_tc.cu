@@ -324,6 +324,66 @@ __device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int
   n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
 }
 
+// 16 accumulator columns of one row: fp32 store, or bf16 delta times the activation
+// derivative (read from the stored forward output). `full` = all 16 columns lie inside N.
+__device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16], int cell, int m,
+                                      int arow, int col0, bool full, float dlo, bool is_tanh) {
+  if (p.epi == EPI_F32) {
+    float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+    if (p.scn == 1) {
+      if (full) {
+        float4* o = reinterpret_cast<float4*>(C + col0);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
+                             __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
+      } else {
+        for (int e = 0; e < 16 && col0 + e < p.N; ++e) C[col0 + e] = __uint_as_float(r[e]);
+      }
+    } else {
+      // transposed output: lanes hold consecutive rows, so each store is one coalesced line
+      const int64_t sc = p.scn;
+      float* o = C + (int64_t)col0 * sc;
+      if (full) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) o[e * sc] = __uint_as_float(r[e]);
+      } else {
+        for (int e = 0; e < 16 && col0 + e < p.N; ++e) o[e * sc] = __uint_as_float(r[e]);
+      }
+    }
+    return;
+  }
+  bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
+  const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
+  if (p.sxn == 1 && p.scn == 1 && full) {
+    const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
+    const uint4 q0 = x4[0], q1 = x4[1];
+    const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+    uint32_t pk[8];
+#pragma unroll
+    for (int e = 0; e < 16; e += 2) {
+      const __nv_bfloat162 y2 = *reinterpret_cast<const __nv_bfloat162*>(&w[e >> 1]);
+      const float y0 = __low2float(y2), y1 = __high2float(y2);
+      const float d0 = is_tanh ? 1.f - y0 * y0 : (y0 > 0.f ? 1.f : dlo);
+      const float d1 = is_tanh ? 1.f - y1 * y1 : (y1 > 0.f ? 1.f : dlo);
+      __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(r[e]) * d0,
+                                                __uint_as_float(r[e + 1]) * d1);
+      pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
+    }
+    uint4* o = reinterpret_cast<uint4*>(C + col0);
+    o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+    return;
+  }
+  for (int e = 0; e < 16; ++e) {
+    const int col = col0 + e;
+    if (col >= p.N) break;
+    const float y = __bfloat162float(X[(int64_t)col * p.sxn]);
+    const float d = is_tanh ? 1.f - y * y : (y > 0.f ? 1.f : dlo);
+    C[(int64_t)col * p.scn] = __float2bfloat16_rn(__uint_as_float(r[e]) * d);
+  }
+}
+
 __device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0, int n0, int n,
                                               uint32_t tbase, int hf, int row) {
   const int m = m0 + row;
@@ -332,63 +392,27 @@ __device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0
   const int g0 = hf ? half : 0, g1 = hf ? ng : half;
   const bool row_ok = m < p.M;
   const int arow = m < p.aux_wrap_at ? m : m - p.aux_wrap_sub;
-  for (int gi = g0; gi < g1; ++gi) {
+  const bool is_tanh = p.act == ACT_TANH;
+  const float dlo = p.act == ACT_RELU ? 0.f : p.slope;
+  int gi = g0;
+  // two 16-column groups per TMEM load where possible
+  for (; gi + 1 < g1; gi += 2) {
+    uint32_t r[32];
+    LIPZ_TMEM_LD32(tbase + gi * 16, r);
+    tmem_wait_ld();
+    if (!row_ok) continue;
+    const int col0 = n0 + gi * 16;
+    const uint32_t(&ra)[16] = *reinterpret_cast<const uint32_t(*)[16]>(&r[0]);
+    const uint32_t(&rb)[16] = *reinterpret_cast<const uint32_t(*)[16]>(&r[16]);
+    epi16(p, ra, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh);
+    if (col0 + 16 < p.N) epi16(p, rb, cell, m, arow, col0 + 16, col0 + 32 <= p.N, dlo, is_tanh);
+  }
+  if (gi < g1) {
     uint32_t r[16];
     LIPZ_TMEM_LD16(tbase + gi * 16, r);
     tmem_wait_ld();
     const int col0 = n0 + gi * 16;
-    if (!row_ok) continue;
-    if (p.epi == EPI_F32) {
-      float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
-      if (p.scn == 1 && col0 + 16 <= p.N) {
-        float4* o = reinterpret_cast<float4*>(C + col0);
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
-                             __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
-      } else {
-#pragma unroll
-        for (int e = 0; e < 16; ++e)
-          if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __uint_as_float(r[e]);
-      }
-    } else {
-      bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
-      const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
-      float v[16];
-      if (p.sxn == 1 && col0 + 16 <= p.N) {
-        const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
-        const uint4 q0 = x4[0], q1 = x4[1];
-        const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
-#pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          const __nv_bfloat162 y2 = *reinterpret_cast<const __nv_bfloat162*>(&w[e >> 1]);
-          v[e] = __uint_as_float(r[e]) * dact(p.act, __low2float(y2), p.slope);
-          v[e + 1] = __uint_as_float(r[e + 1]) * dact(p.act, __high2float(y2), p.slope);
-        }
-      } else {
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const int col = col0 + e;
-          const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
-          v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
-        }
-      }
-      if (p.scn == 1 && col0 + 16 <= p.N) {
-        uint32_t pk[8];
-#pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          __nv_bfloat162 b2 = __floats2bfloat162_rn(v[e], v[e + 1]);
-          pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
-        }
-        uint4* o = reinterpret_cast<uint4*>(C + col0);
-        o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-      } else {
-#pragma unroll
-        for (int e = 0; e < 16; ++e)
-          if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __float2bfloat16_rn(v[e]);
-      }
-    }
+    if (row_ok && col0 < p.N) epi16(p, r, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh);
   }
 }
 
