@@ -35,6 +35,7 @@ struct Descs {
   GemmDesc *tg1, *tg2, *td1, *td2, *bw2d, *bd1, *bw1d, *ba3, *bw3g, *ba2, *bw2g, *ba1, *bw1g;
   GemvDesc* tgv;
   ColSumDesc *cb2d, *cb1d, *cb3g, *cb2g, *cb1g;
+  ColSumDesc* cb_all;  // the five above in one array (one launch)
 };
 
 }  // namespace
@@ -421,6 +422,9 @@ int build_descs(lipz_grid* g, int p) {
       (rc = upload(g, &D.cb3g, cb3g)) || (rc = upload(g, &D.cb2g, cb2g)) ||
       (rc = upload(g, &D.cb1g, cb1g)))
     return rc;
+  std::vector<ColSumDesc> all;
+  for (auto* v : {&cb2d, &cb1d, &cb3g, &cb2g, &cb1g}) all.insert(all.end(), v->begin(), v->end());
+  if ((rc = upload(g, &D.cb_all, all))) return rc;
   return LIPZ_OK;
 }
 
@@ -716,13 +720,9 @@ int train_impl(lipz_grid* g) {
     // the nine backward products of every cell in one launch, then the bias column sums
     std::string msg;
     if (tcb_run_cells(g->tcb[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
-    colsum(g, D.cb2d, C, h);
-    colsum(g, D.cb1d, C, h);
-    colsum(g, D.cb3g, C, x);
-    colsum(g, D.cb2g, C, h);
-    colsum(g, D.cb1g, C, h);
+    colsum(g, D.cb_all, 5 * C, h > x ? h : x);
     CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 6);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 3);
     if (!g->prof) {
       // The discriminator's Adam runs on the side stream, overlapping the generator's Adam and
       // the next evaluation's generator kernel; the grid's stream waits for it before anything

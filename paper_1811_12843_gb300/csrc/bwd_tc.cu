@@ -302,13 +302,15 @@ constexpr int MAX_STAGES = 9;
 
 struct Stage {
   GParams p;
-  int dep;    // stage whose output this one reads (-1: none)
-  int tile0;  // tiles of the cell before this stage
+  int dep;      // stage whose output this one reads (-1: none)
+  int tile0;    // tiles of the cell before this stage
+  int publish;  // a later stage reads this one's output: its tiles are published and counted
+  int pub_end;  // published tiles of the cell up to and including this stage
 };
 
 struct CellPlan {
   Stage st[MAX_STAGES];
-  int n_stages, tiles_per_cell, cells;
+  int n_stages, tiles_per_cell, pub_per_cell, cells;
   int* err;
 };
 
@@ -472,9 +474,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int dep = cp.st[si].dep;
           if (dep >= 0) {
             // the stage reads the output of stage `dep` of this cell: wait for its last tile
-            const GParams& pd = cp.st[dep].p;
-            const int need = cells_done * cp.tiles_per_cell + cp.st[dep].tile0 +
-                             pd.mtiles * pd.ntiles;
+            const int need = cells_done * cp.pub_per_cell + cp.st[dep].pub_end;
             const unsigned long long t0 = globaltimer();
             uint32_t it = 0;
             while (*done_tiles < need) {
@@ -597,10 +597,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
     const int row = q * 32 + lane;
     bool ok = true;
-    int lt = 0;
+    int lt = 0, pub = 0;
     for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
       for (int si = 0; si < cp.n_stages && ok; ++si) {
         const GParams& p = cp.st[si].p;
+        const bool publish = cp.st[si].publish != 0;
         const int nt = p.mtiles * p.ntiles;
         for (int t = 0; t < nt; ++t, ++lt) {
           int m0, n0, n;
@@ -613,25 +614,31 @@ __global__ void __launch_bounds__(THREADS, 1)
           tc_fence_after();
           const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
           epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
-          // publish the tile's global stores to the async proxy (later TMA loads), then count
-          // it. The tile's arrival on bEpi[lt & 1] comes before its arrival on bReg, so no
-          // thread can reach tile lt + 2 (same barrier) before every thread has arrived here.
-          asm volatile("fence.proxy.async;" ::: "memory");
-          mbar_arrive(bEpi + 8 * (lt & 1));
+          if (publish) {
+            // publish the tile's global stores to the async proxy (a later stage loads them by
+            // TMA). The arrival on bEpi[pub & 1] comes before the arrival on bReg, so no thread
+            // can reach the next-but-one published tile (same barrier) before every thread
+            // has arrived here.
+            asm volatile("fence.proxy.async;" ::: "memory");
+            mbar_arrive(bEpi + 8 * (pub & 1));
+          }
           tc_fence_before();
           mbar_arrive(bReg + 8 * R);
-          if (warp == 2) {
-            // one warp counts the tile once all epilogue threads have published their stores
-            if (!mbar_wait_warp(bEpi + 8 * (lt & 1), (uint32_t)((lt >> 1) & 1), abort_flag, err,
-                                17)) {
-              ok = false;
-              break;
+          if (publish) {
+            if (warp == 2) {
+              // one warp counts the tile once all epilogue threads have published their stores
+              if (!mbar_wait_warp(bEpi + 8 * (pub & 1), (uint32_t)((pub >> 1) & 1), abort_flag,
+                                  err, 17)) {
+                ok = false;
+                break;
+              }
+              if (lane == 0) {
+                __threadfence_block();
+                *done_tiles = pub + 1;
+              }
+              __syncwarp();
             }
-            if (lane == 0) {
-              __threadfence_block();
-              *done_tiles = lt + 1;
-            }
-            __syncwarp();
+            ++pub;
           }
         }
       }
@@ -922,17 +929,24 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
   if (ok) {
     // per-cell megakernel: stage order as above; each stage's dependency on an earlier output
     const int deps[9] = {-1, -1, 0, 0, 2, 2, 4, 4, 6};
-    int tile0 = 0;
+    int tile0 = 0, pub = 0;
     for (int k = 0; k < i; ++k) {
+      int publish = 0;
+      for (int j = k + 1; j < i; ++j) publish |= deps[j] == k;
+      const int nt = P->g[k].p.mtiles * P->g[k].p.ntiles;
       P->maps.a[k] = P->g[k].a;
       P->maps.b[k] = P->g[k].b;
       P->cells.st[k].p = P->g[k].p;
       P->cells.st[k].dep = deps[k];
       P->cells.st[k].tile0 = tile0;
-      tile0 += P->g[k].p.mtiles * P->g[k].p.ntiles;
+      P->cells.st[k].publish = publish;
+      tile0 += nt;
+      if (publish) pub += nt;
+      P->cells.st[k].pub_end = pub;
     }
     P->cells.n_stages = i;
     P->cells.tiles_per_cell = tile0;
+    P->cells.pub_per_cell = pub;
     P->cells.cells = C;
     P->cells.err = P->err;
     P->grid_cells = C < sms ? C : sms;
