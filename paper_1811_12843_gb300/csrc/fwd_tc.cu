@@ -43,7 +43,9 @@ constexpr int N3 = 256;                      // generator output columns per MMA
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr int MISC_BYTES = 2048;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + H_BYTES + MISC_BYTES;
+constexpr int BIAS_MAX = 256 + 256 + 1024;  // floats per tile: b1, b2, then b3 (G) or w3, b3 (D)
+constexpr int BIAS_BYTES = 2 * BIAS_MAX * 4;  // double-buffered by tile
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + H_BYTES + MISC_BYTES + BIAS_BYTES;
 
 enum { KIND_G = 0, KIND_D = 1 };
 enum { EPI_TO_H = 0, EPI_LOGIT = 1, EPI_TO_E = 2, EPI_ACT_OUT = 3 };
@@ -114,19 +116,6 @@ __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   return p.train ? __ldg(&p.wsel[prob]) : __ldg(&p.nbr[prob]);
 }
 
-// 32 consecutive fp32 biases (16-byte aligned; the same addresses for every lane of a warp).
-__device__ __forceinline__ void load_bias32(const float* b, float (&bv)[32]) {
-  const float4* b4 = reinterpret_cast<const float4*>(b);
-#pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    const float4 t = __ldg(b4 + q);
-    bv[4 * q] = t.x;
-    bv[4 * q + 1] = t.y;
-    bv[4 * q + 2] = t.z;
-    bv[4 * q + 3] = t.w;
-  }
-}
-
 // Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
 // output that follows it).
 __device__ __forceinline__ float tanh_approx(float x) {
@@ -155,6 +144,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t bH = bReg + 16;
   const uint32_t bPart = bH + 8;
   const uint32_t bFinal = bPart + 8;
+  const uint32_t bBias = bFinal + 8;  // [2]: the tile's biases are in shared memory
+  float* s_bias = reinterpret_cast<float*>(misc + MISC_BYTES);  // [2][BIAS_MAX]
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 256);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 260);
   float* part = reinterpret_cast<float*>(misc + 512);           // [128] partial logits
@@ -172,6 +163,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(bH, 32 * NUM_EPI_WARPS);
     mbar_init(bPart, 32 * NUM_EPI_WARPS / 2);
     mbar_init(bFinal, 1);
+    mbar_init(bBias, 32 * NUM_EPI_WARPS);
+    mbar_init(bBias + 8, 32 * NUM_EPI_WARPS);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -298,7 +291,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     int reg_uses[2] = {0, 0};
     bool ok = true;
-    for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
+    int ltile = 0;
+    const int et = threadIdx.x - 64;  // epilogue thread 0..255
+    for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++ltile) {
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
       const int c = prob_cell(p, prob), slot = prob % 5;
       const int k = prob_individual(p, prob);
@@ -306,6 +301,29 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int rr = m0 + row;
       const bool row_ok = rr < p.rows;
       const int64_t act_off = ((int64_t)prob * p.rows + rr) * HID;
+      // The tile's biases (and D's output weights) go to shared memory once, while the MMAs
+      // run, so that no epilogue waits on a global load. Buffer ltile & 1; a thread cannot
+      // reach tile ltile + 2 before every thread has passed this tile's arrival.
+      float* sb = s_bias + (ltile & 1) * BIAS_MAX;
+      {
+        const int nb3 = p.kind == KIND_D ? HID + 1 : p.x;
+        for (int i = et; i < 512 + nb3; i += 256) {
+          float v;
+          if (i < 256) v = wm[p.off_b1 + i];
+          else if (i < 512) v = wm[p.off_b2 + i - 256];
+          else if (p.kind == KIND_D)
+            v = i < 512 + HID ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
+                              : wm[p.off_b3];
+          else v = wm[p.off_b3 + i - 512];
+          sb[i] = v;
+        }
+        mbar_arrive(bBias + 8 * (ltile & 1));
+        if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
+                            p.err, 8)) {
+          ok = false;
+          break;
+        }
+      }
       for (int j = 0; j < nj && ok; ++j) {
         const Job J = get_job(p, j);
         const int R = J.region;
@@ -316,43 +334,55 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc_fence_after();
         const uint32_t tbase = tmem + lane_base + (uint32_t)(R * HID);
         if (J.epi == EPI_TO_H || J.epi == EPI_ACT_OUT) {
-          const float* bias = wm + (j == 0 ? p.off_b1 : p.off_b2);
+          const float* bias = sb + (j == 0 ? 0 : 256);
           const bool lrelu = p.kind == KIND_D;
           const bool to_h = J.epi == EPI_TO_H;
           bf16* gout = j == 0 ? p.act1 : p.act2;
 #pragma unroll 1
-          for (int cg = hf * 4; cg < hf * 4 + 4; ++cg) {
-            uint32_t r[32];
-            LIPZ_TMEM_LD32(tbase + cg * 32, r);
+          for (int cp = hf * 4; cp < hf * 4 + 4; cp += 2) {
+            uint32_t r2[2][32];
+            LIPZ_TMEM_LD32(tbase + cp * 32, r2[0]);
+            LIPZ_TMEM_LD32(tbase + (cp + 1) * 32, r2[1]);
             tmem_wait_ld();
-            float bv[32];
-            load_bias32(bias + cg * 32, bv);
-            uint32_t pk[16];
 #pragma unroll
-            for (int e = 0; e < 32; e += 2) {
-              float a0 = __uint_as_float(r[e]) + bv[e];
-              float a1 = __uint_as_float(r[e + 1]) + bv[e + 1];
-              a0 = a0 > 0.f ? a0 : (lrelu ? p.slope * a0 : 0.f);
-              a1 = a1 > 0.f ? a1 : (lrelu ? p.slope * a1 : 0.f);
-              pk[e >> 1] = pack_bf16(a0, a1);
-            }
-            if (to_h) {
-              const uint32_t chunk = sH + (uint32_t)((cg >> 1) * H_CHUNK) + (uint32_t)row * 128u;
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const int cg = cp + h2;
+              const uint32_t(&r)[32] = r2[h2];
+              const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
+              uint32_t pk[16];
 #pragma unroll
-              for (int u = 0; u < 4; ++u) {
-                const uint32_t unit = (uint32_t)((cg & 1) * 4 + u);
-                const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
-                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
-                             "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]),
-                             "r"(pk[4 * u + 3])
-                             : "memory");
+              for (int e = 0; e < 32; e += 4) {
+                const float4 bb = b4[e >> 2];
+                float a0 = __uint_as_float(r[e]) + bb.x;
+                float a1 = __uint_as_float(r[e + 1]) + bb.y;
+                float a2 = __uint_as_float(r[e + 2]) + bb.z;
+                float a3 = __uint_as_float(r[e + 3]) + bb.w;
+                const float lo = lrelu ? p.slope : 0.f;
+                a0 = a0 > 0.f ? a0 : lo * a0;
+                a1 = a1 > 0.f ? a1 : lo * a1;
+                a2 = a2 > 0.f ? a2 : lo * a2;
+                a3 = a3 > 0.f ? a3 : lo * a3;
+                pk[e >> 1] = pack_bf16(a0, a1);
+                pk[(e >> 1) + 1] = pack_bf16(a2, a3);
               }
-            }
-            if (gout && row_ok) {
-              uint4* o = reinterpret_cast<uint4*>(gout + act_off + cg * 32);
+              if (to_h) {
+                const uint32_t chunk = sH + (uint32_t)((cg >> 1) * H_CHUNK) + (uint32_t)row * 128u;
 #pragma unroll
-              for (int u = 0; u < 4; ++u)
-                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 4; ++u) {
+                  const uint32_t unit = (uint32_t)((cg & 1) * 4 + u);
+                  const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
+                  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                               "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]),
+                               "r"(pk[4 * u + 3])
+                               : "memory");
+                }
+              }
+              if (gout && row_ok) {
+                uint4* o = reinterpret_cast<uint4*>(gout + act_off + cg * 32);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+              }
             }
           }
           if (to_h) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -360,46 +390,49 @@ __global__ void __launch_bounds__(THREADS, 1)
           mbar_arrive(bReg + 8 * R);
           if (to_h) mbar_arrive(bH);
         } else if (J.epi == EPI_LOGIT) {
-          const float* bias = wm + p.off_b2;
-          const bf16* w3 = p.wb + (int64_t)k * p.pstride + p.off_w3;
+          const float* bias = sb + 256;
+          const float* w3 = sb + 512;
           float acc = 0.f;
 #pragma unroll 1
-          for (int cg = hf * 4; cg < hf * 4 + 4; ++cg) {
-            uint32_t r[32];
-            LIPZ_TMEM_LD32(tbase + cg * 32, r);
+          for (int cp = hf * 4; cp < hf * 4 + 4; cp += 2) {
+            uint32_t r2[2][32];
+            LIPZ_TMEM_LD32(tbase + cp * 32, r2[0]);
+            LIPZ_TMEM_LD32(tbase + (cp + 1) * 32, r2[1]);
             tmem_wait_ld();
-            float bv[32];
-            load_bias32(bias + cg * 32, bv);
-            uint32_t wv[16];
-            {
-              const uint4* w4 = reinterpret_cast<const uint4*>(w3 + cg * 32);
 #pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const uint4 t = __ldg(w4 + q);
-                wv[4 * q] = t.x;
-                wv[4 * q + 1] = t.y;
-                wv[4 * q + 2] = t.z;
-                wv[4 * q + 3] = t.w;
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const int cg = cp + h2;
+              const uint32_t(&r)[32] = r2[h2];
+              const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
+              const float4* w4 = reinterpret_cast<const float4*>(w3 + cg * 32);
+              uint32_t pk[16];
+#pragma unroll
+              for (int e = 0; e < 32; e += 4) {
+                const float4 bb = b4[e >> 2], ww = w4[e >> 2];
+                float a0 = __uint_as_float(r[e]) + bb.x;
+                float a1 = __uint_as_float(r[e + 1]) + bb.y;
+                float a2 = __uint_as_float(r[e + 2]) + bb.z;
+                float a3 = __uint_as_float(r[e + 3]) + bb.w;
+                a0 = a0 > 0.f ? a0 : p.slope * a0;
+                a1 = a1 > 0.f ? a1 : p.slope * a1;
+                a2 = a2 > 0.f ? a2 : p.slope * a2;
+                a3 = a3 > 0.f ? a3 : p.slope * a3;
+                pk[e >> 1] = pack_bf16(a0, a1);
+                pk[(e >> 1) + 1] = pack_bf16(a2, a3);
+                const __nv_bfloat162 q01 = *reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]);
+                const __nv_bfloat162 q23 =
+                    *reinterpret_cast<const __nv_bfloat162*>(&pk[(e >> 1) + 1]);
+                acc = fmaf(__low2float(q01), ww.x, acc);
+                acc = fmaf(__high2float(q01), ww.y, acc);
+                acc = fmaf(__low2float(q23), ww.z, acc);
+                acc = fmaf(__high2float(q23), ww.w, acc);
               }
-            }
-            uint32_t pk[16];
+              if (p.act2 && row_ok) {
+                uint4* o = reinterpret_cast<uint4*>(p.act2 + act_off + cg * 32);
 #pragma unroll
-            for (int e = 0; e < 32; e += 2) {
-              float a0 = __uint_as_float(r[e]) + bv[e];
-              float a1 = __uint_as_float(r[e + 1]) + bv[e + 1];
-              a0 = a0 > 0.f ? a0 : p.slope * a0;
-              a1 = a1 > 0.f ? a1 : p.slope * a1;
-              pk[e >> 1] = pack_bf16(a0, a1);
-              const __nv_bfloat162 q2 = *reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]);
-              const __nv_bfloat162 w2 = *reinterpret_cast<const __nv_bfloat162*>(&wv[e >> 1]);
-              acc = fmaf(__low2float(q2), __low2float(w2), acc);
-              acc = fmaf(__high2float(q2), __high2float(w2), acc);
-            }
-            if (p.act2 && row_ok) {
-              uint4* o = reinterpret_cast<uint4*>(p.act2 + act_off + cg * 32);
-#pragma unroll
-              for (int u = 0; u < 4; ++u)
-                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 4; ++u)
+                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+              }
             }
           }
           tc_fence_before();
@@ -412,13 +445,13 @@ __global__ void __launch_bounds__(THREADS, 1)
               ok = false;
               break;
             }
-            const float logit = acc + part[row] + __ldg(wm + p.off_b3);
+            const float logit = acc + part[row] + sb[512 + HID];
             mbar_arrive(bReg + 8 * R);
             if (row_ok) p.logits[(int64_t)prob * p.rows + rr] = logit;
           }
         } else {
           // generator output block: bias + tanh, bf16, into the fake rows of E[c]
-          const float* bias = wm + p.off_b3;
+          const float* bias = sb + 512;
           const int ng = J.n / 16;
           const int split = (ng + 1) / 2;
           const int g0 = hf ? split : 0, g1 = hf ? ng : split;
@@ -434,7 +467,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
-                const float4 t = __ldg(b4 + q);
+                const float4 t = b4[q];
                 bv[4 * q] = t.x;
                 bv[4 * q + 1] = t.y;
                 bv[4 * q + 2] = t.z;
@@ -520,7 +553,8 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, u
 }  // namespace
 
 bool tc_supported(int z, int h, int x, int B) {
-  return h == tc::HID && z % 16 == 0 && z >= 64 && z <= 256 && x % 16 == 0 && x >= 64 && B >= 1;
+  return h == tc::HID && z % 16 == 0 && z >= 64 && z <= 256 && x % 16 == 0 && x >= 64 &&
+         x <= 1024 && B >= 1;
 }
 
 TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
