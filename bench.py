@@ -51,8 +51,8 @@ TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels, from
 # the ncu launch list in profiles/launches_12x12_bf16_iteration.md (same kernels as this build).
-PHASE_TRAFFIC = {"batch": 41.4e6, "g_fwd": 159.5e6, "d_fwd": 226.9e6, "fitness": 1.7e6,
-                 "select": 0.0, "train_fwd": 160.7e6, "train_bwd": 557.9e6, "adam": 2105.9e6}
+PHASE_TRAFFIC = {"batch": 41.4e6, "g_fwd": 159.9e6, "d_fwd": 226.9e6, "fitness": 1.7e6,
+                 "select": 0.0, "train_fwd": 161.2e6, "train_bwd": 668.5e6, "adam": 2112.0e6}
 
 
 def _peaks():
@@ -345,7 +345,7 @@ def run_reference(args):
     from oracle import lipz_oracle as O
     arch = O.Arch(precision="bf16", batch=BATCH)
     _oracle_state(arch)
-    per_step_cells = 2
+    per_step_cells = 1
     for _ in range(args.warmup):
         _oracle_sample(1e9, max_cells=1)
     times = []
@@ -373,8 +373,8 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
