@@ -61,236 +61,6 @@ __device__ __forceinline__ float dact(int act, float y, float slope) {
   }
 }
 
-// Persistent: CTAs walk the product's tiles (cell, m-tile, n-tile); the accumulator of
-// consecutive tiles alternates between two 256-column TMEM regions, so the epilogue of one
-// tile overlaps the loads and MMAs of the next.
-template <int EPI>
-__global__ void __launch_bounds__(THREADS, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-              const GParams p) {
-  extern __shared__ uint8_t smem_raw[];
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = (raw + 1023u) & ~1023u;
-  uint8_t* gbase = smem_raw + (base - raw);
-  uint8_t* misc = gbase + STAGES * STAGE_BYTES;
-  const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES;
-  const uint32_t bAcc = bEmpty + 8 * STAGES, bReg = bAcc + 16, bFinal = bReg + 16;
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
-
-  const int per_cell = p.mtiles * p.ntiles;
-  const int n_tiles = p.cells * per_cell;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(bFull + 8 * s, 1);
-      mbar_init(bEmpty + 8 * s, 1);
-    }
-    mbar_init(bAcc, 1);
-    mbar_init(bAcc + 8, 1);
-    mbar_init(bReg, 32 * NUM_EPI_WARPS);
-    mbar_init(bReg + 8, 32 * NUM_EPI_WARPS);
-    mbar_init(bFinal, 1);
-    *abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  }
-  if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
-        smem_u32((const void*)tmem_slot)));
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint32_t b_bytes = p.b_mn ? (uint32_t)((p.BN / 64) * MN_BOX_BYTES) : (uint32_t)(p.BN * 128);
-
-  if (warp == 0) {
-    if (lane == 0) {
-      int issued[STAGES] = {0, 0, 0, 0};
-      bool ok = true;
-      int stage = 0;
-      uint32_t phase = 0;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const int cell = tile / per_cell, rem = tile % per_cell;
-        const int m0 = (rem / p.ntiles) * BM, n0 = (rem % p.ntiles) * p.BN;
-        const int za = p.a_sel ? __ldg(&p.a_sel[cell]) : cell;
-        const int zb = p.b_sel ? __ldg(&p.b_sel[cell]) : cell;
-        for (int kc = 0; kc < p.kchunks; ++kc) {
-          if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 11)) {
-            ok = false;
-            break;
-          }
-          const uint32_t full = bFull + 8 * stage;
-          mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
-          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
-          if (p.a_mn) {
-            tma_load_3d(sA, &mA, full, m0, kc * BK, za);
-            tma_load_3d(sA + MN_BOX_BYTES, &mA, full, m0 + 64, kc * BK, za);
-          } else {
-            tma_load_3d(sA, &mA, full, kc * BK, p.a_row0 + m0, za);
-          }
-          if (p.b_mn) {
-            for (int i = 0; i < p.BN / 64; ++i)
-              tma_load_3d(sB + i * MN_BOX_BYTES, &mB, full, n0 + 64 * i, kc * BK, zb);
-          } else {
-            tma_load_3d(sB, &mB, full, kc * BK, p.b_row0 + n0, zb);
-          }
-          issued[stage]++;
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1u;
-          }
-        }
-      }
-      if (!ok) {
-        for (int s = 0; s < STAGES; ++s)
-          if (issued[s] > 0) {
-            volatile int never = 0;
-            mbar_wait(bFull + 8 * s, (uint32_t)((issued[s] - 1) & 1), &never, p.err, 11);
-          }
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      int lt = 0;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++lt) {
-        const int rem = tile % per_cell;
-        const int n0 = (rem % p.ntiles) * p.BN;
-        int n = min(p.BN, p.N - n0);
-        n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
-        const int R = lt & 1, use = lt >> 1;
-        if (use > 0 &&
-            !mbar_wait(bReg + 8 * R, (uint32_t)((use - 1) & 1), abort_flag, p.err, 15)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(R * 256);
-        const uint32_t idesc = idesc_bf16_major(BM, n, p.a_mn, p.b_mn);
-        for (int kc = 0; kc < p.kchunks; ++kc) {
-          if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 12)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ad = p.a_mn ? sw128_mn_desc(sA + kk * 2048, MN_BOX_BYTES)
-                                       : sw128_desc(sA + kk * 32);
-            const uint64_t bd = p.b_mn ? sw128_mn_desc(sB + kk * 2048, MN_BOX_BYTES)
-                                       : sw128_desc(sB + kk * 32);
-            tc_mma(d, ad, bd, idesc, (kc | kk) != 0 ? 1u : 0u);
-          }
-          tc_commit(bEmpty + 8 * stage);
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1u;
-          }
-        }
-        if (!ok) break;
-        tc_commit(bAcc + 8 * R);
-      }
-      // every MMA issued here completes before the tensor memory is released
-      tc_commit(bFinal);
-      volatile int never = 0;
-      mbar_wait(bFinal, 0u, &never, p.err, 14);
-    }
-  } else {
-    const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
-    const int row = q * 32 + lane;
-    int lt = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++lt) {
-      const int cell = tile / per_cell, rem = tile % per_cell;
-      const int m0 = (rem / p.ntiles) * BM, n0 = (rem % p.ntiles) * p.BN;
-      int n = min(p.BN, p.N - n0);
-      n = p.b_mn ? (n + 63) & ~63 : (n + 15) & ~15;
-      const int R = lt & 1, use = lt >> 1;
-      if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(use & 1), abort_flag, p.err, 13)) break;
-      tc_fence_after();
-      const int m = m0 + row;
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
-      const int ng = n / 16;
-      const int half = (ng + 1) / 2;
-      const int g0 = hf ? half : 0, g1 = hf ? ng : half;
-      const bool row_ok = m < p.M;
-      const int arow = m < p.aux_wrap_at ? m : m - p.aux_wrap_sub;
-      for (int gi = g0; gi < g1; ++gi) {
-        uint32_t r[16];
-        LIPZ_TMEM_LD16(tbase + gi * 16, r);
-        tmem_wait_ld();
-        const int col0 = n0 + gi * 16;
-        if (!row_ok) continue;
-        if (EPI == EPI_F32) {
-          float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
-          if (p.scn == 1 && col0 + 16 <= p.N) {
-            float4* o = reinterpret_cast<float4*>(C + col0);
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-              o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
-                                 __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
-          } else {
-#pragma unroll
-            for (int e = 0; e < 16; ++e)
-              if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __uint_as_float(r[e]);
-          }
-        } else {
-          bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
-          const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
-          float v[16];
-          if (p.sxn == 1 && col0 + 16 <= p.N) {
-            const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
-            const uint4 q0 = __ldg(x4), q1 = __ldg(x4 + 1);
-            const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
-#pragma unroll
-            for (int e = 0; e < 16; e += 2) {
-              const __nv_bfloat162 y2 = *reinterpret_cast<const __nv_bfloat162*>(&w[e >> 1]);
-              v[e] = __uint_as_float(r[e]) * dact(p.act, __low2float(y2), p.slope);
-              v[e + 1] = __uint_as_float(r[e + 1]) * dact(p.act, __high2float(y2), p.slope);
-            }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 16; ++e) {
-              const int col = col0 + e;
-              const float y = col < p.N ? __bfloat162float(X[(int64_t)col * p.sxn]) : 0.f;
-              v[e] = __uint_as_float(r[e]) * dact(p.act, y, p.slope);
-            }
-          }
-          if (p.scn == 1 && col0 + 16 <= p.N) {
-            uint32_t pk[8];
-#pragma unroll
-            for (int e = 0; e < 16; e += 2) {
-              __nv_bfloat162 b2 = __floats2bfloat162_rn(v[e], v[e + 1]);
-              pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
-            }
-            uint4* o = reinterpret_cast<uint4*>(C + col0);
-            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 16; ++e)
-              if (col0 + e < p.N) C[(int64_t)(col0 + e) * p.scn] = __float2bfloat16_rn(v[e]);
-          }
-        }
-      }
-      tc_fence_before();
-      mbar_arrive(bReg + 8 * R);
-    }
-  }
-  __syncwarp();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
-  }
-}
-
 // ---------------------------------------------------------------------------------------------
 // The whole backward of one cell in one CTA: the nine products run as consecutive stages of a
 // single tile stream (double-buffered TMEM, one TMA ring). A stage that reads an earlier
@@ -723,14 +493,6 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (cudaFuncSetAttribute(tcb::k_gemm_tc<tcb::EPI_F32>,
-                           cudaFuncAttributeMaxDynamicSharedMemorySize, tcb::SMEM_BYTES) != cudaSuccess ||
-      cudaFuncSetAttribute(tcb::k_gemm_tc<tcb::EPI_DACT>,
-                           cudaFuncAttributeMaxDynamicSharedMemorySize, tcb::SMEM_BYTES) != cudaSuccess) {
-    cudaGetLastError();
-    if (msg) *msg = "cannot reserve shared memory for the tensor-core backward";
-    return nullptr;
-  }
   TcbPlan* P = new TcbPlan();
   memset(P, 0, sizeof *P);
   if (cudaMalloc(&P->err, 4) != cudaSuccess || cudaMemset(P->err, 0, 4) != cudaSuccess) {
@@ -963,22 +725,6 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     return nullptr;
   }
   return P;
-}
-
-int tcb_run(TcbPlan* P, int first, int count, cudaStream_t st, std::string* msg) {
-  for (int i = first; i < first + count && i < P->n; ++i) {
-    Gemm& G = P->g[i];
-    if (G.p.epi == tcb::EPI_DACT)
-      tcb::k_gemm_tc<tcb::EPI_DACT><<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
-    else
-      tcb::k_gemm_tc<tcb::EPI_F32><<<G.grid, tcb::THREADS, tcb::SMEM_BYTES, st>>>(G.a, G.b, G.p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) {
-      if (msg) *msg = std::string("tensor-core backward launch: ") + cudaGetErrorString(e);
-      return 1;
-    }
-  }
-  return 0;
 }
 
 int tcb_run_cells(TcbPlan* P, cudaStream_t st, std::string* msg) {

@@ -40,10 +40,8 @@ struct TcbPlan;
 // hidden == 256, z == 64, x a multiple of 16, 1 <= batch <= 256.
 bool tcb_supported(int z, int h, int x, int B);
 TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* msg);
-// Launches products [first, first + count) of the chain, in order: 0 D1, 1 dW2(D), 2 A3,
-// 3 dW1(D), 4 A2, 5 dW3(G), 6 A1, 7 dW2(G), 8 dW1(G).
-int tcb_run(TcbPlan* p, int first, int count, cudaStream_t st, std::string* msg);
-// All nine products of every cell in one launch (one CTA per cell, stages in the order above).
+// All nine products of every cell in one launch (one CTA per cell), as stages in the order
+// 0 D1, 1 dW2(D), 2 A3, 3 dW1(D), 4 A2, 5 dW3(G), 6 A1, 7 dW2(G), 8 dW1(G).
 int tcb_run_cells(TcbPlan* p, cudaStream_t st, std::string* msg);
 int* tcb_error_flag(TcbPlan* p);
 void tcb_plan_destroy(TcbPlan* p);
