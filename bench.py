@@ -110,6 +110,25 @@ class Clocks:
                 "samples": len(rows)}
 
 
+def allreduce_max(dist, x):
+    """Largest value of x over the ranks (CPU tensors under gloo, CUDA tensors under NCCL)."""
+    import torch
+    if dist is None:
+        return float(x)
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(ms_per_rank_max, steps, world):
+    """(ms per step, grid iterations / s, pair evaluations / s) of the whole job from the
+    slowest rank's time: every rank runs its own 12x12 grid, so the job's pairs are world x."""
+    ms_step = ms_per_rank_max / steps
+    iters_s = 1000.0 / ms_step
+    return ms_step, iters_s * world, PAIRS * world * iters_s
+
+
 def _dist():
     n = int(os.environ.get("WORLD_SIZE", "1"))
     if n > 1:
@@ -162,14 +181,7 @@ def run_ours(args):
     ms = e0.elapsed_time(e1)
     prof0 = L.lipz_profile_read(g.h)
     launches = sum(v[2] for v in prof0.values())
-    t_max = ms
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_max = float(t.item())
-    ms_step = t_max / args.steps
-    iters_s = 1000.0 / ms_step
-    value = PAIRS * world * iters_s
+    ms_step, iters_total, value = aggregate(allreduce_max(dist, ms), args.steps, world)
 
     # ---- per-phase device time (separate pass with phase events on the same stream)
     phase_ms = {k: float("nan") for k in L.PHASES}
@@ -202,7 +214,7 @@ def run_ours(args):
         "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
                    "pairs_per_iter": PAIRS, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (population 2.2 GB + pool 188 MB per iteration)"},
-        "grid_iterations_per_sec": iters_s * world,
+        "grid_iterations_per_sec": iters_total,
         "pair_evals_per_sec_eval_only": PAIRS * world * 1000.0 /
         (phase_ms["batch"] + phase_ms["g_fwd"] + phase_ms["d_fwd"] + phase_ms["fitness"]),
         "phase_ms": phase_ms,
@@ -233,11 +245,7 @@ def _e2e(args, L, g, torch, dist, world):
     t0 = time.perf_counter()
     for i in range(args.steps):
         L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
-    e2e_s = time.perf_counter() - t0
-    if dist:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = allreduce_max(dist, time.perf_counter() - t0)
     return PAIRS * world * args.steps / e2e_s
 
 

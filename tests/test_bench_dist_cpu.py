@@ -1,0 +1,50 @@
+"""The multi-rank reduction of bench.py on CPU: two gloo ranks, the job's numbers come from the
+slowest rank and count every rank's grid (replicas, weak scaling)."""
+
+import os
+import socket
+
+import pytest
+
+torch = pytest.importorskip("torch")
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    import bench
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    ms = 10.0 * (rank + 1)                     # rank 1 is the slow one
+    slowest = bench.allreduce_max(dist, ms)
+    q.put((rank, slowest, bench.aggregate(slowest, 4, world)))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_two_rank_reduction_takes_the_slowest_rank():
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    out = [q.get(timeout=120) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    import bench
+    for rank, slowest, (ms_step, iters, pairs) in out:
+        assert slowest == 20.0
+        assert ms_step == pytest.approx(5.0)
+        assert iters == pytest.approx(2 * 200.0)
+        assert pairs == pytest.approx(2 * 200.0 * bench.PAIRS)

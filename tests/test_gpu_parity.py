@@ -294,3 +294,46 @@ def test_full_size_12x12_bf16_sampled_cells(L):
     src = nbr[np.arange(144), sel["sel_g"]]
     ulp = 2 * np.spacing(np.float32(np.max(np.abs(s.Gw))))
     assert np.max(np.abs(got.Gw - s.Gw[src])) <= 2e-4 * (1 + 1e-5) + ulp
+
+
+def test_bf16_5x5_b256_fifty_iterations_sampled_lockstep(L):
+    """5x5 torus, bf16, B = 256, fifty grid iterations; at a sample of iterations the engine's
+    state is handed to the oracle and one full iteration is compared (the others run
+    unchecked, so drift of any kind accumulates into the checked ones)."""
+    pool = _pool(2, 60000, 784)
+    g = _grid(L, 5, 5, 50, pool, precision="bf16", batch=256, keep_grads=1)
+    checked = {0, 17, 49}
+    for it in range(50):
+        if it in checked:
+            _one_iteration_check(L, g, pool, 2e-2, kink_band=1e-3)
+        else:
+            g.iterate(1)
+    assert g.t == 50
+    s = _to_oracle(g, g.arch)
+    assert np.all(np.isfinite(s.Gw)) and np.all(np.isfinite(s.Dw))
+    assert np.all(s.Gstep >= 1) and np.all(s.Gstep <= 50)
+
+
+def test_large_grid_20x20_bf16_sampled(L):
+    """A 20x20 torus (400 cells, 10,000 pairs per iteration): sampled cells against the oracle,
+    then two iterations with bit-exact selection and bounded weight moves."""
+    pool = _pool(3, 60000, 784)
+    g = _grid(L, 20, 20, 7, pool, precision="bf16")
+    for _ in range(2):
+        s = _to_oracle(g, g.arch)
+        cells = [0, 19, 210, 399]
+        data = O.batches(s, pool, cells=cells)
+        ref = O.eval_neighborhoods(s, data, cells=cells)
+        ev = _check_eval(g, s, ref, 2e-2, cells=cells)
+        sel = g.select()
+        ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                       "fD": ev["fD"].astype(np.float64)})
+        assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+        assert np.array_equal(sel["sel_d"], ref_sel["sel_d"])
+        g.train()
+        got = _to_oracle(g, g.arch)
+        nbr = O.neighbors(20, 20)
+        src = nbr[np.arange(400), sel["sel_d"]]
+        lr = float(np.max(s.Dlr))
+        ulp = 2 * np.spacing(np.float32(np.max(np.abs(s.Dw))))
+        assert np.max(np.abs(got.Dw - s.Dw[src])) <= lr * (1 + 1e-5) + ulp
