@@ -319,7 +319,7 @@ def test_large_grid_20x20_bf16_sampled(L):
     then two iterations with bit-exact selection and bounded weight moves."""
     pool = _pool(3, 60000, 784)
     g = _grid(L, 20, 20, 7, pool, precision="bf16")
-    for _ in range(2):
+    for it in range(2):
         s = _to_oracle(g, g.arch)
         cells = [0, 19, 210, 399]
         data = O.batches(s, pool, cells=cells)
@@ -336,4 +336,8 @@ def test_large_grid_20x20_bf16_sampled(L):
         src = nbr[np.arange(400), sel["sel_d"]]
         lr = float(np.max(s.Dlr))
         ulp = 2 * np.spacing(np.float32(np.max(np.abs(s.Dw))))
-        assert np.max(np.abs(got.Dw - s.Dw[src])) <= lr * (1 + 1e-5) + ulp
+        # Adam moves an element by lr * |m_hat| / (sqrt(v_hat) + eps): at most lr on the first
+        # step, at most lr (1 - beta1) / sqrt(1 - beta2) (about 15.8 lr here) afterwards
+        bound = lr if it == 0 else lr * (1 - 0.5) / np.sqrt(1 - 0.999)
+        assert np.max(np.abs(got.Dw - s.Dw[src])) <= bound * (1 + 1e-5) + ulp
+        assert np.all(got.Dstep == s.Dstep[src] + 1)
