@@ -58,11 +58,30 @@ void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st) {
 // Rows go to E[c][b] (the first B rows of the cell's evaluation input).
 // ------------------------------------------------------------------------------------------
 template <typename T>
+__device__ __forceinline__ void store4(T* dst, float4 v);
+template <>
+__device__ __forceinline__ void store4<float>(float* dst, float4 v) {
+  *reinterpret_cast<float4*>(dst) = v;
+}
+template <>
+__device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+  uint2 pk;
+  pk.x = *reinterpret_cast<uint32_t*>(&lo);
+  pk.y = *reinterpret_cast<uint32_t*>(&hi);
+  *reinterpret_cast<uint2*>(dst) = pk;
+}
+
+// One warp per minibatch row: the row's pool index (one Philox word), a 16-byte-vector copy of
+// the row, then the row's normals, one Philox block (four normals) per lane at a time.
+template <typename T>
 __global__ void k_draw_batch(const float* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
                              T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
                              uint32_t t) {
-  const int b = blockIdx.x, c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
+  if (b >= B) return;
   const float* src;
   if (xin) {
     src = xin + ((int64_t)c * B + b) * x_dim;
@@ -72,14 +91,26 @@ __global__ void k_draw_batch(const float* __restrict__ pool, int64_t n_pool,
     src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
   }
   T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
-  for (int k = threadIdx.x; k < x_dim; k += blockDim.x) dst[k] = from_f<T>(src[k]);
+  const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
+  if (vec) {
+    for (int k = lane * 4; k < x_dim; k += 128)
+      store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
+  } else {
+    for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
+  }
   T* zr = Z + ((int64_t)c * B + b) * z_dim;
-  for (int d = threadIdx.x; d < z_dim; d += blockDim.x) {
-    const uint32_t n = (uint32_t)b * (uint32_t)z_dim + (uint32_t)d;
-    const U4 r = philox_block(seed, 4u, t, (uint32_t)c, n >> 2);
-    const int q = n & 3;
-    const float2 g = q < 2 ? box_muller(r.x, r.y) : box_muller(r.z, r.w);
-    zr[d] = from_f<T>((q & 1) ? g.y : g.x);
+  const uint32_t n0 = (uint32_t)b * (uint32_t)z_dim;
+  // normals n0 .. n0 + z_dim - 1; Philox block i holds normals 4i .. 4i + 3
+  for (uint32_t blk = (n0 >> 2) + lane; blk * 4 < n0 + (uint32_t)z_dim; blk += 32) {
+    const U4 r = philox_block(seed, 4u, t, (uint32_t)c, blk);
+    const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
+    const float v[4] = {g01.x, g01.y, g23.x, g23.y};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t n = blk * 4 + q;
+      if (n >= n0 && n < n0 + (uint32_t)z_dim) zr[n - n0] = from_f<T>(v[q]);
+    }
   }
 }
 
@@ -87,8 +118,8 @@ template <typename T>
 void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
                        cudaStream_t st) {
-  k_draw_batch<T><<<dim3(B, cells), 256, 0, st>>>(pool, n_pool, xin, E, e_cell, Z, B, x_dim,
-                                                  z_dim, seed, t);
+  k_draw_batch<T><<<dim3((B + 7) / 8, cells), 256, 0, st>>>(pool, n_pool, xin, E, e_cell, Z, B,
+                                                            x_dim, z_dim, seed, t);
 }
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
                                        float*, int, int, int, int, uint64_t, uint32_t,
@@ -232,37 +263,51 @@ template void launch_gemv<bf16>(const GemvDesc*, int, int, cudaStream_t);
 // ------------------------------------------------------------------------------------------
 template <typename T>
 __global__ void __launch_bounds__(256) k_colsum(const ColSumDesc* __restrict__ descs) {
+  // A block takes 256 columns of one problem: lane l owns columns 8l .. 8l + 7, warp w the
+  // rows w, w + 8, ...; the 8 partial sums of a column are added in a fixed order.
   const ColSumDesc d = descs[blockIdx.y];
   const int lane = threadIdx.x & 31, rg = threadIdx.x >> 5;
-  const int n = blockIdx.x * 64 + 2 * lane;
-  const T* x = (const T*)d.X;
-  float s0 = 0.f, s1 = 0.f;
-  if (n < d.cols) {
-    const bool pair = n + 1 < d.cols;
-#pragma unroll 4
+  const int n0 = blockIdx.x * 256 + lane * 8;
+  __shared__ float part[8][256];
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (n0 < d.cols) {
+    const T* x = (const T*)d.X;
+    const bool vec = sizeof(T) == 2 && n0 + 8 <= d.cols && (d.ld & 7) == 0 &&
+                     ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
     for (int r = rg; r < d.rows; r += 8) {
-      const T* p = x + (int64_t)r * d.ld + n;
-      s0 += to_f<T>(p[0]);
-      if (pair) s1 += to_f<T>(p[1]);
+      const T* p = x + (int64_t)r * d.ld + n0;
+      if (vec) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4*>(p));
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&w[e]);
+          acc[2 * e] += __low2float(v);
+          acc[2 * e + 1] += __high2float(v);
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (n0 + e < d.cols) acc[e] += to_f<T>(p[e]);
+      }
     }
   }
-  __shared__ float part[8][64];
-  part[rg][2 * lane] = s0;
-  part[rg][2 * lane + 1] = s1;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) part[rg][lane * 8 + e] = acc[e];
   __syncthreads();
-  if (threadIdx.x < 64) {
-    const int c = blockIdx.x * 64 + threadIdx.x;
+  const int col = blockIdx.x * 256 + threadIdx.x;
+  if (col < d.cols) {
     float t = 0.f;
 #pragma unroll
     for (int g = 0; g < 8; ++g) t += part[g][threadIdx.x];
-    if (c < d.cols) d.out[c] = t;
+    d.out[col] = t;
   }
 }
 
 template <typename T>
 void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st) {
   if (n_problems <= 0 || max_cols <= 0) return;
-  k_colsum<T><<<dim3((max_cols + 63) / 64, n_problems), 256, 0, st>>>(descs);
+  k_colsum<T><<<dim3((max_cols + 255) / 256, n_problems), 256, 0, st>>>(descs);
 }
 template void launch_colsum<float>(const ColSumDesc*, int, int, cudaStream_t);
 template void launch_colsum<bf16>(const ColSumDesc*, int, int, cudaStream_t);
@@ -335,7 +380,7 @@ __global__ void k_fitness(const float* __restrict__ logits, int B, float* __rest
 
 void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
                     float* fD, int* flag, cudaStream_t st) {
-  k_fitness<<<cells, 256, 0, st>>>(logits, B, LG, LD, fG, fD, flag);
+  k_fitness<<<cells, 960, 0, st>>>(logits, B, LG, LD, fG, fD, flag);  // one warp per mean
 }
 
 // ------------------------------------------------------------------------------------------
@@ -370,9 +415,11 @@ __global__ void k_select(const float* __restrict__ fG, const float* __restrict__
                          int* __restrict__ src_d, float* __restrict__ lr_g_new,
                          float* __restrict__ lr_d_new, float4* __restrict__ coef_g,
                          float4* __restrict__ coef_d) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  const int gid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = gid >> 1;
   if (c >= cells) return;
-  for (int pop = 0; pop < 2; ++pop) {
+  {
+    const int pop = gid & 1;
     const float* f5 = (pop ? fD : fG) + c * 5;
     const U4 a = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 0u);
     const U4 b = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 1u);
@@ -407,7 +454,7 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
                    int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
                    float4* coef_d, cudaStream_t st) {
-  k_select<<<(cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old,
+  k_select<<<(2 * cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old,
                                                 step_g_old, step_d_old, sel_g, sel_d, src_g, src_d,
                                                 lr_g_new, lr_d_new, coef_g, coef_d);
 }
@@ -457,11 +504,13 @@ __global__ void __launch_bounds__(1024) k_dlogit(
     int64_t wD_stride, int64_t off_w3, const int* __restrict__ src_d, int B, int H, float slope,
     T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride, int64_t off_gw3,
     int64_t off_gb3) {
-  extern __shared__ float dl[];            // [3B] deltas, then [4][H] partial sums
-  float* part = dl + 3 * B;
+  // Lanes own column groups of 8 (threads of the block: H / 8 groups x RG row groups); the RG
+  // partial sums of dW3 are added in a fixed order.
+  extern __shared__ float dl[];  // [3B] deltas, then [RG][H] partial sums
   const int c = blockIdx.x;
-  const int groups = blockDim.x / H;        // row groups (1..4)
-  const int k = threadIdx.x % H, rg = threadIdx.x / H;
+  const int ng = (H + 7) / 8;
+  const int RG = blockDim.x / ng;
+  float* part = dl + 3 * B;
   const float* l = TL + (int64_t)c * 2 * B;
   for (int r = threadIdx.x; r < 3 * B; r += blockDim.x) {
     const float x = r < 2 * B ? l[r] : l[r - B];
@@ -469,26 +518,60 @@ __global__ void __launch_bounds__(1024) k_dlogit(
     dl[r] = (r < B || r >= 2 * B) ? (s - 1.f) / (float)B : s / (float)B;
   }
   __syncthreads();
+  const int gi = threadIdx.x % ng, rg = threadIdx.x / ng;
+  const int k0 = gi * 8;
   const T* w3 = wD + (int64_t)src_d[c] * wD_stride + off_w3;
   const T* g2 = TG2 + (int64_t)c * 2 * B * H;
   T* j2 = J2 + (int64_t)c * 3 * B * H;
-  float acc = 0.f;
-  if (rg < groups) {
-    const float wk = to_f<T>(w3[k]);
-    for (int r = rg; r < 3 * B; r += groups) {
+  float wk[8], acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    wk[e] = k0 + e < H ? to_f<T>(w3[k0 + e]) : 0.f;
+    acc[e] = 0.f;
+  }
+  if (rg < RG) {
+    const bool vec = sizeof(T) == 2 && (H & 7) == 0;
+    for (int r = rg; r < 3 * B; r += RG) {
       const int rr = r < 2 * B ? r : r - B;
-      const float gv = to_f<T>(g2[(int64_t)rr * H + k]);
-      j2[(int64_t)r * H + k] = from_f<T>(dl[r] * wk * (gv > 0.f ? 1.f : slope));
-      if (r < 2 * B) acc = fmaf(dl[r], gv, acc);
+      const float dr = dl[r];
+      if (vec) {
+        // eight bf16 columns in one 16-byte load and store
+        const uint4 q = *reinterpret_cast<const uint4*>(g2 + (int64_t)rr * H + k0);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&w[e]);
+          const float g0 = __low2float(v), g1 = __high2float(v);
+          __nv_bfloat162 y = __floats2bfloat162_rn(dr * wk[2 * e] * (g0 > 0.f ? 1.f : slope),
+                                                   dr * wk[2 * e + 1] * (g1 > 0.f ? 1.f : slope));
+          o[e] = *reinterpret_cast<uint32_t*>(&y);
+          if (r < 2 * B) {
+            acc[2 * e] = fmaf(dr, g0, acc[2 * e]);
+            acc[2 * e + 1] = fmaf(dr, g1, acc[2 * e + 1]);
+          }
+        }
+        *reinterpret_cast<uint4*>(j2 + (int64_t)r * H + k0) = make_uint4(o[0], o[1], o[2], o[3]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          if (k0 + e >= H) break;
+          const float gv = to_f<T>(g2[(int64_t)rr * H + k0 + e]);
+          j2[(int64_t)r * H + k0 + e] = from_f<T>(dr * wk[e] * (gv > 0.f ? 1.f : slope));
+          if (r < 2 * B) acc[e] = fmaf(dr, gv, acc[e]);
+        }
+      }
     }
-    part[rg * H + k] = acc;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (k0 + e < H) part[rg * H + k0 + e] = acc[e];
   }
   __syncthreads();
   float* g = gD + (int64_t)c * gD_stride;
-  if (threadIdx.x < H) {
+  for (int k = threadIdx.x; k < H; k += blockDim.x) {
     float t = 0.f;
-    for (int q = 0; q < groups; ++q) t += part[q * H + threadIdx.x];
-    g[off_gw3 + threadIdx.x] = t;
+    for (int q = 0; q < RG; ++q) t += part[q * H + k];
+    g[off_gw3 + k] = t;
   }
   if (threadIdx.x == 0) {
     float t = 0.f;
@@ -501,11 +584,12 @@ template <typename T>
 void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
                    const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
                    int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st) {
-  int groups = 1024 / H;
-  if (groups > 4) groups = 4;
-  if (groups < 1) groups = 1;
-  const int threads = groups * H;
-  const size_t smem = (3 * (size_t)B + 4 * (size_t)H) * sizeof(float);
+  const int ng = (H + 7) / 8;
+  int rg = 512 / ng;
+  if (rg < 1) rg = 1;
+  if (rg > 16) rg = 16;
+  const int threads = ((rg * ng + 31) / 32) * 32;
+  const size_t smem = (3 * (size_t)B + (size_t)(threads / ng) * H) * sizeof(float);
   k_dlogit<T><<<cells, threads, smem, st>>>(TL, TG2, wD, wD_stride, off_w3, src_d, B, H, slope, J2,
                                             gD, gD_stride, off_gw3, off_gb3);
 }
