@@ -60,7 +60,7 @@ struct lipz_grid {
   std::string err;
 
   // data and work buffers
-  float* pool = nullptr;
+  void* pool = nullptr;  // [pool_n][x_dim] in the population precision
   int64_t pool_n = 0, pool_cap = 0;
   float* xin = nullptr;  // caller-supplied minibatch staging [cells][B][x_dim]
   void *Z = nullptr, *E = nullptr, *H1g = nullptr, *H2g = nullptr, *H1d = nullptr, *H2d = nullptr;
@@ -613,11 +613,11 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
   const int p = g->cur;
   phase_begin(g, LIPZ_PHASE_BATCH);
   if (g->bf)
-    launch_draw_batch<bf16>(g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell, (bf16*)g->Z, C,
-                            B, x, z, g->seed, (uint32_t)g->t, g->st);
+    launch_draw_batch<bf16>((const bf16*)g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell,
+                            (bf16*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, g->st);
   else
-    launch_draw_batch<float>(g->pool, g->pool_n, xin_dev, (float*)g->E, g->e_cell, (float*)g->Z,
-                             C, B, x, z, g->seed, (uint32_t)g->t, g->st);
+    launch_draw_batch<float>((const float*)g->pool, g->pool_n, xin_dev, (float*)g->E, g->e_cell,
+                             (float*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_BATCH, 1);
   if (g->use_tc) {
@@ -925,6 +925,7 @@ int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t 
     return fail(g, LIPZ_ERR_INVALID, "set_data needs a pool of 1..2^32-1 rows of x_dim=%d",
                 g->a.x_dim);
   CK(g, cudaStreamSynchronize(g->st));
+  const size_t n = (size_t)n_rows * dim;
   if (n_rows > g->pool_cap) {
     if (g->pool) {
       for (auto& p : g->allocs)
@@ -933,11 +934,25 @@ int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t 
       g->pool = nullptr;
       g->pool_cap = 0;
     }
-    int rc = dalloc(g, &g->pool, (size_t)n_rows * dim * 4);
+    int rc = dalloc(g, &g->pool, n * (g->bf ? 2 : 4));
     if (rc) return rc;
     g->pool_cap = n_rows;
   }
-  CK(g, cudaMemcpy(g->pool, host_pool, (size_t)n_rows * dim * 4, cudaMemcpyHostToDevice));
+  if (g->bf) {
+    // rounded once here: a drawn row is then the same bf16 row the fp32 pool would give
+    float* tmp = nullptr;
+    CK(g, cudaMalloc(&tmp, n * 4));
+    cudaError_t e = cudaMemcpy(tmp, host_pool, n * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) {
+      launch_to_bf16(tmp, (bf16*)g->pool, (int64_t)n, g->st);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
+    cudaFree(tmp);
+    CK(g, e);
+  } else {
+    CK(g, cudaMemcpy(g->pool, host_pool, n * 4, cudaMemcpyHostToDevice));
+  }
   g->pool_n = n_rows;
   return LIPZ_OK;
 }

@@ -47,7 +47,7 @@ void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout&
 void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st);
 
 template <typename T>
-void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
+void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
                        cudaStream_t st);
 

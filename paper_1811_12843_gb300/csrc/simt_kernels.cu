@@ -73,35 +73,56 @@ __device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
 }
 
 // One warp per minibatch row: the row's pool index (one Philox word), a 16-byte-vector copy of
-// the row, then the row's normals, one Philox block (four normals) per lane at a time.
+// the row, then the row's normals, one Philox block (four normals) per lane at a time. The pool
+// is held in the population's precision, so a drawn row is a plain copy; rows given by the
+// caller (xin, fp32) are rounded here.
 template <typename T>
-__global__ void k_draw_batch(const float* __restrict__ pool, int64_t n_pool,
+__global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
                              T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
                              uint32_t t) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
   if (b >= B) return;
-  const float* src;
+  T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
   if (xin) {
-    src = xin + ((int64_t)c * B + b) * x_dim;
+    const float* src = xin + ((int64_t)c * B + b) * x_dim;
+    const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
+    if (vec) {
+      for (int k = lane * 4; k < x_dim; k += 128)
+        store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
+    } else {
+      for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
+    }
   } else {
     const U4 r = philox_block(seed, 3u, t, (uint32_t)c, (uint32_t)(b >> 2));
     const uint32_t w = (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
-    src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
-  }
-  T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
-  const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
-                   ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
-  if (vec) {
-    for (int k = lane * 4; k < x_dim; k += 128)
-      store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
-  } else {
-    for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
+    const T* src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
+    const int bytes = x_dim * (int)sizeof(T);
+    if ((bytes & 15) == 0 &&
+        ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+      const int n4 = bytes >> 4;
+#pragma unroll 4
+      for (int k = lane; k < n4; k += 32) d4[k] = __ldg(s4 + k);
+    } else {
+      for (int k = lane; k < x_dim; k += 32) dst[k] = src[k];
+    }
   }
   T* zr = Z + ((int64_t)c * B + b) * z_dim;
   const uint32_t n0 = (uint32_t)b * (uint32_t)z_dim;
   // normals n0 .. n0 + z_dim - 1; Philox block i holds normals 4i .. 4i + 3
+  if ((z_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(zr) & (4 * sizeof(T) - 1)) == 0)) {
+    // every block lies inside the row and its four normals are one aligned vector
+    for (int k = lane * 4; k < z_dim; k += 128) {
+      const U4 r = philox_block(seed, 4u, t, (uint32_t)c, (n0 + (uint32_t)k) >> 2);
+      const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
+      store4<T>(zr + k, make_float4(g01.x, g01.y, g23.x, g23.y));
+    }
+    return;
+  }
   for (uint32_t blk = (n0 >> 2) + lane; blk * 4 < n0 + (uint32_t)z_dim; blk += 32) {
     const U4 r = philox_block(seed, 4u, t, (uint32_t)c, blk);
     const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
@@ -115,7 +136,7 @@ __global__ void k_draw_batch(const float* __restrict__ pool, int64_t n_pool,
 }
 
 template <typename T>
-void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
+void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
                        cudaStream_t st) {
   k_draw_batch<T><<<dim3((B + 7) / 8, cells), 256, 0, st>>>(pool, n_pool, xin, E, e_cell, Z, B,
@@ -124,7 +145,7 @@ void launch_draw_batch(const float* pool, int64_t n_pool, const float* xin, T* E
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
                                        float*, int, int, int, int, uint64_t, uint32_t,
                                        cudaStream_t);
-template void launch_draw_batch<bf16>(const float*, int64_t, const float*, bf16*, int64_t, bf16*,
+template void launch_draw_batch<bf16>(const bf16*, int64_t, const float*, bf16*, int64_t, bf16*,
                                       int, int, int, int, uint64_t, uint32_t, cudaStream_t);
 
 // ------------------------------------------------------------------------------------------
