@@ -597,6 +597,24 @@ int create_impl(lipz_grid* g) {
       b.doff = g->ld.off;
       b.src_g = g->src_g;
       b.src_d = g->src_d;
+      // without keep_grads the weight matrices take their Adam step inside the backward
+      b.fuse_adam = g->a.keep_grads ? 0 : 1;
+      const PopView* pops[2][2] = {{&g->G[p], &g->G[1 - p]}, {&g->D[p], &g->D[1 - p]}};
+      TcbBuffers::AdamPop* ap[2] = {&b.adam_g, &b.adam_d};
+      for (int q = 0; q < 2; ++q) {
+        ap[q]->w = pops[q][0]->w;
+        ap[q]->m = pops[q][0]->m;
+        ap[q]->v = pops[q][0]->v;
+        ap[q]->w_new = pops[q][1]->w;
+        ap[q]->m_new = pops[q][1]->m;
+        ap[q]->v_new = pops[q][1]->v;
+        ap[q]->wb_new = pops[q][1]->wb;
+      }
+      b.adam_g.coef = g->coef_g;
+      b.adam_d.coef = g->coef_d;
+      b.beta1 = g->a.beta1;
+      b.beta2 = g->a.beta2;
+      b.eps = g->a.eps;
       std::string msg;
       g->tcb[p] = tcb_plan_create(s, b, &msg);
       if (!g->tcb[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core backward plan: %s", msg.c_str());
@@ -723,6 +741,39 @@ int train_impl(lipz_grid* g) {
     colsum(g, D.cb_all, 5 * C, h > x ? h : x);
     CKL(g);
     phase_end(g, LIPZ_PHASE_TRAIN_BWD, 3);
+    if (!g->a.keep_grads) {
+      // the weight matrices took their Adam step inside the backward: the biases and D's
+      // output layer remain
+      phase_begin(g, LIPZ_PHASE_ADAM);
+      AdamRanges rg{}, rd{};
+      rg.old_p = g->G[p];
+      rg.new_p = g->G[1 - p];
+      rg.grad = g->gG;
+      rg.src = g->src_g;
+      rg.coef = g->coef_g;
+      rg.Ps = g->PGs;
+      rd.old_p = g->D[p];
+      rd.new_p = g->D[1 - p];
+      rd.grad = g->gD;
+      rd.src = g->src_d;
+      rd.coef = g->coef_d;
+      rd.Ps = g->PDs;
+      for (int k : {1, 3, 5}) {
+        rg.off[rg.n] = g->lg.off[k];
+        rg.len[rg.n++] = (int)(g->lg.off[k + 1] - g->lg.off[k]);
+      }
+      for (int k : {1, 3, 4, 5}) {
+        rd.off[rd.n] = g->ld.off[k];
+        rd.len[rd.n++] = (int)(g->ld.off[k + 1] - g->ld.off[k]);
+      }
+      launch_adam_ranges(rg, rd, C, g->a.beta1, g->a.beta2, g->a.eps, g->st);
+      CKL(g);
+      phase_end(g, LIPZ_PHASE_ADAM, 1);
+      g->cur = 1 - p;
+      g->t += 1;
+      g->phase = PH_IDLE;
+      return LIPZ_OK;
+    }
     if (!g->prof) {
       // The discriminator's Adam runs on the side stream, overlapping the generator's Adam and
       // the next evaluation's generator kernel; the grid's stream waits for it before anything

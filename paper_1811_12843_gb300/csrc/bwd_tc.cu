@@ -7,6 +7,10 @@
 // delta^T X and delta W, so no transposed copy is ever written). Epilogues: fp32 store
 // (weight gradients) or bf16 delta times the activation derivative read from the stored
 // forward output. The z coordinate of a weight operand is the cell's selected individual.
+// A weight-gradient tile can instead apply Adam on the spot (EPI_ADAM): the gradient never
+// leaves the accumulator. A loader warp streams the selected individual's old weights and
+// moments by TMA into shared memory, 32 columns at a time, while the epilogue turns the
+// previous chunk into the cell's new weights, moments and bf16 copy.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -23,16 +27,39 @@ using namespace lipz::tc;
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;        // 16 KB
 constexpr int B_BYTES = 256 * BK * 2;       // 32 KB (BN <= 256)
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int MN_BOX_BYTES = 64 * BK * 2;   // one {64 MN, 64 K} box
 constexpr int NUM_EPI_WARPS = 8;
-constexpr int THREADS = 64 + 32 * NUM_EPI_WARPS;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;  // one CTA per SM
+constexpr int EPI_THREADS = 32 * NUM_EPI_WARPS;
+// fused Adam: a chunk is 128 rows x 32 fp32 columns of each of w, m, v (one 128-byte row each,
+// 128-byte swizzle), updated in place, plus the new bf16 copy (64-byte rows, no swizzle)
+constexpr int ADAM_COLS = 32;
+constexpr int ADAM_ARRAY_BYTES = BM * ADAM_COLS * 4;                   // 16 KB
+constexpr int ADAM_WB_BYTES = BM * ADAM_COLS * 2;                      // 8 KB
+constexpr int ADAM_BUF_BYTES = 3 * ADAM_ARRAY_BYTES + ADAM_WB_BYTES;   // 56 KB
 
-enum { EPI_F32 = 0, EPI_DACT = 1 };
+// Without fused Adam: four operand stages. With it: two operand stages, two Adam chunk
+// buffers and one more warp (the Adam loader). One CTA per SM either way.
+template <bool FUSED>
+struct Cfg {
+  static constexpr int STAGES = FUSED ? 2 : 4;
+  static constexpr int ADAM_BUFS = FUSED ? 2 : 0;
+  static constexpr int THREADS = 64 + EPI_THREADS + (FUSED ? 32 : 0);
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + ADAM_BUFS * ADAM_BUF_BYTES + 256;
+};
+
+enum { EPI_F32 = 0, EPI_DACT = 1, EPI_ADAM = 2 };
+
+// Adam of one weight tensor fused into the tile that computes its gradient (Section 3, step 3:
+// the selected individual of the cell takes one Adam step and becomes the cell's new centre).
+// The old snapshot is read and the new one written through the stage's tensor maps.
+struct AdamRef {
+  const int* src;                  // individual each cell trains
+  const float4* coef;              // per cell: lr, 1 / (1 - beta1^t), 1 / (1 - beta2^t), t
+  float beta1, beta2, eps;
+};
 
 struct GParams {
   int cells;
@@ -49,6 +76,7 @@ struct GParams {
   const bf16* aux;
   int64_t aux_cell, sxm, sxn;
   int aux_wrap_at, aux_wrap_sub;  // aux row of m: m < wrap_at ? m : m - wrap_sub
+  AdamRef adam;
   int* err;
 };
 
@@ -87,6 +115,9 @@ struct CellPlan {
 struct StageMaps {
   CUtensorMap a[MAX_STAGES];
   CUtensorMap b[MAX_STAGES];
+  CUtensorMap aw[MAX_STAGES], am[MAX_STAGES], av[MAX_STAGES];  // old w, m, v (EPI_ADAM stages)
+  CUtensorMap nw[MAX_STAGES], nm[MAX_STAGES], nv[MAX_STAGES];  // new w, m, v
+  CUtensorMap nb[MAX_STAGES];                                  // new bf16 copy
 };
 
 __device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int& n0, int& n) {
@@ -188,16 +219,99 @@ __device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0
   }
 }
 
-__global__ void __launch_bounds__(THREADS, 1)
+// Adam epilogue of one weight-gradient tile: for each 32-column chunk, the warp's 16 columns
+// of its row. The chunk's old w, m, v sit in buffer `abuf` as three 128 x 128-byte boxes in the
+// 128-byte swizzle (16-byte unit u of row r at unit u ^ (r & 7)); the new values go back to the
+// same places, the bf16 copy to the buffer's 64-byte-row box, and the loader warp stores the
+// four boxes once every epilogue thread has arrived on aDone. Returns false on a timeout.
+__device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, int n0,
+                                          uint32_t tbase, int hf, int row, uint32_t sAdam,
+                                          uint32_t aFull, uint32_t aDone, int& abuf,
+                                          uint32_t& aph, volatile int* abort_flag, int* err) {
+  const AdamRef& a = p.adam;
+  const float4 cf = __ldg(&a.coef[cell]);
+  const bool row_ok = m0 + row < p.M;
+  const int nch = (min(p.BN, p.N - n0) + ADAM_COLS - 1) / ADAM_COLS;
+  for (int k = 0; k < nch; ++k) {
+    if (!mbar_wait_warp(aFull + 8 * abuf, aph, abort_flag, err, 18)) return false;
+    const int cl = k * ADAM_COLS + 16 * hf;  // first column of this thread, within the tile
+    const uint32_t bb = sAdam + (uint32_t)(abuf * ADAM_BUF_BYTES);
+    const uint32_t rb = bb + (uint32_t)row * 128u;
+    // the TMEM load is warp-collective: every lane takes part, live row or not
+    uint32_t r[16];
+    LIPZ_TMEM_LD16(tbase + cl, r);
+    tmem_wait_ld();
+    if (row_ok && n0 + cl < p.N) {
+      float w[16], mm[16], v[16];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (row & 7)) << 4);
+        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                     : "=f"(w[4 * u]), "=f"(w[4 * u + 1]), "=f"(w[4 * u + 2]), "=f"(w[4 * u + 3])
+                     : "r"(rb + off)
+                     : "memory");
+        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                     : "=f"(mm[4 * u]), "=f"(mm[4 * u + 1]), "=f"(mm[4 * u + 2]),
+                       "=f"(mm[4 * u + 3])
+                     : "r"(rb + ADAM_ARRAY_BYTES + off)
+                     : "memory");
+        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                     : "=f"(v[4 * u]), "=f"(v[4 * u + 1]), "=f"(v[4 * u + 2]), "=f"(v[4 * u + 3])
+                     : "r"(rb + 2 * ADAM_ARRAY_BYTES + off)
+                     : "memory");
+      }
+#pragma unroll
+      for (int e = 0; e < 16; ++e)
+        adam_elem(w[e], mm[e], v[e], __uint_as_float(r[e]), a.beta1, a.beta2, cf.x, cf.y, cf.z,
+                  a.eps);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (row & 7)) << 4);
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(rb + off), "f"(w[4 * u]),
+                     "f"(w[4 * u + 1]), "f"(w[4 * u + 2]), "f"(w[4 * u + 3])
+                     : "memory");
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(rb + ADAM_ARRAY_BYTES + off),
+                     "f"(mm[4 * u]), "f"(mm[4 * u + 1]), "f"(mm[4 * u + 2]), "f"(mm[4 * u + 3])
+                     : "memory");
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(rb + 2 * ADAM_ARRAY_BYTES +
+                                                                      off),
+                     "f"(v[4 * u]), "f"(v[4 * u + 1]), "f"(v[4 * u + 2]), "f"(v[4 * u + 3])
+                     : "memory");
+      }
+      const uint32_t wbr = bb + 3 * ADAM_ARRAY_BYTES + (uint32_t)row * 64u + (uint32_t)hf * 32u;
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(wbr),
+                   "r"(pack_bf16(w[0], w[1])), "r"(pack_bf16(w[2], w[3])),
+                   "r"(pack_bf16(w[4], w[5])), "r"(pack_bf16(w[6], w[7]))
+                   : "memory");
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(wbr + 16),
+                   "r"(pack_bf16(w[8], w[9])), "r"(pack_bf16(w[10], w[11])),
+                   "r"(pack_bf16(w[12], w[13])), "r"(pack_bf16(w[14], w[15]))
+                   : "memory");
+    }
+    // make the new values visible to the TMA store, then hand the chunk to the loader warp
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    mbar_arrive(aDone + 8 * abuf);
+    abuf ^= 1;
+    if (abuf == 0) aph ^= 1u;
+  }
+  return true;
+}
+
+template <bool FUSED>
+__global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     k_bwd_cells(const __grid_constant__ StageMaps maps, const __grid_constant__ CellPlan cp) {
+  constexpr int STAGES = Cfg<FUSED>::STAGES;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  uint8_t* misc = gbase + STAGES * STAGE_BYTES;
+  const uint32_t sAdam = base + STAGES * STAGE_BYTES;  // [ADAM_BUFS][w | m | v] chunks
+  uint8_t* misc = gbase + STAGES * STAGE_BYTES + Cfg<FUSED>::ADAM_BUFS * ADAM_BUF_BYTES;
   const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES;
   const uint32_t bAcc = bEmpty + 8 * STAGES, bReg = bAcc + 16, bFinal = bReg + 16;
-  const uint32_t bEpi = bFinal + 8;  // [2], alternating by tile
+  const uint32_t bEpi = bFinal + 8;    // [2], alternating by tile
+  const uint32_t aFull = bEpi + 16;   // [2] Adam chunk buffers: old values landed
+  const uint32_t aDone = aFull + 16;  // [2] new values written back by the epilogue
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
   volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 200);
@@ -210,11 +324,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     mbar_init(bAcc, 1);
     mbar_init(bAcc + 8, 1);
-    mbar_init(bReg, 32 * NUM_EPI_WARPS);
-    mbar_init(bReg + 8, 32 * NUM_EPI_WARPS);
+    mbar_init(bReg, EPI_THREADS);
+    mbar_init(bReg + 8, EPI_THREADS);
     mbar_init(bFinal, 1);
-    mbar_init(bEpi, 32 * NUM_EPI_WARPS);
-    mbar_init(bEpi + 8, 32 * NUM_EPI_WARPS);
+    mbar_init(bEpi, EPI_THREADS);
+    mbar_init(bEpi + 8, EPI_THREADS);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(aFull + 8 * b, 1);
+      mbar_init(aDone + 8 * b, EPI_THREADS);
+    }
     *abort_flag = 0;
     *done_tiles = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -233,7 +351,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued[STAGES] = {0, 0, 0, 0};
+      int issued[STAGES] = {};
       bool ok = true;
       int stage = 0;
       uint32_t phase = 0;
@@ -363,11 +481,82 @@ __global__ void __launch_bounds__(THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, err, 14);
     }
+  } else if (FUSED && warp == 2 + NUM_EPI_WARPS) {
+    // ===== Adam loader: old w, m, v of every chunk of every EPI_ADAM tile, in tile order, and
+    // the TMA stores of each chunk's new w, m, v and bf16 copy once the epilogue is done =====
+    if (lane == 0) {
+      int buf = 0, issued[2] = {0, 0};
+      int pend_si[2] = {0, 0}, pend_x[2] = {0, 0}, pend_m[2] = {0, 0}, pend_c[2] = {0, 0};
+      bool has[2] = {false, false};
+      bool ok = true;
+      // store the chunk held by buffer b once the epilogue has written it back
+      auto flush = [&](int b) -> bool {
+        if (!mbar_wait(aDone + 8 * b, (uint32_t)((issued[b] - 1) & 1), abort_flag, err, 19))
+          return false;
+        const int si = pend_si[b];
+        const uint32_t bb = sAdam + (uint32_t)(b * ADAM_BUF_BYTES);
+        tma_store_3d(&maps.nw[si], bb, pend_x[b], pend_m[b], pend_c[b]);
+        tma_store_3d(&maps.nm[si], bb + ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
+        tma_store_3d(&maps.nv[si], bb + 2 * ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
+        tma_store_3d(&maps.nb[si], bb + 3 * ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
+        bulk_commit();
+        has[b] = false;
+        return true;
+      };
+      for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
+        for (int si = 0; si < cp.n_stages && ok; ++si) {
+          const GParams& p = cp.st[si].p;
+          if (p.epi != EPI_ADAM) continue;
+          const int zi = __ldg(&p.adam.src[cell]);
+          const int nt = p.mtiles * p.ntiles;
+          for (int t = 0; t < nt && ok; ++t) {
+            const int m0 = (t / p.ntiles) * BM, n0 = (t % p.ntiles) * p.BN;
+            const int nch = (min(p.BN, p.N - n0) + ADAM_COLS - 1) / ADAM_COLS;
+            for (int k = 0; k < nch; ++k) {
+              if (has[buf]) {
+                if (!flush(buf)) {
+                  ok = false;
+                  break;
+                }
+                bulk_wait_read<0>();  // the stores have read the buffer: it may be refilled
+              }
+              const uint32_t full = aFull + 8 * buf;
+              mbar_expect_tx(full, (uint32_t)(3 * ADAM_ARRAY_BYTES));
+              const uint32_t dst = sAdam + (uint32_t)(buf * ADAM_BUF_BYTES);
+              const int x0 = n0 + k * ADAM_COLS;
+              tma_load_3d(dst, &maps.aw[si], full, x0, m0, zi);
+              tma_load_3d(dst + ADAM_ARRAY_BYTES, &maps.am[si], full, x0, m0, zi);
+              tma_load_3d(dst + 2 * ADAM_ARRAY_BYTES, &maps.av[si], full, x0, m0, zi);
+              issued[buf]++;
+              has[buf] = true;
+              pend_si[buf] = si;
+              pend_x[buf] = x0;
+              pend_m[buf] = m0;
+              pend_c[buf] = cell;
+              buf ^= 1;
+            }
+          }
+        }
+      }
+      // the last chunks (oldest first)
+      for (int i = 0; i < 2 && ok; ++i, buf ^= 1)
+        if (has[buf] && !flush(buf)) ok = false;
+      if (!ok) {
+        for (int b = 0; b < 2; ++b)
+          if (issued[b] > 0) {
+            volatile int never = 0;
+            mbar_wait(aFull + 8 * b, (uint32_t)((issued[b] - 1) & 1), &never, err, 19);
+          }
+      }
+      bulk_wait_all();
+    }
   } else {
     const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
     const int row = q * 32 + lane;
     bool ok = true;
     int lt = 0, pub = 0;
+    int abuf = 0;
+    uint32_t aph = 0;
     for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
       for (int si = 0; si < cp.n_stages && ok; ++si) {
         const GParams& p = cp.st[si].p;
@@ -383,7 +572,19 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
           const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
-          epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+          if constexpr (FUSED) {
+            if (p.epi == EPI_ADAM) {
+              if (!adam_tile(p, cell, m0, n0, tbase, hf, row, sAdam, aFull, aDone, abuf, aph,
+                             abort_flag, err)) {
+                ok = false;
+                break;
+              }
+            } else {
+              epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+            }
+          } else {
+            epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+          }
           if (publish) {
             // publish the tile's global stores to the async proxy (a later stage loads them by
             // TMA). The arrival on bEpi[pub & 1] comes before the arrival on bReg, so no thread
@@ -462,8 +663,46 @@ bool map3(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint6
   return true;
 }
 
+// fp32 3-D map over one weight tensor [out][in] of every individual: {in, out, individuals},
+// box {32, 128, 1} (one 128-byte row per output row), 128-byte swizzle.
+bool map3f(CUtensorMap* m, const float* base, uint64_t inner, uint64_t rows, uint64_t depth,
+           uint64_t depth_elems, std::string* msg) {
+  cuuint64_t dims[3] = {inner, rows, depth};
+  cuuint64_t strides[2] = {inner * 4, depth_elems * 4};
+  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::BM, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(base), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (fp32) failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
+// bf16 3-D map over one tensor's bf16 copy of every cell: {in, out, cells}, box {32, 128, 1},
+// no swizzle (64-byte rows).
+bool map3b_rows(CUtensorMap* m, const bf16* base, uint64_t inner, uint64_t rows, uint64_t depth,
+                uint64_t depth_elems, std::string* msg) {
+  cuuint64_t dims[3] = {inner, rows, depth};
+  cuuint64_t strides[2] = {inner * 2, depth_elems * 2};
+  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::BM, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<bf16*>(base), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (bf16 rows) failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
 struct Gemm {
   CUtensorMap a, b;
+  CUtensorMap aw, am, av;      // old w, m, v of the tensor (fused Adam), by individual
+  CUtensorMap nw, nm, nv, nb;  // new w, m, v and bf16 copy, by cell
   tcb::GParams p;
   int grid;
 };
@@ -478,6 +717,7 @@ struct TcbPlan {
   tcb::StageMaps maps;  // the same nine products as one per-cell kernel
   tcb::CellPlan cells;
   int grid_cells;
+  bool fused;  // weight tensors take their Adam step in the backward's epilogue
 };
 
 bool tcb_supported(int z, int h, int x, int B) {
@@ -527,6 +767,31 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     const int tiles = C * G.p.mtiles * G.p.ntiles;
     G.grid = tiles < sms ? tiles : sms;
   };
+  // weight-gradient stage of tensor `off` of a population: Adam in the epilogue when fused
+  // weight-gradient stage of the tensor at `off` of a population, whose gradient tile is
+  // [out = M][in = N] row-major (scm = N, scn = 1): Adam in the epilogue when fused
+  auto fuse = [&](Gemm& G, const TcbBuffers::AdamPop& a, const int* src, int64_t off,
+                  int64_t Ps) {
+    if (!b.fuse_adam) return;
+    if (G.p.scn != 1 || G.p.scm != G.p.N || G.p.N % 16 != 0 || off % 8 != 0 || Ps % 8 != 0) {
+      if (msg) *msg = "fused Adam needs 16-column tensors at 8-element offsets";
+      ok = false;
+      return;
+    }
+    G.p.epi = tcb::EPI_ADAM;
+    G.p.adam.src = src;
+    G.p.adam.coef = a.coef;
+    G.p.adam.beta1 = b.beta1;
+    G.p.adam.beta2 = b.beta2;
+    G.p.adam.eps = b.eps;
+    ok = ok && map3f(&G.aw, a.w + off, G.p.N, G.p.M, NI, Ps, msg) &&
+         map3f(&G.am, a.m + off, G.p.N, G.p.M, NI, Ps, msg) &&
+         map3f(&G.av, a.v + off, G.p.N, G.p.M, NI, Ps, msg) &&
+         map3f(&G.nw, a.w_new + off, G.p.N, G.p.M, C, Ps, msg) &&
+         map3f(&G.nm, a.m_new + off, G.p.N, G.p.M, C, Ps, msg) &&
+         map3f(&G.nv, a.v_new + off, G.p.N, G.p.M, C, Ps, msg) &&
+         map3b_rows(&G.nb, a.wb_new + off, G.p.N, G.p.M, C, Ps, msg);
+  };
 
   // 1. D1 = (J2 @ W2d) * lrelu'(TG1 rows r or r - B): M = 3B rows, N = 256, K = 256
   {
@@ -550,7 +815,8 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Dw + b.doff[2], h, h, NI, b.PDs, 64, msg);
     finish(G);
   }
-  // 2. dW2d^T[i][o] = sum_{r < 2B} TG1[r][i] J2[r][o]: M = i, N = o, K = 2B (TG1 ends at 2B)
+  // 2. dW2d[o][i] = sum_{r < 2B} J2[r][o] TG1[r][i]: M = o, N = i, K = 2B (TG1 ends at 2B).
+  //    An epilogue thread owns one output row o: 16 consecutive parameters per group.
   {
     Gemm& G = P->g[i++];
     G.p = base_params(h, h, 2 * B, 256);
@@ -559,10 +825,11 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.epi = tcb::EPI_F32;
     G.p.C = b.gD + b.doff[2];
     G.p.c_cell = b.PDs;
-    G.p.scm = 1;
-    G.p.scn = h;
-    ok = ok && map3(&G.a, b.TG1, h, 2 * B, C, (uint64_t)2 * B * h, 64, msg) &&
-         map3(&G.b, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg);
+    G.p.scm = h;
+    G.p.scn = 1;
+    fuse(G, b.adam_d, b.src_d, b.doff[2], b.PDs);
+    ok = ok && map3(&G.a, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg) &&
+         map3(&G.b, b.TG1, h, 2 * B, C, (uint64_t)2 * B * h, 64, msg);
     finish(G);
   }
   // 3. A3 = (D1[2B + r] @ W1d) * (1 - F^2): M = B, N = x (tiles of 256), K = 256
@@ -586,19 +853,21 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Dw + b.doff[0], x, h, NI, b.PDs, 64, msg);
     finish(G);
   }
-  // 4. dW1d^T[i][o] = sum_{r < 2B} TX[r][i] D1[r][o]: M = x, N = 256, K = 2B (TX ends at 2B)
+  // 4. dW1d[o][i] = sum_{r < 2B} D1[r][o] TX[r][i]: M = o = 256, N = i = x, K = 2B (TX ends
+  //    at 2B)
   {
     Gemm& G = P->g[i++];
-    G.p = base_params(x, h, 2 * B, 256);
+    G.p = base_params(h, x, 2 * B, 256);
     G.p.a_mn = 1;
     G.p.b_mn = 1;
     G.p.epi = tcb::EPI_F32;
     G.p.C = b.gD + b.doff[0];
     G.p.c_cell = b.PDs;
-    G.p.scm = 1;
-    G.p.scn = x;
-    ok = ok && map3(&G.a, b.TX, x, 2 * B, C, (uint64_t)2 * B * x, 64, msg) &&
-         map3(&G.b, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg);
+    G.p.scm = x;
+    G.p.scn = 1;
+    fuse(G, b.adam_d, b.src_d, b.doff[0], b.PDs);
+    ok = ok && map3(&G.a, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg) &&
+         map3(&G.b, b.TX, x, 2 * B, C, (uint64_t)2 * B * x, 64, msg);
     finish(G);
   }
   // 5. A2 = (A3 @ W3g) * relu'(TH2): M = B, N = 256, K = x
@@ -621,20 +890,20 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Gw + b.goff[4], h, x, NI, b.PGs, 64, msg);
     finish(G);
   }
-  // 6. dW3g^T[i][o] = sum_r TH2[r][i] A3[r][o]: M = 256 (i), N = x (o), K = B; the
-  //    transposed output makes a warp's stores contiguous
+  // 6. dW3g[o][i] = sum_r A3[r][o] TH2[r][i]: M = o = x, N = i = 256, K = B
   {
     Gemm& G = P->g[i++];
-    G.p = base_params(h, x, B, 256);
+    G.p = base_params(x, h, B, 256);
     G.p.a_mn = 1;
     G.p.b_mn = 1;
     G.p.epi = tcb::EPI_F32;
     G.p.C = b.gG + b.goff[4];
     G.p.c_cell = b.PGs;
-    G.p.scm = 1;
-    G.p.scn = h;
-    ok = ok && map3(&G.a, b.TH2, h, B, C, (uint64_t)B * h, 64, msg) &&
-         map3(&G.b, b.A3, x, B, C, (uint64_t)B * x, 64, msg);
+    G.p.scm = h;
+    G.p.scn = 1;
+    fuse(G, b.adam_g, b.src_g, b.goff[4], b.PGs);
+    ok = ok && map3(&G.a, b.A3, x, B, C, (uint64_t)B * x, 64, msg) &&
+         map3(&G.b, b.TH2, h, B, C, (uint64_t)B * h, 64, msg);
     finish(G);
   }
   // 7. A1 = (A2 @ W2g) * relu'(TH1): M = B, N = 256, K = 256
@@ -657,7 +926,7 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Gw + b.goff[2], h, h, NI, b.PGs, 64, msg);
     finish(G);
   }
-  // 8. dW2g^T[i][o] = sum_r TH1[r][i] A2[r][o]: M = 256 (i), N = 256 (o), K = B
+  // 8. dW2g[o][i] = sum_r A2[r][o] TH1[r][i]: M = o = 256, N = i = 256, K = B
   {
     Gemm& G = P->g[i++];
     G.p = base_params(h, h, B, 256);
@@ -666,10 +935,11 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.epi = tcb::EPI_F32;
     G.p.C = b.gG + b.goff[2];
     G.p.c_cell = b.PGs;
-    G.p.scm = 1;
-    G.p.scn = h;
-    ok = ok && map3(&G.a, b.TH1, h, B, C, (uint64_t)B * h, 64, msg) &&
-         map3(&G.b, b.A2, h, B, C, (uint64_t)B * h, 64, msg);
+    G.p.scm = h;
+    G.p.scn = 1;
+    fuse(G, b.adam_g, b.src_g, b.goff[2], b.PGs);
+    ok = ok && map3(&G.a, b.A2, h, B, C, (uint64_t)B * h, 64, msg) &&
+         map3(&G.b, b.TH1, h, B, C, (uint64_t)B * h, 64, msg);
     finish(G);
   }
   // 9. dW1g[o][i] = sum_r A1[r][o] Z[r][i]: M = 256 (o), N = z (i), K = B
@@ -683,6 +953,7 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.c_cell = b.PGs;
     G.p.scm = z;
     G.p.scn = 1;
+    fuse(G, b.adam_g, b.src_g, b.goff[0], b.PGs);
     ok = ok && map3(&G.a, b.A1, h, B, C, (uint64_t)B * h, 64, msg) &&
          map3(&G.b, b.Z, z, B, C, (uint64_t)B * z, 64, msg);
     finish(G);
@@ -698,6 +969,13 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
       const int nt = P->g[k].p.mtiles * P->g[k].p.ntiles;
       P->maps.a[k] = P->g[k].a;
       P->maps.b[k] = P->g[k].b;
+      P->maps.aw[k] = P->g[k].aw;
+      P->maps.am[k] = P->g[k].am;
+      P->maps.av[k] = P->g[k].av;
+      P->maps.nw[k] = P->g[k].nw;
+      P->maps.nm[k] = P->g[k].nm;
+      P->maps.nv[k] = P->g[k].nv;
+      P->maps.nb[k] = P->g[k].nb;
       P->cells.st[k].p = P->g[k].p;
       P->cells.st[k].dep = deps[k];
       P->cells.st[k].tile0 = tile0;
@@ -712,8 +990,15 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     P->cells.cells = C;
     P->cells.err = P->err;
     P->grid_cells = C < sms ? C : sms;
-    if (cudaFuncSetAttribute(tcb::k_bwd_cells, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tcb::SMEM_BYTES) != cudaSuccess) {
+    P->fused = b.fuse_adam != 0;
+    const cudaError_t e =
+        P->fused ? cudaFuncSetAttribute(tcb::k_bwd_cells<true>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        tcb::Cfg<true>::SMEM)
+                 : cudaFuncSetAttribute(tcb::k_bwd_cells<false>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        tcb::Cfg<false>::SMEM);
+    if (e != cudaSuccess) {
       cudaGetLastError();
       if (msg) *msg = "cannot reserve shared memory for the per-cell backward";
       ok = false;
@@ -728,7 +1013,13 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
 }
 
 int tcb_run_cells(TcbPlan* P, cudaStream_t st, std::string* msg) {
-  tcb::k_bwd_cells<<<P->grid_cells, tcb::THREADS, tcb::SMEM_BYTES, st>>>(P->maps, P->cells);
+  if (P->fused)
+    tcb::k_bwd_cells<true><<<P->grid_cells, tcb::Cfg<true>::THREADS, tcb::Cfg<true>::SMEM, st>>>(
+        P->maps, P->cells);
+  else
+    tcb::k_bwd_cells<false>
+        <<<P->grid_cells, tcb::Cfg<false>::THREADS, tcb::Cfg<false>::SMEM, st>>>(P->maps,
+                                                                                 P->cells);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     if (msg) *msg = std::string("per-cell backward launch: ") + cudaGetErrorString(e);

@@ -33,6 +33,17 @@ struct TcbBuffers {
   int64_t PGs, PDs;
   const int64_t *goff, *doff;
   const int *src_g, *src_d;
+  // fuse_adam != 0: the weight-gradient tiles apply Adam instead of storing the gradient (the
+  // biases and D's output layer stay in gG / gD). Per population: the old snapshot (read at
+  // src[cell]), the new one (written at the cell) and the per-cell coefficients.
+  int fuse_adam;
+  struct AdamPop {
+    const float *w, *m, *v;
+    float *w_new, *m_new, *v_new;
+    __nv_bfloat16* wb_new;
+    const float4* coef;
+  } adam_g, adam_d;
+  float beta1, beta2, eps;
 };
 
 struct TcbPlan;

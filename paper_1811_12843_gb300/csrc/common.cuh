@@ -93,6 +93,25 @@ __device__ __forceinline__ float act_bwd(int act, float y, float slope) {
   }
 }
 
+// One Adam step (Kingma & Ba 2015, Algorithm 1) of one parameter, the bias corrections folded
+// into ib1 = 1 / (1 - beta1^t) and ib2 = 1 / (1 - beta2^t). Every operation is spelled out (no
+// contraction left to the compiler), so the stand-alone Adam kernel and the Adam fused into
+// the tensor-core backward give the same bits for the same gradient. The square root and the
+// division of the step use the hardware approximations (a few ulp): the step is about lr in
+// size, so their error lies far below the fp32 rounding of the weight it is added to.
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float r;
+  asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ void adam_elem(float& w, float& m, float& v, float g, float b1,
+                                          float b2, float lr, float ib1, float ib2, float eps) {
+  m = __fmaf_rn(b1, m, __fmul_rn(1.f - b1, g));
+  v = __fmaf_rn(b2, v, __fmul_rn(__fmul_rn(1.f - b2, g), g));
+  const float den = __fadd_rn(sqrt_approx(__fmul_rn(v, ib2)), eps);
+  w = __fsub_rn(w, __fdividef(__fmul_rn(lr, __fmul_rn(m, ib1)), den));
+}
+
 // ---- grouped GEMM problem: C[m, n] = epi( sum_k A[m*sam + k*sak] * B[k*sbk + n*sbn] )
 // Epilogues: EPI_BIAS_ACT: act(acc + bias[n]);  EPI_DACT: acc * act_bwd(aux[m*sxm + n*sxn]);
 // EPI_STORE: acc. Element strides; pointers typed by the launch.

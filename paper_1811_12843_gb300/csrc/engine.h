@@ -79,4 +79,18 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
                  const float4* coef, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
                  float eps, cudaStream_t st);
 
+// Adam + replacement restricted to n parameter ranges [off[q], off[q] + len[q]) of every cell.
+struct AdamRanges {
+  PopView old_p, new_p;
+  const float* grad;
+  const int* src;
+  const float4* coef;
+  int64_t Ps;
+  int n;
+  int64_t off[8];
+  int len[8];
+};
+void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, float beta1,
+                        float beta2, float eps, cudaStream_t st);
+
 }  // namespace lipz

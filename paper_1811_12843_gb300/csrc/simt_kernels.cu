@@ -629,16 +629,10 @@ template void launch_dlogit<bf16>(const float*, const bf16*, const bf16*, int64_
 // ------------------------------------------------------------------------------------------
 __device__ __forceinline__ void adam4(float4& w, float4& m, float4& v, const float4 g, float b1,
                                       float b2, float lr, float ib1, float ib2, float eps) {
-  float* wv = &w.x;
-  float* mv = &m.x;
-  float* vv = &v.x;
-  const float* gv = &g.x;
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    mv[e] = b1 * mv[e] + (1.f - b1) * gv[e];
-    vv[e] = b2 * vv[e] + (1.f - b2) * gv[e] * gv[e];
-    wv[e] = wv[e] - lr * (mv[e] * ib1) / (sqrtf(vv[e] * ib2) + eps);
-  }
+  adam_elem(w.x, m.x, v.x, g.x, b1, b2, lr, ib1, ib2, eps);
+  adam_elem(w.y, m.y, v.y, g.y, b1, b2, lr, ib1, ib2, eps);
+  adam_elem(w.z, m.z, v.z, g.z, b1, b2, lr, ib1, ib2, eps);
+  adam_elem(w.w, m.w, v.w, g.w, b1, b2, lr, ib1, ib2, eps);
 }
 
 __global__ void __launch_bounds__(256) k_adam(PopView old_p, PopView new_p,
@@ -684,10 +678,8 @@ __global__ void __launch_bounds__(256) k_adam(PopView old_p, PopView new_p,
   // tail (P not a multiple of 4)
   if (blockIdx.x == 0 && threadIdx.x < (P & 3)) {
     const int64_t k = (n4 << 2) + threadIdx.x;
-    const float gk = grad[co + k];
-    const float mk = beta1 * old_p.m[so + k] + (1.f - beta1) * gk;
-    const float vk = beta2 * old_p.v[so + k] + (1.f - beta2) * gk * gk;
-    const float wk = old_p.w[so + k] - lr * (mk * ib1) / (sqrtf(vk * ib2) + eps);
+    float wk = old_p.w[so + k], mk = old_p.m[so + k], vk = old_p.v[so + k];
+    adam_elem(wk, mk, vk, grad[co + k], beta1, beta2, lr, ib1, ib2, eps);
     new_p.w[co + k] = wk;
     new_p.m[co + k] = mk;
     new_p.v[co + k] = vk;
@@ -705,6 +697,39 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
   if (per_cell < 1) per_cell = 1;
   dim3 grid(per_cell, cells);
   k_adam<<<grid, 256, 0, st>>>(old_p, new_p, grad, src, coef, P, Ps, beta1, beta2, eps);
+}
+
+// Adam + replacement of listed parameter ranges only (the tensors whose update is not fused
+// into the tensor-core backward: biases and D's output layer), both populations in one launch:
+// block (cell, population), one thread per parameter. Also writes the new snapshot's step and
+// learning rate.
+__global__ void __launch_bounds__(256) k_adam_ranges(AdamRanges r0, AdamRanges r1, float beta1,
+                                                      float beta2, float eps) {
+  const AdamRanges& r = blockIdx.y ? r1 : r0;
+  const int c = blockIdx.x;
+  const int s = r.src[c];
+  const float4 cf = r.coef[c];
+  if (threadIdx.x == 0) {
+    r.new_p.step[c] = (int)cf.w;
+    r.new_p.lr[c] = cf.x;
+  }
+  const int64_t so = (int64_t)s * r.Ps, co = (int64_t)c * r.Ps;
+  for (int q = 0; q < r.n; ++q) {
+    for (int i = threadIdx.x; i < r.len[q]; i += blockDim.x) {
+      const int64_t k = r.off[q] + i;
+      float w = r.old_p.w[so + k], m = r.old_p.m[so + k], v = r.old_p.v[so + k];
+      adam_elem(w, m, v, r.grad[co + k], beta1, beta2, cf.x, cf.y, cf.z, eps);
+      r.new_p.w[co + k] = w;
+      r.new_p.m[co + k] = m;
+      r.new_p.v[co + k] = v;
+      if (r.new_p.wb) r.new_p.wb[co + k] = __float2bfloat16_rn(w);
+    }
+  }
+}
+
+void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, float beta1,
+                        float beta2, float eps, cudaStream_t st) {
+  k_adam_ranges<<<dim3(cells, 2), 256, 0, st>>>(g, d, beta1, beta2, eps);
 }
 
 }  // namespace lipz

@@ -197,6 +197,21 @@ def test_one_iteration_bf16_5x5_b256(L):
     _one_iteration_check(L, g, pool, 2e-2, kink_band=1e-3)
 
 
+@pytest.mark.parametrize("rows,cols,batch", [(3, 3, 100), (2, 3, 129)])
+def test_fused_adam_equals_stored_gradient_path(L, rows, cols, batch):
+    """Unless the gradients are kept, the tensor-core backward applies Adam to the weight
+    matrices inside its epilogue (the gradient never leaves the accumulator). Its state after
+    every iteration must equal, bit for bit, the path that stores the gradients and runs the
+    separate Adam kernel (the one checked against the oracle above)."""
+    pool = _pool(9, 5000, 784)
+    a = _grid(L, rows, cols, 31, pool, precision="bf16", batch=batch)
+    b = _grid(L, rows, cols, 31, pool, precision="bf16", batch=batch, keep_grads=1)
+    for it in range(3):
+        a.iterate(1)
+        b.iterate(1)
+        assert a.export_state() == b.export_state(), it
+
+
 def test_selection_modes_and_mutation(L):
     pool = _pool(8, 4000, 784)
     g = _grid(L, 3, 4, 8, pool, keep_grads=1, tournament_size=5, replace_mode="always",
