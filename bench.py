@@ -43,11 +43,19 @@ EVAL_G_FLOP = 2 * CELLS * 5 * BATCH * G_MAC_ROW
 EVAL_D_FLOP = 2 * CELLS * 30 * BATCH * D_MAC_ROW
 PG = HIDDEN * Z_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + X_DIM * HIDDEN + X_DIM
 PD = HIDDEN * X_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + HIDDEN + 1
-# Adam + replacement per parameter: read w, m, v, g (16 B), write w, m, v (12 B) + bf16 copy (2 B)
-ADAM_BYTES = CELLS * (PG + PD) * 30
 # Training: forward of the selected pair (G layers 1-2 on B rows, D on 2B rows) and backward.
 TRAIN_FWD_FLOP = 2 * CELLS * BATCH * (Z_DIM * HIDDEN + HIDDEN * HIDDEN) + 2 * CELLS * 2 * BATCH * D_MAC_ROW
 TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
+# The backward kernel applies Adam to the weight matrices (G: W1, W2, W3; D: W1, W2) in its
+# epilogue: per such parameter it reads the old w, m, v (12 B) and writes the new w, m, v and
+# the bf16 copy (14 B). Its other algorithmic reads: the bf16 weights of the four matrices the
+# delta chain multiplies by (D: W2, W1; G: W3, W2) and the stored forward activations
+# (J2 3B x h, TG1 2B x h, TX 2B x x, TH1 and TH2 B x h, Z B x z), all bf16.
+W_FUSED = (Z_DIM * HIDDEN + HIDDEN * HIDDEN + X_DIM * HIDDEN) + (HIDDEN * X_DIM + HIDDEN * HIDDEN)
+BWD_ACT = (3 * BATCH * HIDDEN + 2 * BATCH * HIDDEN + 2 * BATCH * X_DIM + 2 * BATCH * HIDDEN
+           + BATCH * Z_DIM)
+TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN)
+                           + 2 * BWD_ACT)
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels, from
 # the ncu launch list in profiles/launches_12x12_bf16_iteration.md (same kernels as this build).
@@ -256,8 +264,9 @@ def _phase_roofs(phase_ms):
             "d_fwd": ("tensor", EVAL_D_FLOP,
                       "discriminator evaluation forward (all 720 slots, 3 fused layers + logit)"),
             "train_fwd": ("tensor", TRAIN_FWD_FLOP, "forward of every cell's selected pair"),
-            "train_bwd": ("tensor", TRAIN_BWD_FLOP, "backward of every cell's selected pair"),
-            "adam": ("hbm", ADAM_BYTES, "Adam + replacement (both populations)")}
+            "train_bwd": ("hbm", TRAIN_BWD_BYTES,
+                          "backward of every cell's selected pair with Adam + replacement of "
+                          "the weight matrices fused in (%.1f GFLOP)" % (TRAIN_BWD_FLOP / 1e9))}
     out = {}
     for ph, (bound, units, what) in work.items():
         t = phase_ms.get(ph)

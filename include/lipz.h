@@ -204,8 +204,10 @@ LIPZ_API int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d);
 /*
  * Per-phase device timing (tracing). Phases: LIPZ_PHASE_BATCH (minibatch draw), _G_FWD and
  * _D_FWD (evaluation forward of all generator / discriminator slots), _FITNESS (BCE losses and
- * fitness), _SELECT, _TRAIN_FWD (forward of the selected pairs), _TRAIN_BWD (their backward),
- * _ADAM (update and replacement). While enabled, every phase is bracketed by CUDA events on
+ * fitness), _SELECT, _TRAIN_FWD (forward of the selected pairs and the logit deltas),
+ * _TRAIN_BWD (their backward; on the tensor-core path one kernel, which also applies Adam to
+ * the weight matrices unless arch.keep_grads is set), _ADAM (bias gradients, then the rest of
+ * the update and replacement). While enabled, every phase is bracketed by CUDA events on
  * the grid's stream. lipz_profile_read waits for the stream and writes, per phase, the summed
  * device milliseconds (ms[n]), the number of phase executions (count[n]) and of kernel launches
  * (launches[n]) since the last read (any pointer may be null; n <= LIPZ_N_PHASES), then resets.

@@ -710,22 +710,21 @@ int train_impl(lipz_grid* g) {
     launch_train_prep<float>((const float*)g->E, g->e_cell, g->sel_g, (float*)g->TX, C, B, x,
                              g->st);
   // forward of the selected pair
+  int n_fwd = 1;
   if (g->use_tc) {
     std::string msg;
     if (tc_run_train_g(g->tc[p], g->st, &msg) || tc_run_train_d(g->tc[p], g->st, &msg))
       return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
-    phase_end(g, LIPZ_PHASE_TRAIN_FWD, 3);
+    n_fwd += 2;
   } else {
     gemm(g, D.tg1, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.tg2, C, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.td1, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemm(g, D.td2, C, 2 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemv(g, D.tgv, C, 2 * B);
-    phase_end(g, LIPZ_PHASE_TRAIN_FWD, 6);
+    n_fwd += 5;
   }
-  CKL(g);
-  phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
-  // logit deltas, then the discriminator's backward
+  // logit deltas (and D's output-layer gradient)
   if (g->bf)
     launch_dlogit<bf16>(g->TL, (const bf16*)g->TG2, g->D[p].wb, g->PDs, g->ld.off[4], g->src_d, C,
                         B, h, g->a.leaky_slope, (bf16*)g->J2, g->gD, g->PDs, g->ld.off[4],
@@ -734,17 +733,21 @@ int train_impl(lipz_grid* g) {
     launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
                          g->ld.off[5], g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_TRAIN_FWD, n_fwd + 1);
+  phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
   if (g->use_tcb) {
-    // the nine backward products of every cell in one launch, then the bias column sums
+    // the nine backward products of every cell in one launch (with Adam on the weight
+    // matrices unless the gradients are kept), then the bias column sums
     std::string msg;
     if (tcb_run_cells(g->tcb[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
-    colsum(g, D.cb_all, 5 * C, h > x ? h : x);
     CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 3);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 1);
+    phase_begin(g, LIPZ_PHASE_ADAM);
+    colsum(g, D.cb_all, 5 * C, h > x ? h : x);
     if (!g->a.keep_grads) {
       // the weight matrices took their Adam step inside the backward: the biases and D's
       // output layer remain
-      phase_begin(g, LIPZ_PHASE_ADAM);
       AdamRanges rg{}, rd{};
       rg.old_p = g->G[p];
       rg.new_p = g->G[1 - p];
@@ -768,7 +771,7 @@ int train_impl(lipz_grid* g) {
       }
       launch_adam_ranges(rg, rd, C, g->a.beta1, g->a.beta2, g->a.eps, g->st);
       CKL(g);
-      phase_end(g, LIPZ_PHASE_ADAM, 1);
+      phase_end(g, LIPZ_PHASE_ADAM, 2);
       g->cur = 1 - p;
       g->t += 1;
       g->phase = PH_IDLE;
@@ -778,7 +781,6 @@ int train_impl(lipz_grid* g) {
       // The discriminator's Adam runs on the side stream, overlapping the generator's Adam and
       // the next evaluation's generator kernel; the grid's stream waits for it before anything
       // reads the discriminator population again (join_side).
-      phase_begin(g, LIPZ_PHASE_ADAM);
       CK(g, cudaEventRecord(g->ev_fork, g->st));
       CK(g, cudaStreamWaitEvent(g->side, g->ev_fork, 0));
       launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs,
@@ -788,7 +790,7 @@ int train_impl(lipz_grid* g) {
       launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs,
                   g->a.beta1, g->a.beta2, g->a.eps, g->st);
       CKL(g);
-      phase_end(g, LIPZ_PHASE_ADAM, 2);
+      phase_end(g, LIPZ_PHASE_ADAM, 3);
       g->cur = 1 - p;
       g->t += 1;
       g->phase = PH_IDLE;
@@ -811,16 +813,16 @@ int train_impl(lipz_grid* g) {
     gemm(g, D.bw1g, C, h, z, EPI_STORE, ACT_NONE, true);
     colsum(g, D.cb1g, C, h);
     CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 17);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 16);
+    phase_begin(g, LIPZ_PHASE_ADAM);
   }
-  phase_begin(g, LIPZ_PHASE_ADAM);
-  // Adam + replacement into the other snapshot
+  // Adam + replacement into the other snapshot (after the bias sums on the tensor-core path)
   launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
   launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
   CKL(g);
-  phase_end(g, LIPZ_PHASE_ADAM, 2);
+  phase_end(g, LIPZ_PHASE_ADAM, g->use_tcb ? 3 : 2);
   g->cur = 1 - p;
   g->t += 1;
   g->phase = PH_IDLE;

@@ -33,19 +33,22 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int MN_BOX_BYTES = 64 * BK * 2;   // one {64 MN, 64 K} box
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int EPI_THREADS = 32 * NUM_EPI_WARPS;
-// fused Adam: a chunk is 128 rows x 32 fp32 columns of each of w, m, v (one 128-byte row each,
-// 128-byte swizzle), updated in place, plus the new bf16 copy (64-byte rows, no swizzle)
+// fused Adam: a chunk is 64 rows (one half of a tile) x 32 fp32 columns of each of w, m, v (one
+// 128-byte row each, 128-byte swizzle), updated in place, plus the new bf16 copy (64-byte rows,
+// no swizzle). Chunks alternate between the two row halves, so each half of the epilogue
+// works through its own two of the four buffers.
 constexpr int ADAM_COLS = 32;
-constexpr int ADAM_ARRAY_BYTES = BM * ADAM_COLS * 4;                   // 16 KB
-constexpr int ADAM_WB_BYTES = BM * ADAM_COLS * 2;                      // 8 KB
-constexpr int ADAM_BUF_BYTES = 3 * ADAM_ARRAY_BYTES + ADAM_WB_BYTES;   // 56 KB
+constexpr int ADAM_ROWS = 64;
+constexpr int ADAM_ARRAY_BYTES = ADAM_ROWS * ADAM_COLS * 4;            // 8 KB
+constexpr int ADAM_WB_BYTES = ADAM_ROWS * ADAM_COLS * 2;               // 4 KB
+constexpr int ADAM_BUF_BYTES = 3 * ADAM_ARRAY_BYTES + ADAM_WB_BYTES;   // 28 KB
 
-// Without fused Adam: four operand stages. With it: two operand stages, two Adam chunk
+// Without fused Adam: four operand stages. With it: two operand stages, four Adam chunk
 // buffers and one more warp (the Adam loader). One CTA per SM either way.
 template <bool FUSED>
 struct Cfg {
   static constexpr int STAGES = FUSED ? 2 : 4;
-  static constexpr int ADAM_BUFS = FUSED ? 2 : 0;
+  static constexpr int ADAM_BUFS = FUSED ? 4 : 0;
   static constexpr int THREADS = 64 + EPI_THREADS + (FUSED ? 32 : 0);
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + ADAM_BUFS * ADAM_BUF_BYTES + 256;
 };
@@ -219,24 +222,28 @@ __device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0
   }
 }
 
-// Adam epilogue of one weight-gradient tile: for each 32-column chunk, the warp's 16 columns
-// of its row. The chunk's old w, m, v sit in buffer `abuf` as three 128 x 128-byte boxes in the
-// 128-byte swizzle (16-byte unit u of row r at unit u ^ (r & 7)); the new values go back to the
-// same places, the bf16 copy to the buffer's 64-byte-row box, and the loader warp stores the
-// four boxes once every epilogue thread has arrived on aDone. Returns false on a timeout.
+// Adam epilogue of one weight-gradient tile: for each 32-column chunk of the thread's row half
+// h, the warp's 16 columns of its row. Chunk number cj of a half sits in buffer 2 (cj & 1) + h
+// (its (cj >> 1)-th use) as three 64 x 128-byte boxes of old w, m, v in the 128-byte swizzle
+// (16-byte unit u of box row r at unit u ^ (r & 7)); the new values go back to the same places,
+// the bf16 copy to the buffer's 64-byte-row box, and the loader warp stores the four boxes once
+// the half's 128 threads have arrived on aDone. Returns false on a timeout.
 __device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, int n0,
                                           uint32_t tbase, int hf, int row, uint32_t sAdam,
-                                          uint32_t aFull, uint32_t aDone, int& abuf,
-                                          uint32_t& aph, volatile int* abort_flag, int* err) {
+                                          uint32_t aFull, uint32_t aDone, int& cj,
+                                          volatile int* abort_flag, int* err) {
   const AdamRef& a = p.adam;
   const float4 cf = __ldg(&a.coef[cell]);
   const bool row_ok = m0 + row < p.M;
+  const int h = row / ADAM_ROWS, rr = row % ADAM_ROWS;
   const int nch = (min(p.BN, p.N - n0) + ADAM_COLS - 1) / ADAM_COLS;
-  for (int k = 0; k < nch; ++k) {
-    if (!mbar_wait_warp(aFull + 8 * abuf, aph, abort_flag, err, 18)) return false;
+  for (int k = 0; k < nch; ++k, ++cj) {
+    const int bi = 2 * (cj & 1) + h;
+    if (!mbar_wait_warp(aFull + 8 * bi, (uint32_t)((cj >> 1) & 1), abort_flag, err, 18))
+      return false;
     const int cl = k * ADAM_COLS + 16 * hf;  // first column of this thread, within the tile
-    const uint32_t bb = sAdam + (uint32_t)(abuf * ADAM_BUF_BYTES);
-    const uint32_t rb = bb + (uint32_t)row * 128u;
+    const uint32_t bb = sAdam + (uint32_t)(bi * ADAM_BUF_BYTES);
+    const uint32_t rb = bb + (uint32_t)rr * 128u;
     // the TMEM load is warp-collective: every lane takes part, live row or not
     uint32_t r[16];
     LIPZ_TMEM_LD16(tbase + cl, r);
@@ -245,7 +252,7 @@ __device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, in
       float w[16], mm[16], v[16];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (row & 7)) << 4);
+        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (rr & 7)) << 4);
         asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
                      : "=f"(w[4 * u]), "=f"(w[4 * u + 1]), "=f"(w[4 * u + 2]), "=f"(w[4 * u + 3])
                      : "r"(rb + off)
@@ -266,7 +273,7 @@ __device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, in
                   a.eps);
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (row & 7)) << 4);
+        const uint32_t off = (uint32_t)(((4 * hf + u) ^ (rr & 7)) << 4);
         asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(rb + off), "f"(w[4 * u]),
                      "f"(w[4 * u + 1]), "f"(w[4 * u + 2]), "f"(w[4 * u + 3])
                      : "memory");
@@ -278,7 +285,7 @@ __device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, in
                      "f"(v[4 * u]), "f"(v[4 * u + 1]), "f"(v[4 * u + 2]), "f"(v[4 * u + 3])
                      : "memory");
       }
-      const uint32_t wbr = bb + 3 * ADAM_ARRAY_BYTES + (uint32_t)row * 64u + (uint32_t)hf * 32u;
+      const uint32_t wbr = bb + 3 * ADAM_ARRAY_BYTES + (uint32_t)rr * 64u + (uint32_t)hf * 32u;
       asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(wbr),
                    "r"(pack_bf16(w[0], w[1])), "r"(pack_bf16(w[2], w[3])),
                    "r"(pack_bf16(w[4], w[5])), "r"(pack_bf16(w[6], w[7]))
@@ -290,9 +297,7 @@ __device__ __forceinline__ bool adam_tile(const GParams& p, int cell, int m0, in
     }
     // make the new values visible to the TMA store, then hand the chunk to the loader warp
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    mbar_arrive(aDone + 8 * abuf);
-    abuf ^= 1;
-    if (abuf == 0) aph ^= 1u;
+    mbar_arrive(aDone + 8 * bi);
   }
   return true;
 }
@@ -310,8 +315,8 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
   const uint32_t bFull = smem_u32(misc), bEmpty = bFull + 8 * STAGES;
   const uint32_t bAcc = bEmpty + 8 * STAGES, bReg = bAcc + 16, bFinal = bReg + 16;
   const uint32_t bEpi = bFinal + 8;    // [2], alternating by tile
-  const uint32_t aFull = bEpi + 16;   // [2] Adam chunk buffers: old values landed
-  const uint32_t aDone = aFull + 16;  // [2] new values written back by the epilogue
+  const uint32_t aFull = bEpi + 16;   // [4] Adam chunk buffers: old values landed
+  const uint32_t aDone = aFull + 32;  // [4] new values written back by the epilogue half
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
   volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 200);
@@ -329,9 +334,9 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     mbar_init(bFinal, 1);
     mbar_init(bEpi, EPI_THREADS);
     mbar_init(bEpi + 8, EPI_THREADS);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < Cfg<FUSED>::ADAM_BUFS; ++b) {
       mbar_init(aFull + 8 * b, 1);
-      mbar_init(aDone + 8 * b, EPI_THREADS);
+      mbar_init(aDone + 8 * b, EPI_THREADS / 2);
     }
     *abort_flag = 0;
     *done_tiles = 0;
@@ -485,11 +490,12 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     // ===== Adam loader: old w, m, v of every chunk of every EPI_ADAM tile, in tile order, and
     // the TMA stores of each chunk's new w, m, v and bf16 copy once the epilogue is done =====
     if (lane == 0) {
-      int buf = 0, issued[2] = {0, 0};
-      int pend_si[2] = {0, 0}, pend_x[2] = {0, 0}, pend_m[2] = {0, 0}, pend_c[2] = {0, 0};
-      bool has[2] = {false, false};
+      constexpr int NB = Cfg<FUSED>::ADAM_BUFS > 0 ? Cfg<FUSED>::ADAM_BUFS : 1;
+      int buf = 0, issued[NB] = {}, pend_si[NB] = {}, pend_x[NB] = {}, pend_m[NB] = {};
+      int pend_c[NB] = {};
+      bool has[NB] = {};
       bool ok = true;
-      // store the chunk held by buffer b once the epilogue has written it back
+      // store the chunk held by buffer b once its epilogue half has written it back
       auto flush = [&](int b) -> bool {
         if (!mbar_wait(aDone + 8 * b, (uint32_t)((issued[b] - 1) & 1), abort_flag, err, 19))
           return false;
@@ -512,7 +518,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
           for (int t = 0; t < nt && ok; ++t) {
             const int m0 = (t / p.ntiles) * BM, n0 = (t % p.ntiles) * p.BN;
             const int nch = (min(p.BN, p.N - n0) + ADAM_COLS - 1) / ADAM_COLS;
-            for (int k = 0; k < nch; ++k) {
+            for (int k = 0; k < 2 * nch; ++k) {
               if (has[buf]) {
                 if (!flush(buf)) {
                   ok = false;
@@ -523,26 +529,28 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
               const uint32_t full = aFull + 8 * buf;
               mbar_expect_tx(full, (uint32_t)(3 * ADAM_ARRAY_BYTES));
               const uint32_t dst = sAdam + (uint32_t)(buf * ADAM_BUF_BYTES);
-              const int x0 = n0 + k * ADAM_COLS;
-              tma_load_3d(dst, &maps.aw[si], full, x0, m0, zi);
-              tma_load_3d(dst + ADAM_ARRAY_BYTES, &maps.am[si], full, x0, m0, zi);
-              tma_load_3d(dst + 2 * ADAM_ARRAY_BYTES, &maps.av[si], full, x0, m0, zi);
+              const int x0 = n0 + (k >> 1) * ADAM_COLS, y0 = m0 + (k & 1) * ADAM_ROWS;
+              tma_load_3d(dst, &maps.aw[si], full, x0, y0, zi);
+              tma_load_3d(dst + ADAM_ARRAY_BYTES, &maps.am[si], full, x0, y0, zi);
+              tma_load_3d(dst + 2 * ADAM_ARRAY_BYTES, &maps.av[si], full, x0, y0, zi);
               issued[buf]++;
               has[buf] = true;
               pend_si[buf] = si;
               pend_x[buf] = x0;
-              pend_m[buf] = m0;
+              pend_m[buf] = y0;
               pend_c[buf] = cell;
-              buf ^= 1;
+              if (++buf == NB) buf = 0;
             }
           }
         }
       }
-      // the last chunks (oldest first)
-      for (int i = 0; i < 2 && ok; ++i, buf ^= 1)
+      // the last chunks, oldest first
+      for (int i = 0; i < NB && ok; ++i) {
         if (has[buf] && !flush(buf)) ok = false;
+        if (++buf == NB) buf = 0;
+      }
       if (!ok) {
-        for (int b = 0; b < 2; ++b)
+        for (int b = 0; b < NB; ++b)
           if (issued[b] > 0) {
             volatile int never = 0;
             mbar_wait(aFull + 8 * b, (uint32_t)((issued[b] - 1) & 1), &never, err, 19);
@@ -555,8 +563,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     const int row = q * 32 + lane;
     bool ok = true;
     int lt = 0, pub = 0;
-    int abuf = 0;
-    uint32_t aph = 0;
+    int cj = 0;  // Adam chunks of this thread's row half so far
     for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
       for (int si = 0; si < cp.n_stages && ok; ++si) {
         const GParams& p = cp.st[si].p;
@@ -574,7 +581,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
           const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(R * 256);
           if constexpr (FUSED) {
             if (p.epi == EPI_ADAM) {
-              if (!adam_tile(p, cell, m0, n0, tbase, hf, row, sAdam, aFull, aDone, abuf, aph,
+              if (!adam_tile(p, cell, m0, n0, tbase, hf, row, sAdam, aFull, aDone, cj,
                              abort_flag, err)) {
                 ok = false;
                 break;
@@ -664,12 +671,12 @@ bool map3(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint6
 }
 
 // fp32 3-D map over one weight tensor [out][in] of every individual: {in, out, individuals},
-// box {32, 128, 1} (one 128-byte row per output row), 128-byte swizzle.
+// box {32, 64, 1} (one 128-byte row per output row), 128-byte swizzle.
 bool map3f(CUtensorMap* m, const float* base, uint64_t inner, uint64_t rows, uint64_t depth,
            uint64_t depth_elems, std::string* msg) {
   cuuint64_t dims[3] = {inner, rows, depth};
   cuuint64_t strides[2] = {inner * 4, depth_elems * 4};
-  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::BM, 1};
+  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::ADAM_ROWS, 1};
   cuuint32_t es[3] = {1, 1, 1};
   CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(base), dims,
                      strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -681,13 +688,13 @@ bool map3f(CUtensorMap* m, const float* base, uint64_t inner, uint64_t rows, uin
   return true;
 }
 
-// bf16 3-D map over one tensor's bf16 copy of every cell: {in, out, cells}, box {32, 128, 1},
+// bf16 3-D map over one tensor's bf16 copy of every cell: {in, out, cells}, box {32, 64, 1},
 // no swizzle (64-byte rows).
 bool map3b_rows(CUtensorMap* m, const bf16* base, uint64_t inner, uint64_t rows, uint64_t depth,
                 uint64_t depth_elems, std::string* msg) {
   cuuint64_t dims[3] = {inner, rows, depth};
   cuuint64_t strides[2] = {inner * 2, depth_elems * 2};
-  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::BM, 1};
+  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::ADAM_ROWS, 1};
   cuuint32_t es[3] = {1, 1, 1};
   CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<bf16*>(base), dims,
                      strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
