@@ -120,7 +120,10 @@ LIPZ_API int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_
 /* Frees everything the grid owns. Null is accepted. */
 LIPZ_API int lipz_grid_destroy(lipz_grid* g);
 
-/* Runs the grid's work on `stream` (a cudaStream_t, owned by the caller; 0 = legacy default). */
+/* Runs the grid's work on `stream` (a cudaStream_t, owned by the caller), or on the grid's own
+ * non-blocking stream (the default, created with the grid) when `stream` is null. Work already
+ * queued completes first. On a created stream consecutive kernels use programmatic dependent
+ * launch; on the legacy or per-thread default stream they keep plain stream order. */
 LIPZ_API int lipz_set_stream(lipz_grid* g, void* stream);
 
 /* Blocks until the grid's stream is idle; reports a non-finite loss seen since the last check. */

@@ -3,7 +3,9 @@
 // The grid owns two population snapshots per population (ping-pong A/B): an iteration reads
 // snapshot `cur` (evaluation, selection, gradients) and writes every cell's new centre into
 // snapshot 1 - cur, so no cell can see a neighbour's half-updated state. Work is enqueued on
-// one CUDA stream; the host waits only when the caller asks for host-side results.
+// one CUDA stream, the kernels with programmatic dependent launch (each kernel's set-up
+// overlaps the previous kernel's tail; its first global access waits for that kernel); the
+// host waits only when the caller asks for host-side results.
 #include <climits>
 #include <cmath>
 #include <cstdarg>
@@ -50,7 +52,8 @@ struct lipz_grid {
   Layout lg{}, ld{};
   int64_t PG = 0, PD = 0, PGs = 0, PDs = 0;
   int64_t e_cell = 0;  // elements per cell of the evaluation input E (6B rows)
-  cudaStream_t st = nullptr;
+  cudaStream_t st = nullptr;      // stream all work is enqueued on
+  cudaStream_t own_st = nullptr;  // the grid's own non-blocking stream (the default)
   int device = 0;
   PopView G[2]{}, D[2]{};
   int cur = 0;
@@ -77,9 +80,6 @@ struct lipz_grid {
   TcPlan* tc[2]{};
   TcbPlan* tcb[2]{};
   bool use_tcb = false;
-  cudaStream_t side = nullptr;  // second stream of the training step (owned)
-  cudaEvent_t ev_fork = nullptr, ev_d1 = nullptr, ev_join = nullptr;
-  bool side_pending = false;    // the side stream's last work is not yet joined into st
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
   bool prof = false;
@@ -172,14 +172,6 @@ void phase_end(lipz_grid* g, int ph, int n_launches) {
   g->open_ev[ph] = nullptr;
 }
 
-// Makes the grid's stream wait for the side stream's outstanding work (the discriminator's
-// Adam step of the last training step), if any.
-cudaError_t join_side(lipz_grid* g) {
-  if (!g->side_pending) return cudaSuccess;
-  g->side_pending = false;
-  return cudaStreamWaitEvent(g->st, g->ev_join, 0);
-}
-
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
 // Layouts (PyTorch Linear convention, W [out][in] row-major).
@@ -230,12 +222,23 @@ GemmDesc gd(const void* A, int64_t sam, int64_t sak, const void* B, int64_t sbk,
   return d;
 }
 
+// Host -> device copy and memset in the order of the grid's stream (which need not be the
+// legacy default stream); the copy returns once the host buffer may be reused.
+int h2d(lipz_grid* g, void* dst, const void* src, size_t bytes) {
+  CK(g, cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
+  return LIPZ_OK;
+}
+int dset(lipz_grid* g, void* dst, int value, size_t bytes) {
+  CK(g, cudaMemsetAsync(dst, value, bytes, g->st));
+  return LIPZ_OK;
+}
+
 template <typename T>
 int upload(lipz_grid* g, T** dst, const std::vector<T>& v) {
   int rc = dalloc(g, dst, v.size() * sizeof(T));
   if (rc) return rc;
-  CK(g, cudaMemcpy(*dst, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice));
-  return LIPZ_OK;
+  return h2d(g, *dst, v.data(), v.size() * sizeof(T));
 }
 
 int build_descs(lipz_grid* g, int p) {
@@ -485,11 +488,10 @@ int alloc_pop(lipz_grid* g, PopView* p, int64_t Ps) {
     return rc;
   p->wb = nullptr;
   if (g->bf && (rc = dalloc(g, &p->wb, n * 2))) return rc;
-  CK(g, cudaMemset(p->w, 0, n * 4));
-  CK(g, cudaMemset(p->m, 0, n * 4));
-  CK(g, cudaMemset(p->v, 0, n * 4));
-  CK(g, cudaMemset(p->step, 0, g->cells * 4));
-  if (p->wb) CK(g, cudaMemset(p->wb, 0, n * 2));
+  if ((rc = dset(g, p->w, 0, n * 4)) || (rc = dset(g, p->m, 0, n * 4)) ||
+      (rc = dset(g, p->v, 0, n * 4)) || (rc = dset(g, p->step, 0, g->cells * 4)) ||
+      (p->wb && (rc = dset(g, p->wb, 0, n * 2))))
+    return rc;
   return LIPZ_OK;
 }
 
@@ -498,10 +500,9 @@ int create_impl(lipz_grid* g) {
   const size_t es = g->esz;
   int rc;
   CK(g, cudaGetDevice(&g->device));
-  CK(g, cudaStreamCreateWithFlags(&g->side, cudaStreamNonBlocking));
-  CK(g, cudaEventCreateWithFlags(&g->ev_fork, cudaEventDisableTiming));
-  CK(g, cudaEventCreateWithFlags(&g->ev_d1, cudaEventDisableTiming));
-  CK(g, cudaEventCreateWithFlags(&g->ev_join, cudaEventDisableTiming));
+  // the grid's own stream (lipz_set_stream may replace it)
+  CK(g, cudaStreamCreateWithFlags(&g->own_st, cudaStreamNonBlocking));
+  g->st = g->own_st;
   make_layouts(g);
   g->e_cell = (int64_t)6 * B * x;
   for (int p = 0; p < 2; ++p) {
@@ -527,10 +528,10 @@ int create_impl(lipz_grid* g) {
       (rc = dalloc(g, &g->gD, (size_t)C * g->PDs * 4)) || (rc = dalloc(g, &g->flag, 4)) ||
       (rc = dalloc(g, &g->xin, CB * x * 4)))
     return rc;
-  CK(g, cudaMemset(g->gG, 0, (size_t)C * g->PGs * 4));
-  CK(g, cudaMemset(g->gD, 0, (size_t)C * g->PDs * 4));
   const int big = INT_MAX;
-  CK(g, cudaMemcpy(g->flag, &big, 4, cudaMemcpyHostToDevice));
+  if ((rc = dset(g, g->gG, 0, (size_t)C * g->PGs * 4)) ||
+      (rc = dset(g, g->gD, 0, (size_t)C * g->PDs * 4)) || (rc = h2d(g, g->flag, &big, 4)))
+    return rc;
   // step 1: random initialisation of snapshot 0
   launch_init_params(g->G[0].w, g->G[0].wb, g->PG, g->PGs, g->lg, C, g->seed, LIPZ_STREAM_INIT_G,
                      g->st);
@@ -538,10 +539,8 @@ int create_impl(lipz_grid* g) {
                      g->st);
   CKL(g);
   std::vector<float> lr(C, g->a.lr);
-  CK(g, cudaMemcpy(g->G[0].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
-  CK(g, cudaMemcpy(g->D[0].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
-  CK(g, cudaMemcpy(g->G[1].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
-  CK(g, cudaMemcpy(g->D[1].lr, lr.data(), C * 4, cudaMemcpyHostToDevice));
+  for (float* d : {g->G[0].lr, g->D[0].lr, g->G[1].lr, g->D[1].lr})
+    if ((rc = h2d(g, d, lr.data(), C * 4))) return rc;
   if ((rc = build_descs(g, 0)) || (rc = build_descs(g, 1))) return rc;
   g->use_tc = g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
   if (g->use_tc) {
@@ -620,7 +619,8 @@ int create_impl(lipz_grid* g) {
       if (!g->tcb[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core backward plan: %s", msg.c_str());
     }
   }
-  CK(g, cudaStreamSynchronize(g->st));
+  // the plans' set-up (allocations, flag resets) ran outside the grid's stream
+  CK(g, cudaDeviceSynchronize());
   return LIPZ_OK;
 }
 
@@ -643,8 +643,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);
-    CK(g, join_side(g));
-    phase_begin(g, LIPZ_PHASE_D_FWD);
+      phase_begin(g, LIPZ_PHASE_D_FWD);
     if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_D_FWD, 1);
   } else {
@@ -654,8 +653,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
     phase_end(g, LIPZ_PHASE_G_FWD, 3);
-    CK(g, join_side(g));
-    phase_begin(g, LIPZ_PHASE_D_FWD);
+      phase_begin(g, LIPZ_PHASE_D_FWD);
     gemm(g, D.d1, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemm(g, D.d2, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemv(g, D.d3, C * 5, 6 * B);
@@ -671,7 +669,6 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
 }
 
 int select_impl(lipz_grid* g) {
-  CK(g, join_side(g));
   if (g->phase != PH_EVALUATED)
     return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
   SelectParams sp;
@@ -697,7 +694,6 @@ int select_impl(lipz_grid* g) {
 }
 
 int train_impl(lipz_grid* g) {
-  CK(g, join_side(g));
   if (g->phase != PH_SELECTED)
     return fail(g, LIPZ_ERR_STATE, "lipz_train_step must follow lipz_select_replace");
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
@@ -777,25 +773,6 @@ int train_impl(lipz_grid* g) {
       g->phase = PH_IDLE;
       return LIPZ_OK;
     }
-    if (!g->prof) {
-      // The discriminator's Adam runs on the side stream, overlapping the generator's Adam and
-      // the next evaluation's generator kernel; the grid's stream waits for it before anything
-      // reads the discriminator population again (join_side).
-      CK(g, cudaEventRecord(g->ev_fork, g->st));
-      CK(g, cudaStreamWaitEvent(g->side, g->ev_fork, 0));
-      launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs,
-                  g->a.beta1, g->a.beta2, g->a.eps, g->side);
-      CK(g, cudaEventRecord(g->ev_join, g->side));
-      g->side_pending = true;
-      launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs,
-                  g->a.beta1, g->a.beta2, g->a.eps, g->st);
-      CKL(g);
-      phase_end(g, LIPZ_PHASE_ADAM, 3);
-      g->cur = 1 - p;
-      g->t += 1;
-      g->phase = PH_IDLE;
-      return LIPZ_OK;
-    }
   } else {
     gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
     colsum(g, D.cb2d, C, h);
@@ -835,17 +812,21 @@ int check_flag(lipz_grid* g) {
                    : (g->tcb[p - 2] ? tcb_error_flag(g->tcb[p - 2]) : nullptr);
     if (!f) continue;
     int code = 0;
-    CK(g, cudaMemcpy(&code, f, 4, cudaMemcpyDeviceToHost));
+    CK(g, cudaMemcpyAsync(&code, f, 4, cudaMemcpyDeviceToHost, g->st));
+    CK(g, cudaStreamSynchronize(g->st));
     if (code) {
-      CK(g, cudaMemset(f, 0, 4));
+      CK(g, cudaMemsetAsync(f, 0, 4, g->st));
+      CK(g, cudaStreamSynchronize(g->st));
       return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
   int v = INT_MAX;
-  CK(g, cudaMemcpy(&v, g->flag, 4, cudaMemcpyDeviceToHost));
+  CK(g, cudaMemcpyAsync(&v, g->flag, 4, cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
   if (v != INT_MAX) {
     const int big = INT_MAX;
-    CK(g, cudaMemcpy(g->flag, &big, 4, cudaMemcpyHostToDevice));
+    int rc = h2d(g, g->flag, &big, 4);
+    if (rc) return rc;
     return fail(g, LIPZ_ERR_NONFINITE, "non-finite loss in cell %d", v);
   }
   return LIPZ_OK;
@@ -934,7 +915,7 @@ int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_t seed, l
 
 int lipz_grid_destroy(lipz_grid* g) {
   if (!g) return LIPZ_OK;
-  if (g->st || true) cudaStreamSynchronize(g->st);
+  cudaStreamSynchronize(g->st);
   for (int p = 0; p < 2; ++p) {
     if (g->tc[p]) tc_plan_destroy(g->tc[p]);
     if (g->tcb[p]) tcb_plan_destroy(g->tcb[p]);
@@ -946,34 +927,27 @@ int lipz_grid_destroy(lipz_grid* g) {
   for (auto e : g->ev_free) cudaEventDestroy(e);
   for (auto e : g->open_ev)
     if (e) cudaEventDestroy(e);
-  if (g->side) {
-    cudaStreamSynchronize(g->side);
-    cudaStreamDestroy(g->side);
-  }
-  for (cudaEvent_t e : {g->ev_fork, g->ev_d1, g->ev_join})
-    if (e) cudaEventDestroy(e);
   for (void* p : g->allocs) cudaFree(p);
+  if (g->own_st) cudaStreamDestroy(g->own_st);
   delete g;
   return LIPZ_OK;
 }
 
 int lipz_set_stream(lipz_grid* g, void* stream) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
-  g->st = (cudaStream_t)stream;
+  CK(g, cudaStreamSynchronize(g->st));  // work already queued stays ordered before the switch
+  g->st = stream ? (cudaStream_t)stream : g->own_st;
   return LIPZ_OK;
 }
 
 int lipz_synchronize(lipz_grid* g) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   CK(g, cudaStreamSynchronize(g->st));
   return check_flag(g);
 }
 
 int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t dim) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   if (!host_pool || n_rows < 1 || n_rows > 0xFFFFFFFFll || dim != g->a.x_dim)
     return fail(g, LIPZ_ERR_INVALID, "set_data needs a pool of 1..2^32-1 rows of x_dim=%d",
                 g->a.x_dim);
@@ -995,7 +969,7 @@ int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t 
     // rounded once here: a drawn row is then the same bf16 row the fp32 pool would give
     float* tmp = nullptr;
     CK(g, cudaMalloc(&tmp, n * 4));
-    cudaError_t e = cudaMemcpy(tmp, host_pool, n * 4, cudaMemcpyHostToDevice);
+    cudaError_t e = cudaMemcpyAsync(tmp, host_pool, n * 4, cudaMemcpyHostToDevice, g->st);
     if (e == cudaSuccess) {
       launch_to_bf16(tmp, (bf16*)g->pool, (int64_t)n, g->st);
       e = cudaGetLastError();
@@ -1004,7 +978,8 @@ int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t 
     cudaFree(tmp);
     CK(g, e);
   } else {
-    CK(g, cudaMemcpy(g->pool, host_pool, n * 4, cudaMemcpyHostToDevice));
+    int rc = h2d(g, g->pool, host_pool, n * 4);
+    if (rc) return rc;
   }
   g->pool_n = n_rows;
   return LIPZ_OK;
@@ -1077,7 +1052,6 @@ int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {
 
 int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   size_t need = 0;
   lipz_state_bytes(g, &need);
   if (!host || bytes != need)
@@ -1095,7 +1069,7 @@ int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
   const int p = g->cur;
   const size_t C = g->cells;
   auto put = [&](const float* src, int64_t P, int64_t Ps) -> int {
-    CK(g, cudaMemcpy2D(o, P * 4, src, Ps * 4, P * 4, C, cudaMemcpyDeviceToHost));
+    CK(g, cudaMemcpy2DAsync(o, P * 4, src, Ps * 4, P * 4, C, cudaMemcpyDeviceToHost, g->st));
     o += C * P * 4;
     return LIPZ_OK;
   };
@@ -1104,19 +1078,19 @@ int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
       (rc = put(g->G[p].v, g->PG, g->PGs)) || (rc = put(g->D[p].w, g->PD, g->PDs)) ||
       (rc = put(g->D[p].m, g->PD, g->PDs)) || (rc = put(g->D[p].v, g->PD, g->PDs)))
     return rc;
-  CK(g, cudaMemcpy(o, g->G[p].step, C * 4, cudaMemcpyDeviceToHost));
+  CK(g, cudaMemcpyAsync(o, g->G[p].step, C * 4, cudaMemcpyDeviceToHost, g->st));
   o += C * 4;
-  CK(g, cudaMemcpy(o, g->D[p].step, C * 4, cudaMemcpyDeviceToHost));
+  CK(g, cudaMemcpyAsync(o, g->D[p].step, C * 4, cudaMemcpyDeviceToHost, g->st));
   o += C * 4;
-  CK(g, cudaMemcpy(o, g->G[p].lr, C * 4, cudaMemcpyDeviceToHost));
+  CK(g, cudaMemcpyAsync(o, g->G[p].lr, C * 4, cudaMemcpyDeviceToHost, g->st));
   o += C * 4;
-  CK(g, cudaMemcpy(o, g->D[p].lr, C * 4, cudaMemcpyDeviceToHost));
+  CK(g, cudaMemcpyAsync(o, g->D[p].lr, C * 4, cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
   return LIPZ_OK;
 }
 
 int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   size_t need = 0;
   lipz_state_bytes(g, &need);
   if (!host || bytes != need) return fail(g, LIPZ_ERR_INVALID, "import_state needs %zu bytes", need);
@@ -1137,7 +1111,7 @@ int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   const int p = g->cur;
   const size_t C = g->cells;
   auto get = [&](float* dst, int64_t P, int64_t Ps) -> int {
-    CK(g, cudaMemcpy2D(dst, Ps * 4, s, P * 4, P * 4, C, cudaMemcpyHostToDevice));
+    CK(g, cudaMemcpy2DAsync(dst, Ps * 4, s, P * 4, P * 4, C, cudaMemcpyHostToDevice, g->st));
     s += C * P * 4;
     return LIPZ_OK;
   };
@@ -1146,13 +1120,13 @@ int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
       (rc = get(g->G[p].v, g->PG, g->PGs)) || (rc = get(g->D[p].w, g->PD, g->PDs)) ||
       (rc = get(g->D[p].m, g->PD, g->PDs)) || (rc = get(g->D[p].v, g->PD, g->PDs)))
     return rc;
-  CK(g, cudaMemcpy(g->G[p].step, s, C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpyAsync(g->G[p].step, s, C * 4, cudaMemcpyHostToDevice, g->st));
   s += C * 4;
-  CK(g, cudaMemcpy(g->D[p].step, s, C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpyAsync(g->D[p].step, s, C * 4, cudaMemcpyHostToDevice, g->st));
   s += C * 4;
-  CK(g, cudaMemcpy(g->G[p].lr, s, C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpyAsync(g->G[p].lr, s, C * 4, cudaMemcpyHostToDevice, g->st));
   s += C * 4;
-  CK(g, cudaMemcpy(g->D[p].lr, s, C * 4, cudaMemcpyHostToDevice));
+  CK(g, cudaMemcpyAsync(g->D[p].lr, s, C * 4, cudaMemcpyHostToDevice, g->st));
   if (g->bf) {
     launch_to_bf16(g->G[p].w, g->G[p].wb, (int64_t)C * g->PGs, g->st);
     launch_to_bf16(g->D[p].w, g->D[p].wb, (int64_t)C * g->PDs, g->st);
@@ -1173,7 +1147,6 @@ int lipz_get_iteration(const lipz_grid* g, int64_t* t) {
 
 int lipz_get_batch(lipz_grid* g, float* x, float* z) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   if (g->phase == PH_IDLE) return fail(g, LIPZ_ERR_STATE, "no evaluation since the last train step");
   const int64_t B = g->a.batch;
   int rc;
@@ -1193,7 +1166,6 @@ int lipz_get_logits(lipz_grid* g, float* logits) {
 
 int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   if (!g->a.keep_grads) return fail(g, LIPZ_ERR_STATE, "grid was created without keep_grads");
   CK(g, cudaStreamSynchronize(g->st));
   const size_t C = g->cells;
@@ -1212,7 +1184,6 @@ int lipz_profile_enable(lipz_grid* g, int enable) {
 
 int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t* launches, int n) {
   if (!g) return LIPZ_ERR_INVALID;
-  CK(g, join_side(g));
   if (n < 0 || n > LIPZ_N_PHASES) return fail(g, LIPZ_ERR_INVALID, "n must be in 0..%d", LIPZ_N_PHASES);
   CK(g, cudaStreamSynchronize(g->st));
   double acc[LIPZ_N_PHASES] = {0};

@@ -353,6 +353,9 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   int* err = cp.err;
+  // the set-up above touched no global memory: from here on the previous kernel's results
+  // are needed (programmatic dependent launch)
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1021,12 +1024,11 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
 
 int tcb_run_cells(TcbPlan* P, cudaStream_t st, std::string* msg) {
   if (P->fused)
-    tcb::k_bwd_cells<true><<<P->grid_cells, tcb::Cfg<true>::THREADS, tcb::Cfg<true>::SMEM, st>>>(
-        P->maps, P->cells);
+    launch_pdl(tcb::k_bwd_cells<true>, dim3(P->grid_cells), dim3(tcb::Cfg<true>::THREADS),
+               tcb::Cfg<true>::SMEM, st, P->maps, P->cells);
   else
-    tcb::k_bwd_cells<false>
-        <<<P->grid_cells, tcb::Cfg<false>::THREADS, tcb::Cfg<false>::SMEM, st>>>(P->maps,
-                                                                                 P->cells);
+    launch_pdl(tcb::k_bwd_cells<false>, dim3(P->grid_cells), dim3(tcb::Cfg<false>::THREADS),
+               tcb::Cfg<false>::SMEM, st, P->maps, P->cells);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     if (msg) *msg = std::string("per-cell backward launch: ") + cudaGetErrorString(e);

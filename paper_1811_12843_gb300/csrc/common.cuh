@@ -10,6 +10,31 @@ namespace lipz {
 
 typedef __nv_bfloat16 bf16;
 
+// ---- programmatic dependent launch: kernels of one grid iteration are launched with
+// programmatic stream serialization, so a kernel is launched while the previous one retires;
+// each waits for the previous kernel to complete and flush its memory (pdl_wait) before it
+// touches global memory. Kernels signal no early completion: the next kernel starts only once
+// every block of the previous one has exited. Without the launch attribute the wait is a no-op.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  // only on an explicitly created stream: the legacy and per-thread default streams are
+  // shared with other work and keep plain stream order
+  cfg.numAttrs = (st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread) ? 0 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---- Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds, key bumped by the Weyl
 // constants between rounds; one round maps (c0, c1, c2, c3) to
 // (hi(M1 c2) ^ c1 ^ k0, lo(M1 c2), hi(M0 c0) ^ c3 ^ k1, lo(M0 c0)).

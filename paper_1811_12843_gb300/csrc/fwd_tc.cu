@@ -179,6 +179,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int nj = n_jobs(p);
+  // the set-up above touched no global memory: from here on the previous kernel's results
+  // are needed (programmatic dependent launch)
+  pdl_wait();
 
   if (warp == 0) {
     // ================================ TMA producer ================================
@@ -667,7 +670,7 @@ namespace {
 int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensorMap& b2,
            const CUtensorMap& b3, const tc::KParams& kp, cudaStream_t st, const char* what,
            std::string* msg) {
-  tc::k_mlp_fwd<<<grid, tc::THREADS, tc::SMEM_BYTES, st>>>(a, b1, b2, b3, kp);
+  launch_pdl(tc::k_mlp_fwd, dim3(grid), dim3(tc::THREADS), tc::SMEM_BYTES, st, a, b1, b2, b3, kp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     if (msg) *msg = std::string(what) + " launch: " + cudaGetErrorString(e);

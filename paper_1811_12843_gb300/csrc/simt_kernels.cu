@@ -81,6 +81,7 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
                              T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
                              uint32_t t) {
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
   if (b >= B) return;
@@ -139,8 +140,8 @@ template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
                        cudaStream_t st) {
-  k_draw_batch<T><<<dim3((B + 7) / 8, cells), 256, 0, st>>>(pool, n_pool, xin, E, e_cell, Z, B,
-                                                            x_dim, z_dim, seed, t);
+  launch_pdl(k_draw_batch<T>, dim3((B + 7) / 8, cells), dim3(256), 0, st, pool, n_pool, xin, E,
+             e_cell, Z, B, x_dim, z_dim, seed, t);
 }
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
                                        float*, int, int, int, int, uint64_t, uint32_t,
@@ -155,6 +156,7 @@ template void launch_draw_batch<bf16>(const bf16*, int64_t, const float*, bf16*,
 template <typename TI, typename TO, int EPI>
 __global__ void __launch_bounds__(256) k_gemm(const GemmDesc* __restrict__ descs, int act,
                                               float slope) {
+  pdl_wait();
   const GemmDesc d = descs[blockIdx.z];
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   if (m0 >= d.M || n0 >= d.N) return;
@@ -234,7 +236,7 @@ void launch_gemm(const GemmDesc* descs, int n_problems, int max_m, int max_n, in
                  float slope, cudaStream_t st) {
   if (n_problems <= 0 || max_m <= 0 || max_n <= 0) return;
   dim3 grid((max_n + 63) / 64, (max_m + 63) / 64, n_problems);
-  k_gemm<TI, TO, EPI><<<grid, 256, 0, st>>>(descs, act, slope);
+  launch_pdl(k_gemm<TI, TO, EPI>, grid, dim3(256), 0, st, descs, act, slope);
 }
 #define LIPZ_INST_GEMM(TI, TO, EPI) \
   template void launch_gemm<TI, TO, EPI>(const GemmDesc*, int, int, int, int, float, cudaStream_t);
@@ -250,6 +252,7 @@ LIPZ_INST_GEMM(bf16, bf16, EPI_DACT)
 // ------------------------------------------------------------------------------------------
 template <typename T>
 __global__ void k_gemv(const GemvDesc* __restrict__ descs) {
+  pdl_wait();
   const GemvDesc d = descs[blockIdx.y];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + warp;
@@ -272,7 +275,7 @@ __global__ void k_gemv(const GemvDesc* __restrict__ descs) {
 template <typename T>
 void launch_gemv(const GemvDesc* descs, int n_problems, int max_rows, cudaStream_t st) {
   if (n_problems <= 0 || max_rows <= 0) return;
-  k_gemv<T><<<dim3((max_rows + 7) / 8, n_problems), 256, 0, st>>>(descs);
+  launch_pdl(k_gemv<T>, dim3((max_rows + 7) / 8, n_problems), dim3(256), 0, st, descs);
 }
 template void launch_gemv<float>(const GemvDesc*, int, int, cudaStream_t);
 template void launch_gemv<bf16>(const GemvDesc*, int, int, cudaStream_t);
@@ -284,6 +287,7 @@ template void launch_gemv<bf16>(const GemvDesc*, int, int, cudaStream_t);
 // ------------------------------------------------------------------------------------------
 template <typename T>
 __global__ void __launch_bounds__(256) k_colsum(const ColSumDesc* __restrict__ descs) {
+  pdl_wait();
   // A block takes 256 columns of one problem: lane l owns columns 8l .. 8l + 7, warp w the
   // rows w, w + 8, ...; the 8 partial sums of a column are added in a fixed order.
   const ColSumDesc d = descs[blockIdx.y];
@@ -328,7 +332,7 @@ __global__ void __launch_bounds__(256) k_colsum(const ColSumDesc* __restrict__ d
 template <typename T>
 void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st) {
   if (n_problems <= 0 || max_cols <= 0) return;
-  k_colsum<T><<<dim3((max_cols + 255) / 256, n_problems), 256, 0, st>>>(descs);
+  launch_pdl(k_colsum<T>, dim3((max_cols + 255) / 256, n_problems), dim3(256), 0, st, descs);
 }
 template void launch_colsum<float>(const ColSumDesc*, int, int, cudaStream_t);
 template void launch_colsum<bf16>(const ColSumDesc*, int, int, cudaStream_t);
@@ -346,6 +350,7 @@ __device__ __forceinline__ float softplusf(float x) { return fmaxf(x, 0.f) + log
 __global__ void k_fitness(const float* __restrict__ logits, int B, float* __restrict__ LG,
                           float* __restrict__ LD, float* __restrict__ fG, float* __restrict__ fD,
                           int* __restrict__ flag) {
+  pdl_wait();
   const int c = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   __shared__ float real_s[5], fake_d[25], fake_g[25];
@@ -401,7 +406,8 @@ __global__ void k_fitness(const float* __restrict__ logits, int B, float* __rest
 
 void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
                     float* fD, int* flag, cudaStream_t st) {
-  k_fitness<<<cells, 960, 0, st>>>(logits, B, LG, LD, fG, fD, flag);  // one warp per mean
+  // one warp per mean
+  launch_pdl(k_fitness, dim3(cells), dim3(960), 0, st, logits, B, LG, LD, fG, fD, flag);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -436,6 +442,7 @@ __global__ void k_select(const float* __restrict__ fG, const float* __restrict__
                          int* __restrict__ src_d, float* __restrict__ lr_g_new,
                          float* __restrict__ lr_d_new, float4* __restrict__ coef_g,
                          float4* __restrict__ coef_d) {
+  pdl_wait();
   const int gid = blockIdx.x * blockDim.x + threadIdx.x;
   const int c = gid >> 1;
   if (c >= cells) return;
@@ -475,9 +482,9 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
                    int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
                    float4* coef_d, cudaStream_t st) {
-  k_select<<<(2 * cells + 127) / 128, 128, 0, st>>>(fG, fD, nbr, cells, p, lr_g_old, lr_d_old,
-                                                step_g_old, step_d_old, sel_g, sel_d, src_g, src_d,
-                                                lr_g_new, lr_d_new, coef_g, coef_d);
+  launch_pdl(k_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, fG, fD, nbr, cells, p,
+             lr_g_old, lr_d_old, step_g_old, step_d_old, sel_g, sel_d, src_g, src_d, lr_g_new,
+             lr_d_new, coef_g, coef_d);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -486,6 +493,7 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
 template <typename T>
 __global__ void k_train_prep(const T* __restrict__ E, int64_t e_cell, const int* __restrict__ sel_g,
                              T* __restrict__ TX, int B, int x_dim) {
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
   if (r >= 2 * B) return;
@@ -505,7 +513,8 @@ __global__ void k_train_prep(const T* __restrict__ E, int64_t e_cell, const int*
 template <typename T>
 void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
                        int x_dim, cudaStream_t st) {
-  k_train_prep<T><<<dim3((2 * B + 7) / 8, cells), 256, 0, st>>>(E, e_cell, sel_g, TX, B, x_dim);
+  launch_pdl(k_train_prep<T>, dim3((2 * B + 7) / 8, cells), dim3(256), 0, st, E, e_cell, sel_g,
+             TX, B, x_dim);
 }
 template void launch_train_prep<float>(const float*, int64_t, const int*, float*, int, int, int,
                                        cudaStream_t);
@@ -525,6 +534,7 @@ __global__ void __launch_bounds__(1024) k_dlogit(
     int64_t wD_stride, int64_t off_w3, const int* __restrict__ src_d, int B, int H, float slope,
     T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride, int64_t off_gw3,
     int64_t off_gb3) {
+  pdl_wait();
   // Lanes own column groups of 8 (threads of the block: H / 8 groups x RG row groups); the RG
   // partial sums of dW3 are added in a fixed order.
   extern __shared__ float dl[];  // [3B] deltas, then [RG][H] partial sums
@@ -611,8 +621,8 @@ void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride
   if (rg > 16) rg = 16;
   const int threads = ((rg * ng + 31) / 32) * 32;
   const size_t smem = (3 * (size_t)B + (size_t)(threads / ng) * H) * sizeof(float);
-  k_dlogit<T><<<cells, threads, smem, st>>>(TL, TG2, wD, wD_stride, off_w3, src_d, B, H, slope, J2,
-                                            gD, gD_stride, off_gw3, off_gb3);
+  launch_pdl(k_dlogit<T>, dim3(cells), dim3(threads), smem, st, TL, TG2, wD, wD_stride, off_w3,
+             src_d, B, H, slope, J2, gD, gD_stride, off_gw3, off_gb3);
 }
 template void launch_dlogit<float>(const float*, const float*, const float*, int64_t, int64_t,
                                    const int*, int, int, int, float, float*, float*, int64_t,
@@ -640,6 +650,7 @@ __global__ void __launch_bounds__(256) k_adam(PopView old_p, PopView new_p,
                                               const int* __restrict__ src,
                                               const float4* __restrict__ coef, int64_t P,
                                               int64_t Ps, float beta1, float beta2, float eps) {
+  pdl_wait();
   const int c = blockIdx.y;
   const int s = src[c];
   const float4 cf = coef[c];
@@ -696,7 +707,8 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
   if (per_cell > target * 4) per_cell = target * 4;
   if (per_cell < 1) per_cell = 1;
   dim3 grid(per_cell, cells);
-  k_adam<<<grid, 256, 0, st>>>(old_p, new_p, grad, src, coef, P, Ps, beta1, beta2, eps);
+  launch_pdl(k_adam, grid, dim3(256), 0, st, old_p, new_p, grad, src, coef, P, Ps, beta1, beta2,
+             eps);
 }
 
 // Adam + replacement of listed parameter ranges only (the tensors whose update is not fused
@@ -705,6 +717,7 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
 // learning rate.
 __global__ void __launch_bounds__(256) k_adam_ranges(AdamRanges r0, AdamRanges r1, float beta1,
                                                       float beta2, float eps) {
+  pdl_wait();
   const AdamRanges& r = blockIdx.y ? r1 : r0;
   const int c = blockIdx.x;
   const int s = r.src[c];
@@ -729,7 +742,7 @@ __global__ void __launch_bounds__(256) k_adam_ranges(AdamRanges r0, AdamRanges r
 
 void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, float beta1,
                         float beta2, float eps, cudaStream_t st) {
-  k_adam_ranges<<<dim3(cells, 2), 256, 0, st>>>(g, d, beta1, beta2, eps);
+  launch_pdl(k_adam_ranges, dim3(cells, 2), dim3(256), 0, st, g, d, beta1, beta2, eps);
 }
 
 }  // namespace lipz
