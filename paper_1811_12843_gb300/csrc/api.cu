@@ -624,7 +624,12 @@ int create_impl(lipz_grid* g) {
   return LIPZ_OK;
 }
 
-int eval_impl(lipz_grid* g, const float* xin_dev) {
+SelectParams select_params(const lipz_grid* g);
+SelectIO select_io(lipz_grid* g);
+
+// Evaluation (minibatch, forwards, fitness); with `then_select` the selection runs in the
+// fitness kernel (the caller reads nothing back in between).
+int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select) {
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
   if (!xin_dev && g->pool_n <= 0)
     return fail(g, LIPZ_ERR_STATE, "no real-data pool: call lipz_set_data first");
@@ -643,7 +648,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);
-      phase_begin(g, LIPZ_PHASE_D_FWD);
+    phase_begin(g, LIPZ_PHASE_D_FWD);
     if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_D_FWD, 1);
   } else {
@@ -653,7 +658,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
     gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
     phase_end(g, LIPZ_PHASE_G_FWD, 3);
-      phase_begin(g, LIPZ_PHASE_D_FWD);
+    phase_begin(g, LIPZ_PHASE_D_FWD);
     gemm(g, D.d1, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemm(g, D.d2, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemv(g, D.d3, C * 5, 6 * B);
@@ -661,17 +666,20 @@ int eval_impl(lipz_grid* g, const float* xin_dev) {
   }
   CKL(g);
   phase_begin(g, LIPZ_PHASE_FITNESS);
-  launch_fitness(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->st);
+  if (then_select)
+    launch_fitness_select(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->nbr,
+                          select_params(g), select_io(g), g->st);
+  else
+    launch_fitness(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_FITNESS, 1);
-  g->phase = PH_EVALUATED;
+  g->phase = then_select ? PH_SELECTED : PH_EVALUATED;
   return LIPZ_OK;
 }
 
-int select_impl(lipz_grid* g) {
-  if (g->phase != PH_EVALUATED)
-    return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
+SelectParams select_params(const lipz_grid* g) {
   SelectParams sp;
+  memset(&sp, 0, sizeof sp);
   sp.seed = g->seed;
   sp.t = (uint32_t)g->t;
   sp.tournament_size = g->a.tournament_size;
@@ -680,13 +688,34 @@ int select_impl(lipz_grid* g) {
   sp.lr_mut_std = g->a.lr_mut_std;
   double thr = std::floor((double)g->a.lr_mut_prob * 4294967296.0);
   sp.lr_mut_thr = (uint64_t)(thr < 0 ? 0 : (thr > 4294967296.0 ? 4294967296.0 : thr));
-  const int p = g->cur;
-  phase_begin(g, LIPZ_PHASE_SELECT);
   sp.beta1 = g->a.beta1;
   sp.beta2 = g->a.beta2;
-  launch_select(g->fG, g->fD, g->nbr, g->cells, sp, g->G[p].lr, g->D[p].lr, g->G[p].step,
-                g->D[p].step, g->sel_g, g->sel_d, g->src_g, g->src_d, g->lrn_g, g->lrn_d,
-                g->coef_g, g->coef_d, g->st);
+  return sp;
+}
+
+SelectIO select_io(lipz_grid* g) {
+  const int p = g->cur;
+  SelectIO io;
+  io.lr_old[0] = g->G[p].lr;
+  io.lr_old[1] = g->D[p].lr;
+  io.step_old[0] = g->G[p].step;
+  io.step_old[1] = g->D[p].step;
+  io.sel[0] = g->sel_g;
+  io.sel[1] = g->sel_d;
+  io.src[0] = g->src_g;
+  io.src[1] = g->src_d;
+  io.lr_new[0] = g->lrn_g;
+  io.lr_new[1] = g->lrn_d;
+  io.coef[0] = g->coef_g;
+  io.coef[1] = g->coef_d;
+  return io;
+}
+
+int select_impl(lipz_grid* g) {
+  if (g->phase != PH_EVALUATED)
+    return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
+  phase_begin(g, LIPZ_PHASE_SELECT);
+  launch_select(g->fG, g->fD, g->nbr, g->cells, select_params(g), select_io(g), g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_SELECT, 1);
   g->phase = PH_SELECTED;
@@ -988,7 +1017,7 @@ int lipz_set_data(lipz_grid* g, const float* host_pool, int64_t n_rows, int32_t 
 int lipz_eval_neighborhoods(lipz_grid* g, float* fit_g, float* fit_d, float* pair_lg,
                             float* pair_ld) {
   if (!g) return LIPZ_ERR_INVALID;
-  int rc = eval_impl(g, nullptr);
+  int rc = eval_impl(g, nullptr, false);
   if (rc) return rc;
   if (fit_g || fit_d || pair_lg || pair_ld) {
     const size_t C = g->cells;
@@ -1024,7 +1053,7 @@ int lipz_iterate(lipz_grid* g, int n_iters) {
   if (n_iters < 0) return fail(g, LIPZ_ERR_INVALID, "n_iters < 0");
   for (int i = 0; i < n_iters; ++i) {
     int rc;
-    if ((rc = eval_impl(g, nullptr)) || (rc = select_impl(g)) || (rc = train_impl(g))) return rc;
+    if ((rc = eval_impl(g, nullptr, true)) || (rc = train_impl(g))) return rc;
   }
   return LIPZ_OK;
 }
@@ -1035,7 +1064,7 @@ int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* f
   const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
   CK(g, cudaMemcpyAsync(g->xin, x_host, bytes, cudaMemcpyHostToDevice, g->st));
   int rc;
-  if ((rc = eval_impl(g, g->xin)) || (rc = select_impl(g)) || (rc = train_impl(g))) return rc;
+  if ((rc = eval_impl(g, g->xin, true)) || (rc = train_impl(g))) return rc;
   const size_t C = g->cells;
   if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
   if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));

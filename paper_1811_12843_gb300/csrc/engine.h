@@ -42,6 +42,17 @@ struct SelectParams {
   float beta1, beta2;
 };
 
+// Where selection reads the old snapshot and writes its results; index 0 = generator, 1 =
+// discriminator population.
+struct SelectIO {
+  const float* lr_old[2];
+  const int* step_old[2];
+  int* sel[2];
+  int* src[2];
+  float* lr_new[2];
+  float4* coef[2];
+};
+
 void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout& lay, int cells,
                         uint64_t seed, uint32_t stream, cudaStream_t st);
 void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st);
@@ -64,10 +75,12 @@ void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD,
 // Also writes, per cell and population, the Adam coefficients of the new centre's next step:
 // (lr, 1 / (1 - beta1^(step+1)), 1 / (1 - beta2^(step+1)), step + 1).
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
-                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old,
-                   const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
-                   int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
-                   float4* coef_d, cudaStream_t st);
+                   const SelectParams& p, const SelectIO& io, cudaStream_t st);
+// Fitness and, in the same kernel, the selection of every cell (when nothing is read back
+// between the two).
+void launch_fitness_select(const float* logits, int cells, int B, float* LG, float* LD,
+                           float* fG, float* fD, int* flag, const int* nbr,
+                           const SelectParams& p, const SelectIO& io, cudaStream_t st);
 template <typename T>
 void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int cells, int B,
                        int x_dim, cudaStream_t st);

@@ -347,13 +347,74 @@ template void launch_colsum<bf16>(const ColSumDesc*, int, int, cudaStream_t);
 // ------------------------------------------------------------------------------------------
 __device__ __forceinline__ float softplusf(float x) { return fmaxf(x, 0.f) + log1pf(expf(-fabsf(x))); }
 
+// ------------------------------------------------------------------------------------------
+// Tournament selection, replacement and learning-rate mutation: one thread per cell.
+// ------------------------------------------------------------------------------------------
+__device__ int tournament_slot(const float* f5, const uint32_t* w, int size) {
+  int remaining[5] = {0, 1, 2, 3, 4};
+  int left = 5, best = -1;
+  for (int m = 0; m < size; ++m) {
+    const int r = (int)mulhi_u32(w[m], (uint32_t)(5 - m));
+    const int e = remaining[r];
+    for (int q = r; q + 1 < left; ++q) remaining[q] = remaining[q + 1];
+    --left;
+    if (best < 0 || f5[e] < f5[best] || (f5[e] == f5[best] && e < best)) best = e;
+  }
+  return best;
+}
+
+__device__ float mutate(float lr, uint64_t seed, uint32_t stream, uint32_t t, uint32_t c,
+                        float std, uint64_t thr) {
+  const U4 r = philox_block(seed, stream, t, c, 0u);
+  if ((uint64_t)r.x >= thr) return lr;
+  const float n = box_muller(r.y, r.z).x;
+  return fmaxf(lr + std * n, 1e-8f);
+}
+
+// Tournament, replacement and lr mutation of population `pop` (0 G, 1 D) of cell c, given the
+// five fitnesses f5 of the cell's neighbourhood; writes the selection, the source individual,
+// the new lr and the Adam coefficients (lr, 1 / (1 - beta1^t), 1 / (1 - beta2^t), t).
+__device__ void select_one(int c, int pop, const float* f5, const int* __restrict__ nbr,
+                           const SelectParams& p, const SelectIO& io) {
+  const U4 a = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 0u);
+  const U4 b = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 1u);
+  const uint32_t w[5] = {a.x, a.y, a.z, a.w, b.x};
+  const int win = tournament_slot(f5, w, p.tournament_size);
+  const int s = p.replace_always ? win : (f5[win] < f5[0] ? win : 0);
+  const int src = nbr[c * 5 + s];
+  float lr = io.lr_old[pop][src];
+  if (p.lr_mutation)
+    lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std, p.lr_mut_thr);
+  const int step1 = io.step_old[pop][src] + 1;
+  // 1 - beta^t = -expm1(t * log1p(-(1 - beta))): 1 - beta is exact in fp32 for beta in
+  // [0.5, 1), and the expm1 form keeps full relative precision for beta^t near 1
+  const float bc1 = -expm1f((float)step1 * log1pf(-(1.f - p.beta1)));
+  const float bc2 = -expm1f((float)step1 * log1pf(-(1.f - p.beta2)));
+  io.coef[pop][c] = make_float4(lr, 1.f / bc1, 1.f / bc2, (float)step1);
+  io.sel[pop][c] = s;
+  io.src[pop][c] = src;
+  io.lr_new[pop][c] = lr;
+}
+
+__global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
+                         const int* __restrict__ nbr, int cells, SelectParams p, SelectIO io) {
+  pdl_wait();
+  const int gid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = gid >> 1;
+  if (c >= cells) return;
+  const int pop = gid & 1;
+  select_one(c, pop, (pop ? fD : fG) + c * 5, nbr, p, io);
+}
+
+template <bool SELECT>
 __global__ void k_fitness(const float* __restrict__ logits, int B, float* __restrict__ LG,
                           float* __restrict__ LD, float* __restrict__ fG, float* __restrict__ fD,
-                          int* __restrict__ flag) {
+                          int* __restrict__ flag, const int* __restrict__ nbr, SelectParams sp,
+                          SelectIO io) {
   pdl_wait();
   const int c = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  __shared__ float real_s[5], fake_d[25], fake_g[25];
+  __shared__ float real_s[5], fake_d[25], fake_g[25], f_s[10];
   const float* lc = logits + (int64_t)c * 5 * 6 * B;
   for (int task = warp; task < 30; task += nw) {
     float s1 = 0.f, s2 = 0.f;
@@ -401,90 +462,34 @@ __global__ void k_fitness(const float* __restrict__ logits, int B, float* __rest
     }
     fG[c * 5 + i] = sg / 5.f;
     fD[c * 5 + i] = sd / 5.f;
+    f_s[i] = sg / 5.f;
+    f_s[5 + i] = sd / 5.f;
+  }
+  if (SELECT) {
+    // the cell's tournaments follow at once: G in thread 0, D in thread 1
+    __syncthreads();
+    if (threadIdx.x < 2) select_one(c, threadIdx.x, f_s + 5 * threadIdx.x, nbr, sp, io);
   }
 }
 
 void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
                     float* fD, int* flag, cudaStream_t st) {
   // one warp per mean
-  launch_pdl(k_fitness, dim3(cells), dim3(960), 0, st, logits, B, LG, LD, fG, fD, flag);
+  launch_pdl(k_fitness<false>, dim3(cells), dim3(960), 0, st, logits, B, LG, LD, fG, fD, flag,
+             (const int*)nullptr, SelectParams{}, SelectIO{});
 }
 
-// ------------------------------------------------------------------------------------------
-// Tournament selection, replacement and learning-rate mutation: one thread per cell.
-// ------------------------------------------------------------------------------------------
-__device__ int tournament_slot(const float* f5, const uint32_t* w, int size) {
-  int remaining[5] = {0, 1, 2, 3, 4};
-  int left = 5, best = -1;
-  for (int m = 0; m < size; ++m) {
-    const int r = (int)mulhi_u32(w[m], (uint32_t)(5 - m));
-    const int e = remaining[r];
-    for (int q = r; q + 1 < left; ++q) remaining[q] = remaining[q + 1];
-    --left;
-    if (best < 0 || f5[e] < f5[best] || (f5[e] == f5[best] && e < best)) best = e;
-  }
-  return best;
-}
-
-__device__ float mutate(float lr, uint64_t seed, uint32_t stream, uint32_t t, uint32_t c,
-                        float std, uint64_t thr) {
-  const U4 r = philox_block(seed, stream, t, c, 0u);
-  if ((uint64_t)r.x >= thr) return lr;
-  const float n = box_muller(r.y, r.z).x;
-  return fmaxf(lr + std * n, 1e-8f);
-}
-
-__global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
-                         const int* __restrict__ nbr, int cells, SelectParams p,
-                         const float* __restrict__ lr_g_old, const float* __restrict__ lr_d_old,
-                         const int* __restrict__ step_g_old, const int* __restrict__ step_d_old,
-                         int* __restrict__ sel_g, int* __restrict__ sel_d, int* __restrict__ src_g,
-                         int* __restrict__ src_d, float* __restrict__ lr_g_new,
-                         float* __restrict__ lr_d_new, float4* __restrict__ coef_g,
-                         float4* __restrict__ coef_d) {
-  pdl_wait();
-  const int gid = blockIdx.x * blockDim.x + threadIdx.x;
-  const int c = gid >> 1;
-  if (c >= cells) return;
-  {
-    const int pop = gid & 1;
-    const float* f5 = (pop ? fD : fG) + c * 5;
-    const U4 a = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 0u);
-    const U4 b = philox_block(p.seed, pop ? 6u : 5u, p.t, (uint32_t)c, 1u);
-    const uint32_t w[5] = {a.x, a.y, a.z, a.w, b.x};
-    const int win = tournament_slot(f5, w, p.tournament_size);
-    const int s = p.replace_always ? win : (f5[win] < f5[0] ? win : 0);
-    const int src = nbr[c * 5 + s];
-    float lr = (pop ? lr_d_old : lr_g_old)[src];
-    if (p.lr_mutation) lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std,
-                                   p.lr_mut_thr);
-    const int step1 = (pop ? step_d_old : step_g_old)[src] + 1;
-    // 1 - beta^t = -expm1(t * log1p(-(1 - beta))): 1 - beta is exact in fp32 for beta in
-    // [0.5, 1), and the expm1 form keeps full relative precision for beta^t near 1
-    const float bc1 = -expm1f((float)step1 * log1pf(-(1.f - p.beta1)));
-    const float bc2 = -expm1f((float)step1 * log1pf(-(1.f - p.beta2)));
-    const float4 cf = make_float4(lr, 1.f / bc1, 1.f / bc2, (float)step1);
-    (pop ? coef_d : coef_g)[c] = cf;
-    if (pop) {
-      sel_d[c] = s;
-      src_d[c] = src;
-      lr_d_new[c] = lr;
-    } else {
-      sel_g[c] = s;
-      src_g[c] = src;
-      lr_g_new[c] = lr;
-    }
-  }
+void launch_fitness_select(const float* logits, int cells, int B, float* LG, float* LD,
+                           float* fG, float* fD, int* flag, const int* nbr,
+                           const SelectParams& p, const SelectIO& io, cudaStream_t st) {
+  launch_pdl(k_fitness<true>, dim3(cells), dim3(960), 0, st, logits, B, LG, LD, fG, fD, flag, nbr,
+             p, io);
 }
 
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
-                   const SelectParams& p, const float* lr_g_old, const float* lr_d_old,
-                   const int* step_g_old, const int* step_d_old, int* sel_g, int* sel_d,
-                   int* src_g, int* src_d, float* lr_g_new, float* lr_d_new, float4* coef_g,
-                   float4* coef_d, cudaStream_t st) {
+                   const SelectParams& p, const SelectIO& io, cudaStream_t st) {
   launch_pdl(k_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, fG, fD, nbr, cells, p,
-             lr_g_old, lr_d_old, step_g_old, step_d_old, sel_g, sel_d, src_g, src_d, lr_g_new,
-             lr_d_new, coef_g, coef_d);
+             io);
 }
 
 // ------------------------------------------------------------------------------------------

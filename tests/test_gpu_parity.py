@@ -212,6 +212,22 @@ def test_fused_adam_equals_stored_gradient_path(L, rows, cols, batch):
         assert a.export_state() == b.export_state(), it
 
 
+@pytest.mark.parametrize("precision", ["fp32", "bf16"])
+def test_iterate_equals_separate_calls(L, precision):
+    """lipz_iterate selects inside the fitness kernel; the result must equal, bit for bit, the
+    separate eval / select / train calls (mutation on, so the lr path is covered too)."""
+    pool = _pool(12, 3000, 784)
+    kw = dict(precision=precision, lr_mutation=1, lr_mut_prob=0.5, lr_mut_std=1e-4)
+    a = _grid(L, 3, 4, 5, pool, **kw)
+    b = _grid(L, 3, 4, 5, pool, **kw)
+    for it in range(2):
+        a.iterate(1)
+        b.eval()
+        b.select()
+        b.train()
+        assert a.export_state() == b.export_state(), it
+
+
 def test_selection_modes_and_mutation(L):
     pool = _pool(8, 4000, 784)
     g = _grid(L, 3, 4, 8, pool, keep_grads=1, tournament_size=5, replace_mode="always",
