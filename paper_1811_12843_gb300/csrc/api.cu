@@ -54,6 +54,9 @@ struct lipz_grid {
   int64_t e_cell = 0;  // elements per cell of the evaluation input E (6B rows)
   cudaStream_t st = nullptr;      // stream all work is enqueued on
   cudaStream_t own_st = nullptr;  // the grid's own non-blocking stream (the default)
+  cudaStream_t copy_st = nullptr;  // host minibatch uploads, overlapping the generator forward
+  cudaEvent_t ev_x = nullptr;      // the upload of the caller's minibatch has landed
+  int* hstat = nullptr;            // pinned host copies of the device error flags
   int device = 0;
   PopView G[2]{}, D[2]{};
   int cur = 0;
@@ -503,6 +506,9 @@ int create_impl(lipz_grid* g) {
   // the grid's own stream (lipz_set_stream may replace it)
   CK(g, cudaStreamCreateWithFlags(&g->own_st, cudaStreamNonBlocking));
   g->st = g->own_st;
+  CK(g, cudaStreamCreateWithFlags(&g->copy_st, cudaStreamNonBlocking));
+  CK(g, cudaEventCreateWithFlags(&g->ev_x, cudaEventDisableTiming));
+  CK(g, cudaMallocHost(&g->hstat, 8 * sizeof(int)));
   make_layouts(g);
   g->e_cell = (int64_t)6 * B * x;
   for (int p = 0; p < 2; ++p) {
@@ -628,19 +634,27 @@ SelectParams select_params(const lipz_grid* g);
 SelectIO select_io(lipz_grid* g);
 
 // Evaluation (minibatch, forwards, fitness); with `then_select` the selection runs in the
-// fitness kernel (the caller reads nothing back in between).
-int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select) {
+// fitness kernel (the caller reads nothing back in between). With `x_ready`, the caller's
+// minibatch xin_dev is still being uploaded: the noise and the generator forward go first,
+// the real rows are copied into place after the event.
+int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
+              cudaEvent_t x_ready = nullptr) {
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
   if (!xin_dev && g->pool_n <= 0)
     return fail(g, LIPZ_ERR_STATE, "no real-data pool: call lipz_set_data first");
   const int p = g->cur;
+  auto draw = [&](int parts, bool pdl) {
+    if (g->bf)
+      launch_draw_batch<bf16>((const bf16*)g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell,
+                              (bf16*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, parts, pdl,
+                              g->st);
+    else
+      launch_draw_batch<float>((const float*)g->pool, g->pool_n, xin_dev, (float*)g->E,
+                               g->e_cell, (float*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t,
+                               parts, pdl, g->st);
+  };
   phase_begin(g, LIPZ_PHASE_BATCH);
-  if (g->bf)
-    launch_draw_batch<bf16>((const bf16*)g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell,
-                            (bf16*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, g->st);
-  else
-    launch_draw_batch<float>((const float*)g->pool, g->pool_n, xin_dev, (float*)g->E, g->e_cell,
-                             (float*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, g->st);
+  draw(x_ready ? DRAW_NOISE : DRAW_REAL | DRAW_NOISE, true);
   CKL(g);
   phase_end(g, LIPZ_PHASE_BATCH, 1);
   if (g->use_tc) {
@@ -648,6 +662,11 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select) {
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);
+    if (x_ready) {
+      CK(g, cudaStreamWaitEvent(g->st, x_ready, 0));
+      draw(DRAW_REAL, false);
+      CKL(g);
+    }
     phase_begin(g, LIPZ_PHASE_D_FWD);
     if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_D_FWD, 1);
@@ -658,6 +677,11 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select) {
     gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
     phase_end(g, LIPZ_PHASE_G_FWD, 3);
+    if (x_ready) {
+      CK(g, cudaStreamWaitEvent(g->st, x_ready, 0));
+      draw(DRAW_REAL, false);
+      CKL(g);
+    }
     phase_begin(g, LIPZ_PHASE_D_FWD);
     gemm(g, D.d1, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
     gemm(g, D.d2, C * 5, 6 * B, h, EPI_BIAS_ACT, ACT_LRELU, false);
@@ -835,23 +859,28 @@ int train_impl(lipz_grid* g) {
   return LIPZ_OK;
 }
 
+// Waits for the grid's stream and reports a bounded wait that expired in a tensor-core kernel
+// or a non-finite loss seen since the last check (one synchronisation: all flags are copied
+// into pinned host memory first); the flags are reset.
 int check_flag(lipz_grid* g) {
-  for (int p = 0; p < 4; ++p) {
-    int* f = p < 2 ? (g->tc[p] ? tc_error_flag(g->tc[p]) : nullptr)
-                   : (g->tcb[p - 2] ? tcb_error_flag(g->tcb[p - 2]) : nullptr);
-    if (!f) continue;
-    int code = 0;
-    CK(g, cudaMemcpyAsync(&code, f, 4, cudaMemcpyDeviceToHost, g->st));
-    CK(g, cudaStreamSynchronize(g->st));
+  int* dev[5] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
+                 g->tc[1] ? tc_error_flag(g->tc[1]) : nullptr,
+                 g->tcb[0] ? tcb_error_flag(g->tcb[0]) : nullptr,
+                 g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr, g->flag};
+  for (int i = 0; i < 5; ++i) {
+    g->hstat[i] = i < 4 ? 0 : INT_MAX;
+    if (dev[i]) CK(g, cudaMemcpyAsync(&g->hstat[i], dev[i], 4, cudaMemcpyDeviceToHost, g->st));
+  }
+  CK(g, cudaStreamSynchronize(g->st));
+  for (int i = 0; i < 4; ++i) {
+    const int code = g->hstat[i];
     if (code) {
-      CK(g, cudaMemsetAsync(f, 0, 4, g->st));
+      CK(g, cudaMemsetAsync(dev[i], 0, 4, g->st));
       CK(g, cudaStreamSynchronize(g->st));
       return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
-  int v = INT_MAX;
-  CK(g, cudaMemcpyAsync(&v, g->flag, 4, cudaMemcpyDeviceToHost, g->st));
-  CK(g, cudaStreamSynchronize(g->st));
+  const int v = g->hstat[4];
   if (v != INT_MAX) {
     const int big = INT_MAX;
     int rc = h2d(g, g->flag, &big, 4);
@@ -958,6 +987,12 @@ int lipz_grid_destroy(lipz_grid* g) {
     if (e) cudaEventDestroy(e);
   for (void* p : g->allocs) cudaFree(p);
   if (g->own_st) cudaStreamDestroy(g->own_st);
+  if (g->copy_st) {
+    cudaStreamSynchronize(g->copy_st);
+    cudaStreamDestroy(g->copy_st);
+  }
+  if (g->ev_x) cudaEventDestroy(g->ev_x);
+  if (g->hstat) cudaFreeHost(g->hstat);
   delete g;
   return LIPZ_OK;
 }
@@ -1062,14 +1097,15 @@ int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* f
   if (!g) return LIPZ_ERR_INVALID;
   if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
   const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
-  CK(g, cudaMemcpyAsync(g->xin, x_host, bytes, cudaMemcpyHostToDevice, g->st));
+  // the upload runs on the copy stream while the noise and the generator forward compute
+  CK(g, cudaMemcpyAsync(g->xin, x_host, bytes, cudaMemcpyHostToDevice, g->copy_st));
+  CK(g, cudaEventRecord(g->ev_x, g->copy_st));
   int rc;
-  if ((rc = eval_impl(g, g->xin, true)) || (rc = train_impl(g))) return rc;
+  if ((rc = eval_impl(g, g->xin, true, g->ev_x)) || (rc = train_impl(g))) return rc;
   const size_t C = g->cells;
   if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
   if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
-  CK(g, cudaStreamSynchronize(g->st));
-  return check_flag(g);
+  return check_flag(g);  // one stream synchronisation for the results and the flags
 }
 
 int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {

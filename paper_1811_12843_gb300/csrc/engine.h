@@ -57,10 +57,13 @@ void launch_init_params(float* w, bf16* wb, int64_t P, int64_t Ps, const Layout&
                         uint64_t seed, uint32_t stream, cudaStream_t st);
 void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st);
 
+// parts: DRAW_REAL (the B real rows into E[c]), DRAW_NOISE (z into Z[c]), or both; pdl = false
+// keeps plain stream order (after an event wait).
+enum { DRAW_REAL = 1, DRAW_NOISE = 2 };
 template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
-                       cudaStream_t st);
+                       int parts, bool pdl, cudaStream_t st);
 
 template <typename TI, typename TO, int EPI>
 void launch_gemm(const GemmDesc* descs, int n_problems, int max_m, int max_n, int act,

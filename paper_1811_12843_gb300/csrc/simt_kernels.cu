@@ -80,13 +80,14 @@ template <typename T>
 __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
                              T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
-                             uint32_t t) {
+                             uint32_t t, int parts) {
   pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
   if (b >= B) return;
   T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
-  if (xin) {
+  if (!(parts & DRAW_REAL)) {
+  } else if (xin) {
     const float* src = xin + ((int64_t)c * B + b) * x_dim;
     const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
                      ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
@@ -112,6 +113,7 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
       for (int k = lane; k < x_dim; k += 32) dst[k] = src[k];
     }
   }
+  if (!(parts & DRAW_NOISE)) return;
   T* zr = Z + ((int64_t)c * B + b) * z_dim;
   const uint32_t n0 = (uint32_t)b * (uint32_t)z_dim;
   // normals n0 .. n0 + z_dim - 1; Philox block i holds normals 4i .. 4i + 3
@@ -139,15 +141,16 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
 template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
-                       cudaStream_t st) {
-  launch_pdl(k_draw_batch<T>, dim3((B + 7) / 8, cells), dim3(256), 0, st, pool, n_pool, xin, E,
-             e_cell, Z, B, x_dim, z_dim, seed, t);
+                       int parts, bool pdl, cudaStream_t st) {
+  launch_kernel(pdl, k_draw_batch<T>, dim3((B + 7) / 8, cells), dim3(256), 0, st, pool, n_pool,
+                xin, E, e_cell, Z, B, x_dim, z_dim, seed, t, parts);
 }
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
-                                       float*, int, int, int, int, uint64_t, uint32_t,
+                                       float*, int, int, int, int, uint64_t, uint32_t, int, bool,
                                        cudaStream_t);
 template void launch_draw_batch<bf16>(const bf16*, int64_t, const float*, bf16*, int64_t, bf16*,
-                                      int, int, int, int, uint64_t, uint32_t, cudaStream_t);
+                                      int, int, int, int, uint64_t, uint32_t, int, bool,
+                                      cudaStream_t);
 
 // ------------------------------------------------------------------------------------------
 // Grouped GEMM on CUDA cores: 64x64 output tile per block, k-slices of 16 staged in shared
