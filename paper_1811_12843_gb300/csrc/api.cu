@@ -36,8 +36,7 @@ struct Descs {
   // training (per parity): forward of the selected pair and its backward
   GemmDesc *tg1, *tg2, *td1, *td2, *bw2d, *bd1, *bw1d, *ba3, *bw3g, *ba2, *bw2g, *ba1, *bw1g;
   GemvDesc* tgv;
-  ColSumDesc *cb2d, *cb1d, *cb3g, *cb2g, *cb1g;
-  ColSumDesc* cb_all;  // the five above in one array (one launch)
+  ColSumDesc *cb1d, *cb3g, *cb2g, *cb1g;  // bias gradients (D's b2 comes from k_dlogit)
 };
 
 }  // namespace
@@ -313,7 +312,7 @@ int build_descs(lipz_grid* g, int p) {
   // ---- training descriptors: weights of the selected individual (wsel = src_g / src_d)
   std::vector<GemmDesc> tg1, tg2, td1, td2, bw2d, bd1, bw1d, ba3, bw3g, ba2, bw2g, ba1, bw1g;
   std::vector<GemvDesc> tgv;
-  std::vector<ColSumDesc> cb2d, cb1d, cb3g, cb2g, cb1g;
+  std::vector<ColSumDesc> cb1d, cb3g, cb2g, cb1g;
   auto selg = [&](GemmDesc d, int c) {
     d.wsel = g->src_g;
     d.wsel_stride = g->PGs;
@@ -379,7 +378,6 @@ int build_descs(lipz_grid* g, int p) {
     tgv.push_back(v);
     // discriminator backward
     bw2d.push_back(gd(J2c, 1, h, TG1c, h, 1, gDc + M.off[2], h, 1, h, h, 2 * B));
-    cb2d.push_back(cs(J2c, gDc + M.off[3], h, 2 * B, h));
     a = seld(gd(J2c, h, 1, eoff(Dw, M.off[2], es), h, 1, D1c, h, 1, 2 * B, h, h), c);
     a.aux = TG1c;
     a.sxm = h;
@@ -424,13 +422,10 @@ int build_descs(lipz_grid* g, int p) {
       (rc = upload(g, &D.ba3, ba3)) || (rc = upload(g, &D.bw3g, bw3g)) ||
       (rc = upload(g, &D.ba2, ba2)) || (rc = upload(g, &D.bw2g, bw2g)) ||
       (rc = upload(g, &D.ba1, ba1)) || (rc = upload(g, &D.bw1g, bw1g)) ||
-      (rc = upload(g, &D.cb2d, cb2d)) || (rc = upload(g, &D.cb1d, cb1d)) ||
+      (rc = upload(g, &D.cb1d, cb1d)) ||
       (rc = upload(g, &D.cb3g, cb3g)) || (rc = upload(g, &D.cb2g, cb2g)) ||
       (rc = upload(g, &D.cb1g, cb1g)))
     return rc;
-  std::vector<ColSumDesc> all;
-  for (auto* v : {&cb2d, &cb1d, &cb3g, &cb2g, &cb1g}) all.insert(all.end(), v->begin(), v->end());
-  if ((rc = upload(g, &D.cb_all, all))) return rc;
   return LIPZ_OK;
 }
 
@@ -777,23 +772,22 @@ int train_impl(lipz_grid* g) {
   if (g->bf)
     launch_dlogit<bf16>(g->TL, (const bf16*)g->TG2, g->D[p].wb, g->PDs, g->ld.off[4], g->src_d, C,
                         B, h, g->a.leaky_slope, (bf16*)g->J2, g->gD, g->PDs, g->ld.off[4],
-                        g->ld.off[5], g->st);
+                        g->ld.off[5], g->ld.off[3], g->st);
   else
     launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
-                         g->ld.off[5], g->st);
+                         g->ld.off[5], g->ld.off[3], g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_TRAIN_FWD, n_fwd + 1);
   phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
   if (g->use_tcb) {
     // the nine backward products of every cell in one launch (with Adam on the weight
-    // matrices unless the gradients are kept), then the bias column sums
+    // matrices unless the gradients are kept; the bias gradients summed in its epilogue)
     std::string msg;
     if (tcb_run_cells(g->tcb[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     CKL(g);
     phase_end(g, LIPZ_PHASE_TRAIN_BWD, 1);
     phase_begin(g, LIPZ_PHASE_ADAM);
-    colsum(g, D.cb_all, 5 * C, h > x ? h : x);
     if (!g->a.keep_grads) {
       // the weight matrices took their Adam step inside the backward: the biases and D's
       // output layer remain
@@ -820,7 +814,7 @@ int train_impl(lipz_grid* g) {
       }
       launch_adam_ranges(rg, rd, C, g->a.beta1, g->a.beta2, g->a.eps, g->st);
       CKL(g);
-      phase_end(g, LIPZ_PHASE_ADAM, 2);
+      phase_end(g, LIPZ_PHASE_ADAM, 1);
       g->cur = 1 - p;
       g->t += 1;
       g->phase = PH_IDLE;
@@ -828,7 +822,6 @@ int train_impl(lipz_grid* g) {
     }
   } else {
     gemm(g, D.bw2d, C, h, h, EPI_STORE, ACT_NONE, true);
-    colsum(g, D.cb2d, C, h);
     gemm(g, D.bd1, 2 * C, 2 * B, h, EPI_DACT, ACT_LRELU, false);
     gemm(g, D.bw1d, C, h, x, EPI_STORE, ACT_NONE, true);
     colsum(g, D.cb1d, C, h);
@@ -843,7 +836,7 @@ int train_impl(lipz_grid* g) {
     gemm(g, D.bw1g, C, h, z, EPI_STORE, ACT_NONE, true);
     colsum(g, D.cb1g, C, h);
     CKL(g);
-    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 16);
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, 15);
     phase_begin(g, LIPZ_PHASE_ADAM);
   }
   // Adam + replacement into the other snapshot (after the bias sums on the tensor-core path)
@@ -852,7 +845,7 @@ int train_impl(lipz_grid* g) {
   launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
   CKL(g);
-  phase_end(g, LIPZ_PHASE_ADAM, g->use_tcb ? 3 : 2);
+  phase_end(g, LIPZ_PHASE_ADAM, 2);
   g->cur = 1 - p;
   g->t += 1;
   g->phase = PH_IDLE;

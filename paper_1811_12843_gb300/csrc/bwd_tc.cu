@@ -33,6 +33,8 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int MN_BOX_BYTES = 64 * BK * 2;   // one {64 MN, 64 K} box
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int EPI_THREADS = 32 * NUM_EPI_WARPS;
+// bias-gradient partial sums: [2 tiles][4 TMEM lane quarters][256 columns] fp32
+constexpr int BIAS_PART_BYTES = 2 * 4 * 256 * 4;
 // fused Adam: a chunk is 64 rows (one half of a tile) x 32 fp32 columns of each of w, m, v (one
 // 128-byte row each, 128-byte swizzle), updated in place, plus the new bf16 copy (64-byte rows,
 // no swizzle). Chunks alternate between the two row halves, so each half of the epilogue
@@ -50,7 +52,8 @@ struct Cfg {
   static constexpr int STAGES = FUSED ? 2 : 4;
   static constexpr int ADAM_BUFS = FUSED ? 4 : 0;
   static constexpr int THREADS = 64 + EPI_THREADS + (FUSED ? 32 : 0);
-  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + ADAM_BUFS * ADAM_BUF_BYTES + 256;
+  static constexpr int SMEM =
+      1024 + STAGES * STAGE_BYTES + ADAM_BUFS * ADAM_BUF_BYTES + 256 + BIAS_PART_BYTES;
 };
 
 enum { EPI_F32 = 0, EPI_DACT = 1, EPI_ADAM = 2 };
@@ -79,6 +82,11 @@ struct GParams {
   const bf16* aux;
   int64_t aux_cell, sxm, sxn;
   int aux_wrap_at, aux_wrap_sub;  // aux row of m: m < wrap_at ? m : m - wrap_sub
+  // EPI_DACT: column sums of the fp32 deltas over rows m < bias_rows go to
+  // bias_out[cell * bias_cell + n] (a bias gradient); null = none
+  float* bias_out;
+  int64_t bias_cell;
+  int bias_rows;
   AdamRef adam;
   int* err;
 };
@@ -133,7 +141,8 @@ __device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int
 // 16 accumulator columns of one row: fp32 store, or bf16 delta times the activation
 // derivative (read from the stored forward output). `full` = all 16 columns lie inside N.
 __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16], int cell, int m,
-                                      int arow, int col0, bool full, float dlo, bool is_tanh) {
+                                      int arow, int col0, bool full, float dlo, bool is_tanh,
+                                      float (&vout)[16]) {
   if (p.epi == EPI_F32) {
     float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
     if (p.scn == 1) {
@@ -172,8 +181,9 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
       const float y0 = __low2float(y2), y1 = __high2float(y2);
       const float d0 = is_tanh ? 1.f - y0 * y0 : (y0 > 0.f ? 1.f : dlo);
       const float d1 = is_tanh ? 1.f - y1 * y1 : (y1 > 0.f ? 1.f : dlo);
-      __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(r[e]) * d0,
-                                                __uint_as_float(r[e + 1]) * d1);
+      vout[e] = __uint_as_float(r[e]) * d0;
+      vout[e + 1] = __uint_as_float(r[e + 1]) * d1;
+      __nv_bfloat162 b2 = __floats2bfloat162_rn(vout[e], vout[e + 1]);
       pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
     }
     uint4* o = reinterpret_cast<uint4*>(C + col0);
@@ -186,12 +196,37 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
     if (col >= p.N) break;
     const float y = __bfloat162float(X[(int64_t)col * p.sxn]);
     const float d = is_tanh ? 1.f - y * y : (y > 0.f ? 1.f : dlo);
-    C[(int64_t)col * p.scn] = __float2bfloat16_rn(__uint_as_float(r[e]) * d);
+    vout[e] = __uint_as_float(r[e]) * d;
+    C[(int64_t)col * p.scn] = __float2bfloat16_rn(vout[e]);
   }
 }
 
-__device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0, int n0, int n,
-                                              uint32_t tbase, int hf, int row) {
+// Sum of v over the 32 lanes of a warp for 16 columns, reduce-scattered: lanes 2j and 2j + 1
+// return the sum of column j. Each partial sum is formed by one lane, in a fixed order.
+__device__ __forceinline__ float warp_colsum16(const float (&v)[16], int lane) {
+  float a8[8], a4[4], a2[2];
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    a8[i] = (b4 ? v[8 + i] : v[i]) + __shfl_xor_sync(0xffffffffu, b4 ? v[i] : v[8 + i], 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    a4[i] = (b3 ? a8[4 + i] : a8[i]) + __shfl_xor_sync(0xffffffffu, b3 ? a8[i] : a8[4 + i], 8);
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+    a2[i] = (b2 ? a4[2 + i] : a4[i]) + __shfl_xor_sync(0xffffffffu, b2 ? a4[i] : a4[2 + i], 4);
+  const float a1 = (b1 ? a2[1] : a2[0]) + __shfl_xor_sync(0xffffffffu, b1 ? a2[0] : a2[1], 2);
+  return a1 + __shfl_xor_sync(0xffffffffu, a1, 1);
+}
+
+// Epilogue of one tile: warp (q, hf) owns TMEM lane quarter q (rows 32q .. 32q + 31) and column
+// half hf. With a bias output, the column sums of the tile's fp32 deltas over the counted rows
+// go through warp_colsum16 and shared memory (one partial per lane quarter, double-buffered by
+// bias tile) and are added in a fixed order into bias_out (stored by the first row tile).
+__device__ __forceinline__ bool epilogue_tile(const GParams& p, int cell, int m0, int n0, int n,
+                                              uint32_t tbase, int hf, int row, int q, int lane,
+                                              float* bpart, int& btile, uint32_t bSum,
+                                              volatile int* abort_flag, int* err) {
   const int m = m0 + row;
   const int ng = n / 16;
   const int half = (ng + 1) / 2;
@@ -200,26 +235,78 @@ __device__ __forceinline__ void epilogue_tile(const GParams& p, int cell, int m0
   const int arow = m < p.aux_wrap_at ? m : m - p.aux_wrap_sub;
   const bool is_tanh = p.act == ACT_TANH;
   const float dlo = p.act == ACT_RELU ? 0.f : p.slope;
+  const bool bias = p.epi == EPI_DACT && p.bias_out != nullptr;
+  const bool brow = row_ok && m < p.bias_rows;
+  float* bp = bpart + (btile & 1) * (4 * 256) + q * 256;
   int gi = g0;
   // two 16-column groups per TMEM load where possible
   for (; gi + 1 < g1; gi += 2) {
     uint32_t r[32];
     LIPZ_TMEM_LD32(tbase + gi * 16, r);
     tmem_wait_ld();
-    if (!row_ok) continue;
     const int col0 = n0 + gi * 16;
     const uint32_t(&ra)[16] = *reinterpret_cast<const uint32_t(*)[16]>(&r[0]);
     const uint32_t(&rb)[16] = *reinterpret_cast<const uint32_t(*)[16]>(&r[16]);
-    epi16(p, ra, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh);
-    if (col0 + 16 < p.N) epi16(p, rb, cell, m, arow, col0 + 16, col0 + 32 <= p.N, dlo, is_tanh);
+    float va[16], vb[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) va[e] = vb[e] = 0.f;
+    if (row_ok) {
+      epi16(p, ra, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va);
+      if (col0 + 16 < p.N)
+        epi16(p, rb, cell, m, arow, col0 + 16, col0 + 32 <= p.N, dlo, is_tanh, vb);
+    }
+    if (bias) {
+      if (!brow) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) va[e] = vb[e] = 0.f;
+      }
+      const float s0 = warp_colsum16(va, lane), s1 = warp_colsum16(vb, lane);
+      if (!(lane & 1)) {
+        bp[gi * 16 + (lane >> 1)] = s0;
+        bp[(gi + 1) * 16 + (lane >> 1)] = s1;
+      }
+    }
   }
   if (gi < g1) {
     uint32_t r[16];
     LIPZ_TMEM_LD16(tbase + gi * 16, r);
     tmem_wait_ld();
     const int col0 = n0 + gi * 16;
-    if (row_ok && col0 < p.N) epi16(p, r, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh);
+    float va[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) va[e] = 0.f;
+    if (row_ok && col0 < p.N) epi16(p, r, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va);
+    if (bias) {
+      if (!brow) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) va[e] = 0.f;
+      }
+      const float s0 = warp_colsum16(va, lane);
+      if (!(lane & 1)) bp[gi * 16 + (lane >> 1)] = s0;
+    }
   }
+  if (bias) {
+    // once every epilogue thread has written its partials (mbarrier bSum[btile & 1]), the
+    // lane-quarter-0 warp of each column half adds the four quarters (fixed order) into the
+    // running sum over row tiles. A buffer is rewritten two bias tiles later, which needs the
+    // TMEM region that this tile's readers (those warps included) release after this.
+    const uint32_t bar = bSum + 8 * (btile & 1);
+    mbar_arrive(bar);
+    if (q == 0) {
+      if (!mbar_wait_warp(bar, (uint32_t)((btile >> 1) & 1), abort_flag, err, 20)) return false;
+      const float* b0 = bpart + (btile & 1) * (4 * 256);
+      for (int col = g0 * 16 + lane; col < g1 * 16; col += 32) {
+        const int gc = n0 + col;
+        if (gc < p.N) {
+          const float t = ((b0[col] + b0[256 + col]) + b0[512 + col]) + b0[768 + col];
+          float* o = p.bias_out + (int64_t)cell * p.bias_cell + gc;
+          *o = m0 == 0 ? t : *o + t;
+        }
+      }
+    }
+    ++btile;
+  }
+  return true;
 }
 
 // Adam epilogue of one weight-gradient tile: for each 32-column chunk of the thread's row half
@@ -317,9 +404,11 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
   const uint32_t bEpi = bFinal + 8;    // [2], alternating by tile
   const uint32_t aFull = bEpi + 16;   // [4] Adam chunk buffers: old values landed
   const uint32_t aDone = aFull + 32;  // [4] new values written back by the epilogue half
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 192);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 196);
-  volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 200);
+  const uint32_t bSum = aDone + 32;   // [2] bias partial sums written, by bias tile
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 224);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 228);
+  volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 232);
+  float* bpart = reinterpret_cast<float*>(misc + 256);  // bias partial sums
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -338,6 +427,8 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
       mbar_init(aFull + 8 * b, 1);
       mbar_init(aDone + 8 * b, EPI_THREADS / 2);
     }
+    mbar_init(bSum, EPI_THREADS);
+    mbar_init(bSum + 8, EPI_THREADS);
     *abort_flag = 0;
     *done_tiles = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -567,6 +658,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     bool ok = true;
     int lt = 0, pub = 0;
     int cj = 0;  // Adam chunks of this thread's row half so far
+    int btile = 0;  // bias-summing tiles so far
     for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
       for (int si = 0; si < cp.n_stages && ok; ++si) {
         const GParams& p = cp.st[si].p;
@@ -589,11 +681,15 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
                 ok = false;
                 break;
               }
-            } else {
-              epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+            } else if (!epilogue_tile(p, cell, m0, n0, n, tbase, hf, row, q, lane, bpart, btile,
+                                      bSum, abort_flag, err)) {
+              ok = false;
+              break;
             }
-          } else {
-            epilogue_tile(p, cell, m0, n0, n, tbase, hf, row);
+          } else if (!epilogue_tile(p, cell, m0, n0, n, tbase, hf, row, q, lane, bpart, btile,
+                                    bSum, abort_flag, err)) {
+            ok = false;
+            break;
           }
           if (publish) {
             // publish the tile's global stores to the async proxy (a later stage loads them by
@@ -821,6 +917,9 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.sxn = 1;
     G.p.aux_wrap_at = 2 * B;
     G.p.aux_wrap_sub = B;
+    G.p.bias_out = b.gD + b.doff[1];  // D's b1: rows of the D loss
+    G.p.bias_cell = b.PDs;
+    G.p.bias_rows = 2 * B;
     ok = ok && map3(&G.a, b.J2, h, 3 * B, C, (uint64_t)3 * B * h, 128, msg) &&
          map3(&G.b, Dw + b.doff[2], h, h, NI, b.PDs, 64, msg);
     finish(G);
@@ -857,6 +956,9 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.scn = 1;
     G.p.aux = (const bf16*)b.TX + (int64_t)B * x;
     G.p.aux_cell = (int64_t)2 * B * x;
+    G.p.bias_out = b.gG + b.goff[5];  // G's b3
+    G.p.bias_cell = b.PGs;
+    G.p.bias_rows = B;
     G.p.sxm = x;
     G.p.sxn = 1;
     ok = ok && map3(&G.a, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 128, msg) &&
@@ -894,6 +996,9 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.scn = 1;
     G.p.aux = (const bf16*)b.TH2;
     G.p.aux_cell = (int64_t)B * h;
+    G.p.bias_out = b.gG + b.goff[3];  // G's b2
+    G.p.bias_cell = b.PGs;
+    G.p.bias_rows = B;
     G.p.sxm = h;
     G.p.sxn = 1;
     ok = ok && map3(&G.a, b.A3, x, B, C, (uint64_t)B * x, 128, msg) &&
@@ -930,6 +1035,9 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.scn = 1;
     G.p.aux = (const bf16*)b.TH1;
     G.p.aux_cell = (int64_t)B * h;
+    G.p.bias_out = b.gG + b.goff[1];  // G's b1
+    G.p.bias_cell = b.PGs;
+    G.p.bias_rows = B;
     G.p.sxm = h;
     G.p.sxn = 1;
     ok = ok && map3(&G.a, b.A2, h, B, C, (uint64_t)B * h, 128, msg) &&

@@ -90,7 +90,8 @@ void launch_train_prep(const T* E, int64_t e_cell, const int* sel_g, T* TX, int 
 template <typename T>
 void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
                    const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
-                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st);
+                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, int64_t off_gb2,
+                   cudaStream_t st);
 void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, const int* src,
                  const float4* coef, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
                  float eps, cudaStream_t st);

@@ -541,15 +541,17 @@ __global__ void __launch_bounds__(1024) k_dlogit(
     const float* __restrict__ TL, const T* __restrict__ TG2, const T* __restrict__ wD,
     int64_t wD_stride, int64_t off_w3, const int* __restrict__ src_d, int B, int H, float slope,
     T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride, int64_t off_gw3,
-    int64_t off_gb3) {
+    int64_t off_gb3, int64_t off_gb2) {
   pdl_wait();
   // Lanes own column groups of 8 (threads of the block: H / 8 groups x RG row groups); the RG
-  // partial sums of dW3 are added in a fixed order.
-  extern __shared__ float dl[];  // [3B] deltas, then [RG][H] partial sums
+  // partial sums of dW3 and of db2 (the column sums of J2 over the D-loss rows) are added in a
+  // fixed order.
+  extern __shared__ float dl[];  // [3B] deltas, then [RG][H] and [RG][H] partial sums
   const int c = blockIdx.x;
   const int ng = (H + 7) / 8;
   const int RG = blockDim.x / ng;
   float* part = dl + 3 * B;
+  float* part2 = part + RG * H;
   const float* l = TL + (int64_t)c * 2 * B;
   for (int r = threadIdx.x; r < 3 * B; r += blockDim.x) {
     const float x = r < 2 * B ? l[r] : l[r - B];
@@ -562,11 +564,12 @@ __global__ void __launch_bounds__(1024) k_dlogit(
   const T* w3 = wD + (int64_t)src_d[c] * wD_stride + off_w3;
   const T* g2 = TG2 + (int64_t)c * 2 * B * H;
   T* j2 = J2 + (int64_t)c * 3 * B * H;
-  float wk[8], acc[8];
+  float wk[8], acc[8], acc2[8];
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     wk[e] = k0 + e < H ? to_f<T>(w3[k0 + e]) : 0.f;
     acc[e] = 0.f;
+    acc2[e] = 0.f;
   }
   if (rg < RG) {
     const bool vec = sizeof(T) == 2 && (H & 7) == 0;
@@ -582,12 +585,15 @@ __global__ void __launch_bounds__(1024) k_dlogit(
         for (int e = 0; e < 4; ++e) {
           const __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&w[e]);
           const float g0 = __low2float(v), g1 = __high2float(v);
-          __nv_bfloat162 y = __floats2bfloat162_rn(dr * wk[2 * e] * (g0 > 0.f ? 1.f : slope),
-                                                   dr * wk[2 * e + 1] * (g1 > 0.f ? 1.f : slope));
+          const float y0 = dr * wk[2 * e] * (g0 > 0.f ? 1.f : slope);
+          const float y1 = dr * wk[2 * e + 1] * (g1 > 0.f ? 1.f : slope);
+          __nv_bfloat162 y = __floats2bfloat162_rn(y0, y1);
           o[e] = *reinterpret_cast<uint32_t*>(&y);
           if (r < 2 * B) {
             acc[2 * e] = fmaf(dr, g0, acc[2 * e]);
             acc[2 * e + 1] = fmaf(dr, g1, acc[2 * e + 1]);
+            acc2[2 * e] += y0;
+            acc2[2 * e + 1] += y1;
           }
         }
         *reinterpret_cast<uint4*>(j2 + (int64_t)r * H + k0) = make_uint4(o[0], o[1], o[2], o[3]);
@@ -596,21 +602,32 @@ __global__ void __launch_bounds__(1024) k_dlogit(
         for (int e = 0; e < 8; ++e) {
           if (k0 + e >= H) break;
           const float gv = to_f<T>(g2[(int64_t)rr * H + k0 + e]);
-          j2[(int64_t)r * H + k0 + e] = from_f<T>(dr * wk[e] * (gv > 0.f ? 1.f : slope));
-          if (r < 2 * B) acc[e] = fmaf(dr, gv, acc[e]);
+          const float yv = dr * wk[e] * (gv > 0.f ? 1.f : slope);
+          j2[(int64_t)r * H + k0 + e] = from_f<T>(yv);
+          if (r < 2 * B) {
+            acc[e] = fmaf(dr, gv, acc[e]);
+            acc2[e] += yv;
+          }
         }
       }
     }
 #pragma unroll
     for (int e = 0; e < 8; ++e)
-      if (k0 + e < H) part[rg * H + k0 + e] = acc[e];
+      if (k0 + e < H) {
+        part[rg * H + k0 + e] = acc[e];
+        part2[rg * H + k0 + e] = acc2[e];
+      }
   }
   __syncthreads();
   float* g = gD + (int64_t)c * gD_stride;
   for (int k = threadIdx.x; k < H; k += blockDim.x) {
-    float t = 0.f;
-    for (int q = 0; q < RG; ++q) t += part[q * H + k];
+    float t = 0.f, t2 = 0.f;
+    for (int q = 0; q < RG; ++q) {
+      t += part[q * H + k];
+      t2 += part2[q * H + k];
+    }
     g[off_gw3 + k] = t;
+    g[off_gb2 + k] = t2;
   }
   if (threadIdx.x == 0) {
     float t = 0.f;
@@ -622,22 +639,23 @@ __global__ void __launch_bounds__(1024) k_dlogit(
 template <typename T>
 void launch_dlogit(const float* TL, const T* TG2, const T* wD, int64_t wD_stride, int64_t off_w3,
                    const int* src_d, int cells, int B, int H, float slope, T* J2, float* gD,
-                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, cudaStream_t st) {
+                   int64_t gD_stride, int64_t off_gw3, int64_t off_gb3, int64_t off_gb2,
+                   cudaStream_t st) {
   const int ng = (H + 7) / 8;
   int rg = 512 / ng;
   if (rg < 1) rg = 1;
   if (rg > 16) rg = 16;
   const int threads = ((rg * ng + 31) / 32) * 32;
-  const size_t smem = (3 * (size_t)B + (size_t)(threads / ng) * H) * sizeof(float);
+  const size_t smem = (3 * (size_t)B + 2 * (size_t)(threads / ng) * H) * sizeof(float);
   launch_pdl(k_dlogit<T>, dim3(cells), dim3(threads), smem, st, TL, TG2, wD, wD_stride, off_w3,
-             src_d, B, H, slope, J2, gD, gD_stride, off_gw3, off_gb3);
+             src_d, B, H, slope, J2, gD, gD_stride, off_gw3, off_gb3, off_gb2);
 }
 template void launch_dlogit<float>(const float*, const float*, const float*, int64_t, int64_t,
                                    const int*, int, int, int, float, float*, float*, int64_t,
-                                   int64_t, int64_t, cudaStream_t);
+                                   int64_t, int64_t, int64_t, cudaStream_t);
 template void launch_dlogit<bf16>(const float*, const bf16*, const bf16*, int64_t, int64_t,
                                   const int*, int, int, int, float, bf16*, float*, int64_t,
-                                  int64_t, int64_t, cudaStream_t);
+                                  int64_t, int64_t, int64_t, cudaStream_t);
 
 // ------------------------------------------------------------------------------------------
 // Adam (Kingma & Ba 2015, Algorithm 1) fused with the replacement copy: the new centre of
