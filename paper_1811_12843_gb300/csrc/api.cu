@@ -561,7 +561,7 @@ int create_impl(lipz_grid* g) {
       b.Dw = g->D[p].w;
       b.PDs = g->PDs;
       b.doff = g->ld.off;
-      b.TX = g->TX;
+      b.sel_g = g->sel_g;
       b.src_g = g->src_g;
       b.src_d = g->src_d;
       b.TH1 = g->TH1;
@@ -578,7 +578,9 @@ int create_impl(lipz_grid* g) {
       TcbShape s{C, B, z, h, x, g->a.leaky_slope, C};
       TcbBuffers b{};
       b.Z = g->Z;
-      b.TX = g->TX;
+      b.E = g->E;
+      b.e_cell = g->e_cell;
+      b.sel_g = g->sel_g;
       b.TH1 = g->TH1;
       b.TH2 = g->TH2;
       b.TG1 = g->TG1;
@@ -748,13 +750,19 @@ int train_impl(lipz_grid* g) {
   const int p = g->cur;
   const Descs& D = g->dsc[p];
   phase_begin(g, LIPZ_PHASE_TRAIN_FWD);
-  if (g->bf)
-    launch_train_prep<bf16>((const bf16*)g->E, g->e_cell, g->sel_g, (bf16*)g->TX, C, B, x, g->st);
-  else
-    launch_train_prep<float>((const float*)g->E, g->e_cell, g->sel_g, (float*)g->TX, C, B, x,
-                             g->st);
+  // the CUDA-core kernels read the discriminator's training input as one array TX; the
+  // tensor-core kernels read it from E in place
+  int n_fwd = 0;
+  if (!(g->use_tc && g->use_tcb)) {
+    if (g->bf)
+      launch_train_prep<bf16>((const bf16*)g->E, g->e_cell, g->sel_g, (bf16*)g->TX, C, B, x,
+                              g->st);
+    else
+      launch_train_prep<float>((const float*)g->E, g->e_cell, g->sel_g, (float*)g->TX, C, B, x,
+                               g->st);
+    n_fwd = 1;
+  }
   // forward of the selected pair
-  int n_fwd = 1;
   if (g->use_tc) {
     std::string msg;
     if (tc_run_train_g(g->tc[p], g->st, &msg) || tc_run_train_d(g->tc[p], g->st, &msg))

@@ -82,6 +82,13 @@ struct GParams {
   const bf16* aux;
   int64_t aux_cell, sxm, sxn;
   int aux_wrap_at, aux_wrap_sub;  // aux row of m: m < wrap_at ? m : m - wrap_sub
+  const int* aux_sel;             // non-null: aux also advances (1 + aux_sel[cell]) * aux_sel_stride
+  int64_t aux_sel_stride;
+  // split K (ksplit > 0): chunks [0, ksplit) read K rows kc * 64 of A and of B's slot 0;
+  // chunks [ksplit, kchunks) read K rows (kc - ksplit) * 64 of A shifted by a_k_off1 and of B's
+  // slot 1 + b_slot_sel[cell]; B is then a 4-D map {n, K rows, slots, cells}
+  int ksplit, a_k_off1;
+  const int* b_slot_sel;
   // EPI_DACT: column sums of the fp32 deltas over rows m < bias_rows go to
   // bias_out[cell * bias_cell + n] (a bias gradient); null = none
   float* bias_out;
@@ -170,6 +177,7 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
   }
   bf16* C = reinterpret_cast<bf16*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
   const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
+  if (p.aux_sel) X += (int64_t)(1 + __ldg(&p.aux_sel[cell])) * p.aux_sel_stride;
   if (p.sxn == 1 && p.scn == 1 && full) {
     const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
     const uint4 q0 = x4[0], q1 = x4[1];
@@ -499,13 +507,20 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
               const uint32_t full = bFull + 8 * stage;
               mbar_expect_tx(full, (uint32_t)A_BYTES + b_bytes);
               const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+              const bool part1 = p.ksplit > 0 && kc >= p.ksplit;
+              const int kk = part1 ? kc - p.ksplit : kc;
+              const int ka = kk * BK + (part1 ? p.a_k_off1 : 0);
               if (p.a_mn) {
-                tma_load_3d(sA, mA, full, m0, kc * BK, za);
-                tma_load_3d(sA + MN_BOX_BYTES, mA, full, m0 + 64, kc * BK, za);
+                tma_load_3d(sA, mA, full, m0, ka, za);
+                tma_load_3d(sA + MN_BOX_BYTES, mA, full, m0 + 64, ka, za);
               } else {
-                tma_load_3d(sA, mA, full, kc * BK, p.a_row0 + m0, za);
+                tma_load_3d(sA, mA, full, ka, p.a_row0 + m0, za);
               }
-              if (p.b_mn) {
+              if (p.ksplit > 0) {
+                const int slot = part1 ? 1 + __ldg(&p.b_slot_sel[cell]) : 0;
+                for (int i = 0; i < p.BN / 64; ++i)
+                  tma_load_4d(sB + i * MN_BOX_BYTES, mB, full, n0 + 64 * i, kk * BK, slot, cell);
+              } else if (p.b_mn) {
                 for (int i = 0; i < p.BN / 64; ++i)
                   tma_load_3d(sB + i * MN_BOX_BYTES, mB, full, n0 + 64 * i, kc * BK, zb);
               } else {
@@ -805,6 +820,24 @@ bool map3b_rows(CUtensorMap* m, const bf16* base, uint64_t inner, uint64_t rows,
   return true;
 }
 
+// bf16 4-D map {inner, rows, slots, depth} (E seen as [cells][6][B][x]); box {64, 64, 1, 1},
+// 128-byte swizzle: rows past `rows` within a slot read as zero.
+bool map4(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t slots,
+          uint64_t depth, uint64_t slot_elems, uint64_t depth_elems, std::string* msg) {
+  cuuint64_t dims[4] = {inner, rows, slots, depth};
+  cuuint64_t strides[3] = {inner * 2, slot_elems * 2, depth_elems * 2};
+  cuuint32_t box[4] = {64, 64, 1, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (4-D) failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
 struct Gemm {
   CUtensorMap a, b;
   CUtensorMap aw, am, av;      // old w, m, v of the tensor (fused Adam), by individual
@@ -954,8 +987,10 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.c_cell = (int64_t)B * x;
     G.p.scm = x;
     G.p.scn = 1;
-    G.p.aux = (const bf16*)b.TX + (int64_t)B * x;
-    G.p.aux_cell = (int64_t)2 * B * x;
+    G.p.aux = (const bf16*)b.E;  // the selected generator's fakes: E[c] slot 1 + sel_g[c]
+    G.p.aux_cell = b.e_cell;
+    G.p.aux_sel = b.sel_g;
+    G.p.aux_sel_stride = (int64_t)B * x;
     G.p.bias_out = b.gG + b.goff[5];  // G's b3
     G.p.bias_cell = b.PGs;
     G.p.bias_rows = B;
@@ -965,11 +1000,17 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
          map3(&G.b, Dw + b.doff[0], x, h, NI, b.PDs, 64, msg);
     finish(G);
   }
-  // 4. dW1d[o][i] = sum_{r < 2B} D1[r][o] TX[r][i]: M = o = 256, N = i = x, K = 2B (TX ends
-  //    at 2B)
+  // 4. dW1d[o][i] = sum_{r < 2B} D1[r][o] X[r][i]: M = o = 256, N = i = x, K = 2B, where X =
+  //    [E[c] rows 0..B-1 (real); E[c] fake rows of slot sel_g[c]] read in place: K splits into
+  //    the two B-row parts (rows past B in a part read as zero), D1 rows shifted by B in the
+  //    second part
   {
     Gemm& G = P->g[i++];
     G.p = base_params(h, x, 2 * B, 256);
+    G.p.kchunks = 2 * ((B + 63) / 64);
+    G.p.ksplit = (B + 63) / 64;
+    G.p.a_k_off1 = B;
+    G.p.b_slot_sel = b.sel_g;
     G.p.a_mn = 1;
     G.p.b_mn = 1;
     G.p.epi = tcb::EPI_F32;
@@ -979,7 +1020,7 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.scn = 1;
     fuse(G, b.adam_d, b.src_d, b.doff[0], b.PDs);
     ok = ok && map3(&G.a, b.D1, h, 3 * B, C, (uint64_t)3 * B * h, 64, msg) &&
-         map3(&G.b, b.TX, x, 2 * B, C, (uint64_t)2 * B * x, 64, msg);
+         map4(&G.b, b.E, x, B, 6, C, (uint64_t)B * x, (uint64_t)b.e_cell, msg);
     finish(G);
   }
   // 5. A2 = (A3 @ W3g) * relu'(TH2): M = B, N = 256, K = x

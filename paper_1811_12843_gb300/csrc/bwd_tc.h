@@ -18,7 +18,8 @@ struct TcbShape {
 };
 
 // Buffers (bf16 unless noted) of one population snapshot:
-//   Z [cells][B][z]; TX [cells][2B][x] (real rows, then the selected fakes);
+//   Z [cells][B][z]; E [cells][6B][x] (the discriminator's training input is E[c] rows
+//   [0, B) and the fake rows of slot sel_g[c], read in place);
 //   TH1, TH2 [cells][B][256] and TG1 [cells][2B][256]: stored forward activations;
 //   J2 [cells][3B][256]: logit deltas through D's last layer (rows: real, fake for L_D, fake
 //   for L_G); D1 [cells][3B][256], A3 [cells][B][x], A2, A1 [cells][B][256]: deltas written
@@ -26,7 +27,10 @@ struct TcbShape {
 //   Gwb, Dwb: bf16 weight copies with tensor offsets goff / doff; src_g, src_d: the individual
 //   each cell trains.
 struct TcbBuffers {
-  const void *Z, *TX, *TH1, *TH2, *TG1, *J2;
+  const void *Z, *TH1, *TH2, *TG1, *J2;
+  const void* E;        // [cells][6B][x]: real rows, then the fakes of slots 0..4
+  int64_t e_cell;
+  const int* sel_g;     // slot of each cell's selected generator (its fakes in E)
   void *D1, *A3, *A2, *A1;
   float *gG, *gD;
   const __nv_bfloat16 *Gwb, *Dwb;

@@ -74,6 +74,10 @@ struct KParams {
   const int* wsel;
   bf16* act1;
   bf16* act2;
+  // two-part training problems (non-null): problem 2c + part of cell c takes B rows of E[c],
+  // slot 0 (the real rows) or slot 1 + part_slot[c] (the selected generator's fakes), through
+  // a 4-D map {x, B, 6, cells}
+  const int* part_slot;
 };
 
 struct Job {
@@ -113,7 +117,8 @@ __device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
   return p.train ? prob : prob / 5;
 }
 __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
-  return p.train ? __ldg(&p.wsel[prob]) : __ldg(&p.nbr[prob]);
+  if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
+  return __ldg(&p.nbr[prob]);
 }
 
 // Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
@@ -207,7 +212,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t full = bFull + 8 * stage;
             mbar_expect_tx(full, bytes);
             const uint32_t sA = sStage + stage * STAGE_BYTES;
-            if (!J.a_from_h) tma_load_3d(sA, &mA, full, kc * BK, m0, c);
+            if (J.a_from_h) {
+            } else if (p.part_slot) {
+              const int cell = prob >> 1;
+              const int slot = (prob & 1) ? 1 + __ldg(&p.part_slot[cell]) : 0;
+              tma_load_4d(sA, &mA, full, kc * BK, m0, slot, cell);
+            } else {
+              tma_load_3d(sA, &mA, full, kc * BK, m0, c);
+            }
             tma_load_3d(sA + A_BYTES, mb, full, kc * BK, J.brow0, k);
             issued[stage]++;
             if (++stage == STAGES) {
@@ -510,7 +522,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // ---- host side -----------------------------------------------------------------------------
 struct TcPlan {
   TcShape s;
-  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mTX;
+  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mE4;
   tc::KParams pg, pd, pgt, pdt;
   int grid_g, grid_d, grid_gt, grid_dt;
   int* err;
@@ -553,6 +565,26 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, u
   return true;
 }
 
+// bf16 4-D map {inner, rows, slots, depth}; box {64, 128, 1, 1}, 128-byte swizzle: rows past
+// `rows` within a slot read as zero.
+bool make_map4(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t slots,
+               uint64_t depth, uint64_t row_bytes, uint64_t slot_bytes, uint64_t depth_bytes,
+               std::string* msg) {
+  cuuint64_t dims[4] = {inner, rows, slots, depth};
+  cuuint64_t strides[3] = {row_bytes, slot_bytes, depth_bytes};
+  cuuint32_t box[4] = {64, (cuuint32_t)tc::BM, 1, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (4-D) failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
 }  // namespace
 
 bool tc_supported(int z, int h, int x, int B) {
@@ -572,7 +604,7 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   const uint64_t C = s.cells, B = s.B, z = s.z, x = s.x, h = s.h;
   bool ok = make_map(&p->mZ, b.Z, z, B, C, z * 2, B * z * 2, 128, msg) &&
             make_map(&p->mE, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 128, msg) &&
-            make_map(&p->mTX, b.TX, x, 2 * B, C, x * 2, 2 * B * x * 2, 128, msg) &&
+            make_map4(&p->mE4, b.E, x, B, 6, C, x * 2, B * x * 2, (uint64_t)b.e_cell * 2, msg) &&
             make_map(&p->mG1, b.Gwb + b.goff[0], z, h, C, z * 2, b.PGs * 2, 256, msg) &&
             make_map(&p->mG2, b.Gwb + b.goff[2], h, h, C, h * 2, b.PGs * 2, 256, msg) &&
             make_map(&p->mG3, b.Gwb + b.goff[4], h, x, C, h * 2, b.PGs * 2, tc::N3, msg) &&
@@ -645,12 +677,13 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   gt.n_tiles = s.cells * g.mtiles;
   gt.act1 = (bf16*)b.TH1;
   gt.act2 = (bf16*)b.TH2;
-  tc::KParams dt = d;  // selected discriminator on [x_c; selected fakes]
+  tc::KParams dt = d;  // selected discriminator on [x_c; selected fakes], read from E
   dt.train = 1;
   dt.wsel = b.src_d;
-  dt.rows = 2 * s.B;
-  dt.mtiles = tiles(2 * s.B);
-  dt.n_tiles = s.cells * dt.mtiles;
+  dt.part_slot = b.sel_g;
+  dt.rows = s.B;
+  dt.mtiles = tiles(s.B);
+  dt.n_tiles = s.cells * 2 * dt.mtiles;
   dt.act1 = (bf16*)b.TG1;
   dt.act2 = (bf16*)b.TG2;
   dt.logits = b.TL;
@@ -695,7 +728,7 @@ int tc_run_train_g(TcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int tc_run_train_d(TcPlan* p, cudaStream_t st, std::string* msg) {
-  return launch(p->grid_dt, p->mTX, p->mD1, p->mD2, p->mD2, p->pdt, st,
+  return launch(p->grid_dt, p->mE4, p->mD1, p->mD2, p->mD2, p->pdt, st,
                 "discriminator training forward", msg);
 }
 

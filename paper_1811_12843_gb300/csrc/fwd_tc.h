@@ -26,8 +26,8 @@ bool tc_supported(int z, int h, int x, int B);
 //   0..4, which the generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5].
 //   Weights: bf16 copies (Gwb, Dwb) and fp32 masters (biases), per-individual strides
 //   PGs / PDs, tensor offsets goff / doff (W1, b1, W2, b2, W3, b3).
-//   Training forward of the selected pairs: TX [cells][2B][x] bf16 (real rows, then the
-//   selected generator's fakes), src_g / src_d [cells] (selected individuals), outputs
+//   Training forward of the selected pairs: the discriminator reads E[c] rows [0, B) and the
+//   fakes of slot sel_g[c] in place, src_g / src_d [cells] (selected individuals), outputs
 //   TH1, TH2 [cells][B][256], TG1, TG2 [cells][2B][256] bf16 and TL [cells][2B] fp32.
 struct TcBuffers {
   void* Z;
@@ -43,7 +43,7 @@ struct TcBuffers {
   const float* Dw;
   int64_t PDs;
   const int64_t* doff;
-  void* TX;
+  const int* sel_g;  // slot of each cell's selected generator (training: its fakes in E)
   const int* src_g;
   const int* src_d;
   void *TH1, *TH2, *TG1, *TG2;
