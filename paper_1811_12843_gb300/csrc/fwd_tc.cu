@@ -321,16 +321,27 @@ __global__ void __launch_bounds__(THREADS, 1)
       // reach tile ltile + 2 before every thread has passed this tile's arrival.
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
       {
+        // every load is issued before the first is stored, so their latencies overlap
         const int nb3 = p.kind == KIND_D ? HID + 1 : p.x;
-        for (int i = et; i < 512 + nb3; i += 256) {
-          float v;
-          if (i < 256) v = wm[p.off_b1 + i];
-          else if (i < 512) v = wm[p.off_b2 + i - 256];
+        constexpr int NV = (BIAS_MAX + 32 * NUM_EPI_WARPS - 1) / (32 * NUM_EPI_WARPS);
+        float v[NV];
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+          const int i = et + u * 32 * NUM_EPI_WARPS;
+          v[u] = 0.f;
+          if (i >= 512 + nb3) continue;
+          if (i < 256) v[u] = wm[p.off_b1 + i];
+          else if (i < 512) v[u] = wm[p.off_b2 + i - 256];
           else if (p.kind == KIND_D)
-            v = i < 512 + HID ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
-                              : wm[p.off_b3];
-          else v = wm[p.off_b3 + i - 512];
-          sb[i] = v;
+            v[u] = i < 512 + HID
+                       ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
+                       : wm[p.off_b3];
+          else v[u] = wm[p.off_b3 + i - 512];
+        }
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+          const int i = et + u * 32 * NUM_EPI_WARPS;
+          if (i < 512 + nb3) sb[i] = v[u];
         }
         mbar_arrive(bBias + 8 * (ltile & 1));
         if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
