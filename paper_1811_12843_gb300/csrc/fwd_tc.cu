@@ -146,8 +146,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t bFull = smem_u32(bars), bEmpty = bFull + 8 * STAGES;
   const uint32_t bAcc = bEmpty + 8 * STAGES;                    // [2]
   const uint32_t bReg = bAcc + 16;                              // [2]
-  const uint32_t bH = bReg + 16;
-  const uint32_t bPart = bH + 8;
+  const uint32_t bH = bReg + 16;      // [4]: 64-column chunk c of the activation is written
+  const uint32_t bPart = bH + 32;
   const uint32_t bFinal = bPart + 8;
   const uint32_t bBias = bFinal + 8;  // [2]: the tile's biases are in shared memory
   float* s_bias = reinterpret_cast<float*>(misc + MISC_BYTES);  // [2][BIAS_MAX]
@@ -165,7 +165,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(bAcc + 8, 1);
     mbar_init(bReg, 32 * NUM_EPI_WARPS);
     mbar_init(bReg + 8, 32 * NUM_EPI_WARPS);
-    mbar_init(bH, 32 * NUM_EPI_WARPS);
+    for (int c = 0; c < HID / BK; ++c) mbar_init(bH + 8 * c, 32 * NUM_EPI_WARPS);
     mbar_init(bPart, 32 * NUM_EPI_WARPS / 2);
     mbar_init(bFinal, 1);
     mbar_init(bBias, 32 * NUM_EPI_WARPS);
@@ -244,7 +244,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       int reg_uses[2] = {0, 0};
-      int h_total = 0, h_seen = 0;
+      int h_total = 0;  // activations written to H so far (each chunk barrier: one phase each)
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         for (int j = 0; j < nj && ok; ++j) {
@@ -255,20 +255,17 @@ __global__ void __launch_bounds__(THREADS, 1)
             ok = false;
             break;
           }
-          if (J.a_from_h) {
-            while (h_seen < h_total) {
-              if (!mbar_wait(bH, (uint32_t)(h_seen & 1), abort_flag, p.err, 3)) {
-                ok = false;
-                break;
-              }
-              ++h_seen;
-            }
-            if (!ok) break;
-          }
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(R * HID);
           const uint32_t idesc = idesc_bf16(BM, J.n);
           for (int kc = 0; kc < J.kchunks; ++kc) {
+            // a layer reading the on-chip activation starts on chunk kc as soon as the epilogue
+            // has written that chunk (write number h_total - 1)
+            if (J.a_from_h &&
+                !mbar_wait(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
+              ok = false;
+              break;
+            }
             if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 4)) {
               ok = false;
               break;
@@ -364,16 +361,15 @@ __global__ void __launch_bounds__(THREADS, 1)
           const bool lrelu = p.kind == KIND_D;
           const bool to_h = J.epi == EPI_TO_H;
           bf16* gout = j == 0 ? p.act1 : p.act2;
+          // chunk by chunk (64 columns, both column halves at once), so that the next layer's
+          // MMAs can start on chunk 0 while the epilogue still writes chunks 1..3
 #pragma unroll 1
-          for (int cp = hf * 4; cp < hf * 4 + 4; cp += 2) {
-            uint32_t r2[2][32];
-            LIPZ_TMEM_LD32(tbase + cp * 32, r2[0]);
-            LIPZ_TMEM_LD32(tbase + (cp + 1) * 32, r2[1]);
-            tmem_wait_ld();
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-              const int cg = cp + h2;
-              const uint32_t(&r)[32] = r2[h2];
+          for (int ch = 0; ch < HID / BK; ++ch) {
+            {
+              const int cg = 2 * ch + hf;  // this warp's 32 columns of the chunk
+              uint32_t r[32];
+              LIPZ_TMEM_LD32(tbase + cg * 32, r);
+              tmem_wait_ld();
               const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
               uint32_t pk[16];
 #pragma unroll
@@ -410,11 +406,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                   o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
               }
             }
+            if (to_h) {
+              asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+              mbar_arrive(bH + 8 * ch);
+            }
           }
-          if (to_h) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           tc_fence_before();
           mbar_arrive(bReg + 8 * R);
-          if (to_h) mbar_arrive(bH);
         } else if (J.epi == EPI_LOGIT) {
           const float* bias = sb + 256;
           const float* w3 = sb + 512;
