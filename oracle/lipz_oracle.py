@@ -24,7 +24,11 @@ Readings where the paper is silent (each is listed in the design doc with its reason)
     by the winner only if the winner's fitness is strictly lower (``if_better``) -- or always;
   * the pair is trained on the same minibatch that was used for its evaluation, with the fake
     batch detached for the discriminator gradient and both gradients taken at the pre-update
-    parameters; one Adam step (Kingma & Ba 2015, Algorithm 1) per iteration;
+    parameters; one Adam step (Kingma & Ba 2015, Algorithm 1) per iteration by default;
+  * with ``train_steps`` K > 1 (an iteration read as an epoch of K minibatch steps, Section 4's
+    footnote equating iteration, generation and epoch), steps k = 1..K-1 train the cell's new
+    centre pair again, each on a fresh minibatch drawn from the step-k streams (stream id +
+    256 k); selection and lr mutation happen once, before step 0;
   * random draws come from Philox4x32-10 (Salmon et al., SC'11) keyed by the seed, with the
     counter (block index, cell, iteration, stream);
   * in bf16 mode every operand of a matrix product (weights, activations, back-propagated
@@ -64,6 +68,8 @@ STREAM_TOUR_G = 5
 STREAM_TOUR_D = 6
 STREAM_MUT_G = 7
 STREAM_MUT_D = 8
+# Minibatch step k of an iteration draws from stream id + STEP_STREAM_STRIDE * k.
+STEP_STREAM_STRIDE = 256
 
 
 def philox4x32_10(ctr: np.ndarray, key: Tuple[int, int]) -> np.ndarray:
@@ -146,6 +152,7 @@ class Arch:
     lr_mut_std: float = 1e-4  # mutation rate (Table 1)
     lr_mut_prob: float = 0.5  # mutation probability (Table 1)
     leaky_slope: float = 0.2
+    train_steps: int = 1      # Adam steps of the new centre pair per iteration
 
 
 def g_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
@@ -321,14 +328,16 @@ def create(rows: int, cols: int, arch: Arch, seed: int) -> State:
                  np.zeros(cells, np.int64), np.full(cells, lr))
 
 
-def draw_batch(seed: int, t: int, cell: int, pool: np.ndarray, arch: Arch
+def draw_batch(seed: int, t: int, cell: int, pool: np.ndarray, arch: Arch, step: int = 0
                ) -> Tuple[np.ndarray, np.ndarray]:
-    """Cell ``cell``'s minibatch at iteration ``t``: B pool rows at indices mulhi(word_b, n)
-    (stream BATCH) and z = B x z_dim normals (stream NOISE), row-major."""
-    w = draw_words(seed, STREAM_BATCH, t, cell, arch.batch)
+    """Cell ``cell``'s minibatch at iteration ``t``, minibatch step ``step``: B pool rows at
+    indices mulhi(word_b, n) (stream BATCH + 256 step) and z = B x z_dim normals (stream
+    NOISE + 256 step), row-major."""
+    off = STEP_STREAM_STRIDE * step
+    w = draw_words(seed, STREAM_BATCH + off, t, cell, arch.batch)
     idx = mulhi(w, pool.shape[0]).astype(np.int64)
     x = pool[idx].astype(np.float64)
-    z = draw_normals(seed, STREAM_NOISE, t, cell, arch.batch * arch.z_dim)
+    z = draw_normals(seed, STREAM_NOISE + off, t, cell, arch.batch * arch.z_dim)
     return x, z.reshape(arch.batch, arch.z_dim)
 
 
@@ -500,9 +509,13 @@ def adam_step(w, m, v, step, g, lr, arch: Arch):
     return w - lr * mhat / (np.sqrt(vhat) + arch.eps), m1, v1, t1
 
 
-def train_step(state: State, sel, data, keep_grads: bool = False):
+def train_step(state: State, sel, data, keep_grads: bool = False,
+               pool: Optional[np.ndarray] = None):
     """Every cell's new centre pair (the selected slots' individuals with their optimiser state)
-    takes one Adam step on the cell's minibatch. Reads only the snapshot ``state``."""
+    takes one Adam step on the cell's minibatch, reading only the snapshot ``state``; with
+    ``arch.train_steps`` K > 1 it then takes K-1 more steps, step k on the cell's fresh step-k
+    minibatch from ``pool``, each at the parameters the previous step left (no selection and no
+    lr mutation in between). The kept gradients are the last step's."""
     a = state.arch
     nbr = neighbors(state.rows, state.cols)
     new = state.copy()
@@ -524,6 +537,18 @@ def train_step(state: State, sel, data, keep_grads: bool = False):
             state.Dw[sd], state.Dm[sd], state.Dv[sd], state.Dstep[sd], gD, lr_d, a)
         new.Glr[c], new.Dlr[c] = lr_g, lr_d
         grads["gG"][c], grads["gD"][c] = gG, gD
+    if a.train_steps > 1 and pool is None:
+        raise ValueError("train_steps > 1 draws its later minibatches from the pool")
+    for k in range(1, a.train_steps):
+        for c in range(state.cells):
+            x, z = draw_batch(state.seed, state.t, c, pool, a, k)
+            gG, gD, info = pair_gradients(new.Gw[c], new.Dw[c], x, z, a)
+            grads["kink"][c] = info["kink"]
+            new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c] = adam_step(
+                new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c], gG, new.Glr[c], a)
+            new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c] = adam_step(
+                new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c], gD, new.Dlr[c], a)
+            grads["gG"][c], grads["gD"][c] = gG, gD
     new.t = state.t + 1
     return (new, grads) if keep_grads else new
 
@@ -537,7 +562,7 @@ def iterate(state: State, pool: Optional[np.ndarray], n_iters: int = 1,
         data = batches(state, pool, x_host)
         ev = eval_neighborhoods(state, data)
         sel = select_replace(state, ev)
-        state = train_step(state, sel, data)
+        state = train_step(state, sel, data, pool=pool)
         if record:
             log.append({"eval": ev, "sel": sel})
     return (state, log) if record else state

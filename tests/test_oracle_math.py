@@ -237,3 +237,58 @@ def test_training_lowers_the_pair_losses():
     F = O.g_forward(O.unflatten(G, O.g_layout(arch)), z, arch)["F"]
     assert _losses_for(G, D1, x, z, arch, F)[1] < losses["LD"]
     assert _losses_for(G1, D, x, z, arch)[0] < losses["LG"]
+
+
+def _torch_adam_step(w, m, v, step, g, lr, arch):
+    """One step of torch.optim.Adam resumed from (m, v, step) (an independent implementation)."""
+    p = torch.tensor(np.array(w, np.float64), requires_grad=True)
+    opt = torch.optim.Adam([p], lr=float(lr), betas=(arch.beta1, arch.beta2), eps=arch.eps)
+    opt.state[p] = {"step": torch.tensor(float(step)),
+                    "exp_avg": torch.tensor(np.array(m, np.float64)),
+                    "exp_avg_sq": torch.tensor(np.array(v, np.float64))}
+    p.grad = torch.tensor(np.array(g, np.float64))
+    opt.step()
+    st = opt.state[p]
+    return (p.detach().numpy(), st["exp_avg"].numpy(), st["exp_avg_sq"].numpy(),
+            int(st["step"].item()))
+
+
+@pytest.mark.parametrize("mutation", [False, True])
+def test_later_minibatch_steps_continue_adam_on_fresh_batches(mutation):
+    """K = 3 minibatch steps per iteration equal the K = 1 iteration followed, in every cell, by
+    two steps of torch.optim.Adam (moments, step count and the cell's lr carried over) on torch
+    autograd gradients of the cell's own pair, on the minibatch of streams BATCH + 256 k and
+    NOISE + 256 k; selection and the lr mutation happen once."""
+    kw = dict(lr=1e-3, lr_mutation=mutation, lr_mut_std=1e-4, lr_mut_prob=0.5)
+    s = _tiny_state(rows=2, cols=3, seed=3, **kw)
+    s3 = _tiny_state(rows=2, cols=3, seed=3, train_steps=3, **kw)
+    pool = np.random.default_rng(2).uniform(-1, 1, size=(40, 5))
+    one = O.iterate(s, pool, 1)
+    three = O.iterate(s3, pool, 1)
+    a = s.arch
+    for c in range(s.cells):
+        G = (one.Gw[c], one.Gm[c], one.Gv[c], int(one.Gstep[c]))
+        D = (one.Dw[c], one.Dm[c], one.Dv[c], int(one.Dstep[c]))
+        for k in (1, 2):
+            idx = O.mulhi(O.draw_words(3, 3 + 256 * k, 0, c, a.batch), pool.shape[0])
+            x = pool[idx.astype(np.int64)]
+            z = O.draw_normals(3, 4 + 256 * k, 0, c, a.batch * a.z_dim).reshape(a.batch, -1)
+            gG, gD = _torch_grads(G[0], D[0], x, z, a)
+            G = _torch_adam_step(*G, gG, one.Glr[c], a)
+            D = _torch_adam_step(*D, gD, one.Dlr[c], a)
+        for got, ref in ((three.Gw[c], G[0]), (three.Gm[c], G[1]), (three.Gv[c], G[2]),
+                         (three.Dw[c], D[0]), (three.Dm[c], D[1]), (three.Dv[c], D[2])):
+            assert np.allclose(got, ref, rtol=1e-11, atol=1e-15)
+        assert three.Gstep[c] == G[3] == 3 and three.Dstep[c] == D[3] == 3
+        assert three.Glr[c] == one.Glr[c] and three.Dlr[c] == one.Dlr[c]
+    assert three.t == 1
+
+
+def test_later_minibatch_steps_draw_fresh_batches():
+    """Step k's minibatch comes from its own streams: no two steps of a cell share their noise,
+    and step 0 is the evaluation minibatch."""
+    a = O.Arch(**TINY)
+    pool = np.random.default_rng(0).uniform(-1, 1, size=(1000, 5))
+    zs = [O.draw_batch(7, 4, 1, pool, a, k)[1] for k in range(3)]
+    assert np.array_equal(zs[0], O.draw_batch(7, 4, 1, pool, a)[1])
+    assert not np.array_equal(zs[0], zs[1]) and not np.array_equal(zs[1], zs[2])
