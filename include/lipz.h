@@ -66,6 +66,9 @@ enum {
   LIPZ_STREAM_INIT_G = 1, LIPZ_STREAM_INIT_D = 2, LIPZ_STREAM_BATCH = 3, LIPZ_STREAM_NOISE = 4,
   LIPZ_STREAM_TOUR_G = 5, LIPZ_STREAM_TOUR_D = 6, LIPZ_STREAM_MUT_G = 7, LIPZ_STREAM_MUT_D = 8
 };
+/* Minibatch step k of an iteration draws its batch from stream LIPZ_STREAM_BATCH + stride * k and
+ * its noise from LIPZ_STREAM_NOISE + stride * k (k = 0 is the evaluation minibatch). */
+enum { LIPZ_STEP_STREAM_STRIDE = 256 };
 
 /*
  * Architecture and hyper-parameters (Table 1, MLP column). Fill with lipz_arch_default and
@@ -100,6 +103,12 @@ typedef struct lipz_arch {
   int32_t keep_grads;      /* 1: keep the last train step's gradients for lipz_get_gradients */
   int32_t force_simt;      /* 1: run the forward on the CUDA-core kernels even where the
                               tensor-core kernels apply (for comparisons) */
+  int32_t train_steps;     /* K >= 1 (default 1): Adam steps of each cell's new centre pair per
+                              iteration. Step 0 uses the evaluation minibatch; step k >= 1
+                              trains the pair again, in place, on a fresh minibatch drawn from
+                              the pool with stream ids + LIPZ_STEP_STREAM_STRIDE * k (also when
+                              the caller supplied step 0's real rows); selection and the lr
+                              mutation happen once, before step 0. K <= 65536. */
 } lipz_arch;
 
 typedef struct lipz_grid lipz_grid;

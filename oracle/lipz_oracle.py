@@ -515,7 +515,8 @@ def train_step(state: State, sel, data, keep_grads: bool = False,
     takes one Adam step on the cell's minibatch, reading only the snapshot ``state``; with
     ``arch.train_steps`` K > 1 it then takes K-1 more steps, step k on the cell's fresh step-k
     minibatch from ``pool``, each at the parameters the previous step left (no selection and no
-    lr mutation in between). The kept gradients are the last step's."""
+    lr mutation in between). The kept gradients are the last step's; ``kink`` is the closest
+    approach of any step's pre-activations to 0."""
     a = state.arch
     nbr = neighbors(state.rows, state.cols)
     new = state.copy()
@@ -543,7 +544,7 @@ def train_step(state: State, sel, data, keep_grads: bool = False,
         for c in range(state.cells):
             x, z = draw_batch(state.seed, state.t, c, pool, a, k)
             gG, gD, info = pair_gradients(new.Gw[c], new.Dw[c], x, z, a)
-            grads["kink"][c] = info["kink"]
+            grads["kink"][c] = min(grads["kink"][c], info["kink"])
             new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c] = adam_step(
                 new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c], gG, new.Glr[c], a)
             new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c] = adam_step(

@@ -50,6 +50,7 @@ class lipz_arch(ctypes.Structure):
         ("lr_mutation", ctypes.c_int32), ("lr_mut_std", ctypes.c_float),
         ("lr_mut_prob", ctypes.c_float), ("leaky_slope", ctypes.c_float),
         ("keep_grads", ctypes.c_int32), ("force_simt", ctypes.c_int32),
+        ("train_steps", ctypes.c_int32),
     ]
 
 

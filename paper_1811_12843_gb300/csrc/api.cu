@@ -474,6 +474,8 @@ int check_arch(const lipz_arch* a) {
       !(a->beta2 >= 0.f && a->beta2 < 1.f) || !(a->eps > 0.f) || !(a->lr_mut_prob >= 0.f) ||
       !(a->lr_mut_prob <= 1.f))
     return fail(nullptr, LIPZ_ERR_INVALID, "bad optimiser / mutation hyper-parameters");
+  if (a->train_steps < 1 || a->train_steps > 65536)
+    return fail(nullptr, LIPZ_ERR_INVALID, "train_steps must be in 1..65536");
   return LIPZ_OK;
 }
 
@@ -630,6 +632,20 @@ int create_impl(lipz_grid* g) {
 SelectParams select_params(const lipz_grid* g);
 SelectIO select_io(lipz_grid* g);
 
+// Minibatch step `step` of the current iteration into E's real rows and Z (the real rows from
+// xin_dev when given, else from the pool).
+void draw_batch(lipz_grid* g, const float* xin_dev, uint32_t step, int parts, bool pdl) {
+  const int C = g->cells, B = g->a.batch, x = g->a.x_dim, z = g->a.z_dim;
+  if (g->bf)
+    launch_draw_batch<bf16>((const bf16*)g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell,
+                            (bf16*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, step, parts, pdl,
+                            g->st);
+  else
+    launch_draw_batch<float>((const float*)g->pool, g->pool_n, xin_dev, (float*)g->E, g->e_cell,
+                             (float*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, step, parts, pdl,
+                             g->st);
+}
+
 // Evaluation (minibatch, forwards, fitness); with `then_select` the selection runs in the
 // fitness kernel (the caller reads nothing back in between). With `x_ready`, the caller's
 // minibatch xin_dev is still being uploaded: the noise and the generator forward go first,
@@ -640,16 +656,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
   if (!xin_dev && g->pool_n <= 0)
     return fail(g, LIPZ_ERR_STATE, "no real-data pool: call lipz_set_data first");
   const int p = g->cur;
-  auto draw = [&](int parts, bool pdl) {
-    if (g->bf)
-      launch_draw_batch<bf16>((const bf16*)g->pool, g->pool_n, xin_dev, (bf16*)g->E, g->e_cell,
-                              (bf16*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t, parts, pdl,
-                              g->st);
-    else
-      launch_draw_batch<float>((const float*)g->pool, g->pool_n, xin_dev, (float*)g->E,
-                               g->e_cell, (float*)g->Z, C, B, x, z, g->seed, (uint32_t)g->t,
-                               parts, pdl, g->st);
-  };
+  auto draw = [&](int parts, bool pdl) { draw_batch(g, xin_dev, 0, parts, pdl); };
   phase_begin(g, LIPZ_PHASE_BATCH);
   draw(x_ready ? DRAW_NOISE : DRAW_REAL | DRAW_NOISE, true);
   CKL(g);
@@ -743,9 +750,9 @@ int select_impl(lipz_grid* g) {
   return LIPZ_OK;
 }
 
-int train_impl(lipz_grid* g) {
-  if (g->phase != PH_SELECTED)
-    return fail(g, LIPZ_ERR_STATE, "lipz_train_step must follow lipz_select_replace");
+// One Adam step of every cell's chosen pair (sel/src/coef) from snapshot cur into the other
+// snapshot, which becomes cur.
+int train_once(lipz_grid* g) {
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
   const int p = g->cur;
   const Descs& D = g->dsc[p];
@@ -824,8 +831,6 @@ int train_impl(lipz_grid* g) {
       CKL(g);
       phase_end(g, LIPZ_PHASE_ADAM, 1);
       g->cur = 1 - p;
-      g->t += 1;
-      g->phase = PH_IDLE;
       return LIPZ_OK;
     }
   } else {
@@ -855,6 +860,49 @@ int train_impl(lipz_grid* g) {
   CKL(g);
   phase_end(g, LIPZ_PHASE_ADAM, 2);
   g->cur = 1 - p;
+  return LIPZ_OK;
+}
+
+// Minibatch step k >= 1 of the iteration: a fresh minibatch, every cell's own centre chosen
+// again (same lr, next Adam step), the centres' fakes, then one Adam step.
+int train_again(lipz_grid* g, uint32_t k) {
+  const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim;
+  phase_begin(g, LIPZ_PHASE_BATCH);
+  draw_batch(g, nullptr, k, DRAW_REAL | DRAW_NOISE, true);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_BATCH, 1);
+  phase_begin(g, LIPZ_PHASE_SELECT);
+  launch_centre_select(C, select_params(g), select_io(g), g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_SELECT, 1);
+  phase_begin(g, LIPZ_PHASE_G_FWD);
+  if (g->use_tc) {
+    std::string msg;
+    if (tc_run_g_centre(g->tc[g->cur], g->st, &msg))
+      return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_G_FWD, 1);
+  } else {
+    // the CUDA-core kernels run the generators of all five slots (slot 0 is the one used)
+    const Descs& D = g->dsc[g->cur];
+    gemm(g, D.g1, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
+    gemm(g, D.g3, C * 5, B, x, EPI_BIAS_ACT, ACT_TANH, false);
+    phase_end(g, LIPZ_PHASE_G_FWD, 3);
+  }
+  CKL(g);
+  return train_once(g);
+}
+
+int train_impl(lipz_grid* g) {
+  if (g->phase != PH_SELECTED)
+    return fail(g, LIPZ_ERR_STATE, "lipz_train_step must follow lipz_select_replace");
+  const int K = g->a.train_steps;
+  if (K > 1 && g->pool_n <= 0)
+    return fail(g, LIPZ_ERR_STATE, "train_steps > 1 draws its minibatches from the pool: call "
+                                   "lipz_set_data first");
+  int rc = train_once(g);
+  for (int k = 1; k < K && !rc; ++k) rc = train_again(g, (uint32_t)k);
+  if (rc) return rc;
   g->t += 1;
   g->phase = PH_IDLE;
   return LIPZ_OK;
@@ -942,6 +990,7 @@ int lipz_arch_default(lipz_arch* a) {
   a->leaky_slope = 0.2f;
   a->keep_grads = 0;
   a->force_simt = 0;
+  a->train_steps = 1;
   return LIPZ_OK;
 }
 

@@ -63,7 +63,7 @@ enum { DRAW_REAL = 1, DRAW_NOISE = 2 };
 template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
-                       int parts, bool pdl, cudaStream_t st);
+                       uint32_t step, int parts, bool pdl, cudaStream_t st);
 
 template <typename TI, typename TO, int EPI>
 void launch_gemm(const GemmDesc* descs, int n_problems, int max_m, int max_n, int act,
@@ -79,6 +79,8 @@ void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD,
 // (lr, 1 / (1 - beta1^(step+1)), 1 / (1 - beta2^(step+1)), step + 1).
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const SelectParams& p, const SelectIO& io, cudaStream_t st);
+// Choice of every cell's own centre (slot 0), for the later minibatch steps of an iteration.
+void launch_centre_select(int cells, const SelectParams& p, const SelectIO& io, cudaStream_t st);
 // Fitness and, in the same kernel, the selection of every cell (when nothing is read back
 // between the two).
 void launch_fitness_select(const float* logits, int cells, int B, float* LG, float* LD,

@@ -78,6 +78,9 @@ struct KParams {
   // slot 0 (the real rows) or slot 1 + part_slot[c] (the selected generator's fakes), through
   // a 4-D map {x, B, 6, cells}
   const int* part_slot;
+  // centre-only generator forward (non-zero): problem c is cell c's own generator on z_c,
+  // written to E[c] as the fakes of slot 0
+  int centre;
 };
 
 struct Job {
@@ -114,11 +117,11 @@ __device__ __forceinline__ int n_jobs(const KParams& p) {
 
 // Problem -> (cell whose activations are the A operand, individual whose weights are B).
 __device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
-  return p.train ? prob : prob / 5;
+  return (p.train || p.centre) ? prob : prob / 5;
 }
 __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
-  return __ldg(&p.nbr[prob]);
+  return p.centre ? prob : __ldg(&p.nbr[prob]);
 }
 
 // Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
@@ -307,7 +310,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int et = threadIdx.x - 64;  // epilogue thread 0..255
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++ltile) {
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
-      const int c = prob_cell(p, prob), slot = prob % 5;
+      const int c = prob_cell(p, prob), slot = p.centre ? 0 : prob % 5;
       const int k = prob_individual(p, prob);
       const float* wm = p.wmaster + (int64_t)k * p.pstride;
       const int rr = m0 + row;
@@ -532,8 +535,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 struct TcPlan {
   TcShape s;
   CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mE4;
-  tc::KParams pg, pd, pgt, pdt;
-  int grid_g, grid_d, grid_gt, grid_dt;
+  tc::KParams pg, pgc, pd, pgt, pdt;
+  int grid_g, grid_gc, grid_d, grid_gt, grid_dt;
   int* err;
 };
 
@@ -666,6 +669,9 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   g.logits = b.logits;
   g.slope = s.slope;
   g.err = p->err;
+  tc::KParams gc = g;  // every cell's own generator only (later minibatch steps)
+  gc.centre = 1;
+  gc.n_tiles = s.cells * g.mtiles;
   tc::KParams d = g;
   d.kind = tc::KIND_D;
   d.rows = 6 * s.B;
@@ -697,11 +703,13 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   dt.act2 = (bf16*)b.TG2;
   dt.logits = b.TL;
   p->pg = g;
+  p->pgc = gc;
   p->pd = d;
   p->pgt = gt;
   p->pdt = dt;
   auto grid = [sms](int n) { return n < sms ? n : sms; };
   p->grid_g = grid(g.n_tiles);
+  p->grid_gc = grid(gc.n_tiles);
   p->grid_d = grid(d.n_tiles);
   p->grid_gt = grid(gt.n_tiles);
   p->grid_dt = grid(dt.n_tiles);
@@ -724,6 +732,11 @@ int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensor
 
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg) {
   return launch(p->grid_g, p->mZ, p->mG1, p->mG2, p->mG3, p->pg, st, "generator forward", msg);
+}
+
+int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg) {
+  return launch(p->grid_gc, p->mZ, p->mG1, p->mG2, p->mG3, p->pgc, st, "centre generator forward",
+                msg);
 }
 
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg) {

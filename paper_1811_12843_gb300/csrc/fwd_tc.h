@@ -57,6 +57,8 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg);
 // Enqueue the generator kernel (fakes of every (cell, slot)) / the discriminator kernel (logits
 // of every (cell, slot)) on `st`. 0 on success.
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
+// Generator forward of every cell's own centre on its z, into E's slot-0 fakes.
+int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
 // Training forward of every cell's selected generator (hidden activations into TH1, TH2) and
 // selected discriminator (TG1, TG2 and the logits TL).

@@ -53,8 +53,9 @@ void launch_to_bf16(const float* w, bf16* wb, int64_t n, cudaStream_t st) {
 }
 
 // ------------------------------------------------------------------------------------------
-// Minibatch of cell c at iteration t: row b = pool row mulhi(word_b, n_pool) of stream BATCH
-// (or row b of the caller's batch), z[b][d] = normal b*z_dim + d of stream NOISE.
+// Minibatch of cell c at iteration t, minibatch step k: row b = pool row mulhi(word_b, n_pool)
+// of stream BATCH + 256 k (or row b of the caller's batch), z[b][d] = normal b*z_dim + d of
+// stream NOISE + 256 k.
 // Rows go to E[c][b] (the first B rows of the cell's evaluation input).
 // ------------------------------------------------------------------------------------------
 template <typename T>
@@ -80,8 +81,9 @@ template <typename T>
 __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
                              T* __restrict__ Z, int B, int x_dim, int z_dim, uint64_t seed,
-                             uint32_t t, int parts) {
+                             uint32_t t, uint32_t step, int parts) {
   pdl_wait();
+  const uint32_t s_batch = 3u + (step << 8), s_noise = 4u + (step << 8);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
   if (b >= B) return;
@@ -98,7 +100,7 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
       for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
     }
   } else {
-    const U4 r = philox_block(seed, 3u, t, (uint32_t)c, (uint32_t)(b >> 2));
+    const U4 r = philox_block(seed, s_batch, t, (uint32_t)c, (uint32_t)(b >> 2));
     const uint32_t w = (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
     const T* src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
     const int bytes = x_dim * (int)sizeof(T);
@@ -120,14 +122,14 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
   if ((z_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(zr) & (4 * sizeof(T) - 1)) == 0)) {
     // every block lies inside the row and its four normals are one aligned vector
     for (int k = lane * 4; k < z_dim; k += 128) {
-      const U4 r = philox_block(seed, 4u, t, (uint32_t)c, (n0 + (uint32_t)k) >> 2);
+      const U4 r = philox_block(seed, s_noise, t, (uint32_t)c, (n0 + (uint32_t)k) >> 2);
       const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
       store4<T>(zr + k, make_float4(g01.x, g01.y, g23.x, g23.y));
     }
     return;
   }
   for (uint32_t blk = (n0 >> 2) + lane; blk * 4 < n0 + (uint32_t)z_dim; blk += 32) {
-    const U4 r = philox_block(seed, 4u, t, (uint32_t)c, blk);
+    const U4 r = philox_block(seed, s_noise, t, (uint32_t)c, blk);
     const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
     const float v[4] = {g01.x, g01.y, g23.x, g23.y};
 #pragma unroll
@@ -141,15 +143,15 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
 template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
-                       int parts, bool pdl, cudaStream_t st) {
+                       uint32_t step, int parts, bool pdl, cudaStream_t st) {
   launch_kernel(pdl, k_draw_batch<T>, dim3((B + 7) / 8, cells), dim3(256), 0, st, pool, n_pool,
-                xin, E, e_cell, Z, B, x_dim, z_dim, seed, t, parts);
+                xin, E, e_cell, Z, B, x_dim, z_dim, seed, t, step, parts);
 }
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
-                                       float*, int, int, int, int, uint64_t, uint32_t, int, bool,
-                                       cudaStream_t);
+                                       float*, int, int, int, int, uint64_t, uint32_t, uint32_t,
+                                       int, bool, cudaStream_t);
 template void launch_draw_batch<bf16>(const bf16*, int64_t, const float*, bf16*, int64_t, bf16*,
-                                      int, int, int, int, uint64_t, uint32_t, int, bool,
+                                      int, int, int, int, uint64_t, uint32_t, uint32_t, int, bool,
                                       cudaStream_t);
 
 // ------------------------------------------------------------------------------------------
@@ -374,6 +376,22 @@ __device__ float mutate(float lr, uint64_t seed, uint32_t stream, uint32_t t, ui
   return fmaxf(lr + std * n, 1e-8f);
 }
 
+// Records the choice of population `pop` (0 G, 1 D) for cell c: slot s, source individual src,
+// the new lr and the Adam coefficients (lr, 1 / (1 - beta1^t), 1 / (1 - beta2^t), t) of the
+// source's next step t.
+__device__ void write_choice(int c, int pop, int s, int src, float lr, const SelectParams& p,
+                             const SelectIO& io) {
+  const int step1 = io.step_old[pop][src] + 1;
+  // 1 - beta^t = -expm1(t * log1p(-(1 - beta))): 1 - beta is exact in fp32 for beta in
+  // [0.5, 1), and the expm1 form keeps full relative precision for beta^t near 1
+  const float bc1 = -expm1f((float)step1 * log1pf(-(1.f - p.beta1)));
+  const float bc2 = -expm1f((float)step1 * log1pf(-(1.f - p.beta2)));
+  io.coef[pop][c] = make_float4(lr, 1.f / bc1, 1.f / bc2, (float)step1);
+  io.sel[pop][c] = s;
+  io.src[pop][c] = src;
+  io.lr_new[pop][c] = lr;
+}
+
 // Tournament, replacement and lr mutation of population `pop` (0 G, 1 D) of cell c, given the
 // five fitnesses f5 of the cell's neighbourhood; writes the selection, the source individual,
 // the new lr and the Adam coefficients (lr, 1 / (1 - beta1^t), 1 / (1 - beta2^t), t).
@@ -388,15 +406,18 @@ __device__ void select_one(int c, int pop, const float* f5, const int* __restric
   float lr = io.lr_old[pop][src];
   if (p.lr_mutation)
     lr = mutate(lr, p.seed, pop ? 8u : 7u, p.t, (uint32_t)c, p.lr_mut_std, p.lr_mut_thr);
-  const int step1 = io.step_old[pop][src] + 1;
-  // 1 - beta^t = -expm1(t * log1p(-(1 - beta))): 1 - beta is exact in fp32 for beta in
-  // [0.5, 1), and the expm1 form keeps full relative precision for beta^t near 1
-  const float bc1 = -expm1f((float)step1 * log1pf(-(1.f - p.beta1)));
-  const float bc2 = -expm1f((float)step1 * log1pf(-(1.f - p.beta2)));
-  io.coef[pop][c] = make_float4(lr, 1.f / bc1, 1.f / bc2, (float)step1);
-  io.sel[pop][c] = s;
-  io.src[pop][c] = src;
-  io.lr_new[pop][c] = lr;
+  write_choice(c, pop, s, src, lr, p, io);
+}
+
+// Later minibatch steps of an iteration: every cell's centre trains again, in place of a
+// selection (slot 0, source individual c, its own lr, no mutation).
+__global__ void k_centre_select(int cells, SelectParams p, SelectIO io) {
+  pdl_wait();
+  const int gid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = gid >> 1;
+  if (c >= cells) return;
+  const int pop = gid & 1;
+  write_choice(c, pop, 0, c, io.lr_old[pop][c], p, io);
 }
 
 __global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
@@ -493,6 +514,10 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const SelectParams& p, const SelectIO& io, cudaStream_t st) {
   launch_pdl(k_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, fG, fD, nbr, cells, p,
              io);
+}
+
+void launch_centre_select(int cells, const SelectParams& p, const SelectIO& io, cudaStream_t st) {
+  launch_pdl(k_centre_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, cells, p, io);
 }
 
 // ------------------------------------------------------------------------------------------

@@ -13,7 +13,8 @@ def oracle_arch(arch) -> O.Arch:
                   tournament_size=arch.tournament_size,
                   replace_mode="always" if arch.replace_mode == 1 else "if_better",
                   lr_mutation=bool(arch.lr_mutation), lr_mut_std=float(arch.lr_mut_std),
-                  lr_mut_prob=float(arch.lr_mut_prob), leaky_slope=float(arch.leaky_slope))
+                  lr_mut_prob=float(arch.lr_mut_prob), leaky_slope=float(arch.leaky_slope),
+                  train_steps=int(arch.train_steps))
 
 
 def max_rel(got, ref) -> float:

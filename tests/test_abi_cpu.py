@@ -64,6 +64,13 @@ def test_create_rejects_bad_arguments_without_a_device(lib):
     with pytest.raises(L.LipzError) as e:
         L.lipz_grid_create(2, 2, bad, 1)
     assert e.value.code == L.LIPZ_ERR_INVALID
+    assert a.train_steps == 1
+    for k in (0, -1, 65537):
+        bad = L.lipz_arch_default()
+        bad.train_steps = k
+        with pytest.raises(L.LipzError) as e:
+            L.lipz_grid_create(2, 2, bad, 1)
+        assert e.value.code == L.LIPZ_ERR_INVALID and "train_steps" in str(e.value)
     bad = L.lipz_arch_default()
     bad.struct_size = 4
     with pytest.raises(L.LipzError):

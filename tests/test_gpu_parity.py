@@ -372,3 +372,118 @@ def test_large_grid_20x20_bf16_sampled(L):
         bound = lr if it == 0 else lr * (1 - 0.5) / np.sqrt(1 - 0.999)
         assert np.max(np.abs(got.Dw - s.Dw[src])) <= bound * (1 + 1e-5) + ulp
         assert np.all(got.Dstep == s.Dstep[src] + 1)
+
+
+def _k_step_iteration_check(L, g, pool, tol, kink_band, loose=False):
+    """One iteration with arch.train_steps = K: the selection bit-exact given the engine's own
+    fitness, then the state after the K Adam steps against the oracle's. The last step's
+    gradients and the moments meet the tolerance in every cell, except a cell whose
+    pre-activations came within rounding distance of a kink in one of the K steps (as in the
+    one-step check; at most a quarter of the cells). With ``loose`` (bf16, where every cell
+    passes that close to a kink, and the worst of some 36 tensors after K steps is taken) a cell
+    may miss the tolerance by less than five times it, the median cell by less than twice: an
+    error of the method (a wrong minibatch, fake slot, step count or moment) is of order one.
+    A weight
+    may miss the tolerance only by less than the K Adam moves (about lr each) that a near-zero
+    gradient can turn either way, and only rarely."""
+    a = oracle_arch(g.arch)
+    K = a.train_steps
+    s = _to_oracle(g, g.arch)
+    data = O.batches(s, pool)
+    ev = g.eval()
+    sel = g.select()
+    ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                   "fD": ev["fD"].astype(np.float64)})
+    assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+    assert np.array_equal(sel["sel_d"], ref_sel["sel_d"])
+    g.train()
+    new, grads = O.train_step(s, ref_sel, data, keep_grads=True, pool=pool)
+    got = _to_oracle(g, g.arch)
+    assert got.t == s.t + 1
+    nbr = O.neighbors(s.rows, s.cols)
+    src_g = nbr[np.arange(s.cells), ref_sel["sel_g"]]
+    assert np.array_equal(got.Gstep, s.Gstep[src_g] + K) and np.array_equal(got.Gstep, new.Gstep)
+    assert np.array_equal(got.Dstep, new.Dstep)
+    assert np.allclose(got.Glr, new.Glr, rtol=1e-6) and np.allclose(got.Dlr, new.Dlr, rtol=1e-6)
+    gg, gd = g.gradients()
+    kinky = grads["kink"] < kink_band
+    worst = np.zeros(s.cells)
+    pairs = [("G", gg, grads["gG"]), ("D", gd, grads["gD"])]
+    for pop in ("G", "D"):
+        pairs += [(pop, getattr(got, pop + f), getattr(new, pop + f)) for f in ("m", "v")]
+    for pop, gpu, ref in pairs:
+        lay = O.g_layout(a) if pop == "G" else O.d_layout(a)
+        for c in range(s.cells):
+            worst[c] = max(worst[c], max(per_tensor(gpu[c:c + 1], ref[c:c + 1], lay).values()))
+    ok = worst < tol
+    assert np.all(ok | kinky), ("mismatch without a kink", np.where(~ok)[0], worst)
+    if loose:
+        assert np.all(worst < 5 * tol) and np.median(worst) < 2 * tol, worst
+    else:
+        assert np.sum(~ok) <= max(1, s.cells // 4), worst
+    for pop, lay in (("G", O.g_layout(a)), ("D", O.d_layout(a))):
+        w_got, w_ref = getattr(got, pop + "w")[ok], getattr(new, pop + "w")[ok]
+        off, flagged, total = 0, 0, 0
+        for name, shape in lay:
+            n = int(np.prod(shape))
+            d = np.abs(w_got[:, off:off + n] - w_ref[:, off:off + n])
+            bad = d > tol * np.max(np.abs(getattr(new, pop + "w")[:, off:off + n]))
+            assert np.all(d[bad] <= 2.5 * K * a.lr), (pop, name, float(np.max(d)))
+            flagged += int(bad.sum())
+            total += d.size
+            off += n
+        assert flagged <= max(20, total // 2000), (pop, flagged)
+
+
+@pytest.mark.parametrize("precision,rows,cols,batch,K", [
+    ("fp32", 2, 2, 100, 3),
+    ("bf16", 3, 3, 129, 2),
+    ("bf16", 2, 3, 100, 4),
+])
+def test_k_minibatch_steps_against_the_oracle(L, precision, rows, cols, batch, K):
+    """train_steps = K: after the selection every cell's new centre pair takes K Adam steps,
+    step k >= 1 on a fresh minibatch of the step-k streams. In bf16 the learning rate is 1e-6:
+    at 2e-4 the elements whose gradient is at bf16 noise level take Adam moves of either sign
+    (about lr each, the same in the one-step check) and those differences feed the next step's
+    gradients, so only the first step would be compared at the tolerance."""
+    pool = _pool(14, 6000, 784)
+    kw = dict(lr_mutation=1, lr_mut_prob=0.5)
+    if precision == "bf16":
+        kw.update(lr=1e-6, lr_mut_std=1e-7)
+    g = _grid(L, rows, cols, 40 + K, pool, precision=precision, batch=batch, keep_grads=1,
+              train_steps=K, **kw)
+    tol = TOL[g.arch.precision]
+    for _ in range(2):
+        _k_step_iteration_check(L, g, pool, tol, 1e-5 if precision == "fp32" else 1e-3,
+                                loose=precision == "bf16")
+
+
+def test_k_minibatch_steps_fused_adam_bit_exact(L):
+    """The in-place later steps through the fused-Adam backward equal the stored-gradient path
+    bit for bit; K = 1 leaves the default iteration unchanged."""
+    pool = _pool(15, 4000, 784)
+    a = _grid(L, 3, 3, 17, pool, precision="bf16", train_steps=3)
+    b = _grid(L, 3, 3, 17, pool, precision="bf16", train_steps=3, keep_grads=1)
+    c = _grid(L, 3, 3, 17, pool, precision="bf16", train_steps=1)
+    d = _grid(L, 3, 3, 17, pool, precision="bf16")
+    for it in range(2):
+        a.iterate(1)
+        b.iterate(1)
+        c.iterate(1)
+        d.iterate(1)
+        assert a.export_state() == b.export_state(), it
+        assert c.export_state() == d.export_state(), it
+    sa = _to_oracle(a, a.arch)
+    assert np.all(sa.Gstep >= 6) and np.all(sa.Gstep % 3 == 0)
+
+
+def test_k_minibatch_steps_need_the_pool(L):
+    """Steps k >= 1 draw from the pool: with caller batches and no pool the training call fails
+    with LIPZ_ERR_STATE instead of reading unset memory."""
+    import lipz_synth
+    g = L.Grid(1, 2, seed=3, train_steps=2)
+    x = lipz_synth.host_batch(2, 2, 100)
+    fg, fd = np.zeros((2, 5), np.float32), np.zeros((2, 5), np.float32)
+    with pytest.raises(L.LipzError) as e:
+        L.lipz_iterate_batch(g.h, x, fg, fd)
+    assert e.value.code == L.LIPZ_ERR_STATE and "pool" in str(e.value)
