@@ -9,6 +9,10 @@ one full grid iteration (minibatch draw, all-pairs evaluation, fitness, selectio
 Adam of every cell's new centre pair).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--train-steps S]
+
+With --train-steps S > 1 every iteration trains each cell's new centre pair S times (the later
+steps on fresh minibatches); the default S = 1 is the headline workload.
 
 With N > 1 (torchrun, one process per GPU) every rank runs its own 12x12 grid (replicas: the
 per-GPU work is fixed, scaling "weak"); value = all ranks' pairs / the slowest rank's time.
@@ -160,7 +164,8 @@ def run_ours(args):
     import paper_1811_12843_gb300 as L
 
     pool = lipz_synth.blob_pool(SEED, n=POOL_N, dim=X_DIM)
-    g = L.Grid(ROWS, COLS, seed=SEED + rank, precision="bf16", batch=BATCH)
+    g = L.Grid(ROWS, COLS, seed=SEED + rank, precision="bf16", batch=BATCH,
+               train_steps=args.train_steps)
     g.set_data(pool)
     stream = torch.cuda.Stream()
     g.set_stream(stream.cuda_stream)
@@ -219,7 +224,9 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
-        "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+        "config": {"workload": _workload(args),
+                   "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+                   "train_steps": args.train_steps,
                    "pairs_per_iter": PAIRS, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (population 2.2 GB + pool 188 MB per iteration)"},
         "grid_iterations_per_sec": iters_total,
@@ -233,7 +240,7 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and args.train_steps == 1:
         line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
     return line
 
@@ -293,9 +300,10 @@ def _roofline(phase_ms):
     return r
 
 
-def _oracle_sample(seconds, max_cells=None):
+def _oracle_sample(seconds, max_cells=None, train_steps=1):
     """Run the oracle's full iteration cell by cell on the 12x12 workload until ``seconds`` of
-    CPU work are spent; return (cells done, elapsed seconds)."""
+    CPU work are spent; return (cells done, elapsed seconds). With ``train_steps`` K > 1 each
+    cell's pair then takes K - 1 more steps on fresh minibatches."""
     import numpy as np
     import lipz_synth
     from oracle import lipz_oracle as O
@@ -318,10 +326,15 @@ def _oracle_sample(seconds, max_cells=None):
                                                      a.tournament_size), a)
         x, z = data[c]
         gG, gD, _ = O.pair_gradients(state.Gw[nbr[c][sg]], state.Dw[nbr[c][sd]], x, z, a)
-        O.adam_step(state.Gw[nbr[c][sg]], state.Gm[nbr[c][sg]], state.Gv[nbr[c][sg]], 0, gG,
-                    a.lr, a)
-        O.adam_step(state.Dw[nbr[c][sd]], state.Dm[nbr[c][sd]], state.Dv[nbr[c][sd]], 0, gD,
-                    a.lr, a)
+        Gn = O.adam_step(state.Gw[nbr[c][sg]], state.Gm[nbr[c][sg]], state.Gv[nbr[c][sg]], 0,
+                         gG, a.lr, a)
+        Dn = O.adam_step(state.Dw[nbr[c][sd]], state.Dm[nbr[c][sd]], state.Dv[nbr[c][sd]], 0,
+                         gD, a.lr, a)
+        for k in range(1, train_steps):
+            x, z = O.draw_batch(state.seed, state.t, c, pool, a, k)
+            gG, gD, _ = O.pair_gradients(Gn[0], Dn[0], x, z, a)
+            Gn = O.adam_step(*Gn, gG, a.lr, a)
+            Dn = O.adam_step(*Dn, gD, a.lr, a)
         done += 1
         c = (c + 1) % CELLS
         el = time.perf_counter() - t0
@@ -355,6 +368,12 @@ def cpu_baseline(seconds):
                       "gradients + Adam per cell), %.1f s, numpy float64 + OpenBLAS" % (done, el)}
 
 
+def _workload(args):
+    if args.train_steps == 1:
+        return WORKLOAD
+    return "%s, %d minibatch steps per iteration" % (WORKLOAD, args.train_steps)
+
+
 def run_reference(args):
     _, rank, world = _dist()
     if rank != 0:
@@ -364,11 +383,11 @@ def run_reference(args):
     _oracle_state(arch)
     per_step_cells = 1
     for _ in range(args.warmup):
-        _oracle_sample(1e9, max_cells=1)
+        _oracle_sample(1e9, max_cells=1, train_steps=args.train_steps)
     times = []
     total_cells = 0
     for _ in range(args.steps):
-        done, el = _oracle_sample(1e9, max_cells=per_step_cells)
+        done, el = _oracle_sample(1e9, max_cells=per_step_cells, train_steps=args.train_steps)
         times.append(el)
         total_cells += done
     el = sum(times)
@@ -377,7 +396,8 @@ def run_reference(args):
             "warmup": args.warmup, "ms_per_step": 1000.0 * el / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded 10-blob 784-dim pool standing in for MNIST)",
-            "config": {"workload": WORKLOAD, "rows": ROWS, "cols": COLS, "global_batch": BATCH,
+            "config": {"workload": _workload(args), "rows": ROWS, "cols": COLS,
+                       "global_batch": BATCH, "train_steps": args.train_steps,
                        "pairs_per_iter": PAIRS, "parallelism": "cpu"},
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
@@ -397,6 +417,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass")
     ap.add_argument("--no-phases", action="store_true", help="skip the per-phase timing pass")
+    ap.add_argument("--train-steps", type=int, default=1,
+                    help="Adam steps per grid iteration (the later ones on fresh minibatches)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
