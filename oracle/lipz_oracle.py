@@ -31,6 +31,12 @@ Readings where the paper is silent (each is listed in the design doc with its reason)
     256 k); selection and lr mutation happen once, before step 0;
   * random draws come from Philox4x32-10 (Salmon et al., SC'11) keyed by the seed, with the
     counter (block index, cell, iteration, stream);
+  * mixture weights (step 4): one ES-(1+1) step per iteration on each cell's weights w over its
+    five neighbourhood generators, scored, in place of FID (no Inception network here), by the
+    squared maximum mean discrepancy (Gretton et al., JMLR 2012) with the Gaussian kernel
+    exp(-||a - b||^2 / x_dim) between the w-weighted fakes of the evaluation and the real
+    minibatch (the same rows the discriminators saw in step 2); a mutation adds sigma N(0, 1)
+    to every weight, clips at 0 and renormalises, and is kept only if it lowers the score;
   * in bf16 mode every operand of a matrix product (weights, activations, back-propagated
     deltas) is rounded to bfloat16 (round to nearest even), products accumulate exactly (here:
     float64), biases, logits, losses, gradients and optimiser state stay unrounded.
@@ -68,6 +74,7 @@ STREAM_TOUR_G = 5
 STREAM_TOUR_D = 6
 STREAM_MUT_G = 7
 STREAM_MUT_D = 8
+STREAM_MIX = 9
 # Minibatch step k of an iteration draws from stream id + STEP_STREAM_STRIDE * k.
 STEP_STREAM_STRIDE = 256
 
@@ -153,6 +160,8 @@ class Arch:
     lr_mut_prob: float = 0.5  # mutation probability (Table 1)
     leaky_slope: float = 0.2
     train_steps: int = 1      # Adam steps of the new centre pair per iteration
+    mixture: bool = False     # evolve each neighbourhood's generator-mixture weights
+    mix_sigma: float = 0.01   # mixture mutation scale (Table 1)
 
 
 def g_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
@@ -302,6 +311,7 @@ class State:
     Dv: np.ndarray
     Dstep: np.ndarray
     Dlr: np.ndarray
+    mix: np.ndarray = None  # [cells, 5] generator-mixture weights of each neighbourhood
 
     @property
     def cells(self) -> int:
@@ -310,7 +320,7 @@ class State:
     def copy(self) -> "State":
         return dataclasses.replace(self, **{f: getattr(self, f).copy() for f in
                                             ("Gw", "Gm", "Gv", "Gstep", "Glr",
-                                             "Dw", "Dm", "Dv", "Dstep", "Dlr")})
+                                             "Dw", "Dm", "Dv", "Dstep", "Dlr", "mix")})
 
 
 def create(rows: int, cols: int, arch: Arch, seed: int) -> State:
@@ -325,7 +335,7 @@ def create(rows: int, cols: int, arch: Arch, seed: int) -> State:
     return State(rows, cols, arch, seed, 0,
                  Gw, np.zeros_like(Gw), np.zeros_like(Gw), np.zeros(cells, np.int64),
                  np.full(cells, lr), Dw, np.zeros_like(Dw), np.zeros_like(Dw),
-                 np.zeros(cells, np.int64), np.full(cells, lr))
+                 np.zeros(cells, np.int64), np.full(cells, lr), np.full((cells, 5), 0.2))
 
 
 def draw_batch(seed: int, t: int, cell: int, pool: np.ndarray, arch: Arch, step: int = 0
@@ -385,6 +395,68 @@ def eval_neighborhoods(state: State, data, cells=None) -> Dict[str, np.ndarray]:
             for i in range(5):
                 LG[c, i, j], LD[c, i, j] = pair_losses(lg[:B], lg[B * (i + 1):B * (i + 2)])
     return {"LG": LG, "LD": LD, "fG": LG.mean(axis=2), "fD": LD.mean(axis=1), "logits": logits}
+
+
+# --------------------------------------------------------------------------------------------
+# Step 4: generator-mixture weights, ES-(1+1).
+# --------------------------------------------------------------------------------------------
+def mixture_blocks(X: np.ndarray, B: int) -> np.ndarray:
+    """S[a][b] = mean of the Gaussian kernel exp(-||X_r - X_s||^2 / dim) over the rows r of block
+    a and s of block b, blocks of B rows (block 0 the real rows, block 1 + i the fakes of
+    generator slot i)."""
+    X = np.asarray(X, np.float64)
+    n, dim = X.shape
+    K = np.empty((n, n))
+    for r in range(n):
+        K[r] = np.exp(-((X - X[r]) ** 2).sum(axis=1) / dim)
+    nb = n // B
+    S = np.empty((nb, nb))
+    for a in range(nb):
+        for b in range(nb):
+            S[a, b] = K[a * B:(a + 1) * B, b * B:(b + 1) * B].mean()
+    return S
+
+
+def mmd2(w: np.ndarray, S: np.ndarray) -> float:
+    """Squared MMD between the mixture sum_i w_i (fakes of slot i) and the real rows, from the
+    block means: sum_ij w_i w_j S[1+i][1+j] - 2 sum_i w_i S[1+i][0] + S[0][0]."""
+    w = np.asarray(w, np.float64)
+    return float(w @ S[1:, 1:] @ w - 2.0 * (w @ S[1:, 0]) + S[0, 0])
+
+
+def mixture_step(w: np.ndarray, S: np.ndarray, normals: np.ndarray, sigma: float):
+    """ES-(1+1): w' = max(w + sigma n, 0) / sum (w kept if that sum is 0); w' replaces w iff
+    mmd2(w') < mmd2(w). Returns (new w, accepted, mmd2(w), mmd2(w'))."""
+    w = np.asarray(w, np.float64)
+    cand = np.maximum(w + sigma * np.asarray(normals, np.float64), 0.0)
+    tot = cand.sum()
+    cand = cand / tot if tot > 0.0 else w.copy()
+    old, new = mmd2(w, S), mmd2(cand, S)
+    acc = new < old
+    return (cand if acc else w.copy()), bool(acc), old, new
+
+
+def mixture_update(state: State, data, cells=None) -> Dict[str, np.ndarray]:
+    """Every cell's ES-(1+1) step on its mixture weights, scored on the evaluation's rows: the
+    real minibatch and the fakes of the five neighbourhood generators on the cell's noise (as
+    the discriminators received them, i.e. rounded to bf16 in bf16 mode). The mutation's five
+    normals are the first five of the cell's stream MIX at the iteration."""
+    a = state.arch
+    rb = _Rounder(a)
+    gl = g_layout(a)
+    nbr = neighbors(state.rows, state.cols)
+    n = state.cells
+    out = {"S": np.zeros((n, 6, 6)), "mix": state.mix.copy(), "accept": np.zeros(n, bool),
+           "score": np.zeros(n), "score_new": np.zeros(n)}
+    for c in (range(n) if cells is None else cells):
+        x, z = data[c]
+        fakes = [g_forward(unflatten(state.Gw[nbr[c][i]], gl), z, a)["F"] for i in range(5)]
+        S = mixture_blocks(rb(np.vstack([x] + fakes)), a.batch)
+        nrm = draw_normals(state.seed, STREAM_MIX, state.t, c, 5)
+        w, acc, old, new = mixture_step(state.mix[c], S, nrm, a.mix_sigma)
+        out["S"][c], out["mix"][c], out["accept"][c] = S, w, acc
+        out["score"][c], out["score_new"][c] = old, new
+    return out
 
 
 # --------------------------------------------------------------------------------------------
@@ -556,27 +628,30 @@ def train_step(state: State, sel, data, keep_grads: bool = False,
 
 def iterate(state: State, pool: Optional[np.ndarray], n_iters: int = 1,
             x_host: Optional[np.ndarray] = None, record: bool = False):
-    """Steps 2, 3 and 5: ``n_iters`` synchronous grid iterations. Returns the new state (and,
+    """Steps 2, 3 (and 4 with ``arch.mixture``) and 5: ``n_iters`` synchronous grid iterations. Returns the new state (and,
     with ``record``, the per-iteration evaluations and selections)."""
     log = []
     for _ in range(n_iters):
         data = batches(state, pool, x_host)
         ev = eval_neighborhoods(state, data)
+        mx = mixture_update(state, data) if state.arch.mixture else None
         sel = select_replace(state, ev)
         state = train_step(state, sel, data, pool=pool)
+        if mx is not None:
+            state.mix = mx["mix"]
         if record:
-            log.append({"eval": ev, "sel": sel})
+            log.append({"eval": ev, "sel": sel, "mix": mx})
     return (state, log) if record else state
 
 
 # --------------------------------------------------------------------------------------------
 # State bytes: the engine's documented export layout (little-endian), so that a state can move
 # between the engine and the oracle.
-#   header (64 bytes): u32 magic 0x5A50494C ("LIPZ"), u32 version 1, i32 rows, i32 cols,
+#   header (64 bytes): u32 magic 0x5A50494C ("LIPZ"), u32 version 2, i32 rows, i32 cols,
 #     i32 z_dim, i32 hidden, i32 x_dim, i32 batch, i32 precision (0 fp32, 1 bf16), i32 0,
 #     i64 t, u64 seed, 8 zero bytes
 #   then f32 Gw[cells][PG], Gm, Gv, Dw[cells][PD], Dm, Dv, i32 Gstep[cells], Dstep[cells],
-#     f32 Glr[cells], Dlr[cells].
+#     f32 Glr[cells], Dlr[cells], f32 mix[cells][5].
 # --------------------------------------------------------------------------------------------
 _MAGIC = 0x5A50494C
 
@@ -584,7 +659,7 @@ _MAGIC = 0x5A50494C
 def state_to_bytes(s: State) -> bytes:
     a = s.arch
     hdr = np.zeros(16, dtype=np.uint32)
-    hdr[0], hdr[1] = _MAGIC, 1
+    hdr[0], hdr[1] = _MAGIC, 2
     hdr[2:10] = [s.rows, s.cols, a.z_dim, a.hidden, a.x_dim, a.batch,
                  1 if a.precision == "bf16" else 0, 0]
     h = hdr.tobytes()
@@ -593,14 +668,15 @@ def state_to_bytes(s: State) -> bytes:
     parts = [h] + [getattr(s, f).astype(np.float32).tobytes()
                    for f in ("Gw", "Gm", "Gv", "Dw", "Dm", "Dv")]
     parts += [s.Gstep.astype(np.int32).tobytes(), s.Dstep.astype(np.int32).tobytes(),
-              s.Glr.astype(np.float32).tobytes(), s.Dlr.astype(np.float32).tobytes()]
+              s.Glr.astype(np.float32).tobytes(), s.Dlr.astype(np.float32).tobytes(),
+              s.mix.astype(np.float32).tobytes()]
     return b"".join(parts)
 
 
 def state_from_bytes(buf: bytes, arch: Arch) -> State:
     hdr = np.frombuffer(buf[:40], dtype=np.int32)
-    if int(np.frombuffer(buf[:4], np.uint32)[0]) != _MAGIC:
-        raise ValueError("not a grid state")
+    if int(np.frombuffer(buf[:4], np.uint32)[0]) != _MAGIC or int(hdr[1]) != 2:
+        raise ValueError("not a version-2 grid state")
     rows, cols = int(hdr[2]), int(hdr[3])
     if (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7])) != (arch.z_dim, arch.hidden,
                                                               arch.x_dim, arch.batch):
@@ -620,6 +696,9 @@ def state_from_bytes(buf: bytes, arch: Arch) -> State:
         v = np.frombuffer(buf[off:off + 4 * cells], dt)
         arrs[f] = v.astype(np.int64 if dt == np.int32 else np.float64)
         off += 4 * cells
+    arrs["mix"] = np.frombuffer(buf[off:off + 20 * cells], np.float32).astype(
+        np.float64).reshape(cells, 5)
+    off += 20 * cells
     if off != len(buf):
         raise ValueError("state size mismatch")
     return State(rows, cols, arch, seed, t, **arrs)
