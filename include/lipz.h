@@ -64,7 +64,8 @@ enum { LIPZ_REPLACE_IF_BETTER = 0, LIPZ_REPLACE_ALWAYS = 1 };
 /* Philox stream ids (fourth counter word). */
 enum {
   LIPZ_STREAM_INIT_G = 1, LIPZ_STREAM_INIT_D = 2, LIPZ_STREAM_BATCH = 3, LIPZ_STREAM_NOISE = 4,
-  LIPZ_STREAM_TOUR_G = 5, LIPZ_STREAM_TOUR_D = 6, LIPZ_STREAM_MUT_G = 7, LIPZ_STREAM_MUT_D = 8
+  LIPZ_STREAM_TOUR_G = 5, LIPZ_STREAM_TOUR_D = 6, LIPZ_STREAM_MUT_G = 7, LIPZ_STREAM_MUT_D = 8,
+  LIPZ_STREAM_MIX = 9
 };
 /* Minibatch step k of an iteration draws its batch from stream LIPZ_STREAM_BATCH + stride * k and
  * its noise from LIPZ_STREAM_NOISE + stride * k (k = 0 is the evaluation minibatch). */
@@ -109,6 +110,10 @@ typedef struct lipz_arch {
                               the pool with stream ids + LIPZ_STEP_STREAM_STRIDE * k (also when
                               the caller supplied step 0's real rows); selection and the lr
                               mutation happen once, before step 0. K <= 65536. */
+  int32_t mixture;         /* 1: every evaluation also takes one ES-(1+1) step of each cell's
+                              generator-mixture weights (Section 3 step 4); see
+                              lipz_get_mixture. Default 0. */
+  float mix_sigma;         /* 0.01: mixture mutation scale (Table 1) */
 } lipz_arch;
 
 typedef struct lipz_grid lipz_grid;
@@ -189,9 +194,10 @@ LIPZ_API int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g,
 
 /*
  * State I/O (checkpoint / resume, and state exchange with other implementations). Layout,
- * little-endian: a 64-byte header {u32 magic 0x5A50494C, u32 version 1, i32 rows, cols, z_dim,
+ * little-endian: a 64-byte header {u32 magic 0x5A50494C, u32 version 2, i32 rows, cols, z_dim,
  * hidden, x_dim, batch, precision, 0, i64 t, u64 seed, 8 zero bytes}, then f32 Gw[cells][PG],
- * Gm, Gv, Dw[cells][PD], Dm, Dv, i32 Gstep[cells], Dstep[cells], f32 Glr[cells], Dlr[cells].
+ * Gm, Gv, Dw[cells][PD], Dm, Dv, i32 Gstep[cells], Dstep[cells], f32 Glr[cells], Dlr[cells],
+ * f32 mix[cells][5] (generator-mixture weights).
  * PG, PD = parameter counts; each individual's vector is, in order, W1 [out][in], b1, W2, b2,
  * W3, b3 (PyTorch Linear layout). Import requires the same rows, cols and arch sizes; it
  * replaces the seed and iteration counter too. Both calls are synchronous.
@@ -210,6 +216,21 @@ LIPZ_API int lipz_get_iteration(const lipz_grid* g, int64_t* t);
 LIPZ_API int lipz_get_batch(lipz_grid* g, float* x, float* z);
 LIPZ_API int lipz_get_logits(lipz_grid* g, float* logits);
 
+/*
+ * Generator mixtures (Section 3 step 4; synchronous, host pointers, each may be null).
+ * weights [cells][5]: every neighbourhood's mixture weights over its generator slots 0..4
+ * (initially 1/5; with arch.mixture each evaluation takes one ES-(1+1) step). blocks
+ * [cells][6][6] and score [cells] (need arch.mixture, else LIPZ_ERR_STATE): of the last
+ * evaluation, S[a][b] = mean over the rows r of block a and s of block b of
+ * exp(-||e_r - e_s||^2 / x_dim), the blocks being the B real rows (0) and the fakes of
+ * generator slots 0..4 (1..5) as the discriminators received them; score = the squared MMD
+ * sum_ij w_i w_j S[1+i][1+j] - 2 sum_i w_i S[1+i][0] + S[0][0] of the weights kept. The step:
+ * w' = max(w + mix_sigma n, 0) / sum (n: the first five normals of stream LIPZ_STREAM_MIX at
+ * the iteration; w kept if the sum is 0) replaces w iff its squared MMD is lower. The score
+ * stands in for the paper's FID (no Inception network here).
+ */
+LIPZ_API int lipz_get_mixture(lipz_grid* g, float* weights, float* blocks, float* score);
+
 /* Gradients of the last train step (needs arch.keep_grads): gG [cells][PG], gD [cells][PD]. */
 LIPZ_API int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d);
 
@@ -219,7 +240,8 @@ LIPZ_API int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d);
  * fitness), _SELECT, _TRAIN_FWD (forward of the selected pairs and the logit deltas),
  * _TRAIN_BWD (their backward; on the tensor-core path one kernel, which also applies Adam to
  * the weight matrices unless arch.keep_grads is set), _ADAM (bias gradients, then the rest of
- * the update and replacement). While enabled, every phase is bracketed by CUDA events on
+ * the update and replacement), _MIXTURE (with arch.mixture: the mixture step at the end of
+ * an evaluation). While enabled, every phase is bracketed by CUDA events on
  * the grid's stream. lipz_profile_read waits for the stream and writes, per phase, the summed
  * device milliseconds (ms[n]), the number of phase executions (count[n]) and of kernel launches
  * (launches[n]) since the last read (any pointer may be null; n <= LIPZ_N_PHASES), then resets.
@@ -227,7 +249,7 @@ LIPZ_API int lipz_get_gradients(lipz_grid* g, float* grad_g, float* grad_d);
 enum {
   LIPZ_PHASE_BATCH = 0, LIPZ_PHASE_G_FWD = 1, LIPZ_PHASE_D_FWD = 2, LIPZ_PHASE_FITNESS = 3,
   LIPZ_PHASE_SELECT = 4, LIPZ_PHASE_TRAIN_FWD = 5, LIPZ_PHASE_TRAIN_BWD = 6,
-  LIPZ_PHASE_ADAM = 7, LIPZ_N_PHASES = 8
+  LIPZ_PHASE_ADAM = 7, LIPZ_PHASE_MIXTURE = 8, LIPZ_N_PHASES = 9
 };
 LIPZ_API int lipz_profile_enable(lipz_grid* g, int enable);
 LIPZ_API int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t* launches, int n);

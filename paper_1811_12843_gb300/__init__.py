@@ -18,7 +18,8 @@ __all__ = [
     "lipz_synchronize", "lipz_set_data", "lipz_eval_neighborhoods", "lipz_select_replace",
     "lipz_train_step", "lipz_iterate", "lipz_iterate_batch", "lipz_state_bytes",
     "lipz_export_state", "lipz_import_state", "lipz_get_iteration", "lipz_get_batch",
-    "lipz_get_logits", "lipz_get_gradients", "lipz_profile_enable", "lipz_profile_read",
+    "lipz_get_logits", "lipz_get_gradients", "lipz_get_mixture", "lipz_profile_enable",
+    "lipz_profile_read",
     "lipz_fitness_from_logits_noalloc", "lipz_last_error", "lipz_status_string", "PHASES",
     "EXPORTED", "Grid", "param_counts",
 ]
@@ -50,7 +51,8 @@ class lipz_arch(ctypes.Structure):
         ("lr_mutation", ctypes.c_int32), ("lr_mut_std", ctypes.c_float),
         ("lr_mut_prob", ctypes.c_float), ("leaky_slope", ctypes.c_float),
         ("keep_grads", ctypes.c_int32), ("force_simt", ctypes.c_int32),
-        ("train_steps", ctypes.c_int32),
+        ("train_steps", ctypes.c_int32), ("mixture", ctypes.c_int32),
+        ("mix_sigma", ctypes.c_float),
     ]
 
 
@@ -77,6 +79,7 @@ _SIGS = {
     "lipz_get_batch": (_I, [_P, _P, _P]),
     "lipz_get_logits": (_I, [_P, _P]),
     "lipz_get_gradients": (_I, [_P, _P, _P]),
+    "lipz_get_mixture": (_I, [_P, _P, _P, _P]),
     "lipz_profile_enable": (_I, [_P, _I]),
     "lipz_profile_read": (_I, [_P, _P, _P, _P, _I]),
     "lipz_fitness_from_logits_noalloc": (_I, [_P, ctypes.c_int32, ctypes.c_int32, _P, _P, _P]),
@@ -213,7 +216,12 @@ def lipz_get_gradients(g, grad_g=None, grad_d=None):
     return _check(g, load().lipz_get_gradients(g, _ptr(grad_g), _ptr(grad_d)))
 
 
-PHASES = ("batch", "g_fwd", "d_fwd", "fitness", "select", "train_fwd", "train_bwd", "adam")
+def lipz_get_mixture(g, weights=None, blocks=None, score=None):
+    return _check(g, load().lipz_get_mixture(g, _ptr(weights), _ptr(blocks), _ptr(score)))
+
+
+PHASES = ("batch", "g_fwd", "d_fwd", "fitness", "select", "train_fwd", "train_bwd", "adam",
+          "mixture")
 
 
 def lipz_profile_enable(g, enable=True):
@@ -342,6 +350,18 @@ class Grid:
         out = np.zeros((self.cells, 5, 6 * self.arch.batch), np.float32)
         lipz_get_logits(self.h, out)
         return out
+
+    def mixture(self, blocks=False):
+        """Mixture weights [cells, 5]; with ``blocks`` also the last evaluation's kernel block
+        means [cells, 6, 6] and squared-MMD scores [cells] (needs arch.mixture)."""
+        w = np.zeros((self.cells, 5), np.float32)
+        if not blocks:
+            lipz_get_mixture(self.h, w)
+            return w
+        S = np.zeros((self.cells, 6, 6), np.float32)
+        sc = np.zeros(self.cells, np.float32)
+        lipz_get_mixture(self.h, w, S, sc)
+        return w, S, sc
 
     def gradients(self):
         gg = np.zeros((self.cells, self.PG), np.float32)

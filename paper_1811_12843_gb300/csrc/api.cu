@@ -78,6 +78,15 @@ struct lipz_grid {
   void *J2 = nullptr, *D1 = nullptr, *A3 = nullptr, *A2 = nullptr, *A1 = nullptr;
   float *gG = nullptr, *gD = nullptr;
   int* flag = nullptr;
+  // generator-mixture weights [cells][5] (always held: part of the state), and with
+  // arch.mixture the score's work buffers: row norms [cells][6B], per-row block sums
+  // [cells][6B][mix_nh][6], block means [cells][6][6], scores [cells]; the CUDA-core path
+  // stores the Gram matrices [cells][6B][6B] first
+  float *mix = nullptr, *rnorm = nullptr, *mixP = nullptr, *mixS = nullptr, *mixScore = nullptr;
+  float* gram = nullptr;
+  GemmDesc* dgram = nullptr;
+  int mix_nh = 1;
+  bool mix_tc = false;
   Descs dsc[2]{};
   TcPlan* tc[2]{};
   TcbPlan* tcb[2]{};
@@ -476,6 +485,8 @@ int check_arch(const lipz_arch* a) {
     return fail(nullptr, LIPZ_ERR_INVALID, "bad optimiser / mutation hyper-parameters");
   if (a->train_steps < 1 || a->train_steps > 65536)
     return fail(nullptr, LIPZ_ERR_INVALID, "train_steps must be in 1..65536");
+  if ((a->mixture != 0 && a->mixture != 1) || !(a->mix_sigma >= 0.f))
+    return fail(nullptr, LIPZ_ERR_INVALID, "mixture must be 0 or 1 and mix_sigma >= 0");
   return LIPZ_OK;
 }
 
@@ -529,8 +540,31 @@ int create_impl(lipz_grid* g) {
       (rc = dalloc(g, &g->A2, CB * h * es)) || (rc = dalloc(g, &g->A1, CB * h * es)) ||
       (rc = dalloc(g, &g->gG, (size_t)C * g->PGs * 4)) ||
       (rc = dalloc(g, &g->gD, (size_t)C * g->PDs * 4)) || (rc = dalloc(g, &g->flag, 4)) ||
-      (rc = dalloc(g, &g->xin, CB * x * 4)))
+      (rc = dalloc(g, &g->xin, CB * x * 4)) || (rc = dalloc(g, &g->mix, C * 5 * 4)))
     return rc;
+  {
+    std::vector<float> w(C * 5, 0.2f);
+    if ((rc = h2d(g, g->mix, w.data(), C * 5 * 4))) return rc;
+  }
+  if (g->a.mixture) {
+    const size_t R = (size_t)6 * B;
+    g->mix_tc = g->bf && !g->a.force_simt && tc_supported(z, h, x, B) && tc_gram_supported(B);
+    g->mix_nh = g->mix_tc ? tc_gram_halves(B) : 1;
+    if ((rc = dalloc(g, &g->rnorm, C * R * 4)) ||
+        (rc = dalloc(g, &g->mixP, C * R * g->mix_nh * 6 * 4)) ||
+        (rc = dalloc(g, &g->mixS, C * 36 * 4)) || (rc = dalloc(g, &g->mixScore, C * 4)) ||
+        (rc = dset(g, g->mixS, 0, C * 36 * 4)) || (rc = dset(g, g->mixScore, 0, C * 4)))
+      return rc;
+    if (!g->mix_tc) {
+      if ((rc = dalloc(g, &g->gram, C * R * R * 4))) return rc;
+      std::vector<GemmDesc> dg;
+      for (int c = 0; c < C; ++c)
+        dg.push_back(gd(eoff(g->E, (int64_t)c * g->e_cell, es), x, 1,
+                        eoff(g->E, (int64_t)c * g->e_cell, es), 1, x,
+                        g->gram + (int64_t)c * R * R, (int64_t)R, 1, (int)R, (int)R, x));
+      if ((rc = upload(g, &g->dgram, dg))) return rc;
+    }
+  }
   const int big = INT_MAX;
   if ((rc = dset(g, g->gG, 0, (size_t)C * g->PGs * 4)) ||
       (rc = dset(g, g->gD, 0, (size_t)C * g->PDs * 4)) || (rc = h2d(g, g->flag, &big, 4)))
@@ -566,6 +600,8 @@ int create_impl(lipz_grid* g) {
       b.sel_g = g->sel_g;
       b.src_g = g->src_g;
       b.src_d = g->src_d;
+      b.rnorm = g->mix_tc ? g->rnorm : nullptr;
+      b.gram_out = g->mix_tc ? g->mixP : nullptr;
       b.TH1 = g->TH1;
       b.TH2 = g->TH2;
       b.TG1 = g->TG1;
@@ -646,6 +682,32 @@ void draw_batch(lipz_grid* g, const float* xin_dev, uint32_t step, int parts, bo
                              g->st);
 }
 
+// Step 4 on the evaluation's rows (E: the real minibatch and the five slots' fakes): squared
+// row norms, the Gaussian-kernel block sums (tensor-core Gram kernel, or a stored Gram matrix
+// on the CUDA-core path), then every cell's ES-(1+1) step on its mixture weights.
+int mixture_impl(lipz_grid* g) {
+  const int C = g->cells, B = g->a.batch, x = g->a.x_dim, R = 6 * B;
+  phase_begin(g, LIPZ_PHASE_MIXTURE);
+  if (g->bf)
+    launch_row_norms<bf16>((const bf16*)g->E, g->e_cell, C, R, x, g->rnorm, g->st);
+  else
+    launch_row_norms<float>((const float*)g->E, g->e_cell, C, R, x, g->rnorm, g->st);
+  CKL(g);
+  if (g->mix_tc) {
+    std::string msg;
+    if (tc_run_gram(g->tc[g->cur], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+  } else {
+    gemm(g, g->dgram, C, R, R, EPI_STORE, ACT_NONE, true);
+    launch_mix_partials(g->gram, g->rnorm, C, R, B, x, g->mixP, g->st);
+  }
+  CKL(g);
+  launch_mix_es(g->mixP, g->mix_nh, C, R, B, g->mix, g->mixS, g->mixScore, g->seed,
+                (uint32_t)g->t, g->a.mix_sigma, g->st);
+  CKL(g);
+  phase_end(g, LIPZ_PHASE_MIXTURE, g->mix_tc ? 3 : 4);
+  return LIPZ_OK;
+}
+
 // Evaluation (minibatch, forwards, fitness); with `then_select` the selection runs in the
 // fitness kernel (the caller reads nothing back in between). With `x_ready`, the caller's
 // minibatch xin_dev is still being uploaded: the noise and the generator forward go first,
@@ -701,6 +763,10 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
     launch_fitness(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_FITNESS, 1);
+  if (g->a.mixture) {
+    int rc = mixture_impl(g);
+    if (rc) return rc;
+  }
   g->phase = then_select ? PH_SELECTED : PH_EVALUATED;
   return LIPZ_OK;
 }
@@ -991,6 +1057,8 @@ int lipz_arch_default(lipz_arch* a) {
   a->keep_grads = 0;
   a->force_simt = 0;
   a->train_steps = 1;
+  a->mixture = 0;
+  a->mix_sigma = 0.01f;
   return LIPZ_OK;
 }
 
@@ -1161,7 +1229,7 @@ int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* f
 int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {
   if (!g || !bytes) return LIPZ_ERR_INVALID;
   const size_t C = g->cells;
-  *bytes = 64 + C * (size_t)(g->PG + g->PD) * 3 * 4 + C * 16;
+  *bytes = 64 + C * (size_t)(g->PG + g->PD) * 3 * 4 + C * 16 + C * 20;
   return LIPZ_OK;
 }
 
@@ -1172,7 +1240,7 @@ int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
   if (!host || bytes != need)
     return fail(g, LIPZ_ERR_INVALID, "export_state needs a %zu-byte buffer", need);
   char* o = (char*)host;
-  uint32_t hdr[10] = {0x5A50494Cu, 1u, (uint32_t)g->rows, (uint32_t)g->cols,
+  uint32_t hdr[10] = {0x5A50494Cu, 2u, (uint32_t)g->rows, (uint32_t)g->cols,
                       (uint32_t)g->a.z_dim, (uint32_t)g->a.hidden, (uint32_t)g->a.x_dim,
                       (uint32_t)g->a.batch, (uint32_t)g->a.precision, 0u};
   memset(o, 0, 64);
@@ -1200,6 +1268,8 @@ int lipz_export_state(lipz_grid* g, void* host, size_t bytes) {
   CK(g, cudaMemcpyAsync(o, g->G[p].lr, C * 4, cudaMemcpyDeviceToHost, g->st));
   o += C * 4;
   CK(g, cudaMemcpyAsync(o, g->D[p].lr, C * 4, cudaMemcpyDeviceToHost, g->st));
+  o += C * 4;
+  CK(g, cudaMemcpyAsync(o, g->mix, C * 20, cudaMemcpyDeviceToHost, g->st));
   CK(g, cudaStreamSynchronize(g->st));
   return LIPZ_OK;
 }
@@ -1212,8 +1282,8 @@ int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   const char* s = (const char*)host;
   uint32_t hdr[10];
   memcpy(hdr, s, 40);
-  if (hdr[0] != 0x5A50494Cu || hdr[1] != 1u)
-    return fail(g, LIPZ_ERR_INVALID, "not a version-1 grid state");
+  if (hdr[0] != 0x5A50494Cu || hdr[1] != 2u)
+    return fail(g, LIPZ_ERR_INVALID, "not a version-2 grid state");
   if ((int)hdr[2] != g->rows || (int)hdr[3] != g->cols || (int)hdr[4] != g->a.z_dim ||
       (int)hdr[5] != g->a.hidden || (int)hdr[6] != g->a.x_dim || (int)hdr[7] != g->a.batch)
     return fail(g, LIPZ_ERR_INVALID, "state shape does not match this grid");
@@ -1242,6 +1312,8 @@ int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   CK(g, cudaMemcpyAsync(g->G[p].lr, s, C * 4, cudaMemcpyHostToDevice, g->st));
   s += C * 4;
   CK(g, cudaMemcpyAsync(g->D[p].lr, s, C * 4, cudaMemcpyHostToDevice, g->st));
+  s += C * 4;
+  CK(g, cudaMemcpyAsync(g->mix, s, C * 20, cudaMemcpyHostToDevice, g->st));
   if (g->bf) {
     launch_to_bf16(g->G[p].w, g->G[p].wb, (int64_t)C * g->PGs, g->st);
     launch_to_bf16(g->D[p].w, g->D[p].wb, (int64_t)C * g->PDs, g->st);
@@ -1267,6 +1339,18 @@ int lipz_get_batch(lipz_grid* g, float* x, float* z) {
   int rc;
   if (x && (rc = act_to_host(g, g->E, g->e_cell, g->cells, B * g->a.x_dim, x))) return rc;
   if (z && (rc = act_to_host(g, g->Z, B * g->a.z_dim, g->cells, B * g->a.z_dim, z))) return rc;
+  return LIPZ_OK;
+}
+
+int lipz_get_mixture(lipz_grid* g, float* weights, float* blocks, float* score) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if ((blocks || score) && !g->a.mixture)
+    return fail(g, LIPZ_ERR_STATE, "grid was created without mixture");
+  const size_t C = g->cells;
+  if (weights) CK(g, cudaMemcpyAsync(weights, g->mix, C * 20, cudaMemcpyDeviceToHost, g->st));
+  if (blocks) CK(g, cudaMemcpyAsync(blocks, g->mixS, C * 144, cudaMemcpyDeviceToHost, g->st));
+  if (score) CK(g, cudaMemcpyAsync(score, g->mixScore, C * 4, cudaMemcpyDeviceToHost, g->st));
+  CK(g, cudaStreamSynchronize(g->st));
   return LIPZ_OK;
 }
 

@@ -79,6 +79,14 @@ void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD,
 // (lr, 1 / (1 - beta1^(step+1)), 1 / (1 - beta2^(step+1)), step + 1).
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const SelectParams& p, const SelectIO& io, cudaStream_t st);
+// Generator-mixture score and ES-(1+1) step (rows = 6B evaluation rows per cell).
+template <typename T>
+void launch_row_norms(const T* E, int64_t e_cell, int cells, int rows, int x, float* out,
+                      cudaStream_t st);
+void launch_mix_partials(const float* gram, const float* rnorm, int cells, int rows, int B, int x,
+                         float* out, cudaStream_t st);
+void launch_mix_es(const float* part, int nh, int cells, int rows, int B, float* mix, float* S,
+                   float* score, uint64_t seed, uint32_t t, float sigma, cudaStream_t st);
 // Choice of every cell's own centre (slot 0), for the later minibatch steps of an iteration.
 void launch_centre_select(int cells, const SelectParams& p, const SelectIO& io, cudaStream_t st);
 // Fitness and, in the same kernel, the selection of every cell (when nothing is read back

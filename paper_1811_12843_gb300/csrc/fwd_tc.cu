@@ -47,8 +47,8 @@ constexpr int BIAS_MAX = 256 + 256 + 1024;  // floats per tile: b1, b2, then b3 
 constexpr int BIAS_BYTES = 2 * BIAS_MAX * 4;  // double-buffered by tile
 constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + H_BYTES + MISC_BYTES + BIAS_BYTES;
 
-enum { KIND_G = 0, KIND_D = 1 };
-enum { EPI_TO_H = 0, EPI_LOGIT = 1, EPI_TO_E = 2, EPI_ACT_OUT = 3 };
+enum { KIND_G = 0, KIND_D = 1, KIND_GRAM = 2 };
+enum { EPI_TO_H = 0, EPI_LOGIT = 1, EPI_TO_E = 2, EPI_ACT_OUT = 3, EPI_GRAM = 4 };
 
 struct KParams {
   int kind;
@@ -81,6 +81,12 @@ struct KParams {
   // centre-only generator forward (non-zero): problem c is cell c's own generator on z_c,
   // written to E[c] as the fakes of slot 0
   int centre;
+  // Gram kind (mixture score): problem c is the Gram matrix of E[c]'s rows with themselves,
+  // reduced in the epilogue to per-row sums of exp(-||e_r - e_s||^2 / x) over the columns s of
+  // each block of B rows. rnorm [cells][rows] holds ||e_r||^2; the sums go to
+  // gram_out[cell][row][half][6], half = 2 * column block + column half of the tile.
+  const float* rnorm;
+  float* gram_out;
 };
 
 struct Job {
@@ -96,7 +102,11 @@ struct Job {
 
 __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   Job J;
-  if (j == 0) {
+  if (p.kind == KIND_GRAM) {
+    // column block j of the Gram matrix: MMA N rounded up to 16 (rows past 6B read as zero)
+    const int n = min(HID, p.rows - j * HID);
+    J = Job{0, p.kc1, (n + 15) & ~15, j & 1, 0, j * HID, HID, EPI_GRAM};
+  } else if (j == 0) {
     J = Job{0, p.kc1, HID, 0, 0, 0, HID, EPI_TO_H};
   } else if (j == 1) {
     const int epi = p.kind == KIND_D ? EPI_LOGIT : (p.train ? EPI_ACT_OUT : EPI_TO_H);
@@ -112,16 +122,17 @@ __device__ __forceinline__ Job get_job(const KParams& p, int j) {
 }
 
 __device__ __forceinline__ int n_jobs(const KParams& p) {
+  if (p.kind == KIND_GRAM) return (p.rows + HID - 1) / HID;
   return (p.kind == KIND_D || p.train) ? 2 : 2 + p.n3;
 }
 
 // Problem -> (cell whose activations are the A operand, individual whose weights are B).
 __device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
-  return (p.train || p.centre) ? prob : prob / 5;
+  return (p.train || p.centre || p.kind == KIND_GRAM) ? prob : prob / 5;
 }
 __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
-  return p.centre ? prob : __ldg(&p.nbr[prob]);
+  return (p.centre || p.kind == KIND_GRAM) ? prob : __ldg(&p.nbr[prob]);
 }
 
 // Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
@@ -312,7 +323,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
       const int c = prob_cell(p, prob), slot = p.centre ? 0 : prob % 5;
       const int k = prob_individual(p, prob);
-      const float* wm = p.wmaster + (int64_t)k * p.pstride;
+      const float* wm = p.wmaster ? p.wmaster + (int64_t)k * p.pstride : nullptr;
       const int rr = m0 + row;
       const bool row_ok = rr < p.rows;
       const int64_t act_off = ((int64_t)prob * p.rows + rr) * HID;
@@ -320,7 +331,17 @@ __global__ void __launch_bounds__(THREADS, 1)
       // run, so that no epilogue waits on a global load. Buffer ltile & 1; a thread cannot
       // reach tile ltile + 2 before every thread has passed this tile's arrival.
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
-      {
+      if (p.kind == KIND_GRAM) {
+        // the squared norms of the cell's rows (the Gram tile's row and column terms)
+        for (int i = et; i < p.rows; i += 32 * NUM_EPI_WARPS)
+          sb[i] = __ldg(&p.rnorm[(int64_t)c * p.rows + i]);
+        mbar_arrive(bBias + 8 * (ltile & 1));
+        if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
+                            p.err, 8)) {
+          ok = false;
+          break;
+        }
+      } else {
         // every load is issued before the first is stored, so their latencies overlap
         const int nb3 = p.kind == KIND_D ? HID + 1 : p.x;
         constexpr int NV = (BIAS_MAX + 32 * NUM_EPI_WARPS - 1) / (32 * NUM_EPI_WARPS);
@@ -476,6 +497,46 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_arrive(bReg + 8 * R);
             if (row_ok) p.logits[(int64_t)prob * p.rows + rr] = logit;
           }
+        } else if (J.epi == EPI_GRAM) {
+          // Gaussian kernel exp(-(|e_r|^2 + |e_s|^2 - 2 e_r.e_s) / x) of this thread's row r
+          // against the warp's 128 columns s, summed per column block of B rows, columns in
+          // increasing order (the block boundary is the same for every lane)
+          const float nr = row_ok ? sb[rr] : 0.f;
+          const float inv_x = 1.f / (float)p.x;
+          float acc[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+          for (int cg = hf * 4; cg < hf * 4 + 4; ++cg) {
+            const int col0 = J.brow0 + cg * 32;
+            if (col0 >= p.rows) break;
+            uint32_t r[32];
+            LIPZ_TMEM_LD32(tbase + cg * 32, r);
+            tmem_wait_ld();
+            int blk = col0 / p.B;
+            int next = (blk + 1) * p.B;
+            float sum = 0.f;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int col = col0 + e;
+              if (col >= next) {
+#pragma unroll
+                for (int t = 0; t < 6; ++t) acc[t] += t == blk ? sum : 0.f;
+                sum = 0.f;
+                ++blk;
+                next += p.B;
+              }
+              if (col < p.rows)
+                sum += __expf(-(nr + sb[col] - 2.f * __uint_as_float(r[e])) * inv_x);
+            }
+#pragma unroll
+            for (int t = 0; t < 6; ++t) acc[t] += t == blk ? sum : 0.f;
+          }
+          tc_fence_before();
+          mbar_arrive(bReg + 8 * R);
+          if (row_ok) {
+            float* o = p.gram_out + (((int64_t)c * p.rows + rr) * (2 * nj) + 2 * j + hf) * 6;
+#pragma unroll
+            for (int t = 0; t < 6; ++t) o[t] = acc[t];
+          }
         } else {
           // generator output block: bias + tanh, bf16, into the fake rows of E[c]
           const float* bias = sb + 512;
@@ -534,9 +595,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 // ---- host side -----------------------------------------------------------------------------
 struct TcPlan {
   TcShape s;
-  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mE4;
-  tc::KParams pg, pgc, pd, pgt, pdt;
-  int grid_g, grid_gc, grid_d, grid_gt, grid_dt;
+  CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mE4, mEB;
+  tc::KParams pg, pgc, pd, pgt, pdt, pgram;
+  int grid_g, grid_gc, grid_d, grid_gt, grid_dt, grid_gram;
   int* err;
 };
 
@@ -616,6 +677,7 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   const uint64_t C = s.cells, B = s.B, z = s.z, x = s.x, h = s.h;
   bool ok = make_map(&p->mZ, b.Z, z, B, C, z * 2, B * z * 2, 128, msg) &&
             make_map(&p->mE, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 128, msg) &&
+            make_map(&p->mEB, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 256, msg) &&
             make_map4(&p->mE4, b.E, x, B, 6, C, x * 2, B * x * 2, (uint64_t)b.e_cell * 2, msg) &&
             make_map(&p->mG1, b.Gwb + b.goff[0], z, h, C, z * 2, b.PGs * 2, 256, msg) &&
             make_map(&p->mG2, b.Gwb + b.goff[2], h, h, C, h * 2, b.PGs * 2, 256, msg) &&
@@ -702,14 +764,31 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   dt.act1 = (bf16*)b.TG1;
   dt.act2 = (bf16*)b.TG2;
   dt.logits = b.TL;
+  tc::KParams gm{};  // Gram matrix of every cell's evaluation rows (mixture score)
+  gm.kind = tc::KIND_GRAM;
+  gm.cells = s.cells;
+  gm.B = s.B;
+  gm.z = s.z;
+  gm.x = s.x;
+  gm.rows = 6 * s.B;
+  gm.mtiles = tiles(6 * s.B);
+  gm.n_tiles = s.cells * gm.mtiles;
+  gm.kc1 = (s.x + tc::BK - 1) / tc::BK;
+  gm.E = (bf16*)b.E;
+  gm.e_cell = b.e_cell;
+  gm.err = p->err;
+  gm.rnorm = b.rnorm;
+  gm.gram_out = b.gram_out;
   p->pg = g;
   p->pgc = gc;
+  p->pgram = gm;
   p->pd = d;
   p->pgt = gt;
   p->pdt = dt;
   auto grid = [sms](int n) { return n < sms ? n : sms; };
   p->grid_g = grid(g.n_tiles);
   p->grid_gc = grid(gc.n_tiles);
+  p->grid_gram = grid(gm.n_tiles);
   p->grid_d = grid(d.n_tiles);
   p->grid_gt = grid(gt.n_tiles);
   p->grid_dt = grid(dt.n_tiles);
@@ -738,6 +817,18 @@ int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg) {
   return launch(p->grid_gc, p->mZ, p->mG1, p->mG2, p->mG3, p->pgc, st, "centre generator forward",
                 msg);
 }
+
+int tc_run_gram(TcPlan* p, cudaStream_t st, std::string* msg) {
+  if (!p->pgram.rnorm || !p->pgram.gram_out || 6 * p->s.B > tc::BIAS_MAX) {
+    if (msg) *msg = "tensor-core Gram kernel: no buffers or batch above 256";
+    return 1;
+  }
+  return launch(p->grid_gram, p->mE, p->mEB, p->mEB, p->mEB, p->pgram, st, "mixture Gram", msg);
+}
+
+int tc_gram_halves(int B) { return 2 * ((6 * B + tc::HID - 1) / tc::HID); }
+
+bool tc_gram_supported(int B) { return 6 * B <= tc::BIAS_MAX; }
 
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg) {
   return launch(p->grid_d, p->mE, p->mD1, p->mD2, p->mD2, p->pd, st, "discriminator forward",

@@ -43,6 +43,10 @@ struct TcBuffers {
   const float* Dw;
   int64_t PDs;
   const int64_t* doff;
+  // mixture score: squared norms of E's rows [cells][6B] fp32 (input) and the Gram kernel's
+  // per-row block sums [cells][6B][tc_gram_halves(B)][6] fp32 (output); null without mixture
+  const float* rnorm;
+  float* gram_out;
   const int* sel_g;  // slot of each cell's selected generator (training: its fakes in E)
   const int* src_g;
   const int* src_d;
@@ -60,6 +64,12 @@ int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
 // Generator forward of every cell's own centre on its z, into E's slot-0 fakes.
 int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
+// Mixture score: for every cell c and row r of E[c], the sums over each block b of B columns
+// s of exp(-||E[c][r] - E[c][s]||^2 / x), into gram_out[c][r][h][b] split over the
+// tc_gram_halves(B) column ranges h (6B <= 1536, i.e. tc_gram_supported).
+int tc_run_gram(TcPlan* p, cudaStream_t st, std::string* msg);
+int tc_gram_halves(int B);
+bool tc_gram_supported(int B);
 // Training forward of every cell's selected generator (hidden activations into TH1, TH2) and
 // selected discriminator (TG1, TG2 and the logits TL).
 int tc_run_train_g(TcPlan* p, cudaStream_t st, std::string* msg);

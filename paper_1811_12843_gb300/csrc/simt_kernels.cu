@@ -796,4 +796,130 @@ void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, flo
   launch_pdl(k_adam_ranges, dim3(cells, 2), dim3(256), 0, st, g, d, beta1, beta2, eps);
 }
 
+// ------------------------------------------------------------------------------------------
+// Generator-mixture score (Section 3 step 4): squared norms of the evaluation rows, the Gaussian
+// kernel's block sums (from a stored Gram matrix on the CUDA-core path), and the ES-(1+1) step.
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_row_norms(const T* __restrict__ E, int64_t e_cell, int rows, int x,
+                            float* __restrict__ out) {
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
+  if (r >= rows) return;
+  const T* e = E + (int64_t)c * e_cell + (int64_t)r * x;
+  float s = 0.f;
+  for (int k = lane; k < x; k += 32) {
+    const float v = to_f<T>(e[k]);
+    s = fmaf(v, v, s);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) out[(int64_t)c * rows + r] = s;
+}
+
+template <typename T>
+void launch_row_norms(const T* E, int64_t e_cell, int cells, int rows, int x, float* out,
+                      cudaStream_t st) {
+  launch_pdl(k_row_norms<T>, dim3((rows + 7) / 8, cells), dim3(256), 0, st, E, e_cell, rows, x,
+             out);
+}
+template void launch_row_norms<float>(const float*, int64_t, int, int, int, float*, cudaStream_t);
+template void launch_row_norms<bf16>(const bf16*, int64_t, int, int, int, float*, cudaStream_t);
+
+// One warp per row r of cell c: for each block b of B columns, the sum over its columns s (in
+// lane-strided order, then a fixed shuffle tree) of exp(-(n_r + n_s - 2 gram[r][s]) / x).
+__global__ void k_mix_partials(const float* __restrict__ gram, const float* __restrict__ rnorm,
+                               int rows, int B, int x, float* __restrict__ out) {
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
+  if (r >= rows) return;
+  const float* gr = gram + ((int64_t)c * rows + r) * rows;
+  const float* n = rnorm + (int64_t)c * rows;
+  const float nr = n[r], inv_x = 1.f / (float)x;
+  for (int b = 0; b < rows / B; ++b) {
+    float s = 0.f;
+    for (int q = b * B + lane; q < (b + 1) * B; q += 32)
+      s += __expf(-(nr + n[q] - 2.f * gr[q]) * inv_x);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) out[((int64_t)c * rows + r) * 6 + b] = s;
+  }
+}
+
+void launch_mix_partials(const float* gram, const float* rnorm, int cells, int rows, int B, int x,
+                         float* out, cudaStream_t st) {
+  launch_pdl(k_mix_partials, dim3((rows + 7) / 8, cells), dim3(256), 0, st, gram, rnorm, rows, B,
+             x, out);
+}
+
+__device__ __forceinline__ float mix_mmd2(const float* w, const float* S) {
+  // sum_ij w_i w_j S[1+i][1+j] - 2 sum_i w_i S[1+i][0] + S[0][0]
+  float q = 0.f, l = 0.f;
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
+    float row = 0.f;
+#pragma unroll
+    for (int j = 0; j < 5; ++j) row = fmaf(w[j], S[(1 + i) * 6 + 1 + j], row);
+    q = fmaf(w[i], row, q);
+    l = fmaf(w[i], S[(1 + i) * 6], l);
+  }
+  return q - 2.f * l + S[0];
+}
+
+// One block per cell: the 6x6 block means S[a][b] = (sum over the rows r of block a and the
+// column ranges h of part[c][r][h][b]) / B^2, then the ES-(1+1) step of the cell's weights w:
+// w' = max(w + sigma n, 0) / sum (n: the first five normals of stream MIX at iteration t; w kept
+// if the sum is 0), kept iff its squared MMD is lower.
+__global__ void k_mix_es(const float* __restrict__ part, int nh, int rows, int B, float* mix,
+                         float* __restrict__ S_out, float* __restrict__ score_out, uint64_t seed,
+                         uint32_t t, float sigma) {
+  pdl_wait();
+  const int c = blockIdx.x;
+  __shared__ float S[36];
+  const int i = threadIdx.x;
+  if (i < 36) {
+    const int a = i / 6, b = i % 6;
+    float s = 0.f;
+    for (int r = a * B; r < (a + 1) * B; ++r)
+      for (int h = 0; h < nh; ++h) s += part[(((int64_t)c * rows + r) * nh + h) * 6 + b];
+    S[i] = s / ((float)B * (float)B);
+    S_out[(int64_t)c * 36 + i] = S[i];
+  }
+  __syncthreads();
+  if (i != 0) return;
+  float w[5], cand[5], nrm[5];
+  const U4 r0 = philox_block(seed, 9u, t, (uint32_t)c, 0u);
+  const U4 r1 = philox_block(seed, 9u, t, (uint32_t)c, 1u);
+  const float2 n01 = box_muller(r0.x, r0.y), n23 = box_muller(r0.z, r0.w),
+               n4 = box_muller(r1.x, r1.y);
+  nrm[0] = n01.x;
+  nrm[1] = n01.y;
+  nrm[2] = n23.x;
+  nrm[3] = n23.y;
+  nrm[4] = n4.x;
+  float tot = 0.f;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    w[k] = mix[c * 5 + k];
+    cand[k] = fmaxf(fmaf(sigma, nrm[k], w[k]), 0.f);
+    tot += cand[k];
+  }
+#pragma unroll
+  for (int k = 0; k < 5; ++k) cand[k] = tot > 0.f ? cand[k] / tot : w[k];
+  const float old = mix_mmd2(w, S), nw = mix_mmd2(cand, S);
+  const bool acc = nw < old;
+  if (acc)
+#pragma unroll
+    for (int k = 0; k < 5; ++k) mix[c * 5 + k] = cand[k];
+  score_out[c] = acc ? nw : old;
+}
+
+void launch_mix_es(const float* part, int nh, int cells, int rows, int B, float* mix, float* S,
+                   float* score, uint64_t seed, uint32_t t, float sigma, cudaStream_t st) {
+  launch_pdl(k_mix_es, dim3(cells), dim3(64), 0, st, part, nh, rows, B, mix, S, score, seed, t,
+             sigma);
+}
+
 }  // namespace lipz
