@@ -9,10 +9,11 @@ one full grid iteration (minibatch draw, all-pairs evaluation, fitness, selectio
 Adam of every cell's new centre pair).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--train-steps S]
+                  [--train-steps S] [--mixture]
 
 With --train-steps S > 1 every iteration trains each cell's new centre pair S times (the later
-steps on fresh minibatches); the default S = 1 is the headline workload.
+steps on fresh minibatches); the default S = 1 is the headline workload. --mixture adds the
+generator-mixture ES-(1+1) step (Gaussian-kernel MMD score) to every evaluation.
 
 With N > 1 (torchrun, one process per GPU) every rank runs its own 12x12 grid (replicas: the
 per-GPU work is fixed, scaling "weak"); value = all ranks' pairs / the slowest rank's time.
@@ -50,6 +51,8 @@ PD = HIDDEN * X_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + HIDDEN + 1
 # Training: forward of the selected pair (G layers 1-2 on B rows, D on 2B rows) and backward.
 TRAIN_FWD_FLOP = 2 * CELLS * BATCH * (Z_DIM * HIDDEN + HIDDEN * HIDDEN) + 2 * CELLS * 2 * BATCH * D_MAC_ROW
 TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
+# Mixture step (--mixture): the Gram matrix of every cell's 6B evaluation rows.
+MIX_FLOP = 2 * CELLS * (6 * BATCH) ** 2 * X_DIM
 # The backward kernel applies Adam to the weight matrices (G: W1, W2, W3; D: W1, W2) in its
 # epilogue: per such parameter it reads the old w, m, v (12 B) and writes the new w, m, v and
 # the bf16 copy (14 B). Its other algorithmic reads: the bf16 weights of the four matrices the
@@ -165,7 +168,7 @@ def run_ours(args):
 
     pool = lipz_synth.blob_pool(SEED, n=POOL_N, dim=X_DIM)
     g = L.Grid(ROWS, COLS, seed=SEED + rank, precision="bf16", batch=BATCH,
-               train_steps=args.train_steps)
+               train_steps=args.train_steps, mixture=1 if args.mixture else 0)
     g.set_data(pool)
     stream = torch.cuda.Stream()
     g.set_stream(stream.cuda_stream)
@@ -240,7 +243,7 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
-    if world == 1 and not args.no_cpu_baseline and args.train_steps == 1:
+    if world == 1 and not args.no_cpu_baseline and args.train_steps == 1 and not args.mixture:
         line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
     return line
 
@@ -271,6 +274,8 @@ def _phase_roofs(phase_ms):
             "d_fwd": ("tensor", EVAL_D_FLOP,
                       "discriminator evaluation forward (all 720 slots, 3 fused layers + logit)"),
             "train_fwd": ("tensor", TRAIN_FWD_FLOP, "forward of every cell's selected pair"),
+            "mixture": ("tensor", MIX_FLOP, "mixture score: Gram of every cell's 6B evaluation "
+                        "rows with the Gaussian kernel and block sums fused, plus the ES step"),
             "train_bwd": ("hbm", TRAIN_BWD_BYTES,
                           "backward of every cell's selected pair with Adam + replacement of "
                           "the weight matrices fused in (%.1f GFLOP)" % (TRAIN_BWD_FLOP / 1e9))}
@@ -300,10 +305,11 @@ def _roofline(phase_ms):
     return r
 
 
-def _oracle_sample(seconds, max_cells=None, train_steps=1):
+def _oracle_sample(seconds, max_cells=None, train_steps=1, mixture=False):
     """Run the oracle's full iteration cell by cell on the 12x12 workload until ``seconds`` of
     CPU work are spent; return (cells done, elapsed seconds). With ``train_steps`` K > 1 each
-    cell's pair then takes K - 1 more steps on fresh minibatches."""
+    cell's pair then takes K - 1 more steps on fresh minibatches; with ``mixture`` each cell also
+    takes its mixture ES step."""
     import numpy as np
     import lipz_synth
     from oracle import lipz_oracle as O
@@ -319,6 +325,8 @@ def _oracle_sample(seconds, max_cells=None, train_steps=1):
         cells = [c]
         data = O.batches(state, pool, cells=cells)
         ev = O.eval_neighborhoods(state, data, cells=cells)
+        if mixture:
+            O.mixture_update(state, data, cells=cells)
         a = state.arch
         sg = O.select_slot(ev["fG"][c], O.draw_words(state.seed, O.STREAM_TOUR_G, state.t, c,
                                                      a.tournament_size), a)
@@ -369,9 +377,12 @@ def cpu_baseline(seconds):
 
 
 def _workload(args):
-    if args.train_steps == 1:
-        return WORKLOAD
-    return "%s, %d minibatch steps per iteration" % (WORKLOAD, args.train_steps)
+    w = WORKLOAD
+    if args.train_steps != 1:
+        w += ", %d minibatch steps per iteration" % args.train_steps
+    if args.mixture:
+        w += ", mixture ES step"
+    return w
 
 
 def run_reference(args):
@@ -383,11 +394,12 @@ def run_reference(args):
     _oracle_state(arch)
     per_step_cells = 1
     for _ in range(args.warmup):
-        _oracle_sample(1e9, max_cells=1, train_steps=args.train_steps)
+        _oracle_sample(1e9, max_cells=1, train_steps=args.train_steps, mixture=args.mixture)
     times = []
     total_cells = 0
     for _ in range(args.steps):
-        done, el = _oracle_sample(1e9, max_cells=per_step_cells, train_steps=args.train_steps)
+        done, el = _oracle_sample(1e9, max_cells=per_step_cells, train_steps=args.train_steps,
+                                  mixture=args.mixture)
         times.append(el)
         total_cells += done
     el = sum(times)
@@ -419,6 +431,8 @@ def main():
     ap.add_argument("--no-phases", action="store_true", help="skip the per-phase timing pass")
     ap.add_argument("--train-steps", type=int, default=1,
                     help="Adam steps per grid iteration (the later ones on fresh minibatches)")
+    ap.add_argument("--mixture", action="store_true",
+                    help="add the generator-mixture ES step to every iteration")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
