@@ -260,10 +260,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       int reg_uses[2] = {0, 0};
       int h_total = 0;  // activations written to H so far (each chunk barrier: one phase each)
       bool ok = true;
+      int jobs_done = 0;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
-        for (int j = 0; j < nj && ok; ++j) {
+        for (int j = 0; j < nj && ok; ++j, ++jobs_done) {
           const Job J = get_job(p, j);
-          const int R = J.region;
+          // the Gram kind alternates the two accumulators over all its jobs (3 per tile)
+          const int R = p.kind == KIND_GRAM ? (jobs_done & 1) : J.region;
           if (reg_uses[R] > 0 &&
               !mbar_wait(bReg + 8 * R, (uint32_t)((reg_uses[R] - 1) & 1), abort_flag, p.err, 2)) {
             ok = false;
@@ -317,7 +319,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     int reg_uses[2] = {0, 0};
     bool ok = true;
-    int ltile = 0;
+    int ltile = 0, jobs_done = 0;
     const int et = threadIdx.x - 64;  // epilogue thread 0..255
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++ltile) {
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
@@ -333,8 +335,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
       if (p.kind == KIND_GRAM) {
         // the squared norms of the cell's rows (the Gram tile's row and column terms)
-        for (int i = et; i < p.rows; i += 32 * NUM_EPI_WARPS)
-          sb[i] = __ldg(&p.rnorm[(int64_t)c * p.rows + i]);
+        // -|e_s|^2 / x for the cell's rows s, zero for the 32 entries past the last row
+        const float ix = 1.f / (float)p.x;
+        for (int i = et; i < p.rows + 32; i += 32 * NUM_EPI_WARPS)
+          sb[i] = i < p.rows ? -__ldg(&p.rnorm[(int64_t)c * p.rows + i]) * ix : 0.f;
         mbar_arrive(bBias + 8 * (ltile & 1));
         if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
                             p.err, 8)) {
@@ -371,9 +375,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         }
       }
-      for (int j = 0; j < nj && ok; ++j) {
+      for (int j = 0; j < nj && ok; ++j, ++jobs_done) {
         const Job J = get_job(p, j);
-        const int R = J.region;
+        const int R = p.kind == KIND_GRAM ? (jobs_done & 1) : J.region;
         if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
           ok = false;
           break;
@@ -498,11 +502,13 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (row_ok) p.logits[(int64_t)prob * p.rows + rr] = logit;
           }
         } else if (J.epi == EPI_GRAM) {
-          // Gaussian kernel exp(-(|e_r|^2 + |e_s|^2 - 2 e_r.e_s) / x) of this thread's row r
-          // against the warp's 128 columns s, summed per column block of B rows, columns in
-          // increasing order (the block boundary is the same for every lane)
+          // Gaussian kernel exp((2 e_r.e_s - |e_r|^2 - |e_s|^2) / x) of this thread's row r
+          // against the warp's 128 columns s, summed per column block of B >= 32 rows: a group
+          // of 32 columns meets at most one block boundary (at column sp of the group, the same
+          // for every lane), columns past the last row count zero; two interleaved partial sums
+          // per side, combined in a fixed order
           const float nr = row_ok ? sb[rr] : 0.f;
-          const float inv_x = 1.f / (float)p.x;
+          const float two_ix = 2.f / (float)p.x;
           float acc[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll 1
           for (int cg = hf * 4; cg < hf * 4 + 4; ++cg) {
@@ -511,24 +517,33 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t r[32];
             LIPZ_TMEM_LD32(tbase + cg * 32, r);
             tmem_wait_ld();
-            int blk = col0 / p.B;
-            int next = (blk + 1) * p.B;
-            float sum = 0.f;
+            const int blk = col0 / p.B;
+            const int sp = (blk + 1) * p.B - col0;
+            const int nv = p.rows - col0;
+            const float4* s4 = reinterpret_cast<const float4*>(sb + col0);
+            float lo0 = 0.f, lo1 = 0.f, hi0 = 0.f, hi1 = 0.f;
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int col = col0 + e;
-              if (col >= next) {
+            for (int q = 0; q < 8; ++q) {
+              const float4 ns = s4[q];
+              const float nsv[4] = {ns.x, ns.y, ns.z, ns.w};
 #pragma unroll
-                for (int t = 0; t < 6; ++t) acc[t] += t == blk ? sum : 0.f;
-                sum = 0.f;
-                ++blk;
-                next += p.B;
+              for (int u = 0; u < 4; ++u) {
+                const int e = 4 * q + u;
+                float v = __expf(fmaf(__uint_as_float(r[e]), two_ix, nr + nsv[u]));
+                v = e < nv ? v : 0.f;
+                const float vl = e < sp ? v : 0.f, vh = e < sp ? 0.f : v;
+                if (e & 1) {
+                  lo1 += vl;
+                  hi1 += vh;
+                } else {
+                  lo0 += vl;
+                  hi0 += vh;
+                }
               }
-              if (col < p.rows)
-                sum += __expf(-(nr + sb[col] - 2.f * __uint_as_float(r[e])) * inv_x);
             }
+            const float lo = lo0 + lo1, hi = hi0 + hi1;
 #pragma unroll
-            for (int t = 0; t < 6; ++t) acc[t] += t == blk ? sum : 0.f;
+            for (int t = 0; t < 6; ++t) acc[t] += t == blk ? lo : (t == blk + 1 ? hi : 0.f);
           }
           tc_fence_before();
           mbar_arrive(bReg + 8 * R);
@@ -819,8 +834,8 @@ int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int tc_run_gram(TcPlan* p, cudaStream_t st, std::string* msg) {
-  if (!p->pgram.rnorm || !p->pgram.gram_out || 6 * p->s.B > tc::BIAS_MAX) {
-    if (msg) *msg = "tensor-core Gram kernel: no buffers or batch above 256";
+  if (!p->pgram.rnorm || !p->pgram.gram_out || !tc_gram_supported(p->s.B)) {
+    if (msg) *msg = "tensor-core Gram kernel: no buffers, or batch outside 32..250";
     return 1;
   }
   return launch(p->grid_gram, p->mE, p->mEB, p->mEB, p->mEB, p->pgram, st, "mixture Gram", msg);
@@ -828,7 +843,9 @@ int tc_run_gram(TcPlan* p, cudaStream_t st, std::string* msg) {
 
 int tc_gram_halves(int B) { return 2 * ((6 * B + tc::HID - 1) / tc::HID); }
 
-bool tc_gram_supported(int B) { return 6 * B <= tc::BIAS_MAX; }
+// B >= 32: a 32-column group meets at most one block boundary; the norms and 32 zero entries
+// past them fit one bias buffer
+bool tc_gram_supported(int B) { return B >= 32 && 6 * B + 32 <= tc::BIAS_MAX; }
 
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg) {
   return launch(p->grid_d, p->mE, p->mD1, p->mD2, p->mD2, p->pd, st, "discriminator forward",

@@ -66,7 +66,7 @@ int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);
 // Mixture score: for every cell c and row r of E[c], the sums over each block b of B columns
 // s of exp(-||E[c][r] - E[c][s]||^2 / x), into gram_out[c][r][h][b] split over the
-// tc_gram_halves(B) column ranges h (6B <= 1536, i.e. tc_gram_supported).
+// tc_gram_halves(B) column ranges h (32 <= B <= 250, i.e. tc_gram_supported).
 int tc_run_gram(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_gram_halves(int B);
 bool tc_gram_supported(int B);

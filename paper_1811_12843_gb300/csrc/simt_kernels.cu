@@ -871,24 +871,36 @@ __device__ __forceinline__ float mix_mmd2(const float* w, const float* S) {
 // One block per cell: the 6x6 block means S[a][b] = (sum over the rows r of block a and the
 // column ranges h of part[c][r][h][b]) / B^2, then the ES-(1+1) step of the cell's weights w:
 // w' = max(w + sigma n, 0) / sum (n: the first five normals of stream MIX at iteration t; w kept
-// if the sum is 0), kept iff its squared MMD is lower.
-__global__ void k_mix_es(const float* __restrict__ part, int nh, int rows, int B, float* mix,
-                         float* __restrict__ S_out, float* __restrict__ score_out, uint64_t seed,
-                         uint32_t t, float sigma) {
+// if the sum is 0), kept iff its squared MMD is lower. Warp a sums block a's rows: lane l takes
+// rows l, l + 32, ... (all h), then a fixed shuffle tree.
+__global__ void __launch_bounds__(192) k_mix_es(const float* __restrict__ part, int nh, int rows,
+                                                int B, float* mix, float* __restrict__ S_out,
+                                                float* __restrict__ score_out, uint64_t seed,
+                                                uint32_t t, float sigma) {
   pdl_wait();
   const int c = blockIdx.x;
   __shared__ float S[36];
-  const int i = threadIdx.x;
-  if (i < 36) {
-    const int a = i / 6, b = i % 6;
-    float s = 0.f;
-    for (int r = a * B; r < (a + 1) * B; ++r)
-      for (int h = 0; h < nh; ++h) s += part[(((int64_t)c * rows + r) * nh + h) * 6 + b];
-    S[i] = s / ((float)B * (float)B);
-    S_out[(int64_t)c * 36 + i] = S[i];
+  const int a = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float acc[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int r = a * B + lane; r < (a + 1) * B; r += 32) {
+    const float* q = part + ((int64_t)c * rows + r) * nh * 6;
+    for (int h = 0; h < nh; ++h) {
+#pragma unroll
+      for (int b = 0; b < 6; ++b) acc[b] += q[h * 6 + b];
+    }
+  }
+#pragma unroll
+  for (int b = 0; b < 6; ++b) {
+    float v = acc[b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) {
+      S[a * 6 + b] = v / ((float)B * (float)B);
+      S_out[(int64_t)c * 36 + a * 6 + b] = S[a * 6 + b];
+    }
   }
   __syncthreads();
-  if (i != 0) return;
+  if (threadIdx.x != 0) return;
   float w[5], cand[5], nrm[5];
   const U4 r0 = philox_block(seed, 9u, t, (uint32_t)c, 0u);
   const U4 r1 = philox_block(seed, 9u, t, (uint32_t)c, 1u);
@@ -909,16 +921,16 @@ __global__ void k_mix_es(const float* __restrict__ part, int nh, int rows, int B
 #pragma unroll
   for (int k = 0; k < 5; ++k) cand[k] = tot > 0.f ? cand[k] / tot : w[k];
   const float old = mix_mmd2(w, S), nw = mix_mmd2(cand, S);
-  const bool acc = nw < old;
-  if (acc)
+  const bool acc_new = nw < old;
+  if (acc_new)
 #pragma unroll
     for (int k = 0; k < 5; ++k) mix[c * 5 + k] = cand[k];
-  score_out[c] = acc ? nw : old;
+  score_out[c] = acc_new ? nw : old;
 }
 
 void launch_mix_es(const float* part, int nh, int cells, int rows, int B, float* mix, float* S,
                    float* score, uint64_t seed, uint32_t t, float sigma, cudaStream_t st) {
-  launch_pdl(k_mix_es, dim3(cells), dim3(64), 0, st, part, nh, rows, B, mix, S, score, seed, t,
+  launch_pdl(k_mix_es, dim3(cells), dim3(192), 0, st, part, nh, rows, B, mix, S, score, seed, t,
              sigma);
 }
 

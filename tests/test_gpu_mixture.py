@@ -70,6 +70,7 @@ def _check_mixture(g, pool, cells=None):
     ("bf16", 3, 3, 100),    # tensor-core Gram kernel: 600 rows = 5 row tiles, 3 column blocks
     ("bf16", 2, 3, 129),    # 774 rows: ragged row tile and a 6-column last block
     ("bf16", 1, 1, 37),     # degenerate torus, one column block of 222
+    ("bf16", 2, 2, 20),     # batch below 32: the stored-Gram path in bf16
 ])
 def test_mixture_step_against_the_oracle(L, precision, rows, cols, batch):
     pool = _pool(21, 4000, 784)
