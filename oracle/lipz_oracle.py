@@ -19,7 +19,10 @@ Training", steps 1-3 and 5) and its settings table (Table 1), written as plain n
 Readings where the paper is silent (each is listed in the design doc with its reason):
   * fitness is a loss for both populations, lower is better: f_G = mean_j L_G, f_D = mean_i L_D;
   * L_D is the SUM of the real-batch and fake-batch BCE means; L_G is the non-saturating loss;
-  * iterations run on a synchronous snapshot of all centres;
+  * iterations run on a synchronous snapshot of all centres; with ``stale_neighbors`` (the
+    asynchronous schedule of Section 3 emulated deterministically) a cell sees its own centre
+    as of the iteration and its four neighbours as they were one iteration earlier (at the
+    first iteration: as they are), both for the evaluation and as selection sources;
   * tournament entrants are distinct slots; a tie goes to the lower slot; the centre is replaced
     by the winner only if the winner's fitness is strictly lower (``if_better``) -- or always;
   * the pair is trained on the same minibatch that was used for its evaluation, with the fake
@@ -161,6 +164,7 @@ class Arch:
     leaky_slope: float = 0.2
     train_steps: int = 1      # Adam steps of the new centre pair per iteration
     mixture: bool = False     # evolve each neighbourhood's generator-mixture weights
+    stale_neighbors: bool = False  # neighbours seen one iteration late (asynchronous cells)
     mix_sigma: float = 0.01   # mixture mutation scale (Table 1)
 
 
@@ -372,11 +376,19 @@ def batches(state: State, pool: Optional[np.ndarray], x_host: Optional[np.ndarra
 # --------------------------------------------------------------------------------------------
 # Step 2: all-pairs evaluation and fitness.
 # --------------------------------------------------------------------------------------------
-def eval_neighborhoods(state: State, data, cells=None) -> Dict[str, np.ndarray]:
+def _slot_state(state: State, prev: Optional[State], s: int) -> State:
+    """The snapshot slot ``s`` of a neighbourhood is read from: the cell's own centre (s = 0)
+    from ``state``; the neighbours from ``prev`` when given (stale neighbours), else ``state``."""
+    return state if (s == 0 or prev is None) else prev
+
+
+def eval_neighborhoods(state: State, data, cells=None, prev: Optional[State] = None
+                       ) -> Dict[str, np.ndarray]:
     """For each cell c and slots (i, j): generator nbr[c][i] against discriminator nbr[c][j] on
     cell c's minibatch. Returns L_G, L_D [cells, 5(i), 5(j)], fitness f_G = mean_j L_G[c, i, :],
     f_D = mean_i L_D[c, :, j], and the logits [cells, 5(j), 6B] (real rows, then the fakes of
-    generator slots 0..4). With ``cells``, only those cells are evaluated (others stay 0)."""
+    generator slots 0..4). With ``cells``, only those cells are evaluated (others stay 0). With
+    ``prev``, the neighbour slots 1..4 hold ``prev``'s individuals (stale neighbours)."""
     a = state.arch
     gl, dl = g_layout(a), d_layout(a)
     nbr = neighbors(state.rows, state.cols)
@@ -387,10 +399,12 @@ def eval_neighborhoods(state: State, data, cells=None) -> Dict[str, np.ndarray]:
     logits = np.zeros((cells, 5, 6 * B))
     for c in (range(cells) if only is None else only):
         x, z = data[c]
-        fakes = [g_forward(unflatten(state.Gw[nbr[c][i]], gl), z, a)["F"] for i in range(5)]
+        fakes = [g_forward(unflatten(_slot_state(state, prev, i).Gw[nbr[c][i]], gl), z, a)["F"]
+                 for i in range(5)]
         X = np.vstack([x] + fakes)
         for j in range(5):
-            lg = d_forward(unflatten(state.Dw[nbr[c][j]], dl), X, a)["logit"]
+            lg = d_forward(unflatten(_slot_state(state, prev, j).Dw[nbr[c][j]], dl), X,
+                           a)["logit"]
             logits[c, j] = lg
             for i in range(5):
                 LG[c, i, j], LD[c, i, j] = pair_losses(lg[:B], lg[B * (i + 1):B * (i + 2)])
@@ -436,7 +450,8 @@ def mixture_step(w: np.ndarray, S: np.ndarray, normals: np.ndarray, sigma: float
     return (cand if acc else w.copy()), bool(acc), old, new
 
 
-def mixture_update(state: State, data, cells=None) -> Dict[str, np.ndarray]:
+def mixture_update(state: State, data, cells=None, prev: Optional[State] = None
+                   ) -> Dict[str, np.ndarray]:
     """Every cell's ES-(1+1) step on its mixture weights, scored on the evaluation's rows: the
     real minibatch and the fakes of the five neighbourhood generators on the cell's noise (as
     the discriminators received them, i.e. rounded to bf16 in bf16 mode). The mutation's five
@@ -450,7 +465,8 @@ def mixture_update(state: State, data, cells=None) -> Dict[str, np.ndarray]:
            "score": np.zeros(n), "score_new": np.zeros(n)}
     for c in (range(n) if cells is None else cells):
         x, z = data[c]
-        fakes = [g_forward(unflatten(state.Gw[nbr[c][i]], gl), z, a)["F"] for i in range(5)]
+        fakes = [g_forward(unflatten(_slot_state(state, prev, i).Gw[nbr[c][i]], gl), z, a)["F"]
+                 for i in range(5)]
         S = mixture_blocks(rb(np.vstack([x] + fakes)), a.batch)
         nrm = draw_normals(state.seed, STREAM_MIX, state.t, c, 5)
         w, acc, old, new = mixture_step(state.mix[c], S, nrm, a.mix_sigma)
@@ -582,13 +598,14 @@ def adam_step(w, m, v, step, g, lr, arch: Arch):
 
 
 def train_step(state: State, sel, data, keep_grads: bool = False,
-               pool: Optional[np.ndarray] = None):
+               pool: Optional[np.ndarray] = None, prev: Optional[State] = None):
     """Every cell's new centre pair (the selected slots' individuals with their optimiser state)
     takes one Adam step on the cell's minibatch, reading only the snapshot ``state``; with
     ``arch.train_steps`` K > 1 it then takes K-1 more steps, step k on the cell's fresh step-k
     minibatch from ``pool``, each at the parameters the previous step left (no selection and no
     lr mutation in between). The kept gradients are the last step's; ``kink`` is the closest
-    approach of any step's pre-activations to 0."""
+    approach of any step's pre-activations to 0. With ``prev`` (stale neighbours), a selected
+    neighbour slot brings ``prev``'s individual."""
     a = state.arch
     nbr = neighbors(state.rows, state.cols)
     new = state.copy()
@@ -597,19 +614,23 @@ def train_step(state: State, sel, data, keep_grads: bool = False,
     for c in range(state.cells):
         sg = int(nbr[c][sel["sel_g"][c]])
         sd = int(nbr[c][sel["sel_d"][c]])
-        lr_g, lr_d = float(state.Glr[sg]), float(state.Dlr[sd])
+        SG = _slot_state(state, prev, int(sel["sel_g"][c]))
+        SD = _slot_state(state, prev, int(sel["sel_d"][c]))
+        lr_g, lr_d = float(SG.Glr[sg]), float(SD.Dlr[sd])
         if a.lr_mutation:
             lr_g = mutate_lr(lr_g, state.seed, STREAM_MUT_G, state.t, c, a)
             lr_d = mutate_lr(lr_d, state.seed, STREAM_MUT_D, state.t, c, a)
         x, z = data[c]
-        gG, gD, info = pair_gradients(state.Gw[sg], state.Dw[sd], x, z, a)
+        gG, gD, info = pair_gradients(SG.Gw[sg], SD.Dw[sd], x, z, a)
         grads["kink"][c] = info["kink"]
         new.Gw[c], new.Gm[c], new.Gv[c], new.Gstep[c] = adam_step(
-            state.Gw[sg], state.Gm[sg], state.Gv[sg], state.Gstep[sg], gG, lr_g, a)
+            SG.Gw[sg], SG.Gm[sg], SG.Gv[sg], SG.Gstep[sg], gG, lr_g, a)
         new.Dw[c], new.Dm[c], new.Dv[c], new.Dstep[c] = adam_step(
-            state.Dw[sd], state.Dm[sd], state.Dv[sd], state.Dstep[sd], gD, lr_d, a)
+            SD.Dw[sd], SD.Dm[sd], SD.Dv[sd], SD.Dstep[sd], gD, lr_d, a)
         new.Glr[c], new.Dlr[c] = lr_g, lr_d
         grads["gG"][c], grads["gD"][c] = gG, gD
+    if a.stale_neighbors and a.train_steps > 1:
+        raise ValueError("stale neighbours are defined for one training step per iteration")
     if a.train_steps > 1 and pool is None:
         raise ValueError("train_steps > 1 draws its later minibatches from the pool")
     for k in range(1, a.train_steps):
@@ -627,18 +648,25 @@ def train_step(state: State, sel, data, keep_grads: bool = False,
 
 
 def iterate(state: State, pool: Optional[np.ndarray], n_iters: int = 1,
-            x_host: Optional[np.ndarray] = None, record: bool = False):
-    """Steps 2, 3 (and 4 with ``arch.mixture``) and 5: ``n_iters`` synchronous grid iterations. Returns the new state (and,
-    with ``record``, the per-iteration evaluations and selections)."""
+            x_host: Optional[np.ndarray] = None, record: bool = False,
+            prev: Optional[State] = None):
+    """Steps 2, 3 (and 4 with ``arch.mixture``) and 5: ``n_iters`` synchronous grid
+    iterations. Returns the new state (and, with ``record``, the per-iteration evaluations and
+    selections). With
+    ``arch.stale_neighbors`` each iteration's neighbours come from the state one iteration
+    older (``prev`` for the first iteration; when None, the first iteration uses ``state``)."""
     log = []
     for _ in range(n_iters):
         data = batches(state, pool, x_host)
-        ev = eval_neighborhoods(state, data)
-        mx = mixture_update(state, data) if state.arch.mixture else None
+        ev = eval_neighborhoods(state, data, prev=prev)
+        mx = mixture_update(state, data, prev=prev) if state.arch.mixture else None
         sel = select_replace(state, ev)
-        state = train_step(state, sel, data, pool=pool)
+        new = train_step(state, sel, data, pool=pool, prev=prev)
         if mx is not None:
-            state.mix = mx["mix"]
+            new.mix = mx["mix"]
+        if state.arch.stale_neighbors:
+            prev = state
+        state = new
         if record:
             log.append({"eval": ev, "sel": sel, "mix": mx})
     return (state, log) if record else state
