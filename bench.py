@@ -9,11 +9,12 @@ one full grid iteration (minibatch draw, all-pairs evaluation, fitness, selectio
 Adam of every cell's new centre pair).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--train-steps S] [--mixture]
+                  [--train-steps S] [--mixture] [--stale-neighbors]
 
 With --train-steps S > 1 every iteration trains each cell's new centre pair S times (the later
 steps on fresh minibatches); the default S = 1 is the headline workload. --mixture adds the
-generator-mixture ES-(1+1) step (Gaussian-kernel MMD score) to every evaluation.
+generator-mixture ES-(1+1) step (Gaussian-kernel MMD score) to every evaluation;
+--stale-neighbors runs the asynchronous schedule (neighbours one iteration late).
 
 With N > 1 (torchrun, one process per GPU) every rank runs its own 12x12 grid (replicas: the
 per-GPU work is fixed, scaling "weak"); value = all ranks' pairs / the slowest rank's time.
@@ -168,7 +169,8 @@ def run_ours(args):
 
     pool = lipz_synth.blob_pool(SEED, n=POOL_N, dim=X_DIM)
     g = L.Grid(ROWS, COLS, seed=SEED + rank, precision="bf16", batch=BATCH,
-               train_steps=args.train_steps, mixture=1 if args.mixture else 0)
+               train_steps=args.train_steps, mixture=1 if args.mixture else 0,
+               stale_neighbors=1 if args.stale_neighbors else 0)
     g.set_data(pool)
     stream = torch.cuda.Stream()
     g.set_stream(stream.cuda_stream)
@@ -243,7 +245,8 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
-    if world == 1 and not args.no_cpu_baseline and args.train_steps == 1 and not args.mixture:
+    if (world == 1 and not args.no_cpu_baseline and args.train_steps == 1 and not args.mixture
+            and not args.stale_neighbors):
         line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
     return line
 
@@ -305,7 +308,7 @@ def _roofline(phase_ms):
     return r
 
 
-def _oracle_sample(seconds, max_cells=None, train_steps=1, mixture=False):
+def _oracle_sample(seconds, max_cells=None, train_steps=1, mixture=False, stale=False):
     """Run the oracle's full iteration cell by cell on the 12x12 workload until ``seconds`` of
     CPU work are spent; return (cells done, elapsed seconds). With ``train_steps`` K > 1 each
     cell's pair then takes K - 1 more steps on fresh minibatches; with ``mixture`` each cell also
@@ -324,9 +327,10 @@ def _oracle_sample(seconds, max_cells=None, train_steps=1, mixture=False):
     while True:
         cells = [c]
         data = O.batches(state, pool, cells=cells)
-        ev = O.eval_neighborhoods(state, data, cells=cells)
+        prev = state if stale else None  # the same work; the sample's weights are synthetic
+        ev = O.eval_neighborhoods(state, data, cells=cells, prev=prev)
         if mixture:
-            O.mixture_update(state, data, cells=cells)
+            O.mixture_update(state, data, cells=cells, prev=prev)
         a = state.arch
         sg = O.select_slot(ev["fG"][c], O.draw_words(state.seed, O.STREAM_TOUR_G, state.t, c,
                                                      a.tournament_size), a)
@@ -382,6 +386,8 @@ def _workload(args):
         w += ", %d minibatch steps per iteration" % args.train_steps
     if args.mixture:
         w += ", mixture ES step"
+    if args.stale_neighbors:
+        w += ", stale neighbours"
     return w
 
 
@@ -394,12 +400,13 @@ def run_reference(args):
     _oracle_state(arch)
     per_step_cells = 1
     for _ in range(args.warmup):
-        _oracle_sample(1e9, max_cells=1, train_steps=args.train_steps, mixture=args.mixture)
+        _oracle_sample(1e9, max_cells=1, train_steps=args.train_steps, mixture=args.mixture,
+                       stale=args.stale_neighbors)
     times = []
     total_cells = 0
     for _ in range(args.steps):
         done, el = _oracle_sample(1e9, max_cells=per_step_cells, train_steps=args.train_steps,
-                                  mixture=args.mixture)
+                                  mixture=args.mixture, stale=args.stale_neighbors)
         times.append(el)
         total_cells += done
     el = sum(times)
@@ -433,6 +440,8 @@ def main():
                     help="Adam steps per grid iteration (the later ones on fresh minibatches)")
     ap.add_argument("--mixture", action="store_true",
                     help="add the generator-mixture ES step to every iteration")
+    ap.add_argument("--stale-neighbors", action="store_true",
+                    help="neighbours seen one iteration late (asynchronous cells)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -114,6 +114,12 @@ typedef struct lipz_arch {
                               generator-mixture weights (Section 3 step 4); see
                               lipz_get_mixture. Default 0. */
   float mix_sigma;         /* 0.01: mixture mutation scale (Table 1) */
+  int32_t stale_neighbors; /* 1: the asynchronous cells of Section 3, emulated deterministically:
+                              an evaluation sees each cell's own centre as of the iteration and
+                              its four neighbours as they were one iteration earlier (the first
+                              iteration after create or lipz_import_state sees them as they
+                              are); a selected neighbour brings that older individual with its
+                              optimiser state. Needs train_steps == 1. Default 0. */
 } lipz_arch;
 
 typedef struct lipz_grid lipz_grid;

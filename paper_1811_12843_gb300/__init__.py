@@ -52,7 +52,7 @@ class lipz_arch(ctypes.Structure):
         ("lr_mut_prob", ctypes.c_float), ("leaky_slope", ctypes.c_float),
         ("keep_grads", ctypes.c_int32), ("force_simt", ctypes.c_int32),
         ("train_steps", ctypes.c_int32), ("mixture", ctypes.c_int32),
-        ("mix_sigma", ctypes.c_float),
+        ("mix_sigma", ctypes.c_float), ("stale_neighbors", ctypes.c_int32),
     ]
 
 

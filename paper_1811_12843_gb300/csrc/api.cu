@@ -57,7 +57,10 @@ struct lipz_grid {
   cudaEvent_t ev_x = nullptr;      // the upload of the caller's minibatch has landed
   int* hstat = nullptr;            // pinned host copies of the device error flags
   int device = 0;
-  PopView G[2]{}, D[2]{};
+  // population snapshots: ping-pong pair, or three in rotation with stale neighbours (the
+  // snapshot being written must not be the one the stale neighbours are read from)
+  PopView G[3]{}, D[3]{};
+  int nsnap = 2;
   int cur = 0;
   int phase = PH_IDLE;
   bool use_tc = false;
@@ -70,7 +73,12 @@ struct lipz_grid {
   float* xin = nullptr;  // caller-supplied minibatch staging [cells][B][x_dim]
   void *Z = nullptr, *E = nullptr, *H1g = nullptr, *H2g = nullptr, *H1d = nullptr, *H2d = nullptr;
   float *logits = nullptr, *LG = nullptr, *LD = nullptr, *fG = nullptr, *fD = nullptr;
-  int *nbr = nullptr, *sel_g = nullptr, *sel_d = nullptr, *src_g = nullptr, *src_d = nullptr;
+  // neighbour tables [cells][5] of individual indices (snapshot * cells + cell) per snapshot
+  // parity: every slot from the current snapshot, or (stale neighbours) slots 1..4 from the
+  // other snapshot, which holds the previous iteration's centres
+  int *nbr_cur[3]{}, *nbr_stale[3]{};
+  bool prev_valid = false;  // the other snapshot holds the previous iteration's centres
+  int *sel_g = nullptr, *sel_d = nullptr, *src_g = nullptr, *src_d = nullptr;
   float *lrn_g = nullptr, *lrn_d = nullptr;
   float4 *coef_g = nullptr, *coef_d = nullptr;  // per cell: lr, 1/bc1, 1/bc2, step + 1
   void *TH1 = nullptr, *TH2 = nullptr, *TX = nullptr, *TG1 = nullptr, *TG2 = nullptr;
@@ -87,9 +95,9 @@ struct lipz_grid {
   GemmDesc* dgram = nullptr;
   int mix_nh = 1;
   bool mix_tc = false;
-  Descs dsc[2]{};
-  TcPlan* tc[2]{};
-  TcbPlan* tcb[2]{};
+  Descs dsc[3]{}, dsc_stale[3]{};
+  TcPlan* tc[3]{};
+  TcbPlan* tcb[3]{};
   bool use_tcb = false;
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
@@ -252,14 +260,19 @@ int upload(lipz_grid* g, T** dst, const std::vector<T>& v) {
   return h2d(g, *dst, v.data(), v.size() * sizeof(T));
 }
 
+// Snapshot written by an iteration that reads snapshot p, and the one it read before p.
+int snap_next(const lipz_grid* g, int p) { return (p + 1) % g->nsnap; }
+int snap_prev(const lipz_grid* g, int p) { return (p + g->nsnap - 1) % g->nsnap; }
+
 int build_descs(lipz_grid* g, int p) {
   const int C = g->cells, B = g->a.batch, z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
   const size_t es = g->esz;
-  const PopView &Gp = g->G[p], &Dp = g->D[p];
+  // both snapshots are one allocation: individual k of the index space is snapshot k / C
+  const PopView &Gp = g->G[0], &Dp = g->D[0];
   const void* Gw = act_w(Gp);
   const void* Dw = act_w(Dp);
   const Layout &L = g->lg, &M = g->ld;
-  std::vector<int> nbr(C * 5);
+  std::vector<int> nbr(C * 5), cur(C * 5), stale(C * 5);
   for (int r = 0; r < g->rows; ++r)
     for (int q = 0; q < g->cols; ++q) {
       int* n = &nbr[(r * g->cols + q) * 5];
@@ -269,54 +282,67 @@ int build_descs(lipz_grid* g, int p) {
       n[3] = r * g->cols + (q - 1 + g->cols) % g->cols;
       n[4] = r * g->cols + (q + 1) % g->cols;
     }
-  std::vector<GemmDesc> g1, g2, g3, d1, d2;
-  std::vector<GemvDesc> d3;
-  for (int c = 0; c < C; ++c)
-    for (int s = 0; s < 5; ++s) {
-      const int k = nbr[c * 5 + s];
-      const int64_t pg = (int64_t)k * g->PGs, pd = (int64_t)k * g->PDs;
-      const int64_t cs = (int64_t)c * 5 + s;
-      GemmDesc a = gd(eoff(g->Z, (int64_t)c * B * z, es), z, 1, eoff(Gw, pg + L.off[0], es), 1, z,
-                      eoff(g->H1g, cs * B * h, es), h, 1, B, h, z);
-      a.bias = Gp.w + pg + L.off[1];
-      g1.push_back(a);
-      GemmDesc b = gd(eoff(g->H1g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[2], es), 1, h,
-                      eoff(g->H2g, cs * B * h, es), h, 1, B, h, h);
-      b.bias = Gp.w + pg + L.off[3];
-      g2.push_back(b);
-      GemmDesc e = gd(eoff(g->H2g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[4], es), 1, h,
-                      eoff(g->E, (int64_t)c * g->e_cell + (int64_t)(1 + s) * B * x, es), x, 1, B,
-                      x, h);
-      e.bias = Gp.w + pg + L.off[5];
-      g3.push_back(e);
-      GemmDesc f = gd(eoff(g->E, (int64_t)c * g->e_cell, es), x, 1, eoff(Dw, pd + M.off[0], es), 1,
-                      x, eoff(g->H1d, cs * 6 * B * h, es), h, 1, 6 * B, h, x);
-      f.bias = Dp.w + pd + M.off[1];
-      d1.push_back(f);
-      GemmDesc q2 = gd(eoff(g->H1d, cs * 6 * B * h, es), h, 1, eoff(Dw, pd + M.off[2], es), 1, h,
-                       eoff(g->H2d, cs * 6 * B * h, es), h, 1, 6 * B, h, h);
-      q2.bias = Dp.w + pd + M.off[3];
-      d2.push_back(q2);
-      GemvDesc v;
-      memset(&v, 0, sizeof v);
-      v.X = eoff(g->H2d, cs * 6 * B * h, es);
-      v.w = eoff(Dw, pd + M.off[4], es);
-      v.bias = Dp.w + pd + M.off[5];
-      v.out = g->logits + cs * 6 * B;
-      v.ld = h;
-      v.rows = 6 * B;
-      v.K = h;
-      d3.push_back(v);
-    }
-  if (p == 0) {
-    int rc = upload(g, &g->nbr, nbr);
-    if (rc) return rc;
+  for (int i = 0; i < C * 5; ++i) {
+    cur[i] = p * C + nbr[i];
+    stale[i] = (i % 5 == 0 ? p : snap_prev(g, p)) * C + nbr[i];
+  }
+  // evaluation descriptors of one neighbour table
+  auto eval_descs = [&](const std::vector<int>& tab, Descs& D) -> int {
+    std::vector<GemmDesc> g1, g2, g3, d1, d2;
+    std::vector<GemvDesc> d3;
+    for (int c = 0; c < C; ++c)
+      for (int s = 0; s < 5; ++s) {
+        const int k = tab[c * 5 + s];
+        const int64_t pg = (int64_t)k * g->PGs, pd = (int64_t)k * g->PDs;
+        const int64_t cs = (int64_t)c * 5 + s;
+        GemmDesc a = gd(eoff(g->Z, (int64_t)c * B * z, es), z, 1, eoff(Gw, pg + L.off[0], es), 1, z,
+                        eoff(g->H1g, cs * B * h, es), h, 1, B, h, z);
+        a.bias = Gp.w + pg + L.off[1];
+        g1.push_back(a);
+        GemmDesc b = gd(eoff(g->H1g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[2], es), 1, h,
+                        eoff(g->H2g, cs * B * h, es), h, 1, B, h, h);
+        b.bias = Gp.w + pg + L.off[3];
+        g2.push_back(b);
+        GemmDesc e = gd(eoff(g->H2g, cs * B * h, es), h, 1, eoff(Gw, pg + L.off[4], es), 1, h,
+                        eoff(g->E, (int64_t)c * g->e_cell + (int64_t)(1 + s) * B * x, es), x, 1, B,
+                        x, h);
+        e.bias = Gp.w + pg + L.off[5];
+        g3.push_back(e);
+        GemmDesc f = gd(eoff(g->E, (int64_t)c * g->e_cell, es), x, 1, eoff(Dw, pd + M.off[0], es), 1,
+                        x, eoff(g->H1d, cs * 6 * B * h, es), h, 1, 6 * B, h, x);
+        f.bias = Dp.w + pd + M.off[1];
+        d1.push_back(f);
+        GemmDesc q2 = gd(eoff(g->H1d, cs * 6 * B * h, es), h, 1, eoff(Dw, pd + M.off[2], es), 1, h,
+                         eoff(g->H2d, cs * 6 * B * h, es), h, 1, 6 * B, h, h);
+        q2.bias = Dp.w + pd + M.off[3];
+        d2.push_back(q2);
+        GemvDesc v;
+        memset(&v, 0, sizeof v);
+        v.X = eoff(g->H2d, cs * 6 * B * h, es);
+        v.w = eoff(Dw, pd + M.off[4], es);
+        v.bias = Dp.w + pd + M.off[5];
+        v.out = g->logits + cs * 6 * B;
+        v.ld = h;
+        v.rows = 6 * B;
+        v.K = h;
+        d3.push_back(v);
+      }
+    int rc;
+    if ((rc = upload(g, &D.g1, g1)) || (rc = upload(g, &D.g2, g2)) ||
+        (rc = upload(g, &D.g3, g3)) || (rc = upload(g, &D.d1, d1)) ||
+        (rc = upload(g, &D.d2, d2)) || (rc = upload(g, &D.d3, d3)))
+      return rc;
+    return LIPZ_OK;
+  };
+  {
+    int rc;
+    if ((rc = upload(g, &g->nbr_cur[p], cur)) || (rc = upload(g, &g->nbr_stale[p], stale)) ||
+        (rc = eval_descs(cur, g->dsc[p])) ||
+        (g->a.stale_neighbors && (rc = eval_descs(stale, g->dsc_stale[p]))))
+      return rc;
   }
   Descs& D = g->dsc[p];
   int rc;
-  if ((rc = upload(g, &D.g1, g1)) || (rc = upload(g, &D.g2, g2)) || (rc = upload(g, &D.g3, g3)) ||
-      (rc = upload(g, &D.d1, d1)) || (rc = upload(g, &D.d2, d2)) || (rc = upload(g, &D.d3, d3)))
-    return rc;
 
   // ---- training descriptors: weights of the selected individual (wsel = src_g / src_d)
   std::vector<GemmDesc> tg1, tg2, td1, td2, bw2d, bd1, bw1d, ba3, bw3g, ba2, bw2g, ba1, bw1g;
@@ -485,24 +511,40 @@ int check_arch(const lipz_arch* a) {
     return fail(nullptr, LIPZ_ERR_INVALID, "bad optimiser / mutation hyper-parameters");
   if (a->train_steps < 1 || a->train_steps > 65536)
     return fail(nullptr, LIPZ_ERR_INVALID, "train_steps must be in 1..65536");
+  if (a->stale_neighbors != 0 && a->stale_neighbors != 1)
+    return fail(nullptr, LIPZ_ERR_INVALID, "stale_neighbors must be 0 or 1");
+  if (a->stale_neighbors && a->train_steps != 1)
+    return fail(nullptr, LIPZ_ERR_INVALID, "stale_neighbors needs train_steps == 1");
   if ((a->mixture != 0 && a->mixture != 1) || !(a->mix_sigma >= 0.f))
     return fail(nullptr, LIPZ_ERR_INVALID, "mixture must be 0 or 1 and mix_sigma >= 0");
   return LIPZ_OK;
 }
 
-int alloc_pop(lipz_grid* g, PopView* p, int64_t Ps) {
-  const size_t n = (size_t)g->cells * Ps;
+// All snapshots of one population in one allocation per array (snapshot s at s * cells
+// individuals), so that an individual index k = snapshot * cells + cell addresses any of them.
+int alloc_pops(lipz_grid* g, PopView* p, int64_t Ps) {
+  const size_t C = g->cells, S = g->nsnap, n = S * C * Ps;
+  PopView& a = p[0];
   int rc;
-  if ((rc = dalloc(g, &p->w, n * 4)) || (rc = dalloc(g, &p->m, n * 4)) ||
-      (rc = dalloc(g, &p->v, n * 4)) || (rc = dalloc(g, &p->step, g->cells * 4)) ||
-      (rc = dalloc(g, &p->lr, g->cells * 4)))
+  if ((rc = dalloc(g, &a.w, n * 4)) || (rc = dalloc(g, &a.m, n * 4)) ||
+      (rc = dalloc(g, &a.v, n * 4)) || (rc = dalloc(g, &a.step, S * C * 4)) ||
+      (rc = dalloc(g, &a.lr, S * C * 4)))
     return rc;
-  p->wb = nullptr;
-  if (g->bf && (rc = dalloc(g, &p->wb, n * 2))) return rc;
-  if ((rc = dset(g, p->w, 0, n * 4)) || (rc = dset(g, p->m, 0, n * 4)) ||
-      (rc = dset(g, p->v, 0, n * 4)) || (rc = dset(g, p->step, 0, g->cells * 4)) ||
-      (p->wb && (rc = dset(g, p->wb, 0, n * 2))))
+  a.wb = nullptr;
+  if (g->bf && (rc = dalloc(g, &a.wb, n * 2))) return rc;
+  if ((rc = dset(g, a.w, 0, n * 4)) || (rc = dset(g, a.m, 0, n * 4)) ||
+      (rc = dset(g, a.v, 0, n * 4)) || (rc = dset(g, a.step, 0, S * C * 4)) ||
+      (a.wb && (rc = dset(g, a.wb, 0, n * 2))))
     return rc;
+  for (size_t s = 1; s < S; ++s) {
+    PopView& b = p[s];
+    b.w = a.w + s * C * Ps;
+    b.m = a.m + s * C * Ps;
+    b.v = a.v + s * C * Ps;
+    b.wb = a.wb ? a.wb + s * C * Ps : nullptr;
+    b.step = a.step + s * C;
+    b.lr = a.lr + s * C;
+  }
   return LIPZ_OK;
 }
 
@@ -519,9 +561,8 @@ int create_impl(lipz_grid* g) {
   CK(g, cudaMallocHost(&g->hstat, 8 * sizeof(int)));
   make_layouts(g);
   g->e_cell = (int64_t)6 * B * x;
-  for (int p = 0; p < 2; ++p) {
-    if ((rc = alloc_pop(g, &g->G[p], g->PGs)) || (rc = alloc_pop(g, &g->D[p], g->PDs))) return rc;
-  }
+  g->nsnap = g->a.stale_neighbors ? 3 : 2;
+  if ((rc = alloc_pops(g, g->G, g->PGs)) || (rc = alloc_pops(g, g->D, g->PDs))) return rc;
   const size_t CB = (size_t)C * B;
   if ((rc = dalloc(g, &g->Z, CB * z * es)) || (rc = dalloc(g, &g->E, (size_t)C * g->e_cell * es)) ||
       (rc = dalloc(g, &g->H1g, CB * 5 * h * es)) || (rc = dalloc(g, &g->H2g, CB * 5 * h * es)) ||
@@ -576,25 +617,27 @@ int create_impl(lipz_grid* g) {
                      g->st);
   CKL(g);
   std::vector<float> lr(C, g->a.lr);
-  for (float* d : {g->G[0].lr, g->D[0].lr, g->G[1].lr, g->D[1].lr})
-    if ((rc = h2d(g, d, lr.data(), C * 4))) return rc;
-  if ((rc = build_descs(g, 0)) || (rc = build_descs(g, 1))) return rc;
+  for (int p = 0; p < g->nsnap; ++p)
+    if ((rc = h2d(g, g->G[p].lr, lr.data(), C * 4)) || (rc = h2d(g, g->D[p].lr, lr.data(), C * 4)) ||
+        (rc = build_descs(g, p)))
+      return rc;
   g->use_tc = g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
   if (g->use_tc) {
-    for (int p = 0; p < 2; ++p) {
-      TcShape s{C, B, z, h, x, g->a.leaky_slope};
+    for (int p = 0; p < g->nsnap; ++p) {
+      TcShape s{C, B, z, h, x, g->a.leaky_slope, g->nsnap * C};
       TcBuffers b{};
       b.Z = g->Z;
       b.E = g->E;
       b.e_cell = g->e_cell;
       b.logits = g->logits;
-      b.nbr = g->nbr;
-      b.Gwb = g->G[p].wb;
-      b.Gw = g->G[p].w;
+      b.nbr = g->nbr_cur[p];
+      b.indiv_off = p * C;
+      b.Gwb = g->G[0].wb;
+      b.Gw = g->G[0].w;
       b.PGs = g->PGs;
       b.goff = g->lg.off;
-      b.Dwb = g->D[p].wb;
-      b.Dw = g->D[p].w;
+      b.Dwb = g->D[0].wb;
+      b.Dw = g->D[0].w;
       b.PDs = g->PDs;
       b.doff = g->ld.off;
       b.sel_g = g->sel_g;
@@ -612,8 +655,8 @@ int create_impl(lipz_grid* g) {
       if (!g->tc[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core plan: %s", msg.c_str());
     }
     g->use_tcb = tcb_supported(z, h, x, B);
-    for (int p = 0; p < 2 && g->use_tcb; ++p) {
-      TcbShape s{C, B, z, h, x, g->a.leaky_slope, C};
+    for (int p = 0; p < g->nsnap && g->use_tcb; ++p) {
+      TcbShape s{C, B, z, h, x, g->a.leaky_slope, g->nsnap * C};
       TcbBuffers b{};
       b.Z = g->Z;
       b.E = g->E;
@@ -629,8 +672,8 @@ int create_impl(lipz_grid* g) {
       b.A1 = g->A1;
       b.gG = g->gG;
       b.gD = g->gD;
-      b.Gwb = g->G[p].wb;
-      b.Dwb = g->D[p].wb;
+      b.Gwb = g->G[0].wb;
+      b.Dwb = g->D[0].wb;
       b.PGs = g->PGs;
       b.PDs = g->PDs;
       b.goff = g->lg.off;
@@ -639,7 +682,10 @@ int create_impl(lipz_grid* g) {
       b.src_d = g->src_d;
       // without keep_grads the weight matrices take their Adam step inside the backward
       b.fuse_adam = g->a.keep_grads ? 0 : 1;
-      const PopView* pops[2][2] = {{&g->G[p], &g->G[1 - p]}, {&g->D[p], &g->D[1 - p]}};
+      // old state: any individual of any snapshot (the selection's source); new: the next
+      // snapshot
+      const int q1 = snap_next(g, p);
+      const PopView* pops[2][2] = {{&g->G[0], &g->G[q1]}, {&g->D[0], &g->D[q1]}};
       TcbBuffers::AdamPop* ap[2] = {&b.adam_g, &b.adam_d};
       for (int q = 0; q < 2; ++q) {
         ap[q]->w = pops[q][0]->w;
@@ -667,6 +713,12 @@ int create_impl(lipz_grid* g) {
 
 SelectParams select_params(const lipz_grid* g);
 SelectIO select_io(lipz_grid* g);
+
+// Neighbour table of the current evaluation: stale neighbours (the other snapshot's
+// individuals in slots 1..4) once the other snapshot holds the previous iteration's centres.
+const int* eval_nbr(const lipz_grid* g) {
+  return g->a.stale_neighbors && g->prev_valid ? g->nbr_stale[g->cur] : g->nbr_cur[g->cur];
+}
 
 // Minibatch step `step` of the current iteration into E's real rows and Z (the real rows from
 // xin_dev when given, else from the pool).
@@ -725,6 +777,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
   phase_end(g, LIPZ_PHASE_BATCH, 1);
   if (g->use_tc) {
     std::string msg;
+    tc_set_nbr(g->tc[p], eval_nbr(g));
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);
@@ -737,7 +790,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
     if (tc_run_d(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_D_FWD, 1);
   } else {
-    const Descs& D = g->dsc[p];
+    const Descs& D = g->a.stale_neighbors && g->prev_valid ? g->dsc_stale[p] : g->dsc[p];
     phase_begin(g, LIPZ_PHASE_G_FWD);
     gemm(g, D.g1, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
     gemm(g, D.g2, C * 5, B, h, EPI_BIAS_ACT, ACT_RELU, false);
@@ -757,7 +810,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
   CKL(g);
   phase_begin(g, LIPZ_PHASE_FITNESS);
   if (then_select)
-    launch_fitness_select(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->nbr,
+    launch_fitness_select(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, eval_nbr(g),
                           select_params(g), select_io(g), g->st);
   else
     launch_fitness(g->logits, C, B, g->LG, g->LD, g->fG, g->fD, g->flag, g->st);
@@ -790,10 +843,10 @@ SelectParams select_params(const lipz_grid* g) {
 SelectIO select_io(lipz_grid* g) {
   const int p = g->cur;
   SelectIO io;
-  io.lr_old[0] = g->G[p].lr;
-  io.lr_old[1] = g->D[p].lr;
-  io.step_old[0] = g->G[p].step;
-  io.step_old[1] = g->D[p].step;
+  io.lr_old[0] = g->G[0].lr;
+  io.lr_old[1] = g->D[0].lr;
+  io.step_old[0] = g->G[0].step;
+  io.step_old[1] = g->D[0].step;
   io.sel[0] = g->sel_g;
   io.sel[1] = g->sel_d;
   io.src[0] = g->src_g;
@@ -809,7 +862,7 @@ int select_impl(lipz_grid* g) {
   if (g->phase != PH_EVALUATED)
     return fail(g, LIPZ_ERR_STATE, "lipz_select_replace must follow lipz_eval_neighborhoods");
   phase_begin(g, LIPZ_PHASE_SELECT);
-  launch_select(g->fG, g->fD, g->nbr, g->cells, select_params(g), select_io(g), g->st);
+  launch_select(g->fG, g->fD, eval_nbr(g), g->cells, select_params(g), select_io(g), g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_SELECT, 1);
   g->phase = PH_SELECTED;
@@ -851,11 +904,11 @@ int train_once(lipz_grid* g) {
   }
   // logit deltas (and D's output-layer gradient)
   if (g->bf)
-    launch_dlogit<bf16>(g->TL, (const bf16*)g->TG2, g->D[p].wb, g->PDs, g->ld.off[4], g->src_d, C,
+    launch_dlogit<bf16>(g->TL, (const bf16*)g->TG2, g->D[0].wb, g->PDs, g->ld.off[4], g->src_d, C,
                         B, h, g->a.leaky_slope, (bf16*)g->J2, g->gD, g->PDs, g->ld.off[4],
                         g->ld.off[5], g->ld.off[3], g->st);
   else
-    launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[p].w, g->PDs, g->ld.off[4], g->src_d,
+    launch_dlogit<float>(g->TL, (const float*)g->TG2, g->D[0].w, g->PDs, g->ld.off[4], g->src_d,
                          C, B, h, g->a.leaky_slope, (float*)g->J2, g->gD, g->PDs, g->ld.off[4],
                          g->ld.off[5], g->ld.off[3], g->st);
   CKL(g);
@@ -873,14 +926,14 @@ int train_once(lipz_grid* g) {
       // the weight matrices took their Adam step inside the backward: the biases and D's
       // output layer remain
       AdamRanges rg{}, rd{};
-      rg.old_p = g->G[p];
-      rg.new_p = g->G[1 - p];
+      rg.old_p = g->G[0];
+      rg.new_p = g->G[snap_next(g, p)];
       rg.grad = g->gG;
       rg.src = g->src_g;
       rg.coef = g->coef_g;
       rg.Ps = g->PGs;
-      rd.old_p = g->D[p];
-      rd.new_p = g->D[1 - p];
+      rd.old_p = g->D[0];
+      rd.new_p = g->D[snap_next(g, p)];
       rd.grad = g->gD;
       rd.src = g->src_d;
       rd.coef = g->coef_d;
@@ -896,7 +949,7 @@ int train_once(lipz_grid* g) {
       launch_adam_ranges(rg, rd, C, g->a.beta1, g->a.beta2, g->a.eps, g->st);
       CKL(g);
       phase_end(g, LIPZ_PHASE_ADAM, 1);
-      g->cur = 1 - p;
+      g->cur = snap_next(g, p);
       return LIPZ_OK;
     }
   } else {
@@ -919,13 +972,13 @@ int train_once(lipz_grid* g) {
     phase_begin(g, LIPZ_PHASE_ADAM);
   }
   // Adam + replacement into the other snapshot (after the bias sums on the tensor-core path)
-  launch_adam(g->G[p], g->G[1 - p], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
+  launch_adam(g->G[0], g->G[snap_next(g, p)], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
-  launch_adam(g->D[p], g->D[1 - p], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
+  launch_adam(g->D[0], g->D[snap_next(g, p)], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs, g->a.beta1,
               g->a.beta2, g->a.eps, g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_ADAM, 2);
-  g->cur = 1 - p;
+  g->cur = snap_next(g, p);
   return LIPZ_OK;
 }
 
@@ -938,7 +991,7 @@ int train_again(lipz_grid* g, uint32_t k) {
   CKL(g);
   phase_end(g, LIPZ_PHASE_BATCH, 1);
   phase_begin(g, LIPZ_PHASE_SELECT);
-  launch_centre_select(C, select_params(g), select_io(g), g->st);
+  launch_centre_select(C, g->cur * C, select_params(g), select_io(g), g->st);
   CKL(g);
   phase_end(g, LIPZ_PHASE_SELECT, 1);
   phase_begin(g, LIPZ_PHASE_G_FWD);
@@ -971,6 +1024,7 @@ int train_impl(lipz_grid* g) {
   if (rc) return rc;
   g->t += 1;
   g->phase = PH_IDLE;
+  g->prev_valid = true;
   return LIPZ_OK;
 }
 
@@ -978,16 +1032,18 @@ int train_impl(lipz_grid* g) {
 // or a non-finite loss seen since the last check (one synchronisation: all flags are copied
 // into pinned host memory first); the flags are reset.
 int check_flag(lipz_grid* g) {
-  int* dev[5] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
+  int* dev[7] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
                  g->tc[1] ? tc_error_flag(g->tc[1]) : nullptr,
+                 g->tc[2] ? tc_error_flag(g->tc[2]) : nullptr,
                  g->tcb[0] ? tcb_error_flag(g->tcb[0]) : nullptr,
-                 g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr, g->flag};
-  for (int i = 0; i < 5; ++i) {
-    g->hstat[i] = i < 4 ? 0 : INT_MAX;
+                 g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr,
+                 g->tcb[2] ? tcb_error_flag(g->tcb[2]) : nullptr, g->flag};
+  for (int i = 0; i < 7; ++i) {
+    g->hstat[i] = i < 6 ? 0 : INT_MAX;
     if (dev[i]) CK(g, cudaMemcpyAsync(&g->hstat[i], dev[i], 4, cudaMemcpyDeviceToHost, g->st));
   }
   CK(g, cudaStreamSynchronize(g->st));
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < 6; ++i) {
     const int code = g->hstat[i];
     if (code) {
       CK(g, cudaMemsetAsync(dev[i], 0, 4, g->st));
@@ -995,7 +1051,7 @@ int check_flag(lipz_grid* g) {
       return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
-  const int v = g->hstat[4];
+  const int v = g->hstat[6];
   if (v != INT_MAX) {
     const int big = INT_MAX;
     int rc = h2d(g, g->flag, &big, 4);
@@ -1059,6 +1115,7 @@ int lipz_arch_default(lipz_arch* a) {
   a->train_steps = 1;
   a->mixture = 0;
   a->mix_sigma = 0.01f;
+  a->stale_neighbors = 0;
   return LIPZ_OK;
 }
 
@@ -1092,7 +1149,7 @@ int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_t seed, l
 int lipz_grid_destroy(lipz_grid* g) {
   if (!g) return LIPZ_OK;
   cudaStreamSynchronize(g->st);
-  for (int p = 0; p < 2; ++p) {
+  for (int p = 0; p < 3; ++p) {
     if (g->tc[p]) tc_plan_destroy(g->tc[p]);
     if (g->tcb[p]) tcb_plan_destroy(g->tcb[p]);
   }
@@ -1314,6 +1371,7 @@ int lipz_import_state(lipz_grid* g, const void* host, size_t bytes) {
   CK(g, cudaMemcpyAsync(g->D[p].lr, s, C * 4, cudaMemcpyHostToDevice, g->st));
   s += C * 4;
   CK(g, cudaMemcpyAsync(g->mix, s, C * 20, cudaMemcpyHostToDevice, g->st));
+  g->prev_valid = false;  // the other snapshot no longer holds this state's predecessor
   if (g->bf) {
     launch_to_bf16(g->G[p].w, g->G[p].wb, (int64_t)C * g->PGs, g->st);
     launch_to_bf16(g->D[p].w, g->D[p].wb, (int64_t)C * g->PDs, g->st);

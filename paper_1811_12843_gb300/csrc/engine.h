@@ -88,7 +88,8 @@ void launch_mix_partials(const float* gram, const float* rnorm, int cells, int r
 void launch_mix_es(const float* part, int nh, int cells, int rows, int B, float* mix, float* S,
                    float* score, uint64_t seed, uint32_t t, float sigma, cudaStream_t st);
 // Choice of every cell's own centre (slot 0), for the later minibatch steps of an iteration.
-void launch_centre_select(int cells, const SelectParams& p, const SelectIO& io, cudaStream_t st);
+void launch_centre_select(int cells, int off, const SelectParams& p, const SelectIO& io,
+                          cudaStream_t st);
 // Fitness and, in the same kernel, the selection of every cell (when nothing is read back
 // between the two).
 void launch_fitness_select(const float* logits, int cells, int B, float* LG, float* LD,

@@ -81,6 +81,7 @@ struct KParams {
   // centre-only generator forward (non-zero): problem c is cell c's own generator on z_c,
   // written to E[c] as the fakes of slot 0
   int centre;
+  int indiv_off;  // centre-only mode: individual index of cell 0's centre (snapshot * cells)
   // Gram kind (mixture score): problem c is the Gram matrix of E[c]'s rows with themselves,
   // reduced in the epilogue to per-row sums of exp(-||e_r - e_s||^2 / x) over the columns s of
   // each block of B rows. rnorm [cells][rows] holds ||e_r||^2; the sums go to
@@ -132,7 +133,8 @@ __device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
 }
 __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
-  return (p.centre || p.kind == KIND_GRAM) ? prob : __ldg(&p.nbr[prob]);
+  if (p.kind == KIND_GRAM) return prob;
+  return p.centre ? p.indiv_off + prob : __ldg(&p.nbr[prob]);
 }
 
 // Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
@@ -689,16 +691,16 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   TcPlan* p = new TcPlan();
   memset(p, 0, sizeof *p);
   p->s = s;
-  const uint64_t C = s.cells, B = s.B, z = s.z, x = s.x, h = s.h;
+  const uint64_t C = s.cells, B = s.B, z = s.z, x = s.x, h = s.h, NI = s.n_indiv;
   bool ok = make_map(&p->mZ, b.Z, z, B, C, z * 2, B * z * 2, 128, msg) &&
             make_map(&p->mE, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 128, msg) &&
             make_map(&p->mEB, b.E, x, 6 * B, C, x * 2, (uint64_t)b.e_cell * 2, 256, msg) &&
             make_map4(&p->mE4, b.E, x, B, 6, C, x * 2, B * x * 2, (uint64_t)b.e_cell * 2, msg) &&
-            make_map(&p->mG1, b.Gwb + b.goff[0], z, h, C, z * 2, b.PGs * 2, 256, msg) &&
-            make_map(&p->mG2, b.Gwb + b.goff[2], h, h, C, h * 2, b.PGs * 2, 256, msg) &&
-            make_map(&p->mG3, b.Gwb + b.goff[4], h, x, C, h * 2, b.PGs * 2, tc::N3, msg) &&
-            make_map(&p->mD1, b.Dwb + b.doff[0], x, h, C, x * 2, b.PDs * 2, 256, msg) &&
-            make_map(&p->mD2, b.Dwb + b.doff[2], h, h, C, h * 2, b.PDs * 2, 256, msg);
+            make_map(&p->mG1, b.Gwb + b.goff[0], z, h, NI, z * 2, b.PGs * 2, 256, msg) &&
+            make_map(&p->mG2, b.Gwb + b.goff[2], h, h, NI, h * 2, b.PGs * 2, 256, msg) &&
+            make_map(&p->mG3, b.Gwb + b.goff[4], h, x, NI, h * 2, b.PGs * 2, tc::N3, msg) &&
+            make_map(&p->mD1, b.Dwb + b.doff[0], x, h, NI, x * 2, b.PDs * 2, 256, msg) &&
+            make_map(&p->mD2, b.Dwb + b.doff[2], h, h, NI, h * 2, b.PDs * 2, 256, msg);
   if (!ok) {
     delete p;
     return nullptr;
@@ -748,6 +750,7 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   g.err = p->err;
   tc::KParams gc = g;  // every cell's own generator only (later minibatch steps)
   gc.centre = 1;
+  gc.indiv_off = b.indiv_off;
   gc.n_tiles = s.cells * g.mtiles;
   tc::KParams d = g;
   d.kind = tc::KIND_D;
@@ -826,6 +829,11 @@ int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensor
 
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg) {
   return launch(p->grid_g, p->mZ, p->mG1, p->mG2, p->mG3, p->pg, st, "generator forward", msg);
+}
+
+void tc_set_nbr(TcPlan* p, const int* nbr) {
+  p->pg.nbr = nbr;
+  p->pd.nbr = nbr;
 }
 
 int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg) {

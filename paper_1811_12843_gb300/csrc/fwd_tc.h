@@ -14,6 +14,7 @@ namespace lipz {
 struct TcShape {
   int cells, B, z, h, x;
   float slope;
+  int n_indiv;  // individuals the weight maps span (both snapshots: 2 * cells)
 };
 
 struct TcPlan;
@@ -23,9 +24,10 @@ bool tc_supported(int z, int h, int x, int B);
 
 // Device buffers of one population snapshot that the tensor-core forward reads and writes.
 //   Z: [cells][B][z] bf16; E: [cells][6B][x] bf16 (rows [0, B) real, then the fakes of slots
-//   0..4, which the generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5].
-//   Weights: bf16 copies (Gwb, Dwb) and fp32 masters (biases), per-individual strides
-//   PGs / PDs, tensor offsets goff / doff (W1, b1, W2, b2, W3, b3).
+//   0..4, which the generator kernel writes); logits [cells][5][6B] fp32; nbr [cells][5]
+//   (individual indices). Weights: bf16 copies (Gwb, Dwb) and fp32 masters (biases) of both
+//   snapshots, individual k = snapshot * cells + cell, per-individual strides PGs / PDs,
+//   tensor offsets goff / doff (W1, b1, W2, b2, W3, b3).
 //   Training forward of the selected pairs: the discriminator reads E[c] rows [0, B) and the
 //   fakes of slot sel_g[c] in place, src_g / src_d [cells] (selected individuals), outputs
 //   TH1, TH2 [cells][B][256], TG1, TG2 [cells][2B][256] bf16 and TL [cells][2B] fp32.
@@ -47,6 +49,7 @@ struct TcBuffers {
   // per-row block sums [cells][6B][tc_gram_halves(B)][6] fp32 (output); null without mixture
   const float* rnorm;
   float* gram_out;
+  int indiv_off;     // individual index of this snapshot's cell 0 (snapshot * cells)
   const int* sel_g;  // slot of each cell's selected generator (training: its fakes in E)
   const int* src_g;
   const int* src_d;
@@ -61,6 +64,8 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg);
 // Enqueue the generator kernel (fakes of every (cell, slot)) / the discriminator kernel (logits
 // of every (cell, slot)) on `st`. 0 on success.
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
+// Neighbour table [cells][5] (individual indices) that the next evaluation runs read.
+void tc_set_nbr(TcPlan* p, const int* nbr);
 // Generator forward of every cell's own centre on its z, into E's slot-0 fakes.
 int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);

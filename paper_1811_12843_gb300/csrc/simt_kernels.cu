@@ -410,14 +410,14 @@ __device__ void select_one(int c, int pop, const float* f5, const int* __restric
 }
 
 // Later minibatch steps of an iteration: every cell's centre trains again, in place of a
-// selection (slot 0, source individual c, its own lr, no mutation).
-__global__ void k_centre_select(int cells, SelectParams p, SelectIO io) {
+// selection (slot 0, source individual off + c, its own lr, no mutation).
+__global__ void k_centre_select(int cells, int off, SelectParams p, SelectIO io) {
   pdl_wait();
   const int gid = blockIdx.x * blockDim.x + threadIdx.x;
   const int c = gid >> 1;
   if (c >= cells) return;
   const int pop = gid & 1;
-  write_choice(c, pop, 0, c, io.lr_old[pop][c], p, io);
+  write_choice(c, pop, 0, off + c, io.lr_old[pop][off + c], p, io);
 }
 
 __global__ void k_select(const float* __restrict__ fG, const float* __restrict__ fD,
@@ -516,8 +516,9 @@ void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
              io);
 }
 
-void launch_centre_select(int cells, const SelectParams& p, const SelectIO& io, cudaStream_t st) {
-  launch_pdl(k_centre_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, cells, p, io);
+void launch_centre_select(int cells, int off, const SelectParams& p, const SelectIO& io,
+                          cudaStream_t st) {
+  launch_pdl(k_centre_select, dim3((2 * cells + 127) / 128), dim3(128), 0, st, cells, off, p, io);
 }
 
 // ------------------------------------------------------------------------------------------

@@ -14,7 +14,9 @@ def oracle_arch(arch) -> O.Arch:
                   replace_mode="always" if arch.replace_mode == 1 else "if_better",
                   lr_mutation=bool(arch.lr_mutation), lr_mut_std=float(arch.lr_mut_std),
                   lr_mut_prob=float(arch.lr_mut_prob), leaky_slope=float(arch.leaky_slope),
-                  train_steps=int(arch.train_steps))
+                  train_steps=int(arch.train_steps), mixture=bool(arch.mixture),
+                  mix_sigma=float(arch.mix_sigma),
+                  stale_neighbors=bool(arch.stale_neighbors))
 
 
 def max_rel(got, ref) -> float:
