@@ -166,10 +166,15 @@ class Arch:
     mixture: bool = False     # evolve each neighbourhood's generator-mixture weights
     stale_neighbors: bool = False  # neighbours seen one iteration late (asynchronous cells)
     mix_sigma: float = 0.01   # mixture mutation scale (Table 1)
+    kind: str = "mlp"         # "mlp" (Table 1, MNIST column) or "dcgan" (CelebA column)
+    ngf: int = 64             # DCGAN generator width (channels 8g, 4g, 2g, g)
+    ndf: int = 64             # DCGAN discriminator width (channels d, 2d, 4d, 8d)
 
 
 def g_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
     """Generator tensors in storage order; weights are [out][in] row-major."""
+    if a.kind == "dcgan":
+        return _dcgan().g_layout(a)
     return [("W1", (a.hidden, a.z_dim)), ("b1", (a.hidden,)),
             ("W2", (a.hidden, a.hidden)), ("b2", (a.hidden,)),
             ("W3", (a.x_dim, a.hidden)), ("b3", (a.x_dim,))]
@@ -177,9 +182,16 @@ def g_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
 
 def d_layout(a: Arch) -> List[Tuple[str, Tuple[int, ...]]]:
     """Discriminator tensors in storage order; weights are [out][in] row-major."""
+    if a.kind == "dcgan":
+        return _dcgan().d_layout(a)
     return [("W1", (a.hidden, a.x_dim)), ("b1", (a.hidden,)),
             ("W2", (a.hidden, a.hidden)), ("b2", (a.hidden,)),
             ("W3", (1, a.hidden)), ("b3", (1,))]
+
+
+def _dcgan():
+    from oracle import dcgan
+    return dcgan
 
 
 def n_params(layout) -> int:
@@ -266,6 +278,8 @@ class _Rounder:
 def g_forward(P: Dict[str, np.ndarray], z: np.ndarray, arch: Arch) -> Dict[str, np.ndarray]:
     """Generator MLP: z -> ReLU(256) -> ReLU(256) -> tanh(784). Returns every activation."""
     rb = _Rounder(arch)
+    if arch.kind == "dcgan":
+        return _dcgan().g_forward(P, z, arch, rb)
     zq = rb(z)
     h1 = rb(np.maximum(zq @ rb(P["W1"]).T + P["b1"], 0.0))
     h2 = rb(np.maximum(h1 @ rb(P["W2"]).T + P["b2"], 0.0))
@@ -280,6 +294,8 @@ def _lrelu(x, slope):
 def d_forward(P: Dict[str, np.ndarray], X: np.ndarray, arch: Arch) -> Dict[str, np.ndarray]:
     """Discriminator MLP: x -> LeakyReLU(256) -> LeakyReLU(256) -> logit (sigmoid in the loss)."""
     rb = _Rounder(arch)
+    if arch.kind == "dcgan":
+        return _dcgan().d_forward(P, X, arch, rb)
     Xq = rb(X)
     g1 = rb(_lrelu(Xq @ rb(P["W1"]).T + P["b1"], arch.leaky_slope))
     g2 = rb(_lrelu(g1 @ rb(P["W2"]).T + P["b2"], arch.leaky_slope))
@@ -333,8 +349,15 @@ def create(rows: int, cols: int, arch: Arch, seed: int) -> State:
         raise ValueError("grid needs rows, cols >= 1")
     gl, dl = g_layout(arch), d_layout(arch)
     cells = rows * cols
-    Gw = np.stack([init_params(seed, STREAM_INIT_G, c, gl) for c in range(cells)])
-    Dw = np.stack([init_params(seed, STREAM_INIT_D, c, dl) for c in range(cells)])
+    if arch.kind == "dcgan":
+        # weights N(0, 0.02^2) and batch-norm scales 1 + N(0, 0.02^2) from the normals of the
+        # cell's init stream (normal k for flat element k)
+        init = lambda stream, c, lay: _dcgan().init_params(
+            draw_normals(seed, stream, 0, c, n_params(lay)), lay)
+    else:
+        init = lambda stream, c, lay: init_params(seed, stream, c, lay)
+    Gw = np.stack([init(STREAM_INIT_G, c, gl) for c in range(cells)])
+    Dw = np.stack([init(STREAM_INIT_D, c, dl) for c in range(cells)])
     lr = float(np.float32(arch.lr))
     return State(rows, cols, arch, seed, 0,
                  Gw, np.zeros_like(Gw), np.zeros_like(Gw), np.zeros(cells, np.int64),
@@ -537,6 +560,8 @@ def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.nd
     the chain rule, layer by layer. Returns flat gradients in the parameter layouts."""
     a = arch
     rb = _Rounder(a)
+    if a.kind == "dcgan":
+        return _dcgan().pair_gradients(Gflat, Dflat, x, z, a, rb, unflatten, pair_losses, sigmoid)
     gl, dl = g_layout(a), d_layout(a)
     G, D = unflatten(Gflat, gl), unflatten(Dflat, dl)
     B = x.shape[0]
