@@ -57,7 +57,7 @@ enum {
   LIPZ_ERR_STATE = 6      /* call out of order (e.g. train before select) */
 };
 
-enum { LIPZ_MLP = 0 };                              /* network family */
+enum { LIPZ_MLP = 0, LIPZ_DCGAN64 = 1 };           /* network family */
 enum { LIPZ_FP32 = 0, LIPZ_BF16 = 1 };              /* arithmetic of the matrix products */
 enum { LIPZ_REPLACE_IF_BETTER = 0, LIPZ_REPLACE_ALWAYS = 1 };
 
@@ -85,7 +85,7 @@ enum { LIPZ_STEP_STREAM_STRIDE = 256 };
  */
 typedef struct lipz_arch {
   uint32_t struct_size;
-  int32_t kind;            /* LIPZ_MLP */
+  int32_t kind;            /* LIPZ_MLP, or LIPZ_DCGAN64 (see ngf) */
   int32_t precision;       /* LIPZ_FP32 or LIPZ_BF16 */
   int32_t z_dim;           /* 64 */
   int32_t hidden;          /* 256 */
@@ -120,6 +120,17 @@ typedef struct lipz_arch {
                               iteration after create or lipz_import_state sees them as they
                               are); a selected neighbour brings that older individual with its
                               optimiser state. Needs train_steps == 1. Default 0. */
+  int32_t ngf;             /* LIPZ_DCGAN64 (Table 1, CelebA column; the DCGAN architecture):
+                              G: z_dim -> ConvT 4x4 -> 8ngf x 4 x 4 -> ConvT 4x4 /2 ->
+                              4ngf x 8 x 8 -> 2ngf x 16 x 16 -> ngf x 32 x 32 (each batch norm in
+                              training mode + ReLU) -> 3 x 64 x 64 tanh; weights [in][out][4][4] */
+  int32_t ndf;             /* D: 3 x 64 x 64 -> Conv 4x4 /2 -> ndf x 32 x 32 -> 2ndf x 16 x 16 ->
+                              4ndf x 8 x 8 -> 8ndf x 4 x 4 (each LeakyReLU) -> Conv 4x4 -> logit;
+                              weights [out][in][4][4], no biases. Needs x_dim == 12288 (CHW
+                              images), train_steps == 1; runs on the CUDA-core kernels. Layout
+                              per generator: W1, gamma1, beta1, ..., W4, gamma4, beta4, W5;
+                              initial weights N(0, 0.02^2), scales 1 + N(0, 0.02^2), shifts 0.
+                              Default 64 (the 512/256/128/64 configuration). */
 } lipz_arch;
 
 typedef struct lipz_grid lipz_grid;

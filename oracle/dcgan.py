@@ -91,7 +91,7 @@ def conv2d(x: np.ndarray, w: np.ndarray, s: int, p: int) -> np.ndarray:
     for ky in range(k):
         for kx in range(k):
             win = xp[:, :, ky:ky + s * (Ho - 1) + 1:s, kx:kx + s * (Wo - 1) + 1:s]
-            y += np.einsum("nchw,oc->nohw", win, w[:, :, ky, kx])
+            y += np.einsum("nchw,oc->nohw", win, w[:, :, ky, kx], optimize=True)
     return y
 
 
@@ -107,8 +107,8 @@ def conv2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
         for kx in range(k):
             sl = (slice(None), slice(None), slice(ky, ky + s * (Ho - 1) + 1, s),
                   slice(kx, kx + s * (Wo - 1) + 1, s))
-            dw[:, :, ky, kx] = np.einsum("nohw,nchw->oc", dy, xp[sl])
-            dxp[sl] += np.einsum("nohw,oc->nchw", dy, w[:, :, ky, kx])
+            dw[:, :, ky, kx] = np.einsum("nohw,nchw->oc", dy, xp[sl], optimize=True)
+            dxp[sl] += np.einsum("nohw,oc->nchw", dy, w[:, :, ky, kx], optimize=True)
     return dxp[:, :, p:p + H, p:p + W], dw
 
 
@@ -122,7 +122,7 @@ def conv_transpose2d(x: np.ndarray, w: np.ndarray, s: int, p: int) -> np.ndarray
     for ky in range(k):
         for kx in range(k):
             full[:, :, ky:ky + s * (H - 1) + 1:s, kx:kx + s * (W - 1) + 1:s] += np.einsum(
-                "nchw,co->nohw", x, w[:, :, ky, kx])
+                "nchw,co->nohw", x, w[:, :, ky, kx], optimize=True)
     return full[:, :, p:Hf - p, p:Wf - p]
 
 
@@ -138,8 +138,8 @@ def conv_transpose2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
     for ky in range(k):
         for kx in range(k):
             d = dfull[:, :, ky:ky + s * (H - 1) + 1:s, kx:kx + s * (W - 1) + 1:s]
-            dx += np.einsum("nohw,co->nchw", d, w[:, :, ky, kx])
-            dw[:, :, ky, kx] = np.einsum("nchw,nohw->co", x, d)
+            dx += np.einsum("nohw,co->nchw", d, w[:, :, ky, kx], optimize=True)
+            dw[:, :, ky, kx] = np.einsum("nchw,nohw->co", x, d, optimize=True)
     return dx, dw
 
 

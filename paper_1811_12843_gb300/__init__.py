@@ -26,7 +26,7 @@ __all__ = [
 
 LIPZ_OK, LIPZ_ERR_INVALID, LIPZ_ERR_CUDA, LIPZ_ERR_OOM = 0, 1, 2, 3
 LIPZ_ERR_NONFINITE, LIPZ_ERR_TIMEOUT, LIPZ_ERR_STATE = 4, 5, 6
-LIPZ_MLP = 0
+LIPZ_MLP, LIPZ_DCGAN64 = 0, 1
 LIPZ_FP32, LIPZ_BF16 = 0, 1
 LIPZ_REPLACE_IF_BETTER, LIPZ_REPLACE_ALWAYS = 0, 1
 
@@ -53,6 +53,7 @@ class lipz_arch(ctypes.Structure):
         ("keep_grads", ctypes.c_int32), ("force_simt", ctypes.c_int32),
         ("train_steps", ctypes.c_int32), ("mixture", ctypes.c_int32),
         ("mix_sigma", ctypes.c_float), ("stale_neighbors", ctypes.c_int32),
+        ("ngf", ctypes.c_int32), ("ndf", ctypes.c_int32),
     ]
 
 
@@ -271,8 +272,14 @@ def arch_default(**overrides) -> lipz_arch:
     return a
 
 
-def param_counts(z_dim, hidden, x_dim):
+def param_counts(z_dim, hidden, x_dim, kind=LIPZ_MLP, ngf=64, ndf=64):
     """(PG, PD): parameters of one generator and one discriminator."""
+    if kind == LIPZ_DCGAN64:
+        ch = [z_dim, 8 * ngf, 4 * ngf, 2 * ngf, ngf]
+        pg = sum(ch[i] * ch[i + 1] * 16 + 2 * ch[i + 1] for i in range(4)) + ngf * 3 * 16
+        dh = [3, ndf, 2 * ndf, 4 * ndf, 8 * ndf]
+        pd = sum(dh[i] * dh[i + 1] * 16 for i in range(4)) + 8 * ndf * 16
+        return pg, pd
     pg = hidden * z_dim + hidden + hidden * hidden + hidden + x_dim * hidden + x_dim
     pd = hidden * x_dim + hidden + hidden * hidden + hidden + hidden + 1
     return pg, pd
@@ -285,7 +292,8 @@ class Grid:
         self.arch = arch if arch is not None else arch_default(**overrides)
         self.rows, self.cols, self.cells = rows, cols, rows * cols
         self.h = lipz_grid_create(rows, cols, self.arch, seed)
-        self.PG, self.PD = param_counts(self.arch.z_dim, self.arch.hidden, self.arch.x_dim)
+        a = self.arch
+        self.PG, self.PD = param_counts(a.z_dim, a.hidden, a.x_dim, a.kind, a.ngf, a.ndf)
 
     def close(self):
         if self.h:

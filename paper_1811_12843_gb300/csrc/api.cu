@@ -17,6 +17,7 @@
 #include "common.cuh"
 #include "engine.h"
 #include "bwd_tc.h"
+#include "dcgan.h"
 #include "fwd_tc.h"
 #include "lipz.h"
 
@@ -98,6 +99,8 @@ struct lipz_grid {
   Descs dsc[3]{}, dsc_stale[3]{};
   TcPlan* tc[3]{};
   TcbPlan* tcb[3]{};
+  DcPlan* dc = nullptr;  // LIPZ_DCGAN64: the convolutional networks' plan
+  bool dcgan = false;
   bool use_tcb = false;
 
   // tracing: event pairs per phase execution, resolved at lipz_profile_read
@@ -196,7 +199,16 @@ int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 // Layouts (PyTorch Linear convention, W [out][in] row-major).
 void make_layouts(lipz_grid* g) {
   const int64_t z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
+  if (g->dcgan) {
+    dc_layouts((int)z, g->a.ngf, g->a.ndf, &g->lg, &g->ld);
+    g->PG = g->lg.off[g->lg.n];
+    g->PD = g->ld.off[g->ld.n];
+    g->PGs = round_up(g->PG, 64);
+    g->PDs = round_up(g->PD, 64);
+    return;
+  }
   auto build = [](Layout& L, const int64_t shapes[6][2]) {
+    L = Layout{};
     L.n = 6;
     L.off[0] = 0;
     for (int t = 0; t < 6; ++t) {
@@ -285,6 +297,12 @@ int build_descs(lipz_grid* g, int p) {
   for (int i = 0; i < C * 5; ++i) {
     cur[i] = p * C + nbr[i];
     stale[i] = (i % 5 == 0 ? p : snap_prev(g, p)) * C + nbr[i];
+  }
+  if (g->dcgan) {
+    int rc;
+    if ((rc = upload(g, &g->nbr_cur[p], cur)) || (rc = upload(g, &g->nbr_stale[p], stale)))
+      return rc;
+    return LIPZ_OK;
   }
   // evaluation descriptors of one neighbour table
   auto eval_descs = [&](const std::vector<int>& tab, Descs& D) -> int {
@@ -495,7 +513,13 @@ int check_arch(const lipz_arch* a) {
   if (a->struct_size != sizeof(lipz_arch))
     return fail(nullptr, LIPZ_ERR_INVALID, "arch.struct_size is %u, expected %zu", a->struct_size,
                 sizeof(lipz_arch));
-  if (a->kind != LIPZ_MLP) return fail(nullptr, LIPZ_ERR_INVALID, "arch.kind must be LIPZ_MLP");
+  if (a->kind != LIPZ_MLP && a->kind != LIPZ_DCGAN64)
+    return fail(nullptr, LIPZ_ERR_INVALID, "arch.kind must be LIPZ_MLP or LIPZ_DCGAN64");
+  if (a->kind == LIPZ_DCGAN64 &&
+      (a->x_dim != 3 * 64 * 64 || a->ngf < 1 || a->ndf < 1 || a->ngf > 512 || a->ndf > 512 ||
+       a->train_steps != 1))
+    return fail(nullptr, LIPZ_ERR_INVALID,
+                "LIPZ_DCGAN64 needs x_dim == 12288, ngf and ndf in 1..512 and train_steps == 1");
   if (a->precision != LIPZ_FP32 && a->precision != LIPZ_BF16)
     return fail(nullptr, LIPZ_ERR_INVALID, "arch.precision must be LIPZ_FP32 or LIPZ_BF16");
   if (a->z_dim < 1 || a->hidden < 1 || a->x_dim < 1 || a->batch < 1 || a->hidden > 1024 ||
@@ -559,6 +583,7 @@ int create_impl(lipz_grid* g) {
   CK(g, cudaStreamCreateWithFlags(&g->copy_st, cudaStreamNonBlocking));
   CK(g, cudaEventCreateWithFlags(&g->ev_x, cudaEventDisableTiming));
   CK(g, cudaMallocHost(&g->hstat, 8 * sizeof(int)));
+  g->dcgan = g->a.kind == LIPZ_DCGAN64;
   make_layouts(g);
   g->e_cell = (int64_t)6 * B * x;
   g->nsnap = g->a.stale_neighbors ? 3 : 2;
@@ -621,7 +646,30 @@ int create_impl(lipz_grid* g) {
     if ((rc = h2d(g, g->G[p].lr, lr.data(), C * 4)) || (rc = h2d(g, g->D[p].lr, lr.data(), C * 4)) ||
         (rc = build_descs(g, p)))
       return rc;
-  g->use_tc = g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
+  g->use_tc = !g->dcgan && g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
+  if (g->dcgan) {
+    DcShape s{C, B, z, g->a.ngf, g->a.ndf, g->bf, g->a.leaky_slope};
+    DcBuffers b{};
+    b.Gw = g->G[0].w;
+    b.Gop = act_w(g->G[0]);
+    b.Dw = g->D[0].w;
+    b.Dop = act_w(g->D[0]);
+    b.PGs = g->PGs;
+    b.PDs = g->PDs;
+    b.goff = g->lg.off;
+    b.doff = g->ld.off;
+    b.Z = g->Z;
+    b.E = g->E;
+    b.e_cell = g->e_cell;
+    b.logits = g->logits;
+    b.src_g = g->src_g;
+    b.src_d = g->src_d;
+    b.gG = g->gG;
+    b.gD = g->gD;
+    std::string msg;
+    g->dc = dc_plan_create(s, b, &msg);
+    if (!g->dc) return fail(g, LIPZ_ERR_OOM, "DCGAN plan: %s", msg.c_str());
+  }
   if (g->use_tc) {
     for (int p = 0; p < g->nsnap; ++p) {
       TcShape s{C, B, z, h, x, g->a.leaky_slope, g->nsnap * C};
@@ -775,7 +823,22 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
   draw(x_ready ? DRAW_NOISE : DRAW_REAL | DRAW_NOISE, true);
   CKL(g);
   phase_end(g, LIPZ_PHASE_BATCH, 1);
-  if (g->use_tc) {
+  if (g->dcgan) {
+    std::string msg;
+    phase_begin(g, LIPZ_PHASE_G_FWD);
+    if (dc_eval_g(g->dc, eval_nbr(g), g->st, &msg))
+      return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_G_FWD, dc_eval_launches(g->dc, 0));
+    if (x_ready) {
+      CK(g, cudaStreamWaitEvent(g->st, x_ready, 0));
+      draw(DRAW_REAL, false);
+      CKL(g);
+    }
+    phase_begin(g, LIPZ_PHASE_D_FWD);
+    if (dc_eval_d(g->dc, eval_nbr(g), g->st, &msg))
+      return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_D_FWD, dc_eval_launches(g->dc, 1));
+  } else if (g->use_tc) {
     std::string msg;
     tc_set_nbr(g->tc[p], eval_nbr(g));
     phase_begin(g, LIPZ_PHASE_G_FWD);
@@ -874,6 +937,23 @@ int select_impl(lipz_grid* g) {
 int train_once(lipz_grid* g) {
   const int C = g->cells, B = g->a.batch, h = g->a.hidden, x = g->a.x_dim, z = g->a.z_dim;
   const int p = g->cur;
+  if (g->dcgan) {
+    // forward and backward of the selected pairs (gradients into gG, gD), then Adam +
+    // replacement into the next snapshot
+    std::string msg;
+    phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
+    if (dc_train(g->dc, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
+    phase_end(g, LIPZ_PHASE_TRAIN_BWD, dc_train_launches(g->dc));
+    phase_begin(g, LIPZ_PHASE_ADAM);
+    launch_adam(g->G[0], g->G[snap_next(g, p)], g->gG, g->src_g, g->coef_g, C, g->PG, g->PGs,
+                g->a.beta1, g->a.beta2, g->a.eps, g->st);
+    launch_adam(g->D[0], g->D[snap_next(g, p)], g->gD, g->src_d, g->coef_d, C, g->PD, g->PDs,
+                g->a.beta1, g->a.beta2, g->a.eps, g->st);
+    CKL(g);
+    phase_end(g, LIPZ_PHASE_ADAM, 2);
+    g->cur = snap_next(g, p);
+    return LIPZ_OK;
+  }
   const Descs& D = g->dsc[p];
   phase_begin(g, LIPZ_PHASE_TRAIN_FWD);
   // the CUDA-core kernels read the discriminator's training input as one array TX; the
@@ -1116,6 +1196,8 @@ int lipz_arch_default(lipz_arch* a) {
   a->mixture = 0;
   a->mix_sigma = 0.01f;
   a->stale_neighbors = 0;
+  a->ngf = 64;
+  a->ndf = 64;
   return LIPZ_OK;
 }
 
@@ -1149,6 +1231,7 @@ int lipz_grid_create(int rows, int cols, const lipz_arch* arch, uint64_t seed, l
 int lipz_grid_destroy(lipz_grid* g) {
   if (!g) return LIPZ_OK;
   cudaStreamSynchronize(g->st);
+  if (g->dc) dc_plan_destroy(g->dc);
   for (int p = 0; p < 3; ++p) {
     if (g->tc[p]) tc_plan_destroy(g->tc[p]);
     if (g->tcb[p]) tcb_plan_destroy(g->tcb[p]);

@@ -1,0 +1,557 @@
+// DCGAN evaluation and training steps of the grid on the CUDA-core kernels (conv_kernels.cu).
+// Every layer of every problem of a phase is one grouped launch: the evaluation's problems are
+// the (cell, slot) pairs, the training's the cells. Weights are read in place from the
+// population (individual index from the neighbour table or the selection), activations are
+// NCHW per sample.
+#include "dcgan.h"
+
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+namespace lipz {
+
+namespace {
+
+int ilog2(int v) {
+  int l = 0;
+  while ((1 << l) < v) ++l;
+  return l;
+}
+
+}  // namespace
+
+void dc_layouts(int z, int ngf, int ndf, Layout* lg, Layout* ld) {
+  const int64_t g = ngf, d = ndf;
+  const int64_t gch[5] = {z, 8 * g, 4 * g, 2 * g, g};
+  Layout L{};
+  int t = 0;
+  int64_t off = 0;
+  auto add = [&](int64_t n, int init, float bound) {
+    L.off[t] = off;
+    L.init[t] = init;
+    L.bound[t] = bound;
+    off += n;
+    ++t;
+  };
+  for (int i = 0; i < 4; ++i) {
+    add(gch[i] * gch[i + 1] * 16, INIT_NORMAL, 0.02f);
+    add(gch[i + 1], INIT_ONE_NORMAL, 0.02f);
+    add(gch[i + 1], INIT_UNIFORM, 0.f);
+  }
+  add(g * 3 * 16, INIT_NORMAL, 0.02f);
+  L.n = t;
+  L.off[t] = off;
+  *lg = L;
+  Layout M{};
+  const int64_t dch[5] = {3, d, 2 * d, 4 * d, 8 * d};
+  L = M;
+  t = 0;
+  off = 0;
+  for (int i = 0; i < 4; ++i) add(dch[i + 1] * dch[i] * 16, INIT_NORMAL, 0.02f);
+  add(8 * d * 16, INIT_NORMAL, 0.02f);
+  L.n = t;
+  L.off[t] = off;
+  *ld = L;
+}
+
+struct DcPlan {
+  DcShape s;
+  DcBuffers b;
+  std::vector<void*> allocs;
+  // evaluation: generator layers (problems cells * 5), discriminator layers (5 problems per
+  // cell, launched cell by cell)
+  ConvDesc* eg[5];
+  BnDesc* ebn[4];
+  ConvDesc* ed[4];
+  LogitDesc* edl;
+  // training (problems = cells)
+  ConvDesc* tg[5];
+  BnDesc* tbn[4];
+  ConvDesc* td[4];
+  LogitDesc* tdl;
+  LogitDesc* tdl_back_d;  // D loss, 2B rows, with the output layer's gradient
+  LogitDesc* tdl_back_g;  // G loss, fake rows
+  ConvDesc* dw[4];        // discriminator weight gradients W4, W3, W2, W1
+  ConvDesc* dd[3];        // D-loss deltas into layers 3, 2, 1
+  ConvDesc* gd[4];        // G-loss deltas into layers 3, 2, 1 and the fakes
+  ConvDesc* gw[5];        // generator weight gradients W5, W4, W3, W2, W1
+  ConvDesc* gdh[4];       // generator deltas dh4, dh3, dh2, dh1
+  BnDesc* gbn[4];         // batch-norm backward of layers 4, 3, 2, 1
+  void* TX;               // [cells][2B][12288] discriminator training input (real, fakes)
+  float* tlogits;         // [cells][2B]
+  void *dl_d, *dl_g;
+  float* part;
+  int64_t part_floats;
+  int splits_dw[4], splits_gw[5];
+  int64_t pstride_dw[4], pstride_gw[5];
+  int eval_launches, train_launches;
+};
+
+namespace {
+
+template <typename T>
+int dev_alloc(DcPlan* p, T** out, size_t bytes, std::string* msg) {
+  void* q = nullptr;
+  if (cudaMalloc(&q, bytes ? bytes : 16) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "cudaMalloc of " + std::to_string(bytes) + " bytes failed";
+    return 1;
+  }
+  p->allocs.push_back(q);
+  *out = (T*)q;
+  return 0;
+}
+
+template <typename T>
+int upload(DcPlan* p, T** out, const std::vector<T>& v, std::string* msg) {
+  if (dev_alloc(p, out, v.size() * sizeof(T), msg)) return 1;
+  if (cudaMemcpy(*out, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "descriptor upload failed";
+    return 1;
+  }
+  return 0;
+}
+
+ConvDesc cdesc(const void* a, int n, int ca, int ha, const void* b, int co, int ho, int s,
+               int pad, void* out) {
+  ConvDesc d;
+  memset(&d, 0, sizeof d);
+  d.a = a;
+  d.b = b;
+  d.out = out;
+  d.n = n;
+  d.ca = ca;
+  d.lha = d.lwa = ilog2(ha);
+  d.co = co;
+  d.lho = d.lwo = ilog2(ho);
+  d.s = s;
+  d.p = pad;
+  return d;
+}
+
+// WGRAD splits: chunks of about 4096 of the K = n * Ha * Wa reduction
+int wgrad_splits(const ConvDesc& d) {
+  const int64_t K = (int64_t)d.n << (d.lha + d.lwa);
+  return (int)std::max<int64_t>(1, std::min<int64_t>(64, K / 4096));
+}
+
+}  // namespace
+
+DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
+  DcPlan* p = new DcPlan();
+  p->s = s;
+  p->b = b;
+  const int C = s.cells, B = s.B, g = s.ngf, d = s.ndf, z = s.z;
+  const size_t es = s.bf ? 2 : 4;
+  const int64_t X = 3 * 64 * 64;
+  auto el = [es](const void* base, int64_t i) { return (const char*)base + i * (int64_t)es; };
+  auto elw = [es](void* base, int64_t i) { return (char*)base + i * (int64_t)es; };
+  // generator channels and sizes per layer (input of layer l: gc[l] x gs[l]^2)
+  const int gc[6] = {z, 8 * g, 4 * g, 2 * g, g, 3};
+  const int gs[6] = {1, 4, 8, 16, 32, 64};
+  const int dc[6] = {3, d, 2 * d, 4 * d, 8 * d, 1};
+  const int ds[6] = {64, 32, 16, 8, 4, 1};
+  int64_t gsz[5], dsz[5];  // per-sample sizes of the generator outputs 1..4 / disc. outputs 1..4
+  for (int l = 1; l <= 4; ++l) {
+    gsz[l] = (int64_t)gc[l] * gs[l] * gs[l];
+    dsz[l] = (int64_t)dc[l] * ds[l] * ds[l];
+  }
+  const int64_t gmax = gsz[4] > gsz[3] ? gsz[4] : gsz[3], dmax = dsz[1];
+  int64_t gall = 0, dall = 0;
+  for (int l = 1; l <= 4; ++l) {
+    gall += gsz[l];
+    dall += dsz[l];
+  }
+  int64_t goffs[5] = {0}, doffs[5] = {0};  // per-sample offsets of stored layers
+  for (int l = 2; l <= 4; ++l) {
+    goffs[l] = goffs[l - 1] + gsz[l - 1];
+    doffs[l] = doffs[l - 1] + dsz[l - 1];
+  }
+  const int PE = C * 5;
+  // ---- buffers
+  float *ec, *emean, *einv, *tc, *tmean, *tinv, *dh;
+  void *eh, *ex, *ey, *th, *ta, *P, *Q, *P2, *Q2, *dcb, *d5;
+  int64_t stats = 15 * (int64_t)g;  // channels of the four batch-normalised layers
+  if (dev_alloc(p, &ec, (size_t)PE * B * gmax * 4, msg) ||
+      dev_alloc(p, &eh, (size_t)PE * B * gmax * es, msg) ||
+      dev_alloc(p, &emean, (size_t)PE * stats * 4, msg) ||
+      dev_alloc(p, &einv, (size_t)PE * stats * 4, msg) ||
+      dev_alloc(p, &ex, (size_t)5 * 6 * B * dmax * es, msg) ||
+      dev_alloc(p, &ey, (size_t)5 * 6 * B * dsz[2] * es, msg) ||
+      dev_alloc(p, &tc, (size_t)C * B * gall * 4, msg) ||
+      dev_alloc(p, &th, (size_t)C * B * gall * es, msg) ||
+      dev_alloc(p, &tmean, (size_t)C * stats * 4, msg) ||
+      dev_alloc(p, &tinv, (size_t)C * stats * 4, msg) ||
+      dev_alloc(p, &p->TX, (size_t)C * 2 * B * X * es, msg) ||
+      dev_alloc(p, &ta, (size_t)C * 2 * B * dall * es, msg) ||
+      dev_alloc(p, &p->tlogits, (size_t)C * 2 * B * 4, msg) ||
+      dev_alloc(p, &p->dl_d, (size_t)C * 2 * B * es, msg) ||
+      dev_alloc(p, &p->dl_g, (size_t)C * B * es, msg) ||
+      dev_alloc(p, &P, (size_t)C * 2 * B * dmax * es, msg) ||
+      dev_alloc(p, &Q, (size_t)C * 2 * B * dmax * es, msg) ||
+      dev_alloc(p, &P2, (size_t)C * B * dmax * es, msg) ||
+      dev_alloc(p, &Q2, (size_t)C * B * dmax * es, msg) ||
+      dev_alloc(p, &dh, (size_t)C * B * gmax * 4, msg) ||
+      dev_alloc(p, &dcb, (size_t)C * B * gmax * es, msg) ||
+      dev_alloc(p, &d5, (size_t)C * B * X * es, msg)) {
+    dc_plan_destroy(p);
+    return nullptr;
+  }
+  int64_t stat_off[5] = {0};  // per-problem offsets of each layer's statistics
+  for (int l = 2; l <= 4; ++l) stat_off[l] = stat_off[l - 1] + gc[l - 1];
+  const int64_t* go = b.goff;
+  const int64_t* dof = b.doff;
+  auto Wg = [&](int l) { return el(b.Gop, go[3 * (l - 1)]); };  // W1..W5 at 0, 3, 6, 9, 12
+  auto Wd = [&](int l) { return el(b.Dop, dof[l - 1]); };
+  std::vector<ConvDesc> v;
+  std::vector<BnDesc> vb;
+  auto bn = [&](const float* c, void* h, float* mean, float* inv, const int* wsel, int idx,
+                int l, int n) {
+    BnDesc q;
+    memset(&q, 0, sizeof q);
+    q.c = c;
+    q.h = h;
+    q.mean = mean;
+    q.inv = inv;
+    q.params = b.Gw;
+    q.wsel = wsel;
+    q.wsel_stride = b.PGs;
+    q.wsel_idx = idx;
+    q.off_gamma = go[3 * (l - 1) + 1];
+    q.off_beta = go[3 * (l - 1) + 2];
+    q.n = n;
+    q.C = gc[l];
+    q.lhw = 2 * ilog2(gs[l]);
+    return q;
+  };
+  bool ok = true;
+  // ---- evaluation: generator of every (cell, slot) on the cell's noise
+  for (int l = 1; l <= 5; ++l) {
+    v.clear();
+    vb.clear();
+    for (int c = 0; c < C; ++c)
+      for (int sl = 0; sl < 5; ++sl) {
+        const int pr = c * 5 + sl;
+        const void* in = l == 1 ? el(b.Z, (int64_t)c * B * z) : el(eh, (int64_t)pr * B * gmax);
+        void* out = l == 5 ? elw(b.E, (int64_t)c * b.e_cell + (int64_t)(1 + sl) * B * X)
+                           : (void*)(ec + (int64_t)pr * B * gmax);
+        ConvDesc q = cdesc(in, B, gc[l - 1], gs[l - 1], Wg(l), gc[l], gs[l], l == 1 ? 1 : 2,
+                           l == 1 ? 0 : 1, out);
+        q.wsel_stride = b.PGs;
+        q.wsel_idx = pr;
+        v.push_back(q);
+        if (l <= 4)
+          vb.push_back(bn(ec + (int64_t)pr * B * gmax, elw(eh, (int64_t)pr * B * gmax),
+                          emean + pr * stats + stat_off[l], einv + pr * stats + stat_off[l],
+                          nullptr, pr, l, B));
+      }
+    ok = ok && !upload(p, &p->eg[l - 1], v, msg);
+    if (l <= 4) ok = ok && !upload(p, &p->ebn[l - 1], vb, msg);
+  }
+  // ---- evaluation: discriminator of every (cell, slot) on E[c] (6B rows), one cell per launch
+  // (buffers ex / ey hold the five problems of one cell)
+  for (int l = 1; l <= 4; ++l) {
+    v.clear();
+    for (int c = 0; c < C; ++c)
+      for (int sl = 0; sl < 5; ++sl) {
+        void* bufs[2] = {elw(ex, (int64_t)sl * 6 * B * dmax), elw(ey, (int64_t)sl * 6 * B * dsz[2])};
+        const void* in = l == 1 ? el(b.E, (int64_t)c * b.e_cell) : bufs[l % 2];
+        void* out = bufs[(l + 1) % 2];
+        ConvDesc q = cdesc(in, 6 * B, dc[l - 1], ds[l - 1], Wd(l), dc[l], ds[l], 2, 1, out);
+        q.wsel_stride = b.PDs;
+        q.wsel_idx = c * 5 + sl;
+        v.push_back(q);
+      }
+    ok = ok && !upload(p, &p->ed[l - 1], v, msg);
+  }
+  {
+    std::vector<LogitDesc> vl;
+    for (int c = 0; c < C; ++c)
+      for (int sl = 0; sl < 5; ++sl) {
+        LogitDesc q;
+        memset(&q, 0, sizeof q);
+        q.a = elw(ey, (int64_t)sl * 6 * B * dsz[2]);  // layer 4's output (4 x 4 x 8d)
+        q.w = Wd(5);
+        q.wsel_stride = b.PDs;
+        q.wsel_idx = c * 5 + sl;
+        q.logits = b.logits + (int64_t)(c * 5 + sl) * 6 * B;
+        q.rows = 6 * B;
+        q.K = (int)dsz[4];
+        vl.push_back(q);
+      }
+    ok = ok && !upload(p, &p->edl, vl, msg);
+  }
+  // ---- training forward: the selected generator on the cell's noise, fakes into TX rows
+  // [B, 2B); the selected discriminator on TX (real rows copied in at run time)
+  auto tgc = [&](int c, int l) { return tc + ((int64_t)c * B) * gall + (int64_t)B * goffs[l]; };
+  auto tgh = [&](int c, int l) { return elw(th, (int64_t)c * B * gall + (int64_t)B * goffs[l]); };
+  auto tda = [&](int c, int l) { return elw(ta, (int64_t)c * 2 * B * dall + (int64_t)2 * B * doffs[l]); };
+  auto tx = [&](int c) { return elw(p->TX, (int64_t)c * 2 * B * X); };
+  for (int l = 1; l <= 5; ++l) {
+    v.clear();
+    vb.clear();
+    for (int c = 0; c < C; ++c) {
+      const void* in = l == 1 ? el(b.Z, (int64_t)c * B * z) : (const void*)tgh(c, l - 1);
+      void* out = l == 5 ? elw(tx(c), (int64_t)B * X) : (void*)tgc(c, l);
+      ConvDesc q = cdesc(in, B, gc[l - 1], gs[l - 1], Wg(l), gc[l], gs[l], l == 1 ? 1 : 2,
+                         l == 1 ? 0 : 1, out);
+      q.wsel = b.src_g;
+      q.wsel_stride = b.PGs;
+      q.wsel_idx = c;
+      v.push_back(q);
+      if (l <= 4)
+        vb.push_back(bn(tgc(c, l), tgh(c, l), tmean + c * stats + stat_off[l],
+                        tinv + c * stats + stat_off[l], b.src_g, c, l, B));
+    }
+    ok = ok && !upload(p, &p->tg[l - 1], v, msg);
+    if (l <= 4) ok = ok && !upload(p, &p->tbn[l - 1], vb, msg);
+  }
+  for (int l = 1; l <= 4; ++l) {
+    v.clear();
+    for (int c = 0; c < C; ++c) {
+      const void* in = l == 1 ? (const void*)tx(c) : (const void*)tda(c, l - 1);
+      ConvDesc q = cdesc(in, 2 * B, dc[l - 1], ds[l - 1], Wd(l), dc[l], ds[l], 2, 1, tda(c, l));
+      q.wsel = b.src_d;
+      q.wsel_stride = b.PDs;
+      q.wsel_idx = c;
+      v.push_back(q);
+    }
+    ok = ok && !upload(p, &p->td[l - 1], v, msg);
+  }
+  {
+    std::vector<LogitDesc> vl, vd, vg;
+    for (int c = 0; c < C; ++c) {
+      LogitDesc q;
+      memset(&q, 0, sizeof q);
+      q.a = tda(c, 4);
+      q.w = Wd(5);
+      q.wsel = b.src_d;
+      q.wsel_stride = b.PDs;
+      q.wsel_idx = c;
+      q.logits = p->tlogits + (int64_t)c * 2 * B;
+      q.rows = 2 * B;
+      q.K = (int)dsz[4];
+      vl.push_back(q);
+      LogitDesc r = q;
+      r.dl = elw(p->dl_d, (int64_t)c * 2 * B);
+      r.da = elw(P, (int64_t)c * 2 * B * dmax);
+      r.dw = b.gD + (int64_t)c * b.PDs + dof[4];
+      vd.push_back(r);
+      LogitDesc t = q;
+      t.a = elw(tda(c, 4), (int64_t)B * dsz[4]);
+      t.rows = B;
+      t.dl = elw(p->dl_g, (int64_t)c * B);
+      t.da = elw(P2, (int64_t)c * B * dmax);
+      t.dw = nullptr;
+      vg.push_back(t);
+    }
+    ok = ok && !upload(p, &p->tdl, vl, msg) && !upload(p, &p->tdl_back_d, vd, msg) &&
+         !upload(p, &p->tdl_back_g, vg, msg);
+  }
+  // ---- discriminator backward (D loss, 2B rows): the delta of layer l's output is in P for
+  // l = 4, 2 and in Q for l = 3, 1
+  int64_t part_need = 0;
+  for (int l = 4; l >= 1; --l) {
+    v.clear();
+    std::vector<ConvDesc> vd;
+    for (int c = 0; c < C; ++c) {
+      void* dout = elw((l % 2 == 0) ? P : Q, (int64_t)c * 2 * B * dmax);
+      const void* prev = l == 1 ? (const void*)tx(c) : (const void*)tda(c, l - 1);
+      // weight gradient: a = delta of the output (dc[l] x ds[l]^2), b = the layer's input
+      ConvDesc w = cdesc(dout, 2 * B, dc[l], ds[l], prev, dc[l - 1], ds[l - 1], 2, 1,
+                         b.gD + (int64_t)c * b.PDs + dof[l - 1]);
+      v.push_back(w);
+      if (l >= 2) {
+        void* din = elw((l % 2 == 0) ? Q : P, (int64_t)c * 2 * B * dmax);
+        ConvDesc q = cdesc(dout, 2 * B, dc[l], ds[l], Wd(l), dc[l - 1], ds[l - 1], 2, 1, din);
+        q.wsel = b.src_d;
+        q.wsel_stride = b.PDs;
+        q.wsel_idx = c;
+        q.aux = tda(c, l - 1);
+        vd.push_back(q);
+      }
+    }
+    const int k = 4 - l;
+    p->splits_dw[k] = wgrad_splits(v[0]);
+    p->pstride_dw[k] = (int64_t)v[0].ca * v[0].co * 16;
+    part_need = std::max<int64_t>(part_need, (int64_t)C * p->splits_dw[k] * p->pstride_dw[k]);
+    ok = ok && !upload(p, &p->dw[k], v, msg);
+    if (l >= 2) ok = ok && !upload(p, &p->dd[k], vd, msg);
+  }
+  // ---- generator loss through the discriminator (fake rows): deltas P2 (l = 4, 2), Q2
+  // (l = 3, 1), then the fakes' delta times tanh' into d5
+  for (int l = 4; l >= 1; --l) {
+    v.clear();
+    for (int c = 0; c < C; ++c) {
+      void* dout = elw((l % 2 == 0) ? P2 : Q2, (int64_t)c * B * dmax);
+      const bool last = l == 1;
+      void* din = last ? elw(d5, (int64_t)c * B * X) : elw((l % 2 == 0) ? Q2 : P2, (int64_t)c * B * dmax);
+      ConvDesc q = cdesc(dout, B, dc[l], ds[l], Wd(l), dc[l - 1], ds[l - 1], 2, 1, din);
+      q.wsel = b.src_d;
+      q.wsel_stride = b.PDs;
+      q.wsel_idx = c;
+      q.aux = last ? elw(tx(c), (int64_t)B * X)
+                   : elw(tda(c, l - 1), (int64_t)B * dsz[l - 1]);
+      v.push_back(q);
+    }
+    ok = ok && !upload(p, &p->gd[4 - l], v, msg);
+  }
+  // ---- generator backward: weight gradient of layer l from its input (h_{l-1} or z) and the
+  // delta of its output (d5, or dc_l in dcb); delta of its input dh_{l-1} (fp32), then the
+  // batch normalisation of layer l - 1
+  for (int l = 5; l >= 1; --l) {
+    v.clear();
+    std::vector<ConvDesc> vd;
+    vb.clear();
+    for (int c = 0; c < C; ++c) {
+      const void* dout = l == 5 ? elw(d5, (int64_t)c * B * X) : elw(dcb, (int64_t)c * B * gmax);
+      const void* in = l == 1 ? el(b.Z, (int64_t)c * B * z) : (const void*)tgh(c, l - 1);
+      ConvDesc w = cdesc(in, B, gc[l - 1], gs[l - 1], dout, gc[l], gs[l], l == 1 ? 1 : 2,
+                         l == 1 ? 0 : 1, b.gG + (int64_t)c * b.PGs + go[3 * (l - 1)]);
+      v.push_back(w);
+      if (l >= 2) {
+        ConvDesc q = cdesc(dout, B, gc[l], gs[l], Wg(l), gc[l - 1], gs[l - 1], 2, 1,
+                           dh + (int64_t)c * B * gmax);
+        q.wsel = b.src_g;
+        q.wsel_stride = b.PGs;
+        q.wsel_idx = c;
+        vd.push_back(q);
+        BnDesc r = bn(tgc(c, l - 1), tgh(c, l - 1), tmean + c * stats + stat_off[l - 1],
+                      tinv + c * stats + stat_off[l - 1], b.src_g, c, l - 1, B);
+        r.dh = dh + (int64_t)c * B * gmax;
+        r.dc = elw(dcb, (int64_t)c * B * gmax);
+        r.dparams = b.gG + (int64_t)c * b.PGs;
+        vb.push_back(r);
+      }
+    }
+    const int k = 5 - l;
+    p->splits_gw[k] = wgrad_splits(v[0]);
+    p->pstride_gw[k] = (int64_t)v[0].ca * v[0].co * 16;
+    part_need = std::max<int64_t>(part_need, (int64_t)C * p->splits_gw[k] * p->pstride_gw[k]);
+    ok = ok && !upload(p, &p->gw[k], v, msg);
+    if (l >= 2) {
+      ok = ok && !upload(p, &p->gdh[k], vd, msg);
+      ok = ok && !upload(p, &p->gbn[k], vb, msg);
+    }
+  }
+  p->part_floats = part_need;
+  ok = ok && !dev_alloc(p, &p->part, (size_t)part_need * 4, msg);
+  if (!ok) {
+    dc_plan_destroy(p);
+    return nullptr;
+  }
+  p->eval_launches = 9 + 5 * C;
+  p->train_launches = 50;
+  return p;
+}
+
+void dc_plan_destroy(DcPlan* p) {
+  if (!p) return;
+  for (void* q : p->allocs) cudaFree(q);
+  delete p;
+}
+
+namespace {
+int check(std::string* msg, const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) return 0;
+  if (msg) *msg = std::string(what) + ": " + cudaGetErrorString(e);
+  return 1;
+}
+}  // namespace
+
+int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
+  const DcShape& s = p->s;
+  const int C = s.cells, B = s.B, g = s.ngf;
+  const int gc[6] = {s.z, 8 * g, 4 * g, 2 * g, g, 3};
+  const int gs[6] = {1, 4, 8, 16, 32, 64};
+  const int PE = C * 5;
+  for (int l = 1; l <= 5; ++l) {
+    launch_conv(CONVT_FWD_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->eg[l - 1], PE,
+                B * gs[l] * gs[l], gc[l], nbr, 1, nullptr, 0, s.slope, st);
+    if (l <= 4) launch_bn_relu(s.bf, p->ebn[l - 1], PE, gc[l], nbr, st);
+  }
+  return check(msg, "DCGAN generator evaluation");
+}
+
+int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
+  const DcShape& s = p->s;
+  const int C = s.cells, B = s.B, d = s.ndf;
+  const int dc[5] = {3, d, 2 * d, 4 * d, 8 * d};
+  const int ds[5] = {64, 32, 16, 8, 4};
+  for (int c = 0; c < C; ++c) {
+    for (int l = 1; l <= 4; ++l)
+      launch_conv(CONV_FWD_MODE, CEPI_LRELU_, s.bf, false, p->ed[l - 1] + c * 5, 5,
+                  6 * B * ds[l] * ds[l], dc[l], nbr, 1, nullptr, 0, s.slope, st);
+    launch_logit_dot(s.bf, p->edl + c * 5, 5, 6 * B, nbr, st);
+  }
+  return check(msg, "DCGAN discriminator evaluation");
+}
+
+int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
+  const DcShape& s = p->s;
+  const int C = s.cells, B = s.B, g = s.ngf, d = s.ndf;
+  const size_t es = s.bf ? 2 : 4;
+  const int64_t X = 3 * 64 * 64;
+  const int gc[6] = {s.z, 8 * g, 4 * g, 2 * g, g, 3};
+  const int gs[6] = {1, 4, 8, 16, 32, 64};
+  const int dc[5] = {3, d, 2 * d, 4 * d, 8 * d};
+  const int ds[5] = {64, 32, 16, 8, 4};
+  // forward of the selected pair
+  for (int l = 1; l <= 5; ++l) {
+    launch_conv(CONVT_FWD_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->tg[l - 1], C,
+                B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0, s.slope, st);
+    if (l <= 4) launch_bn_relu(s.bf, p->tbn[l - 1], C, gc[l], nullptr, st);
+  }
+  // the real rows of every cell's minibatch into TX rows [0, B)
+  if (cudaMemcpy2DAsync(p->TX, 2 * B * X * es, p->b.E, p->b.e_cell * es, B * X * es, C,
+                        cudaMemcpyDeviceToDevice, st) != cudaSuccess) {
+    check(msg, "DCGAN training input copy");
+    return 1;
+  }
+  for (int l = 1; l <= 4; ++l)
+    launch_conv(CONV_FWD_MODE, CEPI_LRELU_, s.bf, false, p->td[l - 1], C,
+                2 * B * ds[l] * ds[l], dc[l], nullptr, 1, nullptr, 0, s.slope, st);
+  launch_logit_dot(s.bf, p->tdl, C, 2 * B, nullptr, st);
+  launch_dc_dlogit(s.bf, p->tlogits, C, B, p->dl_d, p->dl_g, st);
+  // discriminator backward (D loss)
+  launch_logit_back(s.bf, p->tdl_back_d, C, (int)(8 * d * 16), true, s.slope, st);
+  for (int l = 4; l >= 1; --l) {
+    const int k = 4 - l;
+    launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
+                nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
+    if (l >= 2)
+      launch_conv(CONVT_FWD_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
+                  2 * B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0, s.slope,
+                  st);
+  }
+  // the generator loss through the discriminator
+  launch_logit_back(s.bf, p->tdl_back_g, C, (int)(8 * d * 16), false, s.slope, st);
+  for (int l = 4; l >= 1; --l)
+    launch_conv(CONVT_FWD_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
+                p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
+                s.slope, st);
+  // generator backward
+  for (int l = 5; l >= 1; --l) {
+    const int k = 5 - l;
+    launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
+                nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
+    if (l >= 2) {
+      launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
+                  B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
+      launch_bn_relu_backward(s.bf, p->gbn[k], C, gc[l - 1], st);
+    }
+  }
+  return check(msg, "DCGAN training step");
+}
+
+int dc_eval_launches(const DcPlan* p, int part) {
+  return part == 0 ? 9 : p->eval_launches - 9;
+}
+int dc_train_launches(const DcPlan* p) { return p->train_launches; }
+
+}  // namespace lipz

@@ -12,12 +12,15 @@ struct GemvDesc;
 struct ColSumDesc;
 typedef __nv_bfloat16 bf16;
 
-// Flat parameter layout of one individual: tensor t occupies [off[t], off[t+1]); bound[t] is
-// its Xavier bound (0 for biases).
+// Flat parameter layout of one individual: tensor t occupies [off[t], off[t+1]). Its
+// initialisation: init[t] = INIT_UNIFORM: U(-bound, bound) (Xavier; 0 when bound is 0),
+// INIT_NORMAL: bound * N(0, 1), INIT_ONE_NORMAL: 1 + bound * N(0, 1).
+enum { INIT_UNIFORM = 0, INIT_NORMAL = 1, INIT_ONE_NORMAL = 2 };
 struct Layout {
   int n;
-  int64_t off[7];
-  float bound[6];
+  int64_t off[17];
+  float bound[16];
+  int init[16];
 };
 
 // One population snapshot (all cells): fp32 master weights, Adam moments, bf16 copy (bf16
@@ -79,6 +82,71 @@ void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD,
 // (lr, 1 / (1 - beta1^(step+1)), 1 / (1 - beta2^(step+1)), step + 1).
 void launch_select(const float* fG, const float* fD, const int* nbr, int cells,
                    const SelectParams& p, const SelectIO& io, cudaStream_t st);
+// ---- DCGAN (conv_kernels.cu) ---------------------------------------------------------------
+// One grouped implicit-GEMM problem. CONV / CONVT forward: a = input [n][ca][2^lha][2^lwa],
+// b = weights of individual 0 (+ wsel[wsel_idx] * wsel_stride; a launch may pass its own wsel
+// table), out = [n][co][2^lho][2^lwo], aux = the activation whose derivative the epilogue
+// applies (shaped like out). Weight gradient: a = [n][ca][2^lha][2^lwa], b = the gathered
+// operand [n][co][2^lho][2^lwo], out = fp32 [ca][co * 16].
+struct ConvDesc {
+  const void* a;
+  const void* b;
+  const int* wsel;
+  int64_t wsel_stride;
+  int wsel_idx;
+  void* out;
+  const void* aux;
+  int n, ca, lha, lwa, co, lho, lwo, s, p;
+};
+// Training-mode batch normalisation + ReLU of one problem: c = fp32 conv output
+// [n][C][2^lhw], h = activation out, mean / inv [C]; parameters (gamma at off_gamma, beta at
+// off_beta) of individual wsel[wsel_idx] in params (fp32 masters, stride wsel_stride).
+// Backward: dh = fp32 dL/dh, dc = dL/dc out, dparams = this cell's gradient vector.
+struct BnDesc {
+  const float* c;
+  void* h;
+  float* mean;
+  float* inv;
+  const float* params;
+  const int* wsel;
+  int64_t wsel_stride;
+  int wsel_idx;
+  int64_t off_gamma, off_beta;
+  int n, C, lhw;
+  const float* dh;
+  void* dc;
+  float* dparams;
+};
+// Discriminator output layer: a [rows][K] activations, w the weights (individual 0 + wsel),
+// logits [rows] out; backward: dl [rows] in, da [rows][K] out (or null), dw [K] out.
+struct LogitDesc {
+  const void* a;
+  const void* w;
+  const int* wsel;
+  int64_t wsel_stride;
+  int wsel_idx;
+  float* logits;
+  int rows, K;
+  const void* dl;
+  void* da;
+  float* dw;
+};
+enum { CONV_FWD_MODE = 0, CONVT_FWD_MODE = 1, WGRAD_MODE = 2 };
+enum { CEPI_NONE_ = 0, CEPI_LRELU_ = 1, CEPI_TANH_ = 2, CEPI_DLRELU_ = 3, CEPI_DTANH_ = 4 };
+void launch_conv(int mode, int epi, bool bf, bool out_f32, const ConvDesc* descs,
+                 int n_problems, int max_m, int max_n, const int* wsel, int splits, float* part,
+                 int64_t part_stride, float slope, cudaStream_t st);
+void launch_bn_relu(bool bf, const BnDesc* descs, int n_problems, int channels, const int* wsel,
+                    cudaStream_t st);
+void launch_bn_relu_backward(bool bf, const BnDesc* descs, int n_problems, int channels,
+                             cudaStream_t st);
+void launch_logit_dot(bool bf, const LogitDesc* descs, int n_problems, int max_rows,
+                      const int* wsel, cudaStream_t st);
+void launch_dc_dlogit(bool bf, const float* logits, int cells, int B, void* dl_d, void* dl_g,
+                      cudaStream_t st);
+void launch_logit_back(bool bf, const LogitDesc* descs, int n_problems, int K, bool with_dw,
+                       float slope, cudaStream_t st);
+
 // Generator-mixture score and ES-(1+1) step (rows = 6B evaluation rows per cell).
 template <typename T>
 void launch_row_norms(const T* E, int64_t e_cell, int cells, int rows, int x, float* out,

@@ -7,8 +7,10 @@
 namespace lipz {
 
 // ------------------------------------------------------------------------------------------
-// Step 1: Xavier-uniform weights. Element k of the flat vector takes word k of the
-// (stream, 0, individual) sequence; s = word >> 8; q = (2 s + 1 - 2^24) 2^-24; w = a q.
+// Step 1: random weights. Element k of the flat vector takes word k of the
+// (stream, 0, individual) sequence: Xavier-uniform tensors s = word >> 8,
+// q = (2 s + 1 - 2^24) 2^-24, w = a q; normal tensors take normal k (Box-Muller on the two
+// words of block k / 4 that pair with it), w = a n or 1 + a n.
 // ------------------------------------------------------------------------------------------
 __global__ void k_init_params(float* __restrict__ w, bf16* __restrict__ wb, int64_t P,
                               int64_t Ps, Layout lay, uint64_t seed, uint32_t stream) {
@@ -26,9 +28,16 @@ __global__ void k_init_params(float* __restrict__ w, bf16* __restrict__ wb, int6
       int t = 0;
       while (t + 1 < lay.n && k >= lay.off[t + 1]) ++t;
       const float a = lay.bound[t];
-      if (a != 0.f) {
-        const float q = (float)(2 * (int32_t)(words[e] >> 8) + 1 - (1 << 24)) * 5.9604644775390625e-8f;
-        v = a * q;
+      if (lay.init[t] == INIT_UNIFORM) {
+        if (a != 0.f) {
+          const float q =
+              (float)(2 * (int32_t)(words[e] >> 8) + 1 - (1 << 24)) * 5.9604644775390625e-8f;
+          v = a * q;
+        }
+      } else {
+        const float2 nn = e < 2 ? box_muller(r.x, r.y) : box_muller(r.z, r.w);
+        const float n = (e & 1) ? nn.y : nn.x;
+        v = lay.init[t] == INIT_NORMAL ? a * n : 1.f + a * n;
       }
     }
     w[(int64_t)cell * Ps + k] = v;

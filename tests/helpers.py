@@ -16,7 +16,9 @@ def oracle_arch(arch) -> O.Arch:
                   lr_mut_prob=float(arch.lr_mut_prob), leaky_slope=float(arch.leaky_slope),
                   train_steps=int(arch.train_steps), mixture=bool(arch.mixture),
                   mix_sigma=float(arch.mix_sigma),
-                  stale_neighbors=bool(arch.stale_neighbors))
+                  stale_neighbors=bool(arch.stale_neighbors),
+                  kind="dcgan" if arch.kind == 1 else "mlp", ngf=int(arch.ngf),
+                  ndf=int(arch.ndf))
 
 
 def max_rel(got, ref) -> float:
