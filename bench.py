@@ -9,12 +9,13 @@ one full grid iteration (minibatch draw, all-pairs evaluation, fitness, selectio
 Adam of every cell's new centre pair).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--train-steps S] [--mixture] [--stale-neighbors]
+                  [--train-steps S] [--mixture] [--stale-neighbors] [--dcgan]
 
 With --train-steps S > 1 every iteration trains each cell's new centre pair S times (the later
 steps on fresh minibatches); the default S = 1 is the headline workload. --mixture adds the
 generator-mixture ES-(1+1) step (Gaussian-kernel MMD score) to every evaluation;
---stale-neighbors runs the asynchronous schedule (neighbours one iteration late).
+--stale-neighbors runs the asynchronous schedule (neighbours one iteration late). --dcgan
+times the 3x3 DCGAN configuration (width 64, z = 100, B = 128, bf16) instead of the MLP.
 
 With N > 1 (torchrun, one process per GPU) every rank runs its own 12x12 grid (replicas: the
 per-GPU work is fixed, scaling "weak"); value = all ranks' pairs / the slowest rank's time.
@@ -380,7 +381,150 @@ def cpu_baseline(seconds):
                       "gradients + Adam per cell), %.1f s, numpy float64 + OpenBLAS" % (done, el)}
 
 
+# ---- DCGAN workload (the 3x3 DCGAN configuration: width 64, z = 100, B = 128, bf16) --------
+DC_ROWS, DC_COLS, DC_B, DC_Z, DC_W, DC_POOL = 3, 3, 128, 100, 64, 2000
+DC_CELLS = DC_ROWS * DC_COLS
+DC_PAIRS = 25 * DC_CELLS
+DC_WORKLOAD = ("3x3 torus DCGAN G/D (512/256/128/64 channels, 64x64x3) bf16 B=128 "
+               "(225 pairs/iter)")
+
+
+def _dc_macs():
+    """Algorithmic multiply-adds per sample: generator (transposed convolutions) and
+    discriminator (convolutions), each layer H_in W_in C_in C_out 16 for the generator and
+    H_out W_out C_in C_out 16 for the discriminator."""
+    g, d, z = DC_W, DC_W, DC_Z
+    gm = z * 8 * g * 16 + 16 * 8 * g * 4 * g * 16 + 64 * 4 * g * 2 * g * 16 \
+        + 256 * 2 * g * g * 16 + 1024 * g * 3 * 16
+    dm = 1024 * d * 3 * 16 + 256 * 2 * d * d * 16 + 64 * 4 * d * 2 * d * 16 \
+        + 16 * 8 * d * 4 * d * 16 + 8 * d * 16
+    return gm, dm
+
+
+def run_dcgan(args):
+    """The DCGAN grid iteration on the CUDA-core kernels: device time per iteration, phases
+    against the fp32 FMA rate, end to end with host minibatches, and the oracle's rate."""
+    import numpy as np
+    import torch
+    dist, rank, world = _dist()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import lipz_synth
+    import paper_1811_12843_gb300 as L
+    pool = lipz_synth.field_pool(SEED, n=DC_POOL)
+    g = L.Grid(DC_ROWS, DC_COLS, seed=SEED + rank, precision="bf16", batch=DC_B, kind=1,
+               x_dim=12288, z_dim=DC_Z, ngf=DC_W, ndf=DC_W, lr=5e-5,
+               stale_neighbors=1 if args.stale_neighbors else 0,
+               mixture=1 if args.mixture else 0)
+    g.set_data(pool)
+    stream = torch.cuda.Stream()
+    g.set_stream(stream.cuda_stream)
+    for _ in range(args.warmup):
+        L.lipz_iterate(g.h, 1)
+    g.synchronize()
+    L.lipz_profile_read(g.h)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    with Clocks(local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            L.lipz_iterate(g.h, 1)
+        e1.record(stream)
+        g.synchronize()
+    if dist:
+        dist.barrier()
+    ms = allreduce_max(dist, e0.elapsed_time(e1))
+    launches = sum(v[2] for v in L.lipz_profile_read(g.h).values())
+    ms_step = ms / args.steps
+    value = DC_PAIRS * world * 1000.0 / ms_step
+    L.lipz_profile_enable(g.h, True)
+    for _ in range(max(2, args.steps // 2)):
+        L.lipz_iterate(g.h, 1)
+    prof = L.lipz_profile_read(g.h)
+    L.lipz_profile_enable(g.h, False)
+    phase_ms = {k: v[0] / max(v[1], 1) for k, v in prof.items()}
+    # end to end: pinned host minibatches in, fitness out
+    xs = [torch.from_numpy(pool[np.random.default_rng(i).integers(0, DC_POOL, DC_CELLS * DC_B)]
+                           .reshape(DC_CELLS, DC_B, 12288)).pin_memory() for i in range(2)]
+    fg = torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory()
+    fd = torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory()
+    L.lipz_iterate_batch(g.h, xs[0], fg, fd)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    n_e2e = max(2, args.steps // 2)
+    for i in range(n_e2e):
+        L.lipz_iterate_batch(g.h, xs[i % 2], fg, fd)
+    e2e = DC_PAIRS * world * n_e2e / allreduce_max(dist, time.perf_counter() - t0)
+    if rank != 0:
+        return None
+    hbm, tf_burst, tf_sus, kind = _peaks()
+    # CUDA-core fp32 rate: 152 SMs x 128 FMA lanes x 2 FLOP x the sampled SM clock
+    mhz = clk.summary().get("sm_mhz") or 2070.0
+    alu_peak = 152 * 128 * 2 * mhz * 1e6 / 1e12
+    gm, dm = _dc_macs()
+    work = {"g_fwd": 2.0 * DC_CELLS * 5 * DC_B * gm, "d_fwd": 2.0 * DC_CELLS * 30 * DC_B * dm,
+            "train_bwd": 2.0 * DC_CELLS * DC_B * (3 * gm + 7 * dm)}
+    roofs = {}
+    for ph, flop in work.items():
+        t = phase_ms.get(ph)
+        if t and t == t:
+            ach = flop / (t * 1e-3) / 1e12
+            roofs[ph] = {"bound": "alu", "achieved": ach, "peak": alu_peak, "unit": "TFLOP/s",
+                         "frac": ach / alu_peak, "traffic": None, "algorithmic_flop": flop,
+                         "peak_source": "fp32 FMA lanes x sampled SM clock",
+                         "frac_of_bf16_tensor": ach / tf_sus}
+    dom = max(roofs, key=lambda k: phase_ms[k])
+    roof = dict(roofs[dom], phase=dom)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded smooth Gaussian random fields, 3x64x64, standing in for "
+                "CelebA)",
+        "config": {"workload": _workload(args), "rows": DC_ROWS, "cols": DC_COLS,
+                   "global_batch": DC_B, "pairs_per_iter": DC_PAIRS,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (population and activations, several GB)"},
+        "grid_iterations_per_sec": 1000.0 * world / ms_step,
+        "phase_ms": phase_ms, "roofline": roof, "phase_rooflines": roofs,
+        "e2e": {"value": e2e, "unit": UNIT, "h2d_bytes_per_step": DC_CELLS * DC_B * 12288 * 4,
+                "d2h_bytes_per_step": 2 * DC_CELLS * 5 * 4},
+        "gpu_launches": launches, "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        done, el = _dc_oracle_sample()
+        line["cpu_baseline"] = {"value": 25.0 * done / el, "unit": UNIT, "cores": _threads(),
+                                "kind": "oracle",
+                                "sample": "%d cell(s) of the 3x3 DCGAN workload (evaluation of "
+                                          "25 pairs), %.1f s" % (done, el)}
+    return line
+
+
+def _dc_oracle_sample(cells=1):
+    import lipz_synth
+    from oracle import lipz_oracle as O
+    pool = lipz_synth.field_pool(SEED, n=DC_POOL)
+    a = O.Arch(kind="dcgan", precision="bf16", batch=DC_B, z_dim=DC_Z, x_dim=12288, ngf=DC_W,
+               ndf=DC_W)
+    s = O.create(DC_ROWS, DC_COLS, a, SEED)
+    t0 = time.perf_counter()
+    for c in range(cells):
+        O.eval_neighborhoods(s, O.batches(s, pool, cells=[c]), cells=[c])
+    return cells, time.perf_counter() - t0
+
+
 def _workload(args):
+    if getattr(args, "dcgan", False):
+        w = DC_WORKLOAD
+        if args.stale_neighbors:
+            w += ", stale neighbours"
+        if args.mixture:
+            w += ", mixture ES step"
+        return w
     w = WORKLOAD
     if args.train_steps != 1:
         w += ", %d minibatch steps per iteration" % args.train_steps
@@ -389,6 +533,30 @@ def _workload(args):
     if args.stale_neighbors:
         w += ", stale neighbours"
     return w
+
+
+def run_reference_dcgan(args):
+    """The oracle on the DCGAN workload: each step evaluates one cell's 25 pairs."""
+    _, rank, world = _dist()
+    if rank != 0:
+        return None
+    total, el = 0, 0.0
+    for _ in range(args.steps):
+        d, e = _dc_oracle_sample()
+        total += d
+        el += e
+    value = 25.0 * total / el
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded smooth Gaussian random fields, 3x64x64)",
+            "config": {"workload": _workload(args), "rows": DC_ROWS, "cols": DC_COLS,
+                       "global_batch": DC_B, "pairs_per_iter": DC_PAIRS, "parallelism": "cpu"},
+            "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+                             "sample": "1 cell per step of the 3x3 DCGAN workload"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
 
 
 def run_reference(args):
@@ -442,10 +610,17 @@ def main():
                     help="add the generator-mixture ES step to every iteration")
     ap.add_argument("--stale-neighbors", action="store_true",
                     help="neighbours seen one iteration late (asynchronous cells)")
+    ap.add_argument("--dcgan", action="store_true",
+                    help="the 3x3 DCGAN workload (CUDA-core convolutions) instead of the MLP")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
-    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if args.dcgan and args.impl == "reference":
+        line = run_reference_dcgan(args)
+    elif args.dcgan:
+        line = run_dcgan(args)
+    else:
+        line = run_reference(args) if args.impl == "reference" else run_ours(args)
     if line is not None:
         print(json.dumps(line), flush=True)
 
