@@ -16,8 +16,13 @@ namespace lipz {
 //              w[c][o][ky][kx]   (terms whose index is fractional or outside the image vanish)
 //   WGRAD:     y[m][c][ky][kx] = sum_{n,i,j} a[n][m][i][j] b[n][c][s i - p + ky][s j - p + kx]
 //              (split over K = n * Ha * Wa; partial sums reduced in a fixed order)
+//   CONVT2:    CONVT_FWD at stride 2 by output parity class (i mod 2, j mod 2), one class per
+//              block (blockIdx.z = problem * 4 + class): only the taps ky = (i + p) mod 2 + 2 u,
+//              kx = (j + p) mod 2 + 2 v (u, v in {0, 1}) reach a pixel of the class, so K is
+//              4 per input channel instead of 16
 // ------------------------------------------------------------------------------------------
-enum { CONV_FWD = CONV_FWD_MODE, CONVT_FWD = CONVT_FWD_MODE, WGRAD = WGRAD_MODE };
+enum { CONV_FWD = CONV_FWD_MODE, CONVT_FWD = CONVT_FWD_MODE, WGRAD = WGRAD_MODE,
+       CONVT2 = CONVT2_MODE };
 enum { CEPI_NONE = CEPI_NONE_, CEPI_LRELU = CEPI_LRELU_, CEPI_TANH = CEPI_TANH_,
        CEPI_DLRELU = CEPI_DLRELU_, CEPI_DTANH = CEPI_DTANH_ };
 
@@ -26,6 +31,10 @@ __device__ __forceinline__ void conv_dims(const ConvDesc& d, int mode, int& M, i
     M = d.ca;
     N = d.co * 16;
     K = d.n << (d.lha + d.lwa);
+  } else if (mode == CONVT2) {
+    M = d.n << (d.lho + d.lwo - 2);
+    N = d.co;
+    K = d.ca * 4;
   } else {
     M = d.n << (d.lho + d.lwo);
     N = d.co;
@@ -67,6 +76,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
   const int Ha = 1 << d.lha, Wa = 1 << d.lwa;
+  // CONVT2: this block's output class and its first taps
+  const int py = (split >> 1) & 1, px = split & 1;
+  const int ky0 = (py + d.p) & 1, kx0 = (px + d.p) & 1;
+  const int lqy = d.lho - 1, lqx = d.lwo - 1;
   for (int k0 = kb; k0 < ke; k0 += 16) {
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -80,6 +93,14 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
           if (MODE == WGRAD) {
             const int nb = k >> (d.lha + d.lwa), yx = k & ((1 << (d.lha + d.lwa)) - 1);
             v = to_f<TI>(A[(((int64_t)nb * d.ca + m) << (d.lha + d.lwa)) + yx]);
+          } else if (MODE == CONVT2) {
+            const int nb = m >> (lqy + lqx);
+            const int oy = 2 * ((m >> lqx) & ((1 << lqy) - 1)) + py;
+            const int ox = 2 * (m & ((1 << lqx) - 1)) + px;
+            const int c = k >> 2, ky = ky0 + 2 * ((k >> 1) & 1), kx = kx0 + 2 * (k & 1);
+            const int iy = (oy + d.p - ky) >> 1, ix = (ox + d.p - kx) >> 1;
+            if (oy + d.p - ky >= 0 && ox + d.p - kx >= 0 && iy < Ha && ix < Wa)
+              v = to_f<TI>(A[(((int64_t)nb * d.ca + c) << (d.lha + d.lwa)) + (iy << d.lwa) + ix]);
           } else {
             const int nb = m >> (d.lho + d.lwo);
             const int oy = (m >> d.lwo) & ((1 << d.lho) - 1), ox = m & ((1 << d.lwo) - 1);
@@ -124,6 +145,9 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
               v = to_f<TI>(Bm[(((int64_t)nb * d.co + c) << (d.lho + d.lwo)) + (by << d.lwo) + bx]);
           } else if (MODE == CONV_FWD) {
             v = to_f<TI>(Bm[(int64_t)n * K + k]);
+          } else if (MODE == CONVT2) {
+            const int ky = ky0 + 2 * ((k >> 1) & 1), kx = kx0 + 2 * (k & 1);
+            v = to_f<TI>(Bm[((int64_t)(k >> 2) * d.co + n) * 16 + ky * 4 + kx]);
           } else {
             v = to_f<TI>(Bm[((int64_t)(k >> 4) * d.co + n) * 16 + (k & 15)]);
           }
@@ -166,7 +190,16 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
   for (int i = 0; i < 4; ++i) {
     const int m = m0 + tm + i;
     if (m >= M) continue;
-    const int nb = m >> (d.lho + d.lwo), yx = m & ((1 << (d.lho + d.lwo)) - 1);
+    int nb, yx;
+    if (MODE == CONVT2) {
+      nb = m >> (lqy + lqx);
+      const int oy = 2 * ((m >> lqx) & ((1 << lqy) - 1)) + py;
+      const int ox = 2 * (m & ((1 << lqx) - 1)) + px;
+      yx = (oy << d.lwo) + ox;
+    } else {
+      nb = m >> (d.lho + d.lwo);
+      yx = m & ((1 << (d.lho + d.lwo)) - 1);
+    }
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int n = n0 + tn + j;
@@ -205,9 +238,11 @@ template <int MODE, typename TI, typename TO, int EPI>
 void launch_conv_t(const ConvDesc* descs, int n_problems, int max_m, int max_n, const int* wsel,
                    int splits, float* part, int64_t part_stride, float slope, cudaStream_t st) {
   if (n_problems <= 0) return;
-  dim3 grid((max_n + 63) / 64, (max_m + 63) / 64, n_problems * (MODE == WGRAD ? splits : 1));
-  launch_pdl(k_conv<MODE, TI, TO, EPI>, grid, dim3(256), 0, st, descs, wsel,
-             MODE == WGRAD ? splits : 1, part, slope);
+  // CONVT2: max_m counts every output pixel; a class holds a quarter of them
+  const int zs = MODE == WGRAD ? splits : (MODE == CONVT2 ? 4 : 1);
+  if (MODE == CONVT2) max_m = (max_m + 3) / 4;
+  dim3 grid((max_n + 63) / 64, (max_m + 63) / 64, n_problems * zs);
+  launch_pdl(k_conv<MODE, TI, TO, EPI>, grid, dim3(256), 0, st, descs, wsel, zs, part, slope);
   if (MODE == WGRAD)
     launch_pdl(k_wgrad_reduce, dim3(64, n_problems), dim3(256), 0, st, descs, splits,
                (const float*)part, part_stride);
@@ -224,6 +259,21 @@ void launch_conv(int mode, int epi, bool bf, bool out_f32, const ConvDesc* descs
   if (mode == WGRAD) {
     if (bf) LIPZ_CONV(WGRAD, bf16, float, CEPI_NONE);
     else LIPZ_CONV(WGRAD, float, float, CEPI_NONE);
+    return;
+  }
+  if (mode == CONVT2) {
+    if (bf) {
+      if (out_f32) LIPZ_CONV(CONVT2, bf16, float, CEPI_NONE);
+      else if (epi == CEPI_TANH) LIPZ_CONV(CONVT2, bf16, bf16, CEPI_TANH);
+      else if (epi == CEPI_DLRELU) LIPZ_CONV(CONVT2, bf16, bf16, CEPI_DLRELU);
+      else if (epi == CEPI_DTANH) LIPZ_CONV(CONVT2, bf16, bf16, CEPI_DTANH);
+      else LIPZ_CONV(CONVT2, bf16, bf16, CEPI_NONE);
+    } else {
+      if (epi == CEPI_TANH) LIPZ_CONV(CONVT2, float, float, CEPI_TANH);
+      else if (epi == CEPI_DLRELU) LIPZ_CONV(CONVT2, float, float, CEPI_DLRELU);
+      else if (epi == CEPI_DTANH) LIPZ_CONV(CONVT2, float, float, CEPI_DTANH);
+      else LIPZ_CONV(CONVT2, float, float, CEPI_NONE);
+    }
     return;
   }
   if (bf) {

@@ -471,7 +471,8 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int gs[6] = {1, 4, 8, 16, 32, 64};
   const int PE = C * 5;
   for (int l = 1; l <= 5; ++l) {
-    launch_conv(CONVT_FWD_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->eg[l - 1], PE,
+    launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
+                l < 5, p->eg[l - 1], PE,
                 B * gs[l] * gs[l], gc[l], nbr, 1, nullptr, 0, s.slope, st);
     if (l <= 4) launch_bn_relu(s.bf, p->ebn[l - 1], PE, gc[l], nbr, st);
   }
@@ -503,7 +504,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   const int ds[5] = {64, 32, 16, 8, 4};
   // forward of the selected pair
   for (int l = 1; l <= 5; ++l) {
-    launch_conv(CONVT_FWD_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->tg[l - 1], C,
+    launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
+                l < 5, p->tg[l - 1], C,
                 B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0, s.slope, st);
     if (l <= 4) launch_bn_relu(s.bf, p->tbn[l - 1], C, gc[l], nullptr, st);
   }
@@ -525,14 +527,14 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
                 nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
     if (l >= 2)
-      launch_conv(CONVT_FWD_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
+      launch_conv(CONVT2_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
                   2 * B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0, s.slope,
                   st);
   }
   // the generator loss through the discriminator
   launch_logit_back(s.bf, p->tdl_back_g, C, (int)(8 * d * 16), false, s.slope, st);
   for (int l = 4; l >= 1; --l)
-    launch_conv(CONVT_FWD_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
+    launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
                 p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
                 s.slope, st);
   // generator backward
