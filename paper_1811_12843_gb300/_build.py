@@ -19,7 +19,7 @@ OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "liblipz.so")
 
 SOURCES = ["api.cu", "simt_kernels.cu", "fwd_tc.cu", "bwd_tc.cu", "noalloc.cu", "conv_kernels.cu",
-           "dcgan.cu"]
+           "dcgan.cu", "conv_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I" + INCLUDE, "-I" + CSRC]

@@ -648,7 +648,7 @@ int create_impl(lipz_grid* g) {
       return rc;
   g->use_tc = !g->dcgan && g->bf && !g->a.force_simt && tc_supported(z, h, x, B);
   if (g->dcgan) {
-    DcShape s{C, B, z, g->a.ngf, g->a.ndf, g->bf, g->a.leaky_slope};
+    DcShape s{C, B, z, g->a.ngf, g->a.ndf, g->bf, g->a.leaky_slope, g->nsnap * C};
     DcBuffers b{};
     b.Gw = g->G[0].w;
     b.Gop = act_w(g->G[0]);
@@ -1112,18 +1112,19 @@ int train_impl(lipz_grid* g) {
 // or a non-finite loss seen since the last check (one synchronisation: all flags are copied
 // into pinned host memory first); the flags are reset.
 int check_flag(lipz_grid* g) {
-  int* dev[7] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
+  int* dev[8] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
                  g->tc[1] ? tc_error_flag(g->tc[1]) : nullptr,
                  g->tc[2] ? tc_error_flag(g->tc[2]) : nullptr,
                  g->tcb[0] ? tcb_error_flag(g->tcb[0]) : nullptr,
                  g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr,
-                 g->tcb[2] ? tcb_error_flag(g->tcb[2]) : nullptr, g->flag};
-  for (int i = 0; i < 7; ++i) {
-    g->hstat[i] = i < 6 ? 0 : INT_MAX;
+                 g->tcb[2] ? tcb_error_flag(g->tcb[2]) : nullptr,
+                 g->dc ? dc_error_flag(g->dc) : nullptr, g->flag};
+  for (int i = 0; i < 8; ++i) {
+    g->hstat[i] = i < 7 ? 0 : INT_MAX;
     if (dev[i]) CK(g, cudaMemcpyAsync(&g->hstat[i], dev[i], 4, cudaMemcpyDeviceToHost, g->st));
   }
   CK(g, cudaStreamSynchronize(g->st));
-  for (int i = 0; i < 6; ++i) {
+  for (int i = 0; i < 7; ++i) {
     const int code = g->hstat[i];
     if (code) {
       CK(g, cudaMemsetAsync(dev[i], 0, 4, g->st));
@@ -1131,7 +1132,7 @@ int check_flag(lipz_grid* g) {
       return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
-  const int v = g->hstat[6];
+  const int v = g->hstat[7];
   if (v != INT_MAX) {
     const int big = INT_MAX;
     int rc = h2d(g, g->flag, &big, 4);

@@ -7,6 +7,8 @@
 
 #include <cuda_bf16.h>
 
+#include "conv_tc.h"
+
 #include <algorithm>
 #include <cstring>
 #include <vector>
@@ -88,6 +90,17 @@ struct DcPlan {
   int splits_dw[4], splits_gw[5];
   int64_t pstride_dw[4], pstride_gw[5];
   int eval_launches, train_launches;
+  // tensor-core discriminator evaluation (bf16, ndf a multiple of 64): weights re-laid out as
+  // [out][ky][kx][in] for every individual, a TMA map per layer, channel-last activations
+  bool tc = false;
+  bf16* Dwt = nullptr;
+  CUtensorMap mW[4];
+  CtcParams cp[4];
+  ConvTcDesc* tcd[4];
+  LogitDesc* tcl;
+  RelayoutD rel;
+  int* err = nullptr;
+  int sms = 148;
 };
 
 namespace {
@@ -440,6 +453,69 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   }
   p->part_floats = part_need;
   ok = ok && !dev_alloc(p, &p->part, (size_t)part_need * 4, msg);
+  // ---- tensor-core discriminator evaluation
+  p->tc = ok && s.bf && d % 64 == 0 && d * 8 <= 512;
+  if (p->tc) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, dev);
+    ok = !dev_alloc(p, &p->Dwt, (size_t)s.n_indiv * b.PDs * 2, msg) &&
+         !dev_alloc(p, &p->err, 4, msg) && ctc_prepare(msg);
+    if (ok) ok = cudaMemset(p->err, 0, 4) == cudaSuccess;
+    for (int l = 0; l < 6; ++l) p->rel.off[l] = dof[l];
+    for (int l = 0; l < 5; ++l) p->rel.ci[l] = dc[l];
+    p->rel.P = dof[5];
+    for (int l = 1; l <= 4 && ok; ++l) {
+      const int ci = dc[l - 1], co = dc[l];
+      const int nbox = co < 256 ? co : 256;
+      ok = ctc_make_map(&p->mW[l - 1], p->Dwt + dof[l - 1], (uint64_t)ci * 16, co, s.n_indiv,
+                        b.PDs, nbox, msg);
+      CtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = 6 * B;
+      q.ci = ci;
+      q.lhi = ilog2(ds[l - 1]);
+      q.co = co;
+      q.lho = ilog2(ds[l]);
+      q.nchw_in = l == 1 ? 1 : 0;
+      q.kchunks = (ci * 16 + 63) / 64;
+      q.nj = (co + 255) / 256;
+      q.nbox = nbox;
+      q.mtiles = ((6 * B << (2 * q.lho)) + 127) / 128;
+      q.n_tiles = 5 * q.mtiles;
+      q.slope = s.slope;
+      q.err = p->err;
+      p->cp[l - 1] = q;
+      std::vector<ConvTcDesc> vt;
+      for (int c = 0; c < C; ++c)
+        for (int sl = 0; sl < 5; ++sl) {
+          void* bx = elw(ex, (int64_t)sl * 6 * B * dmax);
+          void* by = elw(ey, (int64_t)sl * 6 * B * dsz[2]);
+          ConvTcDesc t;
+          memset(&t, 0, sizeof t);
+          t.in = (const bf16*)(l == 1 ? el(b.E, (int64_t)c * b.e_cell) : (l % 2 == 0 ? bx : by));
+          t.out = (bf16*)(l % 2 == 1 ? bx : by);
+          t.wsel_idx = c * 5 + sl;
+          vt.push_back(t);
+        }
+      ok = ok && !upload(p, &p->tcd[l - 1], vt, msg);
+    }
+    std::vector<LogitDesc> vl;
+    for (int c = 0; c < C; ++c)
+      for (int sl = 0; sl < 5; ++sl) {
+        LogitDesc q;
+        memset(&q, 0, sizeof q);
+        q.a = elw(ey, (int64_t)sl * 6 * B * dsz[2]);
+        q.w = p->Dwt + dof[4];
+        q.wsel_stride = b.PDs;
+        q.wsel_idx = c * 5 + sl;
+        q.logits = b.logits + (int64_t)(c * 5 + sl) * 6 * B;
+        q.rows = 6 * B;
+        q.K = (int)dsz[4];
+        vl.push_back(q);
+      }
+    ok = ok && !upload(p, &p->tcl, vl, msg);
+  }
   if (!ok) {
     dc_plan_destroy(p);
     return nullptr;
@@ -484,6 +560,21 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int C = s.cells, B = s.B, d = s.ndf;
   const int dc[5] = {3, d, 2 * d, 4 * d, 8 * d};
   const int ds[5] = {64, 32, 16, 8, 4};
+  if (p->tc) {
+    // weights in the layout the tensor-core convolution reads, for every individual (they
+    // change after every training step)
+    launch_relayout_d((const bf16*)p->b.Dop, p->Dwt, s.n_indiv, p->b.PDs, p->rel, st);
+    for (int c = 0; c < C; ++c) {
+      for (int l = 1; l <= 4; ++l) {
+        CtcParams q = p->cp[l - 1];
+        q.descs = p->tcd[l - 1] + c * 5;
+        q.wsel = nbr;
+        launch_conv_tc(p->mW[l - 1], q, p->sms, st);
+      }
+      launch_logit_dot(true, p->tcl + c * 5, 5, 6 * B, nbr, st);
+    }
+    return check(msg, "DCGAN discriminator evaluation (tensor cores)");
+  }
   for (int c = 0; c < C; ++c) {
     for (int l = 1; l <= 4; ++l)
       launch_conv(CONV_FWD_MODE, CEPI_LRELU_, s.bf, false, p->ed[l - 1] + c * 5, 5,
@@ -552,8 +643,10 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int dc_eval_launches(const DcPlan* p, int part) {
-  return part == 0 ? 9 : p->eval_launches - 9;
+  return part == 0 ? 9 : p->eval_launches - 9 + (p->tc ? 1 : 0);
 }
+
+int* dc_error_flag(DcPlan* p) { return p && p->tc ? p->err : nullptr; }
 int dc_train_launches(const DcPlan* p) { return p->train_launches; }
 
 }  // namespace lipz

@@ -17,6 +17,7 @@ struct DcShape {
   int cells, B, z, ngf, ndf;
   bool bf;      // bf16 operands (population precision), else fp32
   float slope;  // LeakyReLU slope of the discriminator
+  int n_indiv;  // individuals the population arrays hold (snapshots x cells)
 };
 
 // Populations: fp32 masters and the operand copies (bf16, or the fp32 masters) of every
@@ -62,6 +63,10 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg);
 // Forward and backward of every cell's selected pair (src_g, src_d) on the cell's minibatch
 // (real rows of E, noise Z): the gradients into gG and gD.
 int dc_train(DcPlan* p, cudaStream_t st, std::string* msg);
+
+// Device int that a tensor-core kernel of the plan sets when one of its bounded waits expired
+// (null without them); the host reads and clears it.
+int* dc_error_flag(DcPlan* p);
 
 // Kernel launches of dc_eval_g (part 0), dc_eval_d (part 1) and dc_train.
 int dc_eval_launches(const DcPlan* p, int part);

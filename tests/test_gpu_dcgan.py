@@ -71,6 +71,21 @@ def test_dcgan_eval_parity(L, precision, rows, cols, batch, width):
         assert max_rel(ev[k], ref[k]) < tol, k
 
 
+@pytest.mark.parametrize("rows,cols,batch", [(1, 1, 4), (1, 2, 3)])
+def test_dcgan_tensor_core_discriminator_eval(L, rows, cols, batch):
+    """bf16 with a discriminator width that is a multiple of 64 runs the discriminator's
+    evaluation on the tensor-core implicit-GEMM kernel (channel-last activations, re-laid
+    weights): every logit and loss against the oracle."""
+    pool = _field_pool(5, 30)
+    g = _grid(L, rows, cols, 9, pool, precision="bf16", batch=batch, ngf=8, ndf=64)
+    s = _state(g)
+    ref = O.eval_neighborhoods(s, O.batches(s, pool))
+    ev = g.eval(pairs=True)
+    assert max_rel(g.logits(), ref["logits"]) < 2e-2
+    for k in ("LG", "LD", "fG", "fD"):
+        assert max_rel(ev[k], ref[k]) < 2e-2, k
+
+
 @pytest.mark.parametrize("precision", ["fp32", "bf16"])
 def test_dcgan_one_iteration_parity(L, precision):
     """Selection bit-exact given the engine's fitness; then the last step's gradients and the
