@@ -204,7 +204,8 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
     for (int j = 0; j < 4; ++j) {
       const int n = n0 + tn + j;
       if (n >= N) continue;
-      const int64_t o = (((int64_t)nb * d.co + n) << (d.lho + d.lwo)) + yx;
+      const int64_t o = d.nhwc_out ? ((((int64_t)nb << (d.lho + d.lwo)) + yx) * d.co + n)
+                                   : ((((int64_t)nb * d.co + n) << (d.lho + d.lwo)) + yx);
       float v = acc[i][j];
       if (EPI == CEPI_LRELU) v = v > 0.f ? v : slope * v;
       if (EPI == CEPI_TANH) v = tanhf(v);

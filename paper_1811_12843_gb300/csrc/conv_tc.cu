@@ -70,7 +70,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_wait();
-  const int M = p.rows << (2 * p.lho);
+  // output pixels per problem (per parity class when transposed)
+  const int lq = p.lho - p.transposed;
+  const int M = p.rows << (2 * lq);
   const int nbox = p.nbox;
 
   if (warp == 0) {
@@ -80,7 +82,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
-        const ConvTcDesc d = p.descs[tile / p.mtiles];
+        const int pc = tile / p.mtiles;  // problem (x 4 parity classes when transposed)
+        const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
+        const int cls = p.transposed ? (pc & 3) : 0;
         const int indiv = __ldg(&p.wsel[d.wsel_idx]);
         for (int j = 0; j < p.nj && ok; ++j)
           for (int kc = 0; kc < p.kchunks; ++kc) {
@@ -90,7 +94,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             mbar_expect_tx(bFullB + 8 * stage, (uint32_t)(nbox * BK * 2));
             tma_load_3d(base + stage * STAGE_BYTES + A_BYTES, &mW, bFullB + 8 * stage, kc * BK,
-                        j * 256, indiv);
+                        cls * p.cls_rows + j * 256, indiv);
             issued[stage]++;
             if (++stage == STAGES) {
               stage = 0;
@@ -157,11 +161,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     bool ok = true;
     const int lhi = p.lhi, Hi = 1 << lhi;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
-      const ConvTcDesc d = p.descs[tile / p.mtiles];
+      const int pc = tile / p.mtiles;
+      const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
+      const int cls = p.transposed ? (pc & 3) : 0;
       const int m = (tile % p.mtiles) * BM + r;
       const bool valid = m < M;
-      const int nb = m >> (2 * p.lho), oy = (m >> p.lho) & ((1 << p.lho) - 1),
-                ox = m & ((1 << p.lho) - 1);
+      const int nb = m >> (2 * lq);
+      int oy = (m >> lq) & ((1 << lq) - 1), ox = m & ((1 << lq) - 1);
+      if (p.transposed) {
+        oy = 2 * oy + (cls >> 1);
+        ox = 2 * ox + (cls & 1);
+      }
       for (int j = 0; j < p.nj && ok; ++j)
         for (int kc = 0; kc < p.kchunks; ++kc) {
           if (!mbar_wait_warp(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 27)) {
@@ -197,11 +207,25 @@ __global__ void __launch_bounds__(THREADS, 1)
                            : "memory");
             }
           } else {
-            // channel-last input with ci a multiple of 64: one tap, 64 channels per chunk
+            // channel-last input with ci a multiple of 64: one tap, 64 channels per chunk.
+            // Convolution: tap (ky, kx) of 16, input pixel (2 oy - 1 + ky, 2 ox - 1 + kx).
+            // Transposed (stride 2, pad 1, by class): tap (u, v) of 4, ky = (oy + 1) mod 2 + 2u,
+            // input pixel ((oy + 1 - ky) / 2, (ox + 1 - kx) / 2).
             const int k0 = kc * BK;
             const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
-            const int iy = 2 * oy - 1 + (tap >> 2), ix = 2 * ox - 1 + (tap & 3);
-            const bool in = valid && iy >= 0 && iy < Hi && ix >= 0 && ix < Hi;
+            int iy, ix, ty = 0, tx = 0;
+            if (p.transposed) {
+              const int ky = ((oy + 1) & 1) + 2 * (tap >> 1), kx = ((ox + 1) & 1) + 2 * (tap & 1);
+              ty = oy + 1 - ky;
+              tx = ox + 1 - kx;
+              iy = ty >> 1;
+              ix = tx >> 1;
+            } else {
+              iy = 2 * oy - 1 + (tap >> 2);
+              ix = 2 * ox - 1 + (tap & 3);
+            }
+            const bool in = valid && ty >= 0 && tx >= 0 && iy >= 0 && iy < Hi && ix >= 0 &&
+                            ix < Hi;
             const uint4* src = reinterpret_cast<const uint4*>(
                 d.in + ((((int64_t)nb << (2 * lhi)) + (iy << lhi) + ix) * p.ci + c0));
 #pragma unroll
@@ -229,9 +253,19 @@ __global__ void __launch_bounds__(THREADS, 1)
     int uses[2] = {0, 0}, jobs = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
-      const ConvTcDesc d = p.descs[tile / p.mtiles];
+      const int pc = tile / p.mtiles;
+      const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
+      const int cls = p.transposed ? (pc & 3) : 0;
       const int m = (tile % p.mtiles) * BM + row;
       const bool valid = m < M;
+      const int nb = m >> (2 * lq);
+      int oy = (m >> lq) & ((1 << lq) - 1), ox = m & ((1 << lq) - 1);
+      if (p.transposed) {
+        oy = 2 * oy + (cls >> 1);
+        ox = 2 * ox + (cls & 1);
+      }
+      // output pixel index in the problem's image stack
+      const int64_t pix = ((int64_t)nb << (2 * p.lho)) + (oy << p.lho) + ox;
       for (int j = 0; j < p.nj && ok; ++j, ++jobs) {
         const int R = jobs & 1;
         if (!mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 28)) {
@@ -239,23 +273,46 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
-        for (int g = 0; g < nbox / 32; ++g) {
-          uint32_t v[32];
-          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
+        if (p.out_mode == CTC_TANH_CHW) {
+          // a few output channels (the image's colours): tanh, bf16, channel-major images
+          uint32_t v[16];
+          LIPZ_TMEM_LD16(tmem + lane_base + (uint32_t)(R * 256), v);
           tmem_wait_ld();
-          uint32_t pk[16];
 #pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
-            a = a > 0.f ? a : p.slope * a;
-            b = b > 0.f ? b : p.slope * b;
-            pk[e >> 1] = pack_bf16(a, b);
-          }
-          if (valid) {
-            uint4* o = reinterpret_cast<uint4*>(d.out + (int64_t)m * p.co + j * 256 + g * 32);
+          for (int e = 0; e < 16; ++e)
+            if (valid && e < p.co)
+              d.out[(((int64_t)nb * p.co + e) << (2 * p.lho)) + (oy << p.lho) + ox] =
+                  __float2bfloat16_rn(tanhf(__uint_as_float(v[e])));
+        } else {
+          for (int g = 0; g < nbox / 32; ++g) {
+            uint32_t v[32];
+            LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
+            tmem_wait_ld();
+            if (p.out_mode == CTC_F32_HWC) {
+              if (valid) {
+                float4* o = reinterpret_cast<float4*>(reinterpret_cast<float*>(d.out) +
+                                                      pix * p.co + j * 256 + g * 32);
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-              o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 8; ++u)
+                  o[u] = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
+                                     __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
+              }
+              continue;
+            }
+            uint32_t pk[16];
+#pragma unroll
+            for (int e = 0; e < 32; e += 2) {
+              float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
+              a = a > 0.f ? a : p.slope * a;
+              b = b > 0.f ? b : p.slope * b;
+              pk[e >> 1] = pack_bf16(a, b);
+            }
+            if (valid) {
+              uint4* o = reinterpret_cast<uint4*>(d.out + pix * p.co + j * 256 + g * 32);
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+            }
           }
         }
         tc_fence_before();
@@ -291,7 +348,95 @@ __global__ void k_relayout_d(const bf16* __restrict__ src, bf16* __restrict__ ds
   }
 }
 
+// Generator transposed-convolution weights [in][out][ky][kx] -> by output parity class
+// [class][out][tap][in] (tap (u, v): ky = (py + 1) mod 2 + 2u, kx = (px + 1) mod 2 + 2v), rows
+// of a class cls_rows apart (the padding rows are left as they are: zero).
+__global__ void k_relayout_g(const bf16* __restrict__ src, int64_t src_ps, bf16* __restrict__ dst,
+                             int64_t dst_ps, int n_indiv, RelayoutG r) {
+  pdl_wait();
+  int64_t total = 0;
+  for (int l = 0; l < r.n; ++l) total += (int64_t)r.ci[l] * r.co[l] * 16;
+  total *= n_indiv;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    int64_t per = 0;
+    for (int l = 0; l < r.n; ++l) per += (int64_t)r.ci[l] * r.co[l] * 16;
+    const int64_t ind = e / per;
+    int64_t k = e - ind * per;
+    int l = 0;
+    while (k >= (int64_t)r.ci[l] * r.co[l] * 16) {
+      k -= (int64_t)r.ci[l] * r.co[l] * 16;
+      ++l;
+    }
+    const int ci = r.ci[l], co = r.co[l];
+    // destination k = ((cls * co + o) * 4 + t) * ci + c
+    const int c = (int)(k % ci), t = (int)((k / ci) & 3);
+    const int o = (int)((k / (4 * ci)) % co), cls = (int)(k / (4 * (int64_t)ci * co));
+    const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1), kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
+    dst[ind * dst_ps + r.dst_off[l] + (((int64_t)cls * r.cls_rows[l] + o) * 4 + t) * ci + c] =
+        src[ind * src_ps + r.src_off[l] + (((int64_t)c * co + o) * 4 + ky) * 4 + kx];
+  }
+}
+
+// Training-mode batch normalisation + ReLU on channel-last data: block (channel group of 32,
+// problem); warp w takes pixels w, w + 8, ...; lane = channel; fixed-order reductions.
+__global__ void __launch_bounds__(256) k_bn_relu_hwc(const BnDesc* __restrict__ descs,
+                                                     const int* __restrict__ wsel_override) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int ch = blockIdx.x * 32 + (threadIdx.x & 31);
+  const int w = threadIdx.x >> 5;
+  const int64_t m = (int64_t)d.n << d.lhw;
+  __shared__ float sh[8][32];
+  const bool on = ch < d.C;
+  float s = 0.f;
+  if (on)
+    for (int64_t px = w; px < m; px += 8) s += d.c[px * d.C + ch];
+  sh[w][threadIdx.x & 31] = s;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) tot += sh[i][threadIdx.x & 31];
+  const float mean = tot / (float)m;
+  __syncthreads();
+  float v = 0.f;
+  if (on)
+    for (int64_t px = w; px < m; px += 8) {
+      const float t = d.c[px * d.C + ch] - mean;
+      v = fmaf(t, t, v);
+    }
+  sh[w][threadIdx.x & 31] = v;
+  __syncthreads();
+  float vt = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) vt += sh[i][threadIdx.x & 31];
+  if (!on) return;
+  const float inv = rsqrtf(vt / (float)m + 1e-5f);
+  if (w == 0) {
+    d.mean[ch] = mean;
+    d.inv[ch] = inv;
+  }
+  const int* ws = wsel_override ? wsel_override : d.wsel;
+  const float* P = d.params + (ws ? (int64_t)ws[d.wsel_idx] * d.wsel_stride : 0);
+  const float g = P[d.off_gamma + ch], b = P[d.off_beta + ch];
+  bf16* h = (bf16*)d.h;
+  for (int64_t px = w; px < m; px += 8)
+    h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(g * inv, d.c[px * d.C + ch] - mean, b), 0.f));
+}
+
 }  // namespace ctc
+
+void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
+                       const RelayoutG& r, cudaStream_t st) {
+  launch_pdl(ctc::k_relayout_g, dim3(1216), dim3(256), 0, st, src, src_ps, dst, dst_ps, n_indiv,
+             r);
+}
+
+void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
+                        cudaStream_t st) {
+  launch_pdl(ctc::k_bn_relu_hwc, dim3((channels + 31) / 32, n_problems), dim3(256), 0, st, descs,
+             wsel);
+}
 
 namespace {
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_ctc = nullptr;

@@ -26,12 +26,28 @@ struct ConvTcDesc {
 // squared to co x 2^lho squared; K = 16 ci in (ky, kx, ci) order, kchunks = ceil(K / 64);
 // jobs of nbox = min(co, 256) output channels (nj of them); tiles of 128 output pixels
 // (mtiles per problem). The weight map spans [individual][co][K] bf16.
+// transposed: a stride-2 / pad-1 transposed convolution computed by output parity class (tiles
+// over problem x 4 classes x mtiles; K = 4 ci in (tap, ci) order; the weights of class cls
+// start at row cls * cls_rows of the map). out_mode: CTC_LRELU_HWC (bf16 LeakyReLU,
+// channel-last), CTC_F32_HWC (fp32 raw, channel-last), CTC_TANH_CHW (bf16 tanh, channel-major
+// images; co <= 16).
+enum { CTC_LRELU_HWC = 0, CTC_F32_HWC = 1, CTC_TANH_CHW = 2 };
 struct CtcParams {
   const ConvTcDesc* descs;
   int rows, ci, lhi, co, lho, nchw_in, kchunks, nj, nbox, mtiles, n_tiles;
+  int transposed, out_mode, cls_rows;
   const int* wsel;
   float slope;
   int* err;
+};
+
+// Generator layers 2..5 (n of them): source offsets and sizes [in = ci][out = co][4][4];
+// destination offsets (per individual, stride dst_ps) of the class-major copies with
+// cls_rows rows per class.
+struct RelayoutG {
+  int n;
+  int64_t src_off[4], dst_off[4];
+  int ci[4], co[4], cls_rows[4];
 };
 
 // Offsets and input channels of the five discriminator tensors inside one individual (P its
@@ -48,5 +64,11 @@ bool ctc_prepare(std::string* msg);
 void launch_conv_tc(const CUtensorMap& mW, const CtcParams& p, int sms, cudaStream_t st);
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,
                        cudaStream_t st);
+void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
+                       const RelayoutG& r, cudaStream_t st);
+// Batch normalisation (training mode) + ReLU on fp32 channel-last input into bf16 channel-last
+// output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels).
+void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
+                        cudaStream_t st);
 
 }  // namespace lipz

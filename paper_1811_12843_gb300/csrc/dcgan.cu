@@ -101,6 +101,15 @@ struct DcPlan {
   RelayoutD rel;
   int* err = nullptr;
   int sms = 148;
+  // tensor-core generator evaluation (bf16, ngf a multiple of 64): layers 2-5 by parity class
+  // from class-major weight copies, channel-last activations and batch norm
+  bool tcg = false;
+  bf16* Gwt = nullptr;
+  int64_t gwt_ps = 0;
+  RelayoutG relg;
+  CUtensorMap mG[4];
+  CtcParams gp[4];
+  ConvTcDesc* gtd[4];
 };
 
 namespace {
@@ -185,6 +194,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     doffs[l] = doffs[l - 1] + dsz[l - 1];
   }
   const int PE = C * 5;
+  p->tcg = s.bf && g % 64 == 0;
   // ---- buffers
   float *ec, *emean, *einv, *tc, *tmean, *tinv, *dh;
   void *eh, *ex, *ey, *th, *ta, *P, *Q, *P2, *Q2, *dcb, *d5;
@@ -256,6 +266,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
                            l == 1 ? 0 : 1, out);
         q.wsel_stride = b.PGs;
         q.wsel_idx = pr;
+        q.nhwc_out = (p->tcg && l == 1) ? 1 : 0;
         v.push_back(q);
         if (l <= 4)
           vb.push_back(bn(ec + (int64_t)pr * B * gmax, elw(eh, (int64_t)pr * B * gmax),
@@ -516,6 +527,70 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       }
     ok = ok && !upload(p, &p->tcl, vl, msg);
   }
+  // ---- tensor-core generator evaluation (layers 2-5)
+  if (ok && p->tcg) {
+    if (!p->tc) {
+      int dev = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, dev);
+      ok = !dev_alloc(p, &p->err, 4, msg) && ctc_prepare(msg) &&
+           cudaMemset(p->err, 0, 4) == cudaSuccess;
+    }
+    RelayoutG& r = p->relg;
+    memset(&r, 0, sizeof r);
+    r.n = 4;
+    int64_t off = 0;
+    for (int i = 0; i < 4; ++i) {
+      const int l = i + 2;
+      r.src_off[i] = go[3 * (l - 1)];
+      r.ci[i] = gc[l - 1];
+      r.co[i] = gc[l];
+      r.cls_rows[i] = l == 5 ? 16 : gc[l];
+      r.dst_off[i] = off;
+      off += (int64_t)4 * r.cls_rows[i] * 4 * gc[l - 1];
+    }
+    p->gwt_ps = (off + 63) / 64 * 64;
+    ok = ok && !dev_alloc(p, &p->Gwt, (size_t)s.n_indiv * p->gwt_ps * 2, msg);
+    if (ok) ok = cudaMemset(p->Gwt, 0, (size_t)s.n_indiv * p->gwt_ps * 2) == cudaSuccess;
+    for (int i = 0; i < 4 && ok; ++i) {
+      const int l = i + 2;
+      const int ci = gc[l - 1], co = gc[l];
+      const int nbox = l == 5 ? 16 : (co < 256 ? co : 256);
+      ok = ctc_make_map(&p->mG[i], p->Gwt + r.dst_off[i], (uint64_t)4 * ci, 4 * r.cls_rows[i],
+                        s.n_indiv, p->gwt_ps, nbox, msg);
+      CtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = B;
+      q.ci = ci;
+      q.lhi = ilog2(gs[l - 1]);
+      q.co = co;
+      q.lho = ilog2(gs[l]);
+      q.kchunks = 4 * ci / 64;
+      q.nj = l == 5 ? 1 : (co + 255) / 256;
+      q.nbox = nbox;
+      q.transposed = 1;
+      q.out_mode = l == 5 ? CTC_TANH_CHW : CTC_F32_HWC;
+      q.cls_rows = r.cls_rows[i];
+      q.mtiles = ((B << (2 * (q.lho - 1))) + 127) / 128;
+      q.n_tiles = PE * 4 * q.mtiles;
+      q.slope = s.slope;
+      q.err = p->err;
+      p->gp[i] = q;
+      std::vector<ConvTcDesc> vt;
+      for (int c = 0; c < C; ++c)
+        for (int sl = 0; sl < 5; ++sl) {
+          const int pr = c * 5 + sl;
+          ConvTcDesc t;
+          memset(&t, 0, sizeof t);
+          t.in = (const bf16*)el(eh, (int64_t)pr * B * gmax);
+          t.out = l == 5 ? (bf16*)elw(b.E, (int64_t)c * b.e_cell + (int64_t)(1 + sl) * B * X)
+                         : (bf16*)(ec + (int64_t)pr * B * gmax);
+          t.wsel_idx = pr;
+          vt.push_back(t);
+        }
+      ok = ok && !upload(p, &p->gtd[i], vt, msg);
+    }
+  }
   if (!ok) {
     dc_plan_destroy(p);
     return nullptr;
@@ -546,6 +621,20 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int gc[6] = {s.z, 8 * g, 4 * g, 2 * g, g, 3};
   const int gs[6] = {1, 4, 8, 16, 32, 64};
   const int PE = C * 5;
+  if (p->tcg) {
+    launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
+    launch_conv(CONVT_FWD_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B * 16, gc[1], nbr, 1,
+                nullptr, 0, s.slope, st);
+    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, st);
+    for (int i = 0; i < 4; ++i) {
+      CtcParams q = p->gp[i];
+      q.descs = p->gtd[i];
+      q.wsel = nbr;
+      launch_conv_tc(p->mG[i], q, p->sms, st);
+      if (i < 3) launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, st);
+    }
+    return check(msg, "DCGAN generator evaluation (tensor cores)");
+  }
   for (int l = 1; l <= 5; ++l) {
     launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
                 l < 5, p->eg[l - 1], PE,
@@ -643,10 +732,11 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int dc_eval_launches(const DcPlan* p, int part) {
-  return part == 0 ? 9 : p->eval_launches - 9 + (p->tc ? 1 : 0);
+  if (part == 0) return p->tcg ? 10 : 9;
+  return p->eval_launches - 9 + (p->tc ? 1 : 0);
 }
 
-int* dc_error_flag(DcPlan* p) { return p && p->tc ? p->err : nullptr; }
+int* dc_error_flag(DcPlan* p) { return p && (p->tc || p->tcg) ? p->err : nullptr; }
 int dc_train_launches(const DcPlan* p) { return p->train_launches; }
 
 }  // namespace lipz

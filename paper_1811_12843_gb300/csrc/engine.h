@@ -97,6 +97,7 @@ struct ConvDesc {
   void* out;
   const void* aux;
   int n, ca, lha, lwa, co, lho, lwo, s, p;
+  int nhwc_out;  // CONV / CONVT: store channel-last [n][2^lho][2^lwo][co]
 };
 // Training-mode batch normalisation + ReLU of one problem: c = fp32 conv output
 // [n][C][2^lhw], h = activation out, mean / inv [C]; parameters (gamma at off_gamma, beta at

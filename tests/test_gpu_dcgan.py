@@ -71,13 +71,15 @@ def test_dcgan_eval_parity(L, precision, rows, cols, batch, width):
         assert max_rel(ev[k], ref[k]) < tol, k
 
 
-@pytest.mark.parametrize("rows,cols,batch", [(1, 1, 4), (1, 2, 3)])
-def test_dcgan_tensor_core_discriminator_eval(L, rows, cols, batch):
-    """bf16 with a discriminator width that is a multiple of 64 runs the discriminator's
-    evaluation on the tensor-core implicit-GEMM kernel (channel-last activations, re-laid
-    weights): every logit and loss against the oracle."""
+@pytest.mark.parametrize("rows,cols,batch,ngf", [(1, 1, 4, 8), (1, 2, 3, 8), (1, 1, 4, 64),
+                                                 (2, 1, 5, 64)])
+def test_dcgan_tensor_core_eval(L, rows, cols, batch, ngf):
+    """bf16 with widths that are multiples of 64 runs the evaluation on the tensor-core
+    implicit-GEMM kernel (the discriminator's convolutions; with ngf = 64 also the generator's
+    transposed convolutions by output parity class and channel-last batch norm): every logit
+    and loss against the oracle."""
     pool = _field_pool(5, 30)
-    g = _grid(L, rows, cols, 9, pool, precision="bf16", batch=batch, ngf=8, ndf=64)
+    g = _grid(L, rows, cols, 9, pool, precision="bf16", batch=batch, ngf=ngf, ndf=64)
     s = _state(g)
     ref = O.eval_neighborhoods(s, O.batches(s, pool))
     ev = g.eval(pairs=True)
