@@ -378,41 +378,63 @@ __global__ void k_relayout_g(const bf16* __restrict__ src, int64_t src_ps, bf16*
   }
 }
 
-// Training-mode batch normalisation + ReLU on channel-last data: block (channel group of 32,
-// problem); warp w takes pixels w, w + 8, ...; lane = channel; fixed-order reductions.
-__global__ void __launch_bounds__(256) k_bn_relu_hwc(const BnDesc* __restrict__ descs,
-                                                     const int* __restrict__ wsel_override) {
+// Training-mode batch normalisation + ReLU on channel-last data, in two launches over blocks
+// (group of 32 channels, problem, pixel chunk): each block sums its chunk's values and squares
+// per channel (lane = channel, warps over pixels, fixed order) into part[problem][chunk];
+// the apply blocks combine the chunks' sums in float64 in chunk order (mean, and the variance
+// as E[x^2] - mean^2), normalise, add the shift, apply ReLU and round to bf16.
+constexpr int BN_CHUNKS = 32;
+
+__global__ void __launch_bounds__(256) k_bn_stats_hwc(const BnDesc* __restrict__ descs,
+                                                      float2* __restrict__ part, int cmax) {
   pdl_wait();
   const BnDesc d = descs[blockIdx.y];
   const int ch = blockIdx.x * 32 + (threadIdx.x & 31);
   const int w = threadIdx.x >> 5;
   const int64_t m = (int64_t)d.n << d.lhw;
-  __shared__ float sh[8][32];
-  const bool on = ch < d.C;
-  float s = 0.f;
-  if (on)
-    for (int64_t px = w; px < m; px += 8) s += d.c[px * d.C + ch];
-  sh[w][threadIdx.x & 31] = s;
-  __syncthreads();
-  float tot = 0.f;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) tot += sh[i][threadIdx.x & 31];
-  const float mean = tot / (float)m;
-  __syncthreads();
-  float v = 0.f;
-  if (on)
-    for (int64_t px = w; px < m; px += 8) {
-      const float t = d.c[px * d.C + ch] - mean;
-      v = fmaf(t, t, v);
+  const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
+  __shared__ float sh[8][32][2];
+  float s = 0.f, q = 0.f;
+  if (ch < d.C)
+    for (int64_t px = p0 + w; px < p1; px += 8) {
+      const float v = d.c[px * d.C + ch];
+      s += v;
+      q = fmaf(v, v, q);
     }
-  sh[w][threadIdx.x & 31] = v;
+  sh[w][threadIdx.x & 31][0] = s;
+  sh[w][threadIdx.x & 31][1] = q;
   __syncthreads();
-  float vt = 0.f;
+  if (w == 0 && ch < d.C) {
+    float ts = 0.f, tq = 0.f;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) vt += sh[i][threadIdx.x & 31];
-  if (!on) return;
-  const float inv = rsqrtf(vt / (float)m + 1e-5f);
-  if (w == 0) {
+    for (int i = 0; i < 8; ++i) {
+      ts += sh[i][threadIdx.x & 31][0];
+      tq += sh[i][threadIdx.x & 31][1];
+    }
+    part[((int64_t)blockIdx.y * BN_CHUNKS + blockIdx.z) * cmax + ch] = make_float2(ts, tq);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__ descs,
+                                                      const float2* __restrict__ part, int cmax,
+                                                      const int* __restrict__ wsel_override) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int ch = blockIdx.x * 32 + (threadIdx.x & 31);
+  const int w = threadIdx.x >> 5;
+  if (ch >= d.C) return;
+  const int64_t m = (int64_t)d.n << d.lhw;
+  double ts = 0.0, tq = 0.0;
+  for (int z = 0; z < BN_CHUNKS; ++z) {
+    const float2 v = part[((int64_t)blockIdx.y * BN_CHUNKS + z) * cmax + ch];
+    ts += v.x;
+    tq += v.y;
+  }
+  const double mean_d = ts / (double)m;
+  const double var_d = fmax(tq / (double)m - mean_d * mean_d, 0.0);
+  const float mean = (float)mean_d;
+  const float inv = rsqrtf((float)var_d + 1e-5f);
+  if (w == 0 && blockIdx.z == 0) {
     d.mean[ch] = mean;
     d.inv[ch] = inv;
   }
@@ -420,7 +442,8 @@ __global__ void __launch_bounds__(256) k_bn_relu_hwc(const BnDesc* __restrict__ 
   const float* P = d.params + (ws ? (int64_t)ws[d.wsel_idx] * d.wsel_stride : 0);
   const float g = P[d.off_gamma + ch], b = P[d.off_beta + ch];
   bf16* h = (bf16*)d.h;
-  for (int64_t px = w; px < m; px += 8)
+  const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
+  for (int64_t px = p0 + w; px < p1; px += 8)
     h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(g * inv, d.c[px * d.C + ch] - mean, b), 0.f));
 }
 
@@ -433,9 +456,15 @@ void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
 }
 
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        cudaStream_t st) {
-  launch_pdl(ctc::k_bn_relu_hwc, dim3((channels + 31) / 32, n_problems), dim3(256), 0, st, descs,
+                        float* part, cudaStream_t st) {
+  const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
+  launch_pdl(ctc::k_bn_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels);
+  launch_pdl(ctc::k_bn_apply_hwc, grid, dim3(256), 0, st, descs, (const float2*)part, channels,
              wsel);
+}
+
+int64_t bn_hwc_part_floats(int n_problems, int channels) {
+  return (int64_t)n_problems * ctc::BN_CHUNKS * channels * 2;
 }
 
 namespace {

@@ -67,8 +67,10 @@ void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, cons
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutG& r, cudaStream_t st);
 // Batch normalisation (training mode) + ReLU on fp32 channel-last input into bf16 channel-last
-// output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels).
+// output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels); part holds
+// bn_hwc_part_floats(n_problems, channels) floats of per-chunk sums.
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        cudaStream_t st);
+                        float* part, cudaStream_t st);
+int64_t bn_hwc_part_floats(int n_problems, int channels);
 
 }  // namespace lipz

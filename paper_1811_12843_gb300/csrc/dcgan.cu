@@ -104,6 +104,7 @@ struct DcPlan {
   // tensor-core generator evaluation (bf16, ngf a multiple of 64): layers 2-5 by parity class
   // from class-major weight copies, channel-last activations and batch norm
   bool tcg = false;
+  float* bnpart = nullptr;
   bf16* Gwt = nullptr;
   int64_t gwt_ps = 0;
   RelayoutG relg;
@@ -550,6 +551,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       off += (int64_t)4 * r.cls_rows[i] * 4 * gc[l - 1];
     }
     p->gwt_ps = (off + 63) / 64 * 64;
+    ok = ok && !dev_alloc(p, &p->bnpart, (size_t)bn_hwc_part_floats(PE, 8 * g) * 4, msg);
     ok = ok && !dev_alloc(p, &p->Gwt, (size_t)s.n_indiv * p->gwt_ps * 2, msg);
     if (ok) ok = cudaMemset(p->Gwt, 0, (size_t)s.n_indiv * p->gwt_ps * 2) == cudaSuccess;
     for (int i = 0; i < 4 && ok; ++i) {
@@ -625,13 +627,13 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
     launch_conv(CONVT_FWD_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B * 16, gc[1], nbr, 1,
                 nullptr, 0, s.slope, st);
-    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, st);
+    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->gp[i];
       q.descs = p->gtd[i];
       q.wsel = nbr;
       launch_conv_tc(p->mG[i], q, p->sms, st);
-      if (i < 3) launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, st);
+      if (i < 3) launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, st);
     }
     return check(msg, "DCGAN generator evaluation (tensor cores)");
   }
@@ -732,7 +734,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int dc_eval_launches(const DcPlan* p, int part) {
-  if (part == 0) return p->tcg ? 10 : 9;
+  if (part == 0) return p->tcg ? 14 : 9;
   return p->eval_launches - 9 + (p->tc ? 1 : 0);
 }
 
