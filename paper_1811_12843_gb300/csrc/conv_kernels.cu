@@ -92,7 +92,8 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
         if (m < M && k < ke) {
           if (MODE == WGRAD) {
             const int nb = k >> (d.lha + d.lwa), yx = k & ((1 << (d.lha + d.lwa)) - 1);
-            v = to_f<TI>(A[(((int64_t)nb * d.ca + m) << (d.lha + d.lwa)) + yx]);
+            v = to_f<TI>(A[d.a_hwc ? (((int64_t)nb << (d.lha + d.lwa)) + yx) * d.ca + m
+                                   : (((int64_t)nb * d.ca + m) << (d.lha + d.lwa)) + yx]);
           } else if (MODE == CONVT2) {
             const int nb = m >> (lqy + lqx);
             const int oy = 2 * ((m >> lqx) & ((1 << lqy) - 1)) + py;
@@ -100,7 +101,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
             const int c = k >> 2, ky = ky0 + 2 * ((k >> 1) & 1), kx = kx0 + 2 * (k & 1);
             const int iy = (oy + d.p - ky) >> 1, ix = (ox + d.p - kx) >> 1;
             if (oy + d.p - ky >= 0 && ox + d.p - kx >= 0 && iy < Ha && ix < Wa)
-              v = to_f<TI>(A[(((int64_t)nb * d.ca + c) << (d.lha + d.lwa)) + (iy << d.lwa) + ix]);
+              v = to_f<TI>(A[d.a_hwc ? ((((int64_t)nb << (d.lha + d.lwa)) + (iy << d.lwa) + ix) *
+                                            d.ca + c)
+                                     : (((int64_t)nb * d.ca + c) << (d.lha + d.lwa)) +
+                                           (iy << d.lwa) + ix]);
           } else {
             const int nb = m >> (d.lho + d.lwo);
             const int oy = (m >> d.lwo) & ((1 << d.lho) - 1), ox = m & ((1 << d.lwo) - 1);
@@ -118,7 +122,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
               ix = tx / d.s;
             }
             if (ok && iy >= 0 && iy < Ha && ix >= 0 && ix < Wa)
-              v = to_f<TI>(A[(((int64_t)nb * d.ca + c) << (d.lha + d.lwa)) + (iy << d.lwa) + ix]);
+              v = to_f<TI>(A[d.a_hwc ? ((((int64_t)nb << (d.lha + d.lwa)) + (iy << d.lwa) + ix) *
+                                            d.ca + c)
+                                     : (((int64_t)nb * d.ca + c) << (d.lha + d.lwa)) +
+                                           (iy << d.lwa) + ix]);
           }
         }
         As[kk][mm] = v;
@@ -142,7 +149,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
             const int c = n >> 4, ky = (n >> 2) & 3, kx = n & 3;
             const int by = ay * d.s - d.p + ky, bx = ax * d.s - d.p + kx;
             if (by >= 0 && by < (1 << d.lho) && bx >= 0 && bx < (1 << d.lwo))
-              v = to_f<TI>(Bm[(((int64_t)nb * d.co + c) << (d.lho + d.lwo)) + (by << d.lwo) + bx]);
+              v = to_f<TI>(Bm[d.b_hwc ? ((((int64_t)nb << (d.lho + d.lwo)) + (by << d.lwo) + bx) *
+                                             d.co + c)
+                                      : (((int64_t)nb * d.co + c) << (d.lho + d.lwo)) +
+                                            (by << d.lwo) + bx]);
           } else if (MODE == CONV_FWD) {
             v = to_f<TI>(Bm[(int64_t)n * K + k]);
           } else if (MODE == CONVT2) {
@@ -381,7 +391,7 @@ __global__ void __launch_bounds__(256) k_bn_relu_backward(const BnDesc* __restri
   float sb = 0.f, sg = 0.f;
   for (int64_t e = threadIdx.x; e < m; e += 256) {
     const int64_t nb = e >> d.lhw, q = e & (hw - 1);
-    const int64_t o = ((nb * d.C + ch) << d.lhw) + q;
+    const int64_t o = d.hwc ? e * d.C + ch : ((nb * d.C + ch) << d.lhw) + q;
     const float dy = to_f<TO>(h[o]) > 0.f ? d.dh[o] : 0.f;
     sb += dy;
     sg = fmaf(dy, (d.c[o] - mean) * inv, sg);
@@ -398,7 +408,7 @@ __global__ void __launch_bounds__(256) k_bn_relu_backward(const BnDesc* __restri
   TO* dc = (TO*)d.dc;
   for (int64_t e = threadIdx.x; e < m; e += 256) {
     const int64_t nb = e >> d.lhw, q = e & (hw - 1);
-    const int64_t o = ((nb * d.C + ch) << d.lhw) + q;
+    const int64_t o = d.hwc ? e * d.C + ch : ((nb * d.C + ch) << d.lhw) + q;
     const float dy = to_f<TO>(h[o]) > 0.f ? d.dh[o] : 0.f;
     const float xhat = (d.c[o] - mean) * inv;
     dc[o] = from_f<TO>(g * inv * (dy - k1 - xhat * k2));
@@ -483,7 +493,7 @@ __global__ void k_logit_back(const LogitDesc* __restrict__ descs, int with_dw, f
       s = fmaf(g, av, s);
       if (da) da[(int64_t)r * d.K + k] = from_f<T>(av > 0.f ? g * wk : slope * g * wk);
     }
-    if (with_dw) d.dw[k] = s;
+    if (with_dw) d.dw[d.hwc_c ? (k % d.hwc_c) * 16 + k / d.hwc_c : k] = s;
   }
 }
 

@@ -103,8 +103,11 @@ struct DcPlan {
   int sms = 148;
   // tensor-core generator evaluation (bf16, ngf a multiple of 64): layers 2-5 by parity class
   // from class-major weight copies, channel-last activations and batch norm
-  bool tcg = false;
+  bool tcg = false, tct = false;
   float* bnpart = nullptr;
+  CtcParams tgp[4], tdp[4];
+  ConvTcDesc *tgd[4], *tdd[4];
+  LogitDesc *tdl_tc, *tdl_back_d_tc, *tdl_back_g_tc;
   bf16* Gwt = nullptr;
   int64_t gwt_ps = 0;
   RelayoutG relg;
@@ -196,6 +199,11 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   }
   const int PE = C * 5;
   p->tcg = s.bf && g % 64 == 0;
+  const bool tcd = s.bf && d % 64 == 0 && 8 * d <= 512;
+  // tensor-core training forward (both networks' widths multiples of 64): channel-last
+  // activations, read by the CUDA-core backward kernels in that layout
+  const bool tct = tcd && p->tcg;
+  p->tct = tct;
   // ---- buffers
   float *ec, *emean, *einv, *tc, *tmean, *tinv, *dh;
   void *eh, *ex, *ey, *th, *ta, *P, *Q, *P2, *Q2, *dcb, *d5;
@@ -327,6 +335,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       q.wsel = b.src_g;
       q.wsel_stride = b.PGs;
       q.wsel_idx = c;
+      q.nhwc_out = (tct && l == 1) ? 1 : 0;
       v.push_back(q);
       if (l <= 4)
         vb.push_back(bn(tgc(c, l), tgh(c, l), tmean + c * stats + stat_off[l],
@@ -389,6 +398,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       // weight gradient: a = delta of the output (dc[l] x ds[l]^2), b = the layer's input
       ConvDesc w = cdesc(dout, 2 * B, dc[l], ds[l], prev, dc[l - 1], ds[l - 1], 2, 1,
                          b.gD + (int64_t)c * b.PDs + dof[l - 1]);
+      w.a_hwc = tct;
+      w.b_hwc = tct && l >= 2;
       v.push_back(w);
       if (l >= 2) {
         void* din = elw((l % 2 == 0) ? Q : P, (int64_t)c * 2 * B * dmax);
@@ -397,6 +408,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         q.wsel_stride = b.PDs;
         q.wsel_idx = c;
         q.aux = tda(c, l - 1);
+        q.a_hwc = tct;
+        q.nhwc_out = tct;
         vd.push_back(q);
       }
     }
@@ -421,6 +434,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       q.wsel_idx = c;
       q.aux = last ? elw(tx(c), (int64_t)B * X)
                    : elw(tda(c, l - 1), (int64_t)B * dsz[l - 1]);
+      q.a_hwc = tct;
+      q.nhwc_out = tct && !last;
       v.push_back(q);
     }
     ok = ok && !upload(p, &p->gd[4 - l], v, msg);
@@ -437,6 +452,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       const void* in = l == 1 ? el(b.Z, (int64_t)c * B * z) : (const void*)tgh(c, l - 1);
       ConvDesc w = cdesc(in, B, gc[l - 1], gs[l - 1], dout, gc[l], gs[l], l == 1 ? 1 : 2,
                          l == 1 ? 0 : 1, b.gG + (int64_t)c * b.PGs + go[3 * (l - 1)]);
+      w.a_hwc = tct;
+      w.b_hwc = tct && l < 5;
       v.push_back(w);
       if (l >= 2) {
         ConvDesc q = cdesc(dout, B, gc[l], gs[l], Wg(l), gc[l - 1], gs[l - 1], 2, 1,
@@ -444,12 +461,15 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         q.wsel = b.src_g;
         q.wsel_stride = b.PGs;
         q.wsel_idx = c;
+        q.a_hwc = tct && l < 5;
+        q.nhwc_out = tct;
         vd.push_back(q);
         BnDesc r = bn(tgc(c, l - 1), tgh(c, l - 1), tmean + c * stats + stat_off[l - 1],
                       tinv + c * stats + stat_off[l - 1], b.src_g, c, l - 1, B);
         r.dh = dh + (int64_t)c * B * gmax;
         r.dc = elw(dcb, (int64_t)c * B * gmax);
         r.dparams = b.gG + (int64_t)c * b.PGs;
+        r.hwc = tct;
         vb.push_back(r);
       }
     }
@@ -466,7 +486,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   p->part_floats = part_need;
   ok = ok && !dev_alloc(p, &p->part, (size_t)part_need * 4, msg);
   // ---- tensor-core discriminator evaluation
-  p->tc = ok && s.bf && d % 64 == 0 && d * 8 <= 512;
+  p->tc = ok && tcd;
   if (p->tc) {
     int dev = 0;
     cudaGetDevice(&dev);
@@ -593,12 +613,79 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       ok = ok && !upload(p, &p->gtd[i], vt, msg);
     }
   }
+  // ---- tensor-core training forward (channel-last), and the output layer's descriptors in
+  // the re-laid (tap, channel) order
+  if (ok && tct) {
+    for (int i = 0; i < 4 && ok; ++i) {
+      const int l = i + 2;
+      CtcParams q = p->gp[i];
+      q.mtiles = ((B << (2 * (q.lho - 1))) + 127) / 128;
+      q.n_tiles = C * 4 * q.mtiles;
+      p->tgp[i] = q;
+      std::vector<ConvTcDesc> vt;
+      for (int c = 0; c < C; ++c) {
+        ConvTcDesc t;
+        memset(&t, 0, sizeof t);
+        t.in = (const bf16*)tgh(c, l - 1);
+        t.out = l == 5 ? (bf16*)elw(tx(c), (int64_t)B * X) : (bf16*)tgc(c, l);
+        t.wsel_idx = c;
+        vt.push_back(t);
+      }
+      ok = ok && !upload(p, &p->tgd[i], vt, msg);
+    }
+    for (int l = 1; l <= 4 && ok; ++l) {
+      CtcParams q = p->cp[l - 1];
+      q.rows = 2 * B;
+      q.mtiles = ((2 * B << (2 * q.lho)) + 127) / 128;
+      q.n_tiles = C * q.mtiles;
+      p->tdp[l - 1] = q;
+      std::vector<ConvTcDesc> vt;
+      for (int c = 0; c < C; ++c) {
+        ConvTcDesc t;
+        memset(&t, 0, sizeof t);
+        t.in = (const bf16*)(l == 1 ? (const void*)tx(c) : (const void*)tda(c, l - 1));
+        t.out = (bf16*)tda(c, l);
+        t.wsel_idx = c;
+        vt.push_back(t);
+      }
+      ok = ok && !upload(p, &p->tdd[l - 1], vt, msg);
+    }
+    std::vector<LogitDesc> vl, vd, vg;
+    for (int c = 0; c < C; ++c) {
+      LogitDesc q;
+      memset(&q, 0, sizeof q);
+      q.a = tda(c, 4);
+      q.w = p->Dwt + dof[4];
+      q.wsel = b.src_d;
+      q.wsel_stride = b.PDs;
+      q.wsel_idx = c;
+      q.logits = p->tlogits + (int64_t)c * 2 * B;
+      q.rows = 2 * B;
+      q.K = (int)dsz[4];
+      q.hwc_c = 8 * d;
+      vl.push_back(q);
+      LogitDesc r = q;
+      r.dl = elw(p->dl_d, (int64_t)c * 2 * B);
+      r.da = elw(P, (int64_t)c * 2 * B * dmax);
+      r.dw = b.gD + (int64_t)c * b.PDs + dof[4];
+      vd.push_back(r);
+      LogitDesc t = q;
+      t.a = elw(tda(c, 4), (int64_t)B * dsz[4]);
+      t.rows = B;
+      t.dl = elw(p->dl_g, (int64_t)c * B);
+      t.da = elw(P2, (int64_t)c * B * dmax);
+      t.dw = nullptr;
+      vg.push_back(t);
+    }
+    ok = ok && !upload(p, &p->tdl_tc, vl, msg) && !upload(p, &p->tdl_back_d_tc, vd, msg) &&
+         !upload(p, &p->tdl_back_g_tc, vg, msg);
+  }
   if (!ok) {
     dc_plan_destroy(p);
     return nullptr;
   }
   p->eval_launches = 9 + 5 * C;
-  p->train_launches = 50;
+  p->train_launches = tct ? 54 : 50;
   return p;
 }
 
@@ -685,11 +772,24 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   const int dc[5] = {3, d, 2 * d, 4 * d, 8 * d};
   const int ds[5] = {64, 32, 16, 8, 4};
   // forward of the selected pair
-  for (int l = 1; l <= 5; ++l) {
-    launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
-                l < 5, p->tg[l - 1], C,
-                B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0, s.slope, st);
-    if (l <= 4) launch_bn_relu(s.bf, p->tbn[l - 1], C, gc[l], nullptr, st);
+  if (p->tct) {
+    launch_conv(CONVT_FWD_MODE, CEPI_NONE_, true, true, p->tg[0], C, B * 16, gc[1], nullptr, 1,
+                nullptr, 0, s.slope, st);
+    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, st);
+    for (int i = 0; i < 4; ++i) {
+      CtcParams q = p->tgp[i];
+      q.descs = p->tgd[i];
+      q.wsel = p->b.src_g;
+      launch_conv_tc(p->mG[i], q, p->sms, st);
+      if (i < 3) launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, st);
+    }
+  } else {
+    for (int l = 1; l <= 5; ++l) {
+      launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
+                  l < 5, p->tg[l - 1], C, B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0,
+                  s.slope, st);
+      if (l <= 4) launch_bn_relu(s.bf, p->tbn[l - 1], C, gc[l], nullptr, st);
+    }
   }
   // the real rows of every cell's minibatch into TX rows [0, B)
   if (cudaMemcpy2DAsync(p->TX, 2 * B * X * es, p->b.E, p->b.e_cell * es, B * X * es, C,
@@ -697,13 +797,24 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     check(msg, "DCGAN training input copy");
     return 1;
   }
-  for (int l = 1; l <= 4; ++l)
-    launch_conv(CONV_FWD_MODE, CEPI_LRELU_, s.bf, false, p->td[l - 1], C,
-                2 * B * ds[l] * ds[l], dc[l], nullptr, 1, nullptr, 0, s.slope, st);
-  launch_logit_dot(s.bf, p->tdl, C, 2 * B, nullptr, st);
+  if (p->tct) {
+    for (int l = 1; l <= 4; ++l) {
+      CtcParams q = p->tdp[l - 1];
+      q.descs = p->tdd[l - 1];
+      q.wsel = p->b.src_d;
+      launch_conv_tc(p->mW[l - 1], q, p->sms, st);
+    }
+    launch_logit_dot(true, p->tdl_tc, C, 2 * B, nullptr, st);
+  } else {
+    for (int l = 1; l <= 4; ++l)
+      launch_conv(CONV_FWD_MODE, CEPI_LRELU_, s.bf, false, p->td[l - 1], C,
+                  2 * B * ds[l] * ds[l], dc[l], nullptr, 1, nullptr, 0, s.slope, st);
+    launch_logit_dot(s.bf, p->tdl, C, 2 * B, nullptr, st);
+  }
   launch_dc_dlogit(s.bf, p->tlogits, C, B, p->dl_d, p->dl_g, st);
   // discriminator backward (D loss)
-  launch_logit_back(s.bf, p->tdl_back_d, C, (int)(8 * d * 16), true, s.slope, st);
+  launch_logit_back(s.bf, p->tct ? p->tdl_back_d_tc : p->tdl_back_d, C, (int)(8 * d * 16), true,
+                    s.slope, st);
   for (int l = 4; l >= 1; --l) {
     const int k = 4 - l;
     launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
@@ -714,7 +825,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
                   st);
   }
   // the generator loss through the discriminator
-  launch_logit_back(s.bf, p->tdl_back_g, C, (int)(8 * d * 16), false, s.slope, st);
+  launch_logit_back(s.bf, p->tct ? p->tdl_back_g_tc : p->tdl_back_g, C, (int)(8 * d * 16),
+                    false, s.slope, st);
   for (int l = 4; l >= 1; --l)
     launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
                 p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,

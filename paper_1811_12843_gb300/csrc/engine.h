@@ -97,7 +97,9 @@ struct ConvDesc {
   void* out;
   const void* aux;
   int n, ca, lha, lwa, co, lho, lwo, s, p;
-  int nhwc_out;  // CONV / CONVT: store channel-last [n][2^lho][2^lwo][co]
+  int nhwc_out;  // CONV / CONVT: store (and read aux) channel-last [n][2^lho][2^lwo][co]
+  int a_hwc;     // operand a is channel-last [n][2^lha][2^lwa][ca]
+  int b_hwc;     // WGRAD: operand b is channel-last [n][2^lho][2^lwo][co]
 };
 // Training-mode batch normalisation + ReLU of one problem: c = fp32 conv output
 // [n][C][2^lhw], h = activation out, mean / inv [C]; parameters (gamma at off_gamma, beta at
@@ -117,6 +119,7 @@ struct BnDesc {
   const float* dh;
   void* dc;
   float* dparams;
+  int hwc;  // c, h, dh, dc channel-last [n][2^lhw][C]
 };
 // Discriminator output layer: a [rows][K] activations, w the weights (individual 0 + wsel),
 // logits [rows] out; backward: dl [rows] in, da [rows][K] out (or null), dw [K] out.
@@ -131,6 +134,8 @@ struct LogitDesc {
   const void* dl;
   void* da;
   float* dw;
+  int hwc_c;  // non-zero: a and w are in (tap, channel) order over hwc_c channels; dw is
+              // written in the weights' (channel, tap) order
 };
 enum { CONV_FWD_MODE = 0, CONVT_FWD_MODE = 1, WGRAD_MODE = 2, CONVT2_MODE = 3 };
 enum { CEPI_NONE_ = 0, CEPI_LRELU_ = 1, CEPI_TANH_ = 2, CEPI_DLRELU_ = 3, CEPI_DTANH_ = 4 };

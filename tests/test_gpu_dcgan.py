@@ -88,16 +88,23 @@ def test_dcgan_tensor_core_eval(L, rows, cols, batch, ngf):
         assert max_rel(ev[k], ref[k]) < 2e-2, k
 
 
-@pytest.mark.parametrize("precision", ["fp32", "bf16"])
-def test_dcgan_one_iteration_parity(L, precision):
+@pytest.mark.parametrize("precision,width,rows,cols,batch", [("fp32", 4, 2, 2, 4),
+                                                            ("bf16", 4, 2, 2, 4),
+                                                            ("bf16", 64, 1, 2, 16)])
+def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
     """Selection bit-exact given the engine's fitness; then the last step's gradients and the
     Adam state per cell against the oracle (a cell whose pre-activations came within rounding
-    distance of a kink is excused, as in the MLP checks)."""
+    distance of a kink is excused, as in the MLP checks). Width 64 in bf16 runs the training
+    forward on the tensor-core kernel with channel-last activations. At that width every cell
+    has pre-activations within 1e-8 of a kink, and batch normalisation's backward spreads a
+    flipped derivative over the whole channel: the CUDA-core and the tensor-core paths both
+    reach 1.4-4.7 % there (B = 16), so that case is held to 7.5 % per cell and 5 % median."""
     pool = _field_pool(3, 40)
-    g = _grid(L, 2, 2, 11, pool, precision=precision, keep_grads=1, ngf=4, ndf=4, batch=4)
+    g = _grid(L, rows, cols, 11, pool, precision=precision, keep_grads=1, ngf=width, ndf=width,
+              batch=batch)
     a = oracle_arch(g.arch)
     tol = TOL[g.arch.precision]
-    for it in range(2):
+    for it in range(2 if width < 64 else 1):
         s = _state(g)
         data = O.batches(s, pool)
         ev = g.eval()
@@ -122,6 +129,8 @@ def test_dcgan_one_iteration_parity(L, precision):
         assert np.all(ok | kinky), (it, worst)
         if precision == "fp32":
             assert np.sum(~ok) <= 1, (it, worst)
+        elif width >= 64:
+            assert np.all(worst < 0.075) and np.median(worst) < 0.05, (it, worst)
         else:
             assert np.all(worst < 5 * tol) and np.median(worst) < 2 * tol, (it, worst)
 
