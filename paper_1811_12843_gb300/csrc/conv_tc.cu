@@ -273,16 +273,25 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
-        if (p.out_mode == CTC_TANH_CHW) {
-          // a few output channels (the image's colours): tanh, bf16, channel-major images
+        if (p.out_mode == CTC_TANH_CHW || p.out_mode == CTC_DTANH_CHW) {
+          // a few output channels (the image's colours), channel-major images: tanh, or the
+          // delta times tanh' = 1 - f^2 with f the stored tanh output
           uint32_t v[16];
           LIPZ_TMEM_LD16(tmem + lane_base + (uint32_t)(R * 256), v);
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 16; ++e)
-            if (valid && e < p.co)
-              d.out[(((int64_t)nb * p.co + e) << (2 * p.lho)) + (oy << p.lho) + ox] =
-                  __float2bfloat16_rn(tanhf(__uint_as_float(v[e])));
+            if (valid && e < p.co) {
+              const int64_t o = (((int64_t)nb * p.co + e) << (2 * p.lho)) + (oy << p.lho) + ox;
+              float x = __uint_as_float(v[e]);
+              if (p.out_mode == CTC_TANH_CHW) {
+                x = tanhf(x);
+              } else {
+                const float f = __bfloat162float(d.aux[o]);
+                x = x * (1.f - f * f);
+              }
+              d.out[o] = __float2bfloat16_rn(x);
+            }
         } else {
           for (int g = 0; g < nbox / 32; ++g) {
             uint32_t v[32];
@@ -300,12 +309,32 @@ __global__ void __launch_bounds__(THREADS, 1)
               continue;
             }
             uint32_t pk[16];
+            if (p.out_mode == CTC_DLRELU_HWC) {
+              // the LeakyReLU derivative at the stored activation (same sign as its input)
+              uint4 au[4] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u),
+                             make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+              if (valid) {
+                const uint4* ap =
+                    reinterpret_cast<const uint4*>(d.aux + pix * p.co + j * 256 + g * 32);
 #pragma unroll
-            for (int e = 0; e < 32; e += 2) {
-              float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
-              a = a > 0.f ? a : p.slope * a;
-              b = b > 0.f ? b : p.slope * b;
-              pk[e >> 1] = pack_bf16(a, b);
+                for (int u = 0; u < 4; ++u) au[u] = __ldg(ap + u);
+              }
+              const __nv_bfloat16* ab = reinterpret_cast<const __nv_bfloat16*>(au);
+#pragma unroll
+              for (int e = 0; e < 32; e += 2) {
+                float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
+                a = __bfloat162float(ab[e]) > 0.f ? a : p.slope * a;
+                b = __bfloat162float(ab[e + 1]) > 0.f ? b : p.slope * b;
+                pk[e >> 1] = pack_bf16(a, b);
+              }
+            } else {
+#pragma unroll
+              for (int e = 0; e < 32; e += 2) {
+                float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
+                a = a > 0.f ? a : p.slope * a;
+                b = b > 0.f ? b : p.slope * b;
+                pk[e >> 1] = pack_bf16(a, b);
+              }
             }
             if (valid) {
               uint4* o = reinterpret_cast<uint4*>(d.out + pix * p.co + j * 256 + g * 32);
@@ -447,7 +476,35 @@ __global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__
     h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(g * inv, d.c[px * d.C + ch] - mean, b), 0.f));
 }
 
+// [o][c][ky][kx] -> [o][ky][kx][c] (conv weights in (tap, channel) order).
+__global__ void k_relayout_c(const bf16* __restrict__ src, int64_t src_ps, bf16* __restrict__ dst,
+                             int64_t dst_ps, int n_indiv, RelayoutC r) {
+  pdl_wait();
+  int64_t per = 0;
+  for (int l = 0; l < r.n; ++l) per += (int64_t)r.o[l] * r.c[l] * 16;
+  const int64_t total = per * n_indiv;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t ind = e / per;
+    int64_t k = e - ind * per;
+    int l = 0;
+    while (k >= (int64_t)r.o[l] * r.c[l] * 16) {
+      k -= (int64_t)r.o[l] * r.c[l] * 16;
+      ++l;
+    }
+    const int c = (int)(k % r.c[l]), t = (int)((k / r.c[l]) & 15);
+    const int64_t o = k / (16 * (int64_t)r.c[l]);
+    dst[ind * dst_ps + r.dst_off[l] + k] = src[ind * src_ps + r.src_off[l] + (o * r.c[l] + c) * 16 + t];
+  }
+}
+
 }  // namespace ctc
+
+void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
+                       const RelayoutC& r, cudaStream_t st) {
+  launch_pdl(ctc::k_relayout_c, dim3(1216), dim3(256), 0, st, src, src_ps, dst, dst_ps, n_indiv,
+             r);
+}
 
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutG& r, cudaStream_t st) {

@@ -18,6 +18,7 @@ namespace lipz {
 struct ConvTcDesc {
   const bf16* in;
   bf16* out;
+  const bf16* aux;  // CTC_DLRELU_HWC / CTC_DTANH_CHW: the activation whose derivative applies
   int wsel_idx;
   int pad;
 };
@@ -31,7 +32,10 @@ struct ConvTcDesc {
 // start at row cls * cls_rows of the map). out_mode: CTC_LRELU_HWC (bf16 LeakyReLU,
 // channel-last), CTC_F32_HWC (fp32 raw, channel-last), CTC_TANH_CHW (bf16 tanh, channel-major
 // images; co <= 16).
-enum { CTC_LRELU_HWC = 0, CTC_F32_HWC = 1, CTC_TANH_CHW = 2 };
+// CTC_DLRELU_HWC: bf16 delta times the LeakyReLU derivative at aux (channel-last);
+// CTC_DTANH_CHW: bf16 delta times 1 - aux^2 (aux the tanh output), channel-major images.
+enum { CTC_LRELU_HWC = 0, CTC_F32_HWC = 1, CTC_TANH_CHW = 2, CTC_DLRELU_HWC = 3,
+       CTC_DTANH_CHW = 4 };
 struct CtcParams {
   const ConvTcDesc* descs;
   int rows, ci, lhi, co, lho, nchw_in, kchunks, nj, nbox, mtiles, n_tiles;
@@ -66,6 +70,15 @@ void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, cons
                        cudaStream_t st);
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutG& r, cudaStream_t st);
+// [o][c][ky][kx] -> [o][ky][kx][c] for n weight tensors (o rows, c channels each) from
+// src_off to dst_off of every individual.
+struct RelayoutC {
+  int n;
+  int64_t src_off[4], dst_off[4];
+  int o[4], c[4];
+};
+void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
+                       const RelayoutC& r, cudaStream_t st);
 // Batch normalisation (training mode) + ReLU on fp32 channel-last input into bf16 channel-last
 // output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels); part holds
 // bn_hwc_part_floats(n_problems, channels) floats of per-chunk sums.

@@ -107,6 +107,16 @@ struct DcPlan {
   float* bnpart = nullptr;
   CtcParams tgp[4], tdp[4];
   ConvTcDesc *tgd[4], *tdd[4];
+  // tensor-core input gradients: the discriminator's as parity-class transposed convolutions
+  // (class-major copies of its weights), the generator's as convolutions ((tap, channel)
+  // copies of its transposed-convolution weights)
+  bf16 *Ddt = nullptr, *Gct = nullptr;
+  int64_t ddt_ps = 0, gct_ps = 0;
+  RelayoutG reld;
+  RelayoutC relc;
+  CUtensorMap mDd[4], mGc[4];
+  CtcParams ddp[3], gdp[4], gcp[4];
+  ConvTcDesc *ddd[3], *gdd[4], *gcd[4];
   LogitDesc *tdl_tc, *tdl_back_d_tc, *tdl_back_g_tc;
   bf16* Gwt = nullptr;
   int64_t gwt_ps = 0;
@@ -680,12 +690,132 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     ok = ok && !upload(p, &p->tdl_tc, vl, msg) && !upload(p, &p->tdl_back_d_tc, vd, msg) &&
          !upload(p, &p->tdl_back_g_tc, vg, msg);
   }
+  if (ok && tct) {
+    // discriminator input gradients: layer l's transposed convolution (in dc[l], out dc[l-1])
+    RelayoutG& r = p->reld;
+    memset(&r, 0, sizeof r);
+    r.n = 4;
+    int64_t off = 0;
+    for (int i = 0; i < 4; ++i) {
+      const int l = 4 - i;
+      r.src_off[i] = dof[l - 1];
+      r.ci[i] = dc[l];
+      r.co[i] = dc[l - 1];
+      r.cls_rows[i] = l == 1 ? 16 : dc[l - 1];
+      r.dst_off[i] = off;
+      off += (int64_t)4 * r.cls_rows[i] * 4 * dc[l];
+    }
+    p->ddt_ps = (off + 63) / 64 * 64;
+    ok = !dev_alloc(p, &p->Ddt, (size_t)s.n_indiv * p->ddt_ps * 2, msg) &&
+         cudaMemset(p->Ddt, 0, (size_t)s.n_indiv * p->ddt_ps * 2) == cudaSuccess;
+    for (int i = 0; i < 4 && ok; ++i) {
+      const int l = 4 - i;
+      const int nbox = l == 1 ? 16 : (dc[l - 1] < 256 ? dc[l - 1] : 256);
+      ok = ctc_make_map(&p->mDd[l - 1], p->Ddt + r.dst_off[i], (uint64_t)4 * dc[l],
+                        4 * r.cls_rows[i], s.n_indiv, p->ddt_ps, nbox, msg);
+      for (int chain = 0; chain < 2 && ok; ++chain) {
+        if (chain == 0 && l == 1) continue;  // the D loss needs no input gradient of layer 1
+        const int rows = chain == 0 ? 2 * B : B;
+        CtcParams q;
+        memset(&q, 0, sizeof q);
+        q.rows = rows;
+        q.ci = dc[l];
+        q.lhi = ilog2(ds[l]);
+        q.co = dc[l - 1];
+        q.lho = ilog2(ds[l - 1]);
+        q.kchunks = 4 * dc[l] / 64;
+        q.nj = l == 1 ? 1 : (dc[l - 1] + 255) / 256;
+        q.nbox = nbox;
+        q.transposed = 1;
+        q.out_mode = l == 1 ? CTC_DTANH_CHW : CTC_DLRELU_HWC;
+        q.cls_rows = r.cls_rows[i];
+        q.mtiles = ((rows << (2 * (q.lho - 1))) + 127) / 128;
+        q.n_tiles = C * 4 * q.mtiles;
+        q.slope = s.slope;
+        q.err = p->err;
+        std::vector<ConvTcDesc> vt;
+        for (int c = 0; c < C; ++c) {
+          ConvTcDesc t;
+          memset(&t, 0, sizeof t);
+          t.wsel_idx = c;
+          if (chain == 0) {
+            t.in = (const bf16*)elw((l % 2 == 0) ? P : Q, (int64_t)c * 2 * B * dmax);
+            t.out = (bf16*)elw((l % 2 == 0) ? Q : P, (int64_t)c * 2 * B * dmax);
+            t.aux = (const bf16*)tda(c, l - 1);
+          } else {
+            t.in = (const bf16*)elw((l % 2 == 0) ? P2 : Q2, (int64_t)c * B * dmax);
+            t.out = l == 1 ? (bf16*)elw(d5, (int64_t)c * B * X)
+                           : (bf16*)elw((l % 2 == 0) ? Q2 : P2, (int64_t)c * B * dmax);
+            t.aux = l == 1 ? (const bf16*)elw(tx(c), (int64_t)B * X)
+                           : (const bf16*)elw(tda(c, l - 1), (int64_t)B * dsz[l - 1]);
+          }
+          vt.push_back(t);
+        }
+        if (chain == 0) {
+          p->ddp[4 - l] = q;
+          ok = !upload(p, &p->ddd[4 - l], vt, msg);
+        } else {
+          p->gdp[4 - l] = q;
+          ok = !upload(p, &p->gdd[4 - l], vt, msg);
+        }
+      }
+    }
+    // generator input gradients: layer l's convolution (in gc[l] channels, out gc[l-1])
+    RelayoutC& rc = p->relc;
+    memset(&rc, 0, sizeof rc);
+    rc.n = 4;
+    off = 0;
+    for (int i = 0; i < 4; ++i) {
+      const int l = 5 - i;
+      rc.src_off[i] = go[3 * (l - 1)];
+      rc.o[i] = gc[l - 1];
+      rc.c[i] = gc[l];
+      rc.dst_off[i] = off;
+      off += (int64_t)gc[l - 1] * gc[l] * 16;
+    }
+    p->gct_ps = (off + 63) / 64 * 64;
+    ok = ok && !dev_alloc(p, &p->Gct, (size_t)s.n_indiv * p->gct_ps * 2, msg);
+    for (int i = 0; i < 4 && ok; ++i) {
+      const int l = 5 - i;
+      const int co = gc[l - 1], nbox = co < 256 ? co : 256;
+      ok = ctc_make_map(&p->mGc[i], p->Gct + rc.dst_off[i], (uint64_t)16 * gc[l], co, s.n_indiv,
+                        p->gct_ps, nbox, msg);
+      CtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = B;
+      q.ci = gc[l];
+      q.lhi = ilog2(gs[l]);
+      q.co = co;
+      q.lho = ilog2(gs[l - 1]);
+      q.nchw_in = l == 5 ? 1 : 0;
+      q.kchunks = (16 * gc[l] + 63) / 64;
+      q.nj = (co + 255) / 256;
+      q.nbox = nbox;
+      q.out_mode = CTC_F32_HWC;
+      q.mtiles = ((B << (2 * q.lho)) + 127) / 128;
+      q.n_tiles = C * q.mtiles;
+      q.slope = s.slope;
+      q.err = p->err;
+      p->gcp[i] = q;
+      std::vector<ConvTcDesc> vt;
+      for (int c = 0; c < C; ++c) {
+        ConvTcDesc t;
+        memset(&t, 0, sizeof t);
+        t.in = l == 5 ? (const bf16*)elw(d5, (int64_t)c * B * X)
+                      : (const bf16*)elw(dcb, (int64_t)c * B * gmax);
+        t.out = (bf16*)(dh + (int64_t)c * B * gmax);
+        t.wsel_idx = c;
+        vt.push_back(t);
+      }
+      ok = ok && !upload(p, &p->gcd[i], vt, msg);
+    }
+  }
   if (!ok) {
     dc_plan_destroy(p);
     return nullptr;
   }
   p->eval_launches = 9 + 5 * C;
-  p->train_launches = tct ? 54 : 50;
+  p->train_launches = tct ? 56 : 50;
   return p;
 }
 
@@ -812,6 +942,13 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     launch_logit_dot(s.bf, p->tdl, C, 2 * B, nullptr, st);
   }
   launch_dc_dlogit(s.bf, p->tlogits, C, B, p->dl_d, p->dl_g, st);
+  if (p->tct) {
+    // weights in the layouts the tensor-core input gradients read
+    launch_relayout_g((const bf16*)p->b.Dop, p->b.PDs, p->Ddt, p->ddt_ps, s.n_indiv, p->reld,
+                      st);
+    launch_relayout_c((const bf16*)p->b.Gop, p->b.PGs, p->Gct, p->gct_ps, s.n_indiv, p->relc,
+                      st);
+  }
   // discriminator backward (D loss)
   launch_logit_back(s.bf, p->tct ? p->tdl_back_d_tc : p->tdl_back_d, C, (int)(8 * d * 16), true,
                     s.slope, st);
@@ -819,26 +956,47 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     const int k = 4 - l;
     launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
                 nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
-    if (l >= 2)
+    if (l >= 2 && p->tct) {
+      CtcParams q = p->ddp[k];
+      q.descs = p->ddd[k];
+      q.wsel = p->b.src_d;
+      launch_conv_tc(p->mDd[l - 1], q, p->sms, st);
+    } else if (l >= 2) {
       launch_conv(CONVT2_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
                   2 * B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0, s.slope,
                   st);
+    }
   }
   // the generator loss through the discriminator
   launch_logit_back(s.bf, p->tct ? p->tdl_back_g_tc : p->tdl_back_g, C, (int)(8 * d * 16),
                     false, s.slope, st);
-  for (int l = 4; l >= 1; --l)
-    launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
-                p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
-                s.slope, st);
+  for (int l = 4; l >= 1; --l) {
+    if (p->tct) {
+      CtcParams q = p->gdp[4 - l];
+      q.descs = p->gdd[4 - l];
+      q.wsel = p->b.src_d;
+      launch_conv_tc(p->mDd[l - 1], q, p->sms, st);
+    } else {
+      launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
+                  p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
+                  s.slope, st);
+    }
+  }
   // generator backward
   for (int l = 5; l >= 1; --l) {
     const int k = 5 - l;
     launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
                 nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
     if (l >= 2) {
-      launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
-                  B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
+      if (p->tct) {
+        CtcParams q = p->gcp[k];
+        q.descs = p->gcd[k];
+        q.wsel = p->b.src_g;
+        launch_conv_tc(p->mGc[k], q, p->sms, st);
+      } else {
+        launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
+                    B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
+      }
       launch_bn_relu_backward(s.bf, p->gbn[k], C, gc[l - 1], st);
     }
   }
