@@ -16,13 +16,16 @@ namespace lipz {
 //              w[c][o][ky][kx]   (terms whose index is fractional or outside the image vanish)
 //   WGRAD:     y[m][c][ky][kx] = sum_{n,i,j} a[n][m][i][j] b[n][c][s i - p + ky][s j - p + kx]
 //              (split over K = n * Ha * Wa; partial sums reduced in a fixed order)
+//   DENSE1:    the generator's first layer (1x1 input, kernel 4x4, stride 1, pad 0) as the plain
+//              product y[n][(tap, o)] = sum_c a[n][c] w[c][o][tap] (M = n, N = 16 co, K = ca),
+//              stored channel-last (tap, o) or channel-major (o, tap)
 //   CONVT2:    CONVT_FWD at stride 2 by output parity class (i mod 2, j mod 2), one class per
 //              block (blockIdx.z = problem * 4 + class): only the taps ky = (i + p) mod 2 + 2 u,
 //              kx = (j + p) mod 2 + 2 v (u, v in {0, 1}) reach a pixel of the class, so K is
 //              4 per input channel instead of 16
 // ------------------------------------------------------------------------------------------
 enum { CONV_FWD = CONV_FWD_MODE, CONVT_FWD = CONVT_FWD_MODE, WGRAD = WGRAD_MODE,
-       CONVT2 = CONVT2_MODE };
+       CONVT2 = CONVT2_MODE, DENSE1 = DENSE1_MODE };
 enum { CEPI_NONE = CEPI_NONE_, CEPI_LRELU = CEPI_LRELU_, CEPI_TANH = CEPI_TANH_,
        CEPI_DLRELU = CEPI_DLRELU_, CEPI_DTANH = CEPI_DTANH_ };
 
@@ -35,6 +38,10 @@ __device__ __forceinline__ void conv_dims(const ConvDesc& d, int mode, int& M, i
     M = d.n << (d.lho + d.lwo - 2);
     N = d.co;
     K = d.ca * 4;
+  } else if (mode == DENSE1) {
+    M = d.n;
+    N = d.co * 16;
+    K = d.ca;
   } else {
     M = d.n << (d.lho + d.lwo);
     N = d.co;
@@ -84,13 +91,16 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int idx = tid + 256 * q;
-      // A element (m, k): k fastest
+      // A element (m, k): k fastest (channel-last weight-gradient deltas: m fastest)
       {
-        const int mm = idx >> 4, kk = idx & 15;
+        const bool mfast = MODE == WGRAD && d.a_hwc;
+        const int mm = mfast ? (idx & 63) : (idx >> 4), kk = mfast ? (idx >> 6) : (idx & 15);
         const int m = m0 + mm, k = k0 + kk;
         float v = 0.f;
         if (m < M && k < ke) {
-          if (MODE == WGRAD) {
+          if (MODE == DENSE1) {
+            v = to_f<TI>(A[(int64_t)m * d.ca + k]);
+          } else if (MODE == WGRAD) {
             const int nb = k >> (d.lha + d.lwa), yx = k & ((1 << (d.lha + d.lwa)) - 1);
             v = to_f<TI>(A[d.a_hwc ? (((int64_t)nb << (d.lha + d.lwa)) + yx) * d.ca + m
                                    : (((int64_t)nb * d.ca + m) << (d.lha + d.lwa)) + yx]);
@@ -143,10 +153,24 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
         const int k = k0 + kk, n = n0 + nn;
         float v = 0.f;
         if (n < N && k < ke) {
-          if (MODE == WGRAD) {
+          if (MODE == DENSE1) {
+            // n = tap * co + o
+            const int tap = n / d.co, o = n - tap * d.co;
+            v = to_f<TI>(Bm[((int64_t)k * d.co + o) * 16 + tap]);
+          } else if (MODE == WGRAD) {
             const int nb = k >> (d.lha + d.lwa);
             const int ay = (k >> d.lwa) & (Ha - 1), ax = k & (Wa - 1);
-            const int c = n >> 4, ky = (n >> 2) & 3, kx = n & 3;
+            // channel-last b: n = (tap, c) so that neighbouring threads read neighbouring
+            // channels; otherwise n = (c, tap)
+            int c, tap;
+            if (d.b_hwc) {
+              tap = n / d.co;
+              c = n - tap * d.co;
+            } else {
+              c = n >> 4;
+              tap = n & 15;
+            }
+            const int ky = tap >> 2, kx = tap & 3;
             const int by = ay * d.s - d.p + ky, bx = ax * d.s - d.p + kx;
             if (by >= 0 && by < (1 << d.lho) && bx >= 0 && bx < (1 << d.lwo))
               v = to_f<TI>(Bm[d.b_hwc ? ((((int64_t)nb << (d.lho + d.lwo)) + (by << d.lwo) + bx) *
@@ -189,7 +213,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int n = n0 + tn + j;
-        if (n < N) o[(int64_t)m * N + n] = acc[i][j];
+        if (n < N) {
+          const int e = d.b_hwc ? (n % d.co) * 16 + n / d.co : n;
+          o[(int64_t)m * N + e] = acc[i][j];
+        }
       }
     }
     return;
@@ -201,7 +228,10 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
     const int m = m0 + tm + i;
     if (m >= M) continue;
     int nb, yx;
-    if (MODE == CONVT2) {
+    if (MODE == DENSE1) {
+      nb = m;
+      yx = 0;
+    } else if (MODE == CONVT2) {
       nb = m >> (lqy + lqx);
       const int oy = 2 * ((m >> lqx) & ((1 << lqy) - 1)) + py;
       const int ox = 2 * (m & ((1 << lqx) - 1)) + px;
@@ -214,8 +244,14 @@ __global__ void __launch_bounds__(256) k_conv(const ConvDesc* __restrict__ descs
     for (int j = 0; j < 4; ++j) {
       const int n = n0 + tn + j;
       if (n >= N) continue;
-      const int64_t o = d.nhwc_out ? ((((int64_t)nb << (d.lho + d.lwo)) + yx) * d.co + n)
-                                   : ((((int64_t)nb * d.co + n) << (d.lho + d.lwo)) + yx);
+      int64_t o;
+      if (MODE == DENSE1) {
+        const int tap = n / d.co, oc = n - tap * d.co;
+        o = d.nhwc_out ? (int64_t)m * N + n : ((int64_t)m * d.co + oc) * 16 + tap;
+      } else {
+        o = d.nhwc_out ? ((((int64_t)nb << (d.lho + d.lwo)) + yx) * d.co + n)
+                       : ((((int64_t)nb * d.co + n) << (d.lho + d.lwo)) + yx);
+      }
       float v = acc[i][j];
       if (EPI == CEPI_LRELU) v = v > 0.f ? v : slope * v;
       if (EPI == CEPI_TANH) v = tanhf(v);
@@ -270,6 +306,11 @@ void launch_conv(int mode, int epi, bool bf, bool out_f32, const ConvDesc* descs
   if (mode == WGRAD) {
     if (bf) LIPZ_CONV(WGRAD, bf16, float, CEPI_NONE);
     else LIPZ_CONV(WGRAD, float, float, CEPI_NONE);
+    return;
+  }
+  if (mode == DENSE1) {
+    if (bf) LIPZ_CONV(DENSE1, bf16, float, CEPI_NONE);
+    else LIPZ_CONV(DENSE1, float, float, CEPI_NONE);
     return;
   }
   if (mode == CONVT2) {

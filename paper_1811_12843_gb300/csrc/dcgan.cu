@@ -842,7 +842,7 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int PE = C * 5;
   if (p->tcg) {
     launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
-    launch_conv(CONVT_FWD_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B * 16, gc[1], nbr, 1,
+    launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
                 nullptr, 0, s.slope, st);
     launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, st);
     for (int i = 0; i < 4; ++i) {
@@ -855,9 +855,12 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     return check(msg, "DCGAN generator evaluation (tensor cores)");
   }
   for (int l = 1; l <= 5; ++l) {
-    launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
-                l < 5, p->eg[l - 1], PE,
-                B * gs[l] * gs[l], gc[l], nbr, 1, nullptr, 0, s.slope, st);
+    if (l == 1)
+      launch_conv(DENSE1_MODE, CEPI_NONE_, s.bf, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
+                  nullptr, 0, s.slope, st);
+    else
+      launch_conv(CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->eg[l - 1], PE,
+                  B * gs[l] * gs[l], gc[l], nbr, 1, nullptr, 0, s.slope, st);
     if (l <= 4) launch_bn_relu(s.bf, p->ebn[l - 1], PE, gc[l], nbr, st);
   }
   return check(msg, "DCGAN generator evaluation");
@@ -903,7 +906,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   const int ds[5] = {64, 32, 16, 8, 4};
   // forward of the selected pair
   if (p->tct) {
-    launch_conv(CONVT_FWD_MODE, CEPI_NONE_, true, true, p->tg[0], C, B * 16, gc[1], nullptr, 1,
+    launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
                 nullptr, 0, s.slope, st);
     launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, st);
     for (int i = 0; i < 4; ++i) {
@@ -915,9 +918,12 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     }
   } else {
     for (int l = 1; l <= 5; ++l) {
-      launch_conv(l == 1 ? CONVT_FWD_MODE : CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf,
-                  l < 5, p->tg[l - 1], C, B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0,
-                  s.slope, st);
+      if (l == 1)
+        launch_conv(DENSE1_MODE, CEPI_NONE_, s.bf, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
+                    nullptr, 0, s.slope, st);
+      else
+        launch_conv(CONVT2_MODE, l == 5 ? CEPI_TANH_ : CEPI_NONE_, s.bf, l < 5, p->tg[l - 1], C,
+                    B * gs[l] * gs[l], gc[l], nullptr, 1, nullptr, 0, s.slope, st);
       if (l <= 4) launch_bn_relu(s.bf, p->tbn[l - 1], C, gc[l], nullptr, st);
     }
   }

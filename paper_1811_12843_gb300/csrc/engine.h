@@ -137,7 +137,8 @@ struct LogitDesc {
   int hwc_c;  // non-zero: a and w are in (tap, channel) order over hwc_c channels; dw is
               // written in the weights' (channel, tap) order
 };
-enum { CONV_FWD_MODE = 0, CONVT_FWD_MODE = 1, WGRAD_MODE = 2, CONVT2_MODE = 3 };
+enum { CONV_FWD_MODE = 0, CONVT_FWD_MODE = 1, WGRAD_MODE = 2, CONVT2_MODE = 3,
+       DENSE1_MODE = 4 };
 enum { CEPI_NONE_ = 0, CEPI_LRELU_ = 1, CEPI_TANH_ = 2, CEPI_DLRELU_ = 3, CEPI_DTANH_ = 4 };
 void launch_conv(int mode, int epi, bool bf, bool out_f32, const ConvDesc* descs,
                  int n_problems, int max_m, int max_n, const int* wsel, int splits, float* part,
