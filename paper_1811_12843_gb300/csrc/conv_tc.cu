@@ -358,6 +358,245 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
 }
 
+// ---- weight gradients on tcgen05 -----------------------------------------------------------
+// dW[m][c][tap] = sum over pixels q of A[q][m] * B[(s qy - p + ky, s qx - p + kx)][c], A and B
+// channel-last (M and Cb multiples of 64), as a GEMM with M = channels of A, N = (tap, c) and
+// K = the pixels of A, split into chunks of up to 64 x 64 pixels. Both operands are MN-major:
+// each gather thread writes one pixel row (128 bytes = 64 channels) of one 64-channel atom in
+// the 128-byte swizzle (atoms 8 KB apart). Tiles: (problem, split, M tile of 128, N tile of
+// 256); fp32 partial sums per split go to part[problem][split][M][N] in (tap, c) order.
+constexpr int WG_THREADS = 320;  // warp 1 MMA, warps 2-5 gather, warps 6-9 epilogue
+constexpr int WG_STAGES = 4;
+constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256;
+constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_STAGES)
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constant__ WgtcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* misc = smem_raw + (base - raw) + WG_STAGES * STAGE_BYTES;
+  const uint32_t bars = smem_u32(misc);
+  const uint32_t bFull = bars, bEmpty = bars + 8 * WG_STAGES;
+  const uint32_t bAccF = bars + 16 * WG_STAGES, bAccE = bAccF + 16, bFinal = bAccE + 16;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 240);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 244);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < WG_STAGES; ++s) {
+      mbar_init(bFull + 8 * s, 128);
+      mbar_init(bEmpty + 8 * s, 1);
+    }
+    mbar_init(bAccF, 1);
+    mbar_init(bAccF + 8, 1);
+    mbar_init(bAccE, 128);
+    mbar_init(bAccE + 8, 128);
+    mbar_init(bFinal, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  const int mt_n = p.M / 128, nt_n = p.N / 256;
+  const int per_split = mt_n * nt_n;
+  const int la = p.la, lb = p.lb;
+  const int64_t Kp = (int64_t)p.rows << (2 * la);  // pixels of A per problem
+  auto split_range = [&](int split, int64_t& k0, int64_t& k1) {
+    k0 = (int64_t)split * p.kc;
+    k1 = k0 + p.kc < Kp ? k0 + p.kc : Kp;
+  };
+  if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0, uses[2] = {0, 0}, jobs = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      const uint32_t idesc = idesc_bf16_major(128, 256, 1, 1);
+      for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++jobs) {
+        const int split = (tile / per_split) % p.splits;
+        int64_t k0, k1;
+        split_range(split, k0, k1);
+        const int R = jobs & 1;
+        if (uses[R] > 0 &&
+            !mbar_wait(bAccE + 8 * R, (uint32_t)((uses[R] - 1) & 1), abort_flag, p.err, 31)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dt = tmem + (uint32_t)(R * 256);
+        bool first = true;
+        for (int64_t kb = k0; kb < k1; kb += 64) {
+          if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 32)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            tc_mma(dt, sw128_mn_desc(sA + kk * 2048, 8192), sw128_mn_desc(sB + kk * 2048, 8192),
+                   idesc, first ? 0u : 1u);
+            first = false;
+          }
+          tc_commit(bEmpty + 8 * stage);
+          if (++stage == WG_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        tc_commit(bAccF + 8 * R);
+        uses[R]++;
+      }
+      tc_commit(bFinal);
+      volatile int never = 0;
+      mbar_wait(bFinal, 0u, &never, p.err, 33);
+    }
+  } else if (warp >= 2 && warp < 6) {
+    // gather: thread t copies pixel row (t & 63) of A atom (t >> 6) and of B atoms 2 (t >> 6),
+    // 2 (t >> 6) + 1 with 16-byte cp.async (zero fill outside the image); a stage is marked
+    // full WG_LAG chunks later, once its copy group has landed
+    const int t = threadIdx.x - 64;
+    const int row = t & 63, half = t >> 6;
+    const uint32_t sw = (uint32_t)(row & 7);
+    int stage = 0, arr_stage = 0, pending = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
+      const int prob = tile / (p.splits * per_split);
+      const int split = (tile / per_split) % p.splits;
+      const int mt = (tile % per_split) / nt_n, nt = tile % nt_n;
+      const WgtcDesc d = p.descs[prob];
+      int64_t k0, k1;
+      split_range(split, k0, k1);
+      for (int64_t kb = k0; kb < k1; kb += 64) {
+        if (!mbar_wait_warp(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 34)) {
+          ok = false;
+          break;
+        }
+        const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+        const int64_t q = kb + row;  // pixel of A
+        const bool qv = q < k1;
+        const int nb = (int)(q >> (2 * la));
+        const int ay = (int)((q >> la) & ((1 << la) - 1)), ax = (int)(q & ((1 << la) - 1));
+        {
+          const bf16* src = qv ? d.a + q * p.M + mt * 128 + half * 64 : d.a;
+          const uint32_t dst = sA + (uint32_t)half * 8192u + (uint32_t)row * 128u;
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            cp_async16(dst + (((uint32_t)u ^ sw) << 4), src + (qv ? 8 * u : 0), qv ? 16 : 0);
+        }
+#pragma unroll
+        for (int aa = 0; aa < 2; ++aa) {
+          const int atom = 2 * half + aa;
+          const int n0 = nt * 256 + atom * 64;
+          const int tap = n0 / p.Cb, c0 = n0 - tap * p.Cb;
+          const int by = ay * p.s - p.p + (tap >> 2), bx = ax * p.s - p.p + (tap & 3);
+          const bool in = qv && by >= 0 && by < (1 << lb) && bx >= 0 && bx < (1 << lb);
+          const bf16* src =
+              in ? d.b + ((((int64_t)nb << (2 * lb)) + (by << lb) + bx) * p.Cb + c0) : d.b;
+          const uint32_t dst = sB + (uint32_t)atom * 8192u + (uint32_t)row * 128u;
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            cp_async16(dst + (((uint32_t)u ^ sw) << 4), src + (in ? 8 * u : 0), in ? 16 : 0);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        if (++pending > WG_LAG) {
+          asm volatile("cp.async.wait_group %0;" ::"n"(WG_LAG) : "memory");
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          mbar_arrive(bFull + 8 * arr_stage);
+          arr_stage = arr_stage + 1 == WG_STAGES ? 0 : arr_stage + 1;
+          --pending;
+        }
+        if (++stage == WG_STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    // the last chunks (and, after an expired wait, every copy still in flight)
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    for (; pending > 0; --pending) {
+      mbar_arrive(bFull + 8 * arr_stage);
+      arr_stage = arr_stage + 1 == WG_STAGES ? 0 : arr_stage + 1;
+    }
+  } else if (warp >= 6) {
+    // epilogue: row m of the tile, 256 columns in groups of 32, fp32 partial sums
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
+    int uses[2] = {0, 0}, jobs = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++jobs) {
+      const int prob = tile / (p.splits * per_split);
+      const int split = (tile / per_split) % p.splits;
+      const int mt = (tile % per_split) / nt_n, nt = tile % nt_n;
+      const int R = jobs & 1;
+      if (!mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 35)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float* o = p.part + (((int64_t)prob * p.splits + split) * p.M + mt * 128 + r) * p.N +
+                 nt * 256;
+      for (int g = 0; g < 8; ++g) {
+        uint32_t v[32];
+        LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
+        tmem_wait_ld();
+        float4* o4 = reinterpret_cast<float4*>(o + g * 32);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          o4[u] = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
+                              __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
+      }
+      tc_fence_before();
+      mbar_arrive(bAccE + 8 * R);
+      uses[R]++;
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+}
+
+// part[problem][split][m][(tap, c)] -> dW[m][c][tap], summed over the splits in order; a
+// block turns one row m and 64 channels through shared memory (grid: M * Cb / 64, problems).
+__global__ void __launch_bounds__(256) k_wgrad_tc_reduce(const __grid_constant__ WgtcParams p) {
+  __shared__ float tile[16][65];
+  pdl_wait();
+  const int prob = blockIdx.y;
+  const int cchunks = p.Cb / 64;
+  const int m = blockIdx.x / cchunks, c0 = (blockIdx.x - m * cchunks) * 64;
+  const int64_t MN = (int64_t)p.M * p.N;
+  const float* part = p.part + (int64_t)prob * p.splits * MN + (int64_t)m * p.N + c0;
+  for (int i = threadIdx.x; i < 1024; i += 256) {
+    const int tap = i >> 6, cc = i & 63;
+    const float* src = part + (int64_t)tap * p.Cb + cc;
+    float acc = 0.f;
+    for (int sp = 0; sp < p.splits; ++sp) acc += src[sp * MN];
+    tile[tap][cc] = acc;
+  }
+  __syncthreads();
+  float* out = p.descs[prob].dw + (int64_t)m * p.N + (int64_t)c0 * 16;
+  for (int i = threadIdx.x; i < 1024; i += 256) out[i] = tile[i & 15][i >> 4];
+}
+
 // [out][in][ky][kx] -> [out][ky][kx][in] for the five discriminator tensors of every
 // individual (bf16 copies).
 __global__ void k_relayout_d(const bf16* __restrict__ src, bf16* __restrict__ dst, int n_indiv,
@@ -499,6 +738,22 @@ __global__ void k_relayout_c(const bf16* __restrict__ src, int64_t src_ps, bf16*
 }
 
 }  // namespace ctc
+
+bool wgtc_prepare(std::string* msg) {
+  if (cudaFuncSetAttribute(ctc::k_wgrad_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           ctc::WG_SMEM) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "cannot reserve shared memory for the tensor-core weight gradients";
+    return false;
+  }
+  return true;
+}
+
+void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st) {
+  const int grid = p.n_tiles < sms ? p.n_tiles : sms;
+  launch_pdl(ctc::k_wgrad_tc, dim3(grid), dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, p);
+  launch_pdl(ctc::k_wgrad_tc_reduce, dim3(p.M * (p.Cb / 64), p.n_probs), dim3(256), 0, st, p);
+}
 
 void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutC& r, cudaStream_t st) {

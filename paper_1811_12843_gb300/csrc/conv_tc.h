@@ -62,6 +62,27 @@ struct RelayoutD {
   int64_t P;
 };
 
+// Weight gradients on tcgen05: per problem a = [rows][2^la][2^la][M] and b = the gathered
+// operand [rows][2^lb][2^lb][Cb] (both channel-last, M a multiple of 128, Cb of 64, N = 16 Cb
+// a multiple of 256); dw = the problem's [M][Cb][4][4] fp32 gradient. b's pixel for tap
+// (ky, kx) of a's pixel (y, x) is (s y - p + ky, s x - p + kx). part holds
+// n_probs x splits x M x N floats; split s covers a's pixels [s kc, (s + 1) kc) of each problem
+// (kc a multiple of 64, every split non-empty).
+struct WgtcDesc {
+  const bf16* a;
+  const bf16* b;
+  float* dw;
+};
+struct WgtcParams {
+  const WgtcDesc* descs;
+  int n_probs, rows, M, N, Cb, la, lb, s, p, splits, n_tiles;
+  int64_t kc;
+  float* part;
+  int* err;
+};
+bool wgtc_prepare(std::string* msg);
+void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st);
+
 bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t depth,
                   uint64_t depth_elems, uint32_t box_rows, std::string* msg);
 bool ctc_prepare(std::string* msg);

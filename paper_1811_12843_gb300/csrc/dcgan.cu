@@ -124,6 +124,11 @@ struct DcPlan {
   CUtensorMap mG[4];
   CtcParams gp[4];
   ConvTcDesc* gtd[4];
+  // tensor-core weight gradients of the layers whose channel counts fill the tiles
+  bool wtc_d[4] = {}, wtc_g[5] = {};
+  WgtcParams wdp[4], wgp[5];
+  WgtcDesc *wdd[4] = {}, *wgd[5] = {};
+  float* wpart = nullptr;
 };
 
 namespace {
@@ -809,6 +814,84 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       }
       ok = ok && !upload(p, &p->gcd[i], vt, msg);
     }
+    // weight gradients: a = the output's delta (discriminator) or the layer's input
+    // (generator), M = its channels; b = the other operand, gathered per tap
+    ok = ok && wgtc_prepare(msg);
+    int64_t wneed = 0;
+    auto wplan = [&](WgtcParams& q) {
+      const int64_t Kp = (int64_t)q.rows << (2 * q.la);
+      const int64_t chunks = (Kp + 63) / 64;
+      const int64_t per = (int64_t)C * (q.M / 128) * (q.N / 256);
+      int best = 1;
+      double be = 0;
+      for (int sp = 1; sp <= 64 && sp <= std::max<int64_t>(1, chunks / 8); ++sp) {
+        const int64_t t = per * sp;
+        const double e = (double)t / ((double)((t + p->sms - 1) / p->sms) * p->sms);
+        if (e > be + 1e-9) {
+          be = e;
+          best = sp;
+        }
+      }
+      q.kc = (chunks + best - 1) / best * 64;
+      q.splits = (int)((Kp + q.kc - 1) / q.kc);
+      q.n_tiles = (int)(per * q.splits);
+      q.n_probs = C;
+      q.err = p->err;
+      wneed = std::max<int64_t>(wneed, (int64_t)C * q.splits * q.M * q.N);
+    };
+    for (int l = 4; l >= 2 && ok; --l) {
+      const int k = 4 - l;
+      if (dc[l] % 128 != 0 || dc[l - 1] % 64 != 0) continue;
+      WgtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = 2 * B;
+      q.M = dc[l];
+      q.Cb = dc[l - 1];
+      q.N = 16 * q.Cb;
+      q.la = ilog2(ds[l]);
+      q.lb = ilog2(ds[l - 1]);
+      q.s = 2;
+      q.p = 1;
+      wplan(q);
+      std::vector<WgtcDesc> vw;
+      for (int c = 0; c < C; ++c) {
+        WgtcDesc w;
+        w.a = (const bf16*)elw((l % 2 == 0) ? P : Q, (int64_t)c * 2 * B * dmax);
+        w.b = (const bf16*)tda(c, l - 1);
+        w.dw = b.gD + (int64_t)c * b.PDs + dof[l - 1];
+        vw.push_back(w);
+      }
+      p->wdp[k] = q;
+      p->wtc_d[k] = true;
+      ok = !upload(p, &p->wdd[k], vw, msg);
+    }
+    for (int l = 4; l >= 2 && ok; --l) {
+      const int k = 5 - l;
+      if (gc[l - 1] % 128 != 0 || gc[l] % 64 != 0) continue;
+      WgtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = B;
+      q.M = gc[l - 1];
+      q.Cb = gc[l];
+      q.N = 16 * q.Cb;
+      q.la = ilog2(gs[l - 1]);
+      q.lb = ilog2(gs[l]);
+      q.s = 2;
+      q.p = 1;
+      wplan(q);
+      std::vector<WgtcDesc> vw;
+      for (int c = 0; c < C; ++c) {
+        WgtcDesc w;
+        w.a = (const bf16*)tgh(c, l - 1);
+        w.b = (const bf16*)elw(dcb, (int64_t)c * B * gmax);
+        w.dw = b.gG + (int64_t)c * b.PGs + go[3 * (l - 1)];
+        vw.push_back(w);
+      }
+      p->wgp[k] = q;
+      p->wtc_g[k] = true;
+      ok = !upload(p, &p->wgd[k], vw, msg);
+    }
+    ok = ok && !dev_alloc(p, &p->wpart, (size_t)wneed * 4, msg);
   }
   if (!ok) {
     dc_plan_destroy(p);
@@ -960,8 +1043,15 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
                     s.slope, st);
   for (int l = 4; l >= 1; --l) {
     const int k = 4 - l;
-    launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
-                nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
+    if (p->wtc_d[k]) {
+      WgtcParams q = p->wdp[k];
+      q.descs = p->wdd[k];
+      q.part = p->wpart;
+      launch_wgrad_tc(q, p->sms, st);
+    } else {
+      launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
+                  nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
+    }
     if (l >= 2 && p->tct) {
       CtcParams q = p->ddp[k];
       q.descs = p->ddd[k];
@@ -991,8 +1081,15 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   // generator backward
   for (int l = 5; l >= 1; --l) {
     const int k = 5 - l;
-    launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
-                nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
+    if (p->wtc_g[k]) {
+      WgtcParams q = p->wgp[k];
+      q.descs = p->wgd[k];
+      q.part = p->wpart;
+      launch_wgrad_tc(q, p->sms, st);
+    } else {
+      launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
+                  nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
+    }
     if (l >= 2) {
       if (p->tct) {
         CtcParams q = p->gcp[k];
