@@ -31,6 +31,13 @@ constexpr int B_BYTES = 256 * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 320;  // warp 0 TMA, 1 MMA, 2-5 gather, 6-9 epilogue
 constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr int LAG = 2;  // copy groups a gather thread keeps in flight (< STAGES)
+
+// 16-byte global -> shared copy; bytes = 0 writes zeros (src must still be a valid address)
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes)
+               : "memory");
+}
 
 __global__ void __launch_bounds__(THREADS, 1)
     k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CtcParams p) {
@@ -154,9 +161,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_wait(bFinal, 0u, &never, p.err, 26);
     }
   } else if (warp < 6) {
-    // ---- A operand: thread r gathers row r of every k chunk
+    // ---- A operand: thread r gathers row r of every k chunk. Channel-last rows arrive by
+    // 16-byte cp.async (zero fill outside the image), a stage marked full LAG chunks later once
+    // its copy group has landed; the first layer's CHW rows are converted through registers.
     const int r = threadIdx.x - 64;
-    int stage = 0;
+    int stage = 0, arr_stage = 0, pending = 0;
     uint32_t phase = 0;
     bool ok = true;
     const int lhi = p.lhi, Hi = 1 << lhi;
@@ -226,24 +235,37 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             const bool in = valid && ty >= 0 && tx >= 0 && iy >= 0 && iy < Hi && ix >= 0 &&
                             ix < Hi;
-            const uint4* src = reinterpret_cast<const uint4*>(
-                d.in + ((((int64_t)nb << (2 * lhi)) + (iy << lhi) + ix) * p.ci + c0));
+            const bf16* src =
+                in ? d.in + ((((int64_t)nb << (2 * lhi)) + (iy << lhi) + ix) * p.ci + c0) : d.in;
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              const uint4 v = in ? __ldg(src + u) : make_uint4(0u, 0u, 0u, 0u);
-              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                               row + ((uint32_t)(u ^ (r & 7)) << 4)),
-                           "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                           : "memory");
+            for (int u = 0; u < 8; ++u)
+              cp_async16(row + ((uint32_t)(u ^ (r & 7)) << 4), src + (in ? 8 * u : 0),
+                         in ? 16 : 0);
+            asm volatile("cp.async.commit_group;" ::: "memory");
+            if (++pending > LAG) {
+              asm volatile("cp.async.wait_group %0;" ::"n"(LAG) : "memory");
+              asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+              mbar_arrive(bFullA + 8 * arr_stage);
+              arr_stage = arr_stage + 1 == STAGES ? 0 : arr_stage + 1;
+              --pending;
             }
           }
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          mbar_arrive(bFullA + 8 * stage);
+          if (p.nchw_in) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive(bFullA + 8 * stage);
+          }
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
+    }
+    // the last chunks (and, after an expired wait, every copy still in flight)
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    for (; pending > 0; --pending) {
+      mbar_arrive(bFullA + 8 * arr_stage);
+      arr_stage = arr_stage + 1 == STAGES ? 0 : arr_stage + 1;
     }
   } else {
     // ---- epilogue: LeakyReLU, bf16, channel-last rows
@@ -369,11 +391,6 @@ constexpr int WG_THREADS = 320;  // warp 1 MMA, warps 2-5 gather, warps 6-9 epil
 constexpr int WG_STAGES = 4;
 constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256;
 constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_STAGES)
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes)
-               : "memory");
-}
 
 __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constant__ WgtcParams p) {
   extern __shared__ uint8_t smem_raw[];
