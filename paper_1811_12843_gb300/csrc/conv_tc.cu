@@ -664,44 +664,81 @@ __global__ void k_relayout_g(const bf16* __restrict__ src, int64_t src_ps, bf16*
 }
 
 // Training-mode batch normalisation + ReLU on channel-last data, in two launches over blocks
-// (group of 32 channels, problem, pixel chunk): each block sums its chunk's values and squares
-// per channel (lane = channel, warps over pixels, fixed order) into part[problem][chunk];
-// the apply blocks combine the chunks' sums in float64 in chunk order (mean, and the variance
-// as E[x^2] - mean^2), normalise, add the shift, apply ReLU and round to bf16.
+// (group of 32 channels, problem, pixel chunk): each stats block sums its chunk's values and
+// squares per channel (lane = channel, warps over pixels, fixed order) into
+// part[problem][chunk]; the last block of a (channel group, problem) to finish combines the
+// chunks' sums in float64 in chunk order (mean, and the variance as E[x^2] - mean^2) into the
+// descriptor's mean and inverse deviation. The apply blocks normalise, add the shift, apply
+// ReLU and round to bf16.
 constexpr int BN_CHUNKS = 32;
 
 __global__ void __launch_bounds__(256) k_bn_stats_hwc(const BnDesc* __restrict__ descs,
-                                                      float2* __restrict__ part, int cmax) {
+                                                      float2* __restrict__ part, int cmax,
+                                                      unsigned* __restrict__ counters) {
   pdl_wait();
   const BnDesc d = descs[blockIdx.y];
-  const int ch = blockIdx.x * 32 + (threadIdx.x & 31);
+  const int lane = threadIdx.x & 31;
+  const int ch = blockIdx.x * 32 + lane;
   const int w = threadIdx.x >> 5;
   const int64_t m = (int64_t)d.n << d.lhw;
   const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
   __shared__ float sh[8][32][2];
+  __shared__ int is_last;
   float s = 0.f, q = 0.f;
-  if (ch < d.C)
-    for (int64_t px = p0 + w; px < p1; px += 8) {
+  if (ch < d.C) {
+    int64_t px = p0 + w;
+    for (; px + 24 < p1; px += 32) {
+      float v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = d.c[(px + 8 * u) * d.C + ch];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        s += v[u];
+        q = fmaf(v[u], v[u], q);
+      }
+    }
+    for (; px < p1; px += 8) {
       const float v = d.c[px * d.C + ch];
       s += v;
       q = fmaf(v, v, q);
     }
-  sh[w][threadIdx.x & 31][0] = s;
-  sh[w][threadIdx.x & 31][1] = q;
+  }
+  sh[w][lane][0] = s;
+  sh[w][lane][1] = q;
   __syncthreads();
+  float2* pp = part + (int64_t)blockIdx.y * BN_CHUNKS * cmax;
   if (w == 0 && ch < d.C) {
     float ts = 0.f, tq = 0.f;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      ts += sh[i][threadIdx.x & 31][0];
-      tq += sh[i][threadIdx.x & 31][1];
+      ts += sh[i][lane][0];
+      tq += sh[i][lane][1];
     }
-    part[((int64_t)blockIdx.y * BN_CHUNKS + blockIdx.z) * cmax + ch] = make_float2(ts, tq);
+    pp[(int64_t)blockIdx.z * cmax + ch] = make_float2(ts, tq);
   }
+  __threadfence();
+  __syncthreads();
+  unsigned* cnt = counters + (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
+  if (threadIdx.x == 0) is_last = atomicAdd(cnt, 1u) == BN_CHUNKS - 1;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  if (w == 0 && ch < d.C) {
+    double ts = 0.0, tq = 0.0;
+    for (int z = 0; z < BN_CHUNKS; ++z) {
+      const float2 v = __ldcg(&pp[(int64_t)z * cmax + ch]);
+      ts += v.x;
+      tq += v.y;
+    }
+    const double mean_d = ts / (double)m;
+    const double var_d = fmax(tq / (double)m - mean_d * mean_d, 0.0);
+    d.mean[ch] = (float)mean_d;
+    d.inv[ch] = rsqrtf((float)var_d + 1e-5f);
+  }
+  if (threadIdx.x == 0) *cnt = 0u;
 }
 
 __global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__ descs,
-                                                      const float2* __restrict__ part, int cmax,
                                                       const int* __restrict__ wsel_override) {
   pdl_wait();
   const BnDesc d = descs[blockIdx.y];
@@ -709,27 +746,139 @@ __global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__
   const int w = threadIdx.x >> 5;
   if (ch >= d.C) return;
   const int64_t m = (int64_t)d.n << d.lhw;
-  double ts = 0.0, tq = 0.0;
-  for (int z = 0; z < BN_CHUNKS; ++z) {
-    const float2 v = part[((int64_t)blockIdx.y * BN_CHUNKS + z) * cmax + ch];
-    ts += v.x;
-    tq += v.y;
-  }
-  const double mean_d = ts / (double)m;
-  const double var_d = fmax(tq / (double)m - mean_d * mean_d, 0.0);
-  const float mean = (float)mean_d;
-  const float inv = rsqrtf((float)var_d + 1e-5f);
-  if (w == 0 && blockIdx.z == 0) {
-    d.mean[ch] = mean;
-    d.inv[ch] = inv;
-  }
+  const float mean = d.mean[ch], inv = d.inv[ch];
   const int* ws = wsel_override ? wsel_override : d.wsel;
   const float* P = d.params + (ws ? (int64_t)ws[d.wsel_idx] * d.wsel_stride : 0);
-  const float g = P[d.off_gamma + ch], b = P[d.off_beta + ch];
+  const float sc = P[d.off_gamma + ch] * inv, b = P[d.off_beta + ch];
   bf16* h = (bf16*)d.h;
   const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
-  for (int64_t px = p0 + w; px < p1; px += 8)
-    h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(g * inv, d.c[px * d.C + ch] - mean, b), 0.f));
+  int64_t px = p0 + w;
+  for (; px + 24 < p1; px += 32) {
+    float v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) v[u] = d.c[(px + 8 * u) * d.C + ch];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      h[(px + 8 * u) * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(sc, v[u] - mean, b), 0.f));
+  }
+  for (; px < p1; px += 8)
+    h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(sc, d.c[px * d.C + ch] - mean, b), 0.f));
+}
+
+// Backward through ReLU and the batch normalisation on channel-last bf16 activations, same
+// block layout as the forward: dy = dh where h > 0, xhat = (c - mean) inv; the stats blocks
+// sum dy and dy xhat per channel and chunk, the last block of a (channel group, problem)
+// combines the chunks in float64 in chunk order into dbeta and dgamma (the gradient slots);
+// the apply blocks write dc = gamma inv (dy - dbeta / m - xhat dgamma / m) in bf16.
+__global__ void __launch_bounds__(256) k_bn_back_stats_hwc(const BnDesc* __restrict__ descs,
+                                                           float2* __restrict__ part, int cmax,
+                                                           unsigned* __restrict__ counters) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int lane = threadIdx.x & 31;
+  const int ch = blockIdx.x * 32 + lane;
+  const int w = threadIdx.x >> 5;
+  const int64_t m = (int64_t)d.n << d.lhw;
+  const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
+  __shared__ float sh[8][32][2];
+  __shared__ int is_last;
+  const bf16* h = (const bf16*)d.h;
+  float sb = 0.f, sg = 0.f;
+  if (ch < d.C) {
+    const float mean = d.mean[ch], inv = d.inv[ch];
+    int64_t px = p0 + w;
+    for (; px + 24 < p1; px += 32) {
+      float hv[4], dv[4], cv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int64_t o = (px + 8 * u) * d.C + ch;
+        hv[u] = __bfloat162float(h[o]);
+        dv[u] = d.dh[o];
+        cv[u] = d.c[o];
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float dy = hv[u] > 0.f ? dv[u] : 0.f;
+        sb += dy;
+        sg = fmaf(dy, (cv[u] - mean) * inv, sg);
+      }
+    }
+    for (; px < p1; px += 8) {
+      const int64_t o = px * d.C + ch;
+      const float dy = __bfloat162float(h[o]) > 0.f ? d.dh[o] : 0.f;
+      sb += dy;
+      sg = fmaf(dy, (d.c[o] - mean) * inv, sg);
+    }
+  }
+  sh[w][lane][0] = sb;
+  sh[w][lane][1] = sg;
+  __syncthreads();
+  float2* pp = part + (int64_t)blockIdx.y * BN_CHUNKS * cmax;
+  if (w == 0 && ch < d.C) {
+    float tb = 0.f, tg = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      tb += sh[i][lane][0];
+      tg += sh[i][lane][1];
+    }
+    pp[(int64_t)blockIdx.z * cmax + ch] = make_float2(tb, tg);
+  }
+  __threadfence();
+  __syncthreads();
+  unsigned* cnt = counters + (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
+  if (threadIdx.x == 0) is_last = atomicAdd(cnt, 1u) == BN_CHUNKS - 1;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  if (w == 0 && ch < d.C) {
+    double tb = 0.0, tg = 0.0;
+    for (int z = 0; z < BN_CHUNKS; ++z) {
+      const float2 v = __ldcg(&pp[(int64_t)z * cmax + ch]);
+      tb += v.x;
+      tg += v.y;
+    }
+    d.dparams[d.off_gamma + ch] = (float)tg;
+    d.dparams[d.off_beta + ch] = (float)tb;
+  }
+  if (threadIdx.x == 0) *cnt = 0u;
+}
+
+__global__ void __launch_bounds__(256) k_bn_back_apply_hwc(const BnDesc* __restrict__ descs) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int ch = blockIdx.x * 32 + (threadIdx.x & 31);
+  const int w = threadIdx.x >> 5;
+  if (ch >= d.C) return;
+  const int64_t m = (int64_t)d.n << d.lhw;
+  const float mean = d.mean[ch], inv = d.inv[ch];
+  const float* P = d.params + (d.wsel ? (int64_t)d.wsel[d.wsel_idx] * d.wsel_stride : 0);
+  const float gi = P[d.off_gamma + ch] * inv;
+  const float k1 = d.dparams[d.off_beta + ch] / (float)m;
+  const float k2 = d.dparams[d.off_gamma + ch] / (float)m;
+  const bf16* h = (const bf16*)d.h;
+  bf16* dc = (bf16*)d.dc;
+  const int64_t p0 = m * blockIdx.z / BN_CHUNKS, p1 = m * (blockIdx.z + 1) / BN_CHUNKS;
+  int64_t px = p0 + w;
+  for (; px + 24 < p1; px += 32) {
+    float hv[4], dv[4], cv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t o = (px + 8 * u) * d.C + ch;
+      hv[u] = __bfloat162float(h[o]);
+      dv[u] = d.dh[o];
+      cv[u] = d.c[o];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float dy = hv[u] > 0.f ? dv[u] : 0.f;
+      dc[(px + 8 * u) * d.C + ch] = __float2bfloat16_rn(gi * (dy - k1 - (cv[u] - mean) * inv * k2));
+    }
+  }
+  for (; px < p1; px += 8) {
+    const int64_t o = px * d.C + ch;
+    const float dy = __bfloat162float(h[o]) > 0.f ? d.dh[o] : 0.f;
+    dc[o] = __float2bfloat16_rn(gi * (dy - k1 - (d.c[o] - mean) * inv * k2));
+  }
 }
 
 // [o][c][ky][kx] -> [o][ky][kx][c] (conv weights in (tap, channel) order).
@@ -785,15 +934,27 @@ void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
 }
 
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        float* part, cudaStream_t st) {
+                        float* part, unsigned* counters, cudaStream_t st) {
   const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
-  launch_pdl(ctc::k_bn_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels);
-  launch_pdl(ctc::k_bn_apply_hwc, grid, dim3(256), 0, st, descs, (const float2*)part, channels,
-             wsel);
+  launch_pdl(ctc::k_bn_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels,
+             counters);
+  launch_pdl(ctc::k_bn_apply_hwc, grid, dim3(256), 0, st, descs, wsel);
+}
+
+void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
+                                 float* part, unsigned* counters, cudaStream_t st) {
+  const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
+  launch_pdl(ctc::k_bn_back_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels,
+             counters);
+  launch_pdl(ctc::k_bn_back_apply_hwc, grid, dim3(256), 0, st, descs);
 }
 
 int64_t bn_hwc_part_floats(int n_problems, int channels) {
   return (int64_t)n_problems * ctc::BN_CHUNKS * channels * 2;
+}
+
+int64_t bn_hwc_counters(int n_problems, int channels) {
+  return (int64_t)n_problems * ((channels + 31) / 32);
 }
 
 namespace {

@@ -102,9 +102,15 @@ void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
                        const RelayoutC& r, cudaStream_t st);
 // Batch normalisation (training mode) + ReLU on fp32 channel-last input into bf16 channel-last
 // output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels); part holds
-// bn_hwc_part_floats(n_problems, channels) floats of per-chunk sums.
+// bn_hwc_part_floats(n_problems, channels) floats of per-chunk sums; counters holds
+// bn_hwc_counters(n_problems, channels) zeroed unsigned ints (the launch leaves them zero).
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        float* part, cudaStream_t st);
+                        float* part, unsigned* counters, cudaStream_t st);
+// Backward of launch_bn_relu_hwc (BnDesc: c, h, mean, inv, params, dh fp32, dc bf16, dparams),
+// with the same part and counters buffers.
+void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
+                                 float* part, unsigned* counters, cudaStream_t st);
 int64_t bn_hwc_part_floats(int n_problems, int channels);
+int64_t bn_hwc_counters(int n_problems, int channels);
 
 }  // namespace lipz

@@ -105,6 +105,7 @@ struct DcPlan {
   // from class-major weight copies, channel-last activations and batch norm
   bool tcg = false, tct = false;
   float* bnpart = nullptr;
+  unsigned* bncnt = nullptr;
   CtcParams tgp[4], tdp[4];
   ConvTcDesc *tgd[4], *tdd[4];
   // tensor-core input gradients: the discriminator's as parity-class transposed convolutions
@@ -587,6 +588,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     }
     p->gwt_ps = (off + 63) / 64 * 64;
     ok = ok && !dev_alloc(p, &p->bnpart, (size_t)bn_hwc_part_floats(PE, 8 * g) * 4, msg);
+    ok = ok && !dev_alloc(p, &p->bncnt, (size_t)bn_hwc_counters(PE, 8 * g) * 4, msg);
+    if (ok) ok = cudaMemset(p->bncnt, 0, (size_t)bn_hwc_counters(PE, 8 * g) * 4) == cudaSuccess;
     ok = ok && !dev_alloc(p, &p->Gwt, (size_t)s.n_indiv * p->gwt_ps * 2, msg);
     if (ok) ok = cudaMemset(p->Gwt, 0, (size_t)s.n_indiv * p->gwt_ps * 2) == cudaSuccess;
     for (int i = 0; i < 4 && ok; ++i) {
@@ -898,7 +901,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     return nullptr;
   }
   p->eval_launches = 9 + 5 * C;
-  p->train_launches = tct ? 56 : 50;
+  p->train_launches = tct ? 60 : 50;
   return p;
 }
 
@@ -927,13 +930,14 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
     launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
                 nullptr, 0, s.slope, st);
-    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, st);
+    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->gp[i];
       q.descs = p->gtd[i];
       q.wsel = nbr;
       launch_conv_tc(p->mG[i], q, p->sms, st);
-      if (i < 3) launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, st);
+      if (i < 3)
+        launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, p->bncnt, st);
     }
     return check(msg, "DCGAN generator evaluation (tensor cores)");
   }
@@ -991,13 +995,14 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   if (p->tct) {
     launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
                 nullptr, 0, s.slope, st);
-    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, st);
+    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->tgp[i];
       q.descs = p->tgd[i];
       q.wsel = p->b.src_g;
       launch_conv_tc(p->mG[i], q, p->sms, st);
-      if (i < 3) launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, st);
+      if (i < 3)
+        launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, p->bncnt, st);
     }
   } else {
     for (int l = 1; l <= 5; ++l) {
@@ -1100,7 +1105,10 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
         launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
                     B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
       }
-      launch_bn_relu_backward(s.bf, p->gbn[k], C, gc[l - 1], st);
+      if (p->tct)
+        launch_bn_relu_backward_hwc(p->gbn[k], C, gc[l - 1], p->bnpart, p->bncnt, st);
+      else
+        launch_bn_relu_backward(s.bf, p->gbn[k], C, gc[l - 1], st);
     }
   }
   return check(msg, "DCGAN training step");
