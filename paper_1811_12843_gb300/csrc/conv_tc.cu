@@ -30,13 +30,32 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = 256 * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 320;  // warp 0 TMA, 1 MMA, 2-5 gather, 6-9 epilogue
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+// first-layer input patches: 3 channels x 10 rows x 72 columns (64 interior at column 4)
+constexpr int PATCH_BYTES = 4352;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256 + 3 * PATCH_BYTES;
 constexpr int LAG = 2;  // copy groups a gather thread keeps in flight (< STAGES)
 
 // 16-byte global -> shared copy; bytes = 0 writes zeros (src must still be a valid address)
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes)
                : "memory");
+}
+__device__ __forceinline__ void cp_async8(uint32_t dst, const void* src, int bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(bytes)
+               : "memory");
+}
+
+// Barrier of the four gather warps (named barrier 1) that returns whether any thread passed
+// true.
+__device__ __forceinline__ bool gather_bar_or(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 128, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)pred)
+      : "memory");
+  return r != 0;
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -163,12 +182,85 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp < 6) {
     // ---- A operand: thread r gathers row r of every k chunk. Channel-last rows arrive by
     // 16-byte cp.async (zero fill outside the image), a stage marked full LAG chunks later once
-    // its copy group has landed; the first layer's CHW rows are converted through registers.
+    // its copy group has landed; the first layer's rows are built from staged input patches.
     const int r = threadIdx.x - 64;
     int stage = 0, arr_stage = 0, pending = 0;
     uint32_t phase = 0;
     bool ok = true;
     const int lhi = p.lhi, Hi = 1 << lhi;
+    if (p.nchw_in) {
+      // first layer (3 channels, 64 x 64 CHW images, 32 x 32 outputs, one k chunk of
+      // k = (ky * 4 + kx) * 3 + c over 48 values): a tile's 128 rows are 4 output rows, fed by
+      // a 3 x 10 x 64 input patch that the gather threads copy one tile ahead by 8-byte
+      // cp.async into one of three shared buffers whose halo columns stay zero
+      uint8_t* patches = misc + 256;
+      const uint32_t patch0 = smem_u32(patches);
+      for (int i = r; i < 3 * PATCH_BYTES / 16; i += 128)
+        *reinterpret_cast<uint4*>(patches + 16 * i) = make_uint4(0u, 0u, 0u, 0u);
+      gather_bar_or(false);
+      auto prefetch = [&](int tile, int buf) {
+        if (tile < p.n_tiles) {
+          const ConvTcDesc d = p.descs[tile / p.mtiles];
+          const int m0 = (tile % p.mtiles) * BM;
+          const int nb = m0 >> 10, oy0 = (m0 >> 5) & 31;
+          for (int u = r; u < 480; u += 128) {
+            const int c = u / 160, rem = u - c * 160, pr = rem >> 4, q = rem & 15;
+            const int iy = 2 * oy0 - 1 + pr;
+            const bool in = iy >= 0 && iy < 64;
+            const bf16* src = in ? d.in + ((int64_t)(nb * 3 + c) << 12) + (iy << 6) + 4 * q : d.in;
+            cp_async8(patch0 + (uint32_t)(buf * PATCH_BYTES + ((c * 10 + pr) * 72 + 4 + 4 * q) * 2),
+                      src, in ? 8 : 0);
+          }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+      };
+      prefetch(blockIdx.x, 0);
+      int buf = 0;
+      const int ox = r & 31, oyl = r >> 5;
+      for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
+        prefetch(tile + gridDim.x, buf == 2 ? 0 : buf + 1);
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+        const bool okw = mbar_wait_warp(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 27);
+        if (gather_bar_or(!okw)) {
+          ok = false;
+          break;
+        }
+        const bool valid = (tile % p.mtiles) * BM + r < M;
+        const unsigned short* pb =
+            reinterpret_cast<const unsigned short*>(patches + buf * PATCH_BYTES);
+        const uint32_t row = base + stage * STAGE_BYTES + (uint32_t)r * 128u;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          uint32_t w[4];
+#pragma unroll
+          for (int e2 = 0; e2 < 4; ++e2) {
+            uint32_t hv[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int k = u * 8 + e2 * 2 + h;
+              hv[h] = 0u;
+              if (k < 48) {
+                const int tap = k / 3, c = k - 3 * tap;
+                const int prow = 2 * oyl + (tap >> 2), col = 2 * ox + (tap & 3) + 3;
+                hv[h] = valid ? (uint32_t)pb[(c * 10 + prow) * 72 + col] : 0u;
+              }
+            }
+            w[e2] = hv[0] | (hv[1] << 16);
+          }
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                           row + ((uint32_t)(u ^ (r & 7)) << 4)),
+                       "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                       : "memory");
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_arrive(bFullA + 8 * stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+        buf = buf == 2 ? 0 : buf + 1;
+      }
+    } else
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
       const int pc = tile / p.mtiles;
       const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
@@ -188,34 +280,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           const uint32_t row = base + stage * STAGE_BYTES + (uint32_t)r * 128u;
-          if (p.nchw_in) {
-            // first layer: k = (ky * 4 + kx) * 3 + c over 48 values, CHW image input
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              uint32_t w[4];
-#pragma unroll
-              for (int e2 = 0; e2 < 4; ++e2) {
-                float f[2];
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                  const int k = u * 8 + e2 * 2 + h;
-                  f[h] = 0.f;
-                  if (valid && k < 48) {
-                    const int tap = k / 3, c = k - 3 * tap;
-                    const int iy = 2 * oy - 1 + (tap >> 2), ix = 2 * ox - 1 + (tap & 3);
-                    if (iy >= 0 && iy < Hi && ix >= 0 && ix < Hi)
-                      f[h] = __bfloat162float(
-                          d.in[((int64_t)(nb * 3 + c) << (2 * lhi)) + (iy << lhi) + ix]);
-                  }
-                }
-                w[e2] = pack_bf16(f[0], f[1]);
-              }
-              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                               row + ((uint32_t)(u ^ (r & 7)) << 4)),
-                           "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                           : "memory");
-            }
-          } else {
+          {
             // channel-last input with ci a multiple of 64: one tap, 64 channels per chunk.
             // Convolution: tap (ky, kx) of 16, input pixel (2 oy - 1 + ky, 2 ox - 1 + kx).
             // Transposed (stride 2, pad 1, by class): tap (u, v) of 4, ky = (oy + 1) mod 2 + 2u,
@@ -249,10 +314,6 @@ __global__ void __launch_bounds__(THREADS, 1)
               arr_stage = arr_stage + 1 == STAGES ? 0 : arr_stage + 1;
               --pending;
             }
-          }
-          if (p.nchw_in) {
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            mbar_arrive(bFullA + 8 * stage);
           }
           if (++stage == STAGES) {
             stage = 0;

@@ -26,7 +26,8 @@ struct ConvTcDesc {
 // A launch: problems of `rows` images; 4x4 / stride 2 / pad 1 convolution from ci x 2^lhi
 // squared to co x 2^lho squared; K = 16 ci in (ky, kx, ci) order, kchunks = ceil(K / 64);
 // jobs of nbox = min(co, 256) output channels (nj of them); tiles of 128 output pixels
-// (mtiles per problem). The weight map spans [individual][co][K] bf16.
+// (mtiles per problem). The weight map spans [individual][co][K] bf16. nchw_in: the first
+// layer, which takes only 3-channel channel-major 64 x 64 images (ci 3, lhi 6, lho 5).
 // transposed: a stride-2 / pad-1 transposed convolution computed by output parity class (tiles
 // over problem x 4 classes x mtiles; K = 4 ci in (tap, ci) order; the weights of class cls
 // start at row cls * cls_rows of the map). out_mode: CTC_LRELU_HWC (bf16 LeakyReLU,
