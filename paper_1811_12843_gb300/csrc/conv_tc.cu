@@ -59,7 +59,8 @@ __device__ __forceinline__ bool gather_bar_or(bool pred) {
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
-    k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CtcParams p) {
+    k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mA,
+              const __grid_constant__ CtcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -112,13 +113,37 @@ __global__ void __launch_bounds__(THREADS, 1)
         const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
         const int cls = p.transposed ? (pc & 3) : 0;
         const int indiv = __ldg(&p.wsel[d.wsel_idx]);
+        // channel-last A rows by TMA (a_tma): the tile is 128 consecutive output pixels (class
+        // pixels when transposed) of whole rows; its origin is image n0, row y0
+        const int m0 = (tile % p.mtiles) * BM;
+        const int n0 = m0 >> (2 * lq), y0 = (m0 >> lq) & ((1 << lq) - 1);
         for (int j = 0; j < p.nj && ok; ++j)
           for (int kc = 0; kc < p.kchunks; ++kc) {
             if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 21)) {
               ok = false;
               break;
             }
-            mbar_expect_tx(bFullB + 8 * stage, (uint32_t)(nbox * BK * 2));
+            mbar_expect_tx(bFullB + 8 * stage,
+                           (uint32_t)(nbox * BK * 2 + (p.a_tma ? A_BYTES : 0)));
+            if (p.a_tma) {
+              // Convolution: tap (ky, kx), input rows 2 y - 1 + ky, columns 2 x - 1 + kx (the
+              // map's traversal stride 2). Transposed, class (a, b), tap (u, v): ky = (a + 1)
+              // mod 2 + 2u, input row y + (a + 1 - ky) / 2, column x + (b + 1 - kx) / 2.
+              const int k0 = kc * BK;
+              const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
+              int x, y;
+              if (p.transposed) {
+                const int a = cls >> 1, b = cls & 1;
+                const int ky = ((a + 1) & 1) + 2 * (tap >> 1), kx = ((b + 1) & 1) + 2 * (tap & 1);
+                y = y0 + ((a + 1 - ky) >> 1);
+                x = (b + 1 - kx) >> 1;
+              } else {
+                y = 2 * y0 - 1 + (tap >> 2);
+                x = (tap & 3) - 1;
+              }
+              tma_load_5d(base + stage * STAGE_BYTES, &mA, bFullB + 8 * stage, c0, x, y, n0,
+                          p.transposed ? pc >> 2 : pc);
+            }
             tma_load_3d(base + stage * STAGE_BYTES + A_BYTES, &mW, bFullB + 8 * stage, kc * BK,
                         cls * p.cls_rows + j * 256, indiv);
             issued[stage]++;
@@ -154,7 +179,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           tc_fence_after();
           const uint32_t dt = tmem + (uint32_t)(R * 256);
           for (int kc = 0; kc < p.kchunks; ++kc) {
-            if (!mbar_wait(bFullA + 8 * stage, phase, abort_flag, p.err, 24) ||
+            if ((!p.a_tma && !mbar_wait(bFullA + 8 * stage, phase, abort_flag, p.err, 24)) ||
                 !mbar_wait(bFullB + 8 * stage, phase, abort_flag, p.err, 25)) {
               ok = false;
               break;
@@ -179,7 +204,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 26);
     }
-  } else if (warp < 6) {
+  } else if (warp < 6 && !p.a_tma) {
     // ---- A operand: thread r gathers row r of every k chunk. Channel-last rows arrive by
     // 16-byte cp.async (zero fill outside the image), a stage marked full LAG chunks later once
     // its copy group has landed; the first layer's rows are built from staged input patches.
@@ -328,7 +353,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_arrive(bFullA + 8 * arr_stage);
       arr_stage = arr_stage + 1 == STAGES ? 0 : arr_stage + 1;
     }
-  } else {
+  } else if (warp >= 6) {
     // ---- epilogue: LeakyReLU, bf16, channel-last rows
     const int q = warp & 3;
     const int row = q * 32 + lane;
@@ -1020,10 +1045,8 @@ int64_t bn_hwc_counters(int n_problems, int channels) {
 
 namespace {
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_ctc = nullptr;
-}
 
-bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t depth,
-                  uint64_t depth_elems, uint32_t box_rows, std::string* msg) {
+bool ensure_encode(std::string* msg) {
   if (!g_encode_ctc) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;
@@ -1035,6 +1058,13 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
     }
     g_encode_ctc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
   }
+  return true;
+}
+}  // namespace
+
+bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t depth,
+                  uint64_t depth_elems, uint32_t box_rows, std::string* msg) {
+  if (!ensure_encode(msg)) return false;
   cuuint64_t dims[3] = {K, rows, depth};
   cuuint64_t strides[2] = {K * 2, depth_elems * 2};
   cuuint32_t box[3] = {64, box_rows, 1};
@@ -1050,6 +1080,40 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
   return true;
 }
 
+bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
+                      std::string* msg) {
+  q->a_tma = 0;
+  if (q->nchw_in || q->ci % 64 != 0 || n_probs < 1) return true;
+  const int lq = q->lho - q->transposed;
+  if (lq > 7) return true;
+  const int64_t Wi = (int64_t)1 << q->lhi;
+  const int64_t per = (int64_t)q->rows * Wi * Wi * q->ci;  // elements of one problem's input
+  int64_t pstride = per;
+  if (n_probs > 1) pstride = (int64_t)(descs[1].in - descs[0].in);
+  if (pstride < per || pstride % 8 != 0) return true;
+  for (int k = 1; k < n_probs; ++k)
+    if (descs[k].in != descs[0].in + (int64_t)k * pstride) return true;
+  if (!ensure_encode(msg)) return false;
+  const int stride = q->transposed ? 1 : 2;
+  const int tw = 1 << lq, th = std::min(1 << lq, 128 / tw), tn = std::max(1, 128 / (tw * th));
+  cuuint64_t dims[5] = {(cuuint64_t)q->ci, (cuuint64_t)Wi, (cuuint64_t)Wi, (cuuint64_t)q->rows,
+                        (cuuint64_t)n_probs};
+  cuuint64_t strides[4] = {(cuuint64_t)q->ci * 2, (cuuint64_t)(Wi * q->ci * 2),
+                           (cuuint64_t)(Wi * Wi * q->ci * 2), (cuuint64_t)(pstride * 2)};
+  cuuint32_t box[5] = {64, (cuuint32_t)(tw * stride), (cuuint32_t)(th * stride), (cuuint32_t)tn, 1};
+  cuuint32_t es[5] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1, 1};
+  CUresult r = g_encode_ctc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
+                            const_cast<bf16*>(descs[0].in), dims, strides, box, es,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (convolution activations) failed: " + std::to_string((int)r);
+    return false;
+  }
+  q->a_tma = 1;
+  return true;
+}
+
 bool ctc_prepare(std::string* msg) {
   if (cudaFuncSetAttribute(ctc::k_conv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            ctc::SMEM_BYTES) != cudaSuccess) {
@@ -1060,9 +1124,10 @@ bool ctc_prepare(std::string* msg) {
   return true;
 }
 
-void launch_conv_tc(const CUtensorMap& mW, const CtcParams& p, int sms, cudaStream_t st) {
+void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
+                    cudaStream_t st) {
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
-  launch_pdl(ctc::k_conv_tc, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, p);
+  launch_pdl(ctc::k_conv_tc, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, mA, p);
 }
 
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,

@@ -41,6 +41,7 @@ struct CtcParams {
   const ConvTcDesc* descs;
   int rows, ci, lhi, co, lho, nchw_in, kchunks, nj, nbox, mtiles, n_tiles;
   int transposed, out_mode, cls_rows;
+  int a_tma;  // A rows by TMA through the activation map (set by ctc_make_act_map)
   const int* wsel;
   float slope;
   int* err;
@@ -86,8 +87,16 @@ void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st);
 
 bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t depth,
                   uint64_t depth_elems, uint32_t box_rows, std::string* msg);
+// Activation map of a launch whose problems' channel-last inputs (ci a multiple of 64) sit at
+// a uniform stride from descs[0].in: dims (ci, W, W, rows, problems), a box of 64 channels by
+// the input pixels of 128 output pixels (traversal stride 2 for the convolution, 1 for the
+// parity classes). Sets q->a_tma = 1 when it applies (else 0, and the gather warps load A);
+// false only when the driver refuses the map.
+bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
+                      std::string* msg);
 bool ctc_prepare(std::string* msg);
-void launch_conv_tc(const CUtensorMap& mW, const CtcParams& p, int sms, cudaStream_t st);
+void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
+                    cudaStream_t st);
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,
                        cudaStream_t st);
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,

@@ -125,6 +125,9 @@ struct DcPlan {
   CUtensorMap mG[4];
   CtcParams gp[4];
   ConvTcDesc* gtd[4];
+  // activation maps of the channel-last tensor-core launches (A rows by TMA): evaluation D
+  // and G, training forwards, D-loss and G-loss input gradients, generator input gradients
+  CUtensorMap aEd[4], aEg[4], aTg[4], aTd[4], aDd[3], aGd[4], aGc[4];
   // tensor-core weight gradients of the layers whose channel counts fill the tiles
   bool wtc_d[4] = {}, wtc_g[5] = {};
   WgtcParams wdp[4], wgp[5];
@@ -547,6 +550,10 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
       ok = ok && !upload(p, &p->tcd[l - 1], vt, msg);
+      // one map serves every cell: the chunk buffers are shared
+      ok = ok && ctc_make_act_map(&p->aEd[l - 1], &p->cp[l - 1], vt.data(), 5, msg);
+      for (size_t k = 5; k < vt.size(); ++k)
+        if (vt[k].in != vt[k % 5].in) p->cp[l - 1].a_tma = 0;
     }
     std::vector<LogitDesc> vl;
     for (int c = 0; c < C; ++c)
@@ -629,6 +636,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
       ok = ok && !upload(p, &p->gtd[i], vt, msg);
+      ok = ok && ctc_make_act_map(&p->aEg[i], &p->gp[i], vt.data(), PE, msg);
     }
   }
   // ---- tensor-core training forward (channel-last), and the output layer's descriptors in
@@ -650,6 +658,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->tgd[i], vt, msg);
+      ok = ok && ctc_make_act_map(&p->aTg[i], &p->tgp[i], vt.data(), C, msg);
     }
     for (int l = 1; l <= 4 && ok; ++l) {
       CtcParams q = p->cp[l - 1];
@@ -667,6 +676,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->tdd[l - 1], vt, msg);
+      ok = ok && ctc_make_act_map(&p->aTd[l - 1], &p->tdp[l - 1], vt.data(), C, msg);
     }
     std::vector<LogitDesc> vl, vd, vg;
     for (int c = 0; c < C; ++c) {
@@ -760,9 +770,11 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
         if (chain == 0) {
+          ok = ctc_make_act_map(&p->aDd[4 - l], &q, vt.data(), C, msg);
           p->ddp[4 - l] = q;
           ok = !upload(p, &p->ddd[4 - l], vt, msg);
         } else {
+          ok = ctc_make_act_map(&p->aGd[4 - l], &q, vt.data(), C, msg);
           p->gdp[4 - l] = q;
           ok = !upload(p, &p->gdd[4 - l], vt, msg);
         }
@@ -816,6 +828,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->gcd[i], vt, msg);
+      ok = ok && ctc_make_act_map(&p->aGc[i], &p->gcp[i], vt.data(), C, msg);
     }
     // weight gradients: a = the output's delta (discriminator) or the layer's input
     // (generator), M = its channels; b = the other operand, gathered per tap
@@ -935,7 +948,7 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
       CtcParams q = p->gp[i];
       q.descs = p->gtd[i];
       q.wsel = nbr;
-      launch_conv_tc(p->mG[i], q, p->sms, st);
+      launch_conv_tc(p->mG[i], p->aEg[i], q, p->sms, st);
       if (i < 3)
         launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, p->bncnt, st);
     }
@@ -967,7 +980,7 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
         CtcParams q = p->cp[l - 1];
         q.descs = p->tcd[l - 1] + c * 5;
         q.wsel = nbr;
-        launch_conv_tc(p->mW[l - 1], q, p->sms, st);
+        launch_conv_tc(p->mW[l - 1], p->aEd[l - 1], q, p->sms, st);
       }
       launch_logit_dot(true, p->tcl + c * 5, 5, 6 * B, nbr, st);
     }
@@ -1000,7 +1013,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->tgp[i];
       q.descs = p->tgd[i];
       q.wsel = p->b.src_g;
-      launch_conv_tc(p->mG[i], q, p->sms, st);
+      launch_conv_tc(p->mG[i], p->aTg[i], q, p->sms, st);
       if (i < 3)
         launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, p->bncnt, st);
     }
@@ -1026,7 +1039,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->tdp[l - 1];
       q.descs = p->tdd[l - 1];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mW[l - 1], q, p->sms, st);
+      launch_conv_tc(p->mW[l - 1], p->aTd[l - 1], q, p->sms, st);
     }
     launch_logit_dot(true, p->tdl_tc, C, 2 * B, nullptr, st);
   } else {
@@ -1061,7 +1074,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->ddp[k];
       q.descs = p->ddd[k];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mDd[l - 1], q, p->sms, st);
+      launch_conv_tc(p->mDd[l - 1], p->aDd[k], q, p->sms, st);
     } else if (l >= 2) {
       launch_conv(CONVT2_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
                   2 * B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0, s.slope,
@@ -1076,7 +1089,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->gdp[4 - l];
       q.descs = p->gdd[4 - l];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mDd[l - 1], q, p->sms, st);
+      launch_conv_tc(p->mDd[l - 1], p->aGd[4 - l], q, p->sms, st);
     } else {
       launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
                   p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
@@ -1100,7 +1113,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
         CtcParams q = p->gcp[k];
         q.descs = p->gcd[k];
         q.wsel = p->b.src_g;
-        launch_conv_tc(p->mGc[k], q, p->sms, st);
+        launch_conv_tc(p->mGc[k], p->aGc[k], q, p->sms, st);
       } else {
         launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
                     B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
