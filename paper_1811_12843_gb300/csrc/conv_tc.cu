@@ -700,52 +700,64 @@ __global__ void __launch_bounds__(256) k_wgrad_tc_reduce(const __grid_constant__
   for (int i = threadIdx.x; i < 1024; i += 256) out[i] = tile[i & 15][i >> 4];
 }
 
-// [out][in][ky][kx] -> [out][ky][kx][in] for the five discriminator tensors of every
-// individual (bf16 copies).
-__global__ void k_relayout_d(const bf16* __restrict__ src, bf16* __restrict__ dst, int n_indiv,
-                             int64_t Ps, RelayoutD r) {
+// Weight re-layouts, one block per (output row of one tensor, individual); channels pass
+// through shared memory in chunks of RL_CH so that reads and writes are contiguous runs.
+constexpr int RL_CH = 256;
+struct RelayoutRows {
+  int n;
+  int64_t src_off[5], dst_off[5];
+  int o[5], c[5];
+};
+
+// [o][c][ky][kx] -> [o][ky][kx][c]
+__global__ void __launch_bounds__(256) k_relayout_rows(const bf16* __restrict__ src, int64_t src_ps,
+                                                       bf16* __restrict__ dst, int64_t dst_ps,
+                                                       RelayoutRows r) {
+  __shared__ bf16 sh[16][RL_CH + 2];
   pdl_wait();
-  const int64_t total = (int64_t)n_indiv * r.P;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t ind = e / r.P, k = e - ind * r.P;
-    int l = 0;
-    while (l + 1 < 5 && k >= r.off[l + 1]) ++l;
-    const int64_t i = k - r.off[l];
-    const int ci = r.ci[l];
-    // destination index i = (o * 16 + tap) * ci + c
-    const int64_t c = i % ci, t = (i / ci) & 15, o = i / (16 * (int64_t)ci);
-    dst[ind * Ps + k] = src[ind * Ps + r.off[l] + (o * ci + c) * 16 + t];
+  int row = blockIdx.x, l = 0;
+  while (l + 1 < r.n && row >= r.o[l]) row -= r.o[l++];
+  const int c = r.c[l];
+  const bf16* sp = src + blockIdx.y * src_ps + r.src_off[l] + (int64_t)row * c * 16;
+  bf16* dp = dst + blockIdx.y * dst_ps + r.dst_off[l] + (int64_t)row * c * 16;
+  for (int cb = 0; cb < c; cb += RL_CH) {
+    const int n = c - cb < RL_CH ? c - cb : RL_CH;
+    for (int e = threadIdx.x; e < n * 16; e += 256) sh[e & 15][e >> 4] = sp[cb * 16 + e];
+    __syncthreads();
+    for (int e = threadIdx.x; e < n * 16; e += 256) {
+      const int t = e / n, cc = e - t * n;
+      dp[t * c + cb + cc] = sh[t][cc];
+    }
+    __syncthreads();
   }
 }
 
 // Generator transposed-convolution weights [in][out][ky][kx] -> by output parity class
 // [class][out][tap][in] (tap (u, v): ky = (py + 1) mod 2 + 2u, kx = (px + 1) mod 2 + 2v), rows
-// of a class cls_rows apart (the padding rows are left as they are: zero).
-__global__ void k_relayout_g(const bf16* __restrict__ src, int64_t src_ps, bf16* __restrict__ dst,
-                             int64_t dst_ps, int n_indiv, RelayoutG r) {
+// of a class cls_rows apart (the padding rows are left as they are: zero). One block per
+// (output channel o of one tensor, individual).
+__global__ void __launch_bounds__(256) k_relayout_g(const bf16* __restrict__ src, int64_t src_ps,
+                                                    bf16* __restrict__ dst, int64_t dst_ps,
+                                                    RelayoutG r) {
+  __shared__ bf16 sh[16][RL_CH + 2];
   pdl_wait();
-  int64_t total = 0;
-  for (int l = 0; l < r.n; ++l) total += (int64_t)r.ci[l] * r.co[l] * 16;
-  total *= n_indiv;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    int64_t per = 0;
-    for (int l = 0; l < r.n; ++l) per += (int64_t)r.ci[l] * r.co[l] * 16;
-    const int64_t ind = e / per;
-    int64_t k = e - ind * per;
-    int l = 0;
-    while (k >= (int64_t)r.ci[l] * r.co[l] * 16) {
-      k -= (int64_t)r.ci[l] * r.co[l] * 16;
-      ++l;
+  int o = blockIdx.x, l = 0;
+  while (l + 1 < r.n && o >= r.co[l]) o -= r.co[l++];
+  const int ci = r.ci[l], co = r.co[l];
+  const bf16* sp = src + blockIdx.y * src_ps + r.src_off[l] + (int64_t)o * 16;
+  bf16* dp = dst + blockIdx.y * dst_ps + r.dst_off[l];
+  for (int cb = 0; cb < ci; cb += RL_CH) {
+    const int n = ci - cb < RL_CH ? ci - cb : RL_CH;
+    for (int e = threadIdx.x; e < n * 16; e += 256)
+      sh[e & 15][e >> 4] = sp[(int64_t)(cb + (e >> 4)) * co * 16 + (e & 15)];
+    __syncthreads();
+    for (int e = threadIdx.x; e < n * 16; e += 256) {
+      const int ct = e / n, cc = e - ct * n;  // (class, tap) = ct
+      const int cls = ct >> 2, t = ct & 3;
+      const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1), kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
+      dp[(((int64_t)cls * r.cls_rows[l] + o) * 4 + t) * ci + cb + cc] = sh[ky * 4 + kx][cc];
     }
-    const int ci = r.ci[l], co = r.co[l];
-    // destination k = ((cls * co + o) * 4 + t) * ci + c
-    const int c = (int)(k % ci), t = (int)((k / ci) & 3);
-    const int o = (int)((k / (4 * ci)) % co), cls = (int)(k / (4 * (int64_t)ci * co));
-    const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1), kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
-    dst[ind * dst_ps + r.dst_off[l] + (((int64_t)cls * r.cls_rows[l] + o) * 4 + t) * ci + c] =
-        src[ind * src_ps + r.src_off[l] + (((int64_t)c * co + o) * 4 + ky) * 4 + kx];
+    __syncthreads();
   }
 }
 
@@ -967,28 +979,6 @@ __global__ void __launch_bounds__(256) k_bn_back_apply_hwc(const BnDesc* __restr
   }
 }
 
-// [o][c][ky][kx] -> [o][ky][kx][c] (conv weights in (tap, channel) order).
-__global__ void k_relayout_c(const bf16* __restrict__ src, int64_t src_ps, bf16* __restrict__ dst,
-                             int64_t dst_ps, int n_indiv, RelayoutC r) {
-  pdl_wait();
-  int64_t per = 0;
-  for (int l = 0; l < r.n; ++l) per += (int64_t)r.o[l] * r.c[l] * 16;
-  const int64_t total = per * n_indiv;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t ind = e / per;
-    int64_t k = e - ind * per;
-    int l = 0;
-    while (k >= (int64_t)r.o[l] * r.c[l] * 16) {
-      k -= (int64_t)r.o[l] * r.c[l] * 16;
-      ++l;
-    }
-    const int c = (int)(k % r.c[l]), t = (int)((k / r.c[l]) & 15);
-    const int64_t o = k / (16 * (int64_t)r.c[l]);
-    dst[ind * dst_ps + r.dst_off[l] + k] = src[ind * src_ps + r.src_off[l] + (o * r.c[l] + c) * 16 + t];
-  }
-}
-
 }  // namespace ctc
 
 bool wgtc_prepare(std::string* msg) {
@@ -1009,14 +999,26 @@ void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st) {
 
 void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutC& r, cudaStream_t st) {
-  launch_pdl(ctc::k_relayout_c, dim3(1216), dim3(256), 0, st, src, src_ps, dst, dst_ps, n_indiv,
-             r);
+  ctc::RelayoutRows q;
+  memset(&q, 0, sizeof q);
+  q.n = r.n;
+  int rows = 0;
+  for (int l = 0; l < r.n; ++l) {
+    q.src_off[l] = r.src_off[l];
+    q.dst_off[l] = r.dst_off[l];
+    q.o[l] = r.o[l];
+    q.c[l] = r.c[l];
+    rows += r.o[l];
+  }
+  launch_pdl(ctc::k_relayout_rows, dim3(rows, n_indiv), dim3(256), 0, st, src, src_ps, dst, dst_ps,
+             q);
 }
 
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutG& r, cudaStream_t st) {
-  launch_pdl(ctc::k_relayout_g, dim3(1216), dim3(256), 0, st, src, src_ps, dst, dst_ps, n_indiv,
-             r);
+  int rows = 0;
+  for (int l = 0; l < r.n; ++l) rows += r.co[l];
+  launch_pdl(ctc::k_relayout_g, dim3(rows, n_indiv), dim3(256), 0, st, src, src_ps, dst, dst_ps, r);
 }
 
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
@@ -1132,7 +1134,17 @@ void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParam
 
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,
                        cudaStream_t st) {
-  launch_pdl(ctc::k_relayout_d, dim3(1216), dim3(256), 0, st, src, dst, n_indiv, Ps, r);
+  ctc::RelayoutRows q;
+  memset(&q, 0, sizeof q);
+  q.n = 5;
+  int rows = 0;
+  for (int l = 0; l < 5; ++l) {
+    q.src_off[l] = q.dst_off[l] = r.off[l];
+    q.c[l] = r.ci[l];
+    q.o[l] = (int)((r.off[l + 1] - r.off[l]) / (16 * (int64_t)r.ci[l]));
+    rows += q.o[l];
+  }
+  launch_pdl(ctc::k_relayout_rows, dim3(rows, n_indiv), dim3(256), 0, st, src, Ps, dst, Ps, q);
 }
 
 }  // namespace lipz
