@@ -1,13 +1,17 @@
-// Tensor-core (tcgen05 / TMEM) implicit-GEMM convolution of the DCGAN discriminator's
-// evaluation: y[m][o] = LeakyReLU(sum_k A[m][k] W[o][k]) for the 4x4 / stride 2 / pad 1
-// convolutions, with m = (image, output row, output column) and k = (ky, kx, input channel).
-// Activations are channel-last (NHWC), so the A operand of one 64-wide k chunk is, for a layer
-// with at least 64 input channels, 128 contiguous bytes of one input pixel per row: four warps
-// gather it with 16-byte loads straight into the 128-byte-swizzled K-major layout the MMA
-// reads. The first layer reads the channel-major (CHW) images of the evaluation buffer with
-// scalar loads (K = 48). Weights, re-laid out as [out][ky][kx][in], arrive by TMA. One CTA per
-// SM over 128-row tiles; accumulators (up to 256 columns per job) alternate between two TMEM
-// regions so that the epilogue of one job overlaps the MMAs of the next.
+// Tensor-core (tcgen05 / TMEM) implicit-GEMM convolutions of the DCGAN networks:
+// y[m][o] = epilogue(sum_k A[m][k] W[o][k]) for the 4x4 / stride 2 / pad 1 convolutions, with
+// m = (image, output row, output column) and k = (ky, kx, input channel), and for the stride-2
+// transposed convolutions by output parity class (k = (tap of the class, input channel)).
+// Activations are channel-last (NHWC), so the A operand of one 64-wide k chunk is one tap's 64
+// channels of 128 input pixels: the TMA warp loads it through a 5-D activation map (channels,
+// columns, rows, images, problems) whose traversal stride 2 picks the convolution's input
+// pixels, or whose per-class row/column offset picks the transposed convolution's, straight
+// into the 128-byte-swizzled K-major layout the MMA reads. The 3-channel first layer reads
+// channel-major (CHW) images: four gather warps build its rows (K = 48) from input patches
+// staged in shared memory one tile ahead. Weights, re-laid out as [out][tap][in], arrive by
+// TMA. One CTA per SM over 128-row tiles; accumulators (up to 256 columns per job) alternate
+// between two TMEM regions so that the epilogue of one job overlaps the MMAs of the next.
+// The weight-gradient kernel (k_wgrad_tc) and the channel-last batch norm live here too.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
