@@ -10,6 +10,7 @@
 #include "conv_tc.h"
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <vector>
 
@@ -222,6 +223,15 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   // tensor-core training forward (both networks' widths multiples of 64): channel-last
   // activations, read by the CUDA-core backward kernels in that layout
   const bool tct = tcd && p->tcg;
+  // LIPZ_CONV_GATHER=1: the gather warps load every A tile and the activation maps stay
+  // unused (the tests check that both ways of loading A give bit-identical results)
+  const char* gather_env = getenv("LIPZ_CONV_GATHER");
+  const bool gather_a = gather_env && gather_env[0] == '1';
+  auto act_map = [&](CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n) {
+    if (!ctc_make_act_map(m, q, descs, n, msg)) return false;
+    if (gather_a) q->a_tma = 0;
+    return true;
+  };
   p->tct = tct;
   // ---- buffers
   float *ec, *emean, *einv, *tc, *tmean, *tinv, *dh;
@@ -551,7 +561,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         }
       ok = ok && !upload(p, &p->tcd[l - 1], vt, msg);
       // one map serves every cell: the chunk buffers are shared
-      ok = ok && ctc_make_act_map(&p->aEd[l - 1], &p->cp[l - 1], vt.data(), 5, msg);
+      ok = ok && act_map(&p->aEd[l - 1], &p->cp[l - 1], vt.data(), 5);
       for (size_t k = 5; k < vt.size(); ++k)
         if (vt[k].in != vt[k % 5].in) p->cp[l - 1].a_tma = 0;
     }
@@ -636,7 +646,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
       ok = ok && !upload(p, &p->gtd[i], vt, msg);
-      ok = ok && ctc_make_act_map(&p->aEg[i], &p->gp[i], vt.data(), PE, msg);
+      ok = ok && act_map(&p->aEg[i], &p->gp[i], vt.data(), PE);
     }
   }
   // ---- tensor-core training forward (channel-last), and the output layer's descriptors in
@@ -658,7 +668,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->tgd[i], vt, msg);
-      ok = ok && ctc_make_act_map(&p->aTg[i], &p->tgp[i], vt.data(), C, msg);
+      ok = ok && act_map(&p->aTg[i], &p->tgp[i], vt.data(), C);
     }
     for (int l = 1; l <= 4 && ok; ++l) {
       CtcParams q = p->cp[l - 1];
@@ -676,7 +686,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->tdd[l - 1], vt, msg);
-      ok = ok && ctc_make_act_map(&p->aTd[l - 1], &p->tdp[l - 1], vt.data(), C, msg);
+      ok = ok && act_map(&p->aTd[l - 1], &p->tdp[l - 1], vt.data(), C);
     }
     std::vector<LogitDesc> vl, vd, vg;
     for (int c = 0; c < C; ++c) {
@@ -770,11 +780,11 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
         if (chain == 0) {
-          ok = ctc_make_act_map(&p->aDd[4 - l], &q, vt.data(), C, msg);
+          ok = act_map(&p->aDd[4 - l], &q, vt.data(), C);
           p->ddp[4 - l] = q;
           ok = !upload(p, &p->ddd[4 - l], vt, msg);
         } else {
-          ok = ctc_make_act_map(&p->aGd[4 - l], &q, vt.data(), C, msg);
+          ok = act_map(&p->aGd[4 - l], &q, vt.data(), C);
           p->gdp[4 - l] = q;
           ok = !upload(p, &p->gdd[4 - l], vt, msg);
         }
@@ -828,7 +838,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->gcd[i], vt, msg);
-      ok = ok && ctc_make_act_map(&p->aGc[i], &p->gcp[i], vt.data(), C, msg);
+      ok = ok && act_map(&p->aGc[i], &p->gcp[i], vt.data(), C);
     }
     // weight gradients: a = the output's delta (discriminator) or the layer's input
     // (generator), M = its channels; b = the other operand, gathered per tap

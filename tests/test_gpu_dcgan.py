@@ -166,3 +166,17 @@ def test_dcgan_full_width_3x3_b128_sampled(L):
     X = np.vstack([data[c][0], F])[rows]
     lg = O.d_forward(O.unflatten(s.Dw[c], dl), X, a)["logit"]
     assert max_rel(logits[c, 0, rows], lg) < 2e-2
+
+
+def test_dcgan_tma_and_gathered_activations_agree_bit_for_bit(L, monkeypatch):
+    """The tensor-core convolutions load their channel-last A tiles through activation maps by
+    TMA; with LIPZ_CONV_GATHER=1 the gather warps load them instead. Both hand the MMA the same
+    bytes, so one iteration (evaluation, selection, training) ends in the same state."""
+    pool = _field_pool(6, 40)
+    kw = dict(precision="bf16", ngf=64, ndf=64, batch=16, z_dim=100)
+    a = _grid(L, 2, 2, 7, pool, **kw)
+    a.iterate(1)
+    monkeypatch.setenv("LIPZ_CONV_GATHER", "1")
+    b = _grid(L, 2, 2, 7, pool, **kw)
+    b.iterate(1)
+    assert a.export_state() == b.export_state()
