@@ -517,7 +517,9 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_wait();
-  const int mt_n = p.M / 128, nt_n = p.N / 256;
+  // b_chw: b is a 3-channel channel-major image stack, N = 48 (tap, channel) columns in one
+  // 64-wide tile; M (a multiple of 64) may leave the upper half of a 128-row tile empty
+  const int mt_n = (p.M + 127) / 128, nt_n = p.b_chw ? 1 : p.N / 256;
   const int per_split = mt_n * nt_n;
   const int la = p.la, lb = p.lb;
   const int64_t Kp = (int64_t)p.rows << (2 * la);  // pixels of A per problem
@@ -530,7 +532,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
       int stage = 0, uses[2] = {0, 0}, jobs = 0;
       uint32_t phase = 0;
       bool ok = true;
-      const uint32_t idesc = idesc_bf16_major(128, 256, 1, 1);
+      const uint32_t idesc = idesc_bf16_major(128, p.b_chw ? 64 : 256, 1, 1);
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++jobs) {
         const int split = (tile / per_split) % p.splits;
         int64_t k0, k1;
@@ -599,12 +601,43 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
         const int nb = (int)(q >> (2 * la));
         const int ay = (int)((q >> la) & ((1 << la) - 1)), ax = (int)(q & ((1 << la) - 1));
         {
-          const bf16* src = qv ? d.a + q * p.M + mt * 128 + half * 64 : d.a;
+          const bool av = qv && mt * 128 + half * 64 < p.M;
+          const bf16* src = av ? d.a + q * p.M + mt * 128 + half * 64 : d.a;
           const uint32_t dst = sA + (uint32_t)half * 8192u + (uint32_t)row * 128u;
 #pragma unroll
           for (int u = 0; u < 8; ++u)
-            cp_async16(dst + (((uint32_t)u ^ sw) << 4), src + (qv ? 8 * u : 0), qv ? 16 : 0);
+            cp_async16(dst + (((uint32_t)u ^ sw) << 4), src + (av ? 8 * u : 0), av ? 16 : 0);
         }
+        if (p.b_chw) {
+          // row `row` of the single B atom, columns k = tap * 3 + c (k < 48, zero above);
+          // thread half h writes the 16-byte units 4h .. 4h + 3 (k = 32h .. 32h + 31)
+#pragma unroll
+          for (int uu = 0; uu < 4; ++uu) {
+            const int u = half * 4 + uu;
+            uint32_t w[4];
+#pragma unroll
+            for (int e2 = 0; e2 < 4; ++e2) {
+              uint32_t hv[2];
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const int k = u * 8 + e2 * 2 + h;
+                hv[h] = 0u;
+                if (k < 48 && qv) {
+                  const int tap = k / 3, c = k - 3 * tap;
+                  const int by = ay * p.s - p.p + (tap >> 2), bx = ax * p.s - p.p + (tap & 3);
+                  if (by >= 0 && by < (1 << lb) && bx >= 0 && bx < (1 << lb))
+                    hv[h] = (uint32_t)__bfloat16_as_ushort(
+                        d.b[((int64_t)(nb * 3 + c) << (2 * lb)) + (by << lb) + bx]);
+                }
+              }
+              w[e2] = hv[0] | (hv[1] << 16);
+            }
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                             sB + (uint32_t)row * 128u + (((uint32_t)u ^ sw) << 4)),
+                         "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                         : "memory");
+          }
+        } else
 #pragma unroll
         for (int aa = 0; aa < 2; ++aa) {
           const int atom = 2 * half + aa;
@@ -657,12 +690,15 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
         break;
       }
       tc_fence_after();
+      const bool rv = mt * 128 + r < p.M;
       float* o = p.part + (((int64_t)prob * p.splits + split) * p.M + mt * 128 + r) * p.N +
                  nt * 256;
-      for (int g = 0; g < 8; ++g) {
+      const int groups = p.b_chw ? 2 : 8;
+      for (int g = 0; g < groups; ++g) {
         uint32_t v[32];
         LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
         tmem_wait_ld();
+        if (!rv) continue;
         float4* o4 = reinterpret_cast<float4*>(o + g * 32);
 #pragma unroll
         for (int u = 0; u < 8; ++u)
@@ -680,6 +716,23 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
   tc_fence_after();
   if (warp == 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+}
+
+// b_chw: part[problem][split][m][tap * 3 + c] (64 columns) -> dW[m][c][tap], summed over the
+// splits in order.
+__global__ void __launch_bounds__(256) k_wgrad_tc_reduce_chw(const __grid_constant__ WgtcParams p) {
+  pdl_wait();
+  const int prob = blockIdx.y;
+  const int64_t MN = (int64_t)p.M * p.N;
+  const float* part = p.part + (int64_t)prob * p.splits * MN;
+  float* out = p.descs[prob].dw;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < p.M * 48; e += gridDim.x * blockDim.x) {
+    const int m = e / 48, j = e - m * 48;  // j = c * 16 + tap
+    const int64_t src = (int64_t)m * p.N + (j & 15) * 3 + (j >> 4);
+    float acc = 0.f;
+    for (int sp = 0; sp < p.splits; ++sp) acc += part[sp * MN + src];
+    out[e] = acc;
+  }
 }
 
 // part[problem][split][m][(tap, c)] -> dW[m][c][tap], summed over the splits in order; a
@@ -998,7 +1051,11 @@ bool wgtc_prepare(std::string* msg) {
 void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st) {
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
   launch_pdl(ctc::k_wgrad_tc, dim3(grid), dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, p);
-  launch_pdl(ctc::k_wgrad_tc_reduce, dim3(p.M * (p.Cb / 64), p.n_probs), dim3(256), 0, st, p);
+  if (p.b_chw)
+    launch_pdl(ctc::k_wgrad_tc_reduce_chw, dim3((p.M * 48 + 255) / 256, p.n_probs), dim3(256), 0,
+               st, p);
+  else
+    launch_pdl(ctc::k_wgrad_tc_reduce, dim3(p.M * (p.Cb / 64), p.n_probs), dim3(256), 0, st, p);
 }
 
 void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,

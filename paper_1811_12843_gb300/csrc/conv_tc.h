@@ -66,7 +66,8 @@ struct RelayoutD {
 
 // Weight gradients on tcgen05: per problem a = [rows][2^la][2^la][M] and b = the gathered
 // operand [rows][2^lb][2^lb][Cb] (both channel-last, M a multiple of 128, Cb of 64, N = 16 Cb
-// a multiple of 256); dw = the problem's [M][Cb][4][4] fp32 gradient. b's pixel for tap
+// a multiple of 256; or, with b_chw, b = [rows][3][2^lb][2^lb] channel-major, Cb 3, N 64, M a
+// multiple of 64); dw = the problem's [M][Cb][4][4] fp32 gradient. b's pixel for tap
 // (ky, kx) of a's pixel (y, x) is (s y - p + ky, s x - p + kx). part holds
 // n_probs x splits x M x N floats; split s covers a's pixels [s kc, (s + 1) kc) of each problem
 // (kc a multiple of 64, every split non-empty).
@@ -79,6 +80,7 @@ struct WgtcParams {
   const WgtcDesc* descs;
   int n_probs, rows, M, N, Cb, la, lb, s, p, splits, n_tiles;
   int64_t kc;
+  int b_chw;  // b is 3 channel-major channels (Cb 3, N 64 with 48 used, M a multiple of 64)
   float* part;
   int* err;
 };

@@ -847,7 +847,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     auto wplan = [&](WgtcParams& q) {
       const int64_t Kp = (int64_t)q.rows << (2 * q.la);
       const int64_t chunks = (Kp + 63) / 64;
-      const int64_t per = (int64_t)C * (q.M / 128) * (q.N / 256);
+      const int64_t per = (int64_t)C * ((q.M + 127) / 128) * (q.b_chw ? 1 : q.N / 256);
       int best = 1;
       double be = 0;
       for (int sp = 1; sp <= 64 && sp <= std::max<int64_t>(1, chunks / 8); ++sp) {
@@ -865,15 +865,17 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       q.err = p->err;
       wneed = std::max<int64_t>(wneed, (int64_t)C * q.splits * q.M * q.N);
     };
-    for (int l = 4; l >= 2 && ok; --l) {
+    for (int l = 4; l >= 1 && ok; --l) {
       const int k = 4 - l;
-      if (dc[l] % 128 != 0 || dc[l - 1] % 64 != 0) continue;
+      // layer 1 reads the 3-channel channel-major images (b_chw)
+      if (l == 1 ? dc[1] % 64 != 0 : (dc[l] % 128 != 0 || dc[l - 1] % 64 != 0)) continue;
       WgtcParams q;
       memset(&q, 0, sizeof q);
       q.rows = 2 * B;
       q.M = dc[l];
       q.Cb = dc[l - 1];
-      q.N = 16 * q.Cb;
+      q.b_chw = l == 1;
+      q.N = l == 1 ? 64 : 16 * q.Cb;
       q.la = ilog2(ds[l]);
       q.lb = ilog2(ds[l - 1]);
       q.s = 2;
@@ -883,7 +885,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       for (int c = 0; c < C; ++c) {
         WgtcDesc w;
         w.a = (const bf16*)elw((l % 2 == 0) ? P : Q, (int64_t)c * 2 * B * dmax);
-        w.b = (const bf16*)tda(c, l - 1);
+        w.b = (const bf16*)(l == 1 ? (const void*)tx(c) : (const void*)tda(c, l - 1));
         w.dw = b.gD + (int64_t)c * b.PDs + dof[l - 1];
         vw.push_back(w);
       }
@@ -891,15 +893,17 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       p->wtc_d[k] = true;
       ok = !upload(p, &p->wdd[k], vw, msg);
     }
-    for (int l = 4; l >= 2 && ok; --l) {
+    for (int l = 5; l >= 2 && ok; --l) {
       const int k = 5 - l;
-      if (gc[l - 1] % 128 != 0 || gc[l] % 64 != 0) continue;
+      // layer 5 gathers the 3-channel channel-major delta of the fakes (b_chw)
+      if (l == 5 ? gc[4] % 64 != 0 : (gc[l - 1] % 128 != 0 || gc[l] % 64 != 0)) continue;
       WgtcParams q;
       memset(&q, 0, sizeof q);
       q.rows = B;
       q.M = gc[l - 1];
       q.Cb = gc[l];
-      q.N = 16 * q.Cb;
+      q.b_chw = l == 5;
+      q.N = l == 5 ? 64 : 16 * q.Cb;
       q.la = ilog2(gs[l - 1]);
       q.lb = ilog2(gs[l]);
       q.s = 2;
@@ -909,7 +913,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       for (int c = 0; c < C; ++c) {
         WgtcDesc w;
         w.a = (const bf16*)tgh(c, l - 1);
-        w.b = (const bf16*)elw(dcb, (int64_t)c * B * gmax);
+        w.b = (const bf16*)(l == 5 ? elw(d5, (int64_t)c * B * X) : elw(dcb, (int64_t)c * B * gmax));
         w.dw = b.gG + (int64_t)c * b.PGs + go[3 * (l - 1)];
         vw.push_back(w);
       }
