@@ -36,7 +36,9 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 320;  // warp 0 TMA, 1 MMA, 2-5 gather, 6-9 epilogue
 // first-layer input patches: 3 channels x 10 rows x 72 columns (64 interior at column 4)
 constexpr int PATCH_BYTES = 4352;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256 + 3 * PATCH_BYTES;
+// epilogue staging for coalesced row stores: 32 rows x 36 words per epilogue warp
+constexpr int STG_WORDS = 32 * 36;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256 + 3 * PATCH_BYTES + 4 * STG_WORDS * 4;
 constexpr int LAG = 2;  // copy groups a gather thread keeps in flight (< STAGES)
 
 // 16-byte global -> shared copy; bytes = 0 writes zeros (src must still be a valid address)
@@ -362,6 +364,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    uint32_t* stg = reinterpret_cast<uint32_t*>(misc + 256 + 3 * PATCH_BYTES) + (warp - 6) * STG_WORDS;
     int uses[2] = {0, 0}, jobs = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
@@ -409,17 +412,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t v[32];
             LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
             tmem_wait_ld();
-            if (p.out_mode == CTC_F32_HWC) {
-              if (valid) {
-                float4* o = reinterpret_cast<float4*>(reinterpret_cast<float*>(d.out) +
-                                                      pix * p.co + j * 256 + g * 32);
+            // the row's 32 columns go to the warp's staging rows (fp32 words, or bf16 pairs),
+            // then out in 16-byte pieces, lpr lanes per row, so that each store instruction
+            // writes whole rows' contiguous bytes
+            const bool f32 = p.out_mode == CTC_F32_HWC;
+            if (f32) {
 #pragma unroll
-                for (int u = 0; u < 8; ++u)
-                  o[u] = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
-                                     __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
-              }
-              continue;
-            }
+              for (int u = 0; u < 8; ++u)
+                *reinterpret_cast<uint4*>(stg + lane * 36 + 4 * u) =
+                    make_uint4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+            } else {
             uint32_t pk[16];
             if (p.out_mode == CTC_DLRELU_HWC) {
               // the LeakyReLU derivative at the stored activation (same sign as its input)
@@ -448,12 +450,28 @@ __global__ void __launch_bounds__(THREADS, 1)
                 pk[e >> 1] = pack_bf16(a, b);
               }
             }
-            if (valid) {
-              uint4* o = reinterpret_cast<uint4*>(d.out + pix * p.co + j * 256 + g * 32);
 #pragma unroll
-              for (int u = 0; u < 4; ++u)
-                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+            for (int u = 0; u < 4; ++u)
+              *reinterpret_cast<uint4*>(stg + lane * 36 + 4 * u) =
+                  make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
             }
+            __syncwarp();
+            const int lpr = f32 ? 8 : 4, rpi = 32 / lpr;
+            const int part = lane % lpr;
+            for (int it = 0; it < lpr; ++it) {
+              const int rr = it * rpi + lane / lpr;
+              const int64_t pr = __shfl_sync(0xffffffffu, pix, rr);
+              const int vr = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr);
+              const uint4 w = *reinterpret_cast<const uint4*>(stg + rr * 36 + 4 * part);
+              if (vr) {
+                const int64_t e = pr * p.co + j * 256 + g * 32;
+                if (f32)
+                  *reinterpret_cast<uint4*>(reinterpret_cast<float*>(d.out) + e + 4 * part) = w;
+                else
+                  *reinterpret_cast<uint4*>(d.out + e + 8 * part) = w;
+              }
+            }
+            __syncwarp();
           }
         }
         tc_fence_before();
