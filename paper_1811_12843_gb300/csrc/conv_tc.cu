@@ -497,7 +497,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // 256); fp32 partial sums per split go to part[problem][split][M][N] in (tap, c) order.
 constexpr int WG_THREADS = 320;  // warp 1 MMA, warps 2-5 gather, warps 6-9 epilogue
 constexpr int WG_STAGES = 4;
-constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256;
+constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256 + 4 * STG_WORDS * 4;
 constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_STAGES)
 
 __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constant__ WgtcParams p) {
@@ -692,10 +692,12 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
       arr_stage = arr_stage + 1 == WG_STAGES ? 0 : arr_stage + 1;
     }
   } else if (warp >= 6) {
-    // epilogue: row m of the tile, 256 columns in groups of 32, fp32 partial sums
+    // epilogue: row m of the tile, 256 columns in groups of 32, fp32 partial sums, staged in
+    // shared memory and stored as whole rows (eight lanes per 128-byte row piece)
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
+    uint32_t* stg = reinterpret_cast<uint32_t*>(misc + 256) + (warp - 6) * STG_WORDS;
     int uses[2] = {0, 0}, jobs = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++jobs) {
@@ -708,7 +710,6 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
         break;
       }
       tc_fence_after();
-      const bool rv = mt * 128 + r < p.M;
       float* o = p.part + (((int64_t)prob * p.splits + split) * p.M + mt * 128 + r) * p.N +
                  nt * 256;
       const int groups = p.b_chw ? 2 : 8;
@@ -716,12 +717,18 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
         uint32_t v[32];
         LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
         tmem_wait_ld();
-        if (!rv) continue;
-        float4* o4 = reinterpret_cast<float4*>(o + g * 32);
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-          o4[u] = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
-                              __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
+          *reinterpret_cast<uint4*>(stg + lane * 36 + 4 * u) =
+              make_uint4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+        __syncwarp();
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + (lane >> 3), part = lane & 7;
+          const uint4 w = *reinterpret_cast<const uint4*>(stg + rr * 36 + 4 * part);
+          if (mt * 128 + q4 * 32 + rr < p.M)
+            *reinterpret_cast<uint4*>(o + (int64_t)(rr - lane) * p.N + g * 32 + 4 * part) = w;
+        }
+        __syncwarp();
       }
       tc_fence_before();
       mbar_arrive(bAccE + 8 * R);
