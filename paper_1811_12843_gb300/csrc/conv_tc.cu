@@ -51,6 +51,19 @@ __device__ __forceinline__ void cp_async8(uint32_t dst, const void* src, int byt
                : "memory");
 }
 
+// Barrier of the four epilogue warps (named barrier 2), plain and with an OR vote.
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 2, 128;" ::: "memory"); }
+__device__ __forceinline__ bool epi_bar_or(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 2, 128, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)pred)
+      : "memory");
+  return r != 0;
+}
+
 // Barrier of the four gather warps (named barrier 1) that returns whether any thread passed
 // true.
 __device__ __forceinline__ bool gather_bar_or(bool pred) {
@@ -104,7 +117,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = *tmem_slot;
   pdl_wait();
   // output pixels per problem (per parity class when transposed)
-  const int lq = p.lho - p.transposed;
+  // rows of a problem: output pixels (class pixels when transposed; input pixels in scatter)
+  const int lq = p.scatter ? p.lhi : p.lho - p.transposed;
   const int M = p.rows << (2 * lq);
   const int nbox = p.nbox;
 
@@ -138,7 +152,10 @@ __global__ void __launch_bounds__(THREADS, 1)
               const int k0 = kc * BK;
               const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
               int x, y;
-              if (p.transposed) {
+              if (p.scatter) {
+                y = y0;
+                x = 0;
+              } else if (p.transposed) {
                 const int a = cls >> 1, b = cls & 1;
                 const int ky = ((a + 1) & 1) + 2 * (tap >> 1), kx = ((b + 1) & 1) + 2 * (tap & 1);
                 y = y0 + ((a + 1 - ky) >> 1);
@@ -383,11 +400,67 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int64_t pix = ((int64_t)nb << (2 * p.lho)) + (oy << p.lho) + ox;
       for (int j = 0; j < p.nj && ok; ++j, ++jobs) {
         const int R = jobs & 1;
-        if (!mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 28)) {
+        // the scatter epilogue synchronises the four warps: they leave together
+        const bool okw =
+            mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 28);
+        if (p.scatter ? epi_bar_or(!okw) : !okw) {
           ok = false;
           break;
         }
         tc_fence_after();
+        if (p.scatter) {
+          // input pixel (y0 + q, lane) holds Y[tap * 4 + o] (16 taps, 3 channels); the taps are
+          // added one after the other into the tile's 10 x 66 output window in shared memory
+          // (output row 2 y - 1 + ky, column 2 x - 1 + kx; window origin (2 y0 - 1, -1))
+          float* acc = reinterpret_cast<float*>(stg - (warp - 6) * STG_WORDS);
+          const int et = threadIdx.x - 192;
+          const int m0t = m - row;  // the tile's first input pixel: image img, rows 4 blk ..
+          const int img = m0t >> 10, blk = (m0t >> 7) & 7;
+          for (int i = et; i < 1980; i += 128) acc[i] = 0.f;
+          uint32_t v[32], w[32];  // columns 0..31 (taps 0..7) and 32..63 (taps 8..15)
+          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256), v);
+          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + 32), w);
+          tmem_wait_ld();
+          tc_fence_before();
+          mbar_arrive(bAccE + 8 * R);
+          uses[R]++;
+          epi_bar();
+#pragma unroll
+          for (int tap = 0; tap < 16; ++tap) {
+            float* a = acc + ((2 * q + (tap >> 2)) * 66 + 2 * lane + (tap & 3)) * 3;
+            const uint32_t* y = tap < 8 ? v + tap * 4 : w + (tap - 8) * 4;
+            if (valid) {
+              a[0] += __uint_as_float(y[0]);
+              a[1] += __uint_as_float(y[1]);
+              a[2] += __uint_as_float(y[2]);
+            }
+            epi_bar();
+          }
+          // window rows 2..7 (output rows 8 blk + 1 .. 8 blk + 6) are complete; rows 0, 1, 8, 9
+          // are shared with the blocks above and below and go to the halo buffer
+          const bool tv = m0t < M;
+          if (tv) {
+            for (int i = et; i < 6 * 64 * 3; i += 128) {
+              const int o = i / 384, rem = i - o * 384, lr = 2 + (rem >> 6), gx = rem & 63;
+              const int64_t oi = (((int64_t)img * 3 + o) << 12) + ((8 * blk - 1 + lr) << 6) + gx;
+              float x = acc[(lr * 66 + gx + 1) * 3 + o];
+              if (p.out_mode == CTC_TANH_CHW) {
+                x = tanhf(x);
+              } else {
+                const float f = __bfloat162float(d.aux[oi]);
+                x = x * (1.f - f * f);
+              }
+              d.out[oi] = __float2bfloat16_rn(x);
+            }
+            float* h = p.halo + (((int64_t)pc * p.rows + img) * 8 + blk) * 768;
+            for (int i = et; i < 768; i += 128) {
+              const int pr = i / 192, rem = i - pr * 192, gx = rem / 3, o = rem - gx * 3;
+              h[i] = acc[((pr < 2 ? pr : pr + 6) * 66 + gx + 1) * 3 + o];
+            }
+          }
+          epi_bar();
+          continue;
+        }
         if (p.out_mode == CTC_TANH_CHW || p.out_mode == CTC_DTANH_CHW) {
           // a few output channels (the image's colours), channel-major images: tanh, or the
           // delta times tanh' = 1 - f^2 with f the stored tanh output
@@ -741,6 +814,50 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
   tc_fence_after();
   if (warp == 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+}
+
+// Scatter mode: the output rows 8k - 1 and 8k of every image are shared by row blocks k - 1
+// and k (their halo rows 2, 3 and 0, 1); add them in that order and apply the epilogue (tanh,
+// or the delta times 1 - f^2). Grid: (problem x image); 64 x 64 x 3 outputs per image.
+__global__ void __launch_bounds__(256) k_scatter_fix(const ConvTcDesc* __restrict__ descs,
+                                                     const float* __restrict__ halo, int rows,
+                                                     int out_mode) {
+  pdl_wait();
+  const int pi = blockIdx.x;  // problem * rows + image
+  const ConvTcDesc d = descs[pi / rows];
+  const int img = pi % rows;
+  const float* h = halo + (int64_t)pi * 8 * 768;
+  for (int i = threadIdx.x; i < 9 * 2 * 64 * 3; i += 256) {
+    const int k = i / 384, rem = i - k * 384, t = rem / 192, rem2 = rem - t * 192;
+    const int gx = rem2 / 3, o = rem2 - gx * 3;
+    const int gy = 8 * k - 1 + t;
+    if (gy < 0 || gy > 63) continue;
+    float x = 0.f;
+    if (k > 0) x += h[(k - 1) * 768 + (2 + t) * 192 + gx * 3 + o];
+    if (k < 8) x += h[k * 768 + t * 192 + gx * 3 + o];
+    const int64_t oi = (((int64_t)img * 3 + o) << 12) + (gy << 6) + gx;
+    if (out_mode == CTC_TANH_CHW) {
+      x = tanhf(x);
+    } else {
+      const float f = __bfloat162float(d.aux[oi]);
+      x = x * (1.f - f * f);
+    }
+    d.out[oi] = __float2bfloat16_rn(x);
+  }
+}
+
+// Scatter-mode weights of a 4x4 transposed convolution to 3 channels: src [k][3][16] (64
+// input channels k, 3 outputs j, 16 taps) of every individual -> dst [tap * 4 + j][k] (64 x 64,
+// row j = 3 zero).
+__global__ void k_relayout_s(const bf16* __restrict__ src, int64_t src_ps, int64_t src_off,
+                             bf16* __restrict__ dst) {
+  pdl_wait();
+  const int64_t ind = blockIdx.y;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < 4096; e += gridDim.x * blockDim.x) {
+    const int n = e >> 6, k = e & 63, tap = n >> 2, j = n & 3;
+    dst[ind * 4096 + e] =
+        j < 3 ? src[ind * src_ps + src_off + (k * 3 + j) * 16 + tap] : __float2bfloat16_rn(0.f);
+  }
 }
 
 // b_chw: part[problem][split][m][tap * 3 + c] (64 columns) -> dW[m][c][tap], summed over the
@@ -1172,7 +1289,7 @@ bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int
                       std::string* msg) {
   q->a_tma = 0;
   if (q->nchw_in || q->ci % 64 != 0 || n_probs < 1) return true;
-  const int lq = q->lho - q->transposed;
+  const int lq = q->scatter ? q->lhi : q->lho - q->transposed;
   if (lq > 7) return true;
   const int64_t Wi = (int64_t)1 << q->lhi;
   const int64_t per = (int64_t)q->rows * Wi * Wi * q->ci;  // elements of one problem's input
@@ -1182,7 +1299,7 @@ bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int
   for (int k = 1; k < n_probs; ++k)
     if (descs[k].in != descs[0].in + (int64_t)k * pstride) return true;
   if (!ensure_encode(msg)) return false;
-  const int stride = q->transposed ? 1 : 2;
+  const int stride = q->transposed || q->scatter ? 1 : 2;
   const int tw = 1 << lq, th = std::min(1 << lq, 128 / tw), tn = std::max(1, 128 / (tw * th));
   cuuint64_t dims[5] = {(cuuint64_t)q->ci, (cuuint64_t)Wi, (cuuint64_t)Wi, (cuuint64_t)q->rows,
                         (cuuint64_t)n_probs};
@@ -1216,6 +1333,17 @@ void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParam
                     cudaStream_t st) {
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
   launch_pdl(ctc::k_conv_tc, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, mA, p);
+}
+
+void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_problems, int rows,
+                        int out_mode, cudaStream_t st) {
+  launch_pdl(ctc::k_scatter_fix, dim3(n_problems * rows), dim3(256), 0, st, descs, halo, rows,
+             out_mode);
+}
+
+void launch_relayout_s(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst, int n_indiv,
+                       cudaStream_t st) {
+  launch_pdl(ctc::k_relayout_s, dim3(4, n_indiv), dim3(256), 0, st, src, src_ps, src_off, dst);
 }
 
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,

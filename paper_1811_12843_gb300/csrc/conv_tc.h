@@ -42,6 +42,13 @@ struct CtcParams {
   int rows, ci, lhi, co, lho, nchw_in, kchunks, nj, nbox, mtiles, n_tiles;
   int transposed, out_mode, cls_rows;
   int a_tma;  // A rows by TMA through the activation map (set by ctc_make_act_map)
+  // scatter: a stride-2 transposed convolution to 3 channels (CTC_TANH_CHW / CTC_DTANH_CHW,
+  // ci 64, 32 x 32 -> 64 x 64) as one GEMM over input pixels (N = 16 taps x 4, weights from
+  // launch_relayout_s), each tile of 4 input rows adding its taps into an output window in
+  // shared memory in a fixed order; the rows it shares with the next tile go to halo
+  // (problems x rows x 8 x 768 floats) and launch_scatter_fix completes them
+  int scatter;
+  float* halo;
   const int* wsel;
   float slope;
   int* err;
@@ -97,6 +104,12 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
 bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
                       std::string* msg);
 bool ctc_prepare(std::string* msg);
+void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_problems, int rows,
+                        int out_mode, cudaStream_t st);
+// [individual][64 input channels][3][4][4] at src_off (stride src_ps) -> dst [individual][64
+// rows tap * 4 + output][64], the scatter mode's weights.
+void launch_relayout_s(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst, int n_indiv,
+                       cudaStream_t st);
 void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
                     cudaStream_t st);
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,

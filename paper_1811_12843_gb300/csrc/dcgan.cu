@@ -129,6 +129,15 @@ struct DcPlan {
   // activation maps of the channel-last tensor-core launches (A rows by TMA): evaluation D
   // and G, training forwards, D-loss and G-loss input gradients, generator input gradients
   CUtensorMap aEd[4], aEg[4], aTg[4], aTd[4], aDd[3], aGd[4], aGc[4];
+  // scatter mode (one GEMM over input pixels, see conv_tc.h) for the 64 -> 3 transposed
+  // convolutions: the generator's output layer (evaluation egs, training tgs) and the
+  // G-loss input gradient of discriminator layer 1 (gds)
+  bool scg = false, scd = false;
+  bf16 *Gs = nullptr, *Ds = nullptr;
+  CUtensorMap mGs, mDs, aEgs, aTgs, aGds;
+  CtcParams egs, tgs, gds;
+  float* halo = nullptr;
+  std::vector<ConvTcDesc> h_gtd5, h_tgd5, h_gdd1;
   // tensor-core weight gradients of the layers whose channel counts fill the tiles
   bool wtc_d[4] = {}, wtc_g[5] = {};
   WgtcParams wdp[4], wgp[5];
@@ -646,6 +655,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           vt.push_back(t);
         }
       ok = ok && !upload(p, &p->gtd[i], vt, msg);
+      if (l == 5) p->h_gtd5 = vt;
       ok = ok && act_map(&p->aEg[i], &p->gp[i], vt.data(), PE);
     }
   }
@@ -668,6 +678,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         vt.push_back(t);
       }
       ok = ok && !upload(p, &p->tgd[i], vt, msg);
+      if (l == 5) p->h_tgd5 = vt;
       ok = ok && act_map(&p->aTg[i], &p->tgp[i], vt.data(), C);
     }
     for (int l = 1; l <= 4 && ok; ++l) {
@@ -786,6 +797,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         } else {
           ok = act_map(&p->aGd[4 - l], &q, vt.data(), C);
           p->gdp[4 - l] = q;
+          if (l == 1) p->h_gdd1 = vt;
           ok = !upload(p, &p->gdd[4 - l], vt, msg);
         }
       }
@@ -923,12 +935,59 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     }
     ok = ok && !dev_alloc(p, &p->wpart, (size_t)wneed * 4, msg);
   }
+  // ---- scatter mode for the 64 -> 3 transposed convolutions (its A tiles always come by TMA:
+  // it has no gathered form)
+  p->scg = ok && p->tcg && g == 64;
+  p->scd = ok && tct && d == 64;
+  if (p->scg || p->scd) {
+    auto scatter_params = [&](int rows, int n_probs, int out_mode) {
+      CtcParams q;
+      memset(&q, 0, sizeof q);
+      q.rows = rows;
+      q.ci = 64;
+      q.lhi = 5;
+      q.co = 3;
+      q.lho = 6;
+      q.kchunks = 1;
+      q.nj = 1;
+      q.nbox = 64;
+      q.out_mode = out_mode;
+      q.scatter = 1;
+      q.mtiles = (rows << 10) / 128;
+      q.n_tiles = n_probs * q.mtiles;
+      q.slope = s.slope;
+      q.err = p->err;
+      return q;
+    };
+    ok = !dev_alloc(p, &p->halo, (size_t)std::max(PE, C) * B * 8 * 768 * 4, msg);
+    if (ok && p->scg) {
+      ok = !dev_alloc(p, &p->Gs, (size_t)s.n_indiv * 4096 * 2, msg) &&
+           ctc_make_map(&p->mGs, p->Gs, 64, 64, s.n_indiv, 4096, 64, msg);
+      p->egs = scatter_params(B, PE, CTC_TANH_CHW);
+      p->egs.halo = p->halo;
+      ok = ok && ctc_make_act_map(&p->aEgs, &p->egs, p->h_gtd5.data(), PE, msg);
+      if (ok && tct) {
+        p->tgs = scatter_params(B, C, CTC_TANH_CHW);
+        p->tgs.halo = p->halo;
+        ok = ctc_make_act_map(&p->aTgs, &p->tgs, p->h_tgd5.data(), C, msg);
+      }
+      if (ok && !(p->egs.a_tma && (!tct || p->tgs.a_tma))) p->scg = false;
+    }
+    if (ok && p->scd) {
+      ok = !dev_alloc(p, &p->Ds, (size_t)s.n_indiv * 4096 * 2, msg) &&
+           ctc_make_map(&p->mDs, p->Ds, 64, 64, s.n_indiv, 4096, 64, msg);
+      p->gds = scatter_params(B, C, CTC_DTANH_CHW);
+      p->gds.halo = p->halo;
+      ok = ok && ctc_make_act_map(&p->aGds, &p->gds, p->h_gdd1.data(), C, msg);
+      if (ok && !p->gds.a_tma) p->scd = false;
+    }
+  }
   if (!ok) {
     dc_plan_destroy(p);
     return nullptr;
   }
   p->eval_launches = 9 + 5 * C;
-  p->train_launches = tct ? 60 : 50;
+  p->train_launches = tct ? 60 + (p->scg ? 1 : 0) + (p->scd ? 2 : 0) : 50;
   return p;
 }
 
@@ -958,10 +1017,20 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
                 nullptr, 0, s.slope, st);
     launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, st);
+    if (p->scg)
+      launch_relayout_s((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[12], p->Gs, s.n_indiv, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->gp[i];
       q.descs = p->gtd[i];
       q.wsel = nbr;
+      if (i == 3 && p->scg) {
+        q = p->egs;
+        q.descs = p->gtd[i];
+        q.wsel = nbr;
+        launch_conv_tc(p->mGs, p->aEgs, q, p->sms, st);
+        launch_scatter_fix(p->gtd[i], p->halo, PE, B, CTC_TANH_CHW, st);
+        continue;
+      }
       launch_conv_tc(p->mG[i], p->aEg[i], q, p->sms, st);
       if (i < 3)
         launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, p->bncnt, st);
@@ -1027,6 +1096,14 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->tgp[i];
       q.descs = p->tgd[i];
       q.wsel = p->b.src_g;
+      if (i == 3 && p->scg) {
+        q = p->tgs;
+        q.descs = p->tgd[i];
+        q.wsel = p->b.src_g;
+        launch_conv_tc(p->mGs, p->aTgs, q, p->sms, st);
+        launch_scatter_fix(p->tgd[i], p->halo, C, B, CTC_TANH_CHW, st);
+        continue;
+      }
       launch_conv_tc(p->mG[i], p->aTg[i], q, p->sms, st);
       if (i < 3)
         launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, p->bncnt, st);
@@ -1069,6 +1146,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
                       st);
     launch_relayout_c((const bf16*)p->b.Gop, p->b.PGs, p->Gct, p->gct_ps, s.n_indiv, p->relc,
                       st);
+    if (p->scd)
+      launch_relayout_s((const bf16*)p->b.Dop, p->b.PDs, p->b.doff[0], p->Ds, s.n_indiv, st);
   }
   // discriminator backward (D loss)
   launch_logit_back(s.bf, p->tct ? p->tdl_back_d_tc : p->tdl_back_d, C, (int)(8 * d * 16), true,
@@ -1099,7 +1178,13 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   launch_logit_back(s.bf, p->tct ? p->tdl_back_g_tc : p->tdl_back_g, C, (int)(8 * d * 16),
                     false, s.slope, st);
   for (int l = 4; l >= 1; --l) {
-    if (p->tct) {
+    if (p->tct && l == 1 && p->scd) {
+      CtcParams q = p->gds;
+      q.descs = p->gdd[3];
+      q.wsel = p->b.src_d;
+      launch_conv_tc(p->mDs, p->aGds, q, p->sms, st);
+      launch_scatter_fix(p->gdd[3], p->halo, C, B, CTC_DTANH_CHW, st);
+    } else if (p->tct) {
       CtcParams q = p->gdp[4 - l];
       q.descs = p->gdd[4 - l];
       q.wsel = p->b.src_d;
@@ -1142,7 +1227,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int dc_eval_launches(const DcPlan* p, int part) {
-  if (part == 0) return p->tcg ? 14 : 9;
+  if (part == 0) return p->tcg ? 14 + (p->scg ? 2 : 0) : 9;
   return p->eval_launches - 9 + (p->tc ? 1 : 0);
 }
 
