@@ -425,6 +425,8 @@ __global__ void __launch_bounds__(THREADS, 1)
           mbar_arrive(bAccE + 8 * R);
           uses[R]++;
           epi_bar();
+          // taps with ky < 2 first (warp q writes window rows 2q, 2q + 1: no two warps share a
+          // row), then ky >= 2 (rows 2q + 2, 2q + 3); inside a warp the taps go in order
 #pragma unroll
           for (int tap = 0; tap < 16; ++tap) {
             float* a = acc + ((2 * q + (tap >> 2)) * 66 + 2 * lane + (tap & 3)) * 3;
@@ -434,7 +436,10 @@ __global__ void __launch_bounds__(THREADS, 1)
               a[1] += __uint_as_float(y[1]);
               a[2] += __uint_as_float(y[2]);
             }
-            epi_bar();
+            if (tap == 7 || tap == 15)
+              epi_bar();
+            else
+              __syncwarp();
           }
           // window rows 2..7 (output rows 8 blk + 1 .. 8 blk + 6) are complete; rows 0, 1, 8, 9
           // are shared with the blocks above and below and go to the halo buffer
