@@ -135,8 +135,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int indiv = __ldg(&p.wsel[d.wsel_idx]);
         // channel-last A rows by TMA (a_tma): the tile is 128 consecutive output pixels (class
         // pixels when transposed) of whole rows; its origin is image n0, row y0
-        const int m0 = (tile % p.mtiles) * BM;
+        const int m0 = (tile % p.mtiles) * (p.m2 ? 2 * BM : BM);
         const int n0 = m0 >> (2 * lq), y0 = (m0 >> lq) & ((1 << lq) - 1);
+        // m2: the second 128 rows of a 256-row tile
+        const int n1 = (m0 + BM) >> (2 * lq), y1 = ((m0 + BM) >> lq) & ((1 << lq) - 1);
         for (int j = 0; j < p.nj && ok; ++j)
           for (int kc = 0; kc < p.kchunks; ++kc) {
             if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 21)) {
@@ -144,31 +146,39 @@ __global__ void __launch_bounds__(THREADS, 1)
               break;
             }
             mbar_expect_tx(bFullB + 8 * stage,
-                           (uint32_t)(nbox * BK * 2 + (p.a_tma ? A_BYTES : 0)));
+                           (uint32_t)(nbox * BK * 2 + (p.a_tma ? (p.m2 ? 2 : 1) * A_BYTES : 0)));
             if (p.a_tma) {
               // Convolution: tap (ky, kx), input rows 2 y - 1 + ky, columns 2 x - 1 + kx (the
               // map's traversal stride 2). Transposed, class (a, b), tap (u, v): ky = (a + 1)
               // mod 2 + 2u, input row y + (a + 1 - ky) / 2, column x + (b + 1 - kx) / 2.
               const int k0 = kc * BK;
               const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
-              int x, y;
+              // input row = ym * (tile row origin) + ya
+              int x, ya, ym;
               if (p.scatter) {
-                y = y0;
+                ym = 1;
+                ya = 0;
                 x = 0;
               } else if (p.transposed) {
                 const int a = cls >> 1, b = cls & 1;
                 const int ky = ((a + 1) & 1) + 2 * (tap >> 1), kx = ((b + 1) & 1) + 2 * (tap & 1);
-                y = y0 + ((a + 1 - ky) >> 1);
+                ym = 1;
+                ya = (a + 1 - ky) >> 1;
                 x = (b + 1 - kx) >> 1;
               } else {
-                y = 2 * y0 - 1 + (tap >> 2);
+                ym = 2;
+                ya = (tap >> 2) - 1;
                 x = (tap & 3) - 1;
               }
-              tma_load_5d(base + stage * STAGE_BYTES, &mA, bFullB + 8 * stage, c0, x, y, n0,
-                          p.transposed ? pc >> 2 : pc);
+              const int prob = p.transposed ? pc >> 2 : pc;
+              tma_load_5d(base + stage * STAGE_BYTES, &mA, bFullB + 8 * stage, c0, x,
+                          ym * y0 + ya, n0, prob);
+              if (p.m2)
+                tma_load_5d(base + stage * STAGE_BYTES + A_BYTES, &mA, bFullB + 8 * stage, c0, x,
+                            ym * y1 + ya, n1, prob);
             }
-            tma_load_3d(base + stage * STAGE_BYTES + A_BYTES, &mW, bFullB + 8 * stage, kc * BK,
-                        cls * p.cls_rows + j * 256, indiv);
+            tma_load_3d(base + stage * STAGE_BYTES + (p.m2 ? 2 : 1) * A_BYTES, &mW,
+                        bFullB + 8 * stage, kc * BK, cls * p.cls_rows + j * 256, indiv);
             issued[stage]++;
             if (++stage == STAGES) {
               stage = 0;
@@ -208,11 +218,16 @@ __global__ void __launch_bounds__(THREADS, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+            const uint32_t sA = base + stage * STAGE_BYTES;
+            const uint32_t sB = sA + (p.m2 ? 2 : 1) * A_BYTES;
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
+            for (int kk = 0; kk < BK / 16; ++kk) {
               tc_mma(dt, sw128_desc(sA + kk * 32), sw128_desc(sB + kk * 32), idesc,
                      (kc | kk) != 0 ? 1u : 0u);
+              if (p.m2)
+                tc_mma(dt + (uint32_t)nbox, sw128_desc(sA + A_BYTES + kk * 32),
+                       sw128_desc(sB + kk * 32), idesc, (kc | kk) != 0 ? 1u : 0u);
+            }
             tc_commit(bEmpty + 8 * stage);
             if (++stage == STAGES) {
               stage = 0;
@@ -388,7 +403,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int pc = tile / p.mtiles;
       const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
       const int cls = p.transposed ? (pc & 3) : 0;
-      const int m = (tile % p.mtiles) * BM + row;
+      const int m = (tile % p.mtiles) * (p.m2 ? 2 * BM : BM) + row;
       const bool valid = m < M;
       const int nb = m >> (2 * lq);
       int oy = (m >> lq) & ((1 << lq) - 1), ox = m & ((1 << lq) - 1);
@@ -396,8 +411,6 @@ __global__ void __launch_bounds__(THREADS, 1)
         oy = 2 * oy + (cls >> 1);
         ox = 2 * ox + (cls & 1);
       }
-      // output pixel index in the problem's image stack
-      const int64_t pix = ((int64_t)nb << (2 * p.lho)) + (oy << p.lho) + ox;
       for (int j = 0; j < p.nj && ok; ++j, ++jobs) {
         const int R = jobs & 1;
         // the scatter epilogue synchronises the four warps: they leave together
@@ -486,9 +499,20 @@ __global__ void __launch_bounds__(THREADS, 1)
               d.out[o] = __float2bfloat16_rn(x);
             }
         } else {
+          for (int h = 0; h < (p.m2 ? 2 : 1); ++h) {
+          // row m + 128 h of the tile (its accumulator columns start at h * nbox); valid and
+          // pix shadow the first half's
+          const int mh = m + h * BM;
+          const bool valid = mh < M;
+          int oyh = (mh >> lq) & ((1 << lq) - 1), oxh = mh & ((1 << lq) - 1);
+          if (p.transposed) {
+            oyh = 2 * oyh + (cls >> 1);
+            oxh = 2 * oxh + (cls & 1);
+          }
+          const int64_t pix = ((int64_t)(mh >> (2 * lq)) << (2 * p.lho)) + (oyh << p.lho) + oxh;
           for (int g = 0; g < nbox / 32; ++g) {
             uint32_t v[32];
-            LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
+            LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + h * nbox + g * 32), v);
             tmem_wait_ld();
             // the row's 32 columns go to the warp's staging rows (fp32 words, or bf16 pairs),
             // then out in 16-byte pieces, lpr lanes per row, so that each store instruction
@@ -550,6 +574,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               }
             }
             __syncwarp();
+          }
           }
         }
         tc_fence_before();
@@ -1291,9 +1316,10 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
 }
 
 bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
-                      std::string* msg) {
+                      std::string* msg, bool use_tma) {
   q->a_tma = 0;
-  if (q->nchw_in || q->ci % 64 != 0 || n_probs < 1) return true;
+  q->m2 = 0;
+  if (!use_tma || q->nchw_in || q->ci % 64 != 0 || n_probs < 1) return true;
   const int lq = q->scatter ? q->lhi : q->lho - q->transposed;
   if (lq > 7) return true;
   const int64_t Wi = (int64_t)1 << q->lhi;
@@ -1321,6 +1347,16 @@ bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int
     return false;
   }
   q->a_tma = 1;
+  // 256-row tiles (two accumulators sharing each weight chunk) for narrow weight tiles
+  if (!q->scatter && q->nbox <= 128 &&
+      (q->out_mode == CTC_LRELU_HWC || q->out_mode == CTC_F32_HWC ||
+       q->out_mode == CTC_DLRELU_HWC)) {
+    const int M = q->rows << (2 * lq);
+    const int mt2 = (M + 255) / 256;
+    q->n_tiles = q->n_tiles / q->mtiles * mt2;
+    q->mtiles = mt2;
+    q->m2 = 1;
+  }
   return true;
 }
 

@@ -49,6 +49,9 @@ struct CtcParams {
   // (problems x rows x 8 x 768 floats) and launch_scatter_fix completes them
   int scatter;
   float* halo;
+  // m2: 256-row tiles (set by ctc_make_act_map for channel-last outputs with nbox <= 128): two
+  // 128-row A boxes and two accumulators (columns h * nbox) share each weight chunk
+  int m2;
   const int* wsel;
   float slope;
   int* err;
@@ -99,10 +102,12 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
 // Activation map of a launch whose problems' channel-last inputs (ci a multiple of 64) sit at
 // a uniform stride from descs[0].in: dims (ci, W, W, rows, problems), a box of 64 channels by
 // the input pixels of 128 output pixels (traversal stride 2 for the convolution, 1 for the
-// parity classes). Sets q->a_tma = 1 when it applies (else 0, and the gather warps load A);
-// false only when the driver refuses the map.
+// parity classes). Sets q->a_tma = 1 when it applies (else 0, and the gather warps load A;
+// use_tma = false forces that), and then q->m2 and the 256-row tile count where they apply;
+// q->mtiles and q->n_tiles must count 128-row tiles on entry. False only when the driver
+// refuses the map.
 bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
-                      std::string* msg);
+                      std::string* msg, bool use_tma = true);
 bool ctc_prepare(std::string* msg);
 void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_problems, int rows,
                         int out_mode, cudaStream_t st);

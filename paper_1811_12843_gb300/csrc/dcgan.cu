@@ -237,9 +237,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   const char* gather_env = getenv("LIPZ_CONV_GATHER");
   const bool gather_a = gather_env && gather_env[0] == '1';
   auto act_map = [&](CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n) {
-    if (!ctc_make_act_map(m, q, descs, n, msg)) return false;
-    if (gather_a) q->a_tma = 0;
-    return true;
+    return ctc_make_act_map(m, q, descs, n, msg, !gather_a);
   };
   p->tct = tct;
   // ---- buffers
