@@ -19,7 +19,6 @@
 #include <stdint.h>
 
 #include <string>
-#include <type_traits>
 
 #include "common.cuh"
 #include "conv_tc.h"
@@ -34,8 +33,7 @@ constexpr int BM = 128, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = 256 * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-// warp 0 TMA, 1 MMA, 2-5 gather, 6-9 epilogue, 10-13 gather (the first layer only)
-constexpr int THREADS = 448;
+constexpr int THREADS = 320;  // warp 0 TMA, 1 MMA, 2-5 gather, 6-9 epilogue
 // first-layer input patches: 3 channels x 10 rows x 72 columns (64 interior at column 4)
 constexpr int PATCH_BYTES = 4352;
 // epilogue staging for coalesced row stores: 32 rows x 36 words per epilogue warp
@@ -66,12 +64,12 @@ __device__ __forceinline__ bool epi_bar_or(bool pred) {
   return r != 0;
 }
 
-// Barrier of the eight first-layer gather warps (named barrier 1) that returns whether any
-// thread passed true.
+// Barrier of the four gather warps (named barrier 1) that returns whether any thread passed
+// true.
 __device__ __forceinline__ bool gather_bar_or(bool pred) {
   uint32_t r;
   asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 256, p;\n"
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 128, p;\n"
       " selp.u32 %0, 1, 0, q;\n}"
       : "=r"(r)
       : "r"((uint32_t)pred)
@@ -95,7 +93,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(bFullA + 8 * s, p.nchw_in ? 256 : 128);
+      mbar_init(bFullA + 8 * s, 128);
       mbar_init(bFullB + 8 * s, 1);
       mbar_init(bEmpty + 8 * s, 1);
     }
@@ -244,11 +242,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 26);
     }
-  } else if ((warp < 6 || (warp >= 10 && p.nchw_in)) && !p.a_tma) {
+  } else if (warp < 6 && !p.a_tma) {
     // ---- A operand: thread r gathers row r of every k chunk. Channel-last rows arrive by
     // 16-byte cp.async (zero fill outside the image), a stage marked full LAG chunks later once
     // its copy group has landed; the first layer's rows are built from staged input patches.
-    const int r = warp < 6 ? threadIdx.x - 64 : threadIdx.x - 192;  // 0..255 (first layer)
+    const int r = threadIdx.x - 64;
     int stage = 0, arr_stage = 0, pending = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -260,7 +258,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       // cp.async into one of three shared buffers whose halo columns stay zero
       uint8_t* patches = misc + 256;
       const uint32_t patch0 = smem_u32(patches);
-      for (int i = r; i < 3 * PATCH_BYTES / 16; i += 256)
+      for (int i = r; i < 3 * PATCH_BYTES / 16; i += 128)
         *reinterpret_cast<uint4*>(patches + 16 * i) = make_uint4(0u, 0u, 0u, 0u);
       gather_bar_or(false);
       auto prefetch = [&](int tile, int buf) {
@@ -268,7 +266,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const ConvTcDesc d = p.descs[tile / p.mtiles];
           const int m0 = (tile % p.mtiles) * BM;
           const int nb = m0 >> 10, oy0 = (m0 >> 5) & 31;
-          for (int u = r; u < 480; u += 256) {
+          for (int u = r; u < 480; u += 128) {
             const int c = u / 160, rem = u - c * 160, pr = rem >> 4, q = rem & 15;
             const int iy = 2 * oy0 - 1 + pr;
             const bool in = iy >= 0 && iy < 64;
@@ -281,9 +279,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       };
       prefetch(blockIdx.x, 0);
       int buf = 0;
-      // thread r builds 16-byte units 4 (r >> 7) .. 4 (r >> 7) + 3 of row r & 127
-      const int rr = r & 127, half = r >> 7;
-      const int ox = rr & 31, oyl = rr >> 5;
+      const int ox = r & 31, oyl = r >> 5;
       for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
         prefetch(tile + gridDim.x, buf == 2 ? 0 : buf + 1);
         asm volatile("cp.async.wait_group 1;" ::: "memory");
@@ -292,43 +288,33 @@ __global__ void __launch_bounds__(THREADS, 1)
           ok = false;
           break;
         }
-        const bool valid = (tile % p.mtiles) * BM + rr < M;
+        const bool valid = (tile % p.mtiles) * BM + r < M;
         const unsigned short* pb =
             reinterpret_cast<const unsigned short*>(patches + buf * PATCH_BYTES);
-        const uint32_t row = base + stage * STAGE_BYTES + (uint32_t)rr * 128u;
-        // the unit range as a compile-time constant, so that every k folds to a fixed tap and
-        // channel (half is uniform across a warp)
-        auto build = [&](auto hc) {
-          constexpr int hh = decltype(hc)::value;
+        const uint32_t row = base + stage * STAGE_BYTES + (uint32_t)r * 128u;
 #pragma unroll
-          for (int uu = 0; uu < 4; ++uu) {
-            const int u = hh * 4 + uu;
-            uint32_t w[4];
+        for (int u = 0; u < 8; ++u) {
+          uint32_t w[4];
 #pragma unroll
-            for (int e2 = 0; e2 < 4; ++e2) {
-              uint32_t hv[2];
+          for (int e2 = 0; e2 < 4; ++e2) {
+            uint32_t hv[2];
 #pragma unroll
-              for (int h = 0; h < 2; ++h) {
-                const int k = u * 8 + e2 * 2 + h;
-                hv[h] = 0u;
-                if (k < 48) {
-                  const int tap = k / 3, c = k - 3 * tap;
-                  const int prow = 2 * oyl + (tap >> 2), col = 2 * ox + (tap & 3) + 3;
-                  hv[h] = valid ? (uint32_t)pb[(c * 10 + prow) * 72 + col] : 0u;
-                }
+            for (int h = 0; h < 2; ++h) {
+              const int k = u * 8 + e2 * 2 + h;
+              hv[h] = 0u;
+              if (k < 48) {
+                const int tap = k / 3, c = k - 3 * tap;
+                const int prow = 2 * oyl + (tap >> 2), col = 2 * ox + (tap & 3) + 3;
+                hv[h] = valid ? (uint32_t)pb[(c * 10 + prow) * 72 + col] : 0u;
               }
-              w[e2] = hv[0] | (hv[1] << 16);
             }
-            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                             row + ((uint32_t)(u ^ (rr & 7)) << 4)),
-                         "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                         : "memory");
+            w[e2] = hv[0] | (hv[1] << 16);
           }
-        };
-        if (half == 0)
-          build(std::integral_constant<int, 0>{});
-        else
-          build(std::integral_constant<int, 1>{});
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                           row + ((uint32_t)(u ^ (r & 7)) << 4)),
+                       "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                       : "memory");
+        }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         mbar_arrive(bFullA + 8 * stage);
         if (++stage == STAGES) {
@@ -405,7 +391,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_arrive(bFullA + 8 * arr_stage);
       arr_stage = arr_stage + 1 == STAGES ? 0 : arr_stage + 1;
     }
-  } else if (warp >= 6 && warp < 10) {
+  } else if (warp >= 6) {
     // ---- epilogue: LeakyReLU, bf16, channel-last rows
     const int q = warp & 3;
     const int row = q * 32 + lane;
