@@ -77,10 +77,21 @@ __device__ __forceinline__ bool gather_bar_or(bool pred) {
   return r != 0;
 }
 
+enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4 };
+
+// AK: how the A tiles arrive (AK_CONV / AK_TRANS / AK_SCATTER: TMA through the activation map
+// for the convolution, the parity classes, the scatter mode; AK_NCHW: built from staged
+// first-layer patches; AK_GATHER: gathered channel-last rows, convolution or parity classes as
+// p.transposed says). OM: the out_mode. Each launch runs the instantiation its parameters
+// name, so that a kernel holds only its own code paths.
+template <int AK, int OM>
 __global__ void __launch_bounds__(THREADS, 1)
     k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mA,
               const __grid_constant__ CtcParams p) {
   extern __shared__ uint8_t smem_raw[];
+  constexpr bool kTma = AK == AK_CONV || AK == AK_TRANS || AK == AK_SCATTER;
+  constexpr bool kScatter = AK == AK_SCATTER, kNchw = AK == AK_NCHW;
+  const bool transposed = AK == AK_TRANS || (AK == AK_GATHER && p.transposed);
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
@@ -118,7 +129,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   pdl_wait();
   // output pixels per problem (per parity class when transposed)
   // rows of a problem: output pixels (class pixels when transposed; input pixels in scatter)
-  const int lq = p.scatter ? p.lhi : p.lho - p.transposed;
+  const int lq = kScatter ? p.lhi : p.lho - (transposed ? 1 : 0);
   const int M = p.rows << (2 * lq);
   const int nbox = p.nbox;
 
@@ -130,8 +141,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         const int pc = tile / p.mtiles;  // problem (x 4 parity classes when transposed)
-        const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
-        const int cls = p.transposed ? (pc & 3) : 0;
+        const ConvTcDesc d = p.descs[transposed ? pc >> 2 : pc];
+        const int cls = transposed ? (pc & 3) : 0;
         const int indiv = __ldg(&p.wsel[d.wsel_idx]);
         // channel-last A rows by TMA (a_tma): the tile is 128 consecutive output pixels (class
         // pixels when transposed) of whole rows; its origin is image n0, row y0
@@ -146,8 +157,8 @@ __global__ void __launch_bounds__(THREADS, 1)
               break;
             }
             mbar_expect_tx(bFullB + 8 * stage,
-                           (uint32_t)(nbox * BK * 2 + (p.a_tma ? (p.m2 ? 2 : 1) * A_BYTES : 0)));
-            if (p.a_tma) {
+                           (uint32_t)(nbox * BK * 2 + (kTma ? (p.m2 ? 2 : 1) * A_BYTES : 0)));
+            if constexpr (kTma) {
               // Convolution: tap (ky, kx), input rows 2 y - 1 + ky, columns 2 x - 1 + kx (the
               // map's traversal stride 2). Transposed, class (a, b), tap (u, v): ky = (a + 1)
               // mod 2 + 2u, input row y + (a + 1 - ky) / 2, column x + (b + 1 - kx) / 2.
@@ -155,11 +166,11 @@ __global__ void __launch_bounds__(THREADS, 1)
               const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
               // input row = ym * (tile row origin) + ya
               int x, ya, ym;
-              if (p.scatter) {
+              if (kScatter) {
                 ym = 1;
                 ya = 0;
                 x = 0;
-              } else if (p.transposed) {
+              } else if (transposed) {
                 const int a = cls >> 1, b = cls & 1;
                 const int ky = ((a + 1) & 1) + 2 * (tap >> 1), kx = ((b + 1) & 1) + 2 * (tap & 1);
                 ym = 1;
@@ -170,7 +181,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 ya = (tap >> 2) - 1;
                 x = (tap & 3) - 1;
               }
-              const int prob = p.transposed ? pc >> 2 : pc;
+              const int prob = transposed ? pc >> 2 : pc;
               tma_load_5d(base + stage * STAGE_BYTES, &mA, bFullB + 8 * stage, c0, x,
                           ym * y0 + ya, n0, prob);
               if (p.m2)
@@ -212,7 +223,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           tc_fence_after();
           const uint32_t dt = tmem + (uint32_t)(R * 256);
           for (int kc = 0; kc < p.kchunks; ++kc) {
-            if ((!p.a_tma && !mbar_wait(bFullA + 8 * stage, phase, abort_flag, p.err, 24)) ||
+            if ((!kTma && !mbar_wait(bFullA + 8 * stage, phase, abort_flag, p.err, 24)) ||
                 !mbar_wait(bFullB + 8 * stage, phase, abort_flag, p.err, 25)) {
               ok = false;
               break;
@@ -242,7 +253,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 26);
     }
-  } else if (warp < 6 && !p.a_tma) {
+  } else if (warp < 6 && !kTma) {
     // ---- A operand: thread r gathers row r of every k chunk. Channel-last rows arrive by
     // 16-byte cp.async (zero fill outside the image), a stage marked full LAG chunks later once
     // its copy group has landed; the first layer's rows are built from staged input patches.
@@ -251,7 +262,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t phase = 0;
     bool ok = true;
     const int lhi = p.lhi, Hi = 1 << lhi;
-    if (p.nchw_in) {
+    if constexpr (kNchw) {
       // first layer (3 channels, 64 x 64 CHW images, 32 x 32 outputs, one k chunk of
       // k = (ky * 4 + kx) * 3 + c over 48 values): a tile's 128 rows are 4 output rows, fed by
       // a 3 x 10 x 64 input patch that the gather threads copy one tile ahead by 8-byte
@@ -326,13 +337,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
       const int pc = tile / p.mtiles;
-      const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
-      const int cls = p.transposed ? (pc & 3) : 0;
+      const ConvTcDesc d = p.descs[transposed ? pc >> 2 : pc];
+      const int cls = transposed ? (pc & 3) : 0;
       const int m = (tile % p.mtiles) * BM + r;
       const bool valid = m < M;
       const int nb = m >> (2 * lq);
       int oy = (m >> lq) & ((1 << lq) - 1), ox = m & ((1 << lq) - 1);
-      if (p.transposed) {
+      if (transposed) {
         oy = 2 * oy + (cls >> 1);
         ox = 2 * ox + (cls & 1);
       }
@@ -351,7 +362,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int k0 = kc * BK;
             const int tap = k0 / p.ci, c0 = k0 - tap * p.ci;
             int iy, ix, ty = 0, tx = 0;
-            if (p.transposed) {
+            if (transposed) {
               const int ky = ((oy + 1) & 1) + 2 * (tap >> 1), kx = ((ox + 1) & 1) + 2 * (tap & 1);
               ty = oy + 1 - ky;
               tx = ox + 1 - kx;
@@ -401,13 +412,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
       const int pc = tile / p.mtiles;
-      const ConvTcDesc d = p.descs[p.transposed ? pc >> 2 : pc];
-      const int cls = p.transposed ? (pc & 3) : 0;
+      const ConvTcDesc d = p.descs[transposed ? pc >> 2 : pc];
+      const int cls = transposed ? (pc & 3) : 0;
       const int m = (tile % p.mtiles) * (p.m2 ? 2 * BM : BM) + row;
       const bool valid = m < M;
       const int nb = m >> (2 * lq);
       int oy = (m >> lq) & ((1 << lq) - 1), ox = m & ((1 << lq) - 1);
-      if (p.transposed) {
+      if (transposed) {
         oy = 2 * oy + (cls >> 1);
         ox = 2 * ox + (cls & 1);
       }
@@ -416,12 +427,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         // the scatter epilogue synchronises the four warps: they leave together
         const bool okw =
             mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 28);
-        if (p.scatter ? epi_bar_or(!okw) : !okw) {
+        if (kScatter ? epi_bar_or(!okw) : !okw) {
           ok = false;
           break;
         }
         tc_fence_after();
-        if (p.scatter) {
+        if constexpr (kScatter) {
           // input pixel (y0 + q, lane) holds Y[tap * 4 + o] (16 taps, 3 channels); the taps are
           // added one after the other into the tile's 10 x 66 output window in shared memory
           // (output row 2 y - 1 + ky, column 2 x - 1 + kx; window origin (2 y0 - 1, -1))
@@ -462,7 +473,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               const int o = i / 384, rem = i - o * 384, lr = 2 + (rem >> 6), gx = rem & 63;
               const int64_t oi = (((int64_t)img * 3 + o) << 12) + ((8 * blk - 1 + lr) << 6) + gx;
               float x = acc[(lr * 66 + gx + 1) * 3 + o];
-              if (p.out_mode == CTC_TANH_CHW) {
+              if (OM == CTC_TANH_CHW) {
                 x = tanhf(x);
               } else {
                 const float f = __bfloat162float(d.aux[oi]);
@@ -479,7 +490,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           epi_bar();
           continue;
         }
-        if (p.out_mode == CTC_TANH_CHW || p.out_mode == CTC_DTANH_CHW) {
+        if (OM == CTC_TANH_CHW || OM == CTC_DTANH_CHW) {
           // a few output channels (the image's colours), channel-major images: tanh, or the
           // delta times tanh' = 1 - f^2 with f the stored tanh output
           uint32_t v[16];
@@ -490,7 +501,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (valid && e < p.co) {
               const int64_t o = (((int64_t)nb * p.co + e) << (2 * p.lho)) + (oy << p.lho) + ox;
               float x = __uint_as_float(v[e]);
-              if (p.out_mode == CTC_TANH_CHW) {
+              if (OM == CTC_TANH_CHW) {
                 x = tanhf(x);
               } else {
                 const float f = __bfloat162float(d.aux[o]);
@@ -505,7 +516,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int mh = m + h * BM;
           const bool valid = mh < M;
           int oyh = (mh >> lq) & ((1 << lq) - 1), oxh = mh & ((1 << lq) - 1);
-          if (p.transposed) {
+          if (transposed) {
             oyh = 2 * oyh + (cls >> 1);
             oxh = 2 * oxh + (cls & 1);
           }
@@ -517,7 +528,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             // the row's 32 columns go to the warp's staging rows (fp32 words, or bf16 pairs),
             // then out in 16-byte pieces, lpr lanes per row, so that each store instruction
             // writes whole rows' contiguous bytes
-            const bool f32 = p.out_mode == CTC_F32_HWC;
+            const bool f32 = OM == CTC_F32_HWC;
             if (f32) {
 #pragma unroll
               for (int u = 0; u < 8; ++u)
@@ -525,7 +536,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     make_uint4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
             } else {
             uint32_t pk[16];
-            if (p.out_mode == CTC_DLRELU_HWC) {
+            if (OM == CTC_DLRELU_HWC) {
               // the LeakyReLU derivative at the stored activation (same sign as its input)
               uint4 au[4] = {make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u),
                              make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
@@ -1360,20 +1371,60 @@ bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int
   return true;
 }
 
+namespace {
+using ConvKernel = void (*)(const CUtensorMap, const CUtensorMap, const CtcParams);
+struct ConvVariant {
+  int ak, om;
+  ConvKernel k;
+};
+// the (A kind, out mode) pairs the DCGAN launches use; the gathered form takes them all
+const ConvVariant kConvVariants[] = {
+    {ctc::AK_CONV, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_CONV, CTC_LRELU_HWC>},
+    {ctc::AK_CONV, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_CONV, CTC_F32_HWC>},
+    {ctc::AK_TRANS, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_TRANS, CTC_F32_HWC>},
+    {ctc::AK_TRANS, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_TRANS, CTC_TANH_CHW>},
+    {ctc::AK_TRANS, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_TRANS, CTC_DLRELU_HWC>},
+    {ctc::AK_TRANS, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_TRANS, CTC_DTANH_CHW>},
+    {ctc::AK_SCATTER, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_SCATTER, CTC_TANH_CHW>},
+    {ctc::AK_SCATTER, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_SCATTER, CTC_DTANH_CHW>},
+    {ctc::AK_NCHW, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_NCHW, CTC_LRELU_HWC>},
+    {ctc::AK_NCHW, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_NCHW, CTC_F32_HWC>},
+    {ctc::AK_GATHER, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_LRELU_HWC>},
+    {ctc::AK_GATHER, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_F32_HWC>},
+    {ctc::AK_GATHER, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_GATHER, CTC_TANH_CHW>},
+    {ctc::AK_GATHER, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_DLRELU_HWC>},
+    {ctc::AK_GATHER, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_GATHER, CTC_DTANH_CHW>},
+};
+
+ConvKernel conv_kernel(const CtcParams& p) {
+  const int ak = p.scatter ? ctc::AK_SCATTER
+                 : p.nchw_in ? ctc::AK_NCHW
+                 : p.a_tma   ? (p.transposed ? ctc::AK_TRANS : ctc::AK_CONV)
+                             : ctc::AK_GATHER;
+  for (const ConvVariant& v : kConvVariants)
+    if (v.ak == ak && v.om == p.out_mode) return v.k;
+  return nullptr;
+}
+}  // namespace
+
 bool ctc_prepare(std::string* msg) {
-  if (cudaFuncSetAttribute(ctc::k_conv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           ctc::SMEM_BYTES) != cudaSuccess) {
-    cudaGetLastError();
-    if (msg) *msg = "cannot reserve shared memory for the tensor-core convolution";
-    return false;
-  }
+  for (const ConvVariant& v : kConvVariants)
+    if (cudaFuncSetAttribute(v.k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ctc::SMEM_BYTES) != cudaSuccess) {
+      cudaGetLastError();
+      if (msg) *msg = "cannot reserve shared memory for the tensor-core convolution";
+      return false;
+    }
   return true;
 }
 
-void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
+bool launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
                     cudaStream_t st) {
+  const ConvKernel k = conv_kernel(p);
+  if (!k) return false;
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
-  launch_pdl(ctc::k_conv_tc, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, mA, p);
+  launch_pdl(k, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, mA, p);
+  return true;
 }
 
 void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_problems, int rows,

@@ -115,7 +115,8 @@ void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_proble
 // rows tap * 4 + output][64], the scatter mode's weights.
 void launch_relayout_s(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst, int n_indiv,
                        cudaStream_t st);
-void launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
+// False (and nothing launched) when no kernel variant serves p's A kind and out mode.
+bool launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,
                     cudaStream_t st);
 void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, const RelayoutD& r,
                        cudaStream_t st);

@@ -996,6 +996,11 @@ void dc_plan_destroy(DcPlan* p) {
 }
 
 namespace {
+int no_variant(std::string* msg) {
+  if (msg) *msg = "no tensor-core convolution variant for a layer's A kind and output mode";
+  return 1;
+}
+
 int check(std::string* msg, const char* what) {
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess) return 0;
@@ -1025,11 +1030,11 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
         q = p->egs;
         q.descs = p->gtd[i];
         q.wsel = nbr;
-        launch_conv_tc(p->mGs, p->aEgs, q, p->sms, st);
+        if (!launch_conv_tc(p->mGs, p->aEgs, q, p->sms, st)) return no_variant(msg);
         launch_scatter_fix(p->gtd[i], p->halo, PE, B, CTC_TANH_CHW, st);
         continue;
       }
-      launch_conv_tc(p->mG[i], p->aEg[i], q, p->sms, st);
+      if (!launch_conv_tc(p->mG[i], p->aEg[i], q, p->sms, st)) return no_variant(msg);
       if (i < 3)
         launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, p->bncnt, st);
     }
@@ -1061,7 +1066,7 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
         CtcParams q = p->cp[l - 1];
         q.descs = p->tcd[l - 1] + c * 5;
         q.wsel = nbr;
-        launch_conv_tc(p->mW[l - 1], p->aEd[l - 1], q, p->sms, st);
+        if (!launch_conv_tc(p->mW[l - 1], p->aEd[l - 1], q, p->sms, st)) return no_variant(msg);
       }
       launch_logit_dot(true, p->tcl + c * 5, 5, 6 * B, nbr, st);
     }
@@ -1098,11 +1103,11 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
         q = p->tgs;
         q.descs = p->tgd[i];
         q.wsel = p->b.src_g;
-        launch_conv_tc(p->mGs, p->aTgs, q, p->sms, st);
+        if (!launch_conv_tc(p->mGs, p->aTgs, q, p->sms, st)) return no_variant(msg);
         launch_scatter_fix(p->tgd[i], p->halo, C, B, CTC_TANH_CHW, st);
         continue;
       }
-      launch_conv_tc(p->mG[i], p->aTg[i], q, p->sms, st);
+      if (!launch_conv_tc(p->mG[i], p->aTg[i], q, p->sms, st)) return no_variant(msg);
       if (i < 3)
         launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, p->bncnt, st);
     }
@@ -1128,7 +1133,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->tdp[l - 1];
       q.descs = p->tdd[l - 1];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mW[l - 1], p->aTd[l - 1], q, p->sms, st);
+      if (!launch_conv_tc(p->mW[l - 1], p->aTd[l - 1], q, p->sms, st)) return no_variant(msg);
     }
     launch_logit_dot(true, p->tdl_tc, C, 2 * B, nullptr, st);
   } else {
@@ -1165,7 +1170,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->ddp[k];
       q.descs = p->ddd[k];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mDd[l - 1], p->aDd[k], q, p->sms, st);
+      if (!launch_conv_tc(p->mDd[l - 1], p->aDd[k], q, p->sms, st)) return no_variant(msg);
     } else if (l >= 2) {
       launch_conv(CONVT2_MODE, CEPI_DLRELU_, s.bf, false, p->dd[k], C,
                   2 * B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0, s.slope,
@@ -1180,13 +1185,13 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       CtcParams q = p->gds;
       q.descs = p->gdd[3];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mDs, p->aGds, q, p->sms, st);
+      if (!launch_conv_tc(p->mDs, p->aGds, q, p->sms, st)) return no_variant(msg);
       launch_scatter_fix(p->gdd[3], p->halo, C, B, CTC_DTANH_CHW, st);
     } else if (p->tct) {
       CtcParams q = p->gdp[4 - l];
       q.descs = p->gdd[4 - l];
       q.wsel = p->b.src_d;
-      launch_conv_tc(p->mDd[l - 1], p->aGd[4 - l], q, p->sms, st);
+      if (!launch_conv_tc(p->mDd[l - 1], p->aGd[4 - l], q, p->sms, st)) return no_variant(msg);
     } else {
       launch_conv(CONVT2_MODE, l == 1 ? CEPI_DTANH_ : CEPI_DLRELU_, s.bf, false,
                   p->gd[4 - l], C, B * ds[l - 1] * ds[l - 1], dc[l - 1], nullptr, 1, nullptr, 0,
@@ -1210,7 +1215,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
         CtcParams q = p->gcp[k];
         q.descs = p->gcd[k];
         q.wsel = p->b.src_g;
-        launch_conv_tc(p->mGc[k], p->aGc[k], q, p->sms, st);
+        if (!launch_conv_tc(p->mGc[k], p->aGc[k], q, p->sms, st)) return no_variant(msg);
       } else {
         launch_conv(CONV_FWD_MODE, CEPI_NONE_, s.bf, true, p->gdh[k], C,
                     B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
