@@ -614,6 +614,8 @@ constexpr int WG_STAGES = 4;
 constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256 + 4 * STG_WORDS * 4;
 constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_STAGES)
 
+// BCHW: p.b_chw at compile time (the 3-channel channel-major B operand)
+template <bool BCHW>
 __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constant__ WgtcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -651,7 +653,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
   pdl_wait();
   // b_chw: b is a 3-channel channel-major image stack, N = 48 (tap, channel) columns in one
   // 64-wide tile; M (a multiple of 64) may leave the upper half of a 128-row tile empty
-  const int mt_n = (p.M + 127) / 128, nt_n = p.b_chw ? 1 : p.N / 256;
+  const int mt_n = (p.M + 127) / 128, nt_n = BCHW ? 1 : p.N / 256;
   const int per_split = mt_n * nt_n;
   const int la = p.la, lb = p.lb;
   const int64_t Kp = (int64_t)p.rows << (2 * la);  // pixels of A per problem
@@ -664,7 +666,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
       int stage = 0, uses[2] = {0, 0}, jobs = 0;
       uint32_t phase = 0;
       bool ok = true;
-      const uint32_t idesc = idesc_bf16_major(128, p.b_chw ? 64 : 256, 1, 1);
+      const uint32_t idesc = idesc_bf16_major(128, BCHW ? 64 : 256, 1, 1);
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++jobs) {
         const int split = (tile / per_split) % p.splits;
         int64_t k0, k1;
@@ -740,7 +742,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
           for (int u = 0; u < 8; ++u)
             cp_async16(dst + (((uint32_t)u ^ sw) << 4), src + (av ? 8 * u : 0), av ? 16 : 0);
         }
-        if (p.b_chw) {
+        if constexpr (BCHW) {
           // row `row` of the single B atom, columns k = tap * 3 + c (k < 48, zero above);
           // thread half h writes the 16-byte units 4h .. 4h + 3 (k = 32h .. 32h + 31)
 #pragma unroll
@@ -826,7 +828,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
       tc_fence_after();
       float* o = p.part + (((int64_t)prob * p.splits + split) * p.M + mt * 128 + r) * p.N +
                  nt * 256;
-      const int groups = p.b_chw ? 2 : 8;
+      constexpr int groups = BCHW ? 2 : 8;
       for (int g = 0; g < groups; ++g) {
         uint32_t v[32];
         LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + g * 32), v);
@@ -1222,7 +1224,9 @@ __global__ void __launch_bounds__(256) k_bn_back_apply_hwc(const BnDesc* __restr
 }  // namespace ctc
 
 bool wgtc_prepare(std::string* msg) {
-  if (cudaFuncSetAttribute(ctc::k_wgrad_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(ctc::k_wgrad_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           ctc::WG_SMEM) != cudaSuccess ||
+      cudaFuncSetAttribute(ctc::k_wgrad_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            ctc::WG_SMEM) != cudaSuccess) {
     cudaGetLastError();
     if (msg) *msg = "cannot reserve shared memory for the tensor-core weight gradients";
@@ -1233,7 +1237,8 @@ bool wgtc_prepare(std::string* msg) {
 
 void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st) {
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
-  launch_pdl(ctc::k_wgrad_tc, dim3(grid), dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, p);
+  launch_pdl(p.b_chw ? ctc::k_wgrad_tc<true> : ctc::k_wgrad_tc<false>, dim3(grid),
+             dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, p);
   if (p.b_chw)
     launch_pdl(ctc::k_wgrad_tc_reduce_chw, dim3((p.M * 48 + 255) / 256, p.n_probs), dim3(256), 0,
                st, p);
