@@ -422,6 +422,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         oy = 2 * oy + (cls >> 1);
         ox = 2 * ox + (cls & 1);
       }
+      // CTC_LRELU_LOGIT: this row's share of its image's logit (the 4 x 4 x C output layer on
+      // the bf16 activations, pixel = row mod 16), summed over the jobs
+      float dot = 0.f;
+      const bf16* w5 = nullptr;
+      if constexpr (OM == CTC_LRELU_LOGIT)
+        w5 = p.logit_w + (int64_t)__ldg(&p.wsel[d.wsel_idx]) * p.logit_ws + (int64_t)(m & 15) * p.co;
       for (int j = 0; j < p.nj && ok; ++j, ++jobs) {
         const int R = jobs & 1;
         // the scatter epilogue synchronises the four warps: they leave together
@@ -563,11 +569,31 @@ __global__ void __launch_bounds__(THREADS, 1)
                 pk[e >> 1] = pack_bf16(a, b);
               }
             }
+            if constexpr (OM == CTC_LRELU_LOGIT) {
+              // the output layer instead of storing the activations
+              const uint4* wp = reinterpret_cast<const uint4*>(w5 + j * 256 + g * 32);
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-              *reinterpret_cast<uint4*>(stg + lane * 36 + 4 * u) =
-                  make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+              for (int u = 0; u < 4; ++u) {
+                const uint4 wv = __ldg(wp + u);
+                const uint32_t ww[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const float2 af =
+                      __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[4 * u + e]));
+                  const float2 wf =
+                      __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ww[e]));
+                  dot = fmaf(af.x, wf.x, dot);
+                  dot = fmaf(af.y, wf.y, dot);
+                }
+              }
+            } else {
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<uint4*>(stg + lane * 36 + 4 * u) =
+                    make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
             }
+            }
+            if constexpr (OM == CTC_LRELU_LOGIT) continue;
             __syncwarp();
             const int lpr = f32 ? 8 : 4, rpi = 32 / lpr;
             const int part = lane % lpr;
@@ -591,6 +617,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc_fence_before();
         mbar_arrive(bAccE + 8 * R);
         uses[R]++;
+      }
+      if constexpr (OM == CTC_LRELU_LOGIT) {
+        // an image's 16 pixels are 16 consecutive rows (lanes); fixed-order tree
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+        if (ok && (lane & 15) == 0 && valid) d.logits[m >> 4] = dot;
       }
     }
   }
@@ -1386,6 +1418,7 @@ struct ConvVariant {
 const ConvVariant kConvVariants[] = {
     {ctc::AK_CONV, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_CONV, CTC_LRELU_HWC>},
     {ctc::AK_CONV, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_CONV, CTC_F32_HWC>},
+    {ctc::AK_CONV, CTC_LRELU_LOGIT, ctc::k_conv_tc<ctc::AK_CONV, CTC_LRELU_LOGIT>},
     {ctc::AK_TRANS, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_TRANS, CTC_F32_HWC>},
     {ctc::AK_TRANS, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_TRANS, CTC_TANH_CHW>},
     {ctc::AK_TRANS, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_TRANS, CTC_DLRELU_HWC>},
@@ -1399,6 +1432,7 @@ const ConvVariant kConvVariants[] = {
     {ctc::AK_GATHER, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_GATHER, CTC_TANH_CHW>},
     {ctc::AK_GATHER, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_DLRELU_HWC>},
     {ctc::AK_GATHER, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_GATHER, CTC_DTANH_CHW>},
+    {ctc::AK_GATHER, CTC_LRELU_LOGIT, ctc::k_conv_tc<ctc::AK_GATHER, CTC_LRELU_LOGIT>},
 };
 
 ConvKernel conv_kernel(const CtcParams& p) {

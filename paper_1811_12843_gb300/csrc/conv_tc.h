@@ -21,6 +21,7 @@ struct ConvTcDesc {
   const bf16* aux;  // CTC_DLRELU_HWC / CTC_DTANH_CHW: the activation whose derivative applies
   int wsel_idx;
   int pad;
+  float* logits;  // CTC_LRELU_LOGIT: one logit per image
 };
 
 // A launch: problems of `rows` images; 4x4 / stride 2 / pad 1 convolution from ci x 2^lhi
@@ -35,8 +36,11 @@ struct ConvTcDesc {
 // images; co <= 16).
 // CTC_DLRELU_HWC: bf16 delta times the LeakyReLU derivative at aux (channel-last);
 // CTC_DTANH_CHW: bf16 delta times 1 - aux^2 (aux the tanh output), channel-major images.
+// CTC_LRELU_LOGIT: LeakyReLU as CTC_LRELU_HWC, then the 4 x 4 output layer in the epilogue
+// (4 x 4 outputs; logit_w / logit_ws the output layer's [16 pixels][co] weights of each
+// individual): one logit per image into the descriptor's logits, the activations not stored.
 enum { CTC_LRELU_HWC = 0, CTC_F32_HWC = 1, CTC_TANH_CHW = 2, CTC_DLRELU_HWC = 3,
-       CTC_DTANH_CHW = 4 };
+       CTC_DTANH_CHW = 4, CTC_LRELU_LOGIT = 5 };
 struct CtcParams {
   const ConvTcDesc* descs;
   int rows, ci, lhi, co, lho, nchw_in, kchunks, nj, nbox, mtiles, n_tiles;
@@ -52,6 +56,8 @@ struct CtcParams {
   // m2: 256-row tiles (set by ctc_make_act_map for channel-last outputs with nbox <= 128): two
   // 128-row A boxes and two accumulators (columns h * nbox) share each weight chunk
   int m2;
+  const bf16* logit_w;  // CTC_LRELU_LOGIT
+  int64_t logit_ws;
   const int* wsel;
   float slope;
   int* err;

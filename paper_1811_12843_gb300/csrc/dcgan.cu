@@ -98,7 +98,6 @@ struct DcPlan {
   CUtensorMap mW[4];
   CtcParams cp[4];
   ConvTcDesc* tcd[4];
-  LogitDesc* tcl;
   RelayoutD rel;
   int* err = nullptr;
   int sms = 148;
@@ -553,6 +552,12 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       q.n_tiles = 5 * q.mtiles;
       q.slope = s.slope;
       q.err = p->err;
+      if (l == 4) {
+        // the output layer in layer 4's epilogue: the logits straight into the fitness input
+        q.out_mode = CTC_LRELU_LOGIT;
+        q.logit_w = p->Dwt + dof[4];
+        q.logit_ws = b.PDs;
+      }
       p->cp[l - 1] = q;
       std::vector<ConvTcDesc> vt;
       for (int c = 0; c < C; ++c)
@@ -563,30 +568,19 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
           memset(&t, 0, sizeof t);
           t.in = (const bf16*)(l == 1 ? el(b.E, (int64_t)c * b.e_cell) : (l % 2 == 0 ? bx : by));
           t.out = (bf16*)(l % 2 == 1 ? bx : by);
+          t.logits = b.logits + (int64_t)(c * 5 + sl) * 6 * B;
           t.wsel_idx = c * 5 + sl;
           vt.push_back(t);
         }
       ok = ok && !upload(p, &p->tcd[l - 1], vt, msg);
       // one map serves every cell: the chunk buffers are shared
       ok = ok && act_map(&p->aEd[l - 1], &p->cp[l - 1], vt.data(), 5);
-      for (size_t k = 5; k < vt.size(); ++k)
-        if (vt[k].in != vt[k % 5].in) p->cp[l - 1].a_tma = 0;
+      for (size_t k = 5; k < vt.size() && ok && l >= 2; ++k)
+        if (vt[k].in != vt[k % 5].in) {
+          if (msg) *msg = "DCGAN evaluation buffers differ between cells";
+          ok = false;
+        }
     }
-    std::vector<LogitDesc> vl;
-    for (int c = 0; c < C; ++c)
-      for (int sl = 0; sl < 5; ++sl) {
-        LogitDesc q;
-        memset(&q, 0, sizeof q);
-        q.a = elw(ey, (int64_t)sl * 6 * B * dsz[2]);
-        q.w = p->Dwt + dof[4];
-        q.wsel_stride = b.PDs;
-        q.wsel_idx = c * 5 + sl;
-        q.logits = b.logits + (int64_t)(c * 5 + sl) * 6 * B;
-        q.rows = 6 * B;
-        q.K = (int)dsz[4];
-        vl.push_back(q);
-      }
-    ok = ok && !upload(p, &p->tcl, vl, msg);
   }
   // ---- tensor-core generator evaluation (layers 2-5)
   if (ok && p->tcg) {
@@ -684,6 +678,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       q.rows = 2 * B;
       q.mtiles = ((2 * B << (2 * q.lho)) + 127) / 128;
       q.n_tiles = C * q.mtiles;
+      q.out_mode = CTC_LRELU_HWC;  // training keeps the activations (the backward reads them)
+      q.logit_w = nullptr;
       p->tdp[l - 1] = q;
       std::vector<ConvTcDesc> vt;
       for (int c = 0; c < C; ++c) {
@@ -1068,7 +1064,6 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
         q.wsel = nbr;
         if (!launch_conv_tc(p->mW[l - 1], p->aEd[l - 1], q, p->sms, st)) return no_variant(msg);
       }
-      launch_logit_dot(true, p->tcl + c * 5, 5, 6 * B, nbr, st);
     }
     return check(msg, "DCGAN discriminator evaluation (tensor cores)");
   }
@@ -1231,7 +1226,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
 
 int dc_eval_launches(const DcPlan* p, int part) {
   if (part == 0) return p->tcg ? 14 + (p->scg ? 2 : 0) : 9;
-  return p->eval_launches - 9 + (p->tc ? 1 : 0);
+  return p->eval_launches - 9 + (p->tc ? 1 - p->s.cells : 0);
 }
 
 int* dc_error_flag(DcPlan* p) { return p && (p->tc || p->tcg) ? p->err : nullptr; }
