@@ -101,16 +101,17 @@ struct Job {
   int epi;
 };
 
+template <int KND>
 __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   Job J;
-  if (p.kind == KIND_GRAM) {
+  if (KND == KIND_GRAM) {
     // column block j of the Gram matrix: MMA N rounded up to 16 (rows past 6B read as zero)
     const int n = min(HID, p.rows - j * HID);
     J = Job{0, p.kc1, (n + 15) & ~15, j & 1, 0, j * HID, HID, EPI_GRAM};
   } else if (j == 0) {
     J = Job{0, p.kc1, HID, 0, 0, 0, HID, EPI_TO_H};
   } else if (j == 1) {
-    const int epi = p.kind == KIND_D ? EPI_LOGIT : (p.train ? EPI_ACT_OUT : EPI_TO_H);
+    const int epi = KND == KIND_D ? EPI_LOGIT : (p.train ? EPI_ACT_OUT : EPI_TO_H);
     J = Job{1, HID / BK, HID, 1, 1, 0, HID, epi};
   } else {
     const int nb = j - 2;
@@ -122,18 +123,21 @@ __device__ __forceinline__ Job get_job(const KParams& p, int j) {
   return J;
 }
 
+template <int KND>
 __device__ __forceinline__ int n_jobs(const KParams& p) {
-  if (p.kind == KIND_GRAM) return (p.rows + HID - 1) / HID;
-  return (p.kind == KIND_D || p.train) ? 2 : 2 + p.n3;
+  if (KND == KIND_GRAM) return (p.rows + HID - 1) / HID;
+  return (KND == KIND_D || p.train) ? 2 : 2 + p.n3;
 }
 
 // Problem -> (cell whose activations are the A operand, individual whose weights are B).
+template <int KND>
 __device__ __forceinline__ int prob_cell(const KParams& p, int prob) {
-  return (p.train || p.centre || p.kind == KIND_GRAM) ? prob : prob / 5;
+  return (p.train || p.centre || KND == KIND_GRAM) ? prob : prob / 5;
 }
+template <int KND>
 __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
-  if (p.kind == KIND_GRAM) return prob;
+  if (KND == KIND_GRAM) return prob;
   return p.centre ? p.indiv_off + prob : __ldg(&p.nbr[prob]);
 }
 
@@ -146,6 +150,8 @@ __device__ __forceinline__ float tanh_approx(float x) {
 }
 
 // ---- the kernel ----------------------------------------------------------------------------
+// KND: p.kind at compile time (one variant per network kind, each with only its own paths)
+template <int KND>
 __global__ void __launch_bounds__(THREADS, 1)
     k_mlp_fwd(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB1,
               const __grid_constant__ CUtensorMap mB2, const __grid_constant__ CUtensorMap mB3,
@@ -199,7 +205,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int nj = n_jobs(p);
+  const int nj = n_jobs<KND>(p);
   // the set-up above touched no global memory: from here on the previous kernel's results
   // are needed (programmatic dependent launch)
   pdl_wait();
@@ -213,10 +219,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
-        const int c = prob_cell(p, prob);
-        const int k = prob_individual(p, prob);
+        const int c = prob_cell<KND>(p, prob);
+        const int k = prob_individual<KND>(p, prob);
         for (int j = 0; j < nj && ok; ++j) {
-          const Job J = get_job(p, j);
+          const Job J = get_job<KND>(p, j);
           const CUtensorMap* mb = J.bmap == 0 ? &mB1 : (J.bmap == 1 ? &mB2 : &mB3);
           for (int kc = 0; kc < J.kchunks; ++kc) {
             if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 1)) {
@@ -265,9 +271,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       int jobs_done = 0;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         for (int j = 0; j < nj && ok; ++j, ++jobs_done) {
-          const Job J = get_job(p, j);
+          const Job J = get_job<KND>(p, j);
           // the Gram kind alternates the two accumulators over all its jobs (3 per tile)
-          const int R = p.kind == KIND_GRAM ? (jobs_done & 1) : J.region;
+          const int R = KND == KIND_GRAM ? (jobs_done & 1) : J.region;
           if (reg_uses[R] > 0 &&
               !mbar_wait(bReg + 8 * R, (uint32_t)((reg_uses[R] - 1) & 1), abort_flag, p.err, 2)) {
             ok = false;
@@ -325,8 +331,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int et = threadIdx.x - 64;  // epilogue thread 0..255
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++ltile) {
       const int prob = tile / p.mtiles, m0 = (tile % p.mtiles) * BM;
-      const int c = prob_cell(p, prob), slot = p.centre ? 0 : prob % 5;
-      const int k = prob_individual(p, prob);
+      const int c = prob_cell<KND>(p, prob), slot = p.centre ? 0 : prob % 5;
+      const int k = prob_individual<KND>(p, prob);
       const float* wm = p.wmaster ? p.wmaster + (int64_t)k * p.pstride : nullptr;
       const int rr = m0 + row;
       const bool row_ok = rr < p.rows;
@@ -335,7 +341,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       // run, so that no epilogue waits on a global load. Buffer ltile & 1; a thread cannot
       // reach tile ltile + 2 before every thread has passed this tile's arrival.
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
-      if (p.kind == KIND_GRAM) {
+      if (KND == KIND_GRAM) {
         // the squared norms of the cell's rows (the Gram tile's row and column terms)
         // -|e_s|^2 / x for the cell's rows s, zero for the 32 entries past the last row
         const float ix = 1.f / (float)p.x;
@@ -349,7 +355,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       } else {
         // every load is issued before the first is stored, so their latencies overlap
-        const int nb3 = p.kind == KIND_D ? HID + 1 : p.x;
+        const int nb3 = KND == KIND_D ? HID + 1 : p.x;
         constexpr int NV = (BIAS_MAX + 32 * NUM_EPI_WARPS - 1) / (32 * NUM_EPI_WARPS);
         float v[NV];
 #pragma unroll
@@ -359,7 +365,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (i >= 512 + nb3) continue;
           if (i < 256) v[u] = wm[p.off_b1 + i];
           else if (i < 512) v[u] = wm[p.off_b2 + i - 256];
-          else if (p.kind == KIND_D)
+          else if (KND == KIND_D)
             v[u] = i < 512 + HID
                        ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
                        : wm[p.off_b3];
@@ -378,8 +384,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
       for (int j = 0; j < nj && ok; ++j, ++jobs_done) {
-        const Job J = get_job(p, j);
-        const int R = p.kind == KIND_GRAM ? (jobs_done & 1) : J.region;
+        const Job J = get_job<KND>(p, j);
+        const int R = KND == KIND_GRAM ? (jobs_done & 1) : J.region;
         if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
           ok = false;
           break;
@@ -388,7 +394,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t tbase = tmem + lane_base + (uint32_t)(R * HID);
         if (J.epi == EPI_TO_H || J.epi == EPI_ACT_OUT) {
           const float* bias = sb + (j == 0 ? 0 : 256);
-          const bool lrelu = p.kind == KIND_D;
+          const bool lrelu = KND == KIND_D;
           const bool to_h = J.epi == EPI_TO_H;
           bf16* gout = j == 0 ? p.act1 : p.act2;
           // chunk by chunk (64 columns, both column halves at once), so that the next layer's
@@ -715,7 +721,12 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (cudaFuncSetAttribute(tc::k_mlp_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(tc::k_mlp_fwd<tc::KIND_G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tc::SMEM_BYTES) != cudaSuccess ||
+      cudaFuncSetAttribute(tc::k_mlp_fwd<tc::KIND_D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tc::SMEM_BYTES) != cudaSuccess ||
+      cudaFuncSetAttribute(tc::k_mlp_fwd<tc::KIND_GRAM>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize,
                            tc::SMEM_BYTES) != cudaSuccess) {
     cudaGetLastError();
     if (msg) *msg = "cannot reserve shared memory for the tensor-core forward";
@@ -817,7 +828,10 @@ namespace {
 int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensorMap& b2,
            const CUtensorMap& b3, const tc::KParams& kp, cudaStream_t st, const char* what,
            std::string* msg) {
-  launch_pdl(tc::k_mlp_fwd, dim3(grid), dim3(tc::THREADS), tc::SMEM_BYTES, st, a, b1, b2, b3, kp);
+  auto k = kp.kind == tc::KIND_GRAM ? tc::k_mlp_fwd<tc::KIND_GRAM>
+           : kp.kind == tc::KIND_D  ? tc::k_mlp_fwd<tc::KIND_D>
+                                    : tc::k_mlp_fwd<tc::KIND_G>;
+  launch_pdl(k, dim3(grid), dim3(tc::THREADS), tc::SMEM_BYTES, st, a, b1, b2, b3, kp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     if (msg) *msg = std::string(what) + " launch: " + cudaGetErrorString(e);
