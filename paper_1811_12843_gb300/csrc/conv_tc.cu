@@ -77,7 +77,13 @@ __device__ __forceinline__ bool gather_bar_or(bool pred) {
   return r != 0;
 }
 
-enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4 };
+enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4, AK_NCHW_WIDE = 5 };
+
+// dynamic shared memory of a variant
+constexpr int conv_smem(int ak) {
+  return ak == AK_NCHW ? 1024 + 3 * (A_BYTES + 64 * BK * 2) + 256 + 3 * PATCH_BYTES + 4 * STG_WORDS * 4
+                       : SMEM_BYTES;
+}
 
 // AK: how the A tiles arrive (AK_CONV / AK_TRANS / AK_SCATTER: TMA through the activation map
 // for the convolution, the parity classes, the scatter mode; AK_NCHW: built from staged
@@ -85,12 +91,18 @@ enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4 };
 // p.transposed says). OM: the out_mode. Each launch runs the instantiation its parameters
 // name, so that a kernel holds only its own code paths.
 template <int AK, int OM>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(THREADS, AK == AK_NCHW ? 2 : 1)
     k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mA,
               const __grid_constant__ CtcParams p) {
   extern __shared__ uint8_t smem_raw[];
   constexpr bool kTma = AK == AK_CONV || AK == AK_TRANS || AK == AK_SCATTER;
-  constexpr bool kScatter = AK == AK_SCATTER, kNchw = AK == AK_NCHW;
+  constexpr bool kScatter = AK == AK_SCATTER, kNchw = AK == AK_NCHW || AK == AK_NCHW_WIDE;
+  // AK_NCHW (weight tiles of at most 64 rows): three 24 KB stages and 256 TMEM columns, so
+  // that two CTAs share an SM
+  constexpr bool kCompact = AK == AK_NCHW;
+  constexpr int STAGES = kCompact ? 3 : ctc::STAGES;
+  constexpr uint32_t STAGE_BYTES = kCompact ? A_BYTES + 64 * BK * 2 : ctc::STAGE_BYTES;
+  constexpr uint32_t kTmemCols = kCompact ? 256 : 512, kAccStride = kCompact ? 128 : 256;
   const bool transposed = AK == AK_TRANS || (AK == AK_GATHER && p.transposed);
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -118,8 +130,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
-        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32((const void*)tmem_slot)),
+                 "r"(kTmemCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   tc_fence_before();
@@ -136,7 +149,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (warp == 0) {
     // ---- weights by TMA
     if (lane == 0) {
-      int stage = 0, issued[STAGES] = {0, 0, 0, 0};
+      int stage = 0, issued[STAGES] = {};
       uint32_t phase = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
@@ -221,7 +234,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t dt = tmem + (uint32_t)(R * 256);
+          const uint32_t dt = tmem + (uint32_t)(R * kAccStride);
           for (int kc = 0; kc < p.kchunks; ++kc) {
             if ((!kTma && !mbar_wait(bFullA + 8 * stage, phase, abort_flag, p.err, 24)) ||
                 !mbar_wait(bFullB + 8 * stage, phase, abort_flag, p.err, 25)) {
@@ -448,8 +461,8 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int img = m0t >> 10, blk = (m0t >> 7) & 7;
           for (int i = et; i < 1980; i += 128) acc[i] = 0.f;
           uint32_t v[32], w[32];  // columns 0..31 (taps 0..7) and 32..63 (taps 8..15)
-          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256), v);
-          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + 32), w);
+          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * kAccStride), v);
+          LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * kAccStride + 32), w);
           tmem_wait_ld();
           tc_fence_before();
           mbar_arrive(bAccE + 8 * R);
@@ -500,7 +513,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           // a few output channels (the image's colours), channel-major images: tanh, or the
           // delta times tanh' = 1 - f^2 with f the stored tanh output
           uint32_t v[16];
-          LIPZ_TMEM_LD16(tmem + lane_base + (uint32_t)(R * 256), v);
+          LIPZ_TMEM_LD16(tmem + lane_base + (uint32_t)(R * kAccStride), v);
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 16; ++e)
@@ -529,7 +542,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int64_t pix = ((int64_t)(mh >> (2 * lq)) << (2 * p.lho)) + (oyh << p.lho) + oxh;
           for (int g = 0; g < nbox / 32; ++g) {
             uint32_t v[32];
-            LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * 256 + h * nbox + g * 32), v);
+            LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * kAccStride + h * nbox + g * 32), v);
             tmem_wait_ld();
             // the row's 32 columns go to the warp's staging rows (fp32 words, or bf16 pairs),
             // then out in 16-byte pieces, lpr lanes per row, so that each store instruction
@@ -631,7 +644,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols));
 }
 
 // ---- weight gradients on tcgen05 -----------------------------------------------------------
@@ -1427,6 +1441,8 @@ const ConvVariant kConvVariants[] = {
     {ctc::AK_SCATTER, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_SCATTER, CTC_DTANH_CHW>},
     {ctc::AK_NCHW, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_NCHW, CTC_LRELU_HWC>},
     {ctc::AK_NCHW, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_NCHW, CTC_F32_HWC>},
+    {ctc::AK_NCHW_WIDE, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_NCHW_WIDE, CTC_LRELU_HWC>},
+    {ctc::AK_NCHW_WIDE, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_NCHW_WIDE, CTC_F32_HWC>},
     {ctc::AK_GATHER, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_LRELU_HWC>},
     {ctc::AK_GATHER, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_GATHER, CTC_F32_HWC>},
     {ctc::AK_GATHER, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_GATHER, CTC_TANH_CHW>},
@@ -1435,11 +1451,15 @@ const ConvVariant kConvVariants[] = {
     {ctc::AK_GATHER, CTC_LRELU_LOGIT, ctc::k_conv_tc<ctc::AK_GATHER, CTC_LRELU_LOGIT>},
 };
 
+int conv_ak(const CtcParams& p) {
+  return p.scatter   ? ctc::AK_SCATTER
+         : p.nchw_in ? (p.nbox <= 64 ? ctc::AK_NCHW : ctc::AK_NCHW_WIDE)
+         : p.a_tma   ? (p.transposed ? ctc::AK_TRANS : ctc::AK_CONV)
+                     : ctc::AK_GATHER;
+}
+
 ConvKernel conv_kernel(const CtcParams& p) {
-  const int ak = p.scatter ? ctc::AK_SCATTER
-                 : p.nchw_in ? ctc::AK_NCHW
-                 : p.a_tma   ? (p.transposed ? ctc::AK_TRANS : ctc::AK_CONV)
-                             : ctc::AK_GATHER;
+  const int ak = conv_ak(p);
   for (const ConvVariant& v : kConvVariants)
     if (v.ak == ak && v.om == p.out_mode) return v.k;
   return nullptr;
@@ -1449,7 +1469,7 @@ ConvKernel conv_kernel(const CtcParams& p) {
 bool ctc_prepare(std::string* msg) {
   for (const ConvVariant& v : kConvVariants)
     if (cudaFuncSetAttribute(v.k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             ctc::SMEM_BYTES) != cudaSuccess) {
+                             ctc::conv_smem(v.ak)) != cudaSuccess) {
       cudaGetLastError();
       if (msg) *msg = "cannot reserve shared memory for the tensor-core convolution";
       return false;
@@ -1461,8 +1481,10 @@ bool launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParam
                     cudaStream_t st) {
   const ConvKernel k = conv_kernel(p);
   if (!k) return false;
-  const int grid = p.n_tiles < sms ? p.n_tiles : sms;
-  launch_pdl(k, dim3(grid), dim3(ctc::THREADS), ctc::SMEM_BYTES, st, mW, mA, p);
+  const int ak = conv_ak(p);
+  const int ctas = ak == ctc::AK_NCHW ? 2 * sms : sms;  // the compact variant: two per SM
+  const int grid = p.n_tiles < ctas ? p.n_tiles : ctas;
+  launch_pdl(k, dim3(grid), dim3(ctc::THREADS), ctc::conv_smem(ak), st, mW, mA, p);
   return true;
 }
 
