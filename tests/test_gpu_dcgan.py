@@ -90,7 +90,8 @@ def test_dcgan_tensor_core_eval(L, rows, cols, batch, ngf):
 
 @pytest.mark.parametrize("precision,width,rows,cols,batch", [("fp32", 4, 2, 2, 4),
                                                             ("bf16", 4, 2, 2, 4),
-                                                            ("bf16", 64, 1, 2, 16)])
+                                                            ("bf16", 64, 1, 2, 16),
+                                                            ("bf16", (128, 64), 1, 1, 16)])
 def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
     """Selection bit-exact given the engine's fitness; then the last step's gradients and the
     Adam state per cell against the oracle (a cell whose pre-activations came within rounding
@@ -98,9 +99,16 @@ def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
     forward on the tensor-core kernel with channel-last activations. At that width every cell
     has pre-activations within 1e-8 of a kink, and batch normalisation's backward spreads a
     flipped derivative over the whole channel: the CUDA-core and the tensor-core paths both
-    reach 1.4-4.7 % there (B = 16), so that case is held to 7.5 % per cell and 5 % median."""
+    reach 1.4-4.7 % there (B = 16), so that case is held to 7.5 % per cell and 5 % median.
+    A generator twice as wide (ngf 128, ndf 64) takes the kernel variants the width-64 case
+    does not: the output layer by parity class, and the wide first-layer variant for the
+    generator's input gradient. Its single cell lands at 6.9 % with the tensor cores and 6.8 %
+    with the CUDA-core kernels (measured side by side on the same inputs; the two differ from
+    each other by 7 %), so it is held to the 7.5 % per-cell rule only."""
     pool = _field_pool(3, 40)
-    g = _grid(L, rows, cols, 11, pool, precision=precision, keep_grads=1, ngf=width, ndf=width,
+    ngf, ndf = width if isinstance(width, tuple) else (width, width)
+    width = min(ngf, ndf)
+    g = _grid(L, rows, cols, 11, pool, precision=precision, keep_grads=1, ngf=ngf, ndf=ndf,
               batch=batch)
     a = oracle_arch(g.arch)
     tol = TOL[g.arch.precision]
@@ -130,7 +138,9 @@ def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
         if precision == "fp32":
             assert np.sum(~ok) <= 1, (it, worst)
         elif width >= 64:
-            assert np.all(worst < 0.075) and np.median(worst) < 0.05, (it, worst)
+            assert np.all(worst < 0.075), (it, worst)
+            if ngf == ndf:
+                assert np.median(worst) < 0.05, (it, worst)
         else:
             assert np.all(worst < 5 * tol) and np.median(worst) < 2 * tol, (it, worst)
 
