@@ -77,19 +77,22 @@ __device__ __forceinline__ bool gather_bar_or(bool pred) {
   return r != 0;
 }
 
-enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4, AK_NCHW_WIDE = 5 };
+enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4,
+       AK_NCHW_WIDE = 5 };
 
-// dynamic shared memory of a variant
+// dynamic shared memory of a variant (the compact first-layer variant: three 24 KB stages)
 constexpr int conv_smem(int ak) {
-  return ak == AK_NCHW ? 1024 + 3 * (A_BYTES + 64 * BK * 2) + 256 + 3 * PATCH_BYTES + 4 * STG_WORDS * 4
-                       : SMEM_BYTES;
+  return ak == AK_NCHW
+             ? 1024 + 3 * (A_BYTES + 64 * BK * 2) + 256 + 3 * PATCH_BYTES + 4 * STG_WORDS * 4
+             : SMEM_BYTES;
 }
 
 // AK: how the A tiles arrive (AK_CONV / AK_TRANS / AK_SCATTER: TMA through the activation map
-// for the convolution, the parity classes, the scatter mode; AK_NCHW: built from staged
-// first-layer patches; AK_GATHER: gathered channel-last rows, convolution or parity classes as
-// p.transposed says). OM: the out_mode. Each launch runs the instantiation its parameters
-// name, so that a kernel holds only its own code paths.
+// for the convolution, the parity classes, the scatter mode; AK_NCHW / AK_NCHW_WIDE: built
+// from staged first-layer patches, the former for weight tiles of at most 64 rows in a compact
+// layout that fits two CTAs per SM; AK_GATHER: gathered channel-last rows, convolution or
+// parity classes as p.transposed says). OM: the out_mode. Each launch runs the instantiation
+// its parameters name, so that a kernel holds only its own code paths.
 template <int AK, int OM>
 __global__ void __launch_bounds__(THREADS, AK == AK_NCHW ? 2 : 1)
     k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mA,
