@@ -665,7 +665,9 @@ constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_
 
 // BCHW: p.b_chw at compile time (the 3-channel channel-major B operand)
 template <bool BCHW>
-__global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constant__ WgtcParams p) {
+__global__ void __launch_bounds__(WG_THREADS, 1)
+    k_wgrad_tc(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+               const __grid_constant__ WgtcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -678,7 +680,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < WG_STAGES; ++s) {
-      mbar_init(bFull + 8 * s, 128);
+      mbar_init(bFull + 8 * s, (BCHW || !p.a_tma) ? 128 : 1);
       mbar_init(bEmpty + 8 * s, 1);
     }
     mbar_init(bAccF, 1);
@@ -710,7 +712,57 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
     k0 = (int64_t)split * p.kc;
     k1 = k0 + p.kc < Kp ? k0 + p.kc : Kp;
   };
-  if (warp == 1) {
+  const bool tma = !BCHW && p.a_tma;
+  if (warp == 0 && tma) {
+    // a_tma: both operands by TMA, MN-major rows of 64 channels: A boxes of 64 pixels from the
+    // [problem][pixel][M] map, B boxes of the chunk's 64 A pixels mapped to b's pixels (s y - p
+    // + ky, s x - p + kx) by the 5-D map's traversal stride
+    if (lane == 0) {
+      int stage = 0, issued[WG_STAGES] = {};
+      uint32_t phase = 0;
+      bool ok = true;
+      const int Wa = 1 << la, Ha = Wa;
+      for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
+        const int prob = tile / (p.splits * per_split);
+        const int split = (tile / per_split) % p.splits;
+        const int mt = (tile % per_split) / nt_n, nt = tile % nt_n;
+        int64_t k0, k1;
+        split_range(split, k0, k1);
+        for (int64_t kb = k0; kb < k1; kb += 64) {
+          if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 36)) {
+            ok = false;
+            break;
+          }
+          const uint32_t full = bFull + 8 * stage;
+          mbar_expect_tx(full, (uint32_t)STAGE_BYTES);
+          const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
+          tma_load_3d(sA, &mA, full, mt * 128, (int)kb, prob);
+          tma_load_3d(sA + 8192, &mA, full, mt * 128 + 64, (int)kb, prob);
+          const int nb = (int)(kb >> (2 * la));
+          const int ay0 = (int)((kb >> la) & (Ha - 1)), ax0 = (int)(kb & (Wa - 1));
+#pragma unroll
+          for (int atom = 0; atom < 4; ++atom) {
+            const int n0 = nt * 256 + atom * 64;
+            const int tap = n0 / p.Cb, c0 = n0 - tap * p.Cb;
+            tma_load_5d(sB + atom * 8192, &mB, full, c0, p.s * ax0 - p.p + (tap & 3),
+                        p.s * ay0 - p.p + (tap >> 2), nb, prob);
+          }
+          issued[stage]++;
+          if (++stage == WG_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        for (int st2 = 0; st2 < WG_STAGES; ++st2)
+          if (issued[st2] > 0) {
+            volatile int never = 0;
+            mbar_wait(bFull + 8 * st2, (uint32_t)((issued[st2] - 1) & 1), &never, p.err, 37);
+          }
+      }
+    }
+  } else if (warp == 1) {
     if (lane == 0) {
       int stage = 0, uses[2] = {0, 0}, jobs = 0;
       uint32_t phase = 0;
@@ -756,7 +808,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad_tc(const __grid_constan
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 33);
     }
-  } else if (warp >= 2 && warp < 6) {
+  } else if (warp >= 2 && warp < 6 && !tma) {
     // gather: thread t copies pixel row (t & 63) of A atom (t >> 6) and of B atoms 2 (t >> 6),
     // 2 (t >> 6) + 1 with 16-byte cp.async (zero fill outside the image); a stage is marked
     // full WG_LAG chunks later, once its copy group has landed
@@ -1284,10 +1336,11 @@ bool wgtc_prepare(std::string* msg) {
   return true;
 }
 
-void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st) {
+void launch_wgrad_tc(const CUtensorMap& mA, const CUtensorMap& mB, const WgtcParams& p, int sms,
+                     cudaStream_t st) {
   const int grid = p.n_tiles < sms ? p.n_tiles : sms;
   launch_pdl(p.b_chw ? ctc::k_wgrad_tc<true> : ctc::k_wgrad_tc<false>, dim3(grid),
-             dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, p);
+             dim3(ctc::WG_THREADS), ctc::WG_SMEM, st, mA, mB, p);
   if (p.b_chw)
     launch_pdl(ctc::k_wgrad_tc_reduce_chw, dim3((p.M * 48 + 255) / 256, p.n_probs), dim3(256), 0,
                st, p);
@@ -1468,6 +1521,57 @@ ConvKernel conv_kernel(const CtcParams& p) {
   return nullptr;
 }
 }  // namespace
+
+bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcDesc* descs,
+                    int n_probs, std::string* msg) {
+  q->a_tma = 0;
+  if (q->b_chw || n_probs < 1 || q->M % 64 != 0 || q->Cb % 64 != 0) return true;
+  const int64_t Wa = (int64_t)1 << q->la, Wb = (int64_t)1 << q->lb;
+  const int64_t Kp = (int64_t)q->rows * Wa * Wa;
+  const int64_t per_a = Kp * q->M, per_b = (int64_t)q->rows * Wb * Wb * q->Cb;
+  int64_t sa = per_a, sb = per_b;
+  if (n_probs > 1) {
+    sa = (int64_t)(descs[1].a - descs[0].a);
+    sb = (int64_t)(descs[1].b - descs[0].b);
+  }
+  if (sa < per_a || sb < per_b || sa % 8 != 0 || sb % 8 != 0) return true;
+  for (int k = 1; k < n_probs; ++k)
+    if (descs[k].a != descs[0].a + k * sa || descs[k].b != descs[0].b + k * sb) return true;
+  if (!ensure_encode(msg)) return false;
+  {
+    cuuint64_t dims[3] = {(cuuint64_t)q->M, (cuuint64_t)Kp, (cuuint64_t)n_probs};
+    cuuint64_t strides[2] = {(cuuint64_t)q->M * 2, (cuuint64_t)sa * 2};
+    cuuint32_t box[3] = {64, 64, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    if (g_encode_ctc(mA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<bf16*>(descs[0].a), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+      if (msg) *msg = "cuTensorMapEncodeTiled (weight-gradient A) failed";
+      return false;
+    }
+  }
+  {
+    // the 64 A pixels of a chunk: tw columns of th rows of tn images, in raster order
+    const int tw = (int)std::min<int64_t>(Wa, 64), th = (int)std::min<int64_t>(Wa, 64 / tw);
+    const int tn = std::max(1, 64 / (tw * th));
+    cuuint64_t dims[5] = {(cuuint64_t)q->Cb, (cuuint64_t)Wb, (cuuint64_t)Wb, (cuuint64_t)q->rows,
+                          (cuuint64_t)n_probs};
+    cuuint64_t strides[4] = {(cuuint64_t)q->Cb * 2, (cuuint64_t)(Wb * q->Cb * 2),
+                             (cuuint64_t)(Wb * Wb * q->Cb * 2), (cuuint64_t)sb * 2};
+    cuuint32_t box[5] = {64, (cuuint32_t)(tw * q->s), (cuuint32_t)(th * q->s), (cuuint32_t)tn, 1};
+    cuuint32_t es[5] = {1, (cuuint32_t)q->s, (cuuint32_t)q->s, 1, 1};
+    if (g_encode_ctc(mB, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<bf16*>(descs[0].b), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+      if (msg) *msg = "cuTensorMapEncodeTiled (weight-gradient B) failed";
+      return false;
+    }
+  }
+  q->a_tma = 1;
+  return true;
+}
 
 bool ctc_prepare(std::string* msg) {
   for (const ConvVariant& v : kConvVariants)

@@ -97,11 +97,18 @@ struct WgtcParams {
   int n_probs, rows, M, N, Cb, la, lb, s, p, splits, n_tiles;
   int64_t kc;
   int b_chw;  // b is 3 channel-major channels (Cb 3, N 64 with 48 used, M a multiple of 64)
+  int a_tma;  // both operands by TMA through the maps of wgtc_make_maps (set there)
   float* part;
   int* err;
 };
 bool wgtc_prepare(std::string* msg);
-void launch_wgrad_tc(const WgtcParams& p, int sms, cudaStream_t st);
+// Maps of a weight-gradient launch whose problems' a and b sit at uniform strides (not b_chw):
+// sets q->a_tma = 1 when they apply (else the gather warps load both operands); false only
+// when the driver refuses a map.
+bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcDesc* descs,
+                    int n_probs, std::string* msg);
+void launch_wgrad_tc(const CUtensorMap& mA, const CUtensorMap& mB, const WgtcParams& p, int sms,
+                     cudaStream_t st);
 
 bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t depth,
                   uint64_t depth_elems, uint32_t box_rows, std::string* msg);

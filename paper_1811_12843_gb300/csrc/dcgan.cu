@@ -141,6 +141,7 @@ struct DcPlan {
   bool wtc_d[4] = {}, wtc_g[5] = {};
   WgtcParams wdp[4], wgp[5];
   WgtcDesc *wdd[4] = {}, *wgd[5] = {};
+  CUtensorMap wdA[4], wdB[4], wgA[5], wgB[5];
   float* wpart = nullptr;
 };
 
@@ -895,9 +896,11 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         w.dw = b.gD + (int64_t)c * b.PDs + dof[l - 1];
         vw.push_back(w);
       }
+      ok = wgtc_make_maps(&p->wdA[k], &p->wdB[k], &q, vw.data(), C, msg);
+      if (gather_a) q.a_tma = 0;
       p->wdp[k] = q;
       p->wtc_d[k] = true;
-      ok = !upload(p, &p->wdd[k], vw, msg);
+      ok = ok && !upload(p, &p->wdd[k], vw, msg);
     }
     for (int l = 5; l >= 2 && ok; --l) {
       const int k = 5 - l;
@@ -923,9 +926,11 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
         w.dw = b.gG + (int64_t)c * b.PGs + go[3 * (l - 1)];
         vw.push_back(w);
       }
+      ok = wgtc_make_maps(&p->wgA[k], &p->wgB[k], &q, vw.data(), C, msg);
+      if (gather_a) q.a_tma = 0;
       p->wgp[k] = q;
       p->wtc_g[k] = true;
-      ok = !upload(p, &p->wgd[k], vw, msg);
+      ok = ok && !upload(p, &p->wgd[k], vw, msg);
     }
     ok = ok && !dev_alloc(p, &p->wpart, (size_t)wneed * 4, msg);
   }
@@ -1156,7 +1161,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       WgtcParams q = p->wdp[k];
       q.descs = p->wdd[k];
       q.part = p->wpart;
-      launch_wgrad_tc(q, p->sms, st);
+      launch_wgrad_tc(p->wdA[k], p->wdB[k], q, p->sms, st);
     } else {
       launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->dw[k], C, dc[l], dc[l - 1] * 16,
                   nullptr, p->splits_dw[k], p->part, p->pstride_dw[k], s.slope, st);
@@ -1200,7 +1205,7 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       WgtcParams q = p->wgp[k];
       q.descs = p->wgd[k];
       q.part = p->wpart;
-      launch_wgrad_tc(q, p->sms, st);
+      launch_wgrad_tc(p->wgA[k], p->wgB[k], q, p->sms, st);
     } else {
       launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
                   nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
