@@ -660,7 +660,11 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW ? 2 : 1)
 // 256); fp32 partial sums per split go to part[problem][split][M][N] in (tap, c) order.
 constexpr int WG_THREADS = 320;  // warp 1 MMA, warps 2-5 gather, warps 6-9 epilogue
 constexpr int WG_STAGES = 4;
-constexpr int WG_SMEM = 1024 + WG_STAGES * STAGE_BYTES + 256 + 4 * STG_WORDS * 4;
+// the 3-channel B operand's input patches: 3 channels x 6 rows x 72 columns (64 interior at
+// column 4), three buffers
+constexpr int WG_PATCH_BYTES = 2688;
+constexpr int WG_SMEM =
+    1024 + WG_STAGES * STAGE_BYTES + 256 + 4 * STG_WORDS * 4 + 3 * WG_PATCH_BYTES;
 constexpr int WG_LAG = 2;  // copy groups a gather thread keeps in flight (< WG_STAGES)
 
 // BCHW: p.b_chw at compile time (the 3-channel channel-major B operand)
@@ -680,7 +684,9 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < WG_STAGES; ++s) {
-      mbar_init(bFull + 8 * s, (BCHW || !p.a_tma) ? 128 : 1);
+      // a_tma: the producer's expect-tx arrival (+ the 128 gather threads that build the
+      // 3-channel B operand)
+      mbar_init(bFull + 8 * s, !p.a_tma ? 128 : (BCHW ? 129 : 1));
       mbar_init(bEmpty + 8 * s, 1);
     }
     mbar_init(bAccF, 1);
@@ -712,7 +718,7 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
     k0 = (int64_t)split * p.kc;
     k1 = k0 + p.kc < Kp ? k0 + p.kc : Kp;
   };
-  const bool tma = !BCHW && p.a_tma;
+  const bool tma = p.a_tma;
   if (warp == 0 && tma) {
     // a_tma: both operands by TMA, MN-major rows of 64 channels: A boxes of 64 pixels from the
     // [problem][pixel][M] map, B boxes of the chunk's 64 A pixels mapped to b's pixels (s y - p
@@ -734,10 +740,18 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
             break;
           }
           const uint32_t full = bFull + 8 * stage;
-          mbar_expect_tx(full, (uint32_t)STAGE_BYTES);
+          mbar_expect_tx(full, (uint32_t)(BCHW ? A_BYTES : STAGE_BYTES));
           const uint32_t sA = base + stage * STAGE_BYTES, sB = sA + A_BYTES;
           tma_load_3d(sA, &mA, full, mt * 128, (int)kb, prob);
           tma_load_3d(sA + 8192, &mA, full, mt * 128 + 64, (int)kb, prob);
+          if constexpr (BCHW) {
+            issued[stage]++;
+            if (++stage == WG_STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+            continue;
+          }
           const int nb = (int)(kb >> (2 * la));
           const int ay0 = (int)((kb >> la) & (Ha - 1)), ax0 = (int)(kb & (Wa - 1));
 #pragma unroll
@@ -808,6 +822,101 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 33);
     }
+  } else if (warp >= 2 && warp < 6 && tma && BCHW) {
+    // the 3-channel B operand with A by TMA: a chunk's 64 A pixels are two rows of the 32-wide
+    // A image (first-layer geometry: b is 3 x 64 x 64, s = 2, p = 1), fed by a 3 x 6 x 64
+    // patch of b that the threads copy one chunk ahead by 8-byte cp.async into one of three
+    // buffers (halo columns zero); thread t builds 16-byte units 4 (t >> 6) .. + 3 of row t & 63
+    const int t = threadIdx.x - 64;
+    const int row = t & 63, half = t >> 6;
+    const uint32_t sw = (uint32_t)(row & 7);
+    uint8_t* patches = misc + 256 + 4 * STG_WORDS * 4;
+    const uint32_t patch0 = smem_u32(patches);
+    for (int i = t; i < 3 * WG_PATCH_BYTES / 16; i += 128)
+      *reinterpret_cast<uint4*>(patches + 16 * i) = make_uint4(0u, 0u, 0u, 0u);
+    gather_bar_or(false);
+    // the chunks this CTA builds, in order: (tile, kb) over its tiles and their splits' chunks
+    // (every split holds at least one); the patch prefetch runs one chunk ahead
+    struct Chunk {
+      int tile;
+      int64_t kb, k1;
+    };
+    auto start = [&](Chunk& c, int tile_x) {
+      c.tile = tile_x;
+      if (tile_x < p.n_tiles) {
+        int64_t k0;
+        split_range((tile_x / per_split) % p.splits, k0, c.k1);
+        c.kb = k0;
+      }
+    };
+    auto advance = [&](Chunk& c) {
+      c.kb += 64;
+      if (c.kb >= c.k1) start(c, c.tile + gridDim.x);
+    };
+    auto prefetch = [&](int tile_x, int64_t kb_x, int buf) {
+      if (tile_x < p.n_tiles) {
+        const WgtcDesc dx = p.descs[tile_x / (p.splits * per_split)];
+        const int nb = (int)(kb_x >> 10), ay0 = (int)((kb_x >> 5) & 31);
+        for (int u = t; u < 288; u += 128) {  // 3 channels x 6 rows x 16 pieces of 4
+          const int c = u / 96, rem = u - c * 96, pr = rem >> 4, qq = rem & 15;
+          const int iy = 2 * ay0 - 1 + pr;
+          const bool in = iy >= 0 && iy < 64;
+          const bf16* src = in ? dx.b + ((int64_t)(nb * 3 + c) << 12) + (iy << 6) + 4 * qq : dx.b;
+          cp_async8(patch0 + (uint32_t)(buf * WG_PATCH_BYTES + ((c * 6 + pr) * 72 + 4 + 4 * qq) * 2),
+                    src, in ? 8 : 0);
+        }
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    Chunk cur, nxt;
+    start(cur, blockIdx.x);
+    nxt = cur;
+    prefetch(cur.tile, cur.kb, 0);
+    int buf = 0, stage = 0;
+    uint32_t phase = 0;
+    while (cur.tile < p.n_tiles) {
+      advance(nxt);
+      prefetch(nxt.tile, nxt.kb, buf == 2 ? 0 : buf + 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+      const bool okw = mbar_wait_warp(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 38);
+      if (gather_bar_or(!okw)) break;
+      const bool qv = cur.kb + row < cur.k1;
+      const int ayl = row >> 5, ax = row & 31;
+      const unsigned short* pb = reinterpret_cast<const unsigned short*>(patches + buf * WG_PATCH_BYTES);
+      const uint32_t sB = base + stage * STAGE_BYTES + A_BYTES;
+#pragma unroll
+      for (int uu = 0; uu < 4; ++uu) {
+        const int u = half * 4 + uu;
+        uint32_t w[4];
+#pragma unroll
+        for (int e2 = 0; e2 < 4; ++e2) {
+          uint32_t hv[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int k = u * 8 + e2 * 2 + h;  // k = tap * 3 + c
+            hv[h] = 0u;
+            if (k < 48 && qv) {
+              const int tap = k / 3, c = k - 3 * tap;
+              hv[h] = pb[(c * 6 + 2 * ayl + (tap >> 2)) * 72 + 2 * ax + (tap & 3) + 3];
+            }
+          }
+          w[e2] = hv[0] | (hv[1] << 16);
+        }
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                         sB + (uint32_t)row * 128u + (((uint32_t)u ^ sw) << 4)),
+                     "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                     : "memory");
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(bFull + 8 * stage);
+      if (++stage == WG_STAGES) {
+        stage = 0;
+        phase ^= 1u;
+      }
+      buf = buf == 2 ? 0 : buf + 1;
+      cur = nxt;
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
   } else if (warp >= 2 && warp < 6 && !tma) {
     // gather: thread t copies pixel row (t & 63) of A atom (t >> 6) and of B atoms 2 (t >> 6),
     // 2 (t >> 6) + 1 with 16-byte cp.async (zero fill outside the image); a stage is marked
@@ -1525,7 +1634,10 @@ ConvKernel conv_kernel(const CtcParams& p) {
 bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcDesc* descs,
                     int n_probs, std::string* msg) {
   q->a_tma = 0;
-  if (q->b_chw || n_probs < 1 || q->M % 64 != 0 || q->Cb % 64 != 0) return true;
+  if (n_probs < 1 || q->M % 64 != 0) return true;
+  // b_chw: A by TMA only, B built from staged patches (first-layer geometry only)
+  if (q->b_chw && (q->la != 5 || q->lb != 6 || q->s != 2 || q->p != 1)) return true;
+  if (!q->b_chw && q->Cb % 64 != 0) return true;
   const int64_t Wa = (int64_t)1 << q->la, Wb = (int64_t)1 << q->lb;
   const int64_t Kp = (int64_t)q->rows * Wa * Wa;
   const int64_t per_a = Kp * q->M, per_b = (int64_t)q->rows * Wb * Wb * q->Cb;
@@ -1534,9 +1646,11 @@ bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcD
     sa = (int64_t)(descs[1].a - descs[0].a);
     sb = (int64_t)(descs[1].b - descs[0].b);
   }
+  if (q->b_chw) sb = per_b;  // b is read through the descriptors
   if (sa < per_a || sb < per_b || sa % 8 != 0 || sb % 8 != 0) return true;
   for (int k = 1; k < n_probs; ++k)
-    if (descs[k].a != descs[0].a + k * sa || descs[k].b != descs[0].b + k * sb) return true;
+    if (descs[k].a != descs[0].a + k * sa || (!q->b_chw && descs[k].b != descs[0].b + k * sb))
+      return true;
   if (!ensure_encode(msg)) return false;
   {
     cuuint64_t dims[3] = {(cuuint64_t)q->M, (cuuint64_t)Kp, (cuuint64_t)n_probs};
@@ -1551,7 +1665,7 @@ bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcD
       return false;
     }
   }
-  {
+  if (!q->b_chw) {
     // the 64 A pixels of a chunk: tw columns of th rows of tn images, in raster order
     const int tw = (int)std::min<int64_t>(Wa, 64), th = (int)std::min<int64_t>(Wa, 64 / tw);
     const int tn = std::max(1, 64 / (tw * th));

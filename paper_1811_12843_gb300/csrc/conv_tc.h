@@ -97,14 +97,15 @@ struct WgtcParams {
   int n_probs, rows, M, N, Cb, la, lb, s, p, splits, n_tiles;
   int64_t kc;
   int b_chw;  // b is 3 channel-major channels (Cb 3, N 64 with 48 used, M a multiple of 64)
-  int a_tma;  // both operands by TMA through the maps of wgtc_make_maps (set there)
+  int a_tma;  // operands by TMA through the maps of wgtc_make_maps (set there; with b_chw A only)
   float* part;
   int* err;
 };
 bool wgtc_prepare(std::string* msg);
-// Maps of a weight-gradient launch whose problems' a and b sit at uniform strides (not b_chw):
-// sets q->a_tma = 1 when they apply (else the gather warps load both operands); false only
-// when the driver refuses a map.
+// Maps of a weight-gradient launch whose problems' a (and, without b_chw, b) sit at uniform
+// strides: sets q->a_tma = 1 when they apply (else the gather warps load both operands; with
+// b_chw, a_tma loads A by TMA and builds B from staged patches, for 32 x 32 A images over
+// 64 x 64 b images only); false only when the driver refuses a map.
 bool wgtc_make_maps(CUtensorMap* mA, CUtensorMap* mB, WgtcParams* q, const WgtcDesc* descs,
                     int n_probs, std::string* msg);
 void launch_wgrad_tc(const CUtensorMap& mA, const CUtensorMap& mB, const WgtcParams& p, int sms,
