@@ -67,7 +67,7 @@ TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM *
                            + 2 * BWD_ACT)
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels, from
-# the ncu launch list in profiles/launches_12x12_bf16_iteration.md (same kernels as this build).
+# an ncu launch list (dram__bytes_read.sum + dram__bytes_write.sum) of these same kernels.
 PHASE_TRAFFIC = {"batch": 21.2e6, "g_fwd": 161.4e6, "d_fwd": 226.9e6, "fitness": 1.8e6,
                  "select": 0.0, "train_fwd": 129.0e6, "train_bwd": 2182.6e6, "adam": 3.6e6}
 

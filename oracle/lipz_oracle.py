@@ -16,7 +16,7 @@ Training", steps 1-3 and 5) and its settings table (Table 1), written as plain n
   3. size-2 tournament selection in each neighbourhood, then one gradient (Adam) update of the
      selected pair, with optional Gaussian mutation of the learning rate (step 3, Table 1).
 
-Readings where the paper is silent (each is listed in the design doc with its reason):
+Readings where the paper is silent (each with its reason in the design notes):
   * fitness is a loss for both populations, lower is better: f_G = mean_j L_G, f_D = mean_i L_D;
   * L_D is the SUM of the real-batch and fake-batch BCE means; L_G is the non-saturating loss;
   * iterations run on a synchronous snapshot of all centres; with ``stale_neighbors`` (the
