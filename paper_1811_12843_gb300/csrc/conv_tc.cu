@@ -78,13 +78,16 @@ __device__ __forceinline__ bool gather_bar_or(bool pred) {
 }
 
 enum { AK_CONV = 0, AK_TRANS = 1, AK_SCATTER = 2, AK_NCHW = 3, AK_GATHER = 4,
-       AK_NCHW_WIDE = 5 };
+       AK_NCHW_WIDE = 5, AK_TRANS_C = 6 };
 
-// dynamic shared memory of a variant (the compact first-layer variant: three 24 KB stages)
+// dynamic shared memory of a variant: the compact first layer (three 24 KB stages) and the
+// compact parity classes (256-row tiles of weight tiles of at most 64 rows: two 40 KB stages,
+// no patch buffers) fit two CTAs per SM
 constexpr int conv_smem(int ak) {
   return ak == AK_NCHW
              ? 1024 + 3 * (A_BYTES + 64 * BK * 2) + 256 + 3 * PATCH_BYTES + 4 * STG_WORDS * 4
-             : SMEM_BYTES;
+         : ak == AK_TRANS_C ? 1024 + 2 * (2 * A_BYTES + 64 * BK * 2) + 256 + 4 * STG_WORDS * 4
+                            : SMEM_BYTES;
 }
 
 // AK: how the A tiles arrive (AK_CONV / AK_TRANS / AK_SCATTER: TMA through the activation map
@@ -94,19 +97,23 @@ constexpr int conv_smem(int ak) {
 // parity classes as p.transposed says). OM: the out_mode. Each launch runs the instantiation
 // its parameters name, so that a kernel holds only its own code paths.
 template <int AK, int OM>
-__global__ void __launch_bounds__(THREADS, AK == AK_NCHW ? 2 : 1)
+__global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2 : 1)
     k_conv_tc(const __grid_constant__ CUtensorMap mW, const __grid_constant__ CUtensorMap mA,
               const __grid_constant__ CtcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  constexpr bool kTma = AK == AK_CONV || AK == AK_TRANS || AK == AK_SCATTER;
+  constexpr bool kTma = AK == AK_CONV || AK == AK_TRANS || AK == AK_SCATTER || AK == AK_TRANS_C;
   constexpr bool kScatter = AK == AK_SCATTER, kNchw = AK == AK_NCHW || AK == AK_NCHW_WIDE;
   // AK_NCHW (weight tiles of at most 64 rows): three 24 KB stages and 256 TMEM columns, so
   // that two CTAs share an SM
-  constexpr bool kCompact = AK == AK_NCHW;
-  constexpr int STAGES = kCompact ? 3 : ctc::STAGES;
-  constexpr uint32_t STAGE_BYTES = kCompact ? A_BYTES + 64 * BK * 2 : ctc::STAGE_BYTES;
+  constexpr bool kCompact = AK == AK_NCHW || AK == AK_TRANS_C;
+  constexpr int STAGES = AK == AK_NCHW ? 3 : AK == AK_TRANS_C ? 2 : ctc::STAGES;
+  constexpr uint32_t STAGE_BYTES = AK == AK_NCHW     ? A_BYTES + 64 * BK * 2
+                                   : AK == AK_TRANS_C ? 2 * A_BYTES + 64 * BK * 2
+                                                      : ctc::STAGE_BYTES;
+  // the first layer's patch buffers sit between the barriers and the epilogue staging
+  constexpr int kPatchArea = AK == AK_TRANS_C ? 0 : 3 * PATCH_BYTES;
   constexpr uint32_t kTmemCols = kCompact ? 256 : 512, kAccStride = kCompact ? 128 : 256;
-  const bool transposed = AK == AK_TRANS || (AK == AK_GATHER && p.transposed);
+  const bool transposed = AK == AK_TRANS || AK == AK_TRANS_C || (AK == AK_GATHER && p.transposed);
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
@@ -423,7 +430,7 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW ? 2 : 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-    uint32_t* stg = reinterpret_cast<uint32_t*>(misc + 256 + 3 * PATCH_BYTES) + (warp - 6) * STG_WORDS;
+    uint32_t* stg = reinterpret_cast<uint32_t*>(misc + 256 + kPatchArea) + (warp - 6) * STG_WORDS;
     int uses[2] = {0, 0}, jobs = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
@@ -1602,6 +1609,8 @@ const ConvVariant kConvVariants[] = {
     {ctc::AK_TRANS, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_TRANS, CTC_TANH_CHW>},
     {ctc::AK_TRANS, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_TRANS, CTC_DLRELU_HWC>},
     {ctc::AK_TRANS, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_TRANS, CTC_DTANH_CHW>},
+    {ctc::AK_TRANS_C, CTC_F32_HWC, ctc::k_conv_tc<ctc::AK_TRANS_C, CTC_F32_HWC>},
+    {ctc::AK_TRANS_C, CTC_DLRELU_HWC, ctc::k_conv_tc<ctc::AK_TRANS_C, CTC_DLRELU_HWC>},
     {ctc::AK_SCATTER, CTC_TANH_CHW, ctc::k_conv_tc<ctc::AK_SCATTER, CTC_TANH_CHW>},
     {ctc::AK_SCATTER, CTC_DTANH_CHW, ctc::k_conv_tc<ctc::AK_SCATTER, CTC_DTANH_CHW>},
     {ctc::AK_NCHW, CTC_LRELU_HWC, ctc::k_conv_tc<ctc::AK_NCHW, CTC_LRELU_HWC>},
@@ -1619,7 +1628,8 @@ const ConvVariant kConvVariants[] = {
 int conv_ak(const CtcParams& p) {
   return p.scatter   ? ctc::AK_SCATTER
          : p.nchw_in ? (p.nbox <= 64 ? ctc::AK_NCHW : ctc::AK_NCHW_WIDE)
-         : p.a_tma   ? (p.transposed ? ctc::AK_TRANS : ctc::AK_CONV)
+         : p.a_tma   ? (p.transposed ? (p.m2 && p.nbox <= 64 ? ctc::AK_TRANS_C : ctc::AK_TRANS)
+                                     : ctc::AK_CONV)
                      : ctc::AK_GATHER;
 }
 
@@ -1703,7 +1713,8 @@ bool launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParam
   const ConvKernel k = conv_kernel(p);
   if (!k) return false;
   const int ak = conv_ak(p);
-  const int ctas = ak == ctc::AK_NCHW ? 2 * sms : sms;  // the compact variant: two per SM
+  // the compact variants: two CTAs per SM
+  const int ctas = ak == ctc::AK_NCHW || ak == ctc::AK_TRANS_C ? 2 * sms : sms;
   const int grid = p.n_tiles < ctas ? p.n_tiles : ctas;
   launch_pdl(k, dim3(grid), dim3(ctc::THREADS), ctc::conv_smem(ak), st, mW, mA, p);
   return true;
