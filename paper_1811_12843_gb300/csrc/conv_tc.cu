@@ -450,7 +450,8 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
       float dot = 0.f;
       const bf16* w5 = nullptr;
       if constexpr (OM == CTC_LRELU_LOGIT)
-        w5 = p.logit_w + (int64_t)__ldg(&p.wsel[d.wsel_idx]) * p.logit_ws + (int64_t)(m & 15) * p.co;
+        w5 = p.logit_w + (int64_t)__ldg(&p.wsel[d.wsel_idx]) * p.logit_ws +
+             (int64_t)(m & 15) * p.co;
       for (int j = 0; j < p.nj && ok; ++j, ++jobs) {
         const int R = jobs & 1;
         // the scatter epilogue synchronises the four warps: they leave together
@@ -869,7 +870,8 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
           const int iy = 2 * ay0 - 1 + pr;
           const bool in = iy >= 0 && iy < 64;
           const bf16* src = in ? dx.b + ((int64_t)(nb * 3 + c) << 12) + (iy << 6) + 4 * qq : dx.b;
-          cp_async8(patch0 + (uint32_t)(buf * WG_PATCH_BYTES + ((c * 6 + pr) * 72 + 4 + 4 * qq) * 2),
+          cp_async8(patch0 +
+                        (uint32_t)(buf * WG_PATCH_BYTES + ((c * 6 + pr) * 72 + 4 + 4 * qq) * 2),
                     src, in ? 8 : 0);
         }
       }
@@ -889,7 +891,8 @@ __global__ void __launch_bounds__(WG_THREADS, 1)
       if (gather_bar_or(!okw)) break;
       const bool qv = cur.kb + row < cur.k1;
       const int ayl = row >> 5, ax = row & 31;
-      const unsigned short* pb = reinterpret_cast<const unsigned short*>(patches + buf * WG_PATCH_BYTES);
+      const unsigned short* pb =
+          reinterpret_cast<const unsigned short*>(patches + buf * WG_PATCH_BYTES);
       const uint32_t sB = base + stage * STAGE_BYTES + A_BYTES;
 #pragma unroll
       for (int uu = 0; uu < 4; ++uu) {
@@ -1213,7 +1216,8 @@ __global__ void __launch_bounds__(256) k_relayout_g(const bf16* __restrict__ src
     for (int e = threadIdx.x; e < n * 16; e += 256) {
       const int ct = e / n, cc = e - ct * n;  // (class, tap) = ct
       const int cls = ct >> 2, t = ct & 3;
-      const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1), kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
+      const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1);
+      const int kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
       dp[(((int64_t)cls * r.cls_rows[l] + o) * 4 + t) * ci + cb + cc] = sh[ky * 4 + kx][cc];
     }
     __syncthreads();
@@ -1543,7 +1547,8 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
                             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
-    if (msg) *msg = "cuTensorMapEncodeTiled (convolution weights) failed: " + std::to_string((int)r);
+    if (msg)
+      *msg = "cuTensorMapEncodeTiled (convolution weights) failed: " + std::to_string((int)r);
     return false;
   }
   return true;
@@ -1577,7 +1582,9 @@ bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int
                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
-    if (msg) *msg = "cuTensorMapEncodeTiled (convolution activations) failed: " + std::to_string((int)r);
+    if (msg)
+      *msg = "cuTensorMapEncodeTiled (convolution activations) failed: " +
+             std::to_string((int)r);
     return false;
   }
   q->a_tma = 1;

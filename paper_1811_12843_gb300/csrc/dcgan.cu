@@ -327,7 +327,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     v.clear();
     for (int c = 0; c < C; ++c)
       for (int sl = 0; sl < 5; ++sl) {
-        void* bufs[2] = {elw(ex, (int64_t)sl * 6 * B * dmax), elw(ey, (int64_t)sl * 6 * B * dsz[2])};
+        void* bufs[2] = {elw(ex, (int64_t)sl * 6 * B * dmax),
+                         elw(ey, (int64_t)sl * 6 * B * dsz[2])};
         const void* in = l == 1 ? el(b.E, (int64_t)c * b.e_cell) : bufs[l % 2];
         void* out = bufs[(l + 1) % 2];
         ConvDesc q = cdesc(in, 6 * B, dc[l - 1], ds[l - 1], Wd(l), dc[l], ds[l], 2, 1, out);
@@ -358,7 +359,9 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
   // [B, 2B); the selected discriminator on TX (real rows copied in at run time)
   auto tgc = [&](int c, int l) { return tc + ((int64_t)c * B) * gall + (int64_t)B * goffs[l]; };
   auto tgh = [&](int c, int l) { return elw(th, (int64_t)c * B * gall + (int64_t)B * goffs[l]); };
-  auto tda = [&](int c, int l) { return elw(ta, (int64_t)c * 2 * B * dall + (int64_t)2 * B * doffs[l]); };
+  auto tda = [&](int c, int l) {
+    return elw(ta, (int64_t)c * 2 * B * dall + (int64_t)2 * B * doffs[l]);
+  };
   auto tx = [&](int c) { return elw(p->TX, (int64_t)c * 2 * B * X); };
   for (int l = 1; l <= 5; ++l) {
     v.clear();
@@ -463,7 +466,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     for (int c = 0; c < C; ++c) {
       void* dout = elw((l % 2 == 0) ? P2 : Q2, (int64_t)c * B * dmax);
       const bool last = l == 1;
-      void* din = last ? elw(d5, (int64_t)c * B * X) : elw((l % 2 == 0) ? Q2 : P2, (int64_t)c * B * dmax);
+      void* din = last ? elw(d5, (int64_t)c * B * X)
+                       : elw((l % 2 == 0) ? Q2 : P2, (int64_t)c * B * dmax);
       ConvDesc q = cdesc(dout, B, dc[l], ds[l], Wd(l), dc[l - 1], ds[l - 1], 2, 1, din);
       q.wsel = b.src_d;
       q.wsel_stride = b.PDs;
