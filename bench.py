@@ -609,7 +609,7 @@ def main():
     ap.add_argument("--stale-neighbors", action="store_true",
                     help="neighbours seen one iteration late (asynchronous cells)")
     ap.add_argument("--dcgan", action="store_true",
-                    help="the 3x3 DCGAN workload (CUDA-core convolutions) instead of the MLP")
+                    help="the 3x3 DCGAN workload (tensor-core convolutions) instead of the MLP")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

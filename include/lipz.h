@@ -53,7 +53,7 @@ enum {
   LIPZ_ERR_CUDA = 2,      /* a CUDA runtime/driver call failed; see lipz_last_error */
   LIPZ_ERR_OOM = 3,       /* device or pinned allocation failed */
   LIPZ_ERR_NONFINITE = 4, /* a loss or fitness came out NaN/Inf (first such cell in the message) */
-  LIPZ_ERR_TIMEOUT = 5,   /* reserved for bounded device-side waits */
+  LIPZ_ERR_TIMEOUT = 5,   /* a bounded device-side wait expired (the kernel stopped early) */
   LIPZ_ERR_STATE = 6      /* call out of order (e.g. train before select) */
 };
 
@@ -127,7 +127,9 @@ typedef struct lipz_arch {
   int32_t ndf;             /* D: 3 x 64 x 64 -> Conv 4x4 /2 -> ndf x 32 x 32 -> 2ndf x 16 x 16 ->
                               4ndf x 8 x 8 -> 8ndf x 4 x 4 (each LeakyReLU) -> Conv 4x4 -> logit;
                               weights [out][in][4][4], no biases. Needs x_dim == 12288 (CHW
-                              images), train_steps == 1; runs on the CUDA-core kernels. Layout
+                              images), train_steps == 1. bf16 with ngf, ndf multiples of 64 runs
+                              the convolutions on the tensor cores; fp32 and other widths on
+                              the CUDA-core kernels. Layout
                               per generator: W1, gamma1, beta1, ..., W4, gamma4, beta4, W5;
                               initial weights N(0, 0.02^2), scales 1 + N(0, 0.02^2), shifts 0.
                               Default 64 (the 512/256/128/64 configuration). */
@@ -274,21 +276,24 @@ LIPZ_API int lipz_profile_read(lipz_grid* g, double* ms, int64_t* count, int64_t
 /*
  * Fitness of every cell from logits already in device memory, allocating nothing.
  * Not part of the method: the paper has no counterpart. It is for callers that cannot call
- * cudaMalloc when they need the fitness: code running while a CUDA graph is being captured
- * (allocation calls are not allowed there), a serving loop whose device memory is fully
- * reserved by another allocator (a new allocation would fail), or a latency-critical path
- * that cannot afford the implicit synchronisation of cudaMalloc / cudaFree. The per-pair
- * losses that the computation needs go to one file-scope device array of about 800 KB, which
- * every GPU that loads this library holds until the process exits.
+ * cudaMalloc when they need the fitness: a serving loop whose device memory is fully reserved
+ * by another allocator (a new allocation would fail), or a latency-critical path that cannot
+ * afford the implicit synchronisation of cudaMalloc / cudaFree. The per-pair losses that the
+ * computation needs go to one file-scope device array of about 800 KB, which every GPU that
+ * loads this library holds until the process exits.
  *   logits: device, [cells][5 (j)][6 * batch] fp32, laid out as lipz_get_logits returns it;
  *   fit_g, fit_d: device outputs [cells][5] fp32 (as lipz_eval_neighborhoods computes them);
  *   stream: the cudaStream_t to run on (0 = legacy default). The call is asynchronous.
+ * The library cannot check device buffers: they must hold the sizes above.
  * Limits: 1 <= cells <= LIPZ_NOALLOC_MAX_CELLS and batch >= 1, else LIPZ_ERR_INVALID with
  * nothing launched; a null pointer also gives LIPZ_ERR_INVALID. LIPZ_ERR_CUDA if a CUDA call
  * fails. The first call on a device looks up the array's device address (once per device,
- * with that device current): make that first call before any stream capture. All calls share
- * the array, and each call overwrites what it uses, so two calls whose work overlaps on the
- * GPU (different streams, no ordering) race. Non-finite losses show up as NaN/Inf fitness.
+ * with that device current) and keeps it for the life of the process: make that first call
+ * before any stream capture, and do not use the call across a cudaDeviceReset (the array
+ * moves with the device's primary context). All calls share the array, and each call
+ * overwrites what it uses, so two calls whose work overlaps on the GPU (different streams,
+ * no ordering) race. Non-finite losses are reported only through NaN/Inf fitness values
+ * (lipz_eval_neighborhoods returns LIPZ_ERR_NONFINITE for them; this call has no channel).
  */
 #define LIPZ_NOALLOC_MAX_CELLS 4096
 LIPZ_API int lipz_fitness_from_logits_noalloc(const float* logits, int32_t cells, int32_t batch,

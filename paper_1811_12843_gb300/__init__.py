@@ -29,6 +29,7 @@ LIPZ_ERR_NONFINITE, LIPZ_ERR_TIMEOUT, LIPZ_ERR_STATE = 4, 5, 6
 LIPZ_MLP, LIPZ_DCGAN64 = 0, 1
 LIPZ_FP32, LIPZ_BF16 = 0, 1
 LIPZ_REPLACE_IF_BETTER, LIPZ_REPLACE_ALWAYS = 0, 1
+LIPZ_NOALLOC_MAX_CELLS = 4096
 
 
 def library_path() -> str:
@@ -239,14 +240,39 @@ def lipz_profile_read(g):
     return {p: (float(ms[i]), int(cnt[i]), int(la[i])) for i, p in enumerate(PHASES)}
 
 
+def _device_f32(t, need, what):
+    """Refuse anything but a contiguous float32 CUDA tensor of at least `need` elements: the
+    library launches a kernel on these addresses and cannot check them itself."""
+    ok = (hasattr(t, "is_cuda") and t.is_cuda and str(getattr(t, "dtype", "")) == "torch.float32"
+          and t.is_contiguous())
+    if not ok:
+        raise LipzError(LIPZ_ERR_INVALID, "lipz_fitness_from_logits_noalloc: %s must be a "
+                        "contiguous float32 CUDA tensor" % what)
+    if t.numel() < need:
+        raise LipzError(LIPZ_ERR_INVALID, "lipz_fitness_from_logits_noalloc: %s holds %d "
+                        "elements, %d needed" % (what, t.numel(), need))
+
+
 def lipz_fitness_from_logits_noalloc(logits, cells, batch, fit_g, fit_d, stream=0):
     """Fitness from device logits with no device allocation (all buffers are device tensors
-    the caller owns). Raises LipzError with the status code on failure."""
+    the caller owns). Raises LipzError with the status code on failure; buffers that are not
+    contiguous float32 CUDA tensors of the needed sizes are refused before the library is
+    called."""
+    cells, batch = int(cells), int(batch)
+    # sizes outside the library's limits go through unchecked: the library refuses them itself,
+    # launching nothing
+    if 1 <= cells <= LIPZ_NOALLOC_MAX_CELLS and batch >= 1:
+        _device_f32(logits, cells * 30 * batch, "logits")
+        _device_f32(fit_g, cells * 5, "fit_g")
+        _device_f32(fit_d, cells * 5, "fit_d")
     s = stream if isinstance(stream, int) else getattr(stream, "cuda_stream", stream)
     rc = load().lipz_fitness_from_logits_noalloc(_ptr(logits), int(cells), int(batch),
                                                  _ptr(fit_g), _ptr(fit_d), _P(int(s or 0)))
     if rc != LIPZ_OK:
-        raise LipzError(rc, "lipz_fitness_from_logits_noalloc: " + lipz_status_string(rc))
+        msg = lipz_status_string(rc)
+        if rc == LIPZ_ERR_INVALID:
+            msg += " (cells must be in 1..%d, batch >= 1)" % LIPZ_NOALLOC_MAX_CELLS
+        raise LipzError(rc, "lipz_fitness_from_logits_noalloc: " + msg)
     return rc
 
 

@@ -2,7 +2,9 @@
 //
 // The fitness kernel needs the per-pair losses L_G, L_D of every cell as intermediate storage.
 // Here that storage is one file-scope __device__ array, so a call allocates nothing: it is for
-// callers that cannot call cudaMalloc at the time they need the fitness (see lipz.h).
+// callers that cannot call cudaMalloc at the time they need the fitness (a serving loop whose
+// device memory another allocator has fully reserved, or a latency-critical path that cannot
+// take the implicit synchronisation of cudaMalloc / cudaFree).
 #include <cstring>
 #include <mutex>
 
@@ -21,8 +23,11 @@ static __device__ __align__(256) float g_scratch[2 * 25 * kMaxCells + 64];
 std::mutex g_mu;
 float* g_scratch_addr[kMaxDevices] = {};
 
-// Device address of g_scratch on the current device, looked up once per device. The host
-// symbol g_scratch is only a stand-in for the device array and must not reach a kernel.
+// Device address of g_scratch on the current device, looked up once per device (with that
+// device current) and kept for the life of the process: the array moves if the device's
+// primary context is torn down (cudaDeviceReset), so the call must not be used across one.
+// The host symbol g_scratch is only a stand-in for the device array and must not reach a
+// kernel.
 cudaError_t scratch_address(float** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -60,6 +65,9 @@ extern "C" LIPZ_API int lipz_fitness_from_logits_noalloc(const float* logits, in
     cudaGetLastError();
     return LIPZ_ERR_CUDA;
   }
+  // clear an error left by an unrelated earlier call, so that the check after the launch
+  // reports this launch only
+  cudaGetLastError();
   lipz::launch_fitness(logits, cells, batch, LG, LD, fit_g, fit_d, flag, st);
   if (cudaGetLastError() != cudaSuccess) return LIPZ_ERR_CUDA;
   return LIPZ_OK;

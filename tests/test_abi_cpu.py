@@ -81,3 +81,51 @@ def test_create_rejects_bad_arguments_without_a_device(lib):
 def test_param_counts_match_the_paper_sizes():
     import paper_1811_12843_gb300 as L
     assert L.param_counts(64, 256, 784) == (283920, 267009)
+
+
+def test_noalloc_wrapper_refuses_bad_buffers_before_the_library(lib):
+    """The allocation-free fitness call launches a kernel on the addresses it is given, and the
+    library cannot check them: the wrapper refuses host arrays, wrong dtypes, non-contiguous
+    and short tensors with LIPZ_ERR_INVALID. No device exists here, so a refusal that reached
+    the library would fail differently."""
+    import numpy as np
+    import torch
+    import paper_1811_12843_gb300 as L
+    cells, batch = 2, 3
+    host = np.zeros(cells * 30 * batch, np.float32)
+    out = np.zeros(cells * 5, np.float32)
+    cases = [
+        (host, out, out, "logits"),                                      # numpy, not a device tensor
+        (torch.zeros(cells * 30 * batch), out, out, "logits"),           # CPU tensor
+    ]
+    for logits, fg, fd, what in cases:
+        with pytest.raises(L.LipzError) as e:
+            L.lipz_fitness_from_logits_noalloc(logits, cells, batch, fg, fd)
+        assert e.value.code == L.LIPZ_ERR_INVALID and what in str(e.value)
+
+    class FakeCuda:
+        """Stands in for a CUDA tensor (no device here): only the attributes the check reads."""
+
+        def __init__(self, n, dtype="torch.float32", contiguous=True):
+            self.is_cuda, self.dtype, self._n, self._c = True, dtype, n, contiguous
+
+        def is_contiguous(self):
+            return self._c
+
+        def numel(self):
+            return self._n
+
+        def data_ptr(self):
+            raise AssertionError("the wrapper passed a refused buffer on")
+
+    ok_l, ok_o = FakeCuda(cells * 30 * batch), FakeCuda(cells * 5)
+    bad = [
+        (FakeCuda(cells * 30 * batch - 1), ok_o, ok_o, "logits"),        # one logit short
+        (ok_l, FakeCuda(cells * 5 - 1), ok_o, "fit_g"),                  # short output
+        (ok_l, ok_o, FakeCuda(cells * 5, dtype="torch.float64"), "fit_d"),
+        (FakeCuda(cells * 30 * batch, contiguous=False), ok_o, ok_o, "logits"),
+    ]
+    for logits, fg, fd, what in bad:
+        with pytest.raises(L.LipzError) as e:
+            L.lipz_fitness_from_logits_noalloc(logits, cells, batch, fg, fd)
+        assert e.value.code == L.LIPZ_ERR_INVALID and what in str(e.value)

@@ -1,6 +1,6 @@
-"""The allocation-free fitness entry point, for callers that cannot call cudaMalloc (inside a
-CUDA graph capture, under a fully reserved device memory budget, or on a path that cannot
-take cudaMalloc's implicit synchronisation).
+"""The allocation-free fitness entry point, for callers that cannot call cudaMalloc (a serving
+loop whose device memory another allocator has fully reserved, or a latency-critical path that
+cannot take the implicit synchronisation of cudaMalloc / cudaFree).
 
 Its output must match the fitness that lipz_eval_neighborhoods returns for the same logits,
 on two calls in a row of different sizes (the shared scratch array keeps the previous call's
