@@ -66,10 +66,13 @@ BWD_ACT = (3 * BATCH * HIDDEN + 2 * BATCH * HIDDEN + 2 * BATCH * X_DIM + 2 * BAT
 TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN)
                            + 2 * BWD_ACT)
 
-# DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels, from
-# an ncu launch list (dram__bytes_read.sum + dram__bytes_write.sum) of these same kernels.
-PHASE_TRAFFIC = {"batch": 21.2e6, "g_fwd": 161.4e6, "d_fwd": 226.9e6, "fitness": 1.8e6,
-                 "select": 0.0, "train_fwd": 129.0e6, "train_bwd": 2182.6e6, "adam": 3.6e6}
+# DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels: not
+# measured by this script but taken from ncu captures (dram__bytes_read.sum +
+# dram__bytes_write.sum) of these same kernels, named in PHASE_TRAFFIC_SOURCE. A phase whose
+# kernels changed after its capture has no entry (null traffic).
+PHASE_TRAFFIC = {"batch": 21.2e6, "fitness": 1.8e6, "select": 0.0, "adam": 3.6e6,
+                 "train_bwd": 2182.6e6}
+PHASE_TRAFFIC_SOURCE = "ncu capture summarised in profiles/launches_12x12_bf16_iteration.md"
 
 
 def _peaks():
@@ -248,7 +251,7 @@ def run_ours(args):
     }
     if (world == 1 and not args.no_cpu_baseline and args.train_steps == 1 and not args.mixture
             and not args.stale_neighbors):
-        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds, args.cpu_seconds_single)
     return line
 
 
@@ -292,10 +295,13 @@ def _phase_roofs(phase_ms):
             ach, peak, unit = units / (t * 1e-3) / 1e9, hbm, "GB/s"
             src = peak_kind + " HBM copy"
         else:
-            ach, peak, unit = units / (t * 1e-3) / 1e12, tf_sus, "TFLOP/s"
-            src = peak_kind + " sustained bf16"
+            # the timed region lasts milliseconds, not seconds: the burst rate applies
+            ach, peak, unit = units / (t * 1e-3) / 1e12, tf_burst, "TFLOP/s"
+            src = peak_kind + " burst bf16 (cuBLAS)"
+        tr = PHASE_TRAFFIC.get(ph)
         out[ph] = {"bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
-                   "traffic": PHASE_TRAFFIC.get(ph), "kernel": what, "peak_source": src,
+                   "traffic": tr, "traffic_source": PHASE_TRAFFIC_SOURCE if tr else None,
+                   "kernel": what, "peak_source": src,
                    ("algorithmic_bytes" if bound == "hbm" else "algorithmic_flop"): units}
     return out
 
@@ -374,11 +380,56 @@ def _threads():
     return os.cpu_count() or 1
 
 
-def cpu_baseline(seconds):
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), and its logical core count."""
+    name = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            k, _, v = line.partition(":")
+            if k.strip() == "Model name" and v.strip():
+                name = v.strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if not name:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    k, _, v = line.partition(":")
+                    if k.strip() in ("model name", "Hardware", "CPU part") and v.strip():
+                        name = v.strip()
+                        break
+        except OSError:
+            pass
+    return "%s, %d logical cores" % (name or "unknown CPU", os.cpu_count() or 0)
+
+
+def _single_thread_sample(seconds):
+    """The same oracle sample in a fresh interpreter with one BLAS / OpenMP thread (the thread
+    count of a BLAS library is fixed when it loads)."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json, bench; d, e = bench._oracle_sample(%r); print(json.dumps([d, e]))"
+            % float(seconds))
+    try:
+        out = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
+                             text=True, timeout=seconds * 4 + 120)
+        done, el = json.loads(out.stdout.strip().splitlines()[-1])
+    except (OSError, subprocess.SubprocessError, ValueError, IndexError):
+        return None
+    return {"value": 25.0 * done / el, "unit": UNIT, "cores": 1,
+            "sample": "%d cells, %.1f s, one thread" % (done, el)}
+
+
+def cpu_baseline(seconds, single_seconds=None):
     done, el = _oracle_sample(seconds)
-    return {"value": 25.0 * done / el, "unit": UNIT, "cores": _threads(), "kind": "oracle",
-            "sample": "%d cells of the 12x12 bf16 B=100 workload (eval of 25 pairs + selection + "
-                      "gradients + Adam per cell), %.1f s, numpy float64 + OpenBLAS" % (done, el)}
+    out = {"value": 25.0 * done / el, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+           "sample": "%d cells of the 12x12 bf16 B=100 workload (eval of 25 pairs + selection + "
+                     "gradients + Adam per cell), %.1f s, numpy float64 + OpenBLAS" % (done, el),
+           "cpu_model": cpu_model()}
+    if single_seconds:
+        out["single_thread"] = _single_thread_sample(single_seconds)
+    return out
 
 
 # ---- DCGAN workload (the 3x3 DCGAN configuration: width 64, z = 100, B = 128, bf16) --------
@@ -471,10 +522,10 @@ def run_dcgan(args):
         t = phase_ms.get(ph)
         if t and t == t:
             ach = flop / (t * 1e-3) / 1e12
-            roofs[ph] = {"bound": "tensor", "achieved": ach, "peak": tf_sus,
-                         "unit": "TFLOP/s", "frac": ach / tf_sus, "traffic": None,
+            roofs[ph] = {"bound": "tensor", "achieved": ach, "peak": tf_burst,
+                         "unit": "TFLOP/s", "frac": ach / tf_burst, "traffic": None,
                          "algorithmic_flop": flop,
-                         "peak_source": "bf16 dense, sustained (%s)" % kind}
+                         "peak_source": "%s burst bf16 (cuBLAS)" % kind}
     dom = max(roofs, key=lambda k: phase_ms[k])
     roof = dict(roofs[dom], phase=dom)
     line = {
@@ -496,7 +547,7 @@ def run_dcgan(args):
     if world == 1 and not args.no_cpu_baseline:
         done, el = _dc_oracle_sample()
         line["cpu_baseline"] = {"value": 25.0 * done / el, "unit": UNIT, "cores": _threads(),
-                                "kind": "oracle",
+                                "kind": "oracle", "cpu_model": cpu_model(),
                                 "sample": "%d cell(s) of the 3x3 DCGAN workload (evaluation of "
                                           "25 pairs), %.1f s" % (done, el)}
     return line
@@ -552,7 +603,8 @@ def run_reference_dcgan(args):
                        "global_batch": DC_B, "pairs_per_iter": DC_PAIRS, "parallelism": "cpu"},
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
-                             "sample": "1 cell per step of the 3x3 DCGAN workload"},
+                             "sample": "1 cell per step of the 3x3 DCGAN workload",
+                             "cpu_model": cpu_model()},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
@@ -587,7 +639,7 @@ def run_reference(args):
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
                              "sample": "%d cells per step of the 12x12 bf16 B=100 workload"
-                                       % per_step_cells},
+                                       % per_step_cells, "cpu_model": cpu_model()},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
@@ -599,6 +651,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-seconds-single", type=float, default=10.0,
+                    help="seconds of the one-thread oracle sample (0: skip it)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass")
     ap.add_argument("--no-phases", action="store_true", help="skip the per-phase timing pass")

@@ -555,12 +555,22 @@ def select_replace(state: State, ev) -> Dict[str, np.ndarray]:
 # Step 3b: gradients of the selected pair and the Adam update.
 # --------------------------------------------------------------------------------------------
 def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.ndarray,
-                   arch: Arch) -> Tuple[np.ndarray, np.ndarray, Dict[str, float]]:
+                   arch: Arch, flip: Optional[Dict[str, np.ndarray]] = None
+                   ) -> Tuple[np.ndarray, np.ndarray, Dict[str, float]]:
     """dL_D/dv (fake batch detached) and dL_G/du (through D at its pre-update parameters), by
-    the chain rule, layer by layer. Returns flat gradients in the parameter layouts."""
+    the chain rule, layer by layer. Returns flat gradients in the parameter layouts.
+
+    The derivative of ReLU / LeakyReLU jumps at 0, so an implementation whose pre-activation
+    lands on the other side of 0 (another rounding of the same sum) takes the other branch
+    there. ``flip`` (MLP only) names such elements: {"G1", "G2", "D1", "D2"} -> boolean arrays
+    shaped like the pre-activations that ``info["pre"]`` returns (G: [B, h]; D: [2B, h], real
+    rows then fake rows); a True element takes the other branch of the derivative. The values
+    of the activations are unchanged (they are continuous at 0)."""
     a = arch
     rb = _Rounder(a)
     if a.kind == "dcgan":
+        if flip:
+            raise ValueError("flip is defined for the MLP networks")
         return _dcgan().pair_gradients(Gflat, Dflat, x, z, a, rb, unflatten, pair_losses, sigmoid)
     gl, dl = g_layout(a), d_layout(a)
     G, D = unflatten(Gflat, gl), unflatten(Dflat, dl)
@@ -580,13 +590,24 @@ def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.nd
     dl3 = np.concatenate([dl_d, dl_g])
     g2_3 = np.vstack([g2, g2[B:]])
     g1_3 = np.vstack([g1, g1[B:]])
+    fl = flip or {}
+
+    def side(y, name, rows3=False):
+        # which side of 0 each pre-activation lies on (the activation has its sign), with the
+        # elements named in ``flip`` on the other side; D's fake rows serve both losses
+        pos = y > 0.0
+        f = fl.get(name)
+        if f is not None:
+            pos = pos ^ (np.vstack([f, f[B:]]) if rows3 else f)
+        return pos
+
     w3 = rb(D["W3"])[0]
     gD["W3"][0] = dl_d @ g2
     gD["b3"][0] = dl_d.sum()
-    d2 = rb(dl3[:, None] * w3[None, :] * np.where(g2_3 > 0.0, 1.0, slope))
+    d2 = rb(dl3[:, None] * w3[None, :] * np.where(side(g2_3, "D2", True), 1.0, slope))
     gD["W2"][:] = d2[:2 * B].T @ g1
     gD["b2"][:] = d2[:2 * B].sum(axis=0)
-    d1 = rb((d2 @ rb(D["W2"])) * np.where(g1_3 > 0.0, 1.0, slope))
+    d1 = rb((d2 @ rb(D["W2"])) * np.where(side(g1_3, "D1", True), 1.0, slope))
     gD["W1"][:] = d1[:2 * B].T @ X
     gD["b1"][:] = d1[:2 * B].sum(axis=0)
     # Generator chain: through D's first layer into the fakes, then back through G.
@@ -595,10 +616,10 @@ def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.nd
     a3 = rb(dF * (1.0 - F * F))
     gG["W3"][:] = a3.T @ h2
     gG["b3"][:] = a3.sum(axis=0)
-    a2 = rb((a3 @ rb(G["W3"])) * (h2 > 0.0))
+    a2 = rb((a3 @ rb(G["W3"])) * side(h2, "G2"))
     gG["W2"][:] = a2.T @ h1
     gG["b2"][:] = a2.sum(axis=0)
-    a1 = rb((a2 @ rb(G["W2"])) * (h1 > 0.0))
+    a1 = rb((a2 @ rb(G["W2"])) * side(h1, "G1"))
     gG["W1"][:] = a1.T @ zq
     gG["b1"][:] = a1.sum(axis=0)
     lg, ld = pair_losses(logit[:B], logit[B:])
@@ -606,10 +627,10 @@ def pair_gradients(Gflat: np.ndarray, Dflat: np.ndarray, x: np.ndarray, z: np.nd
     flatD = np.concatenate([gD[n].reshape(-1) for n, _ in dl])
     # Distance of the closest pre-activation to a kink of ReLU / LeakyReLU (where the derivative
     # jumps): a diagnostic for comparisons with implementations that round differently.
-    pre = [zq @ rb(G["W1"]).T + G["b1"], h1 @ rb(G["W2"]).T + G["b2"],
-           X @ rb(D["W1"]).T + D["b1"], g1 @ rb(D["W2"]).T + D["b2"]]
-    kink = min(float(np.min(np.abs(p))) for p in pre)
-    return flatG, flatD, {"LG": lg, "LD": ld, "kink": kink}
+    pre = {"G1": zq @ rb(G["W1"]).T + G["b1"], "G2": h1 @ rb(G["W2"]).T + G["b2"],
+           "D1": X @ rb(D["W1"]).T + D["b1"], "D2": g1 @ rb(D["W2"]).T + D["b2"]}
+    kink = min(float(np.min(np.abs(p))) for p in pre.values())
+    return flatG, flatD, {"LG": lg, "LD": ld, "kink": kink, "pre": pre}
 
 
 def adam_step(w, m, v, step, g, lr, arch: Arch):

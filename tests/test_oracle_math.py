@@ -292,3 +292,46 @@ def test_later_minibatch_steps_draw_fresh_batches():
     zs = [O.draw_batch(7, 4, 1, pool, a, k)[1] for k in range(3)]
     assert np.array_equal(zs[0], O.draw_batch(7, 4, 1, pool, a)[1])
     assert not np.array_equal(zs[0], zs[1]) and not np.array_equal(zs[1], zs[2])
+
+
+@pytest.mark.parametrize("layer,row", [("G1", 3), ("G2", 0), ("D1", 2), ("D1", 9), ("D2", 5),
+                                       ("D2", 11)])
+def test_flipped_derivative_branch_equals_the_other_side_of_the_kink(layer, row):
+    """pair_gradients(flip=...) takes the other branch of a ReLU / LeakyReLU derivative at the
+    named elements (for comparisons with implementations whose pre-activation lands on the other
+    side of 0). Pinned against torch autograd: the bias of the element's unit is set so that
+    the element's pre-activation is +1e-9; flipping it must give the gradients that autograd
+    computes with the pre-activation at -1e-9 (bias lowered by 2e-9), where the derivative is
+    the other branch and every other quantity moves by O(1e-9). D rows 7.. are the fake batch,
+    whose derivative serves both losses."""
+    arch = O.Arch(z_dim=6, hidden=10, x_dim=9, batch=7)
+    rng = np.random.default_rng(11)
+    gl, dl = O.g_layout(arch), O.d_layout(arch)
+    G = rng.normal(scale=0.5, size=O.n_params(gl))
+    D = rng.normal(scale=0.5, size=O.n_params(dl))
+    x = rng.uniform(-1, 1, size=(7, 9))
+    z = rng.normal(size=(7, 6))
+    net, lay = (G, gl) if layer[0] == "G" else (D, dl)
+    bname = "b" + layer[1]
+    off = 0
+    for name, shape in lay:
+        if name == bname:
+            break
+        off += int(np.prod(shape))
+    pre = O.pair_gradients(G, D, x, z, arch)[2]["pre"][layer]
+    unit = int(np.argmax(np.abs(pre[row])))    # a unit that carries a real delta
+    eps = 1e-9
+    net[off + unit] += eps - pre[row, unit]    # now pre[row, unit] = +eps
+    info = O.pair_gradients(G, D, x, z, arch)[2]
+    assert abs(info["pre"][layer][row, unit] - eps) < 1e-12
+    others = np.delete(info["pre"][layer][:, unit], row)
+    assert np.min(np.abs(others)) > 1e-6       # no other row crosses 0 with the shift
+    flip = {layer: np.zeros_like(info["pre"][layer], dtype=bool)}
+    flip[layer][row, unit] = True
+    fG, fD, _ = O.pair_gradients(G, D, x, z, arch, flip=flip)
+    nG, nD, _ = O.pair_gradients(G, D, x, z, arch)
+    net[off + unit] -= 2 * eps                 # pre[row, unit] = -eps
+    tG, tD = _torch_grads(G, D, x, z, arch)
+    assert np.allclose(fG, tG, rtol=1e-6, atol=1e-8) and np.allclose(fD, tD, rtol=1e-6, atol=1e-8)
+    # and the flip mattered: the unflipped gradients are the other side's
+    assert np.max(np.abs(np.concatenate([nG - tG, nD - tD]))) > 1e-4
