@@ -8,7 +8,7 @@ import pytest
 
 from oracle import lipz_oracle as O
 
-from helpers import max_rel, oracle_arch, per_tensor
+from helpers import gradient_parity, max_rel, oracle_arch
 
 pytestmark = pytest.mark.gpu
 
@@ -31,11 +31,12 @@ def _pool(seed, n, dim):
     return lipz_synth.blob_pool(seed, n=n, dim=dim)
 
 
-def _lockstep(g, pool, prev, kink_band):
+def _lockstep(g, pool, prev, label):
     """One stale iteration against the oracle started from the engine's current and previous
     states: evaluation within tolerance, selection bit-exact given the engine's fitness, then
-    the new state's step counts and lrs exactly and its gradients and moments within tolerance
-    (cells at a kink excused, as in the one-step check). Returns the state it started from."""
+    the new state's step counts and lrs exactly, the gradients by the rules of
+    helpers.gradient_parity, and the moments and weights as Adam steps of the selected (possibly
+    older) individual given the engine's own gradient. Returns the state it started from."""
     a = oracle_arch(g.arch)
     s = O.state_from_bytes(g.export_state(), a)
     tol = TOL[g.arch.precision]
@@ -56,17 +57,27 @@ def _lockstep(g, pool, prev, kink_band):
     assert np.array_equal(got.Gstep, new.Gstep) and np.array_equal(got.Dstep, new.Dstep)
     assert np.allclose(got.Glr, new.Glr, rtol=1e-6) and np.allclose(got.Dlr, new.Dlr, rtol=1e-6)
     gg, gd = g.gradients()
-    worst = np.zeros(s.cells)
-    pairs = [("G", gg, grads["gG"]), ("D", gd, grads["gD"]), ("G", got.Gm, new.Gm),
-             ("D", got.Dm, new.Dm)]
-    for pop, gpu, r in pairs:
-        lay = O.g_layout(a) if pop == "G" else O.d_layout(a)
+    nbr = O.neighbors(s.rows, s.cols)
+
+    def source(pop, c):
+        slot = int(ref_sel["sel_" + pop.lower()][c])
+        return O._slot_state(s, prev, slot), int(nbr[c][slot])
+
+    def pair_inputs(c):
+        (SG, kg), (SD, kd) = source("G", c), source("D", c)
+        return (SG.Gw[kg], SD.Dw[kd]) + tuple(data[c])
+
+    gradient_parity(label, a, gg, gd, grads["gG"], grads["gD"], tol, pair_inputs)
+    for pop, gpu_g in (("G", gg), ("D", gd)):
         for c in range(s.cells):
-            worst[c] = max(worst[c], max(per_tensor(gpu[c:c + 1], r[c:c + 1], lay).values()))
-    ok = worst < tol
-    kinky = grads["kink"] < kink_band
-    assert np.all(ok | kinky), ("mismatch without a kink", np.where(~ok)[0], worst)
-    assert np.sum(~ok) <= max(1, s.cells // 4), worst
+            S, k = source(pop, c)
+            w1, m1, v1, _ = O.adam_step(getattr(S, pop + "w")[k], getattr(S, pop + "m")[k],
+                                        getattr(S, pop + "v")[k], getattr(S, pop + "step")[k],
+                                        gpu_g[c].astype(np.float64),
+                                        float(np.float32(getattr(new, pop + "lr")[c])), a)
+            for f, r in (("w", w1), ("m", m1), ("v", v1)):
+                v = getattr(got, pop + f)[c]
+                assert np.max(np.abs(v - r)) <= 1e-6 * np.max(np.abs(r)) + 1e-12, (pop, f, c)
     return s, ref_sel
 
 
@@ -81,7 +92,7 @@ def test_stale_neighbours_lockstep(L, precision, rows, cols, batch):
     g.set_data(pool)
     prev, picked = None, 0
     for it in range(4):
-        s, sel = _lockstep(g, pool, prev, 1e-5 if precision == "fp32" else 1e-3)
+        s, sel = _lockstep(g, pool, prev, "stale %s %dx%d it %d" % (precision, rows, cols, it))
         if it > 0:
             picked += int(np.sum(sel["sel_g"] != 0) + np.sum(sel["sel_d"] != 0))
         prev = s
