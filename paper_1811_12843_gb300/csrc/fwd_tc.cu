@@ -141,14 +141,6 @@ __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   return p.centre ? p.indiv_off + prob : __ldg(&p.nbr[prob]);
 }
 
-// Hardware tanh (relative error below 2^-10.9, i.e. under half a bf16 ulp of the rounded
-// output that follows it).
-__device__ __forceinline__ float tanh_approx(float x) {
-  float y;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
 // ---- the kernel ----------------------------------------------------------------------------
 // KND: p.kind at compile time (one variant per network kind, each with only its own paths)
 template <int KND>
@@ -588,8 +580,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t pk[8];
 #pragma unroll
             for (int e = 0; e < 16; e += 2)
-              pk[e >> 1] = pack_bf16(tanh_approx(__uint_as_float(r[e]) + bv[e]),
-                                     tanh_approx(__uint_as_float(r[e + 1]) + bv[e + 1]));
+              pk[e >> 1] = pack_bf16(tanhf(__uint_as_float(r[e]) + bv[e]),
+                                     tanhf(__uint_as_float(r[e + 1]) + bv[e + 1]));
             if (rr < p.B && col0 < p.x) {
               uint4* o = reinterpret_cast<uint4*>(dst + col0);
               o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);

@@ -61,11 +61,12 @@ def per_tensor(flat_got, flat_ref, layout):
 # instead of float64 products and otherwise the same code, differs from the float64 oracle by
 # up to 2e-2 in a few cells (median 1e-3). The rule is an error budget: every cell within
 # BF16_CEIL x tol, at most one cell in eight above tol, and the median cell within
-# BF16_MEDIAN x tol. A method error (a wrong row, cell, slot or tile tail) is of order one.
+# BF16_MEDIAN x tol (the engine's medians lie at 1e-3 to 5e-3). A method error (a wrong row,
+# cell, slot or tile tail) is of order one.
 FP32_FLIP_BAND = 2e-6
 MAX_FLIPS = 8
 BF16_CEIL = 2.5
-BF16_MEDIAN = 0.5
+BF16_MEDIAN = 0.35
 
 
 def cell_errors(gpu, ref, layout):
