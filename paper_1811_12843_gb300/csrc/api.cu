@@ -78,6 +78,8 @@ struct lipz_grid {
   // parity: every slot from the current snapshot, or (stale neighbours) slots 1..4 from the
   // other snapshot, which holds the previous iteration's centres
   int *nbr_cur[3]{}, *nbr_stale[3]{};
+  // the same tables as work lists of the CTA-pair evaluation kernels (tensor-core path)
+  TcPairs pairs_cur[3]{}, pairs_stale[3]{};
   bool prev_valid = false;  // the other snapshot holds the previous iteration's centres
   int *sel_g = nullptr, *sel_d = nullptr, *src_g = nullptr, *src_d = nullptr;
   float *lrn_g = nullptr, *lrn_d = nullptr;
@@ -303,6 +305,25 @@ int build_descs(lipz_grid* g, int p) {
     if ((rc = upload(g, &g->nbr_cur[p], cur)) || (rc = upload(g, &g->nbr_stale[p], stale)))
       return rc;
     return LIPZ_OK;
+  }
+  // pair lists of both tables for the tensor-core evaluation
+  auto pair_lists = [&](const std::vector<int>& tab, TcPairs& P) -> int {
+    std::vector<int4> gp, dp;
+    std::vector<int2> pl;
+    tc_build_pairs(tab.data(), C, g->nsnap * C, B, &gp, &dp, &pl);
+    int4 *dg = nullptr, *dd = nullptr;
+    int2* dl = nullptr;
+    int rc;
+    if ((rc = upload(g, &dg, gp)) || (rc = upload(g, &dd, dp)) || (rc = upload(g, &dl, pl)))
+      return rc;
+    P = TcPairs{dg, (int)gp.size(), dd, (int)dp.size(), dl};
+    return LIPZ_OK;
+  };
+  {
+    int rc;
+    if ((rc = pair_lists(cur, g->pairs_cur[p])) ||
+        (g->a.stale_neighbors && (rc = pair_lists(stale, g->pairs_stale[p]))))
+      return rc;
   }
   // evaluation descriptors of one neighbour table
   auto eval_descs = [&](const std::vector<int>& tab, Descs& D) -> int {
@@ -767,6 +788,9 @@ SelectIO select_io(lipz_grid* g);
 const int* eval_nbr(const lipz_grid* g) {
   return g->a.stale_neighbors && g->prev_valid ? g->nbr_stale[g->cur] : g->nbr_cur[g->cur];
 }
+const TcPairs* eval_pairs(const lipz_grid* g) {
+  return g->a.stale_neighbors && g->prev_valid ? &g->pairs_stale[g->cur] : &g->pairs_cur[g->cur];
+}
 
 // Minibatch step `step` of the current iteration into E's real rows and Z (the real rows from
 // xin_dev when given, else from the pool).
@@ -840,7 +864,7 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
     phase_end(g, LIPZ_PHASE_D_FWD, dc_eval_launches(g->dc, 1));
   } else if (g->use_tc) {
     std::string msg;
-    tc_set_nbr(g->tc[p], eval_nbr(g));
+    tc_set_nbr(g->tc[p], eval_nbr(g), eval_pairs(g));
     phase_begin(g, LIPZ_PHASE_G_FWD);
     if (tc_run_g(g->tc[p], g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, 1);

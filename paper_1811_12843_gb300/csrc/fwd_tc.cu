@@ -21,7 +21,9 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <cstring>
+#include <vector>
 
 #include "common.cuh"
 #include "fwd_tc.h"
@@ -605,14 +607,522 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+
+// ---- evaluation by CTA pairs (tcgen05 .cta_group::2) ----------------------------------------
+// The two CTAs of a cluster share every weight chunk: each loads half of the chunk's rows
+// (128 of the 256 output columns), holds its own 128 rows of the activations, and the pair's
+// MMAs (M = 256, issued by rank 0) read both halves, so a weight byte brought from L2 serves
+// 256 rows instead of 128. A pair works on one individual:
+//   generator: the individual's 5B rows (the z rows of every cell whose neighbourhood holds it,
+//              in the order of its (cell, slot) problems), two 128-row blocks per pair; the
+//              noise rows are gathered into shared memory by a warp of their own;
+//   discriminator: two 128-row tiles of (cell, slot) problems that share the individual (a
+//              lone tile's partner computes zeros and stores nothing).
+constexpr int HB_BYTES = (HID / 2) * BK * 2;  // 16 KB: half of a 256-row weight box
+constexpr int NUM_PWARPS = 2 + NUM_EPI_WARPS + 1;
+constexpr int P_THREADS = 32 * NUM_PWARPS;
+constexpr int PAIR_EPI_ARRIVALS = 2 * NUM_EPI_WARPS;  // one per epilogue warp of both CTAs
+
+template <int KND>
+struct PCfg;
+// generator: rings of weight halves only (its first layer's A is the gathered noise tile)
+template <>
+struct PCfg<KIND_G> {
+  static constexpr int STAGES = 8, STAGE = HB_BYTES, A_IN = 0, ZBUF = A_BYTES;
+};
+// discriminator: each stage holds the A chunk and the weight half
+template <>
+struct PCfg<KIND_D> {
+  static constexpr int STAGES = 4, STAGE = A_BYTES + HB_BYTES, A_IN = 1, ZBUF = 0;
+};
+template <int KND>
+constexpr int pair_smem_bytes() {
+  return 1024 + PCfg<KND>::STAGES * PCfg<KND>::STAGE + PCfg<KND>::ZBUF + H_BYTES + MISC_BYTES +
+         BIAS_BYTES;
+}
+static_assert(pair_smem_bytes<KIND_G>() <= 232448, "generator pair kernel: shared memory");
+static_assert(pair_smem_bytes<KIND_D>() <= 232448, "discriminator pair kernel: shared memory");
+static_assert(2 * PCfg<KIND_G>::STAGES + 14 <= 32, "barriers must fit below the TMEM slot");
+
+struct PParams {
+  int B, x, rows;  // rows per problem: B (generator) or 6B (discriminator)
+  int kc1, n3;
+  int n_pairs;
+  // generator: {individual, first row of the pair's 256, offset into plist, rows of the
+  // individual}; discriminator: {individual, problem of rank 0, problem of rank 1 (-1: none),
+  // first row of rank 0's tile << 16 | first row of rank 1's tile}; problem = cell * 5 + slot
+  const int4* pairs;
+  const int2* plist;  // generator: (cell, slot) of each problem of an individual, in row order
+  const bf16* Z;      // generator: noise [cells][B][64]
+  const float* wmaster;
+  const bf16* wb;
+  int64_t pstride;
+  int64_t off_b1, off_b2, off_b3, off_w3;
+  bf16* E;
+  int64_t e_cell;
+  float* logits;
+  float slope;
+  int* err;
+};
+
+template <int KND>
+__device__ __forceinline__ Job pair_job(const PParams& p, int j) {
+  if (j == 0) return Job{0, p.kc1, HID, 0, 0, 0, HID, EPI_TO_H};
+  if (j == 1) return Job{1, HID / BK, HID, 1, 1, 0, HID, KND == KIND_D ? EPI_LOGIT : EPI_TO_H};
+  const int nb = j - 2;
+  const int n = min(N3, p.x - nb * N3);
+  return Job{1, HID / BK, (n + 15) & ~15, (nb + p.n3) & 1, 2, nb * N3, N3, EPI_TO_E};
+}
+
+template <int KND>
+__global__ void __launch_bounds__(P_THREADS, 1)
+    k_mlp_fwd_pair(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB1,
+                   const __grid_constant__ CUtensorMap mB2, const __grid_constant__ CUtensorMap mB3,
+                   const PParams p) {
+  using CF = PCfg<KND>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sStage = base;                        // STAGES x ([A] | weight half)
+  const uint32_t sZ = base + CF::STAGES * CF::STAGE;   // generator: the gathered noise rows
+  const uint32_t sH = sZ + CF::ZBUF;                   // on-chip activation (own 128 rows)
+  uint8_t* misc = gbase + CF::STAGES * CF::STAGE + CF::ZBUF + H_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(misc);
+  const uint32_t bFull = smem_u32(bars);               // [STAGES], used in rank 0
+  const uint32_t bEmpty = bFull + 8 * CF::STAGES;      // [STAGES]
+  const uint32_t bAcc = bEmpty + 8 * CF::STAGES;       // [2]
+  const uint32_t bReg = bAcc + 16;                     // [2], rank 0
+  const uint32_t bH = bReg + 16;                       // [4], rank 0
+  const uint32_t bPart = bH + 32;
+  const uint32_t bFinal = bPart + 8;
+  const uint32_t bBias = bFinal + 8;                   // [2]
+  const uint32_t bZfull = bBias + 16;                  // rank 0
+  const uint32_t bZempty = bZfull + 8;
+  float* s_bias = reinterpret_cast<float*>(misc + MISC_BYTES);
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 256);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 260);
+  float* part = reinterpret_cast<float*>(misc + 512);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < CF::STAGES; ++s) {
+      mbar_init(bFull + 8 * s, 1);
+      mbar_init(bEmpty + 8 * s, 1);
+    }
+    for (int r = 0; r < 2; ++r) {
+      mbar_init(bAcc + 8 * r, 1);
+      mbar_init(bReg + 8 * r, PAIR_EPI_ARRIVALS);
+      mbar_init(bBias + 8 * r, 32 * NUM_EPI_WARPS);
+    }
+    for (int c = 0; c < HID / BK; ++c) mbar_init(bH + 8 * c, PAIR_EPI_ARRIVALS);
+    mbar_init(bPart, 32 * NUM_EPI_WARPS / 2);
+    mbar_init(bFinal, 1);
+    mbar_init(bZfull, 2);
+    mbar_init(bZempty, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    // one warp of each CTA of the pair allocates together: the same columns in both
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+  }
+  tc_fence_before();
+  cluster_sync_all();  // no remote arrival before the peer's barriers exist
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // rank 0's barriers that both CTAs arrive on
+  const uint32_t lFull = mapa_shared(bFull, 0), lReg = mapa_shared(bReg, 0);
+  const uint32_t lH = mapa_shared(bH, 0), lZfull = mapa_shared(bZfull, 0);
+  const int nj = KND == KIND_D ? 2 : 2 + p.n3;
+  const int cid = (int)cluster_id_x(), ncl = (int)nclusters_x();
+  pdl_wait();
+
+  if (warp == 0) {
+    // ================================ TMA producer (both CTAs) ================================
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int pi = cid; pi < p.n_pairs && ok; pi += ncl) {
+        const int4 pr = __ldg(&p.pairs[pi]);
+        const int k = pr.x;
+        int a_cell = 0, a_row = p.rows;  // no problem: rows past the end read as zero
+        if (KND == KIND_D) {
+          const int prob = rank ? pr.z : pr.y;
+          if (prob >= 0) {
+            a_cell = prob / 5;
+            a_row = rank ? (pr.w & 0xFFFF) : (pr.w >> 16);
+          }
+        }
+        for (int j = 0; j < nj && ok; ++j) {
+          const Job J = pair_job<KND>(p, j);
+          const CUtensorMap* mb = J.bmap == 0 ? &mB1 : (J.bmap == 1 ? &mB2 : &mB3);
+          const bool a_ring = CF::A_IN && !J.a_from_h;
+          const uint32_t bytes = (a_ring ? (uint32_t)A_BYTES : 0u) + (uint32_t)HB_BYTES;
+          for (int kc = 0; kc < J.kchunks; ++kc) {
+            if (!mbar_wait(bEmpty + 8 * stage, phase ^ 1u, abort_flag, p.err, 1)) {
+              ok = false;
+              break;
+            }
+            // rank 0 expects both CTAs' bytes; the peer's may land first
+            if (leader) mbar_expect_tx(bFull + 8 * stage, 2 * bytes);
+            const uint32_t sS = sStage + stage * CF::STAGE;
+            const uint32_t full = lFull + 8 * stage;
+            if (a_ring) tma_load_3d_cg2(sS, &mA, full, kc * BK, a_row, a_cell);
+            tma_load_3d_cg2(sS + (CF::A_IN ? A_BYTES : 0), mb, full, kc * BK,
+                            J.brow0 + (int)rank * (J.n / 2), k);
+            if (++stage == CF::STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+      if (!ok) {
+        // loads issued here complete on rank 0's barriers: give them time to land before the
+        // CTA leaves
+        const unsigned long long t0 = globaltimer();
+        while (globaltimer() - t0 < 200000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ================================ MMA issuer (rank 0) ================================
+    if (leader && lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int reg_uses[2] = {0, 0};
+      int h_total = 0, zuse = 0;
+      bool ok = true;
+      for (int pi = cid; pi < p.n_pairs && ok; pi += ncl) {
+        for (int j = 0; j < nj && ok; ++j) {
+          const Job J = pair_job<KND>(p, j);
+          const int R = J.region;
+          if (reg_uses[R] > 0 &&
+              !mbar_wait_cl(bReg + 8 * R, (uint32_t)((reg_uses[R] - 1) & 1), abort_flag, p.err, 2)) {
+            ok = false;
+            break;
+          }
+          if (KND == KIND_G && j == 0 &&
+              !mbar_wait_cl(bZfull, (uint32_t)(zuse & 1), abort_flag, p.err, 9)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)(R * HID);
+          const uint32_t idesc = idesc_bf16(2 * BM, J.n);
+          for (int kc = 0; kc < J.kchunks; ++kc) {
+            if (J.a_from_h &&
+                !mbar_wait_cl(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
+              ok = false;
+              break;
+            }
+            if (!mbar_wait_cl(bFull + 8 * stage, phase, abort_flag, p.err, 4)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sS = sStage + stage * CF::STAGE;
+            const uint32_t sA = (KND == KIND_G && j == 0)
+                                    ? sZ
+                                    : (J.a_from_h ? sH + kc * H_CHUNK : sS);
+            const uint32_t sB = sS + (CF::A_IN ? A_BYTES : 0);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              tc_mma_cg2(d, sw128_desc(sA + kk * 32), sw128_desc(sB + kk * 32), idesc,
+                         (kc | kk) != 0 ? 1u : 0u);
+            tc_commit_cg2(bEmpty + 8 * stage, 3);
+            if (++stage == CF::STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (!ok) break;
+          if (KND == KIND_G && j == 0) {
+            tc_commit_cg2(bZempty, 3);
+            ++zuse;
+          }
+          tc_commit_cg2(bAcc + 8 * R, 3);
+          reg_uses[R]++;
+          if (J.epi == EPI_TO_H) ++h_total;
+        }
+      }
+      // every MMA (they write both CTAs' tensor memory) completes before it is released
+      tc_commit_cg2(bFinal, 3);
+      volatile int never = 0;
+      mbar_wait(bFinal, 0u, &never, p.err, 5);
+    }
+  } else if (warp < 2 + NUM_EPI_WARPS) {
+    // ================================ epilogue (own 128 rows) ================================
+    const int ew = warp - 2;
+    const int q = warp & 3;
+    const int hf = ew >> 2;
+    const int row = q * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const int et = threadIdx.x - 64;
+    int reg_uses[2] = {0, 0};
+    bool ok = true;
+    int ltile = 0;
+    // a warp's share of a region, an H chunk: its lanes' writes are done (and, for H, made
+    // visible to the tensor cores) before lane 0 arrives on rank 0's barrier
+    auto warp_arrive = [&](uint32_t bar_cluster) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(bar_cluster);
+    };
+    for (int pi = cid; pi < p.n_pairs && ok; pi += ncl, ++ltile) {
+      const int4 pr = __ldg(&p.pairs[pi]);
+      const int k = pr.x;
+      bool row_ok;
+      bf16* dst = nullptr;   // generator: this row of the fakes
+      int64_t lidx = 0;      // discriminator: this row's logit
+      if (KND == KIND_G) {
+        const int gr = pr.y + (int)rank * BM + row;
+        row_ok = gr < pr.w;
+        if (row_ok) {
+          const int pp = gr / p.B, b = gr - pp * p.B;
+          const int2 cs = __ldg(&p.plist[pr.z + pp]);
+          dst = p.E + (int64_t)cs.x * p.e_cell + (int64_t)((1 + cs.y) * p.B + b) * p.x;
+        }
+      } else {
+        const int prob = rank ? pr.z : pr.y;
+        const int rr = (rank ? (pr.w & 0xFFFF) : (pr.w >> 16)) + row;
+        row_ok = prob >= 0 && rr < p.rows;
+        lidx = (int64_t)prob * p.rows + rr;
+      }
+      const float* wm = p.wmaster + (int64_t)k * p.pstride;
+      float* sb = s_bias + (ltile & 1) * BIAS_MAX;
+      {
+        const int nb3 = KND == KIND_D ? HID + 1 : p.x;
+        constexpr int NV = (BIAS_MAX + 32 * NUM_EPI_WARPS - 1) / (32 * NUM_EPI_WARPS);
+        float v[NV];
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+          const int i = et + u * 32 * NUM_EPI_WARPS;
+          v[u] = 0.f;
+          if (i >= 512 + nb3) continue;
+          if (i < 256) v[u] = wm[p.off_b1 + i];
+          else if (i < 512) v[u] = wm[p.off_b2 + i - 256];
+          else if (KND == KIND_D)
+            v[u] = i < 512 + HID
+                       ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
+                       : wm[p.off_b3];
+          else v[u] = wm[p.off_b3 + i - 512];
+        }
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+          const int i = et + u * 32 * NUM_EPI_WARPS;
+          if (i < 512 + nb3) sb[i] = v[u];
+        }
+        mbar_arrive(bBias + 8 * (ltile & 1));
+        if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
+                            p.err, 8)) {
+          ok = false;
+          break;
+        }
+      }
+      for (int j = 0; j < nj && ok; ++j) {
+        const Job J = pair_job<KND>(p, j);
+        const int R = J.region;
+        if (!mbar_wait_cl_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tbase = tmem + lane_base + (uint32_t)(R * HID);
+        if (J.epi == EPI_TO_H) {
+          const float* bias = sb + (j == 0 ? 0 : 256);
+          const float lo = KND == KIND_D ? p.slope : 0.f;
+#pragma unroll 1
+          for (int ch = 0; ch < HID / BK; ++ch) {
+            const int cg = 2 * ch + hf;
+            uint32_t r[32];
+            LIPZ_TMEM_LD32(tbase + cg * 32, r);
+            tmem_wait_ld();
+            const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
+            uint32_t pk[16];
+#pragma unroll
+            for (int e = 0; e < 32; e += 4) {
+              const float4 bb = b4[e >> 2];
+              float a0 = __uint_as_float(r[e]) + bb.x;
+              float a1 = __uint_as_float(r[e + 1]) + bb.y;
+              float a2 = __uint_as_float(r[e + 2]) + bb.z;
+              float a3 = __uint_as_float(r[e + 3]) + bb.w;
+              a0 = a0 > 0.f ? a0 : lo * a0;
+              a1 = a1 > 0.f ? a1 : lo * a1;
+              a2 = a2 > 0.f ? a2 : lo * a2;
+              a3 = a3 > 0.f ? a3 : lo * a3;
+              pk[e >> 1] = pack_bf16(a0, a1);
+              pk[(e >> 1) + 1] = pack_bf16(a2, a3);
+            }
+            const uint32_t chunk = sH + (uint32_t)(ch * H_CHUNK) + (uint32_t)row * 128u;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const uint32_t unit = (uint32_t)(hf * 4 + u);
+              const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[4 * u]),
+                           "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]), "r"(pk[4 * u + 3])
+                           : "memory");
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            warp_arrive(lH + 8 * ch);
+          }
+          tc_fence_before();
+          warp_arrive(lReg + 8 * R);
+        } else if (J.epi == EPI_LOGIT) {
+          const float* bias = sb + 256;
+          const float* w3 = sb + 512;
+          float acc = 0.f;
+#pragma unroll 1
+          for (int cp = hf * 4; cp < hf * 4 + 4; cp += 2) {
+            uint32_t r2[2][32];
+            LIPZ_TMEM_LD32(tbase + cp * 32, r2[0]);
+            LIPZ_TMEM_LD32(tbase + (cp + 1) * 32, r2[1]);
+            tmem_wait_ld();
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const int cg = cp + h2;
+              const uint32_t(&r)[32] = r2[h2];
+              const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
+              const float4* w4 = reinterpret_cast<const float4*>(w3 + cg * 32);
+#pragma unroll
+              for (int e = 0; e < 32; e += 4) {
+                const float4 bb = b4[e >> 2], ww = w4[e >> 2];
+                float a0 = __uint_as_float(r[e]) + bb.x;
+                float a1 = __uint_as_float(r[e + 1]) + bb.y;
+                float a2 = __uint_as_float(r[e + 2]) + bb.z;
+                float a3 = __uint_as_float(r[e + 3]) + bb.w;
+                a0 = a0 > 0.f ? a0 : p.slope * a0;
+                a1 = a1 > 0.f ? a1 : p.slope * a1;
+                a2 = a2 > 0.f ? a2 : p.slope * a2;
+                a3 = a3 > 0.f ? a3 : p.slope * a3;
+                const uint32_t q01 = pack_bf16(a0, a1), q23 = pack_bf16(a2, a3);
+                const __nv_bfloat162 v01 = *reinterpret_cast<const __nv_bfloat162*>(&q01);
+                const __nv_bfloat162 v23 = *reinterpret_cast<const __nv_bfloat162*>(&q23);
+                acc = fmaf(__low2float(v01), ww.x, acc);
+                acc = fmaf(__high2float(v01), ww.y, acc);
+                acc = fmaf(__low2float(v23), ww.z, acc);
+                acc = fmaf(__high2float(v23), ww.w, acc);
+              }
+            }
+          }
+          tc_fence_before();
+          if (hf == 1) {
+            part[row] = acc;
+            mbar_arrive(bPart);
+            warp_arrive(lReg + 8 * R);
+          } else {
+            if (!mbar_wait_warp(bPart, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 7)) {
+              ok = false;
+              break;
+            }
+            const float logit = acc + part[row] + sb[512 + HID];
+            warp_arrive(lReg + 8 * R);
+            if (row_ok) p.logits[lidx] = logit;
+          }
+        } else {
+          // generator output block: bias + tanh, bf16, into this row's fakes
+          const float* bias = sb + 512;
+          const int ng = J.n / 16;
+          const int split = (ng + 1) / 2;
+          const int g0 = hf ? split : 0, g1 = hf ? ng : split;
+#pragma unroll 1
+          for (int gi = g0; gi < g1; ++gi) {
+            uint32_t r[16];
+            LIPZ_TMEM_LD16(tbase + gi * 16, r);
+            tmem_wait_ld();
+            const int col0 = J.brow0 + gi * 16;
+            const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
+            uint32_t pk[8];
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+              const float4 t = b4[qq];
+              pk[2 * qq] = pack_bf16(tanhf(__uint_as_float(r[4 * qq]) + t.x),
+                                     tanhf(__uint_as_float(r[4 * qq + 1]) + t.y));
+              pk[2 * qq + 1] = pack_bf16(tanhf(__uint_as_float(r[4 * qq + 2]) + t.z),
+                                         tanhf(__uint_as_float(r[4 * qq + 3]) + t.w));
+            }
+            if (row_ok && col0 < p.x) {
+              uint4* o = reinterpret_cast<uint4*>(dst + col0);
+              o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+              o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            }
+          }
+          tc_fence_before();
+          warp_arrive(lReg + 8 * R);
+        }
+        reg_uses[R]++;
+      }
+    }
+  } else if (KND == KIND_G) {
+    // ================================ noise gather (generator) ================================
+    // this CTA's 128 rows of the individual's z rows, 16-byte units in the 128-byte swizzle
+    int zuse = 0;
+    for (int pi = cid; pi < p.n_pairs; pi += ncl, ++zuse) {
+      const int4 pr = __ldg(&p.pairs[pi]);
+      if (zuse > 0 &&
+          !mbar_wait_cl_warp(bZempty, (uint32_t)((zuse - 1) & 1), abort_flag, p.err, 10))
+        break;
+      const int row0 = pr.y + (int)rank * BM;
+#pragma unroll 1
+      for (int t0 = 0; t0 < 32; t0 += 8) {
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int idx = lane + 32 * (t0 + u);
+          const int r = idx >> 3, c16 = idx & 7;
+          const int gr = row0 + r;
+          v[u] = make_uint4(0u, 0u, 0u, 0u);
+          if (gr < pr.w) {
+            const int pp = gr / p.B, b = gr - pp * p.B;
+            const int2 cs = __ldg(&p.plist[pr.z + pp]);
+            v[u] = __ldg(reinterpret_cast<const uint4*>(p.Z + ((int64_t)cs.x * p.B + b) * BK) +
+                         c16);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int idx = lane + 32 * (t0 + u);
+          const int r = idx >> 3, c16 = idx & 7;
+          const uint32_t addr = sZ + (uint32_t)r * 128u + ((uint32_t)(c16 ^ (r & 7)) << 4);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v[u].x),
+                       "r"(v[u].y), "r"(v[u].z), "r"(v[u].w)
+                       : "memory");
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(lZfull);
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while the peer may still arrive on its barriers
+  tc_fence_after();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+  }
+}
+
 }  // namespace tc
 
 // ---- host side -----------------------------------------------------------------------------
 struct TcPlan {
   TcShape s;
   CUtensorMap mZ, mE, mG1, mG2, mG3, mD1, mD2, mE4, mEB;
+  // weight maps of the CTA-pair kernels: boxes of half the output columns (128 rows)
+  CUtensorMap mG1h, mG2h, mG3h, mD1h, mD2h;
   tc::KParams pg, pgc, pd, pgt, pdt, pgram;
+  tc::PParams ppg, ppd;
   int grid_g, grid_gc, grid_d, grid_gt, grid_dt, grid_gram;
+  int ncl_g, ncl_d;        // co-resident clusters of the pair kernels (0: pair path off)
   int* err;
 };
 
@@ -673,6 +1183,89 @@ bool make_map4(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, 
   return true;
 }
 
+// Launch on clusters of two CTAs (the pairs), with programmatic dependent launch on a created
+// stream as launch_kernel does.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cudaStream_t st,
+                         Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * clusters);
+  cfg.blockDim = dim3(tc::P_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  const bool shared = st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread;
+  cfg.attrs = attr;
+  cfg.numAttrs = shared ? 1 : 2;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+// Clusters of two that can be resident at once (one CTA per SM), 0 if the query fails.
+template <typename K>
+int max_pair_clusters(K kernel, size_t smem) {
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(tc::P_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute a;
+  a.id = cudaLaunchAttributeClusterDimension;
+  a.val.clusterDim.x = 2;
+  a.val.clusterDim.y = 1;
+  a.val.clusterDim.z = 1;
+  cfg.attrs = &a;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (const void*)kernel, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+}  // namespace
+
+void tc_build_pairs(const int* nbr, int cells, int n_indiv, int B, std::vector<int4>* gpairs,
+                    std::vector<int4>* dpairs, std::vector<int2>* plist) {
+  std::vector<std::vector<int>> lists(n_indiv);  // problems (cell * 5 + slot) per individual
+  for (int i = 0; i < cells * 5; ++i) lists[nbr[i]].push_back(i);
+  gpairs->clear();
+  dpairs->clear();
+  plist->clear();
+  const int mt = (6 * B + tc::BM - 1) / tc::BM;
+  for (int k = 0; k < n_indiv; ++k) {
+    const std::vector<int>& L = lists[k];
+    if (L.empty()) continue;
+    const int off = (int)plist->size();
+    for (int pr : L) plist->push_back(make_int2(pr / 5, pr % 5));
+    const int nr = (int)L.size() * B;
+    for (int r0 = 0; r0 < nr; r0 += 2 * tc::BM) gpairs->push_back(make_int4(k, r0, off, nr));
+    std::vector<int2> tiles;  // (problem, first row)
+    for (int pr : L)
+      for (int t = 0; t < mt; ++t) tiles.push_back(make_int2(pr, t * tc::BM));
+    for (size_t i = 0; i < tiles.size(); i += 2) {
+      const int2 a = tiles[i];
+      const int2 b = i + 1 < tiles.size() ? tiles[i + 1] : make_int2(-1, 0);
+      dpairs->push_back(make_int4(k, a.x, b.x, (a.y << 16) | b.y));
+    }
+  }
+}
+
+namespace {
+bool env_flag(const char* name) {
+  const char* v = getenv(name);
+  return v && v[0] && v[0] != '0';
+}
 }  // namespace
 
 bool tc_supported(int z, int h, int x, int B) {
@@ -698,7 +1291,12 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
             make_map(&p->mG2, b.Gwb + b.goff[2], h, h, NI, h * 2, b.PGs * 2, 256, msg) &&
             make_map(&p->mG3, b.Gwb + b.goff[4], h, x, NI, h * 2, b.PGs * 2, tc::N3, msg) &&
             make_map(&p->mD1, b.Dwb + b.doff[0], x, h, NI, x * 2, b.PDs * 2, 256, msg) &&
-            make_map(&p->mD2, b.Dwb + b.doff[2], h, h, NI, h * 2, b.PDs * 2, 256, msg);
+            make_map(&p->mD2, b.Dwb + b.doff[2], h, h, NI, h * 2, b.PDs * 2, 256, msg) &&
+            make_map(&p->mG1h, b.Gwb + b.goff[0], z, h, NI, z * 2, b.PGs * 2, 128, msg) &&
+            make_map(&p->mG2h, b.Gwb + b.goff[2], h, h, NI, h * 2, b.PGs * 2, 128, msg) &&
+            make_map(&p->mG3h, b.Gwb + b.goff[4], h, x, NI, h * 2, b.PGs * 2, 128, msg) &&
+            make_map(&p->mD1h, b.Dwb + b.doff[0], x, h, NI, x * 2, b.PDs * 2, 128, msg) &&
+            make_map(&p->mD2h, b.Dwb + b.doff[2], h, h, NI, h * 2, b.PDs * 2, 128, msg);
   if (!ok) {
     delete p;
     return nullptr;
@@ -806,6 +1404,49 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   p->pd = d;
   p->pgt = gt;
   p->pdt = dt;
+  // the CTA-pair evaluation kernels (generator: z == 64, its one noise chunk gathered;
+  // first rows of discriminator tiles packed in 16 bits); LIPZ_FWD_SINGLE=1 keeps the
+  // one-CTA kernels (for comparisons)
+  tc::PParams pp{};
+  pp.B = s.B;
+  pp.x = s.x;
+  pp.n3 = g.n3;
+  pp.Z = (const bf16*)b.Z;
+  pp.E = (bf16*)b.E;
+  pp.e_cell = b.e_cell;
+  pp.logits = b.logits;
+  pp.slope = s.slope;
+  pp.err = p->err;
+  tc::PParams ppg = pp, ppd = pp;
+  ppg.rows = s.B;
+  ppg.kc1 = g.kc1;
+  ppg.wmaster = b.Gw;
+  ppg.wb = b.Gwb;
+  ppg.pstride = b.PGs;
+  ppg.off_b1 = b.goff[1];
+  ppg.off_b2 = b.goff[3];
+  ppg.off_b3 = b.goff[5];
+  ppg.off_w3 = b.goff[4];
+  ppd.rows = 6 * s.B;
+  ppd.kc1 = d.kc1;
+  ppd.wmaster = b.Dw;
+  ppd.wb = b.Dwb;
+  ppd.pstride = b.PDs;
+  ppd.off_b1 = b.doff[1];
+  ppd.off_b2 = b.doff[3];
+  ppd.off_b3 = b.doff[5];
+  ppd.off_w3 = b.doff[4];
+  p->ppg = ppg;
+  p->ppd = ppd;
+  const bool pairs_on = !env_flag("LIPZ_FWD_SINGLE");
+  p->ncl_g = pairs_on && s.z == tc::BK
+                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_G>,
+                                     tc::pair_smem_bytes<tc::KIND_G>())
+                 : 0;
+  p->ncl_d = pairs_on && 6 * s.B < 65536
+                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_D>,
+                                     tc::pair_smem_bytes<tc::KIND_D>())
+                 : 0;
   auto grid = [sms](int n) { return n < sms ? n : sms; };
   p->grid_g = grid(g.n_tiles);
   p->grid_gc = grid(gc.n_tiles);
@@ -833,13 +1474,44 @@ int launch(int grid, const CUtensorMap& a, const CUtensorMap& b1, const CUtensor
 }
 }  // namespace
 
+namespace {
+int launch_pair(int ncl, const CUtensorMap& a, const CUtensorMap& b1, const CUtensorMap& b2,
+                const CUtensorMap& b3, const tc::PParams& pp, bool gen, cudaStream_t st,
+                std::string* msg) {
+  const int clusters = pp.n_pairs < ncl ? pp.n_pairs : ncl;
+  if (clusters <= 0) return 0;
+  cudaError_t e =
+      gen ? launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_G>, clusters,
+                         (size_t)tc::pair_smem_bytes<tc::KIND_G>(), st, a, b1, b2, b3, pp)
+          : launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_D>, clusters,
+                         (size_t)tc::pair_smem_bytes<tc::KIND_D>(), st, a, b1, b2, b3, pp);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    if (msg)
+      *msg = std::string(gen ? "generator" : "discriminator") +
+             " forward (CTA pairs) launch: " + cudaGetErrorString(e);
+    return 1;
+  }
+  return 0;
+}
+}  // namespace
+
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg) {
+  if (p->ncl_g > 0 && p->ppg.pairs)
+    return launch_pair(p->ncl_g, p->mZ, p->mG1h, p->mG2h, p->mG3h, p->ppg, true, st, msg);
   return launch(p->grid_g, p->mZ, p->mG1, p->mG2, p->mG3, p->pg, st, "generator forward", msg);
 }
 
-void tc_set_nbr(TcPlan* p, const int* nbr) {
+void tc_set_nbr(TcPlan* p, const int* nbr, const TcPairs* pairs) {
   p->pg.nbr = nbr;
   p->pd.nbr = nbr;
+  p->ppg.pairs = pairs ? pairs->g : nullptr;
+  p->ppg.n_pairs = pairs ? pairs->ng : 0;
+  p->ppg.plist = pairs ? pairs->plist : nullptr;
+  p->ppd.pairs = pairs ? pairs->d : nullptr;
+  p->ppd.n_pairs = pairs ? pairs->nd : 0;
+  p->ppd.plist = pairs ? pairs->plist : nullptr;
 }
 
 int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg) {
@@ -862,6 +1534,8 @@ int tc_gram_halves(int B) { return 2 * ((6 * B + tc::HID - 1) / tc::HID); }
 bool tc_gram_supported(int B) { return B >= 32 && 6 * B + 32 <= tc::BIAS_MAX; }
 
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg) {
+  if (p->ncl_d > 0 && p->ppd.pairs)
+    return launch_pair(p->ncl_d, p->mE, p->mD1h, p->mD2h, p->mD2h, p->ppd, false, st, msg);
   return launch(p->grid_d, p->mE, p->mD1, p->mD2, p->mD2, p->pd, st, "discriminator forward",
                 msg);
 }

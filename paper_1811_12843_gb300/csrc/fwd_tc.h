@@ -8,6 +8,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <vector>
 
 namespace lipz {
 
@@ -64,8 +65,25 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg);
 // Enqueue the generator kernel (fakes of every (cell, slot)) / the discriminator kernel (logits
 // of every (cell, slot)) on `st`. 0 on success.
 int tc_run_g(TcPlan* p, cudaStream_t st, std::string* msg);
-// Neighbour table [cells][5] (individual indices) that the next evaluation runs read.
-void tc_set_nbr(TcPlan* p, const int* nbr);
+// Work lists of the CTA-pair evaluation kernels for one neighbour table (device arrays built
+// by tc_build_pairs): generator pairs g[ng], discriminator pairs d[nd], and the (cell, slot)
+// problems of every individual (plist) they index.
+struct TcPairs {
+  const int4* g;
+  int ng;
+  const int4* d;
+  int nd;
+  const int2* plist;
+};
+// Host side of TcPairs for the neighbour table nbr [cells][5] (individual indices < n_indiv):
+// per individual its problems in table order; generator pairs {individual, first row of the
+// pair's 256, plist offset, rows = problems x B}; discriminator pairs {individual, problem of
+// the first CTA, problem of the second (-1: none), first rows packed (first << 16 | second)}.
+void tc_build_pairs(const int* nbr, int cells, int n_indiv, int B, std::vector<int4>* gpairs,
+                    std::vector<int4>* dpairs, std::vector<int2>* plist);
+// Neighbour table [cells][5] (individual indices) that the next evaluation runs read, and its
+// pair lists (null: the one-CTA kernels run).
+void tc_set_nbr(TcPlan* p, const int* nbr, const TcPairs* pairs);
 // Generator forward of every cell's own centre on its z, into E's slot-0 fakes.
 int tc_run_g_centre(TcPlan* p, cudaStream_t st, std::string* msg);
 int tc_run_d(TcPlan* p, cudaStream_t st, std::string* msg);

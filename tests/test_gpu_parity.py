@@ -499,3 +499,31 @@ def test_k_minibatch_steps_need_the_pool(L):
     with pytest.raises(L.LipzError) as e:
         L.lipz_iterate_batch(g.h, x, fg, fd)
     assert e.value.code == L.LIPZ_ERR_STATE and "pool" in str(e.value)
+
+
+@pytest.mark.parametrize("rows,cols,batch,stale", [(3, 3, 100, 0), (2, 2, 129, 0), (1, 1, 37, 0),
+                                                   (3, 4, 100, 1), (12, 12, 100, 0)])
+def test_pair_kernels_equal_one_cta_kernels(L, monkeypatch, rows, cols, batch, stale):
+    """The evaluation runs on CTA pairs (two SMs share each weight chunk, M = 256 per MMA);
+    LIPZ_FWD_SINGLE=1 at grid creation keeps the one-CTA kernels (M = 128). Both accumulate
+    every output in the same order, so the logits, the fitness and the whole iteration agree
+    bit for bit: duplicated neighbours (2x2, 1x1), ragged batches and stale neighbours (an
+    individual in one or four problems) included."""
+    pool = _pool(21, 4000, 784)
+    kw = dict(precision="bf16", batch=batch, stale_neighbors=stale)
+    a = _grid(L, rows, cols, 5, pool, **kw)
+    monkeypatch.setenv("LIPZ_FWD_SINGLE", "1")
+    b = _grid(L, rows, cols, 5, pool, **kw)
+    monkeypatch.delenv("LIPZ_FWD_SINGLE")
+    for it in range(3):
+        ea, eb = a.eval(pairs=True), b.eval(pairs=True)
+        assert np.array_equal(a.logits(), b.logits()), it
+        for k in ("LG", "LD", "fG", "fD"):
+            assert np.array_equal(ea[k], eb[k]), (it, k)
+        xa, _ = a.batch()
+        assert np.all(np.isfinite(xa))
+        a.select()
+        b.select()
+        a.train()
+        b.train()
+    assert a.export_state() == b.export_state()
