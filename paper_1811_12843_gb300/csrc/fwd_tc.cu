@@ -21,6 +21,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <vector>
@@ -141,6 +142,20 @@ __device__ __forceinline__ int prob_individual(const KParams& p, int prob) {
   if (p.train) return __ldg(&p.wsel[p.part_slot ? prob >> 1 : prob]);
   if (KND == KIND_GRAM) return prob;
   return p.centre ? p.indiv_off + prob : __ldg(&p.nbr[prob]);
+}
+
+// tanh from its definition, tanh(x) = 1 - 2 / (1 + e^(2x)), with e^(2x) by the hardware base-2
+// exponential, for |x| >= 1/16; below that the Taylor series x - x^3/3 + 2x^5/15 (truncation
+// error under 17 x^7 / 315, relative below 3e-9). Relative error below 1e-5 everywhere (the
+// cancellation in 1 - 2/(1 + e) is largest at |x| = 1/16); |x| is clamped at 16, where the
+// fp32 value is 1.
+__device__ __forceinline__ float tanh_fast(float x) {
+  const float ax = fminf(fabsf(x), 16.f);
+  const float e = ex2_approx(2.8853900817779268f * ax);  // e^(2|x|): 2 log2(e) |x|
+  const float t = 1.f - __fdividef(2.f, 1.f + e);
+  const float x2 = ax * ax;
+  const float s = ax * fmaf(x2, fmaf(x2, 0.13333333333333333f, -0.33333333333333333f), 1.f);
+  return copysignf(ax < 0.0625f ? s : t, x);
 }
 
 // ---- the kernel ----------------------------------------------------------------------------
@@ -582,8 +597,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t pk[8];
 #pragma unroll
             for (int e = 0; e < 16; e += 2)
-              pk[e >> 1] = pack_bf16(tanhf(__uint_as_float(r[e]) + bv[e]),
-                                     tanhf(__uint_as_float(r[e + 1]) + bv[e + 1]));
+              pk[e >> 1] = pack_bf16(tanh_fast(__uint_as_float(r[e]) + bv[e]),
+                                     tanh_fast(__uint_as_float(r[e + 1]) + bv[e + 1]));
             if (rr < p.B && col0 < p.x) {
               uint4* o = reinterpret_cast<uint4*>(dst + col0);
               o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
@@ -619,22 +634,26 @@ __global__ void __launch_bounds__(THREADS, 1)
 //   discriminator: two 128-row tiles of (cell, slot) problems that share the individual (a
 //              lone tile's partner computes zeros and stores nothing).
 constexpr int HB_BYTES = (HID / 2) * BK * 2;  // 16 KB: half of a 256-row weight box
-constexpr int NUM_PWARPS = 2 + NUM_EPI_WARPS + 1;
-constexpr int P_THREADS = 32 * NUM_PWARPS;
-constexpr int PAIR_EPI_ARRIVALS = 2 * NUM_EPI_WARPS;  // one per epilogue warp of both CTAs
 
 template <int KND>
 struct PCfg;
-// generator: rings of weight halves only (its first layer's A is the gathered noise tile)
+// generator: rings of weight halves only (its first layer's A is the gathered noise tile);
+// sixteen epilogue warps (its output epilogue, tanh and the fakes' stores, is the longest)
 template <>
 struct PCfg<KIND_G> {
-  static constexpr int STAGES = 8, STAGE = HB_BYTES, A_IN = 0, ZBUF = A_BYTES;
+  static constexpr int STAGES = 8, STAGE = HB_BYTES, A_IN = 0, ZBUF = A_BYTES, NE = 16;
 };
-// discriminator: each stage holds the A chunk and the weight half
+// discriminator: each stage holds the A chunk and the weight half; eight epilogue warps (two
+// column halves: the logit's two partial dot products are added in the one-CTA kernel's order)
 template <>
 struct PCfg<KIND_D> {
-  static constexpr int STAGES = 4, STAGE = A_BYTES + HB_BYTES, A_IN = 1, ZBUF = 0;
+  static constexpr int STAGES = 4, STAGE = A_BYTES + HB_BYTES, A_IN = 1, ZBUF = 0, NE = 8;
 };
+// warps: producer, MMA issuer, NE epilogue warps, noise gather
+template <int KND>
+constexpr int pair_threads() {
+  return 32 * (3 + PCfg<KND>::NE);
+}
 template <int KND>
 constexpr int pair_smem_bytes() {
   return 1024 + PCfg<KND>::STAGES * PCfg<KND>::STAGE + PCfg<KND>::ZBUF + H_BYTES + MISC_BYTES +
@@ -675,11 +694,14 @@ __device__ __forceinline__ Job pair_job(const PParams& p, int j) {
 }
 
 template <int KND>
-__global__ void __launch_bounds__(P_THREADS, 1)
+__global__ void __launch_bounds__(pair_threads<KND>(), 1)
     k_mlp_fwd_pair(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB1,
                    const __grid_constant__ CUtensorMap mB2, const __grid_constant__ CUtensorMap mB3,
                    const PParams p) {
   using CF = PCfg<KND>;
+  constexpr int NE = CF::NE;               // epilogue warps
+  constexpr int CP = NE / 4;               // column parts (warps per TMEM lane quarter)
+  constexpr int ARRIVALS = 2 * NE;         // one per epilogue warp of both CTAs
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -702,7 +724,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
   float* s_bias = reinterpret_cast<float*>(misc + MISC_BYTES);
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 256);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 260);
-  float* part = reinterpret_cast<float*>(misc + 512);
+  float* part_buf = reinterpret_cast<float*>(misc + 512);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
@@ -714,11 +736,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     }
     for (int r = 0; r < 2; ++r) {
       mbar_init(bAcc + 8 * r, 1);
-      mbar_init(bReg + 8 * r, PAIR_EPI_ARRIVALS);
-      mbar_init(bBias + 8 * r, 32 * NUM_EPI_WARPS);
+      mbar_init(bReg + 8 * r, ARRIVALS);
+      mbar_init(bBias + 8 * r, 32 * NE);
     }
-    for (int c = 0; c < HID / BK; ++c) mbar_init(bH + 8 * c, PAIR_EPI_ARRIVALS);
-    mbar_init(bPart, 32 * NUM_EPI_WARPS / 2);
+    for (int c = 0; c < HID / BK; ++c) mbar_init(bH + 8 * c, ARRIVALS);
+    mbar_init(bPart, 32 * NE / 2);
     mbar_init(bFinal, 1);
     mbar_init(bZfull, 2);
     mbar_init(bZempty, 1);
@@ -805,12 +827,12 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           const Job J = pair_job<KND>(p, j);
           const int R = J.region;
           if (reg_uses[R] > 0 &&
-              !mbar_wait_cl(bReg + 8 * R, (uint32_t)((reg_uses[R] - 1) & 1), abort_flag, p.err, 2)) {
+              !mbar_wait(bReg + 8 * R, (uint32_t)((reg_uses[R] - 1) & 1), abort_flag, p.err, 2)) {
             ok = false;
             break;
           }
           if (KND == KIND_G && j == 0 &&
-              !mbar_wait_cl(bZfull, (uint32_t)(zuse & 1), abort_flag, p.err, 9)) {
+              !mbar_wait(bZfull, (uint32_t)(zuse & 1), abort_flag, p.err, 9)) {
             ok = false;
             break;
           }
@@ -819,11 +841,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
           const uint32_t idesc = idesc_bf16(2 * BM, J.n);
           for (int kc = 0; kc < J.kchunks; ++kc) {
             if (J.a_from_h &&
-                !mbar_wait_cl(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
+                !mbar_wait(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
               ok = false;
               break;
             }
-            if (!mbar_wait_cl(bFull + 8 * stage, phase, abort_flag, p.err, 4)) {
+            if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 4)) {
               ok = false;
               break;
             }
@@ -858,22 +880,23 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, p.err, 5);
     }
-  } else if (warp < 2 + NUM_EPI_WARPS) {
+  } else if (warp < 2 + NE) {
     // ================================ epilogue (own 128 rows) ================================
     const int ew = warp - 2;
-    const int q = warp & 3;
-    const int hf = ew >> 2;
+    const int q = warp & 3;          // TMEM lane quarter this warp may access
+    const int part = ew >> 2;        // column part: HID / CP columns of every region
     const int row = q * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const int et = threadIdx.x - 64;
     int reg_uses[2] = {0, 0};
     bool ok = true;
     int ltile = 0;
-    // a warp's share of a region, an H chunk: its lanes' writes are done (and, for H, made
-    // visible to the tensor cores) before lane 0 arrives on rank 0's barrier
-    auto warp_arrive = [&](uint32_t bar_cluster) {
+    // a warp's share is done (tensor memory read; for H chunks the rows written and made
+    // visible to the tensor cores by every lane's proxy fence): lane 0 arrives on rank 0's
+    // barrier. The H chunk is this CTA's own shared memory, read by this SM's tensor core.
+    auto warp_signal = [&](uint32_t bar_cluster) {
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(bar_cluster);
+      if (lane == 0) mbar_arrive_remote(bar_cluster);
     };
     for (int pi = cid; pi < p.n_pairs && ok; pi += ncl, ++ltile) {
       const int4 pr = __ldg(&p.pairs[pi]);
@@ -899,11 +922,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
       {
         const int nb3 = KND == KIND_D ? HID + 1 : p.x;
-        constexpr int NV = (BIAS_MAX + 32 * NUM_EPI_WARPS - 1) / (32 * NUM_EPI_WARPS);
+        constexpr int NV = (BIAS_MAX + 32 * NE - 1) / (32 * NE);
         float v[NV];
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
-          const int i = et + u * 32 * NUM_EPI_WARPS;
+          const int i = et + u * 32 * NE;
           v[u] = 0.f;
           if (i >= 512 + nb3) continue;
           if (i < 256) v[u] = wm[p.off_b1 + i];
@@ -916,7 +939,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         }
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
-          const int i = et + u * 32 * NUM_EPI_WARPS;
+          const int i = et + u * 32 * NE;
           if (i < 512 + nb3) sb[i] = v[u];
         }
         mbar_arrive(bBias + 8 * (ltile & 1));
@@ -929,25 +952,32 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       for (int j = 0; j < nj && ok; ++j) {
         const Job J = pair_job<KND>(p, j);
         const int R = J.region;
-        if (!mbar_wait_cl_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
+        if (!mbar_wait_warp(bAcc + 8 * R, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 6)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t tbase = tmem + lane_base + (uint32_t)(R * HID);
         if (J.epi == EPI_TO_H) {
+          // chunk by chunk (64 columns; this warp's 64 / CP of each), so that the next layer
+          // starts on chunk 0 while the others are written
           const float* bias = sb + (j == 0 ? 0 : 256);
           const float lo = KND == KIND_D ? p.slope : 0.f;
+          constexpr int W = BK / CP;  // columns of a chunk per warp: 32 or 16
 #pragma unroll 1
           for (int ch = 0; ch < HID / BK; ++ch) {
-            const int cg = 2 * ch + hf;
-            uint32_t r[32];
-            LIPZ_TMEM_LD32(tbase + cg * 32, r);
+            const int col0 = ch * BK + part * W;
+            uint32_t r[W];
+            if (W == 32) {
+              LIPZ_TMEM_LD32(tbase + col0, r);
+            } else {
+              LIPZ_TMEM_LD16(tbase + col0, r);
+            }
             tmem_wait_ld();
-            const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
-            uint32_t pk[16];
+            const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
+            uint32_t pk[W / 2];
 #pragma unroll
-            for (int e = 0; e < 32; e += 4) {
+            for (int e = 0; e < W; e += 4) {
               const float4 bb = b4[e >> 2];
               float a0 = __uint_as_float(r[e]) + bb.x;
               float a1 = __uint_as_float(r[e + 1]) + bb.y;
@@ -962,24 +992,26 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             }
             const uint32_t chunk = sH + (uint32_t)(ch * H_CHUNK) + (uint32_t)row * 128u;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const uint32_t unit = (uint32_t)(hf * 4 + u);
+            for (int u = 0; u < W / 8; ++u) {
+              const uint32_t unit = (uint32_t)(part * (W / 8) + u);
               const uint32_t addr = chunk + ((unit ^ (uint32_t)(row & 7)) << 4);
               asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[4 * u]),
                            "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]), "r"(pk[4 * u + 3])
                            : "memory");
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            warp_arrive(lH + 8 * ch);
+            warp_signal(lH + 8 * ch);
           }
           tc_fence_before();
-          warp_arrive(lReg + 8 * R);
-        } else if (J.epi == EPI_LOGIT) {
+          warp_signal(lReg + 8 * R);
+        } else if (KND == KIND_D && J.epi == EPI_LOGIT) {
+          // LeakyReLU of layer 2, rounded to bf16, dotted with the output weights: each column
+          // half's partial dot product, the halves added as in the one-CTA kernel
           const float* bias = sb + 256;
           const float* w3 = sb + 512;
           float acc = 0.f;
 #pragma unroll 1
-          for (int cp = hf * 4; cp < hf * 4 + 4; cp += 2) {
+          for (int cp = part * 4; cp < part * 4 + 4; cp += 2) {
             uint32_t r2[2][32];
             LIPZ_TMEM_LD32(tbase + cp * 32, r2[0]);
             LIPZ_TMEM_LD32(tbase + (cp + 1) * 32, r2[1]);
@@ -1012,25 +1044,26 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             }
           }
           tc_fence_before();
-          if (hf == 1) {
-            part[row] = acc;
+          if (part == 1) {
+            part_buf[row] = acc;
             mbar_arrive(bPart);
-            warp_arrive(lReg + 8 * R);
+            warp_signal(lReg + 8 * R);
           } else {
             if (!mbar_wait_warp(bPart, (uint32_t)(reg_uses[R] & 1), abort_flag, p.err, 7)) {
               ok = false;
               break;
             }
-            const float logit = acc + part[row] + sb[512 + HID];
-            warp_arrive(lReg + 8 * R);
+            const float logit = acc + part_buf[row] + sb[512 + HID];
+            warp_signal(lReg + 8 * R);
             if (row_ok) p.logits[lidx] = logit;
           }
-        } else {
-          // generator output block: bias + tanh, bf16, into this row's fakes
+        } else if (KND == KIND_G) {
+          // generator output block: bias + tanh, bf16, into this row's fakes; this warp's
+          // share of the block's 16-column groups
           const float* bias = sb + 512;
           const int ng = J.n / 16;
-          const int split = (ng + 1) / 2;
-          const int g0 = hf ? split : 0, g1 = hf ? ng : split;
+          const int per = (ng + CP - 1) / CP;
+          const int g0 = part * per, g1 = min(ng, g0 + per);
 #pragma unroll 1
           for (int gi = g0; gi < g1; ++gi) {
             uint32_t r[16];
@@ -1042,10 +1075,10 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 #pragma unroll
             for (int qq = 0; qq < 4; ++qq) {
               const float4 t = b4[qq];
-              pk[2 * qq] = pack_bf16(tanhf(__uint_as_float(r[4 * qq]) + t.x),
-                                     tanhf(__uint_as_float(r[4 * qq + 1]) + t.y));
-              pk[2 * qq + 1] = pack_bf16(tanhf(__uint_as_float(r[4 * qq + 2]) + t.z),
-                                         tanhf(__uint_as_float(r[4 * qq + 3]) + t.w));
+              pk[2 * qq] = pack_bf16(tanh_fast(__uint_as_float(r[4 * qq]) + t.x),
+                                     tanh_fast(__uint_as_float(r[4 * qq + 1]) + t.y));
+              pk[2 * qq + 1] = pack_bf16(tanh_fast(__uint_as_float(r[4 * qq + 2]) + t.z),
+                                         tanh_fast(__uint_as_float(r[4 * qq + 3]) + t.w));
             }
             if (row_ok && col0 < p.x) {
               uint4* o = reinterpret_cast<uint4*>(dst + col0);
@@ -1054,7 +1087,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             }
           }
           tc_fence_before();
-          warp_arrive(lReg + 8 * R);
+          warp_signal(lReg + 8 * R);
         }
         reg_uses[R]++;
       }
@@ -1066,7 +1099,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     for (int pi = cid; pi < p.n_pairs; pi += ncl, ++zuse) {
       const int4 pr = __ldg(&p.pairs[pi]);
       if (zuse > 0 &&
-          !mbar_wait_cl_warp(bZempty, (uint32_t)((zuse - 1) & 1), abort_flag, p.err, 10))
+          !mbar_wait_warp(bZempty, (uint32_t)((zuse - 1) & 1), abort_flag, p.err, 10))
         break;
       const int row0 = pr.y + (int)rank * BM;
 #pragma unroll 1
@@ -1097,7 +1130,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(lZfull);
+      if (lane == 0) mbar_arrive_remote(lZfull);
     }
   }
 
@@ -1186,11 +1219,11 @@ bool make_map4(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, 
 // Launch on clusters of two CTAs (the pairs), with programmatic dependent launch on a created
 // stream as launch_kernel does.
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cudaStream_t st,
-                         Args... args) {
+cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, int threads, size_t smem,
+                         cudaStream_t st, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * clusters);
-  cfg.blockDim = dim3(tc::P_THREADS);
+  cfg.blockDim = dim3(threads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
@@ -1208,7 +1241,7 @@ cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cu
 
 // Clusters of two that can be resident at once (one CTA per SM), 0 if the query fails.
 template <typename K>
-int max_pair_clusters(K kernel, size_t smem) {
+int max_pair_clusters(K kernel, int threads, size_t smem) {
   if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
       cudaSuccess) {
     cudaGetLastError();
@@ -1216,7 +1249,7 @@ int max_pair_clusters(K kernel, size_t smem) {
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2);
-  cfg.blockDim = dim3(tc::P_THREADS);
+  cfg.blockDim = dim3(threads);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute a;
   a.id = cudaLaunchAttributeClusterDimension;
@@ -1440,13 +1473,16 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   p->ppd = ppd;
   const bool pairs_on = !env_flag("LIPZ_FWD_SINGLE");
   p->ncl_g = pairs_on && s.z == tc::BK
-                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_G>,
+                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_G>, tc::pair_threads<tc::KIND_G>(),
                                      tc::pair_smem_bytes<tc::KIND_G>())
                  : 0;
   p->ncl_d = pairs_on && 6 * s.B < 65536
-                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_D>,
+                 ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_D>, tc::pair_threads<tc::KIND_D>(),
                                      tc::pair_smem_bytes<tc::KIND_D>())
                  : 0;
+  if (env_flag("LIPZ_VERBOSE"))
+    fprintf(stderr, "lipz: tensor-core forward: %d SMs, CTA-pair clusters resident: generator %d, "
+            "discriminator %d\n", sms, p->ncl_g, p->ncl_d);
   auto grid = [sms](int n) { return n < sms ? n : sms; };
   p->grid_g = grid(g.n_tiles);
   p->grid_gc = grid(gc.n_tiles);
@@ -1481,9 +1517,9 @@ int launch_pair(int ncl, const CUtensorMap& a, const CUtensorMap& b1, const CUte
   const int clusters = pp.n_pairs < ncl ? pp.n_pairs : ncl;
   if (clusters <= 0) return 0;
   cudaError_t e =
-      gen ? launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_G>, clusters,
+      gen ? launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_G>, clusters, tc::pair_threads<tc::KIND_G>(),
                          (size_t)tc::pair_smem_bytes<tc::KIND_G>(), st, a, b1, b2, b3, pp)
-          : launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_D>, clusters,
+          : launch_pairs(tc::k_mlp_fwd_pair<tc::KIND_D>, clusters, tc::pair_threads<tc::KIND_D>(),
                          (size_t)tc::pair_smem_bytes<tc::KIND_D>(), st, a, b1, b2, b3, pp);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
