@@ -821,6 +821,7 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
       uint32_t phase = 0;
       int reg_uses[2] = {0, 0};
       int h_total = 0, zuse = 0;
+      int h_seen[HID / BK] = {0, 0, 0, 0};  // activation write each chunk was last waited for
       bool ok = true;
       for (int pi = cid; pi < p.n_pairs && ok; pi += ncl) {
         for (int j = 0; j < nj && ok; ++j) {
@@ -840,10 +841,13 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
           const uint32_t d = tmem + (uint32_t)(R * HID);
           const uint32_t idesc = idesc_bf16(2 * BM, J.n);
           for (int kc = 0; kc < J.kchunks; ++kc) {
-            if (J.a_from_h &&
-                !mbar_wait(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
-              ok = false;
-              break;
+            // (the generator's output blocks read the same activation: wait for it once)
+            if (J.a_from_h && h_seen[kc] != h_total) {
+              if (!mbar_wait(bH + 8 * kc, (uint32_t)((h_total - 1) & 1), abort_flag, p.err, 3)) {
+                ok = false;
+                break;
+              }
+              h_seen[kc] = h_total;
             }
             if (!mbar_wait(bFull + 8 * stage, phase, abort_flag, p.err, 4)) {
               ok = false;
