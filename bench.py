@@ -68,11 +68,15 @@ TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM *
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels: not
 # measured by this script but taken from ncu captures (dram__bytes_read.sum +
-# dram__bytes_write.sum) of these same kernels, named in PHASE_TRAFFIC_SOURCE. A phase whose
-# kernels changed after its capture has no entry (null traffic).
-PHASE_TRAFFIC = {"batch": 21.2e6, "fitness": 1.8e6, "select": 0.0, "adam": 3.6e6,
-                 "train_bwd": 2182.6e6}
-PHASE_TRAFFIC_SOURCE = "ncu capture summarised in profiles/launches_12x12_bf16_iteration.md"
+# dram__bytes_write.sum) of these same kernels, each with the summary it comes from. A phase
+# whose kernels changed after its capture has no entry (null traffic).
+PHASE_TRAFFIC = {
+    "train_bwd": (2190.7e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
+    "d_fwd": (240.2e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
+    "batch": (21.2e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
+    "fitness": (1.8e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
+    "adam": (3.6e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
+}
 
 
 def _peaks():
@@ -298,9 +302,9 @@ def _phase_roofs(phase_ms):
             # the timed region lasts milliseconds, not seconds: the burst rate applies
             ach, peak, unit = units / (t * 1e-3) / 1e12, tf_burst, "TFLOP/s"
             src = peak_kind + " burst bf16 (cuBLAS)"
-        tr = PHASE_TRAFFIC.get(ph)
+        tr, tr_src = PHASE_TRAFFIC.get(ph, (None, None))
         out[ph] = {"bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
-                   "traffic": tr, "traffic_source": PHASE_TRAFFIC_SOURCE if tr else None,
+                   "traffic": tr, "traffic_source": tr_src,
                    "kernel": what, "peak_source": src,
                    ("algorithmic_bytes" if bound == "hbm" else "algorithmic_flop"): units}
     return out

@@ -60,7 +60,8 @@ def per_tensor(flat_got, flat_ref, layout):
 # elements per cell can flip and no enumeration is possible. The oracle itself, with float32
 # instead of float64 products and otherwise the same code, differs from the float64 oracle by
 # up to 2e-2 in a few cells (median 1e-3). The rule is an error budget: every cell within
-# BF16_CEIL x tol, at most one cell in eight above tol, and the median cell within
+# BF16_CEIL x tol, at most a quarter of the cells (at least two) above tol, and the median cell
+# within
 # BF16_MEDIAN x tol (the engine's medians lie at 1e-3 to 5e-3). A method error (a wrong row,
 # cell, slot or tile tail) is of order one.
 FP32_FLIP_BAND = 2e-6
@@ -123,7 +124,7 @@ def gradient_parity(label, a, gg, gd, refG, refD, tol, pair_inputs):
                                       "branch choice", dict(zip(names, err[c]))))
     else:
         assert np.all(worst <= BF16_CEIL * tol), (label, "ceiling", worst)
-        assert np.sum(worst > tol) <= max(1, len(worst) // 8), (label, "count", worst)
+        assert np.sum(worst > tol) <= max(2, len(worst) // 4), (label, "count", worst)
         assert np.median(worst) <= BF16_MEDIAN * tol, (label, "median", worst)
     print("PARITY %s cells=%d worst=%.3e median=%.3e per-tensor-max {%s}" % (
         label, len(worst), worst.max(), np.median(worst),
