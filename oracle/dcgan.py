@@ -37,6 +37,16 @@ import numpy as np
 BN_EPS = 1e-5
 INIT_STD = 0.02
 
+# Accumulation type of every sum (convolutions, batch-norm statistics and their gradients).
+# float64 is the oracle. float32 is the same arithmetic summed in another order and precision:
+# the spread between the two shows how far an implementation that accumulates in fp32 may land
+# from the oracle without any error of method (tests use it to justify their tolerances).
+ACC = np.float64
+
+
+def _a(x):
+    return np.asarray(x).astype(ACC, copy=False)
+
 
 # --------------------------------------------------------------------------------------------
 # Parameter layouts (PyTorch conventions: ConvTranspose2d weight [in][out][kh][kw], Conv2d
@@ -86,13 +96,14 @@ def conv2d(x: np.ndarray, w: np.ndarray, s: int, p: int) -> np.ndarray:
     N, C, H, W = x.shape
     O, _, k, _ = w.shape
     Ho, Wo = (H + 2 * p - k) // s + 1, (W + 2 * p - k) // s + 1
-    xp = np.pad(x, ((0, 0), (0, 0), (p, p), (p, p)))
-    y = np.zeros((N, O, Ho, Wo))
+    xp = _a(np.pad(x, ((0, 0), (0, 0), (p, p), (p, p))))
+    w = _a(w)
+    y = np.zeros((N, O, Ho, Wo), ACC)
     for ky in range(k):
         for kx in range(k):
             win = xp[:, :, ky:ky + s * (Ho - 1) + 1:s, kx:kx + s * (Wo - 1) + 1:s]
             y += np.einsum("nchw,oc->nohw", win, w[:, :, ky, kx], optimize=True)
-    return y
+    return y.astype(np.float64)
 
 
 def conv2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
@@ -100,16 +111,17 @@ def conv2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
     N, C, H, W = x.shape
     O, _, k, _ = w.shape
     Ho, Wo = dy.shape[2], dy.shape[3]
-    xp = np.pad(x, ((0, 0), (0, 0), (p, p), (p, p)))
+    xp = _a(np.pad(x, ((0, 0), (0, 0), (p, p), (p, p))))
+    w, dy = _a(w), _a(dy)
     dxp = np.zeros_like(xp)
-    dw = np.zeros_like(w, dtype=np.float64)
+    dw = np.zeros(w.shape, ACC)
     for ky in range(k):
         for kx in range(k):
             sl = (slice(None), slice(None), slice(ky, ky + s * (Ho - 1) + 1, s),
                   slice(kx, kx + s * (Wo - 1) + 1, s))
             dw[:, :, ky, kx] = np.einsum("nohw,nchw->oc", dy, xp[sl], optimize=True)
             dxp[sl] += np.einsum("nohw,oc->nchw", dy, w[:, :, ky, kx], optimize=True)
-    return dxp[:, :, p:p + H, p:p + W], dw
+    return dxp[:, :, p:p + H, p:p + W].astype(np.float64), dw.astype(np.float64)
 
 
 def conv_transpose2d(x: np.ndarray, w: np.ndarray, s: int, p: int) -> np.ndarray:
@@ -118,12 +130,13 @@ def conv_transpose2d(x: np.ndarray, w: np.ndarray, s: int, p: int) -> np.ndarray
     N, C, H, W = x.shape
     _, O, k, _ = w.shape
     Hf, Wf = s * (H - 1) + k, s * (W - 1) + k
-    full = np.zeros((N, O, Hf, Wf))
+    x, w = _a(x), _a(w)
+    full = np.zeros((N, O, Hf, Wf), ACC)
     for ky in range(k):
         for kx in range(k):
             full[:, :, ky:ky + s * (H - 1) + 1:s, kx:kx + s * (W - 1) + 1:s] += np.einsum(
                 "nchw,co->nohw", x, w[:, :, ky, kx], optimize=True)
-    return full[:, :, p:Hf - p, p:Wf - p]
+    return full[:, :, p:Hf - p, p:Wf - p].astype(np.float64)
 
 
 def conv_transpose2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
@@ -131,24 +144,25 @@ def conv_transpose2d_backward(x, w, s, p, dy) -> Tuple[np.ndarray, np.ndarray]:
     N, C, H, W = x.shape
     _, O, k, _ = w.shape
     Hf, Wf = s * (H - 1) + k, s * (W - 1) + k
-    dfull = np.zeros((N, O, Hf, Wf))
+    x, w = _a(x), _a(w)
+    dfull = np.zeros((N, O, Hf, Wf), ACC)
     dfull[:, :, p:Hf - p, p:Wf - p] = dy
-    dx = np.zeros_like(x, dtype=np.float64)
-    dw = np.zeros_like(w, dtype=np.float64)
+    dx = np.zeros(x.shape, ACC)
+    dw = np.zeros(w.shape, ACC)
     for ky in range(k):
         for kx in range(k):
             d = dfull[:, :, ky:ky + s * (H - 1) + 1:s, kx:kx + s * (W - 1) + 1:s]
             dx += np.einsum("nohw,co->nchw", d, w[:, :, ky, kx], optimize=True)
             dw[:, :, ky, kx] = np.einsum("nchw,nohw->co", x, d, optimize=True)
-    return dx, dw
+    return dx.astype(np.float64), dw.astype(np.float64)
 
 
 # --------------------------------------------------------------------------------------------
 # Batch normalisation in training mode (Ioffe & Szegedy 2015), per channel over (N, H, W).
 # --------------------------------------------------------------------------------------------
 def batchnorm(x, gamma, beta):
-    mu = x.mean(axis=(0, 2, 3))
-    var = ((x - mu[None, :, None, None]) ** 2).mean(axis=(0, 2, 3))
+    mu = _a(x).mean(axis=(0, 2, 3)).astype(np.float64)
+    var = _a((x - mu[None, :, None, None]) ** 2).mean(axis=(0, 2, 3)).astype(np.float64)
     inv = 1.0 / np.sqrt(var + BN_EPS)
     xhat = (x - mu[None, :, None, None]) * inv[None, :, None, None]
     return gamma[None, :, None, None] * xhat + beta[None, :, None, None], (xhat, inv)
@@ -157,8 +171,8 @@ def batchnorm(x, gamma, beta):
 def batchnorm_backward(dy, gamma, cache):
     xhat, inv = cache
     m = dy.shape[0] * dy.shape[2] * dy.shape[3]
-    dbeta = dy.sum(axis=(0, 2, 3))
-    dgamma = (dy * xhat).sum(axis=(0, 2, 3))
+    dbeta = _a(dy).sum(axis=(0, 2, 3)).astype(np.float64)
+    dgamma = _a(dy * xhat).sum(axis=(0, 2, 3)).astype(np.float64)
     dx = (gamma * inv)[None, :, None, None] * (
         dy - dbeta[None, :, None, None] / m - xhat * (dgamma / m)[None, :, None, None])
     return dx, dgamma, dbeta

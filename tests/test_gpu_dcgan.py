@@ -1,14 +1,15 @@
 """GPU parity of the DCGAN networks (Table 1, CelebA column) against the oracle: the
 initialisation, the evaluation of every (cell, slot) pair and one training step of every
-cell's selected pair, at small widths in fp32 and bf16 (1e-4 / 2e-2 max-norm relative), and
-sampled outputs of the 3x3, width-64, B = 128 configuration."""
+cell's selected pair, in fp32 and bf16 at widths 4 and 64 (1e-4 / 2e-2 max-norm relative, or
+2.5 times the oracle's own float32-vs-float64 spread where batch norm makes that larger), and
+one full cell of the 3x3, width-64, B = 128 configuration."""
 
 import numpy as np
 import pytest
 
 from oracle import lipz_oracle as O
 
-from helpers import max_rel, oracle_arch, per_tensor
+from helpers import cell_errors, max_rel, oracle_arch
 
 pytestmark = pytest.mark.gpu
 
@@ -88,31 +89,52 @@ def test_dcgan_tensor_core_eval(L, rows, cols, batch, ngf):
         assert max_rel(ev[k], ref[k]) < 2e-2, k
 
 
+def _spread(a, pairs):
+    """Per cell, the oracle's own spread: the max-norm relative difference (worst tensor)
+    between its gradients with float32 and with float64 accumulation, on the same inputs.
+    pairs: [(G params, D params, x, z, float64 gradients (gG, gD))]."""
+    from oracle import dcgan as DC
+    gl, dl = O.g_layout(a), O.d_layout(a)
+    out = []
+    try:
+        DC.ACC = np.float32
+        for Gf, Df, x, z, (rG, rD) in pairs:
+            fG, fD, _ = O.pair_gradients(Gf, Df, x, z, a)
+            out.append(max(cell_errors(fG[None], rG[None], gl).max(),
+                           cell_errors(fD[None], rD[None], dl).max()))
+    finally:
+        DC.ACC = np.float64
+    return np.array(out)
+
+
+SPREAD_FACTOR = 2.5
+
+
 @pytest.mark.parametrize("precision,width,rows,cols,batch", [("fp32", 4, 2, 2, 4),
                                                             ("bf16", 4, 2, 2, 4),
+                                                            ("fp32", 64, 1, 2, 16),
                                                             ("bf16", 64, 1, 2, 16),
                                                             ("bf16", (128, 64), 1, 1, 16)])
 def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
-    """Selection bit-exact given the engine's fitness; then the last step's gradients and the
-    Adam state per cell against the oracle (a cell whose pre-activations came within rounding
-    distance of a kink is excused, as in the MLP checks). Width 64 in bf16 runs the training
-    forward on the tensor-core kernel with channel-last activations. At that width every cell
-    has pre-activations within 1e-8 of a kink, and batch normalisation's backward spreads a
-    flipped derivative over the whole channel: the CUDA-core and the tensor-core paths both
-    reach 1.4-4.7 % there (B = 16), so that case is held to 7.5 % per cell and 5 % median.
-    A generator twice as wide (ngf 128, ndf 64) takes the kernel variants the width-64 case
-    does not: the output layer by parity class, and the wide first-layer variant for the
-    generator's input gradient. Its single cell lands at 6.9 % with the tensor cores and 6.8 %
-    with the CUDA-core kernels (measured side by side on the same inputs; the two differ from
-    each other by 7 %), so it is held to the 7.5 % per-cell rule only."""
+    """Selection bit-exact given the engine's fitness; then the gradients and the first moments
+    of every cell's trained pair against the oracle. Rule, per cell: the worst tensor within
+    max(tol, 2.5 x the oracle's own spread), the spread being the difference between the
+    oracle with float32 and with float64 accumulation on the same pair and minibatch. Batch
+    normalisation's backward spreads a ReLU derivative that flips at a pre-activation near 0
+    over the whole channel, so summation order alone moves these gradients: at width 64 the
+    oracle's spread is 0.2-0.6 % in fp32 and 4-5 % in bf16 (B = 16), at width 4 it is at the
+    rounding level and the tolerance (1e-4 / 2e-2) binds. Width 64 in bf16 runs the training
+    on the tensor-core kernels, fp32 on the CUDA-core kernels; the wide generator (ngf 128,
+    ndf 64) takes the output layer by parity class and the wide first-layer variant."""
     pool = _field_pool(3, 40)
     ngf, ndf = width if isinstance(width, tuple) else (width, width)
-    width = min(ngf, ndf)
     g = _grid(L, rows, cols, 11, pool, precision=precision, keep_grads=1, ngf=ngf, ndf=ndf,
               batch=batch)
     a = oracle_arch(g.arch)
     tol = TOL[g.arch.precision]
-    for it in range(2 if width < 64 else 1):
+    gl, dl = O.g_layout(a), O.d_layout(a)
+    nbr = O.neighbors(rows, cols)
+    for it in range(2 if min(ngf, ndf) < 64 else 1):
         s = _state(g)
         data = O.batches(s, pool)
         ev = g.eval()
@@ -126,23 +148,19 @@ def test_dcgan_one_iteration_parity(L, precision, width, rows, cols, batch):
         got = _state(g)
         assert np.array_equal(got.Gstep, new.Gstep) and np.array_equal(got.Dstep, new.Dstep)
         gg, gd = g.gradients()
-        worst = np.zeros(s.cells)
-        for pop, gpu, r in (("G", gg, grads["gG"]), ("D", gd, grads["gD"]),
-                            ("G", got.Gm, new.Gm), ("D", got.Dm, new.Dm)):
-            lay = O.g_layout(a) if pop == "G" else O.d_layout(a)
-            for c in range(s.cells):
-                worst[c] = max(worst[c], max(per_tensor(gpu[c:c + 1], r[c:c + 1], lay).values()))
-        ok = worst < tol
-        kinky = grads["kink"] < (1e-5 if precision == "fp32" else 1e-3)
-        assert np.all(ok | kinky), (it, worst)
-        if precision == "fp32":
-            assert np.sum(~ok) <= 1, (it, worst)
-        elif width >= 64:
-            assert np.all(worst < 0.075), (it, worst)
-            if ngf == ndf:
-                assert np.median(worst) < 0.05, (it, worst)
-        else:
-            assert np.all(worst < 5 * tol) and np.median(worst) < 2 * tol, (it, worst)
+        err = np.concatenate([cell_errors(gg, grads["gG"], gl), cell_errors(gd, grads["gD"], dl),
+                              cell_errors(got.Gm, new.Gm, gl), cell_errors(got.Dm, new.Dm, dl)],
+                             axis=1)
+        worst = err.max(axis=1)
+        src_g = nbr[np.arange(s.cells), ref_sel["sel_g"]]
+        src_d = nbr[np.arange(s.cells), ref_sel["sel_d"]]
+        spread = _spread(a, [(s.Gw[src_g[c]], s.Dw[src_d[c]]) + tuple(data[c]) +
+                             ((grads["gG"][c], grads["gD"][c]),) for c in range(s.cells)])
+        bound = np.maximum(tol, SPREAD_FACTOR * spread)
+        print("PARITY dcgan %s width %s it %d worst %s spread %s" % (
+            precision, width, it, " ".join("%.2e" % v for v in worst),
+            " ".join("%.2e" % v for v in spread)))
+        assert np.all(worst <= bound), (it, worst, spread)
 
 
 def test_dcgan_fused_iterate_equals_separate_calls_and_is_deterministic(L):
@@ -159,23 +177,40 @@ def test_dcgan_fused_iterate_equals_separate_calls_and_is_deterministic(L):
 
 def test_dcgan_full_width_3x3_b128_sampled(L):
     """The 3x3 DCGAN configuration (width 64: 512/256/128/64 channels, z = 100, B = 128,
-    bf16): one cell's centre generator on its noise (the full batch, for the batch
-    statistics) and the logits of sampled rows against the oracle."""
+    bf16): every logit of one cell (the real rows and the five generator slots' fakes, through
+    all five discriminator slots), its pair losses and fitness against the oracle computed for
+    that cell, the selection bit-exact, then that cell's training gradients under the rule of
+    the one-iteration check (its oracle spread measured on the same inputs)."""
     pool = _field_pool(1811, 600)
-    g = _grid(L, 3, 3, 1811, pool, precision="bf16", z_dim=100, ngf=64, ndf=64, batch=128)
+    g = _grid(L, 3, 3, 1811, pool, precision="bf16", z_dim=100, ngf=64, ndf=64, batch=128,
+              keep_grads=1)
     s = _state(g)
+    a = s.arch
     c = 4
     data = O.batches(s, pool, cells=[c])
-    g.eval()
-    x, z = g.batch()
-    a = s.arch
-    gl, dl = O.g_layout(a), O.d_layout(a)
-    F = O.g_forward(O.unflatten(s.Gw[c], gl), data[c][1], a)["F"]
+    ref = O.eval_neighborhoods(s, data, cells=[c])
+    ev = g.eval(pairs=True)
     logits = g.logits()
-    rows = np.r_[0:8, 128:136]  # real rows, then the centre generator's fakes
-    X = np.vstack([data[c][0], F])[rows]
-    lg = O.d_forward(O.unflatten(s.Dw[c], dl), X, a)["logit"]
-    assert max_rel(logits[c, 0, rows], lg) < 2e-2
+    assert max_rel(logits[c], ref["logits"][c]) < 2e-2
+    for k in ("LG", "LD", "fG", "fD"):
+        assert max_rel(ev[k][c], ref[k][c]) < 2e-2, k
+    sel = g.select()
+    ref_sel = O.select_replace(s, {"fG": ev["fG"].astype(np.float64),
+                                   "fD": ev["fD"].astype(np.float64)})
+    assert np.array_equal(sel["sel_g"], ref_sel["sel_g"])
+    assert np.array_equal(sel["sel_d"], ref_sel["sel_d"])
+    g.train()
+    gg, gd = g.gradients()
+    nbr = O.neighbors(3, 3)
+    sg, sd = nbr[c][ref_sel["sel_g"][c]], nbr[c][ref_sel["sel_d"][c]]
+    x, z = data[c]
+    rG, rD, _ = O.pair_gradients(s.Gw[sg], s.Dw[sd], x, z, a)
+    gl, dl = O.g_layout(a), O.d_layout(a)
+    worst = max(cell_errors(gg[c:c + 1], rG[None], gl).max(),
+                cell_errors(gd[c:c + 1], rD[None], dl).max())
+    spread = _spread(a, [(s.Gw[sg], s.Dw[sd], x, z, (rG, rD))])[0]
+    print("PARITY dcgan bf16 3x3 B=128 cell %d worst %.4f spread %.4f" % (c, worst, spread))
+    assert worst <= max(2e-2, SPREAD_FACTOR * spread), (worst, spread)
 
 
 def test_dcgan_tma_and_gathered_activations_agree_bit_for_bit(L, monkeypatch):

@@ -175,3 +175,25 @@ def test_initialisation_moments_and_output_range():
     # batch normalisation in training mode: each generator layer's output has zero batch mean
     h = O.g_forward(Gp, z, arch)["cache"][1][2]
     assert np.allclose(h.mean(axis=(0, 2, 3)), Gp["beta2"], atol=1e-12)
+
+
+def test_float32_accumulation_variant_is_the_same_arithmetic():
+    """oracle.dcgan.ACC = float32 sums every convolution and batch-norm statistic in float32
+    (tests use the spread between it and the float64 oracle to set their tolerances). On a
+    small network it must agree with the float64 oracle to float32 rounding, and differ from it
+    (the switch takes effect)."""
+    from oracle import dcgan as DC
+    a = O.Arch(kind="dcgan", precision="fp32", batch=3, z_dim=8, x_dim=12288, ngf=4, ndf=4)
+    s = O.create(1, 1, a, 3)
+    rng = np.random.default_rng(0)
+    x = rng.uniform(-1, 1, size=(3, 12288))
+    z = rng.normal(size=(3, 8))
+    ref = O.pair_gradients(s.Gw[0], s.Dw[0], x, z, a)
+    try:
+        DC.ACC = np.float32
+        got = O.pair_gradients(s.Gw[0], s.Dw[0], x, z, a)
+    finally:
+        DC.ACC = np.float64
+    for r, g in zip(ref[:2], got[:2]):
+        d = np.max(np.abs(g - r)) / np.max(np.abs(r))
+        assert 0 < d < 1e-4, d
