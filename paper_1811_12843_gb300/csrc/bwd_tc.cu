@@ -149,7 +149,7 @@ __device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int
 // derivative (read from the stored forward output). `full` = all 16 columns lie inside N.
 __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16], int cell, int m,
                                       int arow, int col0, bool full, float dlo, bool is_tanh,
-                                      float (&vout)[16]) {
+                                      float (&vout)[16], const uint4* xpre = nullptr) {
   if (p.epi == EPI_F32) {
     float* C = reinterpret_cast<float*>(p.C) + (int64_t)cell * p.c_cell + (int64_t)m * p.scm;
     if (p.scn == 1) {
@@ -179,7 +179,8 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
   const bf16* X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
   if (p.aux_sel) X += (int64_t)(1 + __ldg(&p.aux_sel[cell])) * p.aux_sel_stride;
   if (p.sxn == 1 && p.scn == 1 && full) {
-    const uint4* x4 = reinterpret_cast<const uint4*>(X + col0);
+    // the caller may have loaded this group's forward output ahead (xpre)
+    const uint4* x4 = xpre ? xpre : reinterpret_cast<const uint4*>(X + col0);
     const uint4 q0 = x4[0], q1 = x4[1];
     const uint32_t w[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
     uint32_t pk[8];
@@ -247,8 +248,30 @@ __device__ __forceinline__ bool epilogue_tile(const GParams& p, int cell, int m0
   const bool brow = row_ok && m < p.bias_rows;
   float* bp = bpart + (btile & 1) * (4 * 256) + q * 256;
   int gi = g0;
+  // EPI_DACT reads its row's stored forward output: the next pair of groups' values are loaded
+  // while this pair is converted (one memory latency per tile instead of one per pair)
+  const bool pre = p.epi == EPI_DACT && p.sxn == 1 && p.scn == 1 && row_ok;
+  const bf16* X = nullptr;
+  if (pre) {
+    X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
+    if (p.aux_sel) X += (int64_t)(1 + __ldg(&p.aux_sel[cell])) * p.aux_sel_stride;
+  }
+  auto load_pair = [&](int g, uint4(&d)[4]) {
+    const uint4* x4 = reinterpret_cast<const uint4*>(X + n0 + g * 16);
+    if (n0 + g * 16 + 16 <= p.N) {
+      d[0] = x4[0];
+      d[1] = x4[1];
+    }
+    if (g + 1 < g1 && n0 + g * 16 + 32 <= p.N) {
+      d[2] = x4[2];
+      d[3] = x4[3];
+    }
+  };
+  uint4 xc[4], xn[4];
+  if (pre && gi < g1) load_pair(gi, xc);
   // two 16-column groups per TMEM load where possible
   for (; gi + 1 < g1; gi += 2) {
+    if (pre && gi + 2 < g1) load_pair(gi + 2, xn);
     uint32_t r[32];
     LIPZ_TMEM_LD32(tbase + gi * 16, r);
     tmem_wait_ld();
@@ -259,9 +282,14 @@ __device__ __forceinline__ bool epilogue_tile(const GParams& p, int cell, int m0
 #pragma unroll
     for (int e = 0; e < 16; ++e) va[e] = vb[e] = 0.f;
     if (row_ok) {
-      epi16(p, ra, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va);
+      epi16(p, ra, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va, pre ? &xc[0] : nullptr);
       if (col0 + 16 < p.N)
-        epi16(p, rb, cell, m, arow, col0 + 16, col0 + 32 <= p.N, dlo, is_tanh, vb);
+        epi16(p, rb, cell, m, arow, col0 + 16, col0 + 32 <= p.N, dlo, is_tanh, vb,
+              pre ? &xc[2] : nullptr);
+    }
+    if (pre) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) xc[u] = xn[u];
     }
     if (bias) {
       if (!brow) {
@@ -283,7 +311,8 @@ __device__ __forceinline__ bool epilogue_tile(const GParams& p, int cell, int m0
     float va[16];
 #pragma unroll
     for (int e = 0; e < 16; ++e) va[e] = 0.f;
-    if (row_ok && col0 < p.N) epi16(p, r, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va);
+    if (row_ok && col0 < p.N)
+      epi16(p, r, cell, m, arow, col0, col0 + 16 <= p.N, dlo, is_tanh, va, pre ? &xc[0] : nullptr);
     if (bias) {
       if (!brow) {
 #pragma unroll
