@@ -862,10 +862,13 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
                                     ? sZ
                                     : (J.a_from_h ? sH + kc * H_CHUNK : sS);
             const uint32_t sB = sS + (CF::A_IN ? A_BYTES : 0);
+            // a 16-element K step is 32 bytes: 2 in the descriptors' address field (a 1024-byte
+            // aligned tile plus at most 96 bytes never carries out of it)
+            const uint64_t dA = sw128_desc(sA), dB = sw128_desc(sB);
+            tc_mma_cg2(d, dA, dB, idesc, kc != 0 ? 1u : 0u);
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
-              tc_mma_cg2(d, sw128_desc(sA + kk * 32), sw128_desc(sB + kk * 32), idesc,
-                         (kc | kk) != 0 ? 1u : 0u);
+            for (int kk = 1; kk < BK / 16; ++kk)
+              tc_mma_cg2_acc(d, dA + 2 * kk, dB + 2 * kk, idesc);
             tc_commit_cg2(bEmpty + 8 * stage, 3);
             if (++stage == CF::STAGES) {
               stage = 0;

@@ -308,6 +308,14 @@ __device__ __forceinline__ void tc_mma_cg2(uint32_t d, uint64_t a, uint64_t b, u
       "l"(a), "l"(b), "r"(idesc), "r"(acc)
       : "memory");
 }
+// The same MMA accumulating into D (no predicate to set up).
+__device__ __forceinline__ void tc_mma_cg2_acc(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.eq.u32 p, 1, 1;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc)
+      : "memory");
+}
 // Arrive, once the MMAs issued so far have completed, on the mbarrier at offset `bar` of every
 // CTA in `mask`.
 __device__ __forceinline__ void tc_commit_cg2(uint32_t bar, uint16_t mask) {
