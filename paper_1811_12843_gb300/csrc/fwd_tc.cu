@@ -685,6 +685,15 @@ struct PParams {
   float* logits;
   float slope;
   int* err;
+  // discriminator training forward (train != 0): pair job c * mt + t takes m-tile t of both
+  // parts of cell c through discriminator wsel[c]: rank 0 the B real rows (slot 0 of E[c]),
+  // rank 1 the selected generator's fakes (slot 1 + part_slot[c]); both hidden activations go
+  // to act1 / act2 ([2c + part][B][256] bf16), the logits to logits[(2c + part) B + row]
+  int train, mt;
+  const int* wsel;
+  const int* part_slot;
+  bf16* act1;
+  bf16* act2;
 };
 
 template <int KND>
@@ -775,10 +784,16 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
       uint32_t phase = 0;
       bool ok = true;
       for (int pi = cid; pi < p.n_pairs && ok; pi += ncl) {
-        const int4 pr = __ldg(&p.pairs[pi]);
-        const int k = pr.x;
+        const bool train = KND == KIND_D && p.train;
+        const int4 pr = train ? make_int4(0, 0, 0, 0) : __ldg(&p.pairs[pi]);
+        const int k = train ? __ldg(&p.wsel[pi / p.mt]) : pr.x;
         int a_cell = 0, a_row = p.rows;  // no problem: rows past the end read as zero
-        if (KND == KIND_D) {
+        if (train) {
+          // (rows of the tile past the part's B read the next slot's rows: never stored)
+          const int cell = pi / p.mt, t = pi - cell * p.mt;
+          a_cell = cell;
+          a_row = (rank ? 1 + __ldg(&p.part_slot[cell]) : 0) * p.B + t * BM;
+        } else if (KND == KIND_D) {
           const int prob = rank ? pr.z : pr.y;
           if (prob >= 0) {
             a_cell = prob / 5;
@@ -909,12 +924,17 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
       if (lane == 0) mbar_arrive_remote(bar_cluster);
     };
     for (int pi = cid; pi < p.n_pairs && ok; pi += ncl, ++ltile) {
-      const int4 pr = __ldg(&p.pairs[pi]);
-      const int k = pr.x;
+      const bool train = KND == KIND_D && p.train;
+      const int4 pr = train ? make_int4(0, 0, 0, 0) : __ldg(&p.pairs[pi]);
+      const int k = train ? __ldg(&p.wsel[pi / p.mt]) : pr.x;
       bool row_ok;
       bf16* dst = nullptr;   // generator: this row of the fakes
-      int64_t lidx = 0;      // discriminator: this row's logit
-      if (KND == KIND_G) {
+      int64_t lidx = 0;      // discriminator: this row's logit (training: and activations)
+      if (train) {
+        const int cell = pi / p.mt, rr = (pi - cell * p.mt) * BM + row;
+        row_ok = rr < p.B;
+        lidx = (int64_t)(2 * cell + (int)rank) * p.B + rr;
+      } else if (KND == KIND_G) {
         const int gr = pr.y + (int)rank * BM + row;
         row_ok = gr < pr.w;
         if (row_ok) {
@@ -1009,6 +1029,12 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
                            "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]), "r"(pk[4 * u + 3])
                            : "memory");
             }
+            if (train && j == 0 && row_ok) {
+              uint4* o = reinterpret_cast<uint4*>(p.act1 + lidx * HID + col0);
+#pragma unroll
+              for (int u = 0; u < W / 8; ++u)
+                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+            }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             warp_signal(lH + 8 * ch);
           }
@@ -1032,6 +1058,7 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
               const uint32_t(&r)[32] = r2[h2];
               const float4* b4 = reinterpret_cast<const float4*>(bias + cg * 32);
               const float4* w4 = reinterpret_cast<const float4*>(w3 + cg * 32);
+              uint32_t pk[16];
 #pragma unroll
               for (int e = 0; e < 32; e += 4) {
                 const float4 bb = b4[e >> 2], ww = w4[e >> 2];
@@ -1044,12 +1071,20 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
                 a2 = a2 > 0.f ? a2 : p.slope * a2;
                 a3 = a3 > 0.f ? a3 : p.slope * a3;
                 const uint32_t q01 = pack_bf16(a0, a1), q23 = pack_bf16(a2, a3);
+                pk[e >> 1] = q01;
+                pk[(e >> 1) + 1] = q23;
                 const __nv_bfloat162 v01 = *reinterpret_cast<const __nv_bfloat162*>(&q01);
                 const __nv_bfloat162 v23 = *reinterpret_cast<const __nv_bfloat162*>(&q23);
                 acc = fmaf(__low2float(v01), ww.x, acc);
                 acc = fmaf(__high2float(v01), ww.y, acc);
                 acc = fmaf(__low2float(v23), ww.z, acc);
                 acc = fmaf(__high2float(v23), ww.w, acc);
+              }
+              if (train && row_ok) {
+                uint4* o = reinterpret_cast<uint4*>(p.act2 + lidx * HID + cg * 32);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
               }
             }
           }
@@ -1163,7 +1198,7 @@ struct TcPlan {
   // weight maps of the CTA-pair kernels: boxes of half the output columns (128 rows)
   CUtensorMap mG1h, mG2h, mG3h, mD1h, mD2h;
   tc::KParams pg, pgc, pd, pgt, pdt, pgram;
-  tc::PParams ppg, ppd;
+  tc::PParams ppg, ppd, ppdt;
   int grid_g, grid_gc, grid_d, grid_gt, grid_dt, grid_gram;
   int ncl_g, ncl_d;        // co-resident clusters of the pair kernels (0: pair path off)
   int* err;
@@ -1481,6 +1516,17 @@ TcPlan* tc_plan_create(const TcShape& s, const TcBuffers& b, std::string* msg) {
   ppd.off_w3 = b.doff[4];
   p->ppg = ppg;
   p->ppd = ppd;
+  tc::PParams ppdt = ppd;  // the training discriminators: both parts of a cell on one pair
+  ppdt.train = 1;
+  ppdt.mt = tiles(s.B);
+  ppdt.n_pairs = s.cells * ppdt.mt;
+  ppdt.rows = s.B;
+  ppdt.wsel = b.src_d;
+  ppdt.part_slot = b.sel_g;
+  ppdt.act1 = (bf16*)b.TG1;
+  ppdt.act2 = (bf16*)b.TG2;
+  ppdt.logits = b.TL;
+  p->ppdt = ppdt;
   const bool pairs_on = !env_flag("LIPZ_FWD_SINGLE");
   p->ncl_g = pairs_on && s.z == tc::BK
                  ? max_pair_clusters(tc::k_mlp_fwd_pair<tc::KIND_G>, tc::pair_threads<tc::KIND_G>(),
@@ -1592,6 +1638,8 @@ int tc_run_train_g(TcPlan* p, cudaStream_t st, std::string* msg) {
 }
 
 int tc_run_train_d(TcPlan* p, cudaStream_t st, std::string* msg) {
+  if (p->ncl_d > 0)
+    return launch_pair(p->ncl_d, p->mE, p->mD1h, p->mD2h, p->mD2h, p->ppdt, false, st, msg);
   return launch(p->grid_dt, p->mE4, p->mD1, p->mD2, p->mD2, p->pdt, st,
                 "discriminator training forward", msg);
 }

@@ -608,12 +608,24 @@ __global__ void __launch_bounds__(1024) k_dlogit(
   }
   if (rg < RG) {
     const bool vec = sizeof(T) == 2 && (H & 7) == 0;
-    for (int r = rg; r < 3 * B; r += RG) {
-      const int rr = r < 2 * B ? r : r - B;
-      const float dr = dl[r];
-      if (vec) {
+    // the rows of this thread in groups of four, the four loads issued before any is used (one
+    // memory latency per group); rows are still taken in increasing order
+    constexpr int U = 4;
+    for (int r0 = rg; vec && r0 < 3 * B; r0 += U * RG) {
+      uint4 qv[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int r = r0 + u * RG;
+        const int rr = r < 2 * B ? r : r - B;
+        if (r < 3 * B) qv[u] = *reinterpret_cast<const uint4*>(g2 + (int64_t)rr * H + k0);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int r = r0 + u * RG;
+        if (r >= 3 * B) break;
+        const float dr = dl[r];
         // eight bf16 columns in one 16-byte load and store
-        const uint4 q = *reinterpret_cast<const uint4*>(g2 + (int64_t)rr * H + k0);
+        const uint4 q = qv[u];
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
         uint32_t o[4];
 #pragma unroll
@@ -632,7 +644,12 @@ __global__ void __launch_bounds__(1024) k_dlogit(
           }
         }
         *reinterpret_cast<uint4*>(j2 + (int64_t)r * H + k0) = make_uint4(o[0], o[1], o[2], o[3]);
-      } else {
+      }
+    }
+    for (int r = rg; !vec && r < 3 * B; r += RG) {
+      const int rr = r < 2 * B ? r : r - B;
+      const float dr = dl[r];
+      {
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           if (k0 + e >= H) break;
