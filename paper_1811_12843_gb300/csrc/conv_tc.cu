@@ -18,6 +18,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
 #include <string>
 
 #include "common.cuh"
@@ -1442,6 +1443,146 @@ __global__ void __launch_bounds__(256) k_bn_back_apply_hwc(const BnDesc* __restr
   }
 }
 
+
+// ---- the generator's first layer on tcgen05 -------------------------------------------------
+// A 4x4 transposed convolution of a 1x1 input is the plain product y[n][(tap, o)] =
+// sum_c z[n][c] W[c][o][tap] (Table 1, CelebA column: z of 100 entries to 4 x 4 x 8 ngf). One
+// CTA computes one problem's rows (B <= 128) against 256 consecutive (tap, o) columns: the
+// noise rows are loaded into the 128-byte-swizzled K-major layout (K padded with zeros to 128),
+// the weights arrive by TMA from a [individual][(tap, o)][128] copy (launch_relayout_g1), eight
+// MMAs accumulate in TMEM, and each epilogue thread stores its row's 256 fp32 values
+// channel-last (y[n][tap * co + o], the layout the channel-last batch norm reads).
+constexpr int D1_THREADS = 128;
+constexpr int D1_SMEM = 1024 + 2 * A_BYTES + 2 * B_BYTES + 64;
+
+__global__ void __launch_bounds__(D1_THREADS) k_dense1_tc(const __grid_constant__ CUtensorMap mW,
+                                                          const ConvDesc* __restrict__ descs,
+                                                          const int* __restrict__ wsel_override,
+                                                          int rows, int ca, int N, int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sA = base, sB = base + 2 * A_BYTES;
+  uint8_t* misc = gbase + 2 * A_BYTES + 2 * B_BYTES;
+  const uint32_t bFull = smem_u32(misc), bMma = bFull + 8;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 16);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 20);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * 256;
+  if (threadIdx.x == 0) {
+    mbar_init(bFull, 1);
+    mbar_init(bMma, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  const ConvDesc d = descs[blockIdx.y];
+  const int* ws = wsel_override ? wsel_override : d.wsel;
+  const int indiv = ws ? __ldg(&ws[d.wsel_idx]) : 0;
+  if (threadIdx.x == 0) {
+    mbar_expect_tx(bFull, 2u * B_BYTES);
+    tma_load_3d(sB, &mW, bFull, 0, n0, indiv);
+    tma_load_3d(sB + B_BYTES, &mW, bFull, BK, n0, indiv);
+  }
+  // the noise rows, 8-byte loads (ca a multiple of 4, rows 8-byte aligned); 16-byte unit u of
+  // row r (K elements 8u .. 8u + 7) goes to unit u ^ (r & 7) of its 128-byte row
+  {
+    const bf16* z = (const bf16*)d.a;
+    const int r = threadIdx.x;
+    const uint2* zr = reinterpret_cast<const uint2*>(z + (int64_t)r * ca);
+#pragma unroll 4
+    for (int u = 0; u < 16; ++u) {
+      const int k = 8 * u;
+      uint2 lo = make_uint2(0u, 0u), hi = make_uint2(0u, 0u);
+      if (r < rows) {
+        if (k < ca) lo = zr[k >> 2];
+        if (k + 4 < ca) hi = zr[(k >> 2) + 1];
+      }
+      const uint32_t addr = sA + (uint32_t)((u >> 3) * A_BYTES) + (uint32_t)r * 128u +
+                            ((uint32_t)((u & 7) ^ (r & 7)) << 4);
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(lo.x), "r"(lo.y),
+                   "r"(hi.x), "r"(hi.y)
+                   : "memory");
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (mbar_wait(bFull, 0u, abort_flag, err, 41)) {
+      tc_fence_after();
+      constexpr uint32_t idesc = idesc_bf16(BM, 256);
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)
+          tc_mma(tmem, sw128_desc(sA + c * A_BYTES + kk * 32), sw128_desc(sB + c * B_BYTES + kk * 32),
+                 idesc, (c | kk) != 0 ? 1u : 0u);
+      tc_commit(bMma);
+    }
+  }
+  if (mbar_wait_warp(bMma, 0u, abort_flag, err, 42)) {
+    tc_fence_after();
+    const int row = warp * 32 + lane;
+    float* out = (float*)d.out + (int64_t)row * N + n0;
+#pragma unroll 1
+    for (int g = 0; g < 16; ++g) {
+      uint32_t r[16];
+      LIPZ_TMEM_LD16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(g * 16), r);
+      tmem_wait_ld();
+      if (row < rows && n0 + g * 16 < N) {
+        float4* o = reinterpret_cast<float4*>(out + g * 16);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          o[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                             __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+}
+
+// [individual][c][o][tap] (c < ca) -> [individual][(tap, o)][128], K padded with zeros
+__global__ void k_relayout_g1(const bf16* __restrict__ src, int64_t src_ps, int64_t src_off,
+                              bf16* __restrict__ dst, int64_t dst_ps, int ca, int co,
+                              int n_indiv) {
+  pdl_wait();
+  const int N = 16 * co;
+  const int64_t units = (int64_t)n_indiv * N * 16;  // 16-byte units of the copy
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < units;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int u = (int)(i & 15);
+    const int64_t rn = i >> 4;
+    const int n = (int)(rn % N);
+    const int ind = (int)(rn / N);
+    const int tap = n / co, o = n - tap * co;
+    const bf16* w = src + (int64_t)ind * src_ps + src_off + (int64_t)o * 16 + tap;
+    uint32_t v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int k0 = 8 * u + 2 * e;
+      const unsigned short a = k0 < ca ? __bfloat16_as_ushort(w[(int64_t)k0 * co * 16]) : 0;
+      const unsigned short b =
+          k0 + 1 < ca ? __bfloat16_as_ushort(w[(int64_t)(k0 + 1) * co * 16]) : 0;
+      v[e] = (uint32_t)a | ((uint32_t)b << 16);
+    }
+    *reinterpret_cast<uint4*>(dst + (int64_t)ind * dst_ps + (int64_t)n * 128 + 8 * u) =
+        make_uint4(v[0], v[1], v[2], v[3]);
+  }
+}
+
 }  // namespace ctc
 
 bool wgtc_prepare(std::string* msg) {
@@ -1712,7 +1853,34 @@ bool ctc_prepare(std::string* msg) {
       if (msg) *msg = "cannot reserve shared memory for the tensor-core convolution";
       return false;
     }
+  if (cudaFuncSetAttribute(ctc::k_dense1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           ctc::D1_SMEM) != cudaSuccess) {
+    cudaGetLastError();
+    if (msg) *msg = "cannot reserve shared memory for the generator's first layer";
+    return false;
+  }
   return true;
+}
+
+bool dense1_tc_supported(int rows, int ca, int co) {
+  return rows >= 1 && rows <= ctc::BM && ca >= 1 && ca <= 2 * ctc::BK && ca % 4 == 0 &&
+         (16 * co) % 256 == 0;
+}
+
+void launch_dense1_tc(const CUtensorMap& mW, const ConvDesc* descs, int n_problems,
+                      const int* wsel_override, int rows, int ca, int co, int* err,
+                      cudaStream_t st) {
+  if (n_problems <= 0) return;
+  launch_pdl(ctc::k_dense1_tc, dim3(16 * co / 256, n_problems), dim3(ctc::D1_THREADS),
+             (size_t)ctc::D1_SMEM, st, mW, descs, wsel_override, rows, ca, 16 * co, err);
+}
+
+void launch_relayout_g1(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst,
+                        int64_t dst_ps, int ca, int co, int n_indiv, cudaStream_t st) {
+  const int64_t units = (int64_t)n_indiv * 16 * co * 16;
+  const int blocks = (int)std::min<int64_t>((units + 255) / 256, 4096);
+  launch_pdl(ctc::k_relayout_g1, dim3(blocks), dim3(256), 0, st, src, src_ps, src_off, dst,
+             dst_ps, ca, co, n_indiv);
 }
 
 bool launch_conv_tc(const CUtensorMap& mW, const CUtensorMap& mA, const CtcParams& p, int sms,

@@ -155,6 +155,20 @@ void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const
 // with the same part and counters buffers.
 void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
                                  float* part, unsigned* counters, cudaStream_t st);
+// The generator's first layer (a 4x4 transposed convolution of the 1x1 noise input) as the
+// product y[n][(tap, o)] = sum_c z[n][c] W[c][o][tap] on tcgen05 (DENSE1 descriptors: a = noise
+// rows [n][ca] bf16, 8-byte aligned; out = fp32 channel-last [n][16 co]; the individual from
+// wsel_override or the descriptor's wsel). mW maps the [individual][16 co][128] copy of
+// launch_relayout_g1 (ctc_make_map, K 128, box 256 rows). rows <= 128, ca <= 128 and a multiple
+// of 4, 16 co a multiple of 256 (dense1_tc_supported).
+bool dense1_tc_supported(int rows, int ca, int co);
+void launch_dense1_tc(const CUtensorMap& mW, const ConvDesc* descs, int n_problems,
+                      const int* wsel_override, int rows, int ca, int co, int* err,
+                      cudaStream_t st);
+// [individual][ca][co][4][4] at src_off (stride src_ps) -> dst [individual][(tap, o)][128]
+// (stride dst_ps), K padded with zeros.
+void launch_relayout_g1(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst,
+                        int64_t dst_ps, int ca, int co, int n_indiv, cudaStream_t st);
 int64_t bn_hwc_part_floats(int n_problems, int channels);
 int64_t bn_hwc_counters(int n_problems, int channels);
 

@@ -121,6 +121,10 @@ struct DcPlan {
   LogitDesc *tdl_tc, *tdl_back_d_tc, *tdl_back_g_tc;
   bf16* Gwt = nullptr;
   int64_t gwt_ps = 0;
+  // the generator's first layer on tcgen05: a (tap, o) copy of its weights inside Gwt
+  bool g1tc = false;
+  int64_t g1_off = 0;
+  CUtensorMap mG1;
   RelayoutG relg;
   CUtensorMap mG[4];
   CtcParams gp[4];
@@ -609,12 +613,20 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       r.dst_off[i] = off;
       off += (int64_t)4 * r.cls_rows[i] * 4 * gc[l - 1];
     }
+    p->g1tc = dense1_tc_supported(B, s.z, gc[1]);
+    if (p->g1tc) {
+      p->g1_off = (off + 63) / 64 * 64;
+      off = p->g1_off + (int64_t)16 * gc[1] * 128;
+    }
     p->gwt_ps = (off + 63) / 64 * 64;
     ok = ok && !dev_alloc(p, &p->bnpart, (size_t)bn_hwc_part_floats(PE, 8 * g) * 4, msg);
     ok = ok && !dev_alloc(p, &p->bncnt, (size_t)bn_hwc_counters(PE, 8 * g) * 4, msg);
     if (ok) ok = cudaMemset(p->bncnt, 0, (size_t)bn_hwc_counters(PE, 8 * g) * 4) == cudaSuccess;
     ok = ok && !dev_alloc(p, &p->Gwt, (size_t)s.n_indiv * p->gwt_ps * 2, msg);
     if (ok) ok = cudaMemset(p->Gwt, 0, (size_t)s.n_indiv * p->gwt_ps * 2) == cudaSuccess;
+    if (ok && p->g1tc)
+      ok = ctc_make_map(&p->mG1, p->Gwt + p->g1_off, 128, (uint64_t)16 * gc[1], s.n_indiv,
+                        p->gwt_ps, 256, msg);
     for (int i = 0; i < 4 && ok; ++i) {
       const int l = i + 2;
       const int ci = gc[l - 1], co = gc[l];
@@ -1022,8 +1034,14 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int PE = C * 5;
   if (p->tcg) {
     launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
-    launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
-                nullptr, 0, s.slope, st);
+    if (p->g1tc) {
+      launch_relayout_g1((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[0], p->Gwt + p->g1_off,
+                         p->gwt_ps, s.z, gc[1], s.n_indiv, st);
+      launch_dense1_tc(p->mG1, p->eg[0], PE, nbr, B, s.z, gc[1], p->err, st);
+    } else {
+      launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
+                  nullptr, 0, s.slope, st);
+    }
     launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, st);
     if (p->scg)
       launch_relayout_s((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[12], p->Gs, s.n_indiv, st);
@@ -1096,8 +1114,11 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   const int ds[5] = {64, 32, 16, 8, 4};
   // forward of the selected pair
   if (p->tct) {
-    launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
-                nullptr, 0, s.slope, st);
+    if (p->g1tc)
+      launch_dense1_tc(p->mG1, p->tg[0], C, nullptr, B, s.z, gc[1], p->err, st);
+    else
+      launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
+                  nullptr, 0, s.slope, st);
     launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->tgp[i];
