@@ -620,6 +620,22 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
             }
             if constexpr (OM == CTC_LRELU_LOGIT) continue;
             __syncwarp();
+            if (f32 && p.bn_part) {
+              // batch-norm statistics: sum and sum of squares of column `lane` over the warp's
+              // valid rows, in row order, into this (tile, half, lane quarter)'s slot
+              const unsigned vm = __ballot_sync(0xffffffffu, valid);
+              float bs = 0.f, bq = 0.f;
+#pragma unroll 8
+              for (int rr = 0; rr < 32; ++rr) {
+                const float x = __uint_as_float(stg[rr * 36 + lane]);
+                if ((vm >> rr) & 1u) {
+                  bs += x;
+                  bq = fmaf(x, x, bq);
+                }
+              }
+              const int64_t slot = ((int64_t)tile * (p.m2 ? 2 : 1) + h) * 4 + q;
+              p.bn_part[slot * p.co + j * 256 + g * 32 + lane] = make_float2(bs, bq);
+            }
             const int lpr = f32 ? 8 : 4, rpi = 32 / lpr;
             const int part = lane % lpr;
             for (int it = 0; it < lpr; ++it) {
@@ -1300,6 +1316,54 @@ __global__ void __launch_bounds__(256) k_bn_stats_hwc(const BnDesc* __restrict__
   if (threadIdx.x == 0) *cnt = 0u;
 }
 
+// The statistics when the producing convolution summed them (CtcParams::bn_part): problem pr
+// owns slots [pr T, (pr + 1) T) of part ([slot][C] float2: sum, sum of squares over one lane
+// quarter's rows of one tile). Warp w of the 32 takes slots w, w + 32, ... (four loads in
+// flight, float sums in slot order); warp 0 adds the 32 warp sums in float64 in warp order.
+__global__ void __launch_bounds__(1024) k_bn_finalize_hwc(const BnDesc* __restrict__ descs,
+                                                          const float2* __restrict__ part, int T) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int ch = blockIdx.x * 32 + lane;
+  __shared__ float sh[32][32][2];
+  float s = 0.f, q = 0.f;
+  if (ch < d.C) {
+    const float2* pp = part + (int64_t)blockIdx.y * T * d.C + ch;
+    int t = w;
+    for (; t + 96 < T; t += 128) {
+      float2 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = pp[(int64_t)(t + 32 * u) * d.C];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        s += v[u].x;
+        q += v[u].y;
+      }
+    }
+    for (; t < T; t += 32) {
+      const float2 v = pp[(int64_t)t * d.C];
+      s += v.x;
+      q += v.y;
+    }
+  }
+  sh[w][lane][0] = s;
+  sh[w][lane][1] = q;
+  __syncthreads();
+  if (w == 0 && ch < d.C) {
+    double ts = 0.0, tq = 0.0;
+    for (int i = 0; i < 32; ++i) {
+      ts += sh[i][lane][0];
+      tq += sh[i][lane][1];
+    }
+    const double m = (double)((int64_t)d.n << d.lhw);
+    const double mean_d = ts / m;
+    const double var_d = fmax(tq / m - mean_d * mean_d, 0.0);
+    d.mean[ch] = (float)mean_d;
+    d.inv[ch] = rsqrtf((float)var_d + 1e-5f);
+  }
+}
+
 __global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__ descs,
                                                       const int* __restrict__ wsel_override) {
   pdl_wait();
@@ -1325,6 +1389,58 @@ __global__ void __launch_bounds__(256) k_bn_apply_hwc(const BnDesc* __restrict__
   }
   for (; px < p1; px += 8)
     h[px * d.C + ch] = __float2bfloat16_rn(fmaxf(fmaf(sc, d.c[px * d.C + ch] - mean, b), 0.f));
+}
+
+// The apply pass with four channels per thread (C a multiple of 4, at most 1024): 16-byte
+// loads of the fp32 input and 8-byte stores of the bf16 output, whole rows per warp; block z
+// of a problem takes elements [z E, (z + 1) E) with E = BN_APPLY_ELEMS. Same arithmetic as
+// k_bn_apply_hwc.
+constexpr int BN_APPLY_ELEMS = 32768;
+__global__ void __launch_bounds__(256) k_bn_apply_hwc4(const BnDesc* __restrict__ descs,
+                                                       const int* __restrict__ wsel_override) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int nq = d.C >> 2;
+  const int64_t total = ((int64_t)d.n << d.lhw) * d.C;
+  const int64_t e0 = (int64_t)blockIdx.x * BN_APPLY_ELEMS;
+  if (e0 >= total) return;
+  const int64_t e1 = min(total, e0 + (int64_t)BN_APPLY_ELEMS);
+  // this thread's channel quad is fixed: the step (1024 elements) is a multiple of C
+  const int64_t first = e0 + 4 * threadIdx.x;
+  const int c0 = (int)((first >> 2) % nq) * 4;
+  const int* ws = wsel_override ? wsel_override : d.wsel;
+  const float* P = d.params + (ws ? (int64_t)ws[d.wsel_idx] * d.wsel_stride : 0);
+  float mean[4], sc[4], b[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    mean[u] = d.mean[c0 + u];
+    sc[u] = P[d.off_gamma + c0 + u] * d.inv[c0 + u];
+    b[u] = P[d.off_beta + c0 + u];
+  }
+  const float4* x = reinterpret_cast<const float4*>(d.c);
+  uint2* h = reinterpret_cast<uint2*>(d.h);
+  int64_t e = first;
+  for (; e + 3 * 1024 < e1; e += 4 * 1024) {
+    float4 v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = x[(e + k * 1024) >> 2];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float a0 = fmaxf(fmaf(sc[0], v[k].x - mean[0], b[0]), 0.f);
+      const float a1 = fmaxf(fmaf(sc[1], v[k].y - mean[1], b[1]), 0.f);
+      const float a2 = fmaxf(fmaf(sc[2], v[k].z - mean[2], b[2]), 0.f);
+      const float a3 = fmaxf(fmaf(sc[3], v[k].w - mean[3], b[3]), 0.f);
+      h[(e + k * 1024) >> 2] = make_uint2(pack_bf16(a0, a1), pack_bf16(a2, a3));
+    }
+  }
+  for (; e < e1; e += 1024) {
+    const float4 v = x[e >> 2];
+    const float a0 = fmaxf(fmaf(sc[0], v.x - mean[0], b[0]), 0.f);
+    const float a1 = fmaxf(fmaf(sc[1], v.y - mean[1], b[1]), 0.f);
+    const float a2 = fmaxf(fmaf(sc[2], v.z - mean[2], b[2]), 0.f);
+    const float a3 = fmaxf(fmaf(sc[3], v.w - mean[3], b[3]), 0.f);
+    h[e >> 2] = make_uint2(pack_bf16(a0, a1), pack_bf16(a2, a3));
+  }
 }
 
 // Backward through ReLU and the batch normalisation on channel-last bf16 activations, same
@@ -1633,12 +1749,34 @@ void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
   launch_pdl(ctc::k_relayout_g, dim3(rows, n_indiv), dim3(256), 0, st, src, src_ps, dst, dst_ps, r);
 }
 
+namespace {
+// the apply pass: four channels per thread where the layout allows it
+void bn_apply(const BnDesc* descs, int n_problems, int channels, const int* wsel,
+              int64_t elems, cudaStream_t st) {
+  if (channels % 4 == 0 && channels <= 1024 && 1024 % channels == 0 && elems > 0) {
+    const int64_t blocks = (elems + ctc::BN_APPLY_ELEMS - 1) / ctc::BN_APPLY_ELEMS;
+    launch_pdl(ctc::k_bn_apply_hwc4, dim3((unsigned)blocks, n_problems), dim3(256), 0, st,
+               descs, wsel);
+  } else {
+    const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
+    launch_pdl(ctc::k_bn_apply_hwc, grid, dim3(256), 0, st, descs, wsel);
+  }
+}
+}  // namespace
+
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        float* part, unsigned* counters, cudaStream_t st) {
+                        float* part, unsigned* counters, int64_t elems, cudaStream_t st) {
   const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
   launch_pdl(ctc::k_bn_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels,
              counters);
-  launch_pdl(ctc::k_bn_apply_hwc, grid, dim3(256), 0, st, descs, wsel);
+  bn_apply(descs, n_problems, channels, wsel, elems, st);
+}
+
+void launch_bn_relu_hwc_part(const BnDesc* descs, int n_problems, int channels, const int* wsel,
+                             const float2* part, int slots, int64_t elems, cudaStream_t st) {
+  launch_pdl(ctc::k_bn_finalize_hwc, dim3((channels + 31) / 32, n_problems), dim3(1024), 0, st,
+             descs, part, slots);
+  bn_apply(descs, n_problems, channels, wsel, elems, st);
 }
 
 void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,

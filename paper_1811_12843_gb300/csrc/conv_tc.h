@@ -61,6 +61,11 @@ struct CtcParams {
   const int* wsel;
   float slope;
   int* err;
+  // CTC_F32_HWC: non-null = also the batch-norm statistics of the output: per (tile, 128-row
+  // half, TMEM lane quarter) slot the per-channel sum and sum of squares over its valid rows,
+  // bn_part[slot][co] (slot = (tile * (m2 ? 2 : 1) + half) * 4 + quarter), for
+  // launch_bn_relu_hwc_part
+  float2* bn_part;
 };
 
 // Generator layers 2..5 (n of them): source offsets and sizes [in = ci][out = co][4][4];
@@ -148,11 +153,16 @@ void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
 // Batch normalisation (training mode) + ReLU on fp32 channel-last input into bf16 channel-last
 // output (BnDesc: c, h, mean, inv, params; n images of 2^lhw pixels, C channels); part holds
 // bn_hwc_part_floats(n_problems, channels) floats of per-chunk sums; counters holds
-// bn_hwc_counters(n_problems, channels) zeroed unsigned ints (the launch leaves them zero).
+// bn_hwc_counters(n_problems, channels) zeroed unsigned ints (the launch leaves them zero);
+// elems = the elements of one problem (images x pixels x channels).
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
-                        float* part, unsigned* counters, cudaStream_t st);
+                        float* part, unsigned* counters, int64_t elems, cudaStream_t st);
 // Backward of launch_bn_relu_hwc (BnDesc: c, h, mean, inv, params, dh fp32, dc bf16, dparams),
 // with the same part and counters buffers.
+// The same from statistics that the producing convolution summed into part (bn_part, `slots`
+// slots per problem, consecutive): a finalize launch, then the apply launch.
+void launch_bn_relu_hwc_part(const BnDesc* descs, int n_problems, int channels, const int* wsel,
+                             const float2* part, int slots, int64_t elems, cudaStream_t st);
 void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
                                  float* part, unsigned* counters, cudaStream_t st);
 // The generator's first layer (a 4x4 transposed convolution of the 1x1 noise input) as the

@@ -125,6 +125,9 @@ struct DcPlan {
   bool g1tc = false;
   int64_t g1_off = 0;
   CUtensorMap mG1;
+  // batch-norm statistics of generator layers 2-4 summed in their convolutions' epilogues
+  float2* bnp = nullptr;
+  int bn_slots_e[3] = {0, 0, 0}, bn_slots_t[3] = {0, 0, 0};
   RelayoutG relg;
   CUtensorMap mG[4];
   CtcParams gp[4];
@@ -667,6 +670,19 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       if (l == 5) p->h_gtd5 = vt;
       ok = ok && act_map(&p->aEg[i], &p->gp[i], vt.data(), PE);
     }
+    // the fp32 layers (2-4) sum their batch-norm statistics in the epilogue: slots of
+    // (tile, half, lane quarter), consecutive per problem
+    int64_t bnmax = 0;
+    for (int i = 0; i < 3; ++i) {
+      const CtcParams& q = p->gp[i];
+      bnmax = std::max(bnmax, (int64_t)q.n_tiles * (q.m2 ? 2 : 1) * 4 * q.co);
+    }
+    ok = ok && !dev_alloc(p, &p->bnp, (size_t)bnmax * sizeof(float2), msg);
+    for (int i = 0; i < 3 && ok; ++i) {
+      CtcParams& q = p->gp[i];
+      q.bn_part = p->bnp;
+      p->bn_slots_e[i] = q.n_tiles / PE * (q.m2 ? 2 : 1) * 4;
+    }
   }
   // ---- tensor-core training forward (channel-last), and the output layer's descriptors in
   // the re-laid (tap, channel) order
@@ -689,6 +705,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       ok = ok && !upload(p, &p->tgd[i], vt, msg);
       if (l == 5) p->h_tgd5 = vt;
       ok = ok && act_map(&p->aTg[i], &p->tgp[i], vt.data(), C);
+      if (i < 3)
+        p->bn_slots_t[i] = p->tgp[i].n_tiles / C * (p->tgp[i].m2 ? 2 : 1) * 4;
     }
     for (int l = 1; l <= 4 && ok; ++l) {
       CtcParams q = p->cp[l - 1];
@@ -1042,7 +1060,8 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
       launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
                   nullptr, 0, s.slope, st);
     }
-    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, st);
+    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
+                       st);
     if (p->scg)
       launch_relayout_s((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[12], p->Gs, s.n_indiv, st);
     for (int i = 0; i < 4; ++i) {
@@ -1059,7 +1078,8 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
       }
       if (!launch_conv_tc(p->mG[i], p->aEg[i], q, p->sms, st)) return no_variant(msg);
       if (i < 3)
-        launch_bn_relu_hwc(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnpart, p->bncnt, st);
+        launch_bn_relu_hwc_part(p->ebn[i + 1], PE, gc[i + 2], nbr, p->bnp, p->bn_slots_e[i],
+                                (int64_t)B * gs[i + 2] * gs[i + 2] * gc[i + 2], st);
     }
     return check(msg, "DCGAN generator evaluation (tensor cores)");
   }
@@ -1119,7 +1139,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
     else
       launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
                   nullptr, 0, s.slope, st);
-    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt, st);
+    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
+                       st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->tgp[i];
       q.descs = p->tgd[i];
@@ -1134,7 +1155,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       }
       if (!launch_conv_tc(p->mG[i], p->aTg[i], q, p->sms, st)) return no_variant(msg);
       if (i < 3)
-        launch_bn_relu_hwc(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnpart, p->bncnt, st);
+        launch_bn_relu_hwc_part(p->tbn[i + 1], C, gc[i + 2], nullptr, p->bnp, p->bn_slots_t[i],
+                                (int64_t)B * gs[i + 2] * gs[i + 2] * gc[i + 2], st);
     }
   } else {
     for (int l = 1; l <= 5; ++l) {
