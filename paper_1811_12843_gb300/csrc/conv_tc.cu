@@ -288,7 +288,8 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
     const int lhi = p.lhi, Hi = 1 << lhi;
     if constexpr (kNchw) {
       // first layer (3 channels, 64 x 64 CHW images, 32 x 32 outputs, one k chunk of
-      // k = (ky * 4 + kx) * 3 + c over 48 values): a tile's 128 rows are 4 output rows, fed by
+      // k = c * 16 + ky * 4 + kx over 48 values, the weights' own [out][c][ky][kx] order): a
+      // tile's 128 rows are 4 output rows, fed by
       // a 3 x 10 x 64 input patch that the gather threads copy one tile ahead by 8-byte
       // cp.async into one of three shared buffers whose halo columns stay zero
       uint8_t* patches = misc + 256;
@@ -327,23 +328,22 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
         const unsigned short* pb =
             reinterpret_cast<const unsigned short*>(patches + buf * PATCH_BYTES);
         const uint32_t row = base + stage * STAGE_BYTES + (uint32_t)r * 128u;
+        // group (c, ky) = k / 4: the four kx values are patch columns 2 ox + 3 .. 2 ox + 6 of
+        // patch row c * 10 + 2 oyl + ky, taken from the three aligned words at 2 ox + 2
+        const uint32_t* pw = reinterpret_cast<const uint32_t*>(pb);
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-          uint32_t w[4];
+          uint32_t w[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-          for (int e2 = 0; e2 < 4; ++e2) {
-            uint32_t hv[2];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int k = u * 8 + e2 * 2 + h;
-              hv[h] = 0u;
-              if (k < 48) {
-                const int tap = k / 3, c = k - 3 * tap;
-                const int prow = 2 * oyl + (tap >> 2), col = 2 * ox + (tap & 3) + 3;
-                hv[h] = valid ? (uint32_t)pb[(c * 10 + prow) * 72 + col] : 0u;
-              }
+          for (int hh = 0; hh < 2; ++hh) {
+            const int gidx = 2 * u + hh;  // c * 4 + ky
+            if (gidx < 12 && valid) {
+              const int c = gidx >> 2, ky = gidx & 3;
+              const int e0 = (c * 10 + 2 * oyl + ky) * 72 + 2 * ox + 2;
+              const uint32_t w0 = pw[e0 >> 1], w1 = pw[(e0 >> 1) + 1], w2 = pw[(e0 >> 1) + 2];
+              w[2 * hh] = __byte_perm(w0, w1, 0x5432);
+              w[2 * hh + 1] = __byte_perm(w1, w2, 0x5432);
             }
-            w[e2] = hv[0] | (hv[1] << 16);
           }
           asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
                            row + ((uint32_t)(u ^ (r & 7)) << 4)),
@@ -1734,9 +1734,11 @@ void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
   for (int l = 0; l < r.n; ++l) {
     q.src_off[l] = r.src_off[l];
     q.dst_off[l] = r.dst_off[l];
-    q.o[l] = r.o[l];
+    // a 3-channel tensor is read in its own [out][c][ky][kx] order by the first-layer gather,
+    // straight from src: no rows
+    q.o[l] = r.c[l] == 3 ? 0 : r.o[l];
     q.c[l] = r.c[l];
-    rows += r.o[l];
+    rows += q.o[l];
   }
   launch_pdl(ctc::k_relayout_rows, dim3(rows, n_indiv), dim3(256), 0, st, src, src_ps, dst, dst_ps,
              q);
@@ -2053,7 +2055,8 @@ void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, cons
   for (int l = 0; l < 5; ++l) {
     q.src_off[l] = q.dst_off[l] = r.off[l];
     q.c[l] = r.ci[l];
-    q.o[l] = (int)((r.off[l + 1] - r.off[l]) / (16 * (int64_t)r.ci[l]));
+    // the first layer is read in its own [out][c][ky][kx] order, straight from src: no rows
+    q.o[l] = l == 0 ? 0 : (int)((r.off[l + 1] - r.off[l]) / (16 * (int64_t)r.ci[l]));
     rows += q.o[l];
   }
   launch_pdl(ctc::k_relayout_rows, dim3(rows, n_indiv), dim3(256), 0, st, src, Ps, dst, Ps, q);

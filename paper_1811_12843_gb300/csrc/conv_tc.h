@@ -25,7 +25,8 @@ struct ConvTcDesc {
 };
 
 // A launch: problems of `rows` images; 4x4 / stride 2 / pad 1 convolution from ci x 2^lhi
-// squared to co x 2^lho squared; K = 16 ci in (ky, kx, ci) order, kchunks = ceil(K / 64);
+// squared to co x 2^lho squared; K = 16 ci in (ky, kx, ci) order (the 3-channel first layer:
+// (ci, ky, kx)), kchunks = ceil(K / 64);
 // jobs of nbox = min(co, 256) output channels (nj of them); tiles of 128 output pixels
 // (mtiles per problem). The weight map spans [individual][co][K] bf16. nchw_in: the first
 // layer, which takes only 3-channel channel-major 64 x 64 images (ci 3, lhi 6, lho 5).
@@ -78,7 +79,9 @@ struct RelayoutG {
 };
 
 // Offsets and input channels of the five discriminator tensors inside one individual (P its
-// parameter count): [out][in][ky][kx] -> [out][ky][kx][in].
+// parameter count): [out][in][ky][kx] -> [out][ky][kx][in] for all but the first (3-channel)
+// layer, whose convolution reads its weights in their own order (K = (in, ky, kx)) from the
+// population itself.
 struct RelayoutD {
   int64_t off[6];
   int ci[5];
@@ -142,7 +145,8 @@ void launch_relayout_d(const bf16* src, bf16* dst, int n_indiv, int64_t Ps, cons
 void launch_relayout_g(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_ps, int n_indiv,
                        const RelayoutG& r, cudaStream_t st);
 // [o][c][ky][kx] -> [o][ky][kx][c] for n weight tensors (o rows, c channels each) from
-// src_off to dst_off of every individual.
+// src_off to dst_off of every individual; tensors of 3 channels are left out (the first-layer
+// gather reads them in their own order).
 struct RelayoutC {
   int n;
   int64_t src_off[4], dst_off[4];

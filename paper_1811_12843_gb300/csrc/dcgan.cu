@@ -547,8 +547,9 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     for (int l = 1; l <= 4 && ok; ++l) {
       const int ci = dc[l - 1], co = dc[l];
       const int nbox = co < 256 ? co : 256;
-      ok = ctc_make_map(&p->mW[l - 1], p->Dwt + dof[l - 1], (uint64_t)ci * 16, co, s.n_indiv,
-                        b.PDs, nbox, msg);
+      // the first layer's weights in their own [out][c][ky][kx] order, from the population
+      const bf16* wbase = l == 1 ? (const bf16*)b.Dop + dof[0] : p->Dwt + dof[l - 1];
+      ok = ctc_make_map(&p->mW[l - 1], wbase, (uint64_t)ci * 16, co, s.n_indiv, b.PDs, nbox, msg);
       CtcParams q;
       memset(&q, 0, sizeof q);
       q.rows = 6 * B;
@@ -849,8 +850,13 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     for (int i = 0; i < 4 && ok; ++i) {
       const int l = 5 - i;
       const int co = gc[l - 1], nbox = co < 256 ? co : 256;
-      ok = ctc_make_map(&p->mGc[i], p->Gct + rc.dst_off[i], (uint64_t)16 * gc[l], co, s.n_indiv,
-                        p->gct_ps, nbox, msg);
+      // the output layer's input gradient reads 3-channel images: its weights in their own
+      // [out][c][ky][kx] order, from the population (launch_relayout_c leaves them out)
+      ok = gc[l] == 3
+               ? ctc_make_map(&p->mGc[i], (const bf16*)b.Gop + go[3 * (l - 1)], 48, co,
+                              s.n_indiv, b.PGs, nbox, msg)
+               : ctc_make_map(&p->mGc[i], p->Gct + rc.dst_off[i], (uint64_t)16 * gc[l], co,
+                              s.n_indiv, p->gct_ps, nbox, msg);
       CtcParams q;
       memset(&q, 0, sizeof q);
       q.rows = B;
