@@ -1559,6 +1559,128 @@ __global__ void __launch_bounds__(256) k_bn_back_apply_hwc(const BnDesc* __restr
   }
 }
 
+// The backward passes with four channels per thread (C a multiple of 4 dividing 1024), 1024
+// threads per block, blocks over 4096-element steps: the stats block z of a problem takes steps
+// [S z / 32, S (z + 1) / 32) (S = steps of the problem; the last block also the tail), its
+// threads of one channel quad are added in thread order into part[problem][z][C], and the
+// problem's last block adds the 32 chunks in float64 in chunk order (one counter per problem).
+constexpr int BN_B_THREADS = 1024;
+__global__ void __launch_bounds__(BN_B_THREADS) k_bn_back_stats_hwc4(
+    const BnDesc* __restrict__ descs, float2* __restrict__ part, int cmax,
+    unsigned* __restrict__ counters) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int nq = d.C >> 2;
+  const int64_t m = (int64_t)d.n << d.lhw;
+  const int64_t total = m * d.C, steps = total / 4096;
+  const int z = blockIdx.x;
+  int64_t e = (steps * z / BN_CHUNKS) * 4096 + 4 * threadIdx.x;
+  const int64_t e1 = z == BN_CHUNKS - 1 ? total : (steps * (z + 1) / BN_CHUNKS) * 4096;
+  const int c0 = (4 * threadIdx.x) % d.C;
+  float mean[4], inv[4], sb[4] = {0.f, 0.f, 0.f, 0.f}, sg[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    mean[u] = d.mean[c0 + u];
+    inv[u] = d.inv[c0 + u];
+  }
+  const uint2* h = reinterpret_cast<const uint2*>(d.h);
+  const float4* dh = reinterpret_cast<const float4*>(d.dh);
+  const float4* cc = reinterpret_cast<const float4*>(d.c);
+  for (; e < e1; e += 4096) {
+    const uint2 hv = h[e >> 2];
+    const float4 dv = dh[e >> 2], cv = cc[e >> 2];
+    const float2 h01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hv.x));
+    const float2 h23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hv.y));
+    const float hq[4] = {h01.x, h01.y, h23.x, h23.y};
+    const float dq[4] = {dv.x, dv.y, dv.z, dv.w}, cq[4] = {cv.x, cv.y, cv.z, cv.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float dy = hq[u] > 0.f ? dq[u] : 0.f;
+      sb[u] += dy;
+      sg[u] = fmaf(dy, (cq[u] - mean[u]) * inv[u], sg[u]);
+    }
+  }
+  __shared__ float4 shb[BN_B_THREADS], shg[BN_B_THREADS];
+  __shared__ int is_last;
+  shb[threadIdx.x] = make_float4(sb[0], sb[1], sb[2], sb[3]);
+  shg[threadIdx.x] = make_float4(sg[0], sg[1], sg[2], sg[3]);
+  __syncthreads();
+  float2* pp = part + (int64_t)blockIdx.y * BN_CHUNKS * cmax;
+  if ((int)threadIdx.x < nq) {
+    float4 tb = make_float4(0.f, 0.f, 0.f, 0.f), tg = tb;
+    for (int t = threadIdx.x; t < BN_B_THREADS; t += nq) {
+      const float4 b = shb[t], g = shg[t];
+      tb.x += b.x; tb.y += b.y; tb.z += b.z; tb.w += b.w;
+      tg.x += g.x; tg.y += g.y; tg.z += g.z; tg.w += g.w;
+    }
+    float2* o = pp + (int64_t)z * cmax + 4 * threadIdx.x;
+    o[0] = make_float2(tb.x, tg.x);
+    o[1] = make_float2(tb.y, tg.y);
+    o[2] = make_float2(tb.z, tg.z);
+    o[3] = make_float2(tb.w, tg.w);
+  }
+  __threadfence();
+  __syncthreads();
+  unsigned* cnt = counters + blockIdx.y;
+  if (threadIdx.x == 0) is_last = atomicAdd(cnt, 1u) == BN_CHUNKS - 1;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  for (int ch = threadIdx.x; ch < d.C; ch += BN_B_THREADS) {
+    double tb = 0.0, tg = 0.0;
+    for (int k = 0; k < BN_CHUNKS; ++k) {
+      const float2 v = __ldcg(&pp[(int64_t)k * cmax + ch]);
+      tb += v.x;
+      tg += v.y;
+    }
+    d.dparams[d.off_gamma + ch] = (float)tg;
+    d.dparams[d.off_beta + ch] = (float)tb;
+  }
+  if (threadIdx.x == 0) *cnt = 0u;
+}
+
+// dc = gamma inv (dy - dbeta / m - xhat dgamma / m), four channels per thread, as
+// k_bn_back_apply_hwc; blocks over BN_APPLY_ELEMS elements as k_bn_apply_hwc4.
+__global__ void __launch_bounds__(256) k_bn_back_apply_hwc4(const BnDesc* __restrict__ descs) {
+  pdl_wait();
+  const BnDesc d = descs[blockIdx.y];
+  const int64_t m = (int64_t)d.n << d.lhw;
+  const int64_t total = m * d.C;
+  const int64_t e0 = (int64_t)blockIdx.x * BN_APPLY_ELEMS;
+  if (e0 >= total) return;
+  const int64_t e1 = min(total, e0 + (int64_t)BN_APPLY_ELEMS);
+  const int64_t first = e0 + 4 * threadIdx.x;
+  const int c0 = (int)(first % d.C);
+  const float* P = d.params + (d.wsel ? (int64_t)d.wsel[d.wsel_idx] * d.wsel_stride : 0);
+  float mean[4], inv[4], gi[4], k1[4], k2[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    mean[u] = d.mean[c0 + u];
+    inv[u] = d.inv[c0 + u];
+    gi[u] = P[d.off_gamma + c0 + u] * inv[u];
+    k1[u] = d.dparams[d.off_beta + c0 + u] / (float)m;
+    k2[u] = d.dparams[d.off_gamma + c0 + u] / (float)m;
+  }
+  const uint2* h = reinterpret_cast<const uint2*>(d.h);
+  const float4* dh = reinterpret_cast<const float4*>(d.dh);
+  const float4* cc = reinterpret_cast<const float4*>(d.c);
+  uint2* dc = reinterpret_cast<uint2*>(d.dc);
+  for (int64_t e = first; e < e1; e += 1024) {
+    const uint2 hv = h[e >> 2];
+    const float4 dv = dh[e >> 2], cv = cc[e >> 2];
+    const float2 h01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hv.x));
+    const float2 h23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hv.y));
+    const float hq[4] = {h01.x, h01.y, h23.x, h23.y};
+    const float dq[4] = {dv.x, dv.y, dv.z, dv.w}, cq[4] = {cv.x, cv.y, cv.z, cv.w};
+    float o[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float dy = hq[u] > 0.f ? dq[u] : 0.f;
+      o[u] = gi[u] * (dy - k1[u] - (cq[u] - mean[u]) * inv[u] * k2[u]);
+    }
+    dc[e >> 2] = make_uint2(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]));
+  }
+}
 
 // ---- the generator's first layer on tcgen05 -------------------------------------------------
 // A 4x4 transposed convolution of a 1x1 input is the plain product y[n][(tap, o)] =
@@ -1782,7 +1904,15 @@ void launch_bn_relu_hwc_part(const BnDesc* descs, int n_problems, int channels, 
 }
 
 void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
-                                 float* part, unsigned* counters, cudaStream_t st) {
+                                 float* part, unsigned* counters, int64_t elems, cudaStream_t st) {
+  if (channels % 4 == 0 && channels <= 1024 && 1024 % channels == 0 && elems >= 4096) {
+    launch_pdl(ctc::k_bn_back_stats_hwc4, dim3(ctc::BN_CHUNKS, n_problems),
+               dim3(ctc::BN_B_THREADS), 0, st, descs, (float2*)part, channels, counters);
+    const int64_t blocks = (elems + ctc::BN_APPLY_ELEMS - 1) / ctc::BN_APPLY_ELEMS;
+    launch_pdl(ctc::k_bn_back_apply_hwc4, dim3((unsigned)blocks, n_problems), dim3(256), 0, st,
+               descs);
+    return;
+  }
   const dim3 grid((channels + 31) / 32, n_problems, ctc::BN_CHUNKS);
   launch_pdl(ctc::k_bn_back_stats_hwc, grid, dim3(256), 0, st, descs, (float2*)part, channels,
              counters);

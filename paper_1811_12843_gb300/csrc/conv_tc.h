@@ -161,14 +161,14 @@ void launch_relayout_c(const bf16* src, int64_t src_ps, bf16* dst, int64_t dst_p
 // elems = the elements of one problem (images x pixels x channels).
 void launch_bn_relu_hwc(const BnDesc* descs, int n_problems, int channels, const int* wsel,
                         float* part, unsigned* counters, int64_t elems, cudaStream_t st);
-// Backward of launch_bn_relu_hwc (BnDesc: c, h, mean, inv, params, dh fp32, dc bf16, dparams),
-// with the same part and counters buffers.
 // The same from statistics that the producing convolution summed into part (bn_part, `slots`
 // slots per problem, consecutive): a finalize launch, then the apply launch.
 void launch_bn_relu_hwc_part(const BnDesc* descs, int n_problems, int channels, const int* wsel,
                              const float2* part, int slots, int64_t elems, cudaStream_t st);
+// Backward of launch_bn_relu_hwc (BnDesc: c, h, mean, inv, params, dh fp32, dc bf16, dparams),
+// with the same part and counters buffers; elems = the elements of one problem.
 void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channels,
-                                 float* part, unsigned* counters, cudaStream_t st);
+                                 float* part, unsigned* counters, int64_t elems, cudaStream_t st);
 // The generator's first layer (a 4x4 transposed convolution of the 1x1 noise input) as the
 // product y[n][(tap, o)] = sum_c z[n][c] W[c][o][tap] on tcgen05 (DENSE1 descriptors: a = noise
 // rows [n][ca] bf16, 8-byte aligned; out = fp32 channel-last [n][16 co]; the individual from

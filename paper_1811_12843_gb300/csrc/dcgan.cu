@@ -1274,7 +1274,8 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
                     B * gs[l - 1] * gs[l - 1], gc[l - 1], nullptr, 1, nullptr, 0, s.slope, st);
       }
       if (p->tct)
-        launch_bn_relu_backward_hwc(p->gbn[k], C, gc[l - 1], p->bnpart, p->bncnt, st);
+        launch_bn_relu_backward_hwc(p->gbn[k], C, gc[l - 1], p->bnpart, p->bncnt,
+                                    (int64_t)B * gs[l - 1] * gs[l - 1] * gc[l - 1], st);
       else
         launch_bn_relu_backward(s.bf, p->gbn[k], C, gc[l - 1], st);
     }
