@@ -432,6 +432,11 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
     const int row = q * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     uint32_t* stg = reinterpret_cast<uint32_t*>(misc + 256 + kPatchArea) + (warp - 6) * STG_WORDS;
+    // tma_out (first layer, 64 channels): the tile's 128 rows x 128 bytes go to the staging area
+    // (1024-byte aligned) in the 128-byte swizzle, and one thread stores them by TMA through the
+    // output map (passed as mA, which the first layer's gather does not use)
+    const bool kTmaOut = AK == AK_NCHW && OM == CTC_LRELU_HWC && p.tma_out;
+    const uint32_t tileb = smem_u32(misc + 256 + kPatchArea);
     int uses[2] = {0, 0}, jobs = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
@@ -458,7 +463,7 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
         // the scatter epilogue synchronises the four warps: they leave together
         const bool okw =
             mbar_wait_warp(bAccF + 8 * R, (uint32_t)(uses[R] & 1), abort_flag, p.err, 28);
-        if (kScatter ? epi_bar_or(!okw) : !okw) {
+        if ((kScatter || kTmaOut) ? epi_bar_or(!okw) : !okw) {
           ok = false;
           break;
         }
@@ -552,6 +557,11 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
             oxh = 2 * oxh + (cls & 1);
           }
           const int64_t pix = ((int64_t)(mh >> (2 * lq)) << (2 * p.lho)) + (oyh << p.lho) + oxh;
+          if (kTmaOut) {
+            // the previous tile's store has read the staging area before anyone rewrites it
+            if (threadIdx.x == 192) bulk_wait_read<0>();
+            epi_bar();
+          }
           for (int g = 0; g < nbox / 32; ++g) {
             uint32_t v[32];
             LIPZ_TMEM_LD32(tmem + lane_base + (uint32_t)(R * kAccStride + h * nbox + g * 32), v);
@@ -593,6 +603,18 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
                 b = b > 0.f ? b : p.slope * b;
                 pk[e >> 1] = pack_bf16(a, b);
               }
+            }
+            if (kTmaOut) {
+              // row `row`, 16-byte units 4 g + u of its 128 bytes, in the 128-byte swizzle
+              const uint32_t rb = tileb + (uint32_t)row * 128u;
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                 rb + ((uint32_t)((4 * g + u) ^ (row & 7)) << 4)),
+                             "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]),
+                             "r"(pk[4 * u + 3])
+                             : "memory");
+              continue;
             }
             if constexpr (OM == CTC_LRELU_LOGIT) {
               // the output layer instead of storing the activations
@@ -653,6 +675,15 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
             }
             __syncwarp();
           }
+          if (kTmaOut) {
+            // the four warps' rows are written: one thread stores the tile
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            epi_bar();
+            if (threadIdx.x == 192) {
+              tma_store_3d(&mA, tileb, j * 256, mh - row, pc);
+              bulk_commit();
+            }
+          }
           }
         }
         tc_fence_before();
@@ -667,6 +698,8 @@ __global__ void __launch_bounds__(THREADS, AK == AK_NCHW || AK == AK_TRANS_C ? 2
       }
     }
   }
+  // the last TMA stores of the output have finished before the CTA leaves
+  if (AK == AK_NCHW && OM == CTC_LRELU_HWC && p.tma_out && threadIdx.x == 192) bulk_wait_all();
   __syncwarp();
   tc_fence_before();
   __syncthreads();
@@ -1962,6 +1995,37 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
       *msg = "cuTensorMapEncodeTiled (convolution weights) failed: " + std::to_string((int)r);
     return false;
   }
+  return true;
+}
+
+bool ctc_make_out_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
+                      std::string* msg) {
+  q->tma_out = 0;
+  if (!q->nchw_in || q->out_mode != CTC_LRELU_HWC || q->co != 64 || q->nj != 1 || q->m2 ||
+      n_probs < 1)
+    return true;
+  const int64_t M = (int64_t)q->rows << (2 * q->lho);  // output pixels of a problem
+  if (M % ctc::BM != 0) return true;
+  const int64_t per = M * q->co;
+  int64_t pstride = per;
+  if (n_probs > 1) pstride = (int64_t)(descs[1].out - descs[0].out);
+  if (pstride < per || pstride % 8 != 0 || ((uintptr_t)descs[0].out & 15) != 0) return true;
+  for (int i = 2; i < n_probs; ++i)
+    if ((int64_t)(descs[i].out - descs[0].out) != i * pstride) return true;
+  if (!ensure_encode(msg)) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)q->co, (cuuint64_t)M, (cuuint64_t)n_probs};
+  cuuint64_t strides[2] = {(cuuint64_t)q->co * 2, (cuuint64_t)(pstride * 2)};
+  cuuint32_t box[3] = {64, (cuuint32_t)ctc::BM, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_encode_ctc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, (void*)descs[0].out, dims,
+                            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (convolution output) failed: " + std::to_string((int)r);
+    return false;
+  }
+  q->tma_out = 1;
   return true;
 }
 

@@ -59,6 +59,9 @@ struct CtcParams {
   int m2;
   const bf16* logit_w;  // CTC_LRELU_LOGIT
   int64_t logit_ws;
+  // first layer, CTC_LRELU_HWC, 64 output channels: the output tiles go out by TMA through
+  // the map that ctc_make_out_map builds (passed in place of the activation map)
+  int tma_out;
   const int* wsel;
   float slope;
   int* err;
@@ -130,6 +133,12 @@ bool ctc_make_map(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, u
 // refuses the map.
 bool ctc_make_act_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
                       std::string* msg, bool use_tma = true);
+// Output map of a first-layer launch (nchw_in, CTC_LRELU_HWC, co 64) whose problems' outputs
+// sit at a uniform stride from descs[0].out: dims (64 channels, output pixels, problems), boxes
+// of 128 pixels in the 128-byte swizzle. Sets q->tma_out = 1 when it applies (else 0); false
+// only when the driver refuses the map.
+bool ctc_make_out_map(CUtensorMap* m, CtcParams* q, const ConvTcDesc* descs, int n_probs,
+                      std::string* msg);
 bool ctc_prepare(std::string* msg);
 void launch_scatter_fix(const ConvTcDesc* descs, const float* halo, int n_problems, int rows,
                         int out_mode, cudaStream_t st);

@@ -588,6 +588,8 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       ok = ok && !upload(p, &p->tcd[l - 1], vt, msg);
       // one map serves every cell: the chunk buffers are shared
       ok = ok && act_map(&p->aEd[l - 1], &p->cp[l - 1], vt.data(), 5);
+      // the first layer stores its output by TMA (its gather needs no activation map)
+      if (l == 1) ok = ok && ctc_make_out_map(&p->aEd[0], &p->cp[0], vt.data(), 5, msg);
       for (size_t k = 5; k < vt.size() && ok && l >= 2; ++k)
         if (vt[k].in != vt[k % 5].in) {
           if (msg) *msg = "DCGAN evaluation buffers differ between cells";
@@ -728,6 +730,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       }
       ok = ok && !upload(p, &p->tdd[l - 1], vt, msg);
       ok = ok && act_map(&p->aTd[l - 1], &p->tdp[l - 1], vt.data(), C);
+      if (l == 1) ok = ok && ctc_make_out_map(&p->aTd[0], &p->tdp[0], vt.data(), C, msg);
     }
     std::vector<LogitDesc> vl, vd, vg;
     for (int c = 0; c < C; ++c) {
