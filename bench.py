@@ -668,7 +668,17 @@ def main():
                     help="neighbours seen one iteration late (asynchronous cells)")
     ap.add_argument("--dcgan", action="store_true",
                     help="the 3x3 DCGAN workload (tensor-core convolutions) instead of the MLP")
+    ap.add_argument("--dcgan-grid", default=None, metavar="RxC",
+                    help="with --dcgan: a smaller or larger torus of the same networks (for "
+                         "kernel captures on a small case; not the benchmark configuration)")
     args = ap.parse_args()
+    if args.dcgan_grid:
+        global DC_ROWS, DC_COLS, DC_CELLS, DC_PAIRS, DC_WORKLOAD
+        DC_ROWS, DC_COLS = (int(v) for v in args.dcgan_grid.lower().split("x"))
+        DC_CELLS = DC_ROWS * DC_COLS
+        DC_PAIRS = 25 * DC_CELLS
+        DC_WORKLOAD = ("%dx%d torus DCGAN G/D (512/256/128/64 channels, 64x64x3) bf16 B=128 "
+                       "(%d pairs/iter)" % (DC_ROWS, DC_COLS, DC_PAIRS))
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     if args.dcgan and args.impl == "reference":
