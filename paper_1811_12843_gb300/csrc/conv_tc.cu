@@ -1200,12 +1200,23 @@ __global__ void __launch_bounds__(256) k_wgrad_tc_reduce(const __grid_constant__
   const int m = blockIdx.x / cchunks, c0 = (blockIdx.x - m * cchunks) * 64;
   const int64_t MN = (int64_t)p.M * p.N;
   const float* part = p.part + (int64_t)prob * p.splits * MN + (int64_t)m * p.N + c0;
-  for (int i = threadIdx.x; i < 1024; i += 256) {
-    const int tap = i >> 6, cc = i & 63;
-    const float* src = part + (int64_t)tap * p.Cb + cc;
-    float acc = 0.f;
-    for (int sp = 0; sp < p.splits; ++sp) acc += src[sp * MN];
-    tile[tap][cc] = acc;
+  // the four outputs of a thread, each summed over the splits in split order, with all four
+  // loads of a split issued together
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int sp = 0; sp < p.splits; ++sp) {
+    float v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = threadIdx.x + 256 * u;
+      v[u] = part[(int64_t)sp * MN + (int64_t)(i >> 6) * p.Cb + (i & 63)];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) acc[u] += v[u];
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int i = threadIdx.x + 256 * u;
+    tile[i >> 6][i & 63] = acc[u];
   }
   __syncthreads();
   float* out = p.descs[prob].dw + (int64_t)m * p.N + (int64_t)c0 * 16;
@@ -1854,6 +1865,129 @@ __global__ void k_relayout_g1(const bf16* __restrict__ src, int64_t src_ps, int6
   }
 }
 
+
+// ---- the generator's first-layer weight gradient on tcgen05 ---------------------------------
+// dW1[c][o][tap] = sum_n z[n][c] dc1[n][tap][o], as the product of A = z^T (M = c, padded to
+// 128 with zeros, K = n) and B = dc1 with its columns in (o, tap) order (k_relayout_dc1), both
+// MN-major in the 128-byte swizzle: the noise rows are written into A's atoms by the CTA's
+// threads, B arrives by TMA. One CTA per (256 columns, cell); K = B <= 128 in two chunks; each
+// epilogue thread stores its row's 256 fp32 values, which are contiguous in dW1.
+constexpr int D1W_SMEM = 1024 + 2 * 2 * 8192 + 2 * 4 * 8192 + 64;
+
+__global__ void __launch_bounds__(128) k_dense1_wgrad_tc(const __grid_constant__ CUtensorMap mB,
+                                                         const bf16* __restrict__ z,
+                                                         int64_t z_cell, float* __restrict__ dw,
+                                                         int64_t dw_cell, int rows, int ca, int N,
+                                                         int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sA = base, sB = base + 2 * 16384;  // [chunk][M box][64 k][128 B], [chunk][4][..]
+  uint8_t* misc = gbase + 2 * 16384 + 2 * 32768;
+  const uint32_t bFull = smem_u32(misc), bMma = bFull + 8;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 16);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 20);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * 256, cell = blockIdx.y;
+  if (threadIdx.x == 0) {
+    mbar_init(bFull, 1);
+    mbar_init(bMma, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
+        smem_u32((const void*)tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  if (threadIdx.x == 0) {
+    mbar_expect_tx(bFull, 2u * 4u * 8192u);
+    for (int kc = 0; kc < 2; ++kc)
+      for (int i = 0; i < 4; ++i)
+        tma_load_3d(sB + (uint32_t)(kc * 32768 + i * 8192), &mB, bFull, n0 + 64 * i, kc * 64,
+                    cell);
+  }
+  // A: 16-byte unit u (channels 8u' .. 8u' + 7 of M box b) of k row kr of chunk kc sits at unit
+  // u ^ (kr & 7) of that row; channels past ca and samples past rows are zero
+  {
+    const bf16* zc = z + (int64_t)cell * z_cell;
+    for (int i = threadIdx.x; i < 2 * 2 * 64 * 8; i += 128) {
+      const int u = i & 7, kr = (i >> 3) & 63, b = (i >> 9) & 1, kc = i >> 10;
+      const int n = kc * 64 + kr, c = b * 64 + u * 8;
+      uint2 lo = make_uint2(0u, 0u), hi = make_uint2(0u, 0u);
+      if (n < rows) {
+        const uint2* zr = reinterpret_cast<const uint2*>(zc + (int64_t)n * ca);
+        if (c < ca) lo = zr[c >> 2];
+        if (c + 4 < ca) hi = zr[(c >> 2) + 1];
+      }
+      const uint32_t addr = sA + (uint32_t)(kc * 16384 + b * 8192 + kr * 128) +
+                            ((uint32_t)(u ^ (kr & 7)) << 4);
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(lo.x), "r"(lo.y),
+                   "r"(hi.x), "r"(hi.y)
+                   : "memory");
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (mbar_wait(bFull, 0u, abort_flag, err, 43)) {
+      tc_fence_after();
+      constexpr uint32_t idesc = idesc_bf16_major(BM, 256, 1, 1);
+#pragma unroll
+      for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)
+          tc_mma(tmem, sw128_mn_desc(sA + kc * 16384 + kk * 2048, 8192),
+                 sw128_mn_desc(sB + kc * 32768 + kk * 2048, 8192), idesc, (kc | kk) != 0 ? 1u : 0u);
+      tc_commit(bMma);
+    }
+  }
+  if (mbar_wait_warp(bMma, 0u, abort_flag, err, 44)) {
+    tc_fence_after();
+    const int row = warp * 32 + lane;  // channel c of z
+    float* out = dw + (int64_t)cell * dw_cell + (int64_t)row * N + n0;
+#pragma unroll 1
+    for (int g = 0; g < 16; ++g) {
+      uint32_t r[16];
+      LIPZ_TMEM_LD16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(g * 16), r);
+      tmem_wait_ld();
+      if (row < ca) {
+        float4* o = reinterpret_cast<float4*>(out + g * 16);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          o[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                             __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+}
+
+// dc1 [n][16 taps][co] -> [n][co][16 taps] (bf16), one block per (sample, cell) through shared
+// memory
+__global__ void __launch_bounds__(256) k_relayout_dc1(const bf16* __restrict__ src,
+                                                      int64_t src_cell, bf16* __restrict__ dst,
+                                                      int rows, int co) {
+  extern __shared__ uint8_t smem_dc1[];
+  bf16* sh = reinterpret_cast<bf16*>(smem_dc1);  // [16][co + 2]
+  pdl_wait();
+  const int n = blockIdx.x, cell = blockIdx.y;
+  const bf16* sp = src + (int64_t)cell * src_cell + (int64_t)n * 16 * co;
+  bf16* dp = dst + ((int64_t)cell * rows + n) * 16 * co;
+  for (int i = threadIdx.x; i < 16 * co; i += 256) sh[(i / co) * (co + 2) + (i % co)] = sp[i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < 16 * co; i += 256) dp[i] = sh[(i & 15) * (co + 2) + (i >> 4)];
+}
+
 }  // namespace ctc
 
 bool wgtc_prepare(std::string* msg) {
@@ -2188,12 +2322,41 @@ bool ctc_prepare(std::string* msg) {
       return false;
     }
   if (cudaFuncSetAttribute(ctc::k_dense1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           ctc::D1_SMEM) != cudaSuccess) {
+                           ctc::D1_SMEM) != cudaSuccess ||
+      cudaFuncSetAttribute(ctc::k_dense1_wgrad_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           ctc::D1W_SMEM) != cudaSuccess) {
     cudaGetLastError();
     if (msg) *msg = "cannot reserve shared memory for the generator's first layer";
     return false;
   }
   return true;
+}
+
+bool dense1_wgrad_make_map(CUtensorMap* m, const bf16* dc1t, int rows, int co, int cells,
+                           std::string* msg) {
+  if (!ensure_encode(msg)) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)16 * co, (cuuint64_t)rows, (cuuint64_t)cells};
+  cuuint64_t strides[2] = {(cuuint64_t)16 * co * 2, (cuuint64_t)rows * 16 * co * 2};
+  cuuint32_t box[3] = {64, 64, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_encode_ctc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, (void*)dc1t, dims, strides,
+                            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) *msg = "cuTensorMapEncodeTiled (first-layer deltas) failed: " + std::to_string((int)r);
+    return false;
+  }
+  return true;
+}
+
+void launch_dense1_wgrad_tc(const CUtensorMap& mB, const bf16* z, int64_t z_cell,
+                            const bf16* dc1, int64_t dc1_cell, bf16* dc1t, float* dw,
+                            int64_t dw_cell, int rows, int ca, int co, int cells, int* err,
+                            cudaStream_t st) {
+  launch_pdl(ctc::k_relayout_dc1, dim3(rows, cells), dim3(256), (size_t)16 * (co + 2) * 2, st,
+             dc1, dc1_cell, dc1t, rows, co);
+  launch_pdl(ctc::k_dense1_wgrad_tc, dim3(16 * co / 256, cells), dim3(128),
+             (size_t)ctc::D1W_SMEM, st, mB, z, z_cell, dw, dw_cell, rows, ca, 16 * co, err);
 }
 
 bool dense1_tc_supported(int rows, int ca, int co) {

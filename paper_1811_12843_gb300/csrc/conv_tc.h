@@ -188,6 +188,17 @@ bool dense1_tc_supported(int rows, int ca, int co);
 void launch_dense1_tc(const CUtensorMap& mW, const ConvDesc* descs, int n_problems,
                       const int* wsel_override, int rows, int ca, int co, int* err,
                       cudaStream_t st);
+// The generator's first-layer weight gradient on tcgen05 (the same shape conditions as
+// dense1_tc_supported): dw (fp32 [ca][co][4][4] of each cell, stride dw_cell) = z^T dc1, with
+// z the cells' noise rows [rows][ca] (stride z_cell) and dc1 the layer's batch-norm-backward
+// deltas, channel-last [rows][16][co] (stride dc1_cell); dc1t is a [cells][rows][co][16]
+// scratch that a re-layout launch fills first, and mB its map (dense1_wgrad_make_map).
+bool dense1_wgrad_make_map(CUtensorMap* m, const bf16* dc1t, int rows, int co, int cells,
+                           std::string* msg);
+void launch_dense1_wgrad_tc(const CUtensorMap& mB, const bf16* z, int64_t z_cell,
+                            const bf16* dc1, int64_t dc1_cell, bf16* dc1t, float* dw,
+                            int64_t dw_cell, int rows, int ca, int co, int cells, int* err,
+                            cudaStream_t st);
 // [individual][ca][co][4][4] at src_off (stride src_ps) -> dst [individual][(tap, o)][128]
 // (stride dst_ps), K padded with zeros.
 void launch_relayout_g1(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst,

@@ -125,6 +125,12 @@ struct DcPlan {
   bool g1tc = false;
   int64_t g1_off = 0;
   CUtensorMap mG1;
+  // the generator's first-layer weight gradient on tcgen05: a (o, tap) copy of its deltas
+  bool g1w = false;
+  bf16* dc1t = nullptr;
+  void* dcb = nullptr;  // the generator's batch-norm-backward deltas, [cells][B][gmax]
+  int64_t dcb_cell = 0;
+  CUtensorMap mG1w;
   // batch-norm statistics of generator layers 2-4 summed in their convolutions' epilogues
   float2* bnp = nullptr;
   int bn_slots_e[3] = {0, 0, 0}, bn_slots_t[3] = {0, 0, 0};
@@ -976,6 +982,14 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       ok = ok && !upload(p, &p->wgd[k], vw, msg);
     }
     ok = ok && !dev_alloc(p, &p->wpart, (size_t)wneed * 4, msg);
+    // generator layer 1: z^T times its deltas in (o, tap) order
+    p->g1w = ok && dense1_tc_supported(B, s.z, gc[1]);
+    if (p->g1w) {
+      p->dcb = dcb;
+      p->dcb_cell = (int64_t)B * gmax;
+      ok = !dev_alloc(p, &p->dc1t, (size_t)C * B * 16 * gc[1] * 2, msg) &&
+           dense1_wgrad_make_map(&p->mG1w, p->dc1t, B, gc[1], C, msg);
+    }
   }
   // ---- scatter mode for the 64 -> 3 transposed convolutions (its A tiles always come by TMA:
   // it has no gathered form)
@@ -1262,6 +1276,10 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
       q.descs = p->wgd[k];
       q.part = p->wpart;
       launch_wgrad_tc(p->wgA[k], p->wgB[k], q, p->sms, st);
+    } else if (l == 1 && p->g1w) {
+      launch_dense1_wgrad_tc(p->mG1w, (const bf16*)p->b.Z, (int64_t)B * s.z, (const bf16*)p->dcb,
+                             p->dcb_cell, p->dc1t, p->b.gG + p->b.goff[0], p->b.PGs, B, s.z,
+                             gc[1], C, p->err, st);
     } else {
       launch_conv(WGRAD_MODE, CEPI_NONE_, s.bf, true, p->gw[k], C, gc[l - 1], gc[l] * 16,
                   nullptr, p->splits_gw[k], p->part, p->pstride_gw[k], s.slope, st);
