@@ -1247,8 +1247,11 @@ __global__ void __launch_bounds__(256) k_relayout_rows(const bf16* __restrict__ 
     const int n = c - cb < RL_CH ? c - cb : RL_CH;
     for (int e = threadIdx.x; e < n * 16; e += 256) sh[e & 15][e >> 4] = sp[cb * 16 + e];
     __syncthreads();
+    // (the channel counts are powers of two: a shift instead of a division where they are)
+    const bool pow2 = (n & (n - 1)) == 0;
+    const int ln = __ffs(n) - 1;
     for (int e = threadIdx.x; e < n * 16; e += 256) {
-      const int t = e / n, cc = e - t * n;
+      const int t = pow2 ? e >> ln : e / n, cc = e - t * n;
       dp[t * c + cb + cc] = sh[t][cc];
     }
     __syncthreads();
@@ -1274,8 +1277,10 @@ __global__ void __launch_bounds__(256) k_relayout_g(const bf16* __restrict__ src
     for (int e = threadIdx.x; e < n * 16; e += 256)
       sh[e & 15][e >> 4] = sp[(int64_t)(cb + (e >> 4)) * co * 16 + (e & 15)];
     __syncthreads();
+    const bool pow2 = (n & (n - 1)) == 0;
+    const int ln = __ffs(n) - 1;
     for (int e = threadIdx.x; e < n * 16; e += 256) {
-      const int ct = e / n, cc = e - ct * n;  // (class, tap) = ct
+      const int ct = pow2 ? e >> ln : e / n, cc = e - ct * n;  // (class, tap) = ct
       const int cls = ct >> 2, t = ct & 3;
       const int ky = (((cls >> 1) + 1) & 1) + 2 * (t >> 1);
       const int kx = (((cls & 1) + 1) & 1) + 2 * (t & 1);
