@@ -850,6 +850,9 @@ int eval_impl(lipz_grid* g, const float* xin_dev, bool then_select,
   if (g->dcgan) {
     std::string msg;
     phase_begin(g, LIPZ_PHASE_G_FWD);
+    // stale neighbours read the other snapshot too; otherwise only snapshot p's individuals
+    const bool both = g->a.stale_neighbors && g->prev_valid;
+    dc_set_indiv_range(g->dc, both ? 0 : p * C, both ? 0 : C);
     if (dc_eval_g(g->dc, eval_nbr(g), g->st, &msg))
       return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_G_FWD, dc_eval_launches(g->dc, 0));
@@ -966,6 +969,9 @@ int train_once(lipz_grid* g) {
     // replacement into the next snapshot
     std::string msg;
     phase_begin(g, LIPZ_PHASE_TRAIN_BWD);
+    // the selected individuals come from the evaluation's neighbour table
+    const bool both = g->a.stale_neighbors && g->prev_valid;
+    dc_set_indiv_range(g->dc, both ? 0 : p * C, both ? 0 : C);
     if (dc_train(g->dc, g->st, &msg)) return fail(g, LIPZ_ERR_CUDA, "%s", msg.c_str());
     phase_end(g, LIPZ_PHASE_TRAIN_BWD, dc_train_launches(g->dc));
     phase_begin(g, LIPZ_PHASE_ADAM);

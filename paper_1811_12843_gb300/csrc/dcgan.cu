@@ -131,6 +131,9 @@ struct DcPlan {
   void* dcb = nullptr;  // the generator's batch-norm-backward deltas, [cells][B][gmax]
   int64_t dcb_cell = 0;
   CUtensorMap mG1w;
+  // individuals whose weight copies the next calls need (dc_set_indiv_range): [rl_lo,
+  // rl_lo + rl_n), all when rl_n <= 0
+  int rl_lo = 0, rl_n = 0;
   // batch-norm statistics of generator layers 2-4 summed in their convolutions' epilogues
   float2* bnp = nullptr;
   int bn_slots_e[3] = {0, 0, 0}, bn_slots_t[3] = {0, 0, 0};
@@ -1067,6 +1070,11 @@ int check(std::string* msg, const char* what) {
 }
 }  // namespace
 
+void dc_set_indiv_range(DcPlan* p, int lo, int n) {
+  p->rl_lo = lo;
+  p->rl_n = n;
+}
+
 int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const DcShape& s = p->s;
   const int C = s.cells, B = s.B, g = s.ngf;
@@ -1074,10 +1082,13 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   const int gs[6] = {1, 4, 8, 16, 32, 64};
   const int PE = C * 5;
   if (p->tcg) {
-    launch_relayout_g((const bf16*)p->b.Gop, p->b.PGs, p->Gwt, p->gwt_ps, s.n_indiv, p->relg, st);
+    const int64_t lo = p->rl_n > 0 ? p->rl_lo : 0;
+    const int nI = p->rl_n > 0 ? p->rl_n : s.n_indiv;
+    const bf16* gop = (const bf16*)p->b.Gop + lo * p->b.PGs;
+    launch_relayout_g(gop, p->b.PGs, p->Gwt + lo * p->gwt_ps, p->gwt_ps, nI, p->relg, st);
     if (p->g1tc) {
-      launch_relayout_g1((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[0], p->Gwt + p->g1_off,
-                         p->gwt_ps, s.z, gc[1], s.n_indiv, st);
+      launch_relayout_g1(gop, p->b.PGs, p->b.goff[0], p->Gwt + lo * p->gwt_ps + p->g1_off,
+                         p->gwt_ps, s.z, gc[1], nI, st);
       launch_dense1_tc(p->mG1, p->eg[0], PE, nbr, B, s.z, gc[1], p->err, st);
     } else {
       launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
@@ -1086,7 +1097,7 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
                        st);
     if (p->scg)
-      launch_relayout_s((const bf16*)p->b.Gop, p->b.PGs, p->b.goff[12], p->Gs, s.n_indiv, st);
+      launch_relayout_s(gop, p->b.PGs, p->b.goff[12], p->Gs + lo * 4096, nI, st);
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->gp[i];
       q.descs = p->gtd[i];
@@ -1126,7 +1137,10 @@ int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
   if (p->tc) {
     // weights in the layout the tensor-core convolution reads, for every individual (they
     // change after every training step)
-    launch_relayout_d((const bf16*)p->b.Dop, p->Dwt, s.n_indiv, p->b.PDs, p->rel, st);
+    const int64_t lo = p->rl_n > 0 ? p->rl_lo : 0;
+    const int nI = p->rl_n > 0 ? p->rl_n : s.n_indiv;
+    launch_relayout_d((const bf16*)p->b.Dop + lo * p->b.PDs, p->Dwt + lo * p->b.PDs, nI,
+                      p->b.PDs, p->rel, st);
     for (int c = 0; c < C; ++c) {
       for (int l = 1; l <= 4; ++l) {
         CtcParams q = p->cp[l - 1];
@@ -1215,12 +1229,13 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   launch_dc_dlogit(s.bf, p->tlogits, C, B, p->dl_d, p->dl_g, st);
   if (p->tct) {
     // weights in the layouts the tensor-core input gradients read
-    launch_relayout_g((const bf16*)p->b.Dop, p->b.PDs, p->Ddt, p->ddt_ps, s.n_indiv, p->reld,
-                      st);
-    launch_relayout_c((const bf16*)p->b.Gop, p->b.PGs, p->Gct, p->gct_ps, s.n_indiv, p->relc,
-                      st);
-    if (p->scd)
-      launch_relayout_s((const bf16*)p->b.Dop, p->b.PDs, p->b.doff[0], p->Ds, s.n_indiv, st);
+    const int64_t lo = p->rl_n > 0 ? p->rl_lo : 0;
+    const int nI = p->rl_n > 0 ? p->rl_n : s.n_indiv;
+    const bf16* dop = (const bf16*)p->b.Dop + lo * p->b.PDs;
+    launch_relayout_g(dop, p->b.PDs, p->Ddt + lo * p->ddt_ps, p->ddt_ps, nI, p->reld, st);
+    launch_relayout_c((const bf16*)p->b.Gop + lo * p->b.PGs, p->b.PGs, p->Gct + lo * p->gct_ps,
+                      p->gct_ps, nI, p->relc, st);
+    if (p->scd) launch_relayout_s(dop, p->b.PDs, p->b.doff[0], p->Ds + lo * 4096, nI, st);
   }
   // discriminator backward (D loss)
   launch_logit_back(s.bf, p->tct ? p->tdl_back_d_tc : p->tdl_back_d, C, (int)(8 * d * 16), true,

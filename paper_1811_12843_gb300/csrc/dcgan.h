@@ -57,6 +57,9 @@ void dc_plan_destroy(DcPlan* p);
 // Evaluation forward: every slot's generator on its cell's noise into E's fakes (dc_eval_g),
 // then every slot's discriminator on E[c] into logits (dc_eval_d). nbr [cells][5]: individual
 // of each slot.
+// The individuals [lo, lo + n) whose weights the following evaluation / training reads (the
+// per-iteration weight re-layouts cover only those); n <= 0: all of them.
+void dc_set_indiv_range(DcPlan* p, int lo, int n);
 int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg);
 int dc_eval_d(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg);
 
