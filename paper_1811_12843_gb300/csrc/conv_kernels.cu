@@ -525,6 +525,41 @@ __global__ void k_logit_back(const LogitDesc* __restrict__ descs, int with_dw, f
   const T* a = (const T*)d.a;
   const T* dl = (const T*)d.dl;
   T* da = (T*)d.da;
+  if (sizeof(T) == 2 && (d.K & 1) == 0 && (((uintptr_t)a | (uintptr_t)da) & 3) == 0) {
+    // bf16: two neighbouring k per thread (4-byte loads and stores), eight rows' loads issued
+    // together; each k's sum still runs over the rows in order
+    const int kh = d.K >> 1;
+    for (int k2 = blockIdx.x * blockDim.x + threadIdx.x; k2 < kh; k2 += gridDim.x * blockDim.x) {
+      const int k = 2 * k2;
+      const float w0 = to_f<T>(w[k]), w1 = to_f<T>(w[k + 1]);
+      float s0 = 0.f, s1 = 0.f;
+      const __nv_bfloat162* a2 = reinterpret_cast<const __nv_bfloat162*>(a) + k2;
+      __nv_bfloat162* da2 = reinterpret_cast<__nv_bfloat162*>(da) + k2;
+      for (int r0 = 0; r0 < d.rows; r0 += 8) {
+        float2 av[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          av[u] = r0 + u < d.rows ? __bfloat1622float2(a2[(int64_t)(r0 + u) * kh])
+                                  : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          if (r0 + u >= d.rows) break;
+          const float g = to_f<T>(dl[r0 + u]);
+          s0 = fmaf(g, av[u].x, s0);
+          s1 = fmaf(g, av[u].y, s1);
+          if (da)
+            da2[(int64_t)(r0 + u) * kh] =
+                __floats2bfloat162_rn(av[u].x > 0.f ? g * w0 : slope * g * w0,
+                                      av[u].y > 0.f ? g * w1 : slope * g * w1);
+        }
+      }
+      if (with_dw) {
+        d.dw[d.hwc_c ? (k % d.hwc_c) * 16 + k / d.hwc_c : k] = s0;
+        d.dw[d.hwc_c ? ((k + 1) % d.hwc_c) * 16 + (k + 1) / d.hwc_c : k + 1] = s1;
+      }
+    }
+    return;
+  }
   for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < d.K; k += gridDim.x * blockDim.x) {
     const float wk = to_f<T>(w[k]);
     float s = 0.f;
