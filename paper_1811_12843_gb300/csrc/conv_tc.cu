@@ -1742,10 +1742,29 @@ __global__ void __launch_bounds__(256) k_bn_back_apply_hwc4(const BnDesc* __rest
 constexpr int D1_THREADS = 128;
 constexpr int D1_SMEM = 1024 + 2 * A_BYTES + 2 * B_BYTES + 64;
 
+// Sum of v over the 32 lanes of a warp for 16 columns, reduce-scattered: lanes 2j and 2j + 1
+// return the sum of column j (a fixed tree of lane exchanges).
+__device__ __forceinline__ float colsum16(const float (&v)[16], int lane) {
+  float a8[8], a4[4], a2[2];
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    a8[i] = (b4 ? v[8 + i] : v[i]) + __shfl_xor_sync(0xffffffffu, b4 ? v[i] : v[8 + i], 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    a4[i] = (b3 ? a8[4 + i] : a8[i]) + __shfl_xor_sync(0xffffffffu, b3 ? a8[i] : a8[4 + i], 8);
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+    a2[i] = (b2 ? a4[2 + i] : a4[i]) + __shfl_xor_sync(0xffffffffu, b2 ? a4[i] : a4[2 + i], 4);
+  const float a1 = (b1 ? a2[1] : a2[0]) + __shfl_xor_sync(0xffffffffu, b1 ? a2[0] : a2[1], 2);
+  return a1 + __shfl_xor_sync(0xffffffffu, a1, 1);
+}
+
 __global__ void __launch_bounds__(D1_THREADS) k_dense1_tc(const __grid_constant__ CUtensorMap mW,
                                                           const ConvDesc* __restrict__ descs,
                                                           const int* __restrict__ wsel_override,
-                                                          int rows, int ca, int N, int* err) {
+                                                          int rows, int ca, int N, int* err,
+                                                          float2* __restrict__ bn_part) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -1818,7 +1837,12 @@ __global__ void __launch_bounds__(D1_THREADS) k_dense1_tc(const __grid_constant_
       tc_commit(bMma);
     }
   }
-  if (mbar_wait_warp(bMma, 0u, abort_flag, err, 42)) {
+  // bn_part: the batch-norm sums of this tile's 256 channels of one tap over the problem's rows
+  // (rows past `rows` are zero products): per warp by colsum16 into shared memory (the
+  // operand buffers, free once the accumulator is ready), then the four warps in order
+  float2* red = reinterpret_cast<float2*>(gbase);  // [4 warps][256]
+  const bool mma_ok = mbar_wait_warp(bMma, 0u, abort_flag, err, 42);
+  if (mma_ok) {
     tc_fence_after();
     const int row = warp * 32 + lane;
     float* out = (float*)d.out + (int64_t)row * N + n0;
@@ -1833,6 +1857,32 @@ __global__ void __launch_bounds__(D1_THREADS) k_dense1_tc(const __grid_constant_
         for (int q = 0; q < 4; ++q)
           o[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
                              __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+      }
+      if (bn_part) {
+        float v[16], v2[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          v[e] = __uint_as_float(r[e]);
+          v2[e] = v[e] * v[e];
+        }
+        const float cs = colsum16(v, lane), cq = colsum16(v2, lane);
+        if (!(lane & 1)) red[warp * 256 + g * 16 + (lane >> 1)] = make_float2(cs, cq);
+      }
+    }
+  }
+  if (bn_part) {
+    __syncthreads();
+    if (mma_ok) {
+      const int co = N >> 4, tap = n0 / co, o0 = n0 - tap * co;
+      float2* pp = bn_part + ((int64_t)blockIdx.y * 16 + tap) * co + o0;
+      for (int c = threadIdx.x; c < 256; c += D1_THREADS) {
+        float2 t = red[c];
+#pragma unroll
+        for (int w = 1; w < 4; ++w) {
+          t.x += red[w * 256 + c].x;
+          t.y += red[w * 256 + c].y;
+        }
+        pp[c] = t;
       }
     }
   }
@@ -2371,10 +2421,11 @@ bool dense1_tc_supported(int rows, int ca, int co) {
 
 void launch_dense1_tc(const CUtensorMap& mW, const ConvDesc* descs, int n_problems,
                       const int* wsel_override, int rows, int ca, int co, int* err,
-                      cudaStream_t st) {
+                      cudaStream_t st, float2* bn_part) {
   if (n_problems <= 0) return;
   launch_pdl(ctc::k_dense1_tc, dim3(16 * co / 256, n_problems), dim3(ctc::D1_THREADS),
-             (size_t)ctc::D1_SMEM, st, mW, descs, wsel_override, rows, ca, 16 * co, err);
+             (size_t)ctc::D1_SMEM, st, mW, descs, wsel_override, rows, ca, 16 * co, err,
+             bn_part);
 }
 
 void launch_relayout_g1(const bf16* src, int64_t src_ps, int64_t src_off, bf16* dst,

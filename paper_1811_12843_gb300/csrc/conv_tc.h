@@ -183,11 +183,12 @@ void launch_bn_relu_backward_hwc(const BnDesc* descs, int n_problems, int channe
 // rows [n][ca] bf16, 8-byte aligned; out = fp32 channel-last [n][16 co]; the individual from
 // wsel_override or the descriptor's wsel). mW maps the [individual][16 co][128] copy of
 // launch_relayout_g1 (ctc_make_map, K 128, box 256 rows). rows <= 128, ca <= 128 and a multiple
-// of 4, 16 co a multiple of 256 (dense1_tc_supported).
+// of 4, 16 co a multiple of 256 (dense1_tc_supported). bn_part (nullable): the batch-norm sums
+// of the output, [problem][16 taps][co] float2, for launch_bn_relu_hwc_part with 16 slots.
 bool dense1_tc_supported(int rows, int ca, int co);
 void launch_dense1_tc(const CUtensorMap& mW, const ConvDesc* descs, int n_problems,
                       const int* wsel_override, int rows, int ca, int co, int* err,
-                      cudaStream_t st);
+                      cudaStream_t st, float2* bn_part = nullptr);
 // The generator's first-layer weight gradient on tcgen05 (the same shape conditions as
 // dense1_tc_supported): dw (fp32 [ca][co][4][4] of each cell, stride dw_cell) = z^T dc1, with
 // z the cells' noise rows [rows][ca] (stride z_cell) and dc1 the layer's batch-norm-backward

@@ -684,7 +684,7 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
     }
     // the fp32 layers (2-4) sum their batch-norm statistics in the epilogue: slots of
     // (tile, half, lane quarter), consecutive per problem
-    int64_t bnmax = 0;
+    int64_t bnmax = p->g1tc ? (int64_t)PE * 16 * gc[1] : 0;  // layer 1: a slot per tap
     for (int i = 0; i < 3; ++i) {
       const CtcParams& q = p->gp[i];
       bnmax = std::max(bnmax, (int64_t)q.n_tiles * (q.m2 ? 2 : 1) * 4 * q.co);
@@ -1089,13 +1089,15 @@ int dc_eval_g(DcPlan* p, const int* nbr, cudaStream_t st, std::string* msg) {
     if (p->g1tc) {
       launch_relayout_g1(gop, p->b.PGs, p->b.goff[0], p->Gwt + lo * p->gwt_ps + p->g1_off,
                          p->gwt_ps, s.z, gc[1], nI, st);
-      launch_dense1_tc(p->mG1, p->eg[0], PE, nbr, B, s.z, gc[1], p->err, st);
+      // (its epilogue sums the batch-norm statistics: 16 slots, one per tap)
+      launch_dense1_tc(p->mG1, p->eg[0], PE, nbr, B, s.z, gc[1], p->err, st, p->bnp);
+      launch_bn_relu_hwc_part(p->ebn[0], PE, gc[1], nbr, p->bnp, 16, (int64_t)B * 16 * gc[1], st);
     } else {
       launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->eg[0], PE, B, 16 * gc[1], nbr, 1,
                   nullptr, 0, s.slope, st);
+      launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
+                         st);
     }
-    launch_bn_relu_hwc(p->ebn[0], PE, gc[1], nbr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
-                       st);
     if (p->scg)
       launch_relayout_s(gop, p->b.PGs, p->b.goff[12], p->Gs + lo * 4096, nI, st);
     for (int i = 0; i < 4; ++i) {
@@ -1171,13 +1173,16 @@ int dc_train(DcPlan* p, cudaStream_t st, std::string* msg) {
   const int ds[5] = {64, 32, 16, 8, 4};
   // forward of the selected pair
   if (p->tct) {
-    if (p->g1tc)
-      launch_dense1_tc(p->mG1, p->tg[0], C, nullptr, B, s.z, gc[1], p->err, st);
-    else
+    if (p->g1tc) {
+      launch_dense1_tc(p->mG1, p->tg[0], C, nullptr, B, s.z, gc[1], p->err, st, p->bnp);
+      launch_bn_relu_hwc_part(p->tbn[0], C, gc[1], nullptr, p->bnp, 16, (int64_t)B * 16 * gc[1],
+                              st);
+    } else {
       launch_conv(DENSE1_MODE, CEPI_NONE_, true, true, p->tg[0], C, B, 16 * gc[1], nullptr, 1,
                   nullptr, 0, s.slope, st);
-    launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt, (int64_t)B * 16 * gc[1],
-                       st);
+      launch_bn_relu_hwc(p->tbn[0], C, gc[1], nullptr, p->bnpart, p->bncnt,
+                         (int64_t)B * 16 * gc[1], st);
+    }
     for (int i = 0; i < 4; ++i) {
       CtcParams q = p->tgp[i];
       q.descs = p->tgd[i];
