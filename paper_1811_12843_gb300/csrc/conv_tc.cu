@@ -1140,9 +1140,11 @@ __global__ void __launch_bounds__(256) k_scatter_fix(const ConvTcDesc* __restric
   const ConvTcDesc d = descs[pi / rows];
   const int img = pi % rows;
   const float* h = halo + (int64_t)pi * 8 * 768;
+  // element i: column gx = i mod 64 (neighbouring threads write neighbouring columns), then
+  // channel o, then halo row t and block boundary k
   for (int i = threadIdx.x; i < 9 * 2 * 64 * 3; i += 256) {
-    const int k = i / 384, rem = i - k * 384, t = rem / 192, rem2 = rem - t * 192;
-    const int gx = rem2 / 3, o = rem2 - gx * 3;
+    const int gx = i & 63, r = i >> 6;  // r = (k * 2 + t) * 3 + o
+    const int kt = r / 3, o = r - 3 * kt, k = kt >> 1, t = kt & 1;
     const int gy = 8 * k - 1 + t;
     if (gy < 0 || gy > 63) continue;
     float x = 0.f;
