@@ -485,7 +485,37 @@ __global__ void k_logit_dot(const LogitDesc* __restrict__ descs,
   const T* w = (const T*)d.w + (ws ? (int64_t)ws[d.wsel_idx] * d.wsel_stride : 0);
   const T* x = (const T*)d.a + (int64_t)r * d.K;
   float s = 0.f;
-  for (int k = lane; k < d.K; k += 32) s = fmaf(to_f<T>(x[k]), to_f<T>(w[k]), s);
+  if (sizeof(T) == 2 && (d.K & 255) == 0 && (((uintptr_t)x | (uintptr_t)w) & 15) == 0) {
+    // bf16: eight consecutive k per lane and load (16 bytes), four loads of each operand in
+    // flight; lane l takes k = 256 i + 8 l .. + 7 in order
+    const uint4* x4 = reinterpret_cast<const uint4*>(x) + lane;
+    const uint4* w4 = reinterpret_cast<const uint4*>(w) + lane;
+    const int n = d.K >> 8;
+    for (int i0 = 0; i0 < n; i0 += 4) {
+      uint4 xv[4], wv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u < n) {
+          xv[u] = x4[(i0 + u) * 32];
+          wv[u] = w4[(i0 + u) * 32];
+        }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (i0 + u >= n) break;
+        const uint32_t xa[4] = {xv[u].x, xv[u].y, xv[u].z, xv[u].w};
+        const uint32_t wa[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 xf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xa[e]));
+          const float2 wf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wa[e]));
+          s = fmaf(xf.x, wf.x, s);
+          s = fmaf(xf.y, wf.y, s);
+        }
+      }
+    }
+  } else {
+    for (int k = lane; k < d.K; k += 32) s = fmaf(to_f<T>(x[k]), to_f<T>(w[k]), s);
+  }
 #pragma unroll
   for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if (lane == 0) d.logits[r] = s;

@@ -907,16 +907,17 @@ DcPlan* dc_plan_create(const DcShape& s, const DcBuffers& b, std::string* msg) {
       const int64_t Kp = (int64_t)q.rows << (2 * q.la);
       const int64_t chunks = (Kp + 63) / 64;
       const int64_t per = (int64_t)C * ((q.M + 127) / 128) * (q.b_chw ? 1 : q.N / 256);
-      int best = 1;
-      double be = 0;
-      for (int sp = 1; sp <= 64 && sp <= std::max<int64_t>(1, chunks / 8); ++sp) {
+      // the fewest splits whose wave fill is within 3 % of the best: every split adds an
+      // M x N fp32 partial to write and read back
+      const int sp_max = (int)std::min<int64_t>(64, std::max<int64_t>(1, chunks / 8));
+      auto fill = [&](int sp) {
         const int64_t t = per * sp;
-        const double e = (double)t / ((double)((t + p->sms - 1) / p->sms) * p->sms);
-        if (e > be + 1e-9) {
-          be = e;
-          best = sp;
-        }
-      }
+        return (double)t / ((double)((t + p->sms - 1) / p->sms) * p->sms);
+      };
+      double be = 0;
+      for (int sp = 1; sp <= sp_max; ++sp) be = std::max(be, fill(sp));
+      int best = 1;
+      while (best < sp_max && fill(best) < 0.97 * be) ++best;
       q.kc = (chunks + best - 1) / best * 64;
       q.splits = (int)((Kp + q.kc - 1) / q.kc);
       q.n_tiles = (int)(per * q.splits);
