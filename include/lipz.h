@@ -212,6 +212,17 @@ LIPZ_API int lipz_iterate(lipz_grid* g, int n_iters);
 LIPZ_API int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* fit_d);
 
 /*
+ * The same, pipelined across calls: while this iteration computes, x_next (host, the same
+ * shape, nullable) is uploaded into a second device staging buffer (allocated on the first
+ * call, cells x batch x x_dim fp32), and the next call whose x_host is that same address
+ * skips its upload. The caller must keep x_next's contents unchanged until that call; a call
+ * with another x_host (or lipz_iterate_batch) uploads as usual and the early copy is dropped.
+ * Results, errors and synchronisation as lipz_iterate_batch.
+ */
+LIPZ_API int lipz_iterate_batch_next(lipz_grid* g, const float* x_host, const float* x_next,
+                                     float* fit_g, float* fit_d);
+
+/*
  * State I/O (checkpoint / resume, and state exchange with other implementations). Layout,
  * little-endian: a 64-byte header {u32 magic 0x5A50494C, u32 version 2, i32 rows, cols, z_dim,
  * hidden, x_dim, batch, precision, 0, i64 t, u64 seed, 8 zero bytes}, then f32 Gw[cells][PG],

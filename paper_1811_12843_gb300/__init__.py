@@ -16,7 +16,8 @@ __all__ = [
     "LipzError", "lipz_arch", "arch_default", "library_path", "load",
     "lipz_arch_default", "lipz_grid_create", "lipz_grid_destroy", "lipz_set_stream",
     "lipz_synchronize", "lipz_set_data", "lipz_eval_neighborhoods", "lipz_select_replace",
-    "lipz_train_step", "lipz_iterate", "lipz_iterate_batch", "lipz_state_bytes",
+    "lipz_train_step", "lipz_iterate", "lipz_iterate_batch", "lipz_iterate_batch_next",
+    "lipz_state_bytes",
     "lipz_export_state", "lipz_import_state", "lipz_get_iteration", "lipz_get_batch",
     "lipz_get_logits", "lipz_get_gradients", "lipz_get_mixture", "lipz_profile_enable",
     "lipz_profile_read",
@@ -74,6 +75,7 @@ _SIGS = {
     "lipz_train_step": (_I, [_P]),
     "lipz_iterate": (_I, [_P, _I]),
     "lipz_iterate_batch": (_I, [_P, _P, _P, _P]),
+    "lipz_iterate_batch_next": (_I, [_P, _P, _P, _P, _P]),
     "lipz_state_bytes": (_I, [_P, ctypes.POINTER(ctypes.c_size_t)]),
     "lipz_export_state": (_I, [_P, _P, ctypes.c_size_t]),
     "lipz_import_state": (_I, [_P, _P, ctypes.c_size_t]),
@@ -181,6 +183,12 @@ def lipz_iterate(g, n_iters):
 
 def lipz_iterate_batch(g, x_host, fit_g=None, fit_d=None):
     return _check(g, load().lipz_iterate_batch(g, _ptr(x_host), _ptr(fit_g), _ptr(fit_d)))
+
+
+def lipz_iterate_batch_next(g, x_host, x_next=None, fit_g=None, fit_d=None):
+    """lipz_iterate_batch that uploads the next call's minibatch (x_next) while this one runs."""
+    return _check(g, load().lipz_iterate_batch_next(g, _ptr(x_host), _ptr(x_next), _ptr(fit_g),
+                                                    _ptr(fit_d)))
 
 
 def lipz_state_bytes(g) -> int:

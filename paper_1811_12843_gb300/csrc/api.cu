@@ -56,6 +56,12 @@ struct lipz_grid {
   cudaStream_t own_st = nullptr;  // the grid's own non-blocking stream (the default)
   cudaStream_t copy_st = nullptr;  // host minibatch uploads, overlapping the generator forward
   cudaEvent_t ev_x = nullptr;      // the upload of the caller's minibatch has landed
+  // lipz_iterate_batch_next: a second staging buffer (allocated on first use) and the
+  // minibatch uploaded ahead into buffer pre_buf (0: xin, 1: xin2) from host address pre_host
+  float* xin2 = nullptr;
+  cudaEvent_t ev_x2 = nullptr;
+  const float* pre_host = nullptr;
+  int pre_buf = -1;
   int* hstat = nullptr;            // pinned host copies of the device error flags
   int device = 0;
   // population snapshots: ping-pong pair, or three in rotation with stale neighbours (the
@@ -1281,6 +1287,7 @@ int lipz_grid_destroy(lipz_grid* g) {
     cudaStreamDestroy(g->copy_st);
   }
   if (g->ev_x) cudaEventDestroy(g->ev_x);
+  if (g->ev_x2) cudaEventDestroy(g->ev_x2);
   if (g->hstat) cudaFreeHost(g->hstat);
   delete g;
   return LIPZ_OK;
@@ -1386,6 +1393,8 @@ int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* f
   if (!g) return LIPZ_ERR_INVALID;
   if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
   const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
+  g->pre_buf = -1;  // (a minibatch uploaded ahead into the same buffer is superseded)
+  g->pre_host = nullptr;
   // the upload runs on the copy stream while the noise and the generator forward compute
   CK(g, cudaMemcpyAsync(g->xin, x_host, bytes, cudaMemcpyHostToDevice, g->copy_st));
   CK(g, cudaEventRecord(g->ev_x, g->copy_st));
@@ -1395,6 +1404,51 @@ int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* f
   if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
   if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
   return check_flag(g);  // one stream synchronisation for the results and the flags
+}
+
+int lipz_iterate_batch_next(lipz_grid* g, const float* x_host, const float* x_next,
+                            float* fit_g, float* fit_d) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
+  const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
+  if (!g->xin2) {
+    int rc;
+    if ((rc = dalloc(g, &g->xin2, bytes))) return rc;
+    CK(g, cudaEventCreateWithFlags(&g->ev_x2, cudaEventDisableTiming));
+  }
+  float* const buf[2] = {g->xin, g->xin2};
+  const cudaEvent_t ev[2] = {g->ev_x, g->ev_x2};
+  // this iteration's minibatch: uploaded during the previous call, or now
+  int cur;
+  if (g->pre_buf >= 0 && g->pre_host == x_host) {
+    cur = g->pre_buf;
+  } else {
+    cur = g->pre_buf >= 0 ? 1 - g->pre_buf : 0;
+    CK(g, cudaMemcpyAsync(buf[cur], x_host, bytes, cudaMemcpyHostToDevice, g->copy_st));
+    CK(g, cudaEventRecord(ev[cur], g->copy_st));
+  }
+  g->pre_buf = -1;
+  g->pre_host = nullptr;
+  // the next one into the other buffer, behind it on the copy stream, while this iteration
+  // computes (the other buffer's last reader, the previous iteration, has finished: every call
+  // returns after its iteration is complete)
+  if (x_next) {
+    const int nb = 1 - cur;
+    CK(g, cudaMemcpyAsync(buf[nb], x_next, bytes, cudaMemcpyHostToDevice, g->copy_st));
+    CK(g, cudaEventRecord(ev[nb], g->copy_st));
+    g->pre_buf = nb;
+    g->pre_host = x_next;
+  }
+  int rc;
+  if ((rc = eval_impl(g, buf[cur], true, ev[cur])) || (rc = train_impl(g))) {
+    g->pre_buf = -1;
+    g->pre_host = nullptr;
+    return rc;
+  }
+  const size_t C = g->cells;
+  if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
+  if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
+  return check_flag(g);
 }
 
 int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {

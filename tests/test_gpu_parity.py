@@ -284,6 +284,34 @@ def test_host_batch_iteration(L):
     assert max_rel(got.Dm, new.Dm) < 1e-4
 
 
+def test_host_batch_pipelined_equals_one_call_at_a_time(L):
+    """lipz_iterate_batch_next uploads the next call's minibatch while the current iteration
+    runs; a sequence of calls (cycling two pinned buffers, then a call whose x_host is not the
+    announced one, then plain calls mixed in) ends in the same state and fitnesses as the same
+    minibatches through lipz_iterate_batch, bit for bit."""
+    import torch
+    import lipz_synth
+    pool = _pool(3, 2000, 784)
+    a = _grid(L, 3, 3, 12, pool, precision="bf16")
+    b = _grid(L, 3, 3, 12, pool, precision="bf16")
+    xs = [torch.from_numpy(lipz_synth.host_batch(40 + i, 9, 100)).pin_memory() for i in range(3)]
+    order = [0, 1, 0, 1, 2, 0, 1]
+    fa = [np.zeros((9, 5), np.float32) for _ in range(2)]
+    fb = [np.zeros((9, 5), np.float32) for _ in range(2)]
+    for i, k in enumerate(order):
+        # call 4 announces xs[0] but is followed by xs[2]; call 5 is a plain call
+        nxt = xs[order[i + 1]] if i + 1 < len(order) else None
+        if i == 3:
+            nxt = xs[0]
+        if i == 5:
+            L.lipz_iterate_batch(a.h, xs[k], fa[0], fa[1])
+        else:
+            L.lipz_iterate_batch_next(a.h, xs[k], nxt, fa[0], fa[1])
+        L.lipz_iterate_batch(b.h, xs[k], fb[0], fb[1])
+        assert np.array_equal(fa[0], fb[0]) and np.array_equal(fa[1], fb[1]), i
+    assert a.export_state() == b.export_state()
+
+
 def test_determinism_and_resume(L):
     pool = _pool(4, 2000, 784)
     a = _grid(L, 3, 3, 21, pool, precision="bf16")
