@@ -56,27 +56,28 @@ TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
 # Mixture step (--mixture): the Gram matrix of every cell's 6B evaluation rows.
 MIX_FLOP = 2 * CELLS * (6 * BATCH) ** 2 * X_DIM
 # The backward kernel applies Adam to the weight matrices (G: W1, W2, W3; D: W1, W2) in its
-# epilogue: per such parameter it reads the old w, m, v (12 B) and writes the new w, m, v and
-# the bf16 copy (14 B). Its other algorithmic reads: the bf16 weights of the four matrices the
+# epilogue, and to the remaining parameters (both networks' biases, D's output layer) once a
+# cell's tiles are done: per parameter it reads the old w, m, v (12 B) and writes the new w, m,
+# v and the bf16 copy (14 B), plus the fp32 gradient of the remaining ones (4 B). Its other algorithmic reads: the bf16 weights of the four matrices the
 # delta chain multiplies by (D: W2, W1; G: W3, W2) and the stored forward activations
 # (J2 3B x h, TG1 2B x h, TX 2B x x, TH1 and TH2 B x h, Z B x z), all bf16.
 W_FUSED = (Z_DIM * HIDDEN + HIDDEN * HIDDEN + X_DIM * HIDDEN) + (HIDDEN * X_DIM + HIDDEN * HIDDEN)
 BWD_ACT = (3 * BATCH * HIDDEN + 2 * BATCH * HIDDEN + 2 * BATCH * X_DIM + 2 * BATCH * HIDDEN
            + BATCH * Z_DIM)
-TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN)
-                           + 2 * BWD_ACT)
+W_RANGES = (HIDDEN + HIDDEN + X_DIM) + (HIDDEN + HIDDEN + HIDDEN + 1)  # biases, D's W3 and b3
+TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 30 * W_RANGES
+                           + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN) + 2 * BWD_ACT)
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels: not
 # measured by this script but taken from ncu captures (dram__bytes_read.sum +
 # dram__bytes_write.sum) of these same kernels, each with the summary it comes from. A phase
 # whose kernels changed after its capture has no entry (null traffic).
 PHASE_TRAFFIC = {
-    "train_bwd": (2193.5e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
+    "train_bwd": (2203.5e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
     "d_fwd": (236.7e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
     "g_fwd": (143.8e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
     "batch": (21.2e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
     "fitness": (1.8e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
-    "adam": (3.6e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
 }
 
 

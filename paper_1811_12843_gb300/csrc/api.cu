@@ -599,6 +599,8 @@ int alloc_pops(lipz_grid* g, PopView* p, int64_t Ps) {
   return LIPZ_OK;
 }
 
+void bias_ranges(lipz_grid* g, int p, AdamRanges* rg, AdamRanges* rd);
+
 int create_impl(lipz_grid* g) {
   const int C = g->cells, B = g->a.batch, z = g->a.z_dim, h = g->a.hidden, x = g->a.x_dim;
   const size_t es = g->esz;
@@ -776,6 +778,9 @@ int create_impl(lipz_grid* g) {
       b.beta1 = g->a.beta1;
       b.beta2 = g->a.beta2;
       b.eps = g->a.eps;
+      AdamRanges rr[2];
+      bias_ranges(g, p, &rr[0], &rr[1]);
+      b.ranges = b.fuse_adam ? rr : nullptr;
       std::string msg;
       g->tcb[p] = tcb_plan_create(s, b, &msg);
       if (!g->tcb[p]) return fail(g, LIPZ_ERR_CUDA, "tensor-core backward plan: %s", msg.c_str());
@@ -965,6 +970,33 @@ int select_impl(lipz_grid* g) {
   return LIPZ_OK;
 }
 
+// The Adam ranges left over when the weight matrices take their step inside the backward:
+// the biases of both networks and D's output layer, from snapshot p into the next one.
+void bias_ranges(lipz_grid* g, int p, AdamRanges* rg, AdamRanges* rd) {
+  *rg = AdamRanges{};
+  *rd = AdamRanges{};
+  rg->old_p = g->G[0];
+  rg->new_p = g->G[snap_next(g, p)];
+  rg->grad = g->gG;
+  rg->src = g->src_g;
+  rg->coef = g->coef_g;
+  rg->Ps = g->PGs;
+  rd->old_p = g->D[0];
+  rd->new_p = g->D[snap_next(g, p)];
+  rd->grad = g->gD;
+  rd->src = g->src_d;
+  rd->coef = g->coef_d;
+  rd->Ps = g->PDs;
+  for (int k : {1, 3, 5}) {
+    rg->off[rg->n] = g->lg.off[k];
+    rg->len[rg->n++] = (int)(g->lg.off[k + 1] - g->lg.off[k]);
+  }
+  for (int k : {1, 3, 4, 5}) {
+    rd->off[rd->n] = g->ld.off[k];
+    rd->len[rd->n++] = (int)(g->ld.off[k + 1] - g->ld.off[k]);
+  }
+}
+
 // One Adam step of every cell's chosen pair (sel/src/coef) from snapshot cur into the other
 // snapshot, which becomes cur.
 int train_once(lipz_grid* g) {
@@ -1039,32 +1071,8 @@ int train_once(lipz_grid* g) {
     phase_end(g, LIPZ_PHASE_TRAIN_BWD, 1);
     phase_begin(g, LIPZ_PHASE_ADAM);
     if (!g->a.keep_grads) {
-      // the weight matrices took their Adam step inside the backward: the biases and D's
-      // output layer remain
-      AdamRanges rg{}, rd{};
-      rg.old_p = g->G[0];
-      rg.new_p = g->G[snap_next(g, p)];
-      rg.grad = g->gG;
-      rg.src = g->src_g;
-      rg.coef = g->coef_g;
-      rg.Ps = g->PGs;
-      rd.old_p = g->D[0];
-      rd.new_p = g->D[snap_next(g, p)];
-      rd.grad = g->gD;
-      rd.src = g->src_d;
-      rd.coef = g->coef_d;
-      rd.Ps = g->PDs;
-      for (int k : {1, 3, 5}) {
-        rg.off[rg.n] = g->lg.off[k];
-        rg.len[rg.n++] = (int)(g->lg.off[k + 1] - g->lg.off[k]);
-      }
-      for (int k : {1, 3, 4, 5}) {
-        rd.off[rd.n] = g->ld.off[k];
-        rd.len[rd.n++] = (int)(g->ld.off[k + 1] - g->ld.off[k]);
-      }
-      launch_adam_ranges(rg, rd, C, g->a.beta1, g->a.beta2, g->a.eps, g->st);
-      CKL(g);
-      phase_end(g, LIPZ_PHASE_ADAM, 1);
+      // every Adam step (weight matrices, biases, D's output layer) ran inside the backward
+      phase_end(g, LIPZ_PHASE_ADAM, 0);
       g->cur = snap_next(g, p);
       return LIPZ_OK;
     }

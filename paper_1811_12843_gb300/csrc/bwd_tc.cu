@@ -98,6 +98,19 @@ struct GParams {
   int* err;
 };
 
+// OR of pred over the eight epilogue warps (named barrier 1, 256 threads); also orders their
+// earlier global stores before their later loads.
+__device__ __forceinline__ bool epi_any(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 256, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)pred)
+      : "memory");
+  return r != 0;
+}
+
 __device__ __forceinline__ float dact(int act, float y, float slope) {
   switch (act) {
     case ACT_RELU: return y > 0.f ? 1.f : 0.f;
@@ -128,6 +141,11 @@ struct CellPlan {
   Stage st[MAX_STAGES];
   int n_stages, tiles_per_cell, pub_per_cell, cells;
   int* err;
+  // fused Adam: the biases' and D's output layer's step, applied by the epilogue warps to each
+  // cell once its tiles are done (all of its gradients are then in gG / gD)
+  int has_ranges;
+  AdamRanges rg, rd;
+  float beta1, beta2, eps;
 };
 
 struct StageMaps {
@@ -703,7 +721,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     int lt = 0, pub = 0;
     int cj = 0;  // Adam chunks of this thread's row half so far
     int btile = 0;  // bias-summing tiles so far
-    for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
+    for (int cell = blockIdx.x; cell < cp.cells; cell += gridDim.x) {
       for (int si = 0; si < cp.n_stages && ok; ++si) {
         const GParams& p = cp.st[si].p;
         const bool publish = cp.st[si].publish != 0;
@@ -763,6 +781,37 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
           }
         }
       }
+      if (FUSED && cp.has_ranges) {
+        // the cell's last tile is done by every epilogue thread (its bias sums are in gG / gD):
+        // the remaining Adam ranges of the cell, the eight warps together (they leave
+        // together when any of them gave up)
+        if (epi_any(!ok)) {
+          ok = false;
+          break;
+        }
+        const int et = threadIdx.x - 64;
+        for (int pp = 0; pp < 2; ++pp) {
+          const AdamRanges& r = pp ? cp.rd : cp.rg;
+          const int s = __ldg(&r.src[cell]);
+          const float4 cf = __ldg(&r.coef[cell]);
+          if (et == 0) {
+            r.new_p.step[cell] = (int)cf.w;
+            r.new_p.lr[cell] = cf.x;
+          }
+          const int64_t so = (int64_t)s * r.Ps, co = (int64_t)cell * r.Ps;
+          for (int q = 0; q < r.n; ++q)
+            for (int i = et; i < r.len[q]; i += EPI_THREADS) {
+              const int64_t k = r.off[q] + i;
+              float w = r.old_p.w[so + k], m = r.old_p.m[so + k], v = r.old_p.v[so + k];
+              adam_elem(w, m, v, r.grad[co + k], cp.beta1, cp.beta2, cf.x, cf.y, cf.z, cp.eps);
+              r.new_p.w[co + k] = w;
+              r.new_p.m[co + k] = m;
+              r.new_p.v[co + k] = v;
+              if (r.new_p.wb) r.new_p.wb[co + k] = __float2bfloat16_rn(w);
+            }
+        }
+      }
+      if (!ok) break;
     }
   }
   __syncwarp();
@@ -1179,6 +1228,14 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     P->cells.err = P->err;
     P->grid_cells = C < sms ? C : sms;
     P->fused = b.fuse_adam != 0;
+    P->cells.has_ranges = P->fused && b.ranges ? 1 : 0;
+    if (P->cells.has_ranges) {
+      P->cells.rg = b.ranges[0];
+      P->cells.rd = b.ranges[1];
+      P->cells.beta1 = b.beta1;
+      P->cells.beta2 = b.beta2;
+      P->cells.eps = b.eps;
+    }
     const cudaError_t e =
         P->fused ? cudaFuncSetAttribute(tcb::k_bwd_cells<true>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -9,6 +9,8 @@
 
 #include <string>
 
+#include "engine.h"
+
 namespace lipz {
 
 struct TcbShape {
@@ -48,6 +50,9 @@ struct TcbBuffers {
     const float4* coef;
   } adam_g, adam_d;
   float beta1, beta2, eps;
+  // with fuse_adam: the remaining ranges (biases, D's output layer) of G and D, [2]; each CTA
+  // applies them to its cell after the cell's last tile
+  const AdamRanges* ranges;
 };
 
 struct TcbPlan;

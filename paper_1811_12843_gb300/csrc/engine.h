@@ -182,7 +182,8 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
                  const float4* coef, int cells, int64_t P, int64_t Ps, float beta1, float beta2,
                  float eps, cudaStream_t st);
 
-// Adam + replacement restricted to n parameter ranges [off[q], off[q] + len[q]) of every cell.
+// Adam + replacement restricted to n parameter ranges [off[q], off[q] + len[q]) of every cell
+// (applied by the tensor-core backward to each cell after its last tile).
 struct AdamRanges {
   PopView old_p, new_p;
   const float* grad;
@@ -193,7 +194,6 @@ struct AdamRanges {
   int64_t off[8];
   int len[8];
 };
-void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, float beta1,
-                        float beta2, float eps, cudaStream_t st);
+
 
 }  // namespace lipz

@@ -789,40 +789,6 @@ void launch_adam(const PopView& old_p, const PopView& new_p, const float* grad, 
              eps);
 }
 
-// Adam + replacement of listed parameter ranges only (the tensors whose update is not fused
-// into the tensor-core backward: biases and D's output layer), both populations in one launch:
-// block (cell, population), one thread per parameter. Also writes the new snapshot's step and
-// learning rate.
-__global__ void __launch_bounds__(256) k_adam_ranges(AdamRanges r0, AdamRanges r1, float beta1,
-                                                      float beta2, float eps) {
-  pdl_wait();
-  const AdamRanges& r = blockIdx.y ? r1 : r0;
-  const int c = blockIdx.x;
-  const int s = r.src[c];
-  const float4 cf = r.coef[c];
-  if (threadIdx.x == 0) {
-    r.new_p.step[c] = (int)cf.w;
-    r.new_p.lr[c] = cf.x;
-  }
-  const int64_t so = (int64_t)s * r.Ps, co = (int64_t)c * r.Ps;
-  for (int q = 0; q < r.n; ++q) {
-    for (int i = threadIdx.x; i < r.len[q]; i += blockDim.x) {
-      const int64_t k = r.off[q] + i;
-      float w = r.old_p.w[so + k], m = r.old_p.m[so + k], v = r.old_p.v[so + k];
-      adam_elem(w, m, v, r.grad[co + k], beta1, beta2, cf.x, cf.y, cf.z, eps);
-      r.new_p.w[co + k] = w;
-      r.new_p.m[co + k] = m;
-      r.new_p.v[co + k] = v;
-      if (r.new_p.wb) r.new_p.wb[co + k] = __float2bfloat16_rn(w);
-    }
-  }
-}
-
-void launch_adam_ranges(const AdamRanges& g, const AdamRanges& d, int cells, float beta1,
-                        float beta2, float eps, cudaStream_t st) {
-  launch_pdl(k_adam_ranges, dim3(cells, 2), dim3(256), 0, st, g, d, beta1, beta2, eps);
-}
-
 // ------------------------------------------------------------------------------------------
 // Generator-mixture score (Section 3 step 4): squared norms of the evaluation rows, the Gaussian
 // kernel's block sums (from a stored Gram matrix on the CUDA-core path), and the ES-(1+1) step.
