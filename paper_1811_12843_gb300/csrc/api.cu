@@ -573,14 +573,18 @@ int check_arch(const lipz_arch* a) {
 
 // All snapshots of one population in one allocation per array (snapshot s at s * cells
 // individuals), so that an individual index k = snapshot * cells + cell addresses any of them.
+// w, m and v are three equal parts of one allocation (m = w + n, v = w + 2n floats), so that
+// one 4-D tensor map reaches all three at once (the backward's fused Adam moves a chunk of
+// each with a single TMA load and a single store).
 int alloc_pops(lipz_grid* g, PopView* p, int64_t Ps) {
   const size_t C = g->cells, S = g->nsnap, n = S * C * Ps;
   PopView& a = p[0];
   int rc;
-  if ((rc = dalloc(g, &a.w, n * 4)) || (rc = dalloc(g, &a.m, n * 4)) ||
-      (rc = dalloc(g, &a.v, n * 4)) || (rc = dalloc(g, &a.step, S * C * 4)) ||
+  if ((rc = dalloc(g, &a.w, 3 * n * 4)) || (rc = dalloc(g, &a.step, S * C * 4)) ||
       (rc = dalloc(g, &a.lr, S * C * 4)))
     return rc;
+  a.m = a.w + n;
+  a.v = a.w + 2 * n;
   a.wb = nullptr;
   if (g->bf && (rc = dalloc(g, &a.wb, n * 2))) return rc;
   if ((rc = dset(g, a.w, 0, n * 4)) || (rc = dset(g, a.m, 0, n * 4)) ||

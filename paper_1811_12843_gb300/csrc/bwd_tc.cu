@@ -38,7 +38,10 @@ constexpr int BIAS_PART_BYTES = 2 * 4 * 256 * 4;
 // fused Adam: a chunk is 64 rows (one half of a tile) x 32 fp32 columns of each of w, m, v (one
 // 128-byte row each, 128-byte swizzle), updated in place, plus the new bf16 copy (64-byte rows,
 // no swizzle). Chunks alternate between the two row halves, so each half of the epilogue
-// works through its own two of the four buffers.
+// works through its own two of the four buffers. w, m and v lie a fixed distance apart in
+// memory, so that one TMA box {32, 64, 1, 3} of a 4-D map moves the chunk's three arrays: a
+// tiled TMA operation holds its issuing thread for about 0.2 us whatever its size up to 16 KB,
+// so one box per array made the issuing thread, not the bytes, bound the stream.
 constexpr int ADAM_COLS = 32;
 constexpr int ADAM_ROWS = 64;
 constexpr int ADAM_ARRAY_BYTES = ADAM_ROWS * ADAM_COLS * 4;            // 8 KB
@@ -46,12 +49,12 @@ constexpr int ADAM_WB_BYTES = ADAM_ROWS * ADAM_COLS * 2;               // 4 KB
 constexpr int ADAM_BUF_BYTES = 3 * ADAM_ARRAY_BYTES + ADAM_WB_BYTES;   // 28 KB
 
 // Without fused Adam: four operand stages. With it: two operand stages, four Adam chunk
-// buffers and one more warp (the Adam loader). One CTA per SM either way.
+// buffers and two more warps (the Adam stream's loader and storer). One CTA per SM either way.
 template <bool FUSED>
 struct Cfg {
   static constexpr int STAGES = FUSED ? 2 : 4;
   static constexpr int ADAM_BUFS = FUSED ? 4 : 0;
-  static constexpr int THREADS = 64 + EPI_THREADS + (FUSED ? 32 : 0);
+  static constexpr int THREADS = 64 + EPI_THREADS + (FUSED ? 64 : 0);
   static constexpr int SMEM =
       1024 + STAGES * STAGE_BYTES + ADAM_BUFS * ADAM_BUF_BYTES + 256 + BIAS_PART_BYTES;
 };
@@ -134,12 +137,12 @@ struct Stage {
   int dep;      // stage whose output this one reads (-1: none)
   int tile0;    // tiles of the cell before this stage
   int publish;  // a later stage reads this one's output: its tiles are published and counted
-  int pub_end;  // published tiles of the cell up to and including this stage
 };
 
 struct CellPlan {
   Stage st[MAX_STAGES];
   int n_stages, tiles_per_cell, pub_per_cell, cells;
+  int pub_end[MAX_STAGES];  // tiles of the cell published by the end of stage k
   int* err;
   // fused Adam: the biases' and D's output layer's step, applied by the epilogue warps to each
   // cell once its tiles are done (all of its gradients are then in gG / gD)
@@ -151,9 +154,9 @@ struct CellPlan {
 struct StageMaps {
   CUtensorMap a[MAX_STAGES];
   CUtensorMap b[MAX_STAGES];
-  CUtensorMap aw[MAX_STAGES], am[MAX_STAGES], av[MAX_STAGES];  // old w, m, v (EPI_ADAM stages)
-  CUtensorMap nw[MAX_STAGES], nm[MAX_STAGES], nv[MAX_STAGES];  // new w, m, v
-  CUtensorMap nb[MAX_STAGES];                                  // new bf16 copy
+  CUtensorMap ao[MAX_STAGES];  // old w, m, v (EPI_ADAM stages): {in, out, individual, array}
+  CUtensorMap an[MAX_STAGES];  // new w, m, v: {in, out, cell, array}
+  CUtensorMap nb[MAX_STAGES];  // new bf16 copy
 };
 
 __device__ __forceinline__ void stage_tile(const GParams& p, int t, int& m0, int& n0, int& n) {
@@ -460,6 +463,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
   const uint32_t aFull = bEpi + 16;   // [4] Adam chunk buffers: old values landed
   const uint32_t aDone = aFull + 32;  // [4] new values written back by the epilogue half
   const uint32_t bSum = aDone + 32;   // [2] bias partial sums written, by bias tile
+  const uint32_t aFree = bSum + 16;   // [4] the stores have read the buffer
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(misc + 224);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 228);
   volatile int* done_tiles = reinterpret_cast<volatile int*>(misc + 232);
@@ -481,6 +485,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
     for (int b = 0; b < Cfg<FUSED>::ADAM_BUFS; ++b) {
       mbar_init(aFull + 8 * b, 1);
       mbar_init(aDone + 8 * b, EPI_THREADS / 2);
+      mbar_init(aFree + 8 * b, 1);
     }
     mbar_init(bSum, EPI_THREADS);
     mbar_init(bSum + 8, EPI_THREADS);
@@ -516,7 +521,7 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
           const int dep = cp.st[si].dep;
           if (dep >= 0) {
             // the stage reads the output of stage `dep` of this cell: wait for its last tile
-            const int need = cells_done * cp.pub_per_cell + cp.st[dep].pub_end;
+            const int need = cells_done * cp.pub_per_cell + cp.pub_end[dep];
             const unsigned long long t0 = globaltimer();
             uint32_t it = 0;
             while (*done_tiles < need) {
@@ -642,29 +647,20 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
       volatile int never = 0;
       mbar_wait(bFinal, 0u, &never, err, 14);
     }
-  } else if (FUSED && warp == 2 + NUM_EPI_WARPS) {
-    // ===== Adam loader: old w, m, v of every chunk of every EPI_ADAM tile, in tile order, and
-    // the TMA stores of each chunk's new w, m, v and bf16 copy once the epilogue is done =====
+  } else if (FUSED && warp >= 2 + NUM_EPI_WARPS) {
+    // ===== Adam stream: the old w, m, v of every chunk of every EPI_ADAM tile, in tile order,
+    // into the four buffers in turn, and the new w, m, v and bf16 copy back out. A tiled TMA
+    // operation holds its issuing thread for about 0.2 us, so two warps share the work:
+    //   loader: a chunk's load, once the storer has released the chunk's buffer;
+    //   storer: a chunk's two stores once its epilogue half is done, then, when the stores
+    //           have read the buffer, its release to the loader (releasing it one chunk later,
+    //           to keep a store group in flight, was slower: the stream is bound by the
+    //           latency of each buffer's round trip). =====
+    const bool storer = warp == 3 + NUM_EPI_WARPS;
     if (lane == 0) {
       constexpr int NB = Cfg<FUSED>::ADAM_BUFS > 0 ? Cfg<FUSED>::ADAM_BUFS : 1;
-      int buf = 0, issued[NB] = {}, pend_si[NB] = {}, pend_x[NB] = {}, pend_m[NB] = {};
-      int pend_c[NB] = {};
-      bool has[NB] = {};
+      int buf = 0, uses[NB] = {};
       bool ok = true;
-      // store the chunk held by buffer b once its epilogue half has written it back
-      auto flush = [&](int b) -> bool {
-        if (!mbar_wait(aDone + 8 * b, (uint32_t)((issued[b] - 1) & 1), abort_flag, err, 19))
-          return false;
-        const int si = pend_si[b];
-        const uint32_t bb = sAdam + (uint32_t)(b * ADAM_BUF_BYTES);
-        tma_store_3d(&maps.nw[si], bb, pend_x[b], pend_m[b], pend_c[b]);
-        tma_store_3d(&maps.nm[si], bb + ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
-        tma_store_3d(&maps.nv[si], bb + 2 * ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
-        tma_store_3d(&maps.nb[si], bb + 3 * ADAM_ARRAY_BYTES, pend_x[b], pend_m[b], pend_c[b]);
-        bulk_commit();
-        has[b] = false;
-        return true;
-      };
       for (int cell = blockIdx.x; cell < cp.cells && ok; cell += gridDim.x) {
         for (int si = 0; si < cp.n_stages && ok; ++si) {
           const GParams& p = cp.st[si].p;
@@ -675,44 +671,45 @@ __global__ void __launch_bounds__(Cfg<FUSED>::THREADS, 1)
             const int m0 = (t / p.ntiles) * BM, n0 = (t % p.ntiles) * p.BN;
             const int nch = (min(p.BN, p.N - n0) + ADAM_COLS - 1) / ADAM_COLS;
             for (int k = 0; k < 2 * nch; ++k) {
-              if (has[buf]) {
-                if (!flush(buf)) {
+              const int x0 = n0 + (k >> 1) * ADAM_COLS, y0 = m0 + (k & 1) * ADAM_ROWS;
+              const uint32_t bb = sAdam + (uint32_t)(buf * ADAM_BUF_BYTES);
+              if (storer) {
+                // the (uses[buf] + 1)-th chunk of this buffer is written back
+                if (!mbar_wait(aDone + 8 * buf, (uint32_t)(uses[buf] & 1), abort_flag, err, 19)) {
                   ok = false;
                   break;
                 }
+                tma_store_4d(&maps.an[si], bb, x0, y0, cell, 0);
+                tma_store_3d(&maps.nb[si], bb + 3 * ADAM_ARRAY_BYTES, x0, y0, cell);
+                bulk_commit();
                 bulk_wait_read<0>();  // the stores have read the buffer: it may be refilled
+                mbar_arrive(aFree + 8 * buf);
+              } else {
+                if (uses[buf] > 0 && !mbar_wait(aFree + 8 * buf, (uint32_t)((uses[buf] - 1) & 1),
+                                                abort_flag, err, 21)) {
+                  ok = false;
+                  break;
+                }
+                const uint32_t full = aFull + 8 * buf;
+                mbar_expect_tx(full, (uint32_t)(3 * ADAM_ARRAY_BYTES));
+                tma_load_4d(bb, &maps.ao[si], full, x0, y0, zi, 0);
               }
-              const uint32_t full = aFull + 8 * buf;
-              mbar_expect_tx(full, (uint32_t)(3 * ADAM_ARRAY_BYTES));
-              const uint32_t dst = sAdam + (uint32_t)(buf * ADAM_BUF_BYTES);
-              const int x0 = n0 + (k >> 1) * ADAM_COLS, y0 = m0 + (k & 1) * ADAM_ROWS;
-              tma_load_3d(dst, &maps.aw[si], full, x0, y0, zi);
-              tma_load_3d(dst + ADAM_ARRAY_BYTES, &maps.am[si], full, x0, y0, zi);
-              tma_load_3d(dst + 2 * ADAM_ARRAY_BYTES, &maps.av[si], full, x0, y0, zi);
-              issued[buf]++;
-              has[buf] = true;
-              pend_si[buf] = si;
-              pend_x[buf] = x0;
-              pend_m[buf] = y0;
-              pend_c[buf] = cell;
+              uses[buf]++;
               if (++buf == NB) buf = 0;
             }
           }
         }
       }
-      // the last chunks, oldest first
-      for (int i = 0; i < NB && ok; ++i) {
-        if (has[buf] && !flush(buf)) ok = false;
-        if (++buf == NB) buf = 0;
-      }
-      if (!ok) {
+      if (storer) {
+        bulk_wait_all();
+      } else if (!ok) {
+        // loads issued here land on this CTA's barriers: wait for them before it leaves
         for (int b = 0; b < NB; ++b)
-          if (issued[b] > 0) {
+          if (uses[b] > 0) {
             volatile int never = 0;
-            mbar_wait(aFull + 8 * b, (uint32_t)((issued[b] - 1) & 1), &never, err, 19);
+            mbar_wait(aFull + 8 * b, (uint32_t)((uses[b] - 1) & 1), &never, err, 19);
           }
       }
-      bulk_wait_all();
     }
   } else {
     const int ew = warp - 2, q = warp & 3, hf = ew >> 2;
@@ -862,19 +859,20 @@ bool map3(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint6
   return true;
 }
 
-// fp32 3-D map over one weight tensor [out][in] of every individual: {in, out, individuals},
-// box {32, 64, 1} (one 128-byte row per output row), 128-byte swizzle.
-bool map3f(CUtensorMap* m, const float* base, uint64_t inner, uint64_t rows, uint64_t depth,
-           uint64_t depth_elems, std::string* msg) {
-  cuuint64_t dims[3] = {inner, rows, depth};
-  cuuint64_t strides[2] = {inner * 4, depth_elems * 4};
-  cuuint32_t box[3] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::ADAM_ROWS, 1};
-  cuuint32_t es[3] = {1, 1, 1};
-  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(base), dims,
+// fp32 4-D map over one weight tensor [out][in] of w, m and v of every individual: {in, out,
+// individuals, array}, the arrays `part` floats apart; box {32, 64, 1, 3} (the three arrays'
+// 64 x 128-byte boxes one after another in shared memory), 128-byte swizzle.
+bool map4f(CUtensorMap* m, const float* base, uint64_t inner, uint64_t rows, uint64_t depth,
+           uint64_t depth_elems, uint64_t part, std::string* msg) {
+  cuuint64_t dims[4] = {inner, rows, depth, 3};
+  cuuint64_t strides[3] = {inner * 4, depth_elems * 4, part * 4};
+  cuuint32_t box[4] = {(cuuint32_t)tcb::ADAM_COLS, (cuuint32_t)tcb::ADAM_ROWS, 1, 3};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  CUresult r = g_enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(base), dims,
                      strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
-    if (msg) *msg = "cuTensorMapEncodeTiled (fp32) failed (" + std::to_string((int)r) + ")";
+    if (msg) *msg = "cuTensorMapEncodeTiled (fp32, 4-D) failed (" + std::to_string((int)r) + ")";
     return false;
   }
   return true;
@@ -918,8 +916,8 @@ bool map4(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint6
 
 struct Gemm {
   CUtensorMap a, b;
-  CUtensorMap aw, am, av;      // old w, m, v of the tensor (fused Adam), by individual
-  CUtensorMap nw, nm, nv, nb;  // new w, m, v and bf16 copy, by cell
+  CUtensorMap ao;      // old w, m, v of the tensor (fused Adam), by individual and array
+  CUtensorMap an, nb;  // new w, m, v by cell and array; new bf16 copy by cell
   tcb::GParams p;
   int grid;
 };
@@ -1001,12 +999,17 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
     G.p.adam.beta1 = b.beta1;
     G.p.adam.beta2 = b.beta2;
     G.p.adam.eps = b.eps;
-    ok = ok && map3f(&G.aw, a.w + off, G.p.N, G.p.M, NI, Ps, msg) &&
-         map3f(&G.am, a.m + off, G.p.N, G.p.M, NI, Ps, msg) &&
-         map3f(&G.av, a.v + off, G.p.N, G.p.M, NI, Ps, msg) &&
-         map3f(&G.nw, a.w_new + off, G.p.N, G.p.M, C, Ps, msg) &&
-         map3f(&G.nm, a.m_new + off, G.p.N, G.p.M, C, Ps, msg) &&
-         map3f(&G.nv, a.v_new + off, G.p.N, G.p.M, C, Ps, msg) &&
+    // w, m, v are one allocation in three equal parts: the part size is the 4th dimension's
+    // stride, the same for the old and the new snapshot
+    const int64_t part = a.m - a.w;
+    if (part <= 0 || a.v - a.m != part || a.m_new - a.w_new != part ||
+        a.v_new - a.m_new != part) {
+      if (msg) *msg = "fused Adam needs w, m, v at equal distances";
+      ok = false;
+      return;
+    }
+    ok = ok && map4f(&G.ao, a.w + off, G.p.N, G.p.M, NI, Ps, part, msg) &&
+         map4f(&G.an, a.w_new + off, G.p.N, G.p.M, C, Ps, part, msg) &&
          map3b_rows(&G.nb, a.wb_new + off, G.p.N, G.p.M, C, Ps, msg);
   };
 
@@ -1206,12 +1209,8 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
       const int nt = P->g[k].p.mtiles * P->g[k].p.ntiles;
       P->maps.a[k] = P->g[k].a;
       P->maps.b[k] = P->g[k].b;
-      P->maps.aw[k] = P->g[k].aw;
-      P->maps.am[k] = P->g[k].am;
-      P->maps.av[k] = P->g[k].av;
-      P->maps.nw[k] = P->g[k].nw;
-      P->maps.nm[k] = P->g[k].nm;
-      P->maps.nv[k] = P->g[k].nv;
+      P->maps.ao[k] = P->g[k].ao;
+      P->maps.an[k] = P->g[k].an;
       P->maps.nb[k] = P->g[k].nb;
       P->cells.st[k].p = P->g[k].p;
       P->cells.st[k].dep = deps[k];
@@ -1219,7 +1218,7 @@ TcbPlan* tcb_plan_create(const TcbShape& s, const TcbBuffers& b, std::string* ms
       P->cells.st[k].publish = publish;
       tile0 += nt;
       if (publish) pub += nt;
-      P->cells.st[k].pub_end = pub;
+      P->cells.pub_end[k] = pub;
     }
     P->cells.n_stages = i;
     P->cells.tiles_per_cell = tile0;
