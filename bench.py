@@ -46,15 +46,8 @@ WORKLOAD = "12x12 torus MLP G/D bf16 B=100 (3600 pairs/iter)"
 #   5 * 6B rows x (x*h + h*h + h) MACs per cell.
 G_MAC_ROW = Z_DIM * HIDDEN + HIDDEN * HIDDEN + HIDDEN * X_DIM            # 282,624
 D_MAC_ROW = X_DIM * HIDDEN + HIDDEN * HIDDEN + HIDDEN                    # 266,496
-EVAL_G_FLOP = 2 * CELLS * 5 * BATCH * G_MAC_ROW
-EVAL_D_FLOP = 2 * CELLS * 30 * BATCH * D_MAC_ROW
 PG = HIDDEN * Z_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + X_DIM * HIDDEN + X_DIM
 PD = HIDDEN * X_DIM + HIDDEN + HIDDEN * HIDDEN + HIDDEN + HIDDEN + 1
-# Training: forward of the selected pair (G layers 1-2 on B rows, D on 2B rows) and backward.
-TRAIN_FWD_FLOP = 2 * CELLS * BATCH * (Z_DIM * HIDDEN + HIDDEN * HIDDEN) + 2 * CELLS * 2 * BATCH * D_MAC_ROW
-TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
-# Mixture step (--mixture): the Gram matrix of every cell's 6B evaluation rows.
-MIX_FLOP = 2 * CELLS * (6 * BATCH) ** 2 * X_DIM
 # The backward kernel applies Adam to the weight matrices (G: W1, W2, W3; D: W1, W2) in its
 # epilogue, and to the remaining parameters (both networks' biases, D's output layer) once a
 # cell's tiles are done: per parameter it reads the old w, m, v (12 B) and writes the new w, m,
@@ -65,15 +58,35 @@ W_FUSED = (Z_DIM * HIDDEN + HIDDEN * HIDDEN + X_DIM * HIDDEN) + (HIDDEN * X_DIM 
 BWD_ACT = (3 * BATCH * HIDDEN + 2 * BATCH * HIDDEN + 2 * BATCH * X_DIM + 2 * BATCH * HIDDEN
            + BATCH * Z_DIM)
 W_RANGES = (HIDDEN + HIDDEN + X_DIM) + (HIDDEN + HIDDEN + HIDDEN + 1)  # biases, D's W3 and b3
-TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 30 * W_RANGES
-                           + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN) + 2 * BWD_ACT)
+
+
+def _derive():
+    """The per-iteration work of a ROWS x COLS torus (module globals, so that --grid can set a
+    smaller torus for kernel captures)."""
+    global CELLS, PAIRS, EVAL_G_FLOP, EVAL_D_FLOP, TRAIN_FWD_FLOP, TRAIN_BWD_FLOP, MIX_FLOP
+    global TRAIN_BWD_BYTES
+    CELLS = ROWS * COLS
+    PAIRS = 25 * CELLS
+    EVAL_G_FLOP = 2 * CELLS * 5 * BATCH * G_MAC_ROW
+    EVAL_D_FLOP = 2 * CELLS * 30 * BATCH * D_MAC_ROW
+    # Training: forward of the selected pair (G layers 1-2 on B rows, D on 2B rows), backward.
+    TRAIN_FWD_FLOP = (2 * CELLS * BATCH * (Z_DIM * HIDDEN + HIDDEN * HIDDEN)
+                      + 2 * CELLS * 2 * BATCH * D_MAC_ROW)
+    TRAIN_BWD_FLOP = 2 * CELLS * BATCH * 1479936
+    # Mixture step (--mixture): the Gram matrix of every cell's 6B evaluation rows.
+    MIX_FLOP = 2 * CELLS * (6 * BATCH) ** 2 * X_DIM
+    TRAIN_BWD_BYTES = CELLS * (26 * W_FUSED + 30 * W_RANGES
+                               + 2 * (2 * HIDDEN * HIDDEN + 2 * X_DIM * HIDDEN) + 2 * BWD_ACT)
+
+
+_derive()
 
 # DRAM bytes (read + write) per phase of one iteration, summed over the phase's kernels: not
 # measured by this script but taken from ncu captures (dram__bytes_read.sum +
 # dram__bytes_write.sum) of these same kernels, each with the summary it comes from. A phase
 # whose kernels changed after its capture has no entry (null traffic).
 PHASE_TRAFFIC = {
-    "train_bwd": (2203.5e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
+    "train_bwd": (2195.5e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
     "d_fwd": (236.7e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
     "g_fwd": (143.8e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
     "batch": (21.2e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
@@ -675,10 +688,19 @@ def main():
                     help="neighbours seen one iteration late (asynchronous cells)")
     ap.add_argument("--dcgan", action="store_true",
                     help="the 3x3 DCGAN workload (tensor-core convolutions) instead of the MLP")
+    ap.add_argument("--grid", default=None, metavar="RxC",
+                    help="the MLP workload on a smaller or larger torus (for kernel captures on a "
+                         "small case; not the benchmark configuration; no ncu traffic figures)")
     ap.add_argument("--dcgan-grid", default=None, metavar="RxC",
                     help="with --dcgan: a smaller or larger torus of the same networks (for "
                          "kernel captures on a small case; not the benchmark configuration)")
     args = ap.parse_args()
+    if args.grid:
+        global ROWS, COLS, WORKLOAD, PHASE_TRAFFIC
+        ROWS, COLS = (int(v) for v in args.grid.lower().split("x"))
+        _derive()
+        WORKLOAD = "%dx%d torus MLP G/D bf16 B=100 (%d pairs/iter)" % (ROWS, COLS, PAIRS)
+        PHASE_TRAFFIC = {}
     if args.dcgan_grid:
         global DC_ROWS, DC_COLS, DC_CELLS, DC_PAIRS, DC_WORKLOAD
         DC_ROWS, DC_COLS = (int(v) for v in args.dcgan_grid.lower().split("x"))
