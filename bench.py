@@ -240,7 +240,7 @@ def run_ours(args):
     else:
         e2e_value = _e2e(args, L, g, torch, dist, world)
     h2d = CELLS * BATCH * X_DIM * 4
-    d2h = 2 * CELLS * 5 * 4
+    d2h = 2 * CELLS * 5 * 4 + 8 * 4  # fitnesses and the eight device status words, one copy
     if args.no_phases:
         roof = None
     else:
@@ -279,20 +279,23 @@ def _e2e(args, L, g, torch, dist, world):
     nbuf = 2
     xs = [torch.from_numpy(lipz_synth.host_batch(SEED + 7 + i, CELLS, BATCH, X_DIM)).pin_memory()
           for i in range(nbuf)]
-    fg = torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()
-    fd = torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()
+    # two sets of pinned result buffers: a call's fitnesses land while the next call runs
+    fit = [(torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory(),
+            torch.zeros((CELLS, 5), dtype=torch.float32).pin_memory()) for _ in range(2)]
     for i in range(2):
-        L.lipz_iterate_batch(g.h, xs[i % nbuf], fg, fd)
+        L.lipz_iterate_batch(g.h, xs[i % nbuf], fit[0][0], fit[0][1])
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    # every step's upload is inside the timed region: the first with its own call, each later
-    # one issued by the call before it (lipz_iterate_batch_next overlaps it with that
-    # iteration's compute)
+    # every step's upload and fitness read-back is inside the timed region: the first upload
+    # with its own call, each later one issued by the call before it, which overlaps it with
+    # that iteration's compute; lipz_iterate_batch_async returns once the previous call's
+    # iteration (and its fitness copy) is complete, and lipz_synchronize completes the last
     t0 = time.perf_counter()
     for i in range(args.steps):
         nxt = xs[(i + 1) % nbuf] if i + 1 < args.steps else None
-        L.lipz_iterate_batch_next(g.h, xs[i % nbuf], nxt, fg, fd)
+        L.lipz_iterate_batch_async(g.h, xs[i % nbuf], nxt, fit[i % 2][0], fit[i % 2][1])
+    L.lipz_synchronize(g.h)
     e2e_s = allreduce_max(dist, time.perf_counter() - t0)
     return PAIRS * world * args.steps / e2e_s
 
@@ -525,15 +528,16 @@ def run_dcgan(args):
     # end to end: pinned host minibatches in, fitness out
     xs = [torch.from_numpy(pool[np.random.default_rng(i).integers(0, DC_POOL, DC_CELLS * DC_B)]
                            .reshape(DC_CELLS, DC_B, 12288)).pin_memory() for i in range(2)]
-    fg = torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory()
-    fd = torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory()
-    L.lipz_iterate_batch(g.h, xs[0], fg, fd)
+    fit = [(torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory(),
+            torch.zeros((DC_CELLS, 5), dtype=torch.float32).pin_memory()) for _ in range(2)]
+    L.lipz_iterate_batch(g.h, xs[0], fit[0][0], fit[0][1])
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     n_e2e = max(2, args.steps // 2)
     for i in range(n_e2e):
-        L.lipz_iterate_batch_next(g.h, xs[i % 2], xs[(i + 1) % 2] if i + 1 < n_e2e else None,
-                                  fg, fd)
+        L.lipz_iterate_batch_async(g.h, xs[i % 2], xs[(i + 1) % 2] if i + 1 < n_e2e else None,
+                                   fit[i % 2][0], fit[i % 2][1])
+    L.lipz_synchronize(g.h)
     e2e = DC_PAIRS * world * n_e2e / allreduce_max(dist, time.perf_counter() - t0)
     if rank != 0:
         return None
@@ -565,7 +569,7 @@ def run_dcgan(args):
         "grid_iterations_per_sec": 1000.0 * world / ms_step,
         "phase_ms": phase_ms, "roofline": roof, "phase_rooflines": roofs,
         "e2e": {"value": e2e, "unit": UNIT, "h2d_bytes_per_step": DC_CELLS * DC_B * 12288 * 4,
-                "d2h_bytes_per_step": 2 * DC_CELLS * 5 * 4},
+                "d2h_bytes_per_step": 2 * DC_CELLS * 5 * 4 + 8 * 4},
         "gpu_launches": launches, "clocks": clk.summary(),
     }
     if world == 1 and not args.no_cpu_baseline:

@@ -223,6 +223,27 @@ LIPZ_API int lipz_iterate_batch_next(lipz_grid* g, const float* x_host, const fl
                                      float* fit_g, float* fit_d);
 
 /*
+ * The same one call ahead (a pipeline one iteration deep), for a caller that keeps the GPU
+ * busy across calls: the call enqueues this iteration (and x_next's upload) and then waits
+ * only for the PREVIOUS call's iteration. When it returns, the previous call's fit_g / fit_d
+ * hold that iteration's fitnesses, and the return code reports the previous iteration's device
+ * status (LIPZ_ERR_NONFINITE, LIPZ_ERR_TIMEOUT) or an error in enqueueing this one; the first
+ * call returns without waiting. This call's fit_g / fit_d are written when the next call (or
+ * lipz_synchronize) returns: the caller must leave them, x_host and x_next alone until then,
+ * so two sets of result buffers alternate. lipz_synchronize completes the last call (its
+ * fitnesses included) and reports its
+ * status; any other call on the grid may report it instead. After an error the pipeline is
+ * drained (this call's iteration has completed too and is not reported separately). An upload
+ * into a staging buffer waits on the device for the iteration that last read it. Results are
+ * bit-identical to lipz_iterate_batch on the same minibatches. Per iteration the fitnesses
+ * and device status words are gathered on the device and come back in one copy into a pinned
+ * slot of the grid; the fitnesses are copied into fit_g / fit_d (any host memory) when the
+ * call completes.
+ */
+LIPZ_API int lipz_iterate_batch_async(lipz_grid* g, const float* x_host, const float* x_next,
+                                      float* fit_g, float* fit_d);
+
+/*
  * State I/O (checkpoint / resume, and state exchange with other implementations). Layout,
  * little-endian: a 64-byte header {u32 magic 0x5A50494C, u32 version 2, i32 rows, cols, z_dim,
  * hidden, x_dim, batch, precision, 0, i64 t, u64 seed, 8 zero bytes}, then f32 Gw[cells][PG],

@@ -17,6 +17,7 @@ __all__ = [
     "lipz_arch_default", "lipz_grid_create", "lipz_grid_destroy", "lipz_set_stream",
     "lipz_synchronize", "lipz_set_data", "lipz_eval_neighborhoods", "lipz_select_replace",
     "lipz_train_step", "lipz_iterate", "lipz_iterate_batch", "lipz_iterate_batch_next",
+    "lipz_iterate_batch_async",
     "lipz_state_bytes",
     "lipz_export_state", "lipz_import_state", "lipz_get_iteration", "lipz_get_batch",
     "lipz_get_logits", "lipz_get_gradients", "lipz_get_mixture", "lipz_profile_enable",
@@ -76,6 +77,7 @@ _SIGS = {
     "lipz_iterate": (_I, [_P, _I]),
     "lipz_iterate_batch": (_I, [_P, _P, _P, _P]),
     "lipz_iterate_batch_next": (_I, [_P, _P, _P, _P, _P]),
+    "lipz_iterate_batch_async": (_I, [_P, _P, _P, _P, _P]),
     "lipz_state_bytes": (_I, [_P, ctypes.POINTER(ctypes.c_size_t)]),
     "lipz_export_state": (_I, [_P, _P, ctypes.c_size_t]),
     "lipz_import_state": (_I, [_P, _P, ctypes.c_size_t]),
@@ -189,6 +191,13 @@ def lipz_iterate_batch_next(g, x_host, x_next=None, fit_g=None, fit_d=None):
     """lipz_iterate_batch that uploads the next call's minibatch (x_next) while this one runs."""
     return _check(g, load().lipz_iterate_batch_next(g, _ptr(x_host), _ptr(x_next), _ptr(fit_g),
                                                     _ptr(fit_d)))
+
+
+def lipz_iterate_batch_async(g, x_host, x_next=None, fit_g=None, fit_d=None):
+    """lipz_iterate_batch_next one call ahead: enqueues this iteration, returns once the previous
+    call's has completed (its fitness buffers filled, its device status returned)."""
+    return _check(g, load().lipz_iterate_batch_async(g, _ptr(x_host), _ptr(x_next), _ptr(fit_g),
+                                                     _ptr(fit_d)))
 
 
 def lipz_state_bytes(g) -> int:

@@ -63,6 +63,18 @@ struct lipz_grid {
   const float* pre_host = nullptr;
   int pre_buf = -1;
   int* hstat = nullptr;            // pinned host copies of the device error flags
+  // lipz_iterate_batch_async: per call slot (alternating) a pinned copy of its iteration's
+  // fitnesses and device status words (gathered on the device into `astage` first: one copy)
+  // with the caller's result pointers, and an event at its end; per staging buffer an event
+  // after the last iteration that read it (an upload into the buffer waits for it)
+  float* astage = nullptr;         // device [2 cells 5 fitnesses][8 status words]
+  float* hstat_a = nullptr;        // pinned [2 slots][the same]
+  float* a_fit[2][2] = {};         // per slot: the caller's fit_g, fit_d
+  cudaEvent_t ev_it[2] = {nullptr, nullptr};
+  cudaEvent_t ev_buf[2] = {nullptr, nullptr};
+  bool buf_read[2] = {false, false};
+  int a_last = 1;                  // slot of the newest call
+  bool a_pending = false;          // the newest call's status is still to be reported
   int device = 0;
   // population snapshots: ping-pong pair, or three in rotation with stale neighbours (the
   // snapshot being written must not be the one the stale neighbours are read from)
@@ -1159,28 +1171,30 @@ int train_impl(lipz_grid* g) {
 // Waits for the grid's stream and reports a bounded wait that expired in a tensor-core kernel
 // or a non-finite loss seen since the last check (one synchronisation: all flags are copied
 // into pinned host memory first); the flags are reset.
-int check_flag(lipz_grid* g) {
-  int* dev[8] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
-                 g->tc[1] ? tc_error_flag(g->tc[1]) : nullptr,
-                 g->tc[2] ? tc_error_flag(g->tc[2]) : nullptr,
-                 g->tcb[0] ? tcb_error_flag(g->tcb[0]) : nullptr,
-                 g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr,
-                 g->tcb[2] ? tcb_error_flag(g->tcb[2]) : nullptr,
-                 g->dc ? dc_error_flag(g->dc) : nullptr, g->flag};
-  for (int i = 0; i < 8; ++i) {
-    g->hstat[i] = i < 7 ? 0 : INT_MAX;
-    if (dev[i]) CK(g, cudaMemcpyAsync(&g->hstat[i], dev[i], 4, cudaMemcpyDeviceToHost, g->st));
-  }
-  CK(g, cudaStreamSynchronize(g->st));
+// The device flags of every kernel that can stop early, and the non-finite-loss flag.
+void flag_ptrs(lipz_grid* g, int* (&dev)[8]) {
+  int* d[8] = {g->tc[0] ? tc_error_flag(g->tc[0]) : nullptr,
+               g->tc[1] ? tc_error_flag(g->tc[1]) : nullptr,
+               g->tc[2] ? tc_error_flag(g->tc[2]) : nullptr,
+               g->tcb[0] ? tcb_error_flag(g->tcb[0]) : nullptr,
+               g->tcb[1] ? tcb_error_flag(g->tcb[1]) : nullptr,
+               g->tcb[2] ? tcb_error_flag(g->tcb[2]) : nullptr,
+               g->dc ? dc_error_flag(g->dc) : nullptr, g->flag};
+  for (int i = 0; i < 8; ++i) dev[i] = d[i];
+}
+
+// Status from pinned copies st[8] of the device flags (the queued work has completed): a
+// raised flag is reset on the device and reported.
+int flag_status(lipz_grid* g, int* const (&dev)[8], const int* st) {
   for (int i = 0; i < 7; ++i) {
-    const int code = g->hstat[i];
+    const int code = st[i];
     if (code) {
       CK(g, cudaMemsetAsync(dev[i], 0, 4, g->st));
       CK(g, cudaStreamSynchronize(g->st));
       return fail(g, LIPZ_ERR_TIMEOUT, "tensor-core kernel stopped: bounded wait %d expired", code);
     }
   }
-  const int v = g->hstat[7];
+  const int v = st[7];
   if (v != INT_MAX) {
     const int big = INT_MAX;
     int rc = h2d(g, g->flag, &big, 4);
@@ -1188,6 +1202,34 @@ int check_flag(lipz_grid* g) {
     return fail(g, LIPZ_ERR_NONFINITE, "non-finite loss in cell %d", v);
   }
   return LIPZ_OK;
+}
+
+// Completes a pending lipz_iterate_batch_async call: waits for its iteration and copies its
+// fitnesses to the caller (its status is left to the device flags, which stay raised until a
+// check reads and resets them).
+int deliver_pending(lipz_grid* g) {
+  if (!g->a_pending) return LIPZ_OK;
+  g->a_pending = false;
+  CK(g, cudaEventSynchronize(g->ev_it[g->a_last]));
+  const size_t n5 = (size_t)g->cells * 5;
+  const float* hp = g->hstat_a + g->a_last * (2 * n5 + 8);
+  if (g->a_fit[g->a_last][0]) memcpy(g->a_fit[g->a_last][0], hp, n5 * 4);
+  if (g->a_fit[g->a_last][1]) memcpy(g->a_fit[g->a_last][1], hp + n5, n5 * 4);
+  return LIPZ_OK;
+}
+
+int check_flag(lipz_grid* g) {
+  // a pending pipelined call completes first; the flags read here cover its iteration too
+  int rc0 = deliver_pending(g);
+  if (rc0) return rc0;
+  int* dev[8];
+  flag_ptrs(g, dev);
+  for (int i = 0; i < 8; ++i) {
+    g->hstat[i] = i < 7 ? 0 : INT_MAX;
+    if (dev[i]) CK(g, cudaMemcpyAsync(&g->hstat[i], dev[i], 4, cudaMemcpyDeviceToHost, g->st));
+  }
+  CK(g, cudaStreamSynchronize(g->st));
+  return flag_status(g, dev, g->hstat);
 }
 
 float bf16_bits_to_float(uint16_t b) {
@@ -1301,6 +1343,11 @@ int lipz_grid_destroy(lipz_grid* g) {
   if (g->ev_x) cudaEventDestroy(g->ev_x);
   if (g->ev_x2) cudaEventDestroy(g->ev_x2);
   if (g->hstat) cudaFreeHost(g->hstat);
+  if (g->hstat_a) cudaFreeHost(g->hstat_a);
+  for (int i = 0; i < 2; ++i) {
+    if (g->ev_it[i]) cudaEventDestroy(g->ev_it[i]);
+    if (g->ev_buf[i]) cudaEventDestroy(g->ev_buf[i]);
+  }
   delete g;
   return LIPZ_OK;
 }
@@ -1404,6 +1451,9 @@ int lipz_iterate(lipz_grid* g, int n_iters) {
 int lipz_iterate_batch(lipz_grid* g, const float* x_host, float* fit_g, float* fit_d) {
   if (!g) return LIPZ_ERR_INVALID;
   if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
+  // a pipelined call's iteration may still read a staging buffer
+  int rc0 = deliver_pending(g);
+  if (rc0) return rc0;
   const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
   g->pre_buf = -1;  // (a minibatch uploaded ahead into the same buffer is superseded)
   g->pre_host = nullptr;
@@ -1422,6 +1472,8 @@ int lipz_iterate_batch_next(lipz_grid* g, const float* x_host, const float* x_ne
                             float* fit_g, float* fit_d) {
   if (!g) return LIPZ_ERR_INVALID;
   if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
+  int rc0 = deliver_pending(g);
+  if (rc0) return rc0;
   const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
   if (!g->xin2) {
     int rc;
@@ -1461,6 +1513,92 @@ int lipz_iterate_batch_next(lipz_grid* g, const float* x_host, const float* x_ne
   if (fit_g) CK(g, cudaMemcpyAsync(fit_g, g->fG, C * 20, cudaMemcpyDeviceToHost, g->st));
   if (fit_d) CK(g, cudaMemcpyAsync(fit_d, g->fD, C * 20, cudaMemcpyDeviceToHost, g->st));
   return check_flag(g);
+}
+
+int lipz_iterate_batch_async(lipz_grid* g, const float* x_host, const float* x_next,
+                             float* fit_g, float* fit_d) {
+  if (!g) return LIPZ_ERR_INVALID;
+  if (!x_host) return fail(g, LIPZ_ERR_INVALID, "x_host is null");
+  const size_t bytes = (size_t)g->cells * g->a.batch * g->a.x_dim * 4;
+  if (!g->xin2) {
+    int rc;
+    if ((rc = dalloc(g, &g->xin2, bytes))) return rc;
+    CK(g, cudaEventCreateWithFlags(&g->ev_x2, cudaEventDisableTiming));
+  }
+  const size_t C = g->cells, n5 = C * 5, stage_words = 2 * n5 + 8;
+  if (!g->hstat_a) {
+    int rc0;
+    if ((rc0 = dalloc(g, &g->astage, stage_words * 4))) return rc0;
+    CK(g, cudaMallocHost(&g->hstat_a, 2 * stage_words * 4));
+    for (int i = 0; i < 2; ++i) {
+      CK(g, cudaEventCreateWithFlags(&g->ev_it[i], cudaEventDisableTiming));
+      CK(g, cudaEventCreateWithFlags(&g->ev_buf[i], cudaEventDisableTiming));
+    }
+  }
+  float* const buf[2] = {g->xin, g->xin2};
+  const cudaEvent_t ev[2] = {g->ev_x, g->ev_x2};
+  // an upload into a staging buffer waits for the last iteration that read it (which may
+  // still be running: this call does not wait for the previous one before enqueueing)
+  auto upload = [&](int b, const float* src) -> int {
+    if (g->buf_read[b]) CK(g, cudaStreamWaitEvent(g->copy_st, g->ev_buf[b], 0));
+    CK(g, cudaMemcpyAsync(buf[b], src, bytes, cudaMemcpyHostToDevice, g->copy_st));
+    CK(g, cudaEventRecord(ev[b], g->copy_st));
+    return LIPZ_OK;
+  };
+  int rc, cur;
+  if (g->pre_buf >= 0 && g->pre_host == x_host) {
+    cur = g->pre_buf;
+  } else {
+    cur = g->pre_buf >= 0 ? 1 - g->pre_buf : 0;
+    if ((rc = upload(cur, x_host))) return rc;
+  }
+  g->pre_buf = -1;
+  g->pre_host = nullptr;
+  if (x_next) {
+    if ((rc = upload(1 - cur, x_next))) return rc;
+    g->pre_buf = 1 - cur;
+    g->pre_host = x_next;
+  }
+  if ((rc = eval_impl(g, buf[cur], true, ev[cur])) || (rc = train_impl(g))) {
+    g->pre_buf = -1;
+    g->pre_host = nullptr;
+    return rc;
+  }
+  // this iteration's fitnesses and status words, gathered and copied into this call's slot
+  const int slot = 1 - g->a_last;
+  int* dev[8];
+  flag_ptrs(g, dev);
+  StatusFlags fl;
+  for (int i = 0; i < 8; ++i) fl.p[i] = dev[i];
+  launch_gather_status(g->fG, g->fD, (int)n5, fl, g->astage, true, g->st);
+  CKL(g);
+  float* hs = g->hstat_a + slot * stage_words;
+  CK(g, cudaMemcpyAsync(hs, g->astage, stage_words * 4, cudaMemcpyDeviceToHost, g->st));
+  g->a_fit[slot][0] = fit_g;
+  g->a_fit[slot][1] = fit_d;
+  CK(g, cudaEventRecord(g->ev_it[slot], g->st));
+  // the staging buffer is free once the iteration and its small copies are done (an upload
+  // started earlier would hold up those copies, and the next iteration behind them)
+  CK(g, cudaEventRecord(g->ev_buf[cur], g->st));
+  g->buf_read[cur] = true;
+  const bool had = g->a_pending;
+  const int prev = g->a_last;
+  g->a_last = slot;
+  g->a_pending = true;
+  if (!had) return LIPZ_OK;
+  // the previous call's iteration (and its copy) has completed once this returns
+  CK(g, cudaEventSynchronize(g->ev_it[prev]));
+  const float* hp = g->hstat_a + prev * stage_words;
+  if (g->a_fit[prev][0]) memcpy(g->a_fit[prev][0], hp, n5 * 4);
+  if (g->a_fit[prev][1]) memcpy(g->a_fit[prev][1], hp + n5, n5 * 4);
+  rc = flag_status(g, dev, reinterpret_cast<const int*>(hp + 2 * n5));
+  if (rc) {
+    // the flags are sticky until reset: drain this call too, whose copies may repeat the
+    // report, and leave nothing pending
+    CK(g, cudaStreamSynchronize(g->st));
+    g->a_pending = false;
+  }
+  return rc;
 }
 
 int lipz_state_bytes(const lipz_grid* g, size_t* bytes) {

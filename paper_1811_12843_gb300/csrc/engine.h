@@ -76,6 +76,13 @@ void launch_gemv(const GemvDesc* descs, int n_problems, int max_rows, cudaStream
 template <typename T>
 void launch_colsum(const ColSumDesc* descs, int n_problems, int max_cols, cudaStream_t st);
 
+// device status words of one iteration (error flags of the kernels that can stop early, the
+// non-finite-loss flag last), any of them null
+struct StatusFlags {
+  const int* p[8];
+};
+void launch_gather_status(const float* fG, const float* fD, int n, const StatusFlags& fl,
+                          float* out, bool pdl, cudaStream_t st);
 void launch_fitness(const float* logits, int cells, int B, float* LG, float* LD, float* fG,
                     float* fD, int* flag, cudaStream_t st);
 // Also writes, per cell and population, the Adam coefficients of the new centre's next step:

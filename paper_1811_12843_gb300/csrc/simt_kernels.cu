@@ -927,4 +927,24 @@ void launch_mix_es(const float* part, int nh, int cells, int rows, int B, float*
              sigma);
 }
 
+// The iteration's results for one host copy: out[0, n) = fG, out[n, 2n) = fD (n = cells * 5),
+// then the eight status words (a null flag reads as its all-clear value: 0 for the first
+// seven, INT_MAX for the last).
+__global__ void k_gather_status(const float* __restrict__ fG, const float* __restrict__ fD, int n,
+                                StatusFlags fl, float* __restrict__ out) {
+  pdl_wait();
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < 2 * n; i += gridDim.x * blockDim.x)
+    out[i] = i < n ? fG[i] : fD[i - n];
+  if (blockIdx.x == 0 && threadIdx.x < 8) {
+    const int* f = fl.p[threadIdx.x];
+    reinterpret_cast<int*>(out + 2 * n)[threadIdx.x] =
+        f ? *f : (threadIdx.x < 7 ? 0 : 0x7FFFFFFF);
+  }
+}
+
+void launch_gather_status(const float* fG, const float* fD, int n, const StatusFlags& fl,
+                          float* out, bool pdl, cudaStream_t st) {
+  launch_kernel(pdl, k_gather_status, dim3(2), dim3(256), 0, st, fG, fD, n, fl, out);
+}
+
 }  // namespace lipz

@@ -312,6 +312,63 @@ def test_host_batch_pipelined_equals_one_call_at_a_time(L):
     assert a.export_state() == b.export_state()
 
 
+def test_host_batch_async_equals_one_call_at_a_time(L):
+    """lipz_iterate_batch_async runs one call ahead: it enqueues its iteration and returns once
+    the previous call's has completed, with that call's fitnesses in its (alternating, pinned)
+    result buffers. A sequence of calls (a minibatch announced and then not used, a synchronous
+    call in between, lipz_synchronize to finish) gives the same fitnesses and state as the same
+    minibatches through lipz_iterate_batch, bit for bit; uploads into a staging buffer wait for
+    the iteration that last read it (a call never waits for its own iteration)."""
+    import torch
+    import lipz_synth
+    pool = _pool(3, 2000, 784)
+    a = _grid(L, 3, 3, 12, pool, precision="bf16")
+    b = _grid(L, 3, 3, 12, pool, precision="bf16")
+    xs = [torch.from_numpy(lipz_synth.host_batch(50 + i, 9, 100)).pin_memory() for i in range(3)]
+    order = [0, 1, 2, 0, 1, 2, 0, 1, 0]
+    res = [[torch.zeros((9, 5), dtype=torch.float32).pin_memory() for _ in range(2)]
+           for _ in range(2)]
+    ref = []
+    fb = [np.zeros((9, 5), np.float32) for _ in range(2)]
+    pending = None  # index of the call whose results the next call completes
+    for i, k in enumerate(order):
+        nxt = xs[order[i + 1]] if i + 1 < len(order) else None
+        if i == 4:
+            nxt = xs[0]  # announced, then call 5 uses xs[2]: the early upload is dropped
+        L.lipz_iterate_batch(b.h, xs[k], fb[0], fb[1])
+        ref.append((fb[0].copy(), fb[1].copy()))
+        if i == 6:
+            # a synchronous call in between completes the pending one first
+            L.lipz_iterate_batch(a.h, xs[k], res[i % 2][0], res[i % 2][1])
+        else:
+            L.lipz_iterate_batch_async(a.h, xs[k], nxt, res[i % 2][0], res[i % 2][1])
+        if pending is not None:
+            got = res[pending % 2]
+            assert np.array_equal(got[0].numpy(), ref[pending][0]), pending
+            assert np.array_equal(got[1].numpy(), ref[pending][1]), pending
+        pending = None if i == 6 else i
+        if i == 6:
+            assert np.array_equal(res[0][0].numpy(), ref[6][0])
+    L.lipz_synchronize(a.h)
+    last = len(order) - 1
+    assert np.array_equal(res[last % 2][0].numpy(), ref[last][0])
+    assert np.array_equal(res[last % 2][1].numpy(), ref[last][1])
+    assert a.export_state() == b.export_state()
+    # a non-finite loss of call n is reported by call n + 1 (or by lipz_synchronize)
+    s = _to_oracle(a, a.arch)
+    s.Dw[2, 5] = np.nan
+    a.import_state(O.state_to_bytes(s))
+    L.lipz_iterate_batch_async(a.h, xs[0], xs[1], res[0][0], res[0][1])
+    with pytest.raises(L.LipzError) as e:
+        L.lipz_iterate_batch_async(a.h, xs[1], None, res[1][0], res[1][1])
+    assert e.value.code == L.LIPZ_ERR_NONFINITE
+    L.lipz_synchronize(a.h)  # drained: nothing left to report
+    s.Dw[2, 5] = 0.0
+    a.import_state(O.state_to_bytes(s))
+    L.lipz_iterate_batch_async(a.h, xs[0], None, res[0][0], res[0][1])
+    L.lipz_synchronize(a.h)
+
+
 def test_determinism_and_resume(L):
     pool = _pool(4, 2000, 784)
     a = _grid(L, 3, 3, 21, pool, precision="bf16")
