@@ -216,9 +216,7 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
       __nv_bfloat162 b2 = __floats2bfloat162_rn(vout[e], vout[e + 1]);
       pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
     }
-    uint4* o = reinterpret_cast<uint4*>(C + col0);
-    o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-    o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+    st_global_v8(C + col0, pk);  // rows and column groups are 32-byte aligned here
     return;
   }
   for (int e = 0; e < 16; ++e) {
@@ -277,15 +275,18 @@ __device__ __forceinline__ bool epilogue_tile(const GParams& p, int cell, int m0
     X = p.aux + (int64_t)cell * p.aux_cell + (int64_t)arow * p.sxm;
     if (p.aux_sel) X += (int64_t)(1 + __ldg(&p.aux_sel[cell])) * p.aux_sel_stride;
   }
+  // (16 bf16 of a row per 256-bit load: the stored outputs' rows are 32-byte aligned)
   auto load_pair = [&](int g, uint4(&d)[4]) {
-    const uint4* x4 = reinterpret_cast<const uint4*>(X + n0 + g * 16);
+    const bf16* x = X + n0 + g * 16;
     if (n0 + g * 16 + 16 <= p.N) {
-      d[0] = x4[0];
-      d[1] = x4[1];
+      const U8 v = ld_global_v8(x);
+      d[0] = v.a;
+      d[1] = v.b;
     }
     if (g + 1 < g1 && n0 + g * 16 + 32 <= p.N) {
-      d[2] = x4[2];
-      d[3] = x4[3];
+      const U8 v = ld_global_v8(x + 16);
+      d[2] = v.a;
+      d[3] = v.b;
     }
   };
   uint4 xc[4], xn[4];

@@ -99,6 +99,23 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, uint32_t sr
       "r"(x), "r"(y), "r"(z), "r"(w), "r"(src)
       : "memory");
 }
+// 256-bit global accesses (32-byte aligned): one per 16 bf16 of a row, half the L1 wavefronts
+// of two 16-byte accesses when the lanes of a warp touch 32 different rows
+struct U8 {
+  uint4 a, b;
+};
+__device__ __forceinline__ U8 ld_global_v8(const void* p) {
+  uint32_t r0, r1, r2, r3, r4, r5, r6, r7;
+  asm("ld.global.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3), "=r"(r4), "=r"(r5), "=r"(r6), "=r"(r7)
+               : "l"(p));
+  return U8{make_uint4(r0, r1, r2, r3), make_uint4(r4, r5, r6, r7)};
+}
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t (&v)[8]) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]),
+               "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
