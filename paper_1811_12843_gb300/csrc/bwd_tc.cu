@@ -216,7 +216,9 @@ __device__ __forceinline__ void epi16(const GParams& p, const uint32_t (&r)[16],
       __nv_bfloat162 b2 = __floats2bfloat162_rn(vout[e], vout[e + 1]);
       pk[e >> 1] = *reinterpret_cast<uint32_t*>(&b2);
     }
-    st_global_v8(C + col0, pk);  // rows and column groups are 32-byte aligned here
+    // rows and column groups are 32-byte aligned here
+    st_global_v8(C + col0, make_uint4(pk[0], pk[1], pk[2], pk[3]),
+                 make_uint4(pk[4], pk[5], pk[6], pk[7]));
     return;
   }
   for (int e = 0; e < 16; ++e) {

@@ -448,10 +448,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
               }
               if (gout && row_ok) {
-                uint4* o = reinterpret_cast<uint4*>(gout + act_off + cg * 32);
+                bf16* o = gout + act_off + cg * 32;  // 256-bit stores: 32-byte aligned rows
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 4; u += 2)
+                  st_global_v8(o + 8 * u, make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                                     pk[4 * u + 3]),
+                               make_uint4(pk[4 * u + 4], pk[4 * u + 5], pk[4 * u + 6],
+                                          pk[4 * u + 7]));
               }
             }
             if (to_h) {
@@ -500,10 +503,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 acc = fmaf(__high2float(q23), ww.w, acc);
               }
               if (p.act2 && row_ok) {
-                uint4* o = reinterpret_cast<uint4*>(p.act2 + act_off + cg * 32);
+                bf16* o = p.act2 + act_off + cg * 32;
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 4; u += 2)
+                  st_global_v8(o + 8 * u, make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                                     pk[4 * u + 3]),
+                               make_uint4(pk[4 * u + 4], pk[4 * u + 5], pk[4 * u + 6],
+                                          pk[4 * u + 7]));
               }
             }
           }
@@ -602,11 +608,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int e = 0; e < 16; e += 2)
               pk[e >> 1] = pack_bf16(tanh_fast(__uint_as_float(r[e]) + bv[e]),
                                      tanh_fast(__uint_as_float(r[e + 1]) + bv[e + 1]));
-            if (rr < p.B && col0 < p.x) {
-              uint4* o = reinterpret_cast<uint4*>(dst + col0);
-              o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-              o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-            }
+            if (rr < p.B && col0 < p.x)  // one 256-bit store per row and 16 columns
+              st_global_v8(dst + col0, make_uint4(pk[0], pk[1], pk[2], pk[3]),
+                           make_uint4(pk[4], pk[5], pk[6], pk[7]));
           }
           tc_fence_before();
           mbar_arrive(bReg + 8 * R);
@@ -1030,10 +1034,13 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
                            : "memory");
             }
             if (train && j == 0 && row_ok) {
-              uint4* o = reinterpret_cast<uint4*>(p.act1 + lidx * HID + col0);
+              bf16* o = p.act1 + lidx * HID + col0;  // 256-bit stores: 32-byte aligned rows
 #pragma unroll
-              for (int u = 0; u < W / 8; ++u)
-                o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+              for (int u = 0; u < W / 8; u += 2)
+                st_global_v8(o + 8 * u, make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                                   pk[4 * u + 3]),
+                             make_uint4(pk[4 * u + 4], pk[4 * u + 5], pk[4 * u + 6],
+                                        pk[4 * u + 7]));
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             warp_signal(lH + 8 * ch);
@@ -1081,10 +1088,13 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
                 acc = fmaf(__high2float(v23), ww.w, acc);
               }
               if (train && row_ok) {
-                uint4* o = reinterpret_cast<uint4*>(p.act2 + lidx * HID + cg * 32);
+                bf16* o = p.act2 + lidx * HID + cg * 32;
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                  o[u] = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                for (int u = 0; u < 4; u += 2)
+                  st_global_v8(o + 8 * u, make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                                     pk[4 * u + 3]),
+                               make_uint4(pk[4 * u + 4], pk[4 * u + 5], pk[4 * u + 6],
+                                          pk[4 * u + 7]));
               }
             }
           }
@@ -1125,11 +1135,10 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
               pk[2 * qq + 1] = pack_bf16(tanh_fast(__uint_as_float(r[4 * qq + 2]) + t.z),
                                          tanh_fast(__uint_as_float(r[4 * qq + 3]) + t.w));
             }
-            if (row_ok && col0 < p.x) {
-              uint4* o = reinterpret_cast<uint4*>(dst + col0);
-              o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-              o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-            }
+            if (row_ok && col0 < p.x)  // one 256-bit store per row and 16 columns (E's rows,
+                                       // slots and cells are 32-byte aligned: x % 16 == 0)
+              st_global_v8(dst + col0, make_uint4(pk[0], pk[1], pk[2], pk[3]),
+                           make_uint4(pk[4], pk[5], pk[6], pk[7]));
           }
           tc_fence_before();
           warp_signal(lReg + 8 * R);
