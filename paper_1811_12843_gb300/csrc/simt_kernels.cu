@@ -82,10 +82,13 @@ __device__ __forceinline__ void store4<bf16>(bf16* dst, float4 v) {
   *reinterpret_cast<uint2*>(dst) = pk;
 }
 
-// One warp per minibatch row: the row's pool index (one Philox word), a 16-byte-vector copy of
-// the row, then the row's normals, one Philox block (four normals) per lane at a time. The pool
-// is held in the population's precision, so a drawn row is a plain copy; rows given by the
-// caller (xin, fp32) are rounded here.
+// Four minibatch rows per warp: one Philox block gives the four rows' pool indices, and the
+// rows' 16-byte-vector copies are issued together (every load, then every store), so a warp
+// waits for memory once; then each row's normals, one Philox block (four normals) per lane at
+// a time. The pool is held in the population's precision, so a drawn row is a plain copy;
+// rows given by the caller (xin, fp32) are rounded here.
+constexpr int DRAW_RPW = 4;
+
 template <typename T>
 __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
                              const float* __restrict__ xin, T* __restrict__ E, int64_t e_cell,
@@ -94,57 +97,96 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
   pdl_wait();
   const uint32_t s_batch = 3u + (step << 8), s_noise = 4u + (step << 8);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
-  if (b >= B) return;
-  T* dst = E + (int64_t)c * e_cell + (int64_t)b * x_dim;
+  const int q = blockIdx.x * (blockDim.x >> 5) + warp, c = blockIdx.y;
+  const int b0 = q * DRAW_RPW;
+  if (b0 >= B) return;
+  const int nb = min(DRAW_RPW, B - b0);
+  T* const dst0 = E + (int64_t)c * e_cell + (int64_t)b0 * x_dim;
   if (!(parts & DRAW_REAL)) {
   } else if (xin) {
-    const float* src = xin + ((int64_t)c * B + b) * x_dim;
-    const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
-                     ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
-    if (vec) {
-      for (int k = lane * 4; k < x_dim; k += 128)
-        store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
-    } else {
-      for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
+    for (int i = 0; i < nb; ++i) {
+      T* dst = dst0 + (int64_t)i * x_dim;
+      const float* src = xin + ((int64_t)c * B + b0 + i) * x_dim;
+      const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
+                       ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
+      if (vec) {
+        for (int k = lane * 4; k < x_dim; k += 128)
+          store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
+      } else {
+        for (int k = lane; k < x_dim; k += 32) dst[k] = from_f<T>(src[k]);
+      }
     }
   } else {
-    const U4 r = philox_block(seed, s_batch, t, (uint32_t)c, (uint32_t)(b >> 2));
-    const uint32_t w = (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
-    const T* src = pool + (int64_t)mulhi_u32(w, (uint32_t)n_pool) * x_dim;
+    // rows 4q .. 4q + 3 take the four words of Philox block q
+    const U4 r = philox_block(seed, s_batch, t, (uint32_t)c, (uint32_t)q);
+    const uint32_t wd[DRAW_RPW] = {r.x, r.y, r.z, r.w};
     const int bytes = x_dim * (int)sizeof(T);
-    if ((bytes & 15) == 0 &&
-        ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
-      const uint4* s4 = reinterpret_cast<const uint4*>(src);
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
-      const int n4 = bytes >> 4;
+    const int n4 = bytes >> 4;
+    const bool vec = (bytes & 15) == 0 &&
+                     ((reinterpret_cast<uintptr_t>(pool) | reinterpret_cast<uintptr_t>(E)) & 15) == 0 &&
+                     ((e_cell * (int64_t)sizeof(T)) & 15) == 0;
+    if (vec && n4 > 128) {
+      // long rows (images): row by row, four vectors of a row in flight per lane
+      for (int i = 0; i < nb; ++i) {
+        const uint4* s4 = reinterpret_cast<const uint4*>(
+            pool + (int64_t)mulhi_u32(wd[i], (uint32_t)n_pool) * x_dim);
+        uint4* d4 = reinterpret_cast<uint4*>(dst0 + (int64_t)i * x_dim);
 #pragma unroll 4
-      for (int k = lane; k < n4; k += 32) d4[k] = __ldg(s4 + k);
+        for (int k = lane; k < n4; k += 32) d4[k] = __ldg(s4 + k);
+      }
+    } else if (vec) {
+      uint4 v[DRAW_RPW][4];
+#pragma unroll
+      for (int i = 0; i < DRAW_RPW; ++i) {
+        const uint4* s4 = reinterpret_cast<const uint4*>(
+            pool + (int64_t)mulhi_u32(wd[i], (uint32_t)n_pool) * x_dim);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int k = lane + 32 * u;
+          if (i < nb && k < n4) v[i][u] = __ldg(s4 + k);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < DRAW_RPW; ++i) {
+        uint4* d4 = reinterpret_cast<uint4*>(dst0 + (int64_t)i * x_dim);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int k = lane + 32 * u;
+          if (i < nb && k < n4) d4[k] = v[i][u];
+        }
+      }
     } else {
-      for (int k = lane; k < x_dim; k += 32) dst[k] = src[k];
+      for (int i = 0; i < nb; ++i) {
+        const T* src = pool + (int64_t)mulhi_u32(wd[i], (uint32_t)n_pool) * x_dim;
+        T* dst = dst0 + (int64_t)i * x_dim;
+        for (int k = lane; k < x_dim; k += 32) dst[k] = src[k];
+      }
     }
   }
   if (!(parts & DRAW_NOISE)) return;
-  T* zr = Z + ((int64_t)c * B + b) * z_dim;
-  const uint32_t n0 = (uint32_t)b * (uint32_t)z_dim;
-  // normals n0 .. n0 + z_dim - 1; Philox block i holds normals 4i .. 4i + 3
-  if ((z_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(zr) & (4 * sizeof(T) - 1)) == 0)) {
-    // every block lies inside the row and its four normals are one aligned vector
-    for (int k = lane * 4; k < z_dim; k += 128) {
-      const U4 r = philox_block(seed, s_noise, t, (uint32_t)c, (n0 + (uint32_t)k) >> 2);
-      const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
-      store4<T>(zr + k, make_float4(g01.x, g01.y, g23.x, g23.y));
+  for (int i = 0; i < nb; ++i) {
+    const int b = b0 + i;
+    T* zr = Z + ((int64_t)c * B + b) * z_dim;
+    const uint32_t n0 = (uint32_t)b * (uint32_t)z_dim;
+    // normals n0 .. n0 + z_dim - 1; Philox block i holds normals 4i .. 4i + 3
+    if ((z_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(zr) & (4 * sizeof(T) - 1)) == 0)) {
+      // every block lies inside the row and its four normals are one aligned vector
+      for (int k = lane * 4; k < z_dim; k += 128) {
+        const U4 rn = philox_block(seed, s_noise, t, (uint32_t)c, (n0 + (uint32_t)k) >> 2);
+        const float2 g01 = box_muller(rn.x, rn.y), g23 = box_muller(rn.z, rn.w);
+        store4<T>(zr + k, make_float4(g01.x, g01.y, g23.x, g23.y));
+      }
+      continue;
     }
-    return;
-  }
-  for (uint32_t blk = (n0 >> 2) + lane; blk * 4 < n0 + (uint32_t)z_dim; blk += 32) {
-    const U4 r = philox_block(seed, s_noise, t, (uint32_t)c, blk);
-    const float2 g01 = box_muller(r.x, r.y), g23 = box_muller(r.z, r.w);
-    const float v[4] = {g01.x, g01.y, g23.x, g23.y};
+    for (uint32_t blk = (n0 >> 2) + lane; blk * 4 < n0 + (uint32_t)z_dim; blk += 32) {
+      const U4 rn = philox_block(seed, s_noise, t, (uint32_t)c, blk);
+      const float2 g01 = box_muller(rn.x, rn.y), g23 = box_muller(rn.z, rn.w);
+      const float vv[4] = {g01.x, g01.y, g23.x, g23.y};
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint32_t n = blk * 4 + q;
-      if (n >= n0 && n < n0 + (uint32_t)z_dim) zr[n - n0] = from_f<T>(v[q]);
+      for (int qq = 0; qq < 4; ++qq) {
+        const uint32_t n = blk * 4 + qq;
+        if (n >= n0 && n < n0 + (uint32_t)z_dim) zr[n - n0] = from_f<T>(vv[qq]);
+      }
     }
   }
 }
@@ -153,7 +195,8 @@ template <typename T>
 void launch_draw_batch(const T* pool, int64_t n_pool, const float* xin, T* E, int64_t e_cell,
                        T* Z, int cells, int B, int x_dim, int z_dim, uint64_t seed, uint32_t t,
                        uint32_t step, int parts, bool pdl, cudaStream_t st) {
-  launch_kernel(pdl, k_draw_batch<T>, dim3((B + 7) / 8, cells), dim3(256), 0, st, pool, n_pool,
+  launch_kernel(pdl, k_draw_batch<T>, dim3((B + 8 * DRAW_RPW - 1) / (8 * DRAW_RPW), cells),
+                dim3(256), 0, st, pool, n_pool,
                 xin, E, e_cell, Z, B, x_dim, z_dim, seed, t, step, parts);
 }
 template void launch_draw_batch<float>(const float*, int64_t, const float*, float*, int64_t,
