@@ -615,7 +615,7 @@ template void launch_train_prep<bf16>(const bf16*, int64_t, const int*, bf16*, i
 // One block per cell, one thread per hidden unit.
 // ------------------------------------------------------------------------------------------
 template <typename T>
-__global__ void __launch_bounds__(1024) k_dlogit(
+__global__ void __launch_bounds__(512) k_dlogit(
     const float* __restrict__ TL, const T* __restrict__ TG2, const T* __restrict__ wD,
     int64_t wD_stride, int64_t off_w3, const int* __restrict__ src_d, int B, int H, float slope,
     T* __restrict__ J2, float* __restrict__ gD, int64_t gD_stride, int64_t off_gw3,
@@ -651,9 +651,9 @@ __global__ void __launch_bounds__(1024) k_dlogit(
   }
   if (rg < RG) {
     const bool vec = sizeof(T) == 2 && (H & 7) == 0;
-    // the rows of this thread in groups of four, the four loads issued before any is used (one
+    // the rows of this thread in groups of eight, the eight loads issued before any is used (one
     // memory latency per group); rows are still taken in increasing order
-    constexpr int U = 4;
+    constexpr int U = 8;
     for (int r0 = rg; vec && r0 < 3 * B; r0 += U * RG) {
       uint4 qv[U];
 #pragma unroll
