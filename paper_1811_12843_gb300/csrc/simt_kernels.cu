@@ -109,7 +109,20 @@ __global__ void k_draw_batch(const T* __restrict__ pool, int64_t n_pool,
       const float* src = xin + ((int64_t)c * B + b0 + i) * x_dim;
       const bool vec = (x_dim & 3) == 0 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0) &&
                        ((reinterpret_cast<uintptr_t>(dst) & (4 * sizeof(T) - 1)) == 0);
-      if (vec) {
+      if (vec && x_dim <= 1024) {
+        // the row's (up to eight per lane) 16-byte loads issued before its stores
+        float4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int k = lane * 4 + 128 * u;
+          if (k < x_dim) v[u] = __ldg(reinterpret_cast<const float4*>(src + k));
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int k = lane * 4 + 128 * u;
+          if (k < x_dim) store4<T>(dst + k, v[u]);
+        }
+      } else if (vec) {
         for (int k = lane * 4; k < x_dim; k += 128)
           store4<T>(dst + k, __ldg(reinterpret_cast<const float4*>(src + k)));
       } else {
