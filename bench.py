@@ -86,9 +86,9 @@ _derive()
 # dram__bytes_write.sum) of these same kernels, each with the summary it comes from. A phase
 # whose kernels changed after its capture has no entry (null traffic).
 PHASE_TRAFFIC = {
-    "train_bwd": (2195.5e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
-    "d_fwd": (236.7e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
-    "g_fwd": (143.8e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
+    "train_bwd": (2198.7e6, "profiles/k_bwd_cells_fused_adam_12x12_bf16.md"),
+    "d_fwd": (236.6e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
+    "g_fwd": (146.4e6, "profiles/k_mlp_fwd_pair_eval_12x12_bf16.md"),
     "batch": (21.2e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
     "fitness": (1.8e6, "profiles/launches_12x12_bf16_iteration.md (earlier DRAM capture)"),
 }
