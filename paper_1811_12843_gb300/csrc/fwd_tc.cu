@@ -927,6 +927,32 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(bar_cluster);
     };
+    // a tile's biases (and the discriminator's output weights): this thread's share, loaded
+    // from global memory one tile ahead, so that a tile's staging waits on no memory latency
+    // (the generator's first layer, one K chunk, does not cover it)
+    constexpr int NV = (BIAS_MAX + 32 * NE - 1) / (32 * NE);
+    auto load_bias = [&](int kk, float (&v)[NV]) {
+      const float* wm = p.wmaster + (int64_t)kk * p.pstride;
+      const int nb3 = KND == KIND_D ? HID + 1 : p.x;
+#pragma unroll
+      for (int u = 0; u < NV; ++u) {
+        const int i = et + u * 32 * NE;
+        v[u] = 0.f;
+        if (i >= 512 + nb3) continue;
+        if (i < 256) v[u] = wm[p.off_b1 + i];
+        else if (i < 512) v[u] = wm[p.off_b2 + i - 256];
+        else if (KND == KIND_D)
+          v[u] = i < 512 + HID
+                     ? __bfloat162float(p.wb[(int64_t)kk * p.pstride + p.off_w3 + i - 512])
+                     : wm[p.off_b3];
+        else v[u] = wm[p.off_b3 + i - 512];
+      }
+    };
+    auto tile_individual = [&](int q) {
+      return (KND == KIND_D && p.train) ? __ldg(&p.wsel[q / p.mt]) : __ldg(&p.pairs[q]).x;
+    };
+    float vb[NV];
+    if (cid < p.n_pairs) load_bias(tile_individual(cid), vb);
     for (int pi = cid; pi < p.n_pairs && ok; pi += ncl, ++ltile) {
       const bool train = KND == KIND_D && p.train;
       const int4 pr = train ? make_int4(0, 0, 0, 0) : __ldg(&p.pairs[pi]);
@@ -952,30 +978,17 @@ __global__ void __launch_bounds__(pair_threads<KND>(), 1)
         row_ok = prob >= 0 && rr < p.rows;
         lidx = (int64_t)prob * p.rows + rr;
       }
-      const float* wm = p.wmaster + (int64_t)k * p.pstride;
+      (void)k;
       float* sb = s_bias + (ltile & 1) * BIAS_MAX;
       {
         const int nb3 = KND == KIND_D ? HID + 1 : p.x;
-        constexpr int NV = (BIAS_MAX + 32 * NE - 1) / (32 * NE);
-        float v[NV];
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
           const int i = et + u * 32 * NE;
-          v[u] = 0.f;
-          if (i >= 512 + nb3) continue;
-          if (i < 256) v[u] = wm[p.off_b1 + i];
-          else if (i < 512) v[u] = wm[p.off_b2 + i - 256];
-          else if (KND == KIND_D)
-            v[u] = i < 512 + HID
-                       ? __bfloat162float(p.wb[(int64_t)k * p.pstride + p.off_w3 + i - 512])
-                       : wm[p.off_b3];
-          else v[u] = wm[p.off_b3 + i - 512];
+          if (i < 512 + nb3) sb[i] = vb[u];
         }
-#pragma unroll
-        for (int u = 0; u < NV; ++u) {
-          const int i = et + u * 32 * NE;
-          if (i < 512 + nb3) sb[i] = v[u];
-        }
+        // the next tile's, in flight while this one computes
+        if (pi + ncl < p.n_pairs) load_bias(tile_individual(pi + ncl), vb);
         mbar_arrive(bBias + 8 * (ltile & 1));
         if (!mbar_wait_warp(bBias + 8 * (ltile & 1), (uint32_t)((ltile >> 1) & 1), abort_flag,
                             p.err, 8)) {
