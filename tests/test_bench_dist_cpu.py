@@ -48,3 +48,28 @@ def test_two_rank_reduction_takes_the_slowest_rank():
         assert ms_step == pytest.approx(5.0)
         assert iters == pytest.approx(2 * 200.0)
         assert pairs == pytest.approx(2 * 200.0 * bench.PAIRS)
+
+
+def test_grid_option_scales_the_work_with_the_cells():
+    """bench.py --grid RxC (small-case kernel captures) re-derives every per-iteration work
+    figure from the cell count: evaluation and training FLOP and the backward's algorithmic
+    bytes are per-cell sums, so a 6x6 torus has a quarter of the 12x12 figures."""
+    import importlib.util
+    import pathlib
+    path = pathlib.Path(__file__).resolve().parents[1] / "bench.py"
+    spec = importlib.util.spec_from_file_location("bench_grid_probe", path)
+    b = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(b)
+    full = (b.CELLS, b.PAIRS, b.EVAL_G_FLOP, b.EVAL_D_FLOP, b.TRAIN_FWD_FLOP, b.TRAIN_BWD_FLOP,
+            b.MIX_FLOP, b.TRAIN_BWD_BYTES)
+    assert full[0] == 144 and full[1] == 3600
+    b.ROWS, b.COLS = 6, 6
+    b._derive()
+    small = (b.CELLS, b.PAIRS, b.EVAL_G_FLOP, b.EVAL_D_FLOP, b.TRAIN_FWD_FLOP, b.TRAIN_BWD_FLOP,
+             b.MIX_FLOP, b.TRAIN_BWD_BYTES)
+    for f, s in zip(full, small):
+        assert s * 4 == f
+    # the evaluation's FLOP: 2 B rows x (z h + h h + h x) per generator slot, 2 x 6B rows x
+    # (x h + h h + h) per discriminator slot, 5 slots of each per cell
+    assert b.EVAL_G_FLOP == 2 * 36 * 5 * 100 * (64 * 256 + 256 * 256 + 256 * 784)
+    assert b.EVAL_D_FLOP == 2 * 36 * 30 * 100 * (784 * 256 + 256 * 256 + 256)
