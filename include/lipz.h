@@ -159,7 +159,9 @@ LIPZ_API int lipz_grid_destroy(lipz_grid* g);
  * launch; on the legacy or per-thread default stream they keep plain stream order. */
 LIPZ_API int lipz_set_stream(lipz_grid* g, void* stream);
 
-/* Blocks until the grid's stream is idle; reports a non-finite loss seen since the last check. */
+/* Blocks until the grid's stream is idle; reports a non-finite loss or an expired bounded wait
+ * seen since the last check, and completes a pending lipz_iterate_batch_async call (its
+ * fitnesses are copied to the caller's buffers). */
 LIPZ_API int lipz_synchronize(lipz_grid* g);
 
 /*
