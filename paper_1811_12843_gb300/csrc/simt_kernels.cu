@@ -507,12 +507,28 @@ __global__ void k_fitness(const float* __restrict__ logits, int B, float* __rest
   const float* lc = logits + (int64_t)c * 5 * 6 * B;
   for (int task = warp; task < 30; task += nw) {
     float s1 = 0.f, s2 = 0.f;
-    if (task < 5) {
-      const float* l = lc + (int64_t)task * 6 * B;
+    const bool real = task < 5;
+    const int i = real ? 0 : (task - 5) / 5, j = real ? task : (task - 5) % 5;
+    const float* l = lc + (int64_t)j * 6 * B + (real ? 0 : (int64_t)(1 + i) * B);
+    if (B <= 128) {
+      // a lane's (up to four) logits loaded before any is used: one memory latency per mean;
+      // the terms are still added in increasing row order
+      float x[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) x[u] = lane + 32 * u < B ? l[lane + 32 * u] : 0.f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (lane + 32 * u >= B) break;
+        if (real) {
+          s1 += softplusf(-x[u]);
+        } else {
+          s1 += softplusf(x[u]);
+          s2 += softplusf(-x[u]);
+        }
+      }
+    } else if (real) {
       for (int b = lane; b < B; b += 32) s1 += softplusf(-l[b]);
     } else {
-      const int i = (task - 5) / 5, j = (task - 5) % 5;
-      const float* l = lc + (int64_t)j * 6 * B + (int64_t)(1 + i) * B;
       for (int b = lane; b < B; b += 32) {
         s1 += softplusf(l[b]);
         s2 += softplusf(-l[b]);
